@@ -1,0 +1,369 @@
+#!/usr/bin/env python
+"""Benchmark of the GB300 repair path: repaired document tokens/s and p50 repair
+latency per request, with the roofline fraction of the dominant kernel.
+
+One step = one request through all four C-ABI calls (assemble, compress,
+forward, apply) on one stream, captured once into a CUDA graph and replayed.
+Default workload: the Llama-3.1-8B-shaped cache (32 layers, 8 KV heads,
+head_dim 128, d_model 4096) with the d_c 512 / d_b 1024 / 6-block repairer,
+one request of 10 chunks x 512 tokens.  Inputs are seeded and synthetic; the
+pool (1 GiB) and the assembled cache (0.67 GB) exceed the 129 MB L2, so no
+explicit L2 flush is needed between steps.
+
+    python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+
+For N > 1 (torchrun, one process per GPU) every rank repairs its own request
+stream with a weight replica: requests never interact, so there is no
+collective; value = all ranks' tokens / the slowest rank's time.
+`--impl reference` times the CPU oracle (float64 numpy) on a bounded prefix
+of the same request instead.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "repaired doc tokens/s and p50 repair latency per request (1 GB300, % roofline)"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="llama8b")
+    ap.add_argument("--no-graph", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return p["hbm_gbs"], p["bf16_tflops"], p["bf16_tflops_sustained"], "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def workload_desc(case):
+    t, r = case.target, case.repairer
+    lens = case.plan.request_lengths()
+    nreq = len(lens)
+    nch = len(case.plan.chunk_idx)
+    return (f"{case.recipe.name}: target L{t.n_layers} H_kv{t.n_kv_heads} d_h{t.head_dim} "
+            f"d_model{t.d_model} {t.cache_dtype}; repairer d_c{r.d_c} d_b{r.d_b} B{r.n_blocks} "
+            f"{r.n_heads} heads MLP{r.mlp_hidden // r.d_b}x d_seg{r.d_seg}; {nreq} request(s), "
+            f"{nch} chunks, {sum(lens)} tokens")
+
+
+def sample_clocks(dev_index):
+    path = tempfile.mktemp(prefix="cr_clocks_", suffix=".csv")
+    q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    try:
+        f = open(path, "w")
+        p = subprocess.Popen(["nvidia-smi", f"--query-gpu={q}", "--format=csv,noheader,nounits",
+                              "-lms", "200", "-i", str(dev_index)], stdout=f,
+                             stderr=subprocess.DEVNULL)
+        return p, f, path
+    except Exception:
+        return None, None, path
+
+
+def stop_clocks(handle):
+    p, f, path = handle
+    if p is None:
+        return None
+    p.terminate()
+    try:
+        p.wait(timeout=5)
+    except Exception:
+        p.kill()
+    f.close()
+    rows = []
+    with open(path) as fh:
+        for line in fh:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) >= 9 and parts[1].replace(".", "").isdigit():
+                rows.append(parts)
+    os.unlink(path)
+    if not rows:
+        return None
+    sm = [float(r[1]) for r in rows]
+    names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+    reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+    return {"sm_mhz": statistics.median(sm), "sm_max_mhz": float(rows[0][2]),
+            "power_w_max": max(float(r[3]) for r in rows if r[3].replace(".", "").isdigit())
+            if any(r[3].replace(".", "").isdigit() for r in rows) else None,
+            "reasons": reasons, "samples": len(rows)}
+
+
+def oracle_sample(case, n_chunks):
+    """Run the oracle on the first n_chunks of request 0 (a document prefix); returns
+    (tokens, seconds)."""
+    import numpy as np
+    import oracle as O
+    p = case.plan
+    sel = p.chunk_idx[p.cu_chunks[0]:p.cu_chunks[1]][:n_chunks]
+    kvs, embs = [], []
+    for c in sel:
+        kv, emb = case.pool_rows(int(p.chunk_start[c]), int(p.chunk_len[c]))
+        kvs.append(kv)
+        embs.append(emb)
+    kv, emb = np.concatenate(kvs), np.concatenate(embs)
+    lens = p.chunk_len[sel]
+    cid = np.concatenate([np.full(l, i, np.int32) for i, l in enumerate(lens)])
+    pos = np.arange(len(cid), dtype=np.int32)
+    t, r = case.target, case.repairer
+    t0 = time.perf_counter()
+    O.repair_request(kv, emb, cid, pos, case.weights, cache_dtype=t.cache_dtype,
+                     n_layers=t.n_layers, n_kv_heads=t.n_kv_heads, head_dim=t.head_dim,
+                     n_heads=r.n_heads)
+    return len(cid), time.perf_counter() - t0
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import fixtures as F
+    case = F.make_case(args.workload)
+    n_chunks = 1
+    times, toks = [], 0
+    for i in range(args.warmup + args.steps):
+        n, s = oracle_sample(case, n_chunks)
+        if i >= args.warmup:
+            times.append(s)
+            toks = n
+    total = sum(times)
+    value = toks * len(times) / total
+    cores = os.cpu_count()
+    sample = f"first {n_chunks} chunk ({toks} tokens) of the request, full repair incl. head"
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * total / len(times), "p50_ms": 1e3 * statistics.median(times),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded), random-init repairer",
+        "config": {"workload": workload_desc(case), "sample": sample},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }))
+
+
+def run_ours(args):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    import fixtures as F
+    from paper_2609_35139_gb300 import RepairSession, build, cr, dims_from, pack_host_weights
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    build.build()
+    cr.lib()
+    cr.cr_clear_device_status()
+
+    case = F.make_case(args.workload)
+    t, r = dims_from(case.target, case.repairer)
+    pw = pack_host_weights(case.weights, case.repairer.n_blocks)
+    p = case.plan
+    kvp_h, embp_h = case.pool()
+    to_dev = lambda a: (torch.from_numpy(a.view(np.int16)).view(torch.bfloat16)
+                        if a.dtype == np.uint16 else torch.from_numpy(a)).cuda()
+    kvp, embp = to_dev(kvp_h), to_dev(embp_h)
+    N = p.n_tokens
+    sess = RepairSession(t, r, pw, max_tokens=N)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        sess.repair(kvp, embp, p.chunk_start, p.chunk_len, p.chunk_idx, p.cu_chunks)
+
+    # ---- per-call timing (eager), for the stage breakdown and the roofline
+    a = sess.assemble(kvp, embp, p.chunk_start, p.chunk_len, p.chunk_idx, p.cu_chunks)
+    calls = [("assemble", lambda: sess.assemble(kvp, embp, p.chunk_start, p.chunk_len,
+                                                p.chunk_idx, p.cu_chunks)),
+             ("compress", lambda: sess.compress(a)),
+             ("forward", lambda: sess.forward(a)),
+             ("apply", lambda: sess.apply(a))]
+    for _ in range(3):
+        for _, fn in calls:
+            fn()
+    torch.cuda.synchronize()
+    stage_ms = {k: [] for k, _ in calls}
+    for _ in range(10):
+        for name, fn in calls:
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            stage_ms[name].append((e0, e1))
+    torch.cuda.synchronize()
+    stages = {k: statistics.median(e0.elapsed_time(e1) for e0, e1 in v) for k, v in stage_ms.items()}
+
+    # ---- the timed step: graph replay
+    use_graph = not args.no_graph
+    if use_graph:
+        g = torch.cuda.CUDAGraph()
+        step()
+        torch.cuda.synchronize()
+        with torch.cuda.graph(g):
+            step()
+        run = g.replay
+    else:
+        run = step
+    for _ in range(args.warmup):
+        run()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clk = sample_clocks(local)
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    evs[0].record(stream)
+    for i in range(args.steps):
+        run()
+        evs[i + 1].record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks = stop_clocks(clk)
+    per_step = [evs[i].elapsed_time(evs[i + 1]) for i in range(args.steps)]
+    total_ms = evs[0].elapsed_time(evs[-1])
+    if world > 1:
+        tt = torch.tensor([total_ms], device="cuda")
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms = float(tt.item())
+    value = world * N * args.steps / (total_ms / 1e3)
+    st, word = cr.cr_get_device_status()
+    if st != cr.CR_OK:
+        raise RuntimeError(f"device status {word}")
+
+    # ---- end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(case, sess, kvp_h, embp_h, args, world)
+
+    # ---- roofline of the dominant kernel (the KV residual head, one launch)
+    hbm, tf_burst, tf_sus, src = load_peaks()
+    tg, rp = case.target, case.repairer
+    head_flops = 2.0 * N * rp.d_b * tg.d_kv
+    head_tf = head_flops / (stages["apply"] * 1e-3) / 1e12
+    es = 2 if tg.cache_dtype == "bf16" else 4
+    gather_bytes = 2.0 * N * (tg.d_kv + tg.d_model) * es
+    roofline = {"kernel": "cr_apply_residual (KV residual head GEMM + residual add)",
+                "bound": "tensor", "achieved": head_tf, "peak": tf_sus, "unit": "TFLOP/s",
+                "frac": head_tf / tf_sus, "traffic": None,
+                "peak_source": f"{src} bf16_tflops_sustained",
+                "algorithmic": f"2*N*d_b*D_KV = {head_flops:.3e} flop per launch"}
+    stage_roofline = {
+        "assemble_hbm_frac": gather_bytes / (stages["assemble"] * 1e-3) / 1e9 / hbm,
+        "apply_tensor_frac": roofline["frac"],
+    }
+    launches_per_step = 1 + (2 + 4 + (2 if tg.cache_dtype == "f32" else 0) - (1 if rp.n_blocks == 0 else 0)) \
+        + 7 * rp.n_blocks + 1 + 1
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        n_chunks = 2
+        ntok, secs = oracle_sample(case, n_chunks)
+        cpu = {"value": ntok / secs, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+               "sample": f"first {n_chunks} chunks ({ntok} tokens) of the request, full repair "
+                         f"incl. head, float64 numpy, {secs:.1f} s"}
+    if rank == 0:
+        out = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
+            "p50_ms": statistics.median(per_step),
+            "p90_ms": sorted(per_step)[int(0.9 * (len(per_step) - 1))],
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded caches, embeddings, chunk map; random-init Xavier repairer)",
+            "config": {"workload": workload_desc(case), "n_tokens": N, "cuda_graph": use_graph,
+                       "l2": "no flush: pool 1 GiB and assembled cache 0.67 GB exceed L2",
+                       "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+            "roofline": roofline, "stage_roofline": stage_roofline,
+            "stages_ms": stages, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": launches_per_step * args.steps, "clocks": clocks,
+        }
+        print(json.dumps(out))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def run_e2e(case, sess, kvp_h, embp_h, args, world):
+    """Host pool in pinned memory -> the request's chunks copied to a device staging
+    pool -> the four calls -> repaired cache copied back to pinned host memory."""
+    import numpy as np
+    import torch
+    from paper_2609_35139_gb300 import cr
+
+    p = case.plan
+    sel = p.chunk_idx[p.cu_chunks[0]:p.cu_chunks[1]]
+    lens = p.chunk_len[sel]
+    starts = p.chunk_start[sel]
+    pin = lambda a: (torch.from_numpy(a.view(np.int16)).view(torch.bfloat16)
+                     if a.dtype == np.uint16 else torch.from_numpy(a)).pin_memory()
+    kv_h, emb_h = pin(kvp_h), pin(embp_h)
+    N = int(lens.sum())
+    stage_kv = torch.empty(N, kv_h.shape[1], dtype=kv_h.dtype, device="cuda")
+    stage_emb = torch.empty(N, emb_h.shape[1], dtype=emb_h.dtype, device="cuda")
+    out_h = torch.empty(N, kv_h.shape[1], dtype=kv_h.dtype).pin_memory()
+    st_start = np.concatenate([[0], np.cumsum(lens)[:-1]]).astype(np.int64)
+    idx = np.arange(len(sel), dtype=np.int32)
+    cu = np.array([0, len(sel)], np.int32)
+
+    def step():
+        for k in range(len(sel)):
+            a, n, d = int(starts[k]), int(lens[k]), int(st_start[k])
+            stage_kv[d:d + n].copy_(kv_h[a:a + n], non_blocking=True)
+            stage_emb[d:d + n].copy_(emb_h[a:a + n], non_blocking=True)
+        sess.repair(stage_kv, stage_emb, st_start, lens, idx, cu)
+        out_h.copy_(sess.kv[:N], non_blocking=True)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / args.steps
+    es = kv_h.element_size()
+    return {"value": world * N / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
+            "h2d_bytes_per_step": int(N * (kv_h.shape[1] + emb_h.shape[1]) * es),
+            "d2h_bytes_per_step": int(N * kv_h.shape[1] * es),
+            "path": "pinned host chunks -> device staging (copy engine) -> four C-ABI calls -> "
+                    "pinned host repaired cache"}
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,226 @@
+/*
+ * cr.h - C ABI of the GB300 (sm_103a) CacheRepair online repair library.
+ *
+ * The library repairs a stale multi-chunk KV cache with the lightweight
+ * repair network of "CacheRepair: Learning to Repair Cross-Chunk Context in
+ * RAG for KV Cache Fusion" (arxiv 2609.35139):
+ *
+ *     KV_hat = R_theta(KV_stale, D_r)  ~  KV_joint          (Sec. 2.2)
+ *
+ * in four calls that run back to back on one CUDA stream:
+ *
+ *   cr_assemble_stale     concatenate canonical chunk caches      (Sec. 4.1)
+ *   cr_compress_features  StaleEncoder, token fusion, P_b(s)      (Sec. 4.1)
+ *   cr_repair_forward     B Repair Blocks, final LayerNorm        (Sec. 4.1)
+ *   cr_apply_residual     KV residual head, in-place residual add,
+ *                         optional global RoPE on K               (Sec. 4.1)
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * Ownership: the caller owns and allocates every buffer (device memory
+ *   unless a parameter says "host").  The library allocates no memory and
+ *   keeps no per-call state; scratch lives in a caller workspace of
+ *   cr_workspace_bytes() bytes.  Calls on different streams with different
+ *   workspaces may run concurrently.
+ * Asynchrony: calls enqueue kernels on `stream` (a cudaStream_t; NULL is the
+ *   legacy default stream) and return without synchronising.  Host arrays
+ *   are read before the call returns.  Nothing is allocated or synchronised,
+ *   so a sequence of calls can be captured into a CUDA graph.
+ * Layouts: row-major.  A cache row is one token: kv[t, j] with
+ *   j = ((layer * 2 + kv) * n_kv_heads + head) * head_dim + d, kv = 0 for K,
+ *   D_KV = 2 * n_layers * n_kv_heads * head_dim.  K is canonical (no RoPE,
+ *   Sec. 4.1 "Chunk-cache preparation").  Weight matrices are bf16 (uint16
+ *   bit patterns) stored [out_features, in_features]; biases, LayerNorm
+ *   parameters and sigma vectors are fp32.
+ * Alignment: every device pointer must be 16-byte aligned and every row
+ *   stride a multiple of 16 bytes (TMA requirement), else CR_ERR_INVALID_ARG.
+ * Errors: arguments are validated on the host before anything is enqueued
+ *   (CR_ERR_INVALID_ARG, CR_ERR_UNSUPPORTED for shapes the kernels do not
+ *   implement); launch failures return CR_ERR_CUDA.  A kernel that detects
+ *   a problem on the device (an index out of range, a pipeline wait that
+ *   timed out) records it in a device status word instead of trapping; read
+ *   it with cr_get_device_status().  Once set, later kernels give up their
+ *   waits early, so a bad state never hangs the GPU.
+ */
+#ifndef CR_H_
+#define CR_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum cr_status {
+    CR_OK = 0,
+    CR_ERR_INVALID_ARG = 1,
+    CR_ERR_UNSUPPORTED = 2,
+    CR_ERR_CUDA = 3,
+    CR_ERR_DEVICE_INDEX = 4,
+    CR_ERR_TIMEOUT = 5
+} cr_status;
+
+typedef enum cr_dtype { CR_F32 = 0, CR_BF16 = 1 } cr_dtype;
+
+/* Global RoPE on repaired K: none (canonical K out) or R_M(p_t) (Sec. 4.1). */
+typedef enum cr_rope_mode { CR_ROPE_NONE = 0, CR_ROPE_GLOBAL = 1 } cr_rope_mode;
+
+/* Frozen target LLM cache shape (Sec. 4.1: S = 2 L H_KV segments of d_h). */
+typedef struct cr_target_dims {
+    int32_t n_layers;     /* L_M */
+    int32_t n_kv_heads;   /* H_KV */
+    int32_t head_dim;     /* d_h: 64 or 128 */
+    int32_t d_model;      /* width of the target's token embedding E_M(x_t) */
+    int32_t cache_dtype;  /* cr_dtype of the cache and embeddings */
+} cr_target_dims;
+
+/* Repairer shape (Sec. 4.1; App. A Table "repair-scales").  d_c is the
+ * StaleEncoder/P_tok output width, d_b the backbone width (d_c = d_b in the
+ * paper's repairers).  Attention heads are d_b / n_heads wide (32 or 64). */
+typedef struct cr_repairer_dims {
+    int32_t d_seg;        /* per-segment projection width, 8 or 16 */
+    int32_t d_c;
+    int32_t d_b;          /* multiple of 128, at most 1024 */
+    int32_t n_blocks;     /* B */
+    int32_t n_heads;
+    int32_t mlp_hidden;   /* MLP width (ratio * d_b) */
+    float ln_eps;         /* LayerNorm epsilon */
+    float rope_theta;     /* base of the repairer's own RoPE on Q and K */
+} cr_repairer_dims;
+
+/* One Repair Block (pre-LN attention + MLP).  Device pointers. */
+typedef struct cr_block_weights {
+    const float* ln1_g;      /* [d_b] */
+    const float* ln1_b;      /* [d_b] */
+    const uint16_t* w_qkv;   /* [3 d_b, d_b]: rows 0..d_b-1 Q, then K, then V */
+    const float* b_qkv;      /* [3 d_b] */
+    const uint16_t* w_o;     /* [d_b, d_b] */
+    const float* b_o;        /* [d_b] */
+    const float* ln2_g;      /* [d_b] */
+    const float* ln2_b;      /* [d_b] */
+    const uint16_t* w_fc1;   /* [mlp_hidden, d_b] */
+    const float* b_fc1;      /* [mlp_hidden] */
+    const uint16_t* w_fc2;   /* [d_b, mlp_hidden] */
+    const float* b_fc2;      /* [d_b] */
+} cr_block_weights;
+
+/* All repairer parameters (device pointers, except `blocks`, a HOST array of
+ * n_blocks entries whose members are device pointers). */
+typedef struct cr_weights {
+    const uint16_t* w_seg;   /* [S, d_seg, d_h]: segment s's d_h -> d_seg map */
+    const float* b_seg;      /* [S, d_seg] */
+    const uint16_t* w_map;   /* [d_c, S d_seg] */
+    const float* b_map;      /* [d_c] */
+    const uint16_t* w_tok;   /* [d_c, d_model]  (P_tok) */
+    const float* b_tok;      /* [d_c] */
+    const uint16_t* w_fuse;  /* [d_b, 2 d_c]  (F on [s ; P_tok E]) */
+    const float* b_fuse;     /* [d_b] */
+    const uint16_t* w_rein;  /* [B d_b, d_c]: P_1 .. P_B stacked */
+    const float* b_rein;     /* [B d_b] */
+    const cr_block_weights* blocks;  /* HOST array [B] */
+    const float* lnf_g;      /* [d_b] final LayerNorm */
+    const float* lnf_b;      /* [d_b] */
+    const uint16_t* w_out;   /* [D_KV, d_b]  KV residual head */
+    const float* b_out;      /* [D_KV] */
+    const float* sigma_stale;  /* [D_KV] input scale (Sec. 4.2 "Normalization") */
+    const float* sigma_delta;  /* [D_KV] residual scale */
+} cr_weights;
+
+/* Bytes of scratch workspace the calls need for requests of up to
+ * max_tokens assembled tokens (all requests of one call together).
+ * Returns 0 if the dimensions are invalid. */
+size_t cr_workspace_bytes(const cr_target_dims* target, const cr_repairer_dims* rep,
+                          int64_t max_tokens);
+
+/*
+ * cr_assemble_stale - concatenate the selected canonical chunk caches of
+ * each request in document order into KV^c_stale (Sec. 4.1 "Chunk-cache
+ * preparation": with K stored without RoPE, assembly is a pure copy; the
+ * method places K at its global position only after repair).
+ *
+ * kv_pool  [n_pool_tokens, D_KV], emb_pool [n_pool_tokens, d_model]
+ *          (cache dtype): independently prefilled chunks back to back.
+ * chunk_start [n_pool_chunks] (HOST, int64), chunk_len [n_pool_chunks] (HOST):
+ *          pool chunk c occupies rows chunk_start[c] .. + chunk_len[c].
+ * chunk_idx (HOST): pool chunk ids of all requests, request r using
+ *          chunk_idx[cu_chunks[r] .. cu_chunks[r+1]) in document order.
+ * cu_chunks [n_req + 1] (HOST).
+ * Outputs (device, caller-sized for max_tokens rows):
+ *   kv_out [N, D_KV], emb_out [N, d_model]   stale cache and embeddings
+ *   chunk_id  [N] int32  c(t): index of t's chunk within its request
+ *   chunk_end [N] int32  exclusive request-local end of t's chunk
+ *   pos       [N] int32  p_t: position of t within its request
+ *   cu_seqlens_dev [n_req + 1] int32 token offsets of the requests
+ *   cu_seqlens_host [n_req + 1] (HOST, written before return)
+ * Errors: CR_ERR_INVALID_ARG for an out-of-range or empty chunk, a chunk
+ *   outside the pool, an empty request, N > max_tokens, or more than 512
+ *   selected chunks / 256 requests in one call.
+ */
+cr_status cr_assemble_stale(const cr_target_dims* target, const void* kv_pool,
+                            const void* emb_pool, int64_t n_pool_tokens,
+                            const int64_t* chunk_start, const int32_t* chunk_len,
+                            int32_t n_pool_chunks, const int32_t* chunk_idx,
+                            const int32_t* cu_chunks, int32_t n_req, void* kv_out,
+                            void* emb_out, int64_t max_tokens, int32_t* chunk_id,
+                            int32_t* chunk_end, int32_t* pos, int32_t* cu_seqlens_dev,
+                            int32_t* cu_seqlens_host, void* stream);
+
+/*
+ * cr_compress_features - StaleEncoder and token fusion (Sec. 4.1):
+ *   s_t   = W_map [W_seg,s (kv_t,s / sigma_stale,s) + b_seg,s]_s + b_map
+ *   h^0_t = F([s_t ; P_tok E_M(x_t)])
+ *   r_b   = P_b(s)  for every block b (stale-feature reinjection)
+ * kv [N, D_KV], emb [N, d_model] (cache dtype, from cr_assemble_stale).
+ * h0_out   [N, d_b] fp32  backbone input h^0.
+ * rein_out [N, B d_b] bf16  P_b(s_t) at columns b*d_b .. (b+1)*d_b.
+ * workspace: cr_workspace_bytes(.., max_tokens >= N) bytes, 256-B aligned.
+ */
+cr_status cr_compress_features(const cr_target_dims* target, const cr_repairer_dims* rep,
+                               const cr_weights* w, const void* kv, const void* emb,
+                               int64_t n_tokens, float* h0_out, uint16_t* rein_out,
+                               void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * cr_repair_forward - the B Repair Blocks and the final LayerNorm (Sec. 4.1):
+ *   h^b = RepairBlock_b(h^{b-1} + P_b(s); A, p),   y_f = LN(h^B)
+ * with the block-causal mask A_ij = 1[c(j) <= c(i)] inside each request and
+ * the repairer's RoPE on Q, K at positions p.
+ * h0 [N, d_b] fp32 and rein [N, B d_b] bf16 from cr_compress_features;
+ * chunk_end, pos [N] from cr_assemble_stale; cu_seqlens_host [n_req+1] HOST.
+ * yf_out [N, d_b] bf16.
+ */
+cr_status cr_repair_forward(const cr_target_dims* target, const cr_repairer_dims* rep,
+                            const cr_weights* w, const float* h0, const uint16_t* rein,
+                            const int32_t* chunk_end, const int32_t* pos,
+                            const int32_t* cu_seqlens_host, int32_t n_req, int64_t n_tokens,
+                            uint16_t* yf_out, void* workspace, size_t workspace_bytes,
+                            void* stream);
+
+/*
+ * cr_apply_residual - KV residual head and residual add, in place (Sec. 4.1):
+ *   z_t = W_out y_f,t + b_out;   kv_t <- round(kv_t + sigma_delta * z_t)
+ * and, for CR_ROPE_GLOBAL, K segments rotated by R_M(p_t) (rotate-half pairs
+ * (d, d + d_h/2), angle p_t * inv_freq[d]) before the single rounding to the
+ * cache dtype (round to nearest even).
+ * yf [N, d_b] bf16; kv_inout [N, D_KV] cache dtype; pos [N] device int32;
+ * inv_freq_host [head_dim/2] HOST fp32, the target's RoPE frequencies
+ * (may be NULL for CR_ROPE_NONE).
+ */
+cr_status cr_apply_residual(const cr_target_dims* target, const cr_repairer_dims* rep,
+                            const cr_weights* w, const uint16_t* yf, int64_t n_tokens,
+                            void* kv_inout, const int32_t* pos, const float* inv_freq_host,
+                            int32_t rope_mode, void* stream);
+
+/* Device status word: out[0] = first error (0 none, 1 wait timeout, 2 device
+ * index out of range), out[1] = site, out[2] = block.  Synchronises the
+ * device.  cr_clear_device_status() resets it to zero. */
+cr_status cr_get_device_status(uint32_t out[3]);
+cr_status cr_clear_device_status(void);
+
+const char* cr_status_str(cr_status s);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* CR_H_ */

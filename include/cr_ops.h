@@ -1,0 +1,85 @@
+/*
+ * cr_ops.h - the kernels inside the four cr.h calls, exposed one by one so
+ * that each step of the repair path can be checked on its own.  Same
+ * conventions as cr.h (caller-owned device buffers, 16-byte alignment,
+ * asynchronous on `stream`, host-side validation, no allocation).
+ */
+#ifndef CR_OPS_H_
+#define CR_OPS_H_
+
+#include "cr.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Epilogues of cr_linear. */
+typedef enum cr_linear_epi {
+    CR_EPI_BF16 = 0,      /* out(bf16)  = A W^T + bias                         */
+    CR_EPI_GELU_BF16 = 1, /* out(bf16)  = GELU_erf(A W^T + bias)  (MLP, R4)    */
+    CR_EPI_ADD_F32 = 2,   /* out(fp32) += A W^T + bias      (residual stream)  */
+    CR_EPI_F32 = 3        /* out(fp32)  = A W^T + bias                         */
+} cr_linear_epi;
+
+/*
+ * cr_linear - out = epi(A W^T + bias) on the tcgen05 tensor cores, bf16
+ * operands, fp32 accumulation (every linear of Sec. 4.1).
+ * A [M, K] bf16 with row stride lda elements; W [N, K] bf16 (row stride K);
+ * bias [N] fp32 or NULL; out [M, N] with row stride ldo elements.
+ * K must be a multiple of 8; M, N >= 1.
+ */
+cr_status cr_linear(const uint16_t* A, int64_t lda, const uint16_t* W, const float* bias,
+                    int64_t M, int64_t N, int64_t K, void* out, int64_t ldo, int32_t epi,
+                    void* stream);
+
+/*
+ * cr_layernorm - u = LN(x + add) * gamma + beta per row (biased variance,
+ * eps), fp32 statistics (R4).  x [M, D] fp32 (row stride D).  If `add` is
+ * non-NULL ([M, D] bf16, row stride ld_add), x + add is also written to
+ * x_out ([M, D] fp32; may equal x).  u [M, D] bf16.  D a multiple of 128,
+ * at most 1024.
+ */
+cr_status cr_layernorm(const float* x, const uint16_t* add, int64_t ld_add, float* x_out,
+                       const float* gamma, const float* beta, float eps, int64_t M, int64_t D,
+                       uint16_t* u, void* stream);
+
+/*
+ * cr_chunk_causal_attention - softmax(Q K^T / sqrt(d) masked to
+ * c(j) <= c(i)) V per head and request (Sec. 4.1, block-causal mask).
+ * qkv [N, 3 d_b] bf16: Q at columns [0, d_b), K at [d_b, 2 d_b), V at
+ * [2 d_b, 3 d_b); head h at h*d .. (h+1)*d inside each (d = d_b / n_heads,
+ * 32 or 64; RoPE already applied).  chunk_end [N] int32 (request-local
+ * exclusive end of each token's chunk; key j is visible to query i iff
+ * j < chunk_end[i]).  cu_seqlens_host [n_req + 1] HOST.  out [N, d_b] bf16.
+ */
+cr_status cr_chunk_causal_attention(const uint16_t* qkv, int32_t d_b, int32_t n_heads,
+                                    const int32_t* chunk_end, const int32_t* cu_seqlens_host,
+                                    int32_t n_req, int64_t n_tokens, uint16_t* out,
+                                    void* stream);
+
+/*
+ * cr_qkv_rope - the repair block's QKV linear with the repairer RoPE fused
+ * into its epilogue: qkv = u W_qkv^T + b_qkv, then Q and K of every head
+ * rotated (rotate-half pairs, angle pos[t] * theta^(-2i/d)).
+ * u [N, d_b] bf16; w_qkv [3 d_b, d_b]; qkv [N, 3 d_b] bf16.
+ */
+cr_status cr_qkv_rope(const uint16_t* u, const uint16_t* w_qkv, const float* b_qkv,
+                      const int32_t* pos, int64_t n_tokens, int32_t d_b, int32_t n_heads,
+                      float rope_theta, uint16_t* qkv, void* stream);
+
+/*
+ * cr_segment_project - StaleEncoder stage 1 (Sec. 4.1):
+ *   y[t, s*d_seg + k] = sum_d W_seg[s,k,d] kv[t, s*d_h + d] / sigma_stale[s*d_h + d]
+ *                       + b_seg[s,k]
+ * kv [N, D_KV] bf16; y [N, S*d_seg] bf16.  workspace: at least
+ * S*d_seg*d_h*2 bytes (holds W_seg with 1/sigma folded in).
+ */
+cr_status cr_segment_project(const cr_target_dims* target, int32_t d_seg, const uint16_t* kv,
+                             int64_t n_tokens, const uint16_t* w_seg, const float* b_seg,
+                             const float* sigma_stale, uint16_t* y, void* workspace,
+                             size_t workspace_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* CR_OPS_H_ */

@@ -45,10 +45,10 @@ from dataclasses import dataclass
 from typing import Dict, List, Optional, Sequence
 
 import numpy as np
-from scipy.special import erf
+import torch
 
 __all__ = [
-    "dtype_to_f64", "round_to_cache", "assemble_stale", "stale_encoder", "token_fusion",
+    "dtype_to_f64", "round_to_cache", "assemble_stale", "segment_projection", "stale_encoder", "token_fusion",
     "reinjection", "layer_norm", "gelu", "rope_rotate_half", "block_causal_mask",
     "block_causal_attention", "repair_block", "repair_backbone", "residual_head",
     "apply_residual", "global_rope_k", "repair_request", "weight_shapes", "param_groups",
@@ -104,7 +104,10 @@ def round_to_cache(x: np.ndarray, dtype: str) -> np.ndarray:
 
 
 def _bf16_mat(w: np.ndarray) -> np.ndarray:
-    return dtype_to_f64(w, "bf16")
+    """bf16 bit patterns -> float64; float arrays (already converted) pass through."""
+    if w.dtype == np.uint16:
+        return dtype_to_f64(w, "bf16")
+    return np.asarray(w, dtype=np.float64)
 
 
 def _vec(v: np.ndarray) -> np.ndarray:
@@ -143,22 +146,43 @@ def assemble_stale(kv_pool: np.ndarray, emb_pool: np.ndarray, chunk_start: np.nd
 
 
 # ------------------------------------------------------------------ Sec. 4.1: StaleEncoder, fusion
+def segment_projection(kv: np.ndarray, sigma_stale: np.ndarray, w_seg: np.ndarray,
+                       b_seg: np.ndarray, head_dim: int,
+                       cache_dtype: Optional[str] = None) -> np.ndarray:
+    """StaleEncoder stage 1 (Sec. 4.1): y[t, s] = W_seg,s (kv_t,s / sigma_stale,s) + b_seg,s.
+
+    kv: [n, D_KV] (float64, or the stored cache with `cache_dtype`); segment s
+    is the slice [s d_h, (s+1) d_h) (R9).  Returns [n, S * d_seg], the S
+    outputs concatenated in segment order.
+    """
+    x = dtype_to_f64(kv, cache_dtype) if cache_dtype else kv
+    n = x.shape[0]
+    S = x.shape[1] // head_dim
+    W = _bf16_mat(w_seg)                                         # [S, d_seg, d_h]
+    x = (x / _vec(sigma_stale)[None, :]).reshape(n, S, head_dim)
+    y = np.matmul(x.transpose(1, 0, 2), W.transpose(0, 2, 1)).transpose(1, 0, 2)
+    return (y + _vec(b_seg)[None]).reshape(n, -1)
+
+
 def stale_encoder(kv: np.ndarray, sigma_stale: np.ndarray, w_seg: np.ndarray, b_seg: np.ndarray,
-                  w_map: np.ndarray, b_map: np.ndarray, head_dim: int) -> np.ndarray:
+                  w_map: np.ndarray, b_map: np.ndarray, head_dim: int,
+                  cache_dtype: Optional[str] = None, rows_per_step: int = 256) -> np.ndarray:
     """s_t = StaleEncoder(KV^c_stale,t / sigma_stale)  (Sec. 4.1).
 
-    kv: [N, D_KV] float64.  The input is divided elementwise by sigma_stale;
-    segment s (one layer, head, K/V component; R9) has its own d_h -> d_seg
-    linear; the S outputs are concatenated and mapped to d_c (R1, R3).
+    Stage 1 (`segment_projection`): one d_h -> d_seg linear per segment on the
+    cache divided by sigma_stale; stage 2: the concatenated S outputs mapped
+    to d_c (R1, R3).  Tokens are independent, so they are processed
+    `rows_per_step` at a time to bound memory.
     """
     n = kv.shape[0]
-    S = kv.shape[1] // head_dim
-    x = kv / _vec(sigma_stale)[None, :]
-    x = x.reshape(n, S, head_dim)
-    W = _bf16_mat(w_seg)                                  # [S, d_seg, d_h]
-    y = np.einsum("nsd,skd->nsk", x, W) + _vec(b_seg)[None]   # per-segment linear
-    y = y.reshape(n, -1)                                  # concat over segments
-    return y @ _bf16_mat(w_map).T + _vec(b_map)
+    W = _bf16_mat(w_seg)
+    Wm = _bf16_mat(w_map)
+    out = np.empty((n, Wm.shape[0]))
+    for a in range(0, n, rows_per_step):
+        y = segment_projection(kv[a:a + rows_per_step], sigma_stale, W, b_seg, head_dim,
+                               cache_dtype)
+        out[a:a + rows_per_step] = y @ Wm.T + _vec(b_map)
+    return out
 
 
 def token_fusion(s: np.ndarray, emb: np.ndarray, w_tok, b_tok, w_fuse, b_fuse) -> np.ndarray:
@@ -182,7 +206,7 @@ def layer_norm(x: np.ndarray, g, b, eps: float) -> np.ndarray:
 
 def gelu(x: np.ndarray) -> np.ndarray:
     """erf-form GELU, x * Phi(x) (R4)."""
-    return 0.5 * x * (1.0 + erf(x / math.sqrt(2.0)))
+    return 0.5 * x * (1.0 + torch.erf(torch.from_numpy(x / math.sqrt(2.0))).numpy())
 
 
 def rope_rotate_half(x: np.ndarray, pos: np.ndarray, inv_freq: np.ndarray) -> np.ndarray:
@@ -209,20 +233,24 @@ def block_causal_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray,
                            chunk_id: np.ndarray) -> np.ndarray:
     """Multi-head softmax attention under the block-causal mask, one request.
 
-    q, k, v: [N, n_heads, d_head] (RoPE already applied to q, k).  For each
-    head: scores = q k^T / sqrt(d_head); disallowed pairs get -inf; softmax
-    over each row (max-subtracted); output = P v  (R7).
+    q, k, v: [N, n_heads, d_head] (RoPE already applied to q, k).  Query i
+    attends to the keys j with c(j) <= c(i) (R7).  Chunk ids are
+    non-decreasing along the request, so for every query of chunk c that set
+    is the prefix of tokens up to the end of chunk c; the softmax
+    (max-subtracted) of q k^T / sqrt(d_head) is taken over exactly that set.
     """
     n, nh, dh = q.shape
-    allow = block_causal_mask(chunk_id)
     out = np.empty_like(q)
-    for h in range(nh):
-        sc = (q[:, h, :] @ k[:, h, :].T) / math.sqrt(dh)
-        sc = np.where(allow, sc, -np.inf)
-        sc = sc - sc.max(axis=1, keepdims=True)
-        p = np.exp(sc)
-        p = p / p.sum(axis=1, keepdims=True)
-        out[:, h, :] = p @ v[:, h, :]
+    assert np.all(np.diff(chunk_id) >= 0), "chunk ids must be non-decreasing"
+    for c in np.unique(chunk_id):
+        rows = np.nonzero(chunk_id == c)[0]
+        end = int(np.nonzero(chunk_id <= c)[0].max()) + 1      # keys j with c(j) <= c
+        for h in range(nh):
+            sc = (q[rows, h, :] @ k[:end, h, :].T) / math.sqrt(dh)
+            sc = sc - sc.max(axis=1, keepdims=True)
+            p = np.exp(sc)
+            p = p / p.sum(axis=1, keepdims=True)
+            out[rows, h, :] = p @ v[:end, h, :]
     return out
 
 
@@ -322,10 +350,10 @@ def repair_request(kv: np.ndarray, emb: np.ndarray, chunk_id: np.ndarray, pos: n
     dtype; the result's `repaired` is the exact repaired cache, to be
     rounded with `round_to_cache` for a bit-level comparison.
     """
-    kv64 = dtype_to_f64(kv, cache_dtype)
+    w = {k_: (_bf16_mat(v_) if v_.dtype == np.uint16 else v_) for k_, v_ in w.items()}
     emb64 = dtype_to_f64(emb, cache_dtype)
-    s = stale_encoder(kv64, w["sigma_stale"], w["w_seg"], w["b_seg"], w["w_map"], w["b_map"],
-                      head_dim)
+    s = stale_encoder(kv, w["sigma_stale"], w["w_seg"], w["b_seg"], w["w_map"], w["b_map"],
+                      head_dim, cache_dtype=cache_dtype)
     h0 = token_fusion(s, emb64, w["w_tok"], w["b_tok"], w["w_fuse"], w["b_fuse"])
     rein = [reinjection(s, w["w_rein"][b], w["b_rein"][b]) for b in range(w["w_rein"].shape[0])]
     blocks: List[np.ndarray] = []
@@ -334,7 +362,8 @@ def repair_request(kv: np.ndarray, emb: np.ndarray, chunk_id: np.ndarray, pos: n
     z = rep = rot = None
     if with_head:
         z = residual_head(hB, w["lnf_g"], w["lnf_b"], w["w_out"], w["b_out"], eps, cols=head_cols)
-        base = kv64 if head_cols is None else kv64[:, head_cols]
+        kv64 = dtype_to_f64(kv if head_cols is None else kv[:, head_cols], cache_dtype)
+        base = kv64
         sd = w["sigma_delta"] if head_cols is None else w["sigma_delta"][head_cols]
         rep = apply_residual(base, z, sd)
         if inv_freq_target is not None and head_cols is None:

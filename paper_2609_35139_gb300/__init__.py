@@ -1,0 +1,9 @@
+"""GB300-native (sm_103a) CacheRepair online repair path.
+
+The compute lives in libcacherepair.so (csrc/, C ABI in include/cr.h); this
+package is its build script and a ctypes binding with the same names.
+"""
+from . import build, cr  # noqa: F401
+from .session import RepairSession, pack_host_weights, host_to_device, dims_from  # noqa: F401
+
+__all__ = ["build", "cr", "RepairSession", "pack_host_weights", "host_to_device", "dims_from"]

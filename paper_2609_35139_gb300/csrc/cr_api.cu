@@ -1,0 +1,644 @@
+// C ABI of the repair library (include/cr.h, include/cr_ops.h): host-side
+// validation, workspace carving and the launch sequence of each call.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <mutex>
+#include <string.h>
+
+#include "cr_internal.h"
+
+// Device status word (first error code, site, block); one copy per device
+// that loads the library.  Kernels receive its address as a parameter.
+__device__ unsigned g_cr_status[4];
+
+namespace cr {
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_mu;
+unsigned* g_status_ptr[kMaxDevices];
+int g_sms[kMaxDevices];
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+int current_device() {
+    int d = -1;
+    if (cudaGetDevice(&d) != cudaSuccess || d < 0 || d >= kMaxDevices) return -1;
+    return d;
+}
+
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+struct Dims {
+    int64_t L, H, dh, dmodel, S, D;
+    bool f32;
+    int64_t dseg, dc, db, B, nh, hd, hid;
+};
+
+Dims dims_of(const cr_target_dims* t, const cr_repairer_dims* r) {
+    Dims d{};
+    d.L = t->n_layers;
+    d.H = t->n_kv_heads;
+    d.dh = t->head_dim;
+    d.dmodel = t->d_model;
+    d.S = 2 * d.L * d.H;
+    d.D = d.S * d.dh;
+    d.f32 = t->cache_dtype == CR_F32;
+    if (r) {
+        d.dseg = r->d_seg;
+        d.dc = r->d_c;
+        d.db = r->d_b;
+        d.B = r->n_blocks;
+        d.nh = r->n_heads;
+        d.hd = r->n_heads > 0 ? r->d_b / r->n_heads : 0;
+        d.hid = r->mlp_hidden;
+    }
+    return d;
+}
+
+cr_status check_target(const cr_target_dims* t) {
+    if (!t) return CR_ERR_INVALID_ARG;
+    if (t->n_layers < 1 || t->n_kv_heads < 1 || t->d_model < 8 || (t->d_model % 8) != 0)
+        return CR_ERR_INVALID_ARG;
+    if (t->cache_dtype != CR_F32 && t->cache_dtype != CR_BF16) return CR_ERR_INVALID_ARG;
+    if (t->head_dim != 64 && t->head_dim != 128) return CR_ERR_UNSUPPORTED;
+    return CR_OK;
+}
+
+cr_status check_repairer(const cr_repairer_dims* r) {
+    if (!r) return CR_ERR_INVALID_ARG;
+    if (r->n_blocks < 0 || r->n_blocks > 64 || r->n_heads < 1 || r->d_c < 16 ||
+        r->mlp_hidden < 16 || !(r->ln_eps > 0.0f) || !(r->rope_theta > 0.0f))
+        return CR_ERR_INVALID_ARG;
+    if (r->d_b % r->n_heads != 0) return CR_ERR_INVALID_ARG;
+    if (r->d_seg != 8 && r->d_seg != 16) return CR_ERR_UNSUPPORTED;
+    if (r->d_c % 16 != 0 || r->mlp_hidden % 16 != 0) return CR_ERR_UNSUPPORTED;
+    if (r->d_b % 128 != 0 || r->d_b > 1024 || r->d_b < 128) return CR_ERR_UNSUPPORTED;
+    const int hd = r->d_b / r->n_heads;
+    if (hd != 32 && hd != 64) return CR_ERR_UNSUPPORTED;
+    return CR_OK;
+}
+
+struct WsLayout {
+    size_t wfold, kvb, embb, y, se, x, u, qkv, o, g, total;
+};
+
+WsLayout ws_layout(const Dims& d, int64_t n) {
+    WsLayout w{};
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        const size_t o = off;
+        off += align256(bytes);
+        return o;
+    };
+    const size_t N = static_cast<size_t>(n);
+    w.wfold = take(static_cast<size_t>(d.S * d.dseg * d.dh) * 2);
+    w.kvb = take(d.f32 ? N * d.D * 2 : 0);
+    w.embb = take(d.f32 ? N * d.dmodel * 2 : 0);
+    w.y = take(N * d.S * d.dseg * 2);
+    w.se = take(N * 2 * d.dc * 2);
+    w.x = take(N * d.db * 4);
+    w.u = take(N * d.db * 2);
+    w.qkv = take(N * 3 * d.db * 2);
+    w.o = take(N * d.db * 2);
+    w.g = take(N * d.hid * 2);
+    w.total = off;
+    return w;
+}
+
+template <typename T>
+T* at(void* base, size_t off) {
+    return reinterpret_cast<T*>(static_cast<uint8_t*>(base) + off);
+}
+
+void repairer_inv_freq(float* out, int dim, float theta) {
+    for (int i = 0; i < dim / 2; ++i)
+        out[i] = static_cast<float>(pow(static_cast<double>(theta), -2.0 * i / dim));
+}
+
+bool all_aligned() { return true; }
+template <typename P, typename... R>
+bool all_aligned(const P* p, R... rest) {
+    return p != nullptr && aligned16(p) && all_aligned(rest...);
+}
+
+}  // namespace
+
+cr_status cuda_check(cudaError_t e) { return e == cudaSuccess ? CR_OK : CR_ERR_CUDA; }
+
+int current_device_index() { return current_device(); }
+
+unsigned* device_status_ptr() {
+    const int d = current_device();
+    if (d < 0) return nullptr;
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (!g_status_ptr[d]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_cr_status) != cudaSuccess) return nullptr;
+        g_status_ptr[d] = static_cast<unsigned*>(p);
+    }
+    return g_status_ptr[d];
+}
+
+int num_sms() {
+    const int d = current_device();
+    if (d < 0) return 1;
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (!g_sms[d]) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, d) != cudaSuccess || n < 1)
+            n = 1;
+        g_sms[d] = n;
+    }
+    return g_sms[d];
+}
+
+bool make_tmap_2d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, uint64_t inner,
+                  uint64_t outer, uint64_t row_stride_bytes, uint32_t box_inner,
+                  uint32_t box_outer, CUtensorMapSwizzle swz) {
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        if (!g_encode) {
+            void* fn = nullptr;
+            cudaDriverEntryPointQueryResult q;
+            if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                                 cudaEnableDefault, &q) != cudaSuccess ||
+                q != cudaDriverEntryPointSuccess || !fn)
+                return false;
+            g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+        }
+    }
+    if (!aligned16(base) || (row_stride_bytes % 16) != 0 || inner == 0 || outer == 0) return false;
+    const cuuint64_t dims[2] = {inner, outer};
+    const cuuint64_t strides[1] = {row_stride_bytes};
+    const cuuint32_t box[2] = {box_inner, box_outer};
+    const cuuint32_t estr[2] = {1, 1};
+    return g_encode(m, dt, 2, const_cast<void*>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace cr
+
+using namespace cr;
+
+extern "C" {
+
+const char* cr_status_str(cr_status s) {
+    switch (s) {
+        case CR_OK: return "ok";
+        case CR_ERR_INVALID_ARG: return "invalid argument";
+        case CR_ERR_UNSUPPORTED: return "unsupported shape";
+        case CR_ERR_CUDA: return "CUDA error";
+        case CR_ERR_DEVICE_INDEX: return "device-detected index out of range";
+        case CR_ERR_TIMEOUT: return "device pipeline wait timed out";
+    }
+    return "unknown status";
+}
+
+cr_status cr_get_device_status(uint32_t out[3]) {
+    if (!out) return CR_ERR_INVALID_ARG;
+    unsigned h[4] = {0, 0, 0, 0};
+    if (cudaDeviceSynchronize() != cudaSuccess) return CR_ERR_CUDA;
+    if (cudaMemcpyFromSymbol(h, g_cr_status, sizeof(h)) != cudaSuccess) return CR_ERR_CUDA;
+    out[0] = h[0];
+    out[1] = h[1];
+    out[2] = h[2];
+    if (h[0] == CR_DEV_TIMEOUT) return CR_ERR_TIMEOUT;
+    if (h[0] == CR_DEV_INDEX) return CR_ERR_DEVICE_INDEX;
+    return CR_OK;
+}
+
+cr_status cr_clear_device_status(void) {
+    const unsigned z[4] = {0, 0, 0, 0};
+    if (cudaMemcpyToSymbol(g_cr_status, z, sizeof(z)) != cudaSuccess) return CR_ERR_CUDA;
+    return cudaDeviceSynchronize() == cudaSuccess ? CR_OK : CR_ERR_CUDA;
+}
+
+size_t cr_workspace_bytes(const cr_target_dims* target, const cr_repairer_dims* rep,
+                          int64_t max_tokens) {
+    if (check_target(target) != CR_OK || check_repairer(rep) != CR_OK || max_tokens < 0) return 0;
+    return ws_layout(dims_of(target, rep), max_tokens).total;
+}
+
+cr_status cr_assemble_stale(const cr_target_dims* target, const void* kv_pool,
+                            const void* emb_pool, int64_t n_pool_tokens,
+                            const int64_t* chunk_start, const int32_t* chunk_len,
+                            int32_t n_pool_chunks, const int32_t* chunk_idx,
+                            const int32_t* cu_chunks, int32_t n_req, void* kv_out,
+                            void* emb_out, int64_t max_tokens, int32_t* chunk_id,
+                            int32_t* chunk_end, int32_t* pos, int32_t* cu_seqlens_dev,
+                            int32_t* cu_seqlens_host, void* stream) {
+    cr_status s = check_target(target);
+    if (s != CR_OK) return s;
+    if (!chunk_start || !chunk_len || !chunk_idx || !cu_chunks || !cu_seqlens_host)
+        return CR_ERR_INVALID_ARG;
+    if (n_req < 1 || n_req > kMaxReq || n_pool_chunks < 1 || n_pool_tokens < 1)
+        return CR_ERR_INVALID_ARG;
+    if (!all_aligned(kv_pool, emb_pool, kv_out, emb_out, chunk_id, chunk_end, pos, cu_seqlens_dev))
+        return CR_ERR_INVALID_ARG;
+    const Dims d = dims_of(target, nullptr);
+    const int64_t es = d.f32 ? 4 : 2;
+    GatherParams* p = new GatherParams();   // ~17 KB: keep it off the caller's stack
+    memset(p, 0, sizeof(*p));
+    if (cu_chunks[0] != 0) {
+        delete p;
+        return CR_ERR_INVALID_ARG;
+    }
+    int64_t t = 0;
+    int n_seg = 0;
+    p->cu_seqlens_host[0] = 0;
+    for (int r = 0; r < n_req; ++r) {
+        const int a = cu_chunks[r], b = cu_chunks[r + 1];
+        if (b <= a || b - a > kMaxSegs) {
+            delete p;
+            return CR_ERR_INVALID_ARG;
+        }
+        int64_t local = 0;
+        for (int k = a; k < b; ++k) {
+            const int c = chunk_idx[k];
+            if (c < 0 || c >= n_pool_chunks || n_seg >= kMaxSegs) {
+                delete p;
+                return CR_ERR_INVALID_ARG;
+            }
+            const int64_t st = chunk_start[c], ln = chunk_len[c];
+            if (ln < 1 || st < 0 || st + ln > n_pool_tokens) {
+                delete p;
+                return CR_ERR_INVALID_ARG;
+            }
+            GatherSeg& g = p->seg[n_seg++];
+            g.src_row = st;
+            g.dst_row = t;
+            g.len = static_cast<int32_t>(ln);
+            g.chunk_local = k - a;
+            g.local_start = static_cast<int32_t>(local);
+            local += ln;
+            t += ln;
+            if (local > INT32_MAX / 2) {
+                delete p;
+                return CR_ERR_INVALID_ARG;
+            }
+        }
+        p->cu_seqlens_host[r + 1] = static_cast<int32_t>(t);
+    }
+    if (t > max_tokens || t > INT32_MAX / 2) {
+        delete p;
+        return CR_ERR_INVALID_ARG;
+    }
+    p->kv_pool = static_cast<const uint8_t*>(kv_pool);
+    p->emb_pool = static_cast<const uint8_t*>(emb_pool);
+    p->kv_out = static_cast<uint8_t*>(kv_out);
+    p->emb_out = static_cast<uint8_t*>(emb_out);
+    p->kv_row_bytes = d.D * es;
+    p->emb_row_bytes = d.dmodel * es;
+    p->chunk_id = chunk_id;
+    p->chunk_end = chunk_end;
+    p->pos = pos;
+    p->cu_seqlens = cu_seqlens_dev;
+    p->n_tokens = t;
+    p->n_pool_tokens = n_pool_tokens;
+    p->n_seg = n_seg;
+    p->n_req = n_req;
+    p->status = device_status_ptr();
+    for (int r = 0; r <= n_req; ++r) cu_seqlens_host[r] = p->cu_seqlens_host[r];
+    s = p->status ? launch_gather(*p, static_cast<cudaStream_t>(stream)) : CR_ERR_CUDA;
+    delete p;
+    return s;
+}
+
+static cr_status check_weights_compress(const Dims& d, const cr_weights* w) {
+    if (!w) return CR_ERR_INVALID_ARG;
+    if (!all_aligned(w->w_seg, w->b_seg, w->w_map, w->b_map, w->w_tok, w->b_tok, w->w_fuse,
+                     w->b_fuse, w->sigma_stale))
+        return CR_ERR_INVALID_ARG;
+    if (d.B > 0 && !all_aligned(w->w_rein, w->b_rein)) return CR_ERR_INVALID_ARG;
+    return CR_OK;
+}
+
+cr_status cr_compress_features(const cr_target_dims* target, const cr_repairer_dims* rep,
+                               const cr_weights* w, const void* kv, const void* emb,
+                               int64_t n_tokens, float* h0_out, uint16_t* rein_out,
+                               void* workspace, size_t workspace_bytes, void* stream) {
+    cr_status s = check_target(target);
+    if (s == CR_OK) s = check_repairer(rep);
+    if (s != CR_OK) return s;
+    const Dims d = dims_of(target, rep);
+    if (n_tokens < 1 || n_tokens > INT32_MAX / 2) return CR_ERR_INVALID_ARG;
+    if ((s = check_weights_compress(d, w)) != CR_OK) return s;
+    if (!all_aligned(kv, emb, h0_out, workspace)) return CR_ERR_INVALID_ARG;
+    if (d.B > 0 && !all_aligned(rein_out)) return CR_ERR_INVALID_ARG;
+    const WsLayout L = ws_layout(d, n_tokens);
+    if (workspace_bytes < L.total) return CR_ERR_INVALID_ARG;
+    unsigned* status = device_status_ptr();
+    if (!status) return CR_ERR_CUDA;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int64_t N = n_tokens;
+
+    uint16_t* wfold = at<uint16_t>(workspace, L.wfold);
+    if ((s = launch_fold_sigma(w->w_seg, w->sigma_stale, static_cast<int>(d.S),
+                               static_cast<int>(d.dseg), static_cast<int>(d.dh), wfold, st)) != CR_OK)
+        return s;
+    const uint16_t* kvb = static_cast<const uint16_t*>(kv);
+    const uint16_t* embb = static_cast<const uint16_t*>(emb);
+    if (d.f32) {
+        uint16_t* k2 = at<uint16_t>(workspace, L.kvb);
+        uint16_t* e2 = at<uint16_t>(workspace, L.embb);
+        if ((s = launch_to_bf16(static_cast<const float*>(kv), N * d.D, k2, st)) != CR_OK) return s;
+        if ((s = launch_to_bf16(static_cast<const float*>(emb), N * d.dmodel, e2, st)) != CR_OK)
+            return s;
+        kvb = k2;
+        embb = e2;
+    }
+    uint16_t* y = at<uint16_t>(workspace, L.y);
+    SegParams sp{};
+    sp.M = static_cast<int32_t>(N);
+    sp.S = static_cast<int32_t>(d.S);
+    sp.d_seg = static_cast<int32_t>(d.dseg);
+    sp.b_seg = w->b_seg;
+    sp.y = y;
+    sp.status = status;
+    if ((s = launch_segproj(kvb, d.D, wfold, static_cast<int>(d.dh), sp, st)) != CR_OK) return s;
+
+    uint16_t* se = at<uint16_t>(workspace, L.se);   // [N, 2 d_c] = [s ; P_tok E]
+    GemmParams gp{};
+    gp.status = status;
+    gp.bias = w->b_map;
+    gp.out = se;
+    gp.ldo = 2 * d.dc;
+    if ((s = launch_gemm(y, d.S * d.dseg, w->w_map, N, d.dc, d.S * d.dseg, EPI_BF16, gp, nullptr,
+                         0, st)) != CR_OK)
+        return s;
+    gp.bias = w->b_tok;
+    gp.out = se + d.dc;
+    if ((s = launch_gemm(embb, d.dmodel, w->w_tok, N, d.dc, d.dmodel, EPI_BF16, gp, nullptr, 0,
+                         st)) != CR_OK)
+        return s;
+    gp.bias = w->b_fuse;
+    gp.out = h0_out;
+    gp.ldo = d.db;
+    if ((s = launch_gemm(se, 2 * d.dc, w->w_fuse, N, d.db, 2 * d.dc, EPI_F32, gp, nullptr, 0,
+                         st)) != CR_OK)
+        return s;
+    if (d.B > 0) {
+        gp.bias = w->b_rein;
+        gp.out = rein_out;
+        gp.ldo = d.B * d.db;
+        if ((s = launch_gemm(se, 2 * d.dc, w->w_rein, N, d.B * d.db, d.dc, EPI_BF16, gp, nullptr,
+                             0, st)) != CR_OK)
+            return s;
+    }
+    return CR_OK;
+}
+
+static cr_status attn_params(const Dims& d, const int32_t* chunk_end,
+                             const int32_t* cu_seqlens_host, int n_req, int64_t N, uint16_t* out,
+                             unsigned* status, AttnParams* p) {
+    if (!cu_seqlens_host || n_req < 1 || n_req > kMaxReq) return CR_ERR_INVALID_ARG;
+    if (cu_seqlens_host[0] != 0 || cu_seqlens_host[n_req] != N) return CR_ERR_INVALID_ARG;
+    memset(p, 0, sizeof(*p));
+    int items = 0;
+    for (int r = 0; r < n_req; ++r) {
+        const int len = cu_seqlens_host[r + 1] - cu_seqlens_host[r];
+        if (len < 1) return CR_ERR_INVALID_ARG;
+        p->req_start[r] = cu_seqlens_host[r];
+        p->tile_prefix[r] = items;
+        items += (len + 127) / 128;
+    }
+    p->req_start[n_req] = cu_seqlens_host[n_req];
+    p->tile_prefix[n_req] = items;
+    p->chunk_end = chunk_end;
+    p->out = out;
+    p->d_b = static_cast<int32_t>(d.db);
+    p->n_heads = static_cast<int32_t>(d.nh);
+    p->n_req = n_req;
+    p->n_items = items;
+    p->scale_log2 = static_cast<float>(1.4426950408889634 / sqrt(static_cast<double>(d.hd)));
+    p->status = status;
+    return CR_OK;
+}
+
+cr_status cr_repair_forward(const cr_target_dims* target, const cr_repairer_dims* rep,
+                            const cr_weights* w, const float* h0, const uint16_t* rein,
+                            const int32_t* chunk_end, const int32_t* pos,
+                            const int32_t* cu_seqlens_host, int32_t n_req, int64_t n_tokens,
+                            uint16_t* yf_out, void* workspace, size_t workspace_bytes,
+                            void* stream) {
+    cr_status s = check_target(target);
+    if (s == CR_OK) s = check_repairer(rep);
+    if (s != CR_OK) return s;
+    const Dims d = dims_of(target, rep);
+    if (!w || n_tokens < 1 || n_tokens > INT32_MAX / 2) return CR_ERR_INVALID_ARG;
+    if (!all_aligned(h0, chunk_end, pos, yf_out, workspace, w->lnf_g, w->lnf_b))
+        return CR_ERR_INVALID_ARG;
+    if (d.B > 0 && (!w->blocks || !all_aligned(rein))) return CR_ERR_INVALID_ARG;
+    for (int b = 0; b < d.B; ++b) {
+        const cr_block_weights& k = w->blocks[b];
+        if (!all_aligned(k.ln1_g, k.ln1_b, k.w_qkv, k.b_qkv, k.w_o, k.b_o, k.ln2_g, k.ln2_b,
+                         k.w_fc1, k.b_fc1, k.w_fc2, k.b_fc2))
+            return CR_ERR_INVALID_ARG;
+    }
+    const WsLayout L = ws_layout(d, n_tokens);
+    if (workspace_bytes < L.total) return CR_ERR_INVALID_ARG;
+    const int64_t N = n_tokens;
+    float* x = at<float>(workspace, L.x);
+    uint16_t* u = at<uint16_t>(workspace, L.u);
+    uint16_t* qkv = at<uint16_t>(workspace, L.qkv);
+    uint16_t* o = at<uint16_t>(workspace, L.o);
+    uint16_t* g = at<uint16_t>(workspace, L.g);
+    AttnParams* ap = new AttnParams();
+    s = attn_params(d, chunk_end, cu_seqlens_host, n_req, N, o, nullptr, ap);
+    unsigned* status = (s == CR_OK) ? device_status_ptr() : nullptr;
+    if (s == CR_OK && !status) s = CR_ERR_CUDA;
+    if (s != CR_OK) {
+        delete ap;
+        return s;
+    }
+    ap->status = status;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    GemmParams gq{};
+    gq.status = status;
+    gq.pos = pos;
+    gq.rope_dim = static_cast<int32_t>(d.hd);
+    gq.rope_cols = static_cast<int32_t>(2 * d.db);
+    repairer_inv_freq(gq.inv_freq, static_cast<int>(d.hd), rep->rope_theta);
+    GemmParams gr{};
+    gr.status = status;
+    for (int b = 0; b < d.B && s == CR_OK; ++b) {
+        const cr_block_weights& k = w->blocks[b];
+        // x = h^{b-1} + P_b(s);  u = LN1(x)
+        s = launch_layernorm(b == 0 ? h0 : x, rein + b * d.db, d.B * d.db, x, k.ln1_g, k.ln1_b,
+                             rep->ln_eps, N, d.db, u, st);
+        if (s != CR_OK) break;
+        gq.bias = k.b_qkv;
+        gq.out = qkv;
+        gq.ldo = 3 * d.db;
+        s = launch_gemm(u, d.db, k.w_qkv, N, 3 * d.db, d.db, EPI_QKV_ROPE, gq, nullptr, 0, st);
+        if (s != CR_OK) break;
+        s = launch_attention(qkv, N, static_cast<int>(d.hd), *ap, st);
+        if (s != CR_OK) break;
+        gr.bias = k.b_o;
+        gr.out = x;
+        gr.ldo = d.db;
+        s = launch_gemm(o, d.db, k.w_o, N, d.db, d.db, EPI_ADD_F32, gr, nullptr, 0, st);
+        if (s != CR_OK) break;
+        s = launch_layernorm(x, nullptr, 0, x, k.ln2_g, k.ln2_b, rep->ln_eps, N, d.db, u, st);
+        if (s != CR_OK) break;
+        gr.bias = k.b_fc1;
+        gr.out = g;
+        gr.ldo = d.hid;
+        s = launch_gemm(u, d.db, k.w_fc1, N, d.hid, d.db, EPI_GELU_BF16, gr, nullptr, 0, st);
+        if (s != CR_OK) break;
+        gr.bias = k.b_fc2;
+        gr.out = x;
+        gr.ldo = d.db;
+        s = launch_gemm(g, d.hid, k.w_fc2, N, d.db, d.hid, EPI_ADD_F32, gr, nullptr, 0, st);
+    }
+    delete ap;
+    if (s != CR_OK) return s;
+    return launch_layernorm(d.B > 0 ? x : h0, nullptr, 0, nullptr, w->lnf_g, w->lnf_b,
+                            rep->ln_eps, N, d.db, yf_out, st);
+}
+
+cr_status cr_apply_residual(const cr_target_dims* target, const cr_repairer_dims* rep,
+                            const cr_weights* w, const uint16_t* yf, int64_t n_tokens,
+                            void* kv_inout, const int32_t* pos, const float* inv_freq_host,
+                            int32_t rope_mode, void* stream) {
+    cr_status s = check_target(target);
+    if (s == CR_OK) s = check_repairer(rep);
+    if (s != CR_OK) return s;
+    const Dims d = dims_of(target, rep);
+    if (!w || n_tokens < 1 || n_tokens > INT32_MAX / 2) return CR_ERR_INVALID_ARG;
+    if (rope_mode != CR_ROPE_NONE && rope_mode != CR_ROPE_GLOBAL) return CR_ERR_INVALID_ARG;
+    if (!all_aligned(yf, kv_inout, pos, w->w_out, w->b_out, w->sigma_delta))
+        return CR_ERR_INVALID_ARG;
+    if (rope_mode == CR_ROPE_GLOBAL && !inv_freq_host) return CR_ERR_INVALID_ARG;
+    const int bn = d.f32 ? 128 : 256;
+    if (d.D % bn != 0) return CR_ERR_UNSUPPORTED;
+    unsigned* status = device_status_ptr();
+    if (!status) return CR_ERR_CUDA;
+    GemmParams gp{};
+    gp.status = status;
+    gp.bias = w->b_out;
+    gp.sigma = w->sigma_delta;
+    gp.pos = pos;
+    gp.rope_dim = static_cast<int32_t>(d.dh);
+    gp.rope_on = rope_mode == CR_ROPE_GLOBAL ? 1 : 0;
+    gp.n_kv_heads = static_cast<int32_t>(d.H);
+    if (gp.rope_on)
+        for (int i = 0; i < d.dh / 2; ++i) gp.inv_freq[i] = inv_freq_host[i];
+    return launch_gemm(yf, d.db, w->w_out, n_tokens, d.D, d.db, d.f32 ? EPI_KV_F32 : EPI_KV_BF16,
+                       gp, kv_inout, d.D, static_cast<cudaStream_t>(stream));
+}
+
+// ------------------------------------------------------------------ cr_ops.h
+cr_status cr_linear(const uint16_t* A, int64_t lda, const uint16_t* W, const float* bias,
+                    int64_t M, int64_t N, int64_t K, void* out, int64_t ldo, int32_t epi,
+                    void* stream) {
+    if (M < 1 || N < 1 || K < 8 || (K % 8) != 0 || (N % 16) != 0 || lda < K || ldo < N)
+        return CR_ERR_INVALID_ARG;
+    if (M > INT32_MAX / 2 || N > INT32_MAX / 2 || K > INT32_MAX / 2) return CR_ERR_INVALID_ARG;
+    if (epi < CR_EPI_BF16 || epi > CR_EPI_F32) return CR_ERR_INVALID_ARG;
+    if (!all_aligned(A, W, out) || (bias && !aligned16(bias))) return CR_ERR_INVALID_ARG;
+    const int64_t es = (epi == CR_EPI_ADD_F32 || epi == CR_EPI_F32) ? 4 : 2;
+    if ((lda * 2) % 16 != 0 || (ldo * es) % 16 != 0) return CR_ERR_INVALID_ARG;
+    unsigned* status = device_status_ptr();
+    if (!status) return CR_ERR_CUDA;
+    GemmParams gp{};
+    gp.status = status;
+    gp.bias = bias;
+    gp.out = out;
+    gp.ldo = ldo;
+    static const int map[4] = {EPI_BF16, EPI_GELU_BF16, EPI_ADD_F32, EPI_F32};
+    return launch_gemm(A, lda, W, M, N, K, map[epi], gp, nullptr, 0,
+                       static_cast<cudaStream_t>(stream));
+}
+
+cr_status cr_layernorm(const float* x, const uint16_t* add, int64_t ld_add, float* x_out,
+                       const float* gamma, const float* beta, float eps, int64_t M, int64_t D,
+                       uint16_t* u, void* stream) {
+    if (M < 1 || D < 128 || D > 1024 || (D % 128) != 0 || !(eps > 0.0f)) return CR_ERR_INVALID_ARG;
+    if (!all_aligned(x, gamma, beta, u)) return CR_ERR_INVALID_ARG;
+    if (add && (!all_aligned(add, x_out) || ld_add < D || (ld_add % 8) != 0))
+        return CR_ERR_INVALID_ARG;
+    return launch_layernorm(x, add, ld_add, x_out, gamma, beta, eps, M, D, u,
+                            static_cast<cudaStream_t>(stream));
+}
+
+cr_status cr_chunk_causal_attention(const uint16_t* qkv, int32_t d_b, int32_t n_heads,
+                                    const int32_t* chunk_end, const int32_t* cu_seqlens_host,
+                                    int32_t n_req, int64_t n_tokens, uint16_t* out,
+                                    void* stream) {
+    if (n_heads < 1 || d_b < 1 || d_b % n_heads != 0 || n_tokens < 1 || n_tokens > INT32_MAX / 2)
+        return CR_ERR_INVALID_ARG;
+    const int hd = d_b / n_heads;
+    if (hd != 32 && hd != 64) return CR_ERR_UNSUPPORTED;
+    if (!all_aligned(qkv, chunk_end, out)) return CR_ERR_INVALID_ARG;
+    Dims d{};
+    d.db = d_b;
+    d.nh = n_heads;
+    d.hd = hd;
+    AttnParams* ap = new AttnParams();
+    cr_status s = attn_params(d, chunk_end, cu_seqlens_host, n_req, n_tokens, out, nullptr, ap);
+    if (s == CR_OK) {
+        ap->status = device_status_ptr();
+        s = ap->status ? launch_attention(qkv, n_tokens, hd, *ap, static_cast<cudaStream_t>(stream))
+                       : CR_ERR_CUDA;
+    }
+    delete ap;
+    return s;
+}
+
+cr_status cr_qkv_rope(const uint16_t* u, const uint16_t* w_qkv, const float* b_qkv,
+                      const int32_t* pos, int64_t n_tokens, int32_t d_b, int32_t n_heads,
+                      float rope_theta, uint16_t* qkv, void* stream) {
+    if (n_heads < 1 || d_b < 128 || d_b % 128 != 0 || d_b % n_heads != 0 || n_tokens < 1 ||
+        n_tokens > INT32_MAX / 2 || !(rope_theta > 0.0f))
+        return CR_ERR_INVALID_ARG;
+    const int hd = d_b / n_heads;
+    if (hd != 32 && hd != 64) return CR_ERR_UNSUPPORTED;
+    if (!all_aligned(u, w_qkv, pos, qkv) || (b_qkv && !aligned16(b_qkv))) return CR_ERR_INVALID_ARG;
+    unsigned* status = device_status_ptr();
+    if (!status) return CR_ERR_CUDA;
+    GemmParams gq{};
+    gq.status = status;
+    gq.pos = pos;
+    gq.bias = b_qkv;
+    gq.out = qkv;
+    gq.ldo = 3 * d_b;
+    gq.rope_dim = hd;
+    gq.rope_cols = 2 * d_b;
+    repairer_inv_freq(gq.inv_freq, hd, rope_theta);
+    return launch_gemm(u, d_b, w_qkv, n_tokens, 3 * d_b, d_b, EPI_QKV_ROPE, gq, nullptr, 0,
+                       static_cast<cudaStream_t>(stream));
+}
+
+cr_status cr_segment_project(const cr_target_dims* target, int32_t d_seg, const uint16_t* kv,
+                             int64_t n_tokens, const uint16_t* w_seg, const float* b_seg,
+                             const float* sigma_stale, uint16_t* y, void* workspace,
+                             size_t workspace_bytes, void* stream) {
+    cr_status s = check_target(target);
+    if (s != CR_OK) return s;
+    if (d_seg != 8 && d_seg != 16) return CR_ERR_UNSUPPORTED;
+    if (n_tokens < 1 || n_tokens > INT32_MAX / 2) return CR_ERR_INVALID_ARG;
+    if (!all_aligned(kv, w_seg, b_seg, sigma_stale, y, workspace)) return CR_ERR_INVALID_ARG;
+    const Dims d = dims_of(target, nullptr);
+    if (workspace_bytes < static_cast<size_t>(d.S * d_seg * d.dh) * 2) return CR_ERR_INVALID_ARG;
+    unsigned* status = device_status_ptr();
+    if (!status) return CR_ERR_CUDA;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    uint16_t* wfold = static_cast<uint16_t*>(workspace);
+    if ((s = launch_fold_sigma(w_seg, sigma_stale, static_cast<int>(d.S), d_seg,
+                               static_cast<int>(d.dh), wfold, st)) != CR_OK)
+        return s;
+    SegParams sp{};
+    sp.M = static_cast<int32_t>(n_tokens);
+    sp.S = static_cast<int32_t>(d.S);
+    sp.d_seg = d_seg;
+    sp.b_seg = b_seg;
+    sp.y = y;
+    sp.status = status;
+    return launch_segproj(kv, d.D, wfold, static_cast<int>(d.dh), sp, st);
+}
+
+}  // extern "C"

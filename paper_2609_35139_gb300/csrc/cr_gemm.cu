@@ -1,0 +1,489 @@
+// tcgen05 GEMM for every dense linear of the repair path (Sec. 4.1):
+//   C[M, N] = A[M, K] * W[N, K]^T + bias, with a fused epilogue.
+//
+// Design (sm_103a, one CTA per SM, persistent):
+//   warp 0      TMA producer: A and W k-slices (64 wide, 128B swizzle) into a
+//               STAGES-deep shared-memory ring; for the residual epilogue also
+//               the stale cache tile [128, BN] of the output.
+//   warp 1      allocates TMEM, one elected lane issues tcgen05.mma
+//               (M = 128, N = BN, K = 16) into a double-buffered fp32
+//               accumulator (2 x BN TMEM columns), commits to mbarriers.
+//   warps 2..5  epilogue: tcgen05.ld 32 lanes x 16 columns, bias, then one of
+//               bf16 store / GELU / fp32 residual add / RoPE on Q,K /
+//               in-place "kv + sigma_delta * z" (+ R_M on K) on the staged
+//               cache tile, written back with TMA stores.
+// Tiles are walked W-tile-major (all M tiles of one N tile back to back), so
+// a W tile is read from HBM once and reused from L2 while the small A
+// operand stays L2-resident.
+#include <cuda_bf16.h>
+
+#include "cr_internal.h"
+#include "cr_ptx.cuh"
+
+namespace cr {
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 64;
+constexpr uint32_t A_BYTES = BM * BK * 2;
+
+template <int BN, int EPI>
+struct GemmCfg {
+    static constexpr bool kKV = (EPI == EPI_KV_BF16 || EPI == EPI_KV_F32);
+    static constexpr int kKVEsize = (EPI == EPI_KV_F32) ? 4 : 2;
+    static constexpr uint32_t kBBytes = BN * BK * 2;
+    static constexpr uint32_t kStageBytes = A_BYTES + kBBytes;
+    static constexpr int kStages = kKV ? (BN == 256 ? 3 : 4) : (BN == 256 ? 4 : 6);
+    static constexpr uint32_t kKVBytes = kKV ? BM * BN * kKVEsize : 0;
+    static constexpr int kKVBoxCols = 128 / kKVEsize;          // one 128-byte swizzle row
+    static constexpr int kKVBoxes = kKV ? BN / kKVBoxCols : 0;
+    static constexpr uint32_t kTmemCols = 2 * BN;
+    static constexpr uint32_t kSmemBytes = 1024 + kStages * kStageBytes + kKVBytes + 256;
+};
+
+__device__ __forceinline__ float gelu_erf(float x) {
+    return 0.5f * x * (1.0f + erff(x * 0.70710678118654752440f));
+}
+
+// 16 consecutive bf16 of a [128 x (64*k)] tile stored as 128B-swizzled boxes
+// of 64 columns; col multiple of 16.  Returns the byte offsets of its two
+// 16-byte chunks.
+__device__ __forceinline__ void swz_offsets_bf16(int row, int col, uint32_t* o0, uint32_t* o1) {
+    const int box = col >> 6;
+    const int ch = (col & 63) >> 3;
+    const uint32_t base = box * 16384 + row * 128;
+    *o0 = base + (((ch) ^ (row & 7)) << 4);
+    *o1 = base + (((ch + 1) ^ (row & 7)) << 4);
+}
+
+__device__ __forceinline__ void load16_bf16_smem(const uint8_t* tile, int row, int col, float* v) {
+    uint32_t o0, o1;
+    swz_offsets_bf16(row, col, &o0, &o1);
+    const uint4 a = *reinterpret_cast<const uint4*>(tile + o0);
+    const uint4 b = *reinterpret_cast<const uint4*>(tile + o1);
+    const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        v[2 * i] = __uint_as_float(w[i] << 16);
+        v[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+    }
+}
+
+__device__ __forceinline__ void store16_bf16_smem(uint8_t* tile, int row, int col, const float* v) {
+    uint32_t o0, o1;
+    swz_offsets_bf16(row, col, &o0, &o1);
+    uint4 a, b;
+    a.x = pack_bf16x2(v[0], v[1]);
+    a.y = pack_bf16x2(v[2], v[3]);
+    a.z = pack_bf16x2(v[4], v[5]);
+    a.w = pack_bf16x2(v[6], v[7]);
+    b.x = pack_bf16x2(v[8], v[9]);
+    b.y = pack_bf16x2(v[10], v[11]);
+    b.z = pack_bf16x2(v[12], v[13]);
+    b.w = pack_bf16x2(v[14], v[15]);
+    *reinterpret_cast<uint4*>(tile + o0) = a;
+    *reinterpret_cast<uint4*>(tile + o1) = b;
+}
+
+// fp32 tile: boxes of 32 columns (128 B rows), 4 chunks of 4 floats.
+__device__ __forceinline__ uint32_t swz_offset_f32(int row, int col, int k) {
+    const int box = col >> 5;
+    const int ch = ((col & 31) >> 2) + k;
+    return box * 16384 + row * 128 + ((ch ^ (row & 7)) << 4);
+}
+
+__device__ __forceinline__ void load16_f32_smem(const uint8_t* tile, int row, int col, float* v) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const float4 a = *reinterpret_cast<const float4*>(tile + swz_offset_f32(row, col, k));
+        v[4 * k] = a.x;
+        v[4 * k + 1] = a.y;
+        v[4 * k + 2] = a.z;
+        v[4 * k + 3] = a.w;
+    }
+}
+
+__device__ __forceinline__ void store16_f32_smem(uint8_t* tile, int row, int col, const float* v) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+        *reinterpret_cast<float4*>(tile + swz_offset_f32(row, col, k)) =
+            make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
+}
+
+__device__ __forceinline__ void store16_bf16_global(uint16_t* dst, const float* v) {
+    uint4 a, b;
+    a.x = pack_bf16x2(v[0], v[1]);
+    a.y = pack_bf16x2(v[2], v[3]);
+    a.z = pack_bf16x2(v[4], v[5]);
+    a.w = pack_bf16x2(v[6], v[7]);
+    b.x = pack_bf16x2(v[8], v[9]);
+    b.y = pack_bf16x2(v[10], v[11]);
+    b.z = pack_bf16x2(v[12], v[13]);
+    b.w = pack_bf16x2(v[14], v[15]);
+    reinterpret_cast<uint4*>(dst)[0] = a;
+    reinterpret_cast<uint4*>(dst)[1] = b;
+}
+
+__device__ __forceinline__ void add_bias16(float* v, const float* bias, int col) {
+    if (bias) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] += __ldg(bias + col + i);
+    }
+}
+
+__device__ __forceinline__ void rotate16(float* a, float* b, float p, const float* inv_freq, int j0) {
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        float s, c;
+        sincos_prod(p, inv_freq[j0 + i], &s, &c);
+        const float x = a[i], y = b[i];
+        a[i] = x * c - y * s;
+        b[i] = y * c + x * s;
+    }
+}
+
+template <int BN, int EPI>
+__global__ void __launch_bounds__(192, 1)
+    gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                const __grid_constant__ CUtensorMap tmC, const __grid_constant__ GemmParams p) {
+    using Cfg = GemmCfg<BN, EPI>;
+    constexpr int STAGES = Cfg::kStages;
+    constexpr uint32_t IDESC = idesc_bf16(BM, BN, false, false);
+
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    uint8_t* kv_tile = smem + STAGES * Cfg::kStageBytes;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(kv_tile + Cfg::kKVBytes);
+    uint64_t* full = bars;
+    uint64_t* empty = bars + STAGES;
+    uint64_t* tfull = bars + 2 * STAGES;
+    uint64_t* tempty = tfull + 2;
+    uint64_t* kvfull = tempty + 2;
+    uint64_t* kvempty = kvfull + 1;
+    uint64_t* drain = kvempty + 1;
+    uint64_t* epi_done = drain + 1;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(epi_done + 1);
+    int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
+
+    const uint32_t warp = warp_id(), lane = lane_id();
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&tfull[s], 1);
+            mbar_init(&tempty[s], 4);
+        }
+        mbar_init(kvfull, 1);
+        mbar_init(kvempty, 1);
+        mbar_init(drain, 1);
+        mbar_init(epi_done, 128);
+        *abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == 1) tmem_alloc(tmem_slot, Cfg::kTmemCols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+    const WaitCtx wc{abort_flag, p.status};
+
+    const int total = p.num_m * p.num_n;
+    const int num_k = (p.K + BK - 1) / BK;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ------------------------------------------------ TMA producer
+            tma_prefetch(&tmA);
+            tma_prefetch(&tmB);
+            if constexpr (Cfg::kKV) tma_prefetch(&tmC);
+            uint32_t stage = 0, phase = 0, kv_phase = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+                const int m0 = (t % p.num_m) * BM;
+                const int n0 = (t / p.num_m) * BN;
+                if constexpr (Cfg::kKV) {
+                    if (!(ok = mbar_wait(kvempty, kv_phase ^ 1u, wc, 101))) break;
+                    mbar_expect_tx(kvfull, Cfg::kKVBytes);
+                    for (int b = 0; b < Cfg::kKVBoxes; ++b)
+                        tma_load_2d(kv_tile + b * 16384, &tmC, kvfull, n0 + b * Cfg::kKVBoxCols,
+                                    m0);
+                    kv_phase ^= 1u;
+                }
+                for (int kb = 0; kb < num_k; ++kb) {
+                    if (!(ok = mbar_wait(&empty[stage], phase ^ 1u, wc, 102))) break;
+                    uint8_t* sa = smem + stage * Cfg::kStageBytes;
+                    mbar_expect_tx(&full[stage], Cfg::kStageBytes);
+                    tma_load_2d(sa, &tmA, &full[stage], kb * BK, m0);
+                    tma_load_2d(sa + A_BYTES, &tmB, &full[stage], kb * BK, n0);
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+            }
+            if (!ok) {  // let copies already in flight land before the CTA exits
+                const uint64_t t0 = globaltimer();
+                while (globaltimer() - t0 < 50000ull) {
+                }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // ------------------------------------------------ MMA issuer
+            uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+                if (!(ok = mbar_wait(&tempty[acc], acc_phase ^ 1u, wc, 201))) break;
+                tc_fence_after();
+                const uint32_t d = tmem_base + acc * BN;
+                for (int kb = 0; kb < num_k; ++kb) {
+                    if (!(ok = mbar_wait(&full[stage], phase, wc, 202))) break;
+                    tc_fence_after();
+                    const uint32_t sa = smem_u32(smem + stage * Cfg::kStageBytes);
+                    const uint32_t sb = sa + A_BYTES;
+#pragma unroll
+                    for (int k = 0; k < BK / 16; ++k) {
+                        const uint64_t da = smem_desc(sa + k * 32, 16, 1024, SWZ_128B);
+                        const uint64_t db = smem_desc(sb + k * 32, 16, 1024, SWZ_128B);
+                        mma_bf16_ss(d, da, db, IDESC, (kb | k) != 0 ? 1u : 0u);
+                    }
+                    mma_commit(&empty[stage]);
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+                if (!ok) break;
+                mma_commit(&tfull[acc]);
+                acc ^= 1u;
+                if (acc == 0) acc_phase ^= 1u;
+            }
+            // all MMAs of this thread retire before TMEM can be released
+            mma_commit(drain);
+            mbar_wait(drain, 0, wc, 203);
+        }
+    } else {
+        // ---------------------------------------------------- epilogue (warps 2..5)
+        const uint32_t quad = warp & 3u;
+        const int r = static_cast<int>(quad * 32 + lane);     // row inside the tile
+        uint32_t acc = 0, acc_phase = 0, kv_phase = 0;
+        for (int t = blockIdx.x; t < total; t += gridDim.x) {
+            const int m0 = (t % p.num_m) * BM;
+            const int n0 = (t / p.num_m) * BN;
+            bool ok = mbar_wait(&tfull[acc], acc_phase, wc, 301);
+            if constexpr (Cfg::kKV) ok = ok && mbar_wait(kvfull, kv_phase, wc, 302);
+            if (!__all_sync(0xffffffffu, ok)) break;
+            tc_fence_after();
+            const int row = m0 + r;
+            const bool row_ok = row < p.M;
+            const uint32_t taddr = tmem_base + ((quad * 32u) << 16) + acc * BN;
+
+            if constexpr (EPI == EPI_QKV_ROPE) {
+                const int hd = p.rope_dim;
+                const float pr = row_ok ? static_cast<float>(__ldg(p.pos + row)) : 0.0f;
+                uint16_t* orow = reinterpret_cast<uint16_t*>(p.out) + static_cast<int64_t>(row) * p.ldo;
+                for (int h0 = 0; h0 < BN; h0 += hd) {
+                    const bool rot = (n0 + h0) < p.rope_cols;
+                    for (int j = 0; j < hd / 2; j += 16) {
+                        float a[16], b[16];
+                        tmem_ld16(taddr + h0 + j, a);
+                        tmem_ld16(taddr + h0 + hd / 2 + j, b);
+                        tmem_wait_ld();
+                        const int ca = n0 + h0 + j, cb = n0 + h0 + hd / 2 + j;
+                        add_bias16(a, p.bias, ca);
+                        add_bias16(b, p.bias, cb);
+                        if (rot) rotate16(a, b, pr, p.inv_freq, j);
+                        if (row_ok) {
+                            store16_bf16_global(orow + ca, a);
+                            store16_bf16_global(orow + cb, b);
+                        }
+                    }
+                }
+            } else if constexpr (Cfg::kKV) {
+                const int dh = p.rope_dim;
+                const float pr = row_ok ? static_cast<float>(__ldg(p.pos + row)) : 0.0f;
+                for (int s0 = 0; s0 < BN; s0 += dh) {
+                    const int gseg = (n0 + s0) / dh;
+                    const bool rot = p.rope_on && (((gseg / p.n_kv_heads) & 1) == 0);
+                    for (int j = 0; j < dh / 2; j += 16) {
+                        float a[16], b[16], ka[16], kb[16];
+                        tmem_ld16(taddr + s0 + j, a);
+                        tmem_ld16(taddr + s0 + dh / 2 + j, b);
+                        const int ta = s0 + j, tb = s0 + dh / 2 + j;   // tile columns
+                        if constexpr (EPI == EPI_KV_BF16) {
+                            load16_bf16_smem(kv_tile, r, ta, ka);
+                            load16_bf16_smem(kv_tile, r, tb, kb);
+                        } else {
+                            load16_f32_smem(kv_tile, r, ta, ka);
+                            load16_f32_smem(kv_tile, r, tb, kb);
+                        }
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            const int ga = n0 + ta + i, gb = n0 + tb + i;
+                            ka[i] = fmaf(__ldg(p.sigma + ga), a[i] + __ldg(p.bias + ga), ka[i]);
+                            kb[i] = fmaf(__ldg(p.sigma + gb), b[i] + __ldg(p.bias + gb), kb[i]);
+                        }
+                        if (rot) rotate16(ka, kb, pr, p.inv_freq, j);
+                        if constexpr (EPI == EPI_KV_BF16) {
+                            store16_bf16_smem(kv_tile, r, ta, ka);
+                            store16_bf16_smem(kv_tile, r, tb, kb);
+                        } else {
+                            store16_f32_smem(kv_tile, r, ta, ka);
+                            store16_f32_smem(kv_tile, r, tb, kb);
+                        }
+                    }
+                }
+            } else {
+                for (int c = 0; c < BN; c += 16) {
+                    float v[16];
+                    __syncwarp();
+                    tmem_ld16(taddr + c, v);
+                    tmem_wait_ld();
+                    const int col = n0 + c;
+                    if (col >= p.N || !row_ok) continue;
+                    add_bias16(v, p.bias, col);
+                    if constexpr (EPI == EPI_BF16 || EPI == EPI_GELU_BF16) {
+                        if constexpr (EPI == EPI_GELU_BF16) {
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) v[i] = gelu_erf(v[i]);
+                        }
+                        store16_bf16_global(
+                            reinterpret_cast<uint16_t*>(p.out) + static_cast<int64_t>(row) * p.ldo + col, v);
+                    } else {
+                        float* o = reinterpret_cast<float*>(p.out) + static_cast<int64_t>(row) * p.ldo + col;
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            float4 x = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                            if constexpr (EPI == EPI_ADD_F32) {
+                                const float4 y = reinterpret_cast<const float4*>(o)[q];
+                                x.x += y.x;
+                                x.y += y.y;
+                                x.z += y.z;
+                                x.w += y.w;
+                            }
+                            reinterpret_cast<float4*>(o)[q] = x;
+                        }
+                    }
+                }
+            }
+            // accumulator buffer free for the MMA warp
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[acc]);
+            if constexpr (Cfg::kKV) {
+                // every epilogue thread's tile writes -> async proxy; then lane 0
+                // of warp 2, after a bounded wait for all 128 threads, stores the
+                // tile with TMA and hands the buffer back to the producer
+                fence_async_smem();
+                mbar_arrive(epi_done);
+                if (warp == 2) {
+                    bool ok2 = true;
+                    if (lane == 0) {
+                        ok2 = mbar_wait(epi_done, kv_phase, wc, 303);
+                        if (ok2) {
+                            for (int b = 0; b < Cfg::kKVBoxes; ++b)
+                                tma_store_2d(&tmC, kv_tile + b * 16384, n0 + b * Cfg::kKVBoxCols, m0);
+                            tma_store_commit();
+                            tma_store_wait_read0();
+                            mbar_arrive(kvempty);
+                        }
+                    }
+                    if (!__shfl_sync(0xffffffffu, ok2 ? 1 : 0, 0)) break;
+                }
+                kv_phase ^= 1u;
+            }
+            acc ^= 1u;
+            if (acc == 0) acc_phase ^= 1u;
+        }
+        if constexpr (Cfg::kKV) {
+            if (warp == 2 && lane == 0) tma_store_wait0();
+        }
+    }
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc(tmem_base, Cfg::kTmemCols);
+    }
+}
+
+template <int BN, int EPI>
+cr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
+                    const GemmParams& p, cudaStream_t st) {
+    using Cfg = GemmCfg<BN, EPI>;
+    auto kern = gemm_kernel<BN, EPI>;
+    static unsigned long long attr_done = 0;   // one per template instantiation
+    const cr_status sa = ensure_smem_attr(kern, static_cast<int>(Cfg::kSmemBytes), &attr_done);
+    if (sa != CR_OK) return sa;
+    const int tiles = p.num_m * p.num_n;
+    const int grid = tiles < num_sms() ? tiles : num_sms();
+    kern<<<grid, 192, Cfg::kSmemBytes, st>>>(ta, tb, tc, p);
+    return cuda_check(cudaGetLastError());
+}
+
+}  // namespace
+
+cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t M, int64_t N,
+                      int64_t K, int epi, GemmParams p, void* kv_base, int64_t ld_kv,
+                      cudaStream_t st) {
+    const bool kv = (epi == EPI_KV_BF16 || epi == EPI_KV_F32);
+    int BN;
+    if (epi == EPI_KV_F32)
+        BN = 128;
+    else if (kv)
+        BN = 256;
+    else
+        BN = (N >= 2048) ? 256 : 128;
+    if (kv && (N % BN) != 0) return CR_ERR_UNSUPPORTED;
+    if (epi == EPI_QKV_ROPE && (BN % p.rope_dim) != 0) return CR_ERR_UNSUPPORTED;
+    p.M = static_cast<int32_t>(M);
+    p.N = static_cast<int32_t>(N);
+    p.K = static_cast<int32_t>(K);
+    p.num_m = static_cast<int32_t>((M + BM - 1) / BM);
+    p.num_n = static_cast<int32_t>((N + BN - 1) / BN);
+    CUtensorMap ta, tb, tc;
+    if (!make_tmap_2d(&ta, A, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, K, M, lda * 2, BK, BM,
+                      CU_TENSOR_MAP_SWIZZLE_128B))
+        return CR_ERR_INVALID_ARG;
+    if (!make_tmap_2d(&tb, W, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, K, N, K * 2, BK, BN,
+                      CU_TENSOR_MAP_SWIZZLE_128B))
+        return CR_ERR_INVALID_ARG;
+    tc = ta;
+    if (kv) {
+        const bool f32 = (epi == EPI_KV_F32);
+        if (!make_tmap_2d(&tc, kv_base,
+                          f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                          N, M, ld_kv * (f32 ? 4 : 2), f32 ? 32 : 64, BM,
+                          CU_TENSOR_MAP_SWIZZLE_128B))
+            return CR_ERR_INVALID_ARG;
+    }
+    switch (epi) {
+        case EPI_BF16:
+            return BN == 256 ? launch_bn<256, EPI_BF16>(ta, tb, tc, p, st)
+                             : launch_bn<128, EPI_BF16>(ta, tb, tc, p, st);
+        case EPI_GELU_BF16:
+            return BN == 256 ? launch_bn<256, EPI_GELU_BF16>(ta, tb, tc, p, st)
+                             : launch_bn<128, EPI_GELU_BF16>(ta, tb, tc, p, st);
+        case EPI_ADD_F32:
+            return BN == 256 ? launch_bn<256, EPI_ADD_F32>(ta, tb, tc, p, st)
+                             : launch_bn<128, EPI_ADD_F32>(ta, tb, tc, p, st);
+        case EPI_F32:
+            return BN == 256 ? launch_bn<256, EPI_F32>(ta, tb, tc, p, st)
+                             : launch_bn<128, EPI_F32>(ta, tb, tc, p, st);
+        case EPI_QKV_ROPE:
+            return BN == 256 ? launch_bn<256, EPI_QKV_ROPE>(ta, tb, tc, p, st)
+                             : launch_bn<128, EPI_QKV_ROPE>(ta, tb, tc, p, st);
+        case EPI_KV_BF16:
+            return launch_bn<256, EPI_KV_BF16>(ta, tb, tc, p, st);
+        case EPI_KV_F32:
+            return launch_bn<128, EPI_KV_F32>(ta, tb, tc, p, st);
+        default:
+            return CR_ERR_INVALID_ARG;
+    }
+}
+
+}  // namespace cr

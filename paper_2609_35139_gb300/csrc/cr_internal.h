@@ -1,0 +1,140 @@
+// Internal declarations shared by the library's translation units.
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "cr.h"
+#include "cr_ops.h"
+
+// Device status codes (status word element 0).
+enum : unsigned { CR_DEV_OK = 0u, CR_DEV_TIMEOUT = 1u, CR_DEV_INDEX = 2u };
+
+namespace cr {
+
+constexpr int kMaxSegs = 512;   // selected chunks per cr_assemble_stale call
+constexpr int kMaxReq = 256;    // requests per call
+
+// ------------------------------------------------------------------ gather
+struct GatherSeg {
+    int64_t src_row;     // first pool row of the chunk
+    int64_t dst_row;     // first output row
+    int32_t len;         // rows
+    int32_t chunk_local; // c(t) of the chunk inside its request
+    int32_t local_start; // request-local position of the chunk's first token
+    int32_t pad;
+};
+struct GatherParams {
+    const uint8_t* kv_pool;
+    const uint8_t* emb_pool;
+    uint8_t* kv_out;
+    uint8_t* emb_out;
+    int64_t kv_row_bytes;
+    int64_t emb_row_bytes;
+    int32_t* chunk_id;
+    int32_t* chunk_end;
+    int32_t* pos;
+    int32_t* cu_seqlens;
+    int64_t n_tokens;
+    int64_t n_pool_tokens;
+    unsigned* status;
+    int32_t n_seg;
+    int32_t n_req;
+    int32_t cu_seqlens_host[kMaxReq + 1];
+    GatherSeg seg[kMaxSegs];
+};
+
+// ------------------------------------------------------------------ GEMM
+enum GemmEpi : int {
+    EPI_BF16 = 0,
+    EPI_GELU_BF16 = 1,
+    EPI_ADD_F32 = 2,
+    EPI_F32 = 3,
+    EPI_QKV_ROPE = 4,   // bf16 out, repairer RoPE on columns < rope_cols
+    EPI_KV_BF16 = 5,    // in-place residual add on a bf16 cache tile (+ global RoPE on K)
+    EPI_KV_F32 = 6      // same for an fp32 cache
+};
+
+struct GemmParams {
+    int32_t M, N, K;
+    int32_t num_m, num_n;
+    const float* bias;       // [N] or null
+    void* out;               // non-KV epilogues
+    int64_t ldo;             // elements
+    const int32_t* pos;      // [M] (RoPE epilogues)
+    int32_t rope_dim;        // head dim the RoPE pairs live in
+    int32_t rope_cols;       // QKV: columns [0, rope_cols) are rotated (Q and K)
+    int32_t rope_on;         // KV: rotate K segments
+    int32_t n_kv_heads;      // KV: segment s is K iff (s / n_kv_heads) is even
+    const float* sigma;      // KV: sigma_delta [N]
+    unsigned* status;
+    float inv_freq[64];      // RoPE frequencies, rope_dim / 2 entries
+};
+
+// ------------------------------------------------------------------ segment projection
+struct SegParams {
+    int32_t M;           // tokens
+    int32_t S;           // segments
+    int32_t d_seg;       // 8 or 16
+    int32_t num_m, num_g;
+    const float* b_seg;  // [S, d_seg]
+    uint16_t* y;         // [M, S * d_seg]
+    unsigned* status;
+};
+
+// ------------------------------------------------------------------ attention
+struct AttnParams {
+    const int32_t* chunk_end;
+    uint16_t* out;           // [N, d_b]
+    int32_t d_b;
+    int32_t n_heads;
+    int32_t n_req;
+    int32_t n_items;         // total (request, q-tile) pairs
+    float scale_log2;        // log2(e) / sqrt(d)
+    unsigned* status;
+    int32_t req_start[kMaxReq + 1];   // cu_seqlens
+    int32_t tile_prefix[kMaxReq + 1]; // cumulative q tiles
+};
+
+// ------------------------------------------------------------------ host helpers
+unsigned* device_status_ptr();          // per current device, nullptr on failure
+int num_sms();                          // SMs of the current device
+cr_status cuda_check(cudaError_t e);
+bool make_tmap_2d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, uint64_t inner,
+                  uint64_t outer, uint64_t row_stride_bytes, uint32_t box_inner,
+                  uint32_t box_outer, CUtensorMapSwizzle swz);
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Raise a kernel's dynamic shared-memory limit once per device (the first,
+// uncaptured call does it, so later calls can be captured into CUDA graphs).
+int current_device_index();
+// `done` must be a static owned by the caller's kernel-specific code (one per kernel).
+template <typename K>
+cr_status ensure_smem_attr(K kern, int bytes, unsigned long long* done) {
+    const int d = current_device_index();
+    if (d < 0) return CR_ERR_CUDA;
+    const unsigned long long bit = 1ull << (d & 63);
+    if (__atomic_load_n(done, __ATOMIC_ACQUIRE) & bit) return CR_OK;
+    const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e != cudaSuccess) return CR_ERR_CUDA;
+    __atomic_fetch_or(done, bit, __ATOMIC_ACQ_REL);
+    return CR_OK;
+}
+
+// Launchers (validated arguments).
+cr_status launch_gather(const GatherParams& p, cudaStream_t st);
+cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t M, int64_t N,
+                      int64_t K, int epi, GemmParams p, void* kv_base, int64_t ld_kv,
+                      cudaStream_t st);
+cr_status launch_segproj(const uint16_t* kv, int64_t ld_kv, const uint16_t* wfold, int head_dim,
+                         SegParams p, cudaStream_t st);
+cr_status launch_fold_sigma(const uint16_t* w_seg, const float* sigma, int S, int d_seg,
+                            int head_dim, uint16_t* wfold, cudaStream_t st);
+cr_status launch_to_bf16(const float* x, int64_t n, uint16_t* y, cudaStream_t st);
+cr_status launch_layernorm(const float* x, const uint16_t* add, int64_t ld_add, float* x_out,
+                           const float* g, const float* b, float eps, int64_t M, int64_t D,
+                           uint16_t* u, cudaStream_t st);
+cr_status launch_attention(const uint16_t* qkv, int64_t n_tokens, int head_dim,
+                           const AttnParams& p, cudaStream_t st);
+
+}  // namespace cr

@@ -1,0 +1,179 @@
+// Bandwidth-bound kernels of the repair path:
+//   gather_kernel     stale-cache assembly (Sec. 4.1, "Chunk-cache
+//                     preparation": canonical chunk caches concatenated in
+//                     document order; a pure copy, K is not rotated)
+//   layernorm_kernel  LayerNorm of the residual stream (optionally adding the
+//                     block's reinjection P_b(s) first, Sec. 4.1 eq. for h^b)
+//   to_bf16_kernel    fp32 cache/embedding -> bf16 operands for the tensor cores
+#include <cuda_bf16.h>
+
+#include "cr_internal.h"
+#include "cr_ptx.cuh"
+
+namespace cr {
+namespace {
+
+// One CTA per output row (grid-stride).  A row is one token's D_KV cache
+// values plus its d_model embedding values, each copied with 16-byte vectors,
+// four loads in flight per thread before the matching stores.
+__global__ void __launch_bounds__(512) gather_kernel(const __grid_constant__ GatherParams p) {
+    for (int64_t t = blockIdx.x; t < p.n_tokens; t += gridDim.x) {
+        int lo = 0, hi = p.n_seg - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (p.seg[mid].dst_row <= t)
+                lo = mid;
+            else
+                hi = mid - 1;
+        }
+        const GatherSeg& sg = p.seg[lo];
+        const int64_t off = t - sg.dst_row;
+        const int64_t src = sg.src_row + off;
+        if (off < 0 || off >= sg.len || src < 0 || src >= p.n_pool_tokens) {
+            if (threadIdx.x == 0) report(p.status, CR_DEV_INDEX, 1);
+            continue;
+        }
+        if (threadIdx.x == 0) {
+            p.chunk_id[t] = sg.chunk_local;
+            p.pos[t] = static_cast<int32_t>(sg.local_start + off);
+            p.chunk_end[t] = sg.local_start + sg.len;
+        }
+        for (int part = 0; part < 2; ++part) {
+            const int64_t rb = part == 0 ? p.kv_row_bytes : p.emb_row_bytes;
+            const uint4* s = reinterpret_cast<const uint4*>((part == 0 ? p.kv_pool : p.emb_pool) + src * rb);
+            uint4* d = reinterpret_cast<uint4*>((part == 0 ? p.kv_out : p.emb_out) + t * rb);
+            const int64_t nv = rb >> 4;
+            for (int64_t base = threadIdx.x; base < nv; base += 4 * blockDim.x) {
+                uint4 v[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int64_t i = base + u * blockDim.x;
+                    if (i < nv) v[u] = __ldcs(s + i);
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int64_t i = base + u * blockDim.x;
+                    if (i < nv) d[i] = v[u];
+                }
+            }
+        }
+    }
+    if (blockIdx.x == 0 && static_cast<int>(threadIdx.x) <= p.n_req)
+        p.cu_seqlens[threadIdx.x] = p.cu_seqlens_host[threadIdx.x];
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+// One warp per row, VPL float4 per lane (D = 128 * VPL); two-pass statistics
+// from registers (mean, then mean squared deviation: biased variance).
+template <int VPL>
+__global__ void __launch_bounds__(256) layernorm_kernel(const float* x,
+                                                        const uint16_t* __restrict__ add,
+                                                        int64_t ld_add, float* x_out,
+                                                        const float* __restrict__ g,
+                                                        const float* __restrict__ b, float eps,
+                                                        int64_t M, uint16_t* __restrict__ u) {
+    constexpr int D = VPL * 128;
+    const int64_t row = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (row >= M) return;
+    float4 v[VPL];
+    const float4* xr = reinterpret_cast<const float4*>(x + row * D);
+#pragma unroll
+    for (int k = 0; k < VPL; ++k) v[k] = xr[lane + 32 * k];
+    if (add) {
+        const uint2* ar = reinterpret_cast<const uint2*>(add + row * ld_add);
+        float4* xo = reinterpret_cast<float4*>(x_out + row * D);
+#pragma unroll
+        for (int k = 0; k < VPL; ++k) {
+            const uint2 a = ar[lane + 32 * k];
+            v[k].x += bf16_lo(a.x);
+            v[k].y += bf16_hi(a.x);
+            v[k].z += bf16_lo(a.y);
+            v[k].w += bf16_hi(a.y);
+            xo[lane + 32 * k] = v[k];
+        }
+    }
+    float s = 0.f;
+#pragma unroll
+    for (int k = 0; k < VPL; ++k) s += (v[k].x + v[k].y) + (v[k].z + v[k].w);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    const float mean = s * (1.0f / D);
+    float q = 0.f;
+#pragma unroll
+    for (int k = 0; k < VPL; ++k) {
+        const float a = v[k].x - mean, bb = v[k].y - mean, c = v[k].z - mean, d = v[k].w - mean;
+        q += (a * a + bb * bb) + (c * c + d * d);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
+    const float rstd = rsqrtf(q * (1.0f / D) + eps);
+    const float4* g4 = reinterpret_cast<const float4*>(g);
+    const float4* b4 = reinterpret_cast<const float4*>(b);
+    uint2* ur = reinterpret_cast<uint2*>(u + row * D);
+#pragma unroll
+    for (int k = 0; k < VPL; ++k) {
+        const float4 gg = __ldg(g4 + lane + 32 * k);
+        const float4 bq = __ldg(b4 + lane + 32 * k);
+        uint2 w;
+        w.x = pack_bf16x2((v[k].x - mean) * rstd * gg.x + bq.x, (v[k].y - mean) * rstd * gg.y + bq.y);
+        w.y = pack_bf16x2((v[k].z - mean) * rstd * gg.z + bq.z, (v[k].w - mean) * rstd * gg.w + bq.w);
+        ur[lane + 32 * k] = w;
+    }
+}
+
+__global__ void to_bf16_kernel(const float* __restrict__ x, int64_t n, uint16_t* __restrict__ y) {
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const __nv_bfloat16 b = __float2bfloat16_rn(x[i]);
+        y[i] = *reinterpret_cast<const uint16_t*>(&b);
+    }
+}
+
+}  // namespace
+
+cr_status launch_gather(const GatherParams& p, cudaStream_t st) {
+    if (p.n_tokens <= 0) return CR_OK;
+    int64_t grid = static_cast<int64_t>(num_sms()) * 4;
+    if (grid > p.n_tokens) grid = p.n_tokens;
+    gather_kernel<<<static_cast<int>(grid), 512, 0, st>>>(p);
+    return cuda_check(cudaGetLastError());
+}
+
+cr_status launch_layernorm(const float* x, const uint16_t* add, int64_t ld_add, float* x_out,
+                           const float* g, const float* b, float eps, int64_t M, int64_t D,
+                           uint16_t* u, cudaStream_t st) {
+    if (M <= 0) return CR_OK;
+    const int rows_per_block = 8;
+    const int grid = static_cast<int>((M + rows_per_block - 1) / rows_per_block);
+    switch (D) {
+#define CR_LN_CASE(V)                                                                       \
+    case V * 128:                                                                           \
+        layernorm_kernel<V><<<grid, 256, 0, st>>>(x, add, ld_add, x_out, g, b, eps, M, u); \
+        break;
+        CR_LN_CASE(1)
+        CR_LN_CASE(2)
+        CR_LN_CASE(3)
+        CR_LN_CASE(4)
+        CR_LN_CASE(5)
+        CR_LN_CASE(6)
+        CR_LN_CASE(7)
+        CR_LN_CASE(8)
+#undef CR_LN_CASE
+        default:
+            return CR_ERR_UNSUPPORTED;
+    }
+    return cuda_check(cudaGetLastError());
+}
+
+cr_status launch_to_bf16(const float* x, int64_t n, uint16_t* y, cudaStream_t st) {
+    if (n <= 0) return CR_OK;
+    int64_t blocks = (n + 255) / 256;
+    if (blocks > static_cast<int64_t>(num_sms()) * 16) blocks = static_cast<int64_t>(num_sms()) * 16;
+    to_bf16_kernel<<<static_cast<int>(blocks), 256, 0, st>>>(x, n, y);
+    return cuda_check(cudaGetLastError());
+}
+
+}  // namespace cr

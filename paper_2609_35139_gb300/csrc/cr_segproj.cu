@@ -1,0 +1,257 @@
+// StaleEncoder stage 1 (Sec. 4.1): every one of the S = 2 L H_KV segments of
+// a token has its own d_h -> d_seg linear, applied to the cache divided by
+// sigma_stale.  Per token this reads D_KV cache values and does 2 D_KV d_seg
+// flops, i.e. 16 flop/byte at d_seg = 16: the kernel is bound by HBM, and the
+// tensor cores only have to keep up with the stream of cache tiles.
+//
+// Work item: 128 tokens x G = 16 consecutive segments.  Warp 0 streams, per
+// segment, the [128 x d_h] cache slice (TMA, 128B swizzle) and the segment's
+// [16 x d_h] weight rows (1/sigma already folded in) through a ring of
+// shared-memory stages; warp 1 issues one M=128, N=16 MMA chain per segment
+// into its own 16 TMEM columns (two 256-column buffers); warps 2..5 add the
+// bias and store d_seg bf16 values per segment.  For d_seg = 8 the weight box
+// still spans 16 rows (the next segment's rows, or TMA zero fill past the
+// end); those 8 extra output columns are computed and discarded.
+#include "cr_internal.h"
+#include "cr_ptx.cuh"
+
+namespace cr {
+namespace {
+
+constexpr int SP_G = 16;          // segments per work item
+constexpr int SP_N = 16;          // MMA N (>= d_seg)
+
+template <int DH>
+struct SegCfg {
+    static constexpr int kBoxes = DH / 64;                 // 64-column swizzle boxes per slice
+    static constexpr uint32_t kABytes = 128 * DH * 2;
+    static constexpr uint32_t kBBytes = SP_N * DH * 2;
+    static constexpr uint32_t kStageBytes = kABytes + kBBytes;
+    static constexpr int kStages = (DH == 128) ? 5 : 8;
+    static constexpr uint32_t kSmemBytes = 1024 + kStages * kStageBytes + 256;
+};
+
+__global__ void fold_sigma_kernel(const uint16_t* __restrict__ w, const float* __restrict__ sigma,
+                                  int64_t n, int d_seg, int dh, uint16_t* __restrict__ out) {
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t d = i % dh;
+        const int64_t s = i / (static_cast<int64_t>(d_seg) * dh);
+        const float wv = __uint_as_float(static_cast<uint32_t>(w[i]) << 16);
+        const float v = wv / sigma[s * dh + d];
+        const __nv_bfloat16 b = __float2bfloat16_rn(v);
+        out[i] = *reinterpret_cast<const uint16_t*>(&b);
+    }
+}
+
+template <int DH>
+__global__ void __launch_bounds__(192, 1)
+    segproj_kernel(const __grid_constant__ CUtensorMap tmKV, const __grid_constant__ CUtensorMap tmW,
+                   const __grid_constant__ SegParams p) {
+    using Cfg = SegCfg<DH>;
+    constexpr int STAGES = Cfg::kStages;
+    constexpr uint32_t IDESC = idesc_bf16(128, SP_N, false, false);
+    constexpr uint32_t TMEM_COLS = 512;
+
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * Cfg::kStageBytes);
+    uint64_t* full = bars;
+    uint64_t* empty = bars + STAGES;
+    uint64_t* tfull = bars + 2 * STAGES;
+    uint64_t* tempty = tfull + 2;
+    uint64_t* drain = tempty + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
+
+    const uint32_t warp = warp_id(), lane = lane_id();
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&tfull[s], 1);
+            mbar_init(&tempty[s], 4);
+        }
+        mbar_init(drain, 1);
+        *abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == 1) tmem_alloc(tmem_slot, TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+    const WaitCtx wc{abort_flag, p.status};
+    const int total = p.num_m * p.num_g;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            tma_prefetch(&tmKV);
+            tma_prefetch(&tmW);
+            uint32_t stage = 0, phase = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+                const int m0 = (t % p.num_m) * 128;
+                const int s0 = (t / p.num_m) * SP_G;
+                const int ns = min(SP_G, p.S - s0);
+                for (int g = 0; g < ns; ++g) {
+                    if (!(ok = mbar_wait(&empty[stage], phase ^ 1u, wc, 111))) break;
+                    uint8_t* sa = smem + stage * Cfg::kStageBytes;
+                    uint8_t* sb = sa + Cfg::kABytes;
+                    const int seg = s0 + g;
+                    mbar_expect_tx(&full[stage], Cfg::kStageBytes);
+#pragma unroll
+                    for (int b = 0; b < Cfg::kBoxes; ++b) {
+                        tma_load_2d(sa + b * 16384, &tmKV, &full[stage], seg * DH + b * 64, m0);
+                        tma_load_2d(sb + b * (SP_N * 128), &tmW, &full[stage], b * 64,
+                                    seg * p.d_seg);
+                    }
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+            }
+            if (!ok) {
+                const uint64_t t0 = globaltimer();
+                while (globaltimer() - t0 < 50000ull) {
+                }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+                const int s0 = (t / p.num_m) * SP_G;
+                const int ns = min(SP_G, p.S - s0);
+                if (!(ok = mbar_wait(&tempty[acc], acc_phase ^ 1u, wc, 211))) break;
+                tc_fence_after();
+                for (int g = 0; g < ns; ++g) {
+                    if (!(ok = mbar_wait(&full[stage], phase, wc, 212))) break;
+                    tc_fence_after();
+                    const uint32_t d = tmem_base + acc * 256 + g * SP_N;
+                    const uint32_t sa = smem_u32(smem + stage * Cfg::kStageBytes);
+                    const uint32_t sb = sa + Cfg::kABytes;
+#pragma unroll
+                    for (int b = 0; b < Cfg::kBoxes; ++b) {
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            const uint64_t da = smem_desc(sa + b * 16384 + k * 32, 16, 1024, SWZ_128B);
+                            const uint64_t db =
+                                smem_desc(sb + b * (SP_N * 128) + k * 32, 16, 1024, SWZ_128B);
+                            mma_bf16_ss(d, da, db, IDESC, (b | k) != 0 ? 1u : 0u);
+                        }
+                    }
+                    mma_commit(&empty[stage]);
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+                if (!ok) break;
+                mma_commit(&tfull[acc]);
+                acc ^= 1u;
+                if (acc == 0) acc_phase ^= 1u;
+            }
+            mma_commit(drain);
+            mbar_wait(drain, 0, wc, 213);
+        }
+    } else {
+        const uint32_t quad = warp & 3u;
+        const int r = static_cast<int>(quad * 32 + lane);
+        const int ldy = p.S * p.d_seg;
+        uint32_t acc = 0, acc_phase = 0;
+        for (int t = blockIdx.x; t < total; t += gridDim.x) {
+            const int m0 = (t % p.num_m) * 128;
+            const int s0 = (t / p.num_m) * SP_G;
+            const int ns = min(SP_G, p.S - s0);
+            const bool ok = mbar_wait(&tfull[acc], acc_phase, wc, 311);
+            if (!__all_sync(0xffffffffu, ok)) break;
+            tc_fence_after();
+            const int row = m0 + r;
+            const uint32_t taddr = tmem_base + ((quad * 32u) << 16) + acc * 256;
+            uint16_t* yrow = p.y + static_cast<int64_t>(row) * ldy;
+            for (int g = 0; g < ns; ++g) {
+                float v[16];
+                __syncwarp();
+                tmem_ld16(taddr + g * SP_N, v);
+                tmem_wait_ld();
+                const int seg = s0 + g;
+                const float* bs = p.b_seg + seg * p.d_seg;
+                if (row < p.M) {
+                    uint32_t w[8];
+#pragma unroll
+                    const int dm = p.d_seg - 1;   // d_seg is 8 or 16; columns >= d_seg are dropped
+                    for (int i = 0; i < 8; ++i)
+                        w[i] = pack_bf16x2(v[2 * i] + __ldg(bs + ((2 * i) & dm)),
+                                           v[2 * i + 1] + __ldg(bs + ((2 * i + 1) & dm)));
+                    uint4* dst = reinterpret_cast<uint4*>(yrow + seg * p.d_seg);
+                    dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
+                    if (p.d_seg == 16) dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[acc]);
+            acc ^= 1u;
+            if (acc == 0) acc_phase ^= 1u;
+        }
+    }
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc(tmem_base, TMEM_COLS);
+    }
+}
+
+template <int DH>
+cr_status launch_dh(const CUtensorMap& tk, const CUtensorMap& tw, const SegParams& p,
+                    cudaStream_t st) {
+    using Cfg = SegCfg<DH>;
+    auto kern = segproj_kernel<DH>;
+    static unsigned long long attr_done = 0;   // one per template instantiation
+    const cr_status sa = ensure_smem_attr(kern, static_cast<int>(Cfg::kSmemBytes), &attr_done);
+    if (sa != CR_OK) return sa;
+    const int items = p.num_m * p.num_g;
+    const int grid = items < num_sms() ? items : num_sms();
+    kern<<<grid, 192, Cfg::kSmemBytes, st>>>(tk, tw, p);
+    return cuda_check(cudaGetLastError());
+}
+
+}  // namespace
+
+cr_status launch_fold_sigma(const uint16_t* w_seg, const float* sigma, int S, int d_seg,
+                            int head_dim, uint16_t* wfold, cudaStream_t st) {
+    const int64_t n = static_cast<int64_t>(S) * d_seg * head_dim;
+    const int threads = 256;
+    int64_t blocks = (n + threads - 1) / threads;
+    if (blocks > 4 * 1024) blocks = 4 * 1024;
+    fold_sigma_kernel<<<static_cast<int>(blocks), threads, 0, st>>>(w_seg, sigma, n, d_seg,
+                                                                     head_dim, wfold);
+    return cuda_check(cudaGetLastError());
+}
+
+cr_status launch_segproj(const uint16_t* kv, int64_t ld_kv, const uint16_t* wfold, int head_dim,
+                         SegParams p, cudaStream_t st) {
+    if (head_dim != 64 && head_dim != 128) return CR_ERR_UNSUPPORTED;
+    if (p.d_seg != 8 && p.d_seg != 16) return CR_ERR_UNSUPPORTED;
+    p.num_m = (p.M + 127) / 128;
+    p.num_g = (p.S + SP_G - 1) / SP_G;
+    CUtensorMap tk, tw;
+    const uint64_t dkv = static_cast<uint64_t>(p.S) * head_dim;
+    if (!make_tmap_2d(&tk, kv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dkv, p.M, ld_kv * 2, 64, 128,
+                      CU_TENSOR_MAP_SWIZZLE_128B))
+        return CR_ERR_INVALID_ARG;
+    if (!make_tmap_2d(&tw, wfold, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, head_dim,
+                      static_cast<uint64_t>(p.S) * p.d_seg, head_dim * 2, 64, SP_N,
+                      CU_TENSOR_MAP_SWIZZLE_128B))
+        return CR_ERR_INVALID_ARG;
+    return head_dim == 128 ? launch_dh<128>(tk, tw, p, st) : launch_dh<64>(tk, tw, p, st);
+}
+
+}  // namespace cr

@@ -1,0 +1,150 @@
+"""Each kernel of the repair path against the oracle's step, through the C ABI."""
+import numpy as np
+import pytest
+import torch
+
+import fixtures as F
+import oracle as O
+from paper_2609_35139_gb300 import build, cr
+from parity_util import as_f64, assert_close, to_dev, to_host
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    build.build()
+    L = cr.lib()
+    cr.cr_clear_device_status()
+    yield L
+    st, word = cr.cr_get_device_status()
+    assert st == cr.CR_OK, f"device status {word}"
+
+
+def _bf16(g, shape, scale=1.0):
+    return F.f32_to_bf16((g.standard_normal(shape) * scale).astype(np.float32))
+
+
+@pytest.mark.parametrize("M,N,K", [(128, 128, 64), (300, 256, 200), (77, 3072, 1024),
+                                   (513, 1024, 4096), (40, 48, 8), (1000, 512, 8192)])
+@pytest.mark.parametrize("epi", [cr.CR_EPI_BF16, cr.CR_EPI_GELU_BF16, cr.CR_EPI_ADD_F32, cr.CR_EPI_F32])
+def test_linear(M, N, K, epi):
+    g = np.random.default_rng(M * 7 + N + K + epi)
+    A = _bf16(g, (M, K))
+    W = _bf16(g, (N, K), 1.0 / np.sqrt(K))
+    bias = g.standard_normal(N).astype(np.float32)
+    ref = as_f64(A) @ as_f64(W).T + bias
+    f32 = epi in (cr.CR_EPI_ADD_F32, cr.CR_EPI_F32)
+    init = g.standard_normal((M, N)).astype(np.float32)
+    out = to_dev(init) if f32 else torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
+    cr.cr_linear(to_dev(A), to_dev(W), to_dev(bias), out, epi)
+    torch.cuda.synchronize()
+    got = to_host(out)
+    if epi == cr.CR_EPI_GELU_BF16:
+        ref = O.gelu(ref)
+    if epi == cr.CR_EPI_ADD_F32:
+        ref = ref + init
+    if f32:
+        assert_close(got, ref, 1e-5, 1e-4, f"linear f32 {M}x{N}x{K}")
+    else:   # one bf16 rounding of the output
+        assert_close(got, ref, 3e-3, 1.5e-2, f"linear bf16 {M}x{N}x{K}")
+
+
+@pytest.mark.parametrize("D", [128, 512, 1024])
+def test_layernorm_with_reinjection_add(D):
+    g = np.random.default_rng(D)
+    M = 301
+    x = (g.standard_normal((M, D)) * 3 + 0.5).astype(np.float32)
+    add = _bf16(g, (M, 2 * D))          # strided slice of a wider matrix, like P_b(s)
+    gam = (1 + 0.2 * g.standard_normal(D)).astype(np.float32)
+    bet = (0.1 * g.standard_normal(D)).astype(np.float32)
+    xd = to_dev(x)
+    xo = torch.empty_like(xd)
+    u = torch.empty(M, D, dtype=torch.bfloat16, device="cuda")
+    addd = to_dev(add)
+    cr.cr_layernorm(xd, to_dev(gam), to_dev(bet), 1e-5, u, add=addd[:, D:], ld_add=2 * D, x_out=xo)
+    torch.cuda.synchronize()
+    xs = x.astype(np.float64) + as_f64(add)[:, D:]
+    np.testing.assert_allclose(to_host(xo), xs, rtol=1e-6, atol=1e-6)
+    assert_close(to_host(u), O.layer_norm(xs, gam, bet, 1e-5), 3e-3, 1.5e-2, "layernorm")
+
+
+def _chunk_ids(lens):
+    return np.concatenate([np.full(n, i, np.int32) for i, n in enumerate(lens)])
+
+
+@pytest.mark.parametrize("hd", [32, 64])
+@pytest.mark.parametrize("reqs", [
+    [[64, 64]],                      # two chunks, one tile
+    [[300]],                          # single chunk: bidirectional, ragged tail
+    [[1] * 150],                      # unit chunks: token-causal
+    [[130, 77, 200, 1, 95]],          # ragged chunk map across several tiles
+    [[129, 40], [5], [300, 256, 3]],  # several requests (varlen)
+])
+def test_chunk_causal_attention(hd, reqs):
+    g = np.random.default_rng(hd + sum(map(sum, reqs)))
+    nh = 4 if hd == 32 else 8
+    db = nh * hd
+    lens = [sum(r) for r in reqs]
+    N = sum(lens)
+    qkv = _bf16(g, (N, 3 * db))
+    cend = []
+    for r in reqs:
+        e = np.cumsum(r)
+        cend.append(np.concatenate([np.full(n, e[i], np.int32) for i, n in enumerate(r)]))
+    cend = np.concatenate(cend)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    out = torch.full((N, db), float("nan"), dtype=torch.bfloat16, device="cuda")
+    cr.cr_chunk_causal_attention(to_dev(qkv), db, nh, to_dev(cend), cu, out)
+    torch.cuda.synchronize()
+    got = to_host(out)
+    q = as_f64(qkv)
+    want = np.empty((N, db))
+    for r, req in enumerate(reqs):
+        a, b = cu[r], cu[r + 1]
+        sl = lambda off: q[a:b, off:off + db].reshape(b - a, nh, hd)
+        want[a:b] = O.block_causal_attention(sl(0), sl(db), sl(2 * db), _chunk_ids(req)).reshape(b - a, db)
+    assert not np.isnan(as_f64(got)).any()
+    assert_close(got, want, 8e-3, 4e-2, f"attention hd={hd} {reqs}")
+
+
+@pytest.mark.parametrize("db,nh", [(128, 4), (512, 8), (1024, 16)])
+def test_qkv_rope(db, nh):
+    g = np.random.default_rng(db)
+    N = 333
+    u = _bf16(g, (N, db))
+    W = _bf16(g, (3 * db, db), 1 / np.sqrt(db))
+    b = (0.1 * g.standard_normal(3 * db)).astype(np.float32)
+    pos = g.integers(0, 9000, N).astype(np.int32)
+    out = torch.empty(N, 3 * db, dtype=torch.bfloat16, device="cuda")
+    cr.cr_qkv_rope(to_dev(u), to_dev(W), to_dev(b), to_dev(pos), db, nh, 1e4, out)
+    torch.cuda.synchronize()
+    hd = db // nh
+    y = as_f64(u) @ as_f64(W).T + b
+    f = O.repair_inv_freq(hd, 1e4)
+    q = O.rope_rotate_half(y[:, :db].reshape(N, nh, hd), pos, f).reshape(N, db)
+    k = O.rope_rotate_half(y[:, db:2 * db].reshape(N, nh, hd), pos, f).reshape(N, db)
+    want = np.concatenate([q, k, y[:, 2 * db:]], axis=1)
+    assert_close(to_host(out), want, 4e-3, 2e-2, "qkv+rope")
+
+
+@pytest.mark.parametrize("name", ["tiny", "small", "llama8b"])
+def test_segment_projection(name):
+    c = F.make_case(name)
+    t, r = c.target, c.repairer
+    rows = 300 if name != "llama8b" else 1000
+    kv, _ = c.pool_rows(0, rows)
+    if t.cache_dtype == "f32":
+        kv = F.f32_to_bf16(kv)          # the op consumes bf16 (fp32 caches are converted first)
+    w = c.weights
+    from paper_2609_35139_gb300 import dims_from
+    td, _ = dims_from(t, r)
+    y = torch.empty(rows, t.n_segments * r.d_seg, dtype=torch.bfloat16, device="cuda")
+    ws = torch.empty(t.n_segments * r.d_seg * t.head_dim * 2, dtype=torch.uint8, device="cuda")
+    cr.cr_segment_project(td, r.d_seg, to_dev(kv), to_dev(w["w_seg"]), to_dev(w["b_seg"]),
+                          to_dev(w["sigma_stale"]), y, ws)
+    torch.cuda.synchronize()
+    want = O.segment_projection(kv, w["sigma_stale"], w["w_seg"], w["b_seg"], t.head_dim, "bf16")
+    assert_close(to_host(y), want, 4e-3, 2.5e-2, f"segment projection {name}")

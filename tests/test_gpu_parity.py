@@ -1,0 +1,296 @@
+"""End-to-end parity: the four C-ABI calls against the oracle, on every workload.
+
+The GPU path runs exactly as bench.py runs it (RepairSession: assemble,
+compress, forward, apply on one stream).  Small workloads are compared on
+every output; the full-size ones on every intermediate and on a sample of
+repaired rows (all D_KV coordinates of each sampled token) that the oracle's
+head computes one by one.
+"""
+import numpy as np
+import pytest
+import torch
+
+import fixtures as F
+import oracle as O
+from paper_2609_35139_gb300 import RepairSession, cr, dims_from, pack_host_weights
+from parity_util import (as_f64, assert_close, check_repaired_cache, rel_errors, residual_cosine,
+                         to_dev, to_host)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2609_35139_gb300 import build
+    build.build()
+    cr.lib()
+    cr.cr_clear_device_status()
+    yield
+    st, word = cr.cr_get_device_status()
+    assert st == cr.CR_OK, f"device status {word}"
+
+
+class GpuRun:
+    """One pass of the repair chain on a case, keeping the intermediates on the host."""
+
+    def __init__(self, case, rope_mode=cr.CR_ROPE_NONE, weights=None, pool=None, patch=None):
+        t, r = dims_from(case.target, case.repairer)
+        w = weights if weights is not None else case.weights
+        self.pw = pack_host_weights(w, case.repairer.n_blocks)
+        kvp, embp = pool if pool is not None else case.pool()
+        p = case.plan
+        self.sess = RepairSession(t, r, self.pw, max_tokens=p.n_tokens)
+        s = self.sess
+        self.a = s.assemble(to_dev(kvp), to_dev(embp), p.chunk_start, p.chunk_len, p.chunk_idx,
+                            p.cu_chunks)
+        n = self.a.n_tokens
+        torch.cuda.synchronize()
+        self.kv_stale = to_host(s.kv[:n])
+        self.emb = to_host(s.emb[:n])
+        self.chunk_id = to_host(s.chunk_id[:n])
+        self.chunk_end = to_host(s.chunk_end[:n])
+        self.pos = to_host(s.pos[:n])
+        self.cu_dev = to_host(s.cu_seqlens[:len(p.cu_chunks)])
+        if patch is not None:
+            patch(s, n)
+        s.compress(self.a)
+        s.forward(self.a)
+        s.apply(self.a, case.inv_freq_target, rope_mode)
+        torch.cuda.synchronize()
+        self.h0 = to_host(s.h0[:n])
+        self.rein = to_host(s.rein[:n])
+        self.yf = to_host(s.yf[:n])
+        self.kv = to_host(s.kv[:n])
+
+
+def oracle_request(case, assembled, r, rows=None, rope=False, weights=None):
+    """Oracle pass over request r; head only on `rows` (request-local) if given."""
+    t, rp = case.target, case.repairer
+    w = weights if weights is not None else case.weights
+    a, b = assembled["cu_seqlens"][r], assembled["cu_seqlens"][r + 1]
+    kv, emb = assembled["kv"][a:b], assembled["emb"][a:b]
+    res = O.repair_request(kv, emb, assembled["chunk_id"][a:b], assembled["pos"][a:b], w,
+                           cache_dtype=t.cache_dtype, n_layers=t.n_layers,
+                           n_kv_heads=t.n_kv_heads, head_dim=t.head_dim, n_heads=rp.n_heads,
+                           inv_freq_target=case.inv_freq_target if rope else None,
+                           with_head=rows is None)
+    if rows is not None:
+        z = O.residual_head(res.blocks[-1][rows] if res.blocks else res.h0[rows], w["lnf_g"],
+                            w["lnf_b"], w["w_out"], w["b_out"], rp.ln_eps)
+        rep = O.apply_residual(O.dtype_to_f64(kv[rows], t.cache_dtype), z, w["sigma_delta"])
+        if rope:
+            rep = O.global_rope_k(rep, assembled["pos"][a:b][rows], case.inv_freq_target,
+                                  t.n_layers, t.n_kv_heads, t.head_dim)
+        res.repaired = rep
+    return res
+
+
+def oracle_assemble(case, pool=None):
+    kvp, embp = pool if pool is not None else case.pool()
+    p = case.plan
+    return O.assemble_stale(kvp, embp, p.chunk_start, p.chunk_len, p.chunk_idx, p.cu_chunks)
+
+
+def check_assembly(g: GpuRun, a):
+    assert np.array_equal(g.kv_stale.view(np.uint8), np.ascontiguousarray(a["kv"]).view(np.uint8))
+    assert np.array_equal(g.emb.view(np.uint8), np.ascontiguousarray(a["emb"]).view(np.uint8))
+    assert np.array_equal(g.chunk_id, a["chunk_id"])
+    assert np.array_equal(g.chunk_end, a["chunk_end"])
+    assert np.array_equal(g.pos, a["pos"])
+    assert np.array_equal(g.cu_dev, a["cu_seqlens"])
+
+
+def check_request(case, g: GpuRun, a, r, res, rows=None, rope=False):
+    t = case.target
+    lo, hi = a["cu_seqlens"][r], a["cu_seqlens"][r + 1]
+    report = {}
+    report["h0"] = assert_close(g.h0[lo:hi], res.h0, 1e-2, 6e-2, "h0 (compress)")
+    B = case.repairer.n_blocks
+    db = case.repairer.d_b
+    for b in range(B):
+        report[f"rein{b}"] = assert_close(g.rein[lo:hi, b * db:(b + 1) * db], res.rein[b], 1e-2,
+                                          6e-2, f"P_{b}(s)")
+    report["yf"] = assert_close(g.yf[lo:hi], res.yf, 2.5e-2, 0.2, "y_f (forward)")
+    sel = np.arange(hi - lo) if rows is None else rows
+    got = g.kv[lo:hi][sel]
+    exact = res.repaired if rows is not None else (res.repaired_rot if rope else res.repaired)
+    if rope and rows is None:
+        exact = res.repaired_rot
+    report["cache"] = check_repaired_cache(got, exact, t, t.cache_dtype)
+    if not rope:
+        report["resid_cos"] = residual_cosine(got, g.kv_stale[lo:hi][sel], exact, t.cache_dtype)
+        assert report["resid_cos"] >= 0.99, report
+    return report
+
+
+# ------------------------------------------------------------------ small workloads, every output
+@pytest.mark.parametrize("name", ["tiny", "tiny_affine", "small", "small_multi"])
+def test_parity_small(name):
+    case = F.make_case(name)
+    g = GpuRun(case)
+    a = oracle_assemble(case)
+    check_assembly(g, a)
+    for r in range(len(a["cu_seqlens"]) - 1):
+        res = oracle_request(case, a, r)
+        rep = check_request(case, g, a, r, res)
+        print(name, r, rep)
+
+
+@pytest.mark.parametrize("name", ["small", "tiny"])
+def test_parity_global_rope(name):
+    case = F.make_case(name)
+    g = GpuRun(case, rope_mode=cr.CR_ROPE_GLOBAL)
+    a = oracle_assemble(case)
+    res = oracle_request(case, a, 0, rope=True)
+    print(name, check_request(case, g, a, 0, res, rope=True))
+
+
+def test_no_blocks_degenerate():
+    case = F.make_case("tiny_affine", repairer=F.RepairerDims(8, 64, 128, 0, 4, 512))
+    g = GpuRun(case)
+    a = oracle_assemble(case)
+    check_request(case, g, a, 0, oracle_request(case, a, 0))
+
+
+# ------------------------------------------------------------------ invariants on the GPU
+def test_zero_head_returns_stale_bit_for_bit():
+    case = F.make_case("small")
+    w = dict(case.weights, w_out=np.zeros_like(case.weights["w_out"]),
+             b_out=np.zeros_like(case.weights["b_out"]))
+    g = GpuRun(case, weights=w)
+    assert np.array_equal(g.kv, g.kv_stale)
+
+
+def test_causality_bit_identical_on_gpu():
+    case = F.make_case("small")
+    kvp, embp = case.pool()
+    g1 = GpuRun(case, pool=(kvp, embp))
+    # perturb the pool chunks that become request chunks 2.. (document order)
+    p = case.plan
+    kv2, emb2 = kvp.copy(), embp.copy()
+    rng = np.random.default_rng(3)
+    for c in p.chunk_idx[2:]:
+        a, n = p.chunk_start[c], p.chunk_len[c]
+        kv2[a:a + n] = F.f32_to_bf16(rng.standard_normal((n, kvp.shape[1])).astype(np.float32))
+        emb2[a:a + n] = F.f32_to_bf16(0.02 * rng.standard_normal((n, embp.shape[1])).astype(np.float32))
+    g2 = GpuRun(case, pool=(kv2, emb2))
+    cut = int(np.searchsorted(g1.chunk_id, 2))
+    assert cut > 0
+    for x, y in ((g1.h0, g2.h0), (g1.yf, g2.yf), (g1.kv, g2.kv)):
+        assert np.array_equal(x[:cut], y[:cut])
+        assert not np.array_equal(x[cut:], y[cut:])
+
+
+def test_permutation_within_chunk_permutes_outputs():
+    case = F.make_case("small")
+    g1 = GpuRun(case)
+    lo = int(np.searchsorted(g1.chunk_id, 2))
+    hi = int(np.searchsorted(g1.chunk_id, 3))
+    perm = np.arange(len(g1.chunk_id))
+    perm[lo:hi] = lo + np.random.default_rng(4).permutation(hi - lo)
+    pt = torch.from_numpy(perm).cuda()
+
+    def patch(s, n):   # move cache rows, embeddings and positions together
+        s.kv[:n] = s.kv[:n][pt]
+        s.emb[:n] = s.emb[:n][pt]
+        s.pos[:n] = s.pos[:n][pt]
+
+    g2 = GpuRun(case, patch=patch)
+    assert_close(g2.yf, g1.yf[perm], 5e-3, 5e-2, "permuted y_f")
+    assert_close(g2.kv, g1.kv[perm], 2e-3, 3e-2, "permuted repaired cache")
+
+
+def test_batch_equals_single_requests():
+    """Requests never interact: each request's outputs in a batch equal a solo run."""
+    case = F.make_case("small_multi")
+    g = GpuRun(case)
+    p = case.plan
+    for r in range(len(p.cu_chunks) - 1):
+        sel = p.chunk_idx[p.cu_chunks[r]:p.cu_chunks[r + 1]]
+        solo = F.make_case("small_multi", requests=[[int(c) for c in sel]])
+        gs = GpuRun(solo)
+        lo, hi = g.cu_dev[r], g.cu_dev[r + 1]
+        assert_close(gs.yf, g.yf[lo:hi], 1e-6, 1e-5, "solo vs batched y_f")
+        assert_close(gs.kv, g.kv[lo:hi], 1e-6, 1e-5, "solo vs batched cache")
+
+
+# ------------------------------------------------------------------ full-size workloads
+def _sample_rows(chunk_id, n_random=160, seed=0):
+    n = len(chunk_id)
+    starts = np.nonzero(np.diff(np.concatenate([[-1], chunk_id])))[0]
+    edge = np.concatenate([np.arange(s, min(s + 4, n)) for s in starts] + [[n - 1]])
+    rnd = np.random.default_rng(seed).choice(n, size=min(n_random, n), replace=False)
+    return np.unique(np.concatenate([edge, rnd]))
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("name", ["qwen3b", "llama8b", "qwen7b"])
+def test_parity_full_size(name):
+    case = F.make_case(name)
+    g = GpuRun(case)
+    a = oracle_assemble(case)
+    check_assembly(g, a)
+    rows = _sample_rows(a["chunk_id"])
+    res = oracle_request(case, a, 0, rows=rows)
+    print(name, check_request(case, g, a, 0, res, rows=rows))
+
+
+@pytest.mark.slow
+def test_parity_full_size_global_rope():
+    case = F.make_case("qwen3b")
+    g = GpuRun(case, rope_mode=cr.CR_ROPE_GLOBAL)
+    a = oracle_assemble(case)
+    rows = _sample_rows(a["chunk_id"], 64)
+    res = oracle_request(case, a, 0, rows=rows, rope=True)
+    print(check_request(case, g, a, 0, res, rows=rows, rope=True))
+
+
+@pytest.mark.slow
+def test_parity_batched_sampled_requests():
+    """16 varlen requests (about 128k tokens, a 18 GB pool); the oracle checks the
+    first and the last request; assembly is checked bit for bit on all of them."""
+    case = F.make_case("batched")
+    p = case.plan
+    # device pool built chunk by chunk (the host never holds all of it at once)
+    t = case.target
+    kvp = torch.empty(p.n_pool_tokens, t.d_kv, dtype=torch.bfloat16, device="cuda")
+    embp = torch.empty(p.n_pool_tokens, t.d_model, dtype=torch.bfloat16, device="cuda")
+    for c in range(len(p.chunk_len)):
+        s0, n = int(p.chunk_start[c]), int(p.chunk_len[c])
+        kv, emb = case.pool_rows(s0, n)
+        kvp[s0:s0 + n] = to_dev(kv)
+        embp[s0:s0 + n] = to_dev(emb)
+    tdims, rdims = dims_from(case.target, case.repairer)
+    pw = pack_host_weights(case.weights, case.repairer.n_blocks)
+    sess = RepairSession(tdims, rdims, pw, max_tokens=p.n_tokens)
+    asm = sess.assemble(kvp, embp, p.chunk_start, p.chunk_len, p.chunk_idx, p.cu_chunks)
+    torch.cuda.synchronize()
+    n = asm.n_tokens
+    stale_rows = {}
+    for r in (0, 15):
+        lo, hi = asm.cu_seqlens[r], asm.cu_seqlens[r + 1]
+        stale_rows[r] = (to_host(sess.kv[lo:hi]), to_host(sess.emb[lo:hi]))
+    sess.compress(asm)
+    sess.forward(asm)
+    sess.apply(asm)
+    torch.cuda.synchronize()
+    for r in (0, 15):
+        lo, hi = asm.cu_seqlens[r], asm.cu_seqlens[r + 1]
+        sel, kvs, embs = case.request_pool_rows(r)
+        kv_r, emb_r = np.concatenate(kvs), np.concatenate(embs)
+        assert np.array_equal(stale_rows[r][0], kv_r) and np.array_equal(stale_rows[r][1], emb_r)
+        lens = p.chunk_len[sel]
+        cid = np.concatenate([np.full(l, i, np.int32) for i, l in enumerate(lens)])
+        pos = np.arange(hi - lo, dtype=np.int32)
+        assert np.array_equal(to_host(sess.chunk_id[lo:hi]), cid)
+        assert np.array_equal(to_host(sess.pos[lo:hi]), pos)
+        rows = _sample_rows(cid, 96, seed=r)
+        asm_r = dict(kv=kv_r, emb=emb_r, chunk_id=cid, pos=pos,
+                     cu_seqlens=np.array([0, hi - lo], np.int32))
+        res = oracle_request(case, asm_r, 0, rows=rows)
+        g = type("G", (), {})()
+        g.h0, g.rein = to_host(sess.h0[lo:hi]), to_host(sess.rein[lo:hi])
+        g.yf, g.kv, g.kv_stale = to_host(sess.yf[lo:hi]), to_host(sess.kv[lo:hi]), stale_rows[r][0]
+        print("batched", r, check_request(case, g, asm_r, 0, res, rows=rows))

@@ -1,0 +1,117 @@
+"""The C-ABI library builds for sm_103a, loads without a GPU, exports every
+symbol include/*.h declares, and validates arguments on the host (no device
+work is attempted for invalid calls)."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from paper_2609_35139_gb300 import build, cr
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    build.build()
+    return cr.lib()
+
+
+def _declared():
+    names = set()
+    for h in ("cr.h", "cr_ops.h"):
+        with open(os.path.join(ROOT, "include", h)) as f:
+            src = f.read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        names |= set(re.findall(r"\b(cr_[a-z0-9_]+)\s*\(", src))
+    return sorted(names)
+
+
+def test_every_declared_symbol_is_exported(L):
+    declared = _declared()
+    assert len(declared) >= 13
+    for name in declared:
+        assert hasattr(L, name), name
+    assert set(declared) == set(cr.EXPORTED)
+
+
+def test_library_is_built_for_sm103a_only():
+    # the build passes exactly one -gencode for compute_103a / sm_103a
+    assert build.ARCH == ["-gencode", "arch=compute_103a,code=sm_103a"]
+
+
+def test_status_strings(L):
+    for s in range(6):
+        assert L.cr_status_str(s)
+    assert L.cr_status_str(99) == b"unknown status"
+
+
+def _dims(name="small"):
+    import fixtures as F
+    from paper_2609_35139_gb300 import dims_from
+    c = F.make_case(name)
+    return c, dims_from(c.target, c.repairer)
+
+
+def test_workspace_bytes_host_logic(L):
+    c, (t, r) = _dims("llama8b")
+    w1 = cr.cr_workspace_bytes(t, r, 1)
+    w2 = cr.cr_workspace_bytes(t, r, 5120)
+    assert 0 < w1 < w2
+    # dominated by per-token buffers: y, s|e, x, u, qkv, o, g (bf16 / fp32 x)
+    per_tok = (512 * 16 * 2 + 2 * 512 * 2 + 1024 * 4 + 1024 * 2 + 3 * 1024 * 2 + 1024 * 2
+               + 4096 * 2)
+    assert abs((w2 - w1) - 5119 * per_tok) < 64 * 256
+    bad = cr.repairer_dims(16, 512, 1000, 6, 16, 4096)   # d_b not a multiple of 128
+    assert cr.cr_workspace_bytes(t, bad, 10) == 0
+    bad = cr.repairer_dims(16, 512, 1024, 6, 8, 4096)    # 128-dim heads: unsupported
+    assert cr.cr_workspace_bytes(t, bad, 10) == 0
+
+
+FAKE = 0x10000   # 16-byte aligned, never dereferenced: validation fails first
+
+
+def _assemble(L, t, chunk_idx, cu, chunk_len=(10, 20, 30), n_pool=60, max_tokens=1000, ptr=FAKE):
+    cs = np.array([0, 10, 30], np.int64)
+    cl = np.array(chunk_len, np.int32)
+    ci = np.array(chunk_idx, np.int32)
+    cc = np.array(cu, np.int32)
+    cuh = np.zeros(len(cc), np.int32)
+    return L.cr_assemble_stale(ctypes.byref(t), ptr, ptr, n_pool, cs.ctypes.data, cl.ctypes.data,
+                               len(cl), ci.ctypes.data, cc.ctypes.data, len(cc) - 1, ptr, ptr,
+                               max_tokens, ptr, ptr, ptr, ptr, cuh.ctypes.data, None)
+
+
+def test_assemble_rejects_bad_inputs_on_host(L):
+    c, (t, r) = _dims()
+    assert _assemble(L, t, [0, 5], [0, 2]) == cr.CR_ERR_INVALID_ARG        # chunk id out of range
+    assert _assemble(L, t, [0, -1], [0, 2]) == cr.CR_ERR_INVALID_ARG
+    assert _assemble(L, t, [0, 1], [0, 0, 2]) == cr.CR_ERR_INVALID_ARG     # empty request
+    assert _assemble(L, t, [0, 2], [0, 2], n_pool=50) == cr.CR_ERR_INVALID_ARG   # chunk past pool
+    assert _assemble(L, t, [0, 1], [0, 2], chunk_len=(10, 0, 30)) == cr.CR_ERR_INVALID_ARG
+    assert _assemble(L, t, [2, 1], [0, 2], max_tokens=40) == cr.CR_ERR_INVALID_ARG  # 50 > 40
+    assert _assemble(L, t, [0, 1], [0, 2], ptr=FAKE + 8) == cr.CR_ERR_INVALID_ARG  # misaligned
+    bad = cr.target_dims(4, 2, 96, 512, "bf16")
+    assert _assemble(L, bad, [0, 1], [0, 2]) == cr.CR_ERR_UNSUPPORTED
+
+
+def test_other_calls_reject_bad_inputs_on_host(L):
+    c, (t, r) = _dims()
+    w = cr.cr_weights()
+    # null weights -> invalid before any device work
+    assert L.cr_compress_features(ctypes.byref(t), ctypes.byref(r), ctypes.byref(w), FAKE, FAKE,
+                                  10, FAKE, FAKE, FAKE, 1 << 30, None) == cr.CR_ERR_INVALID_ARG
+    assert L.cr_apply_residual(ctypes.byref(t), ctypes.byref(r), ctypes.byref(w), FAKE, 10, FAKE,
+                               FAKE, None, 1, None) == cr.CR_ERR_INVALID_ARG
+    assert L.cr_linear(FAKE, 64, FAKE, None, 10, 30, 64, FAKE, 30, 0, None) == cr.CR_ERR_INVALID_ARG
+    assert L.cr_linear(FAKE, 64, FAKE, None, 10, 32, 60, FAKE, 32, 0, None) == cr.CR_ERR_INVALID_ARG
+    assert L.cr_layernorm(FAKE, None, 0, None, FAKE, FAKE, 1e-5, 4, 100, FAKE, None) == \
+        cr.CR_ERR_INVALID_ARG
+    cu = np.array([0, 100], np.int32)
+    assert L.cr_chunk_causal_attention(FAKE, 1024, 8, FAKE, cu.ctypes.data, 1, 100, FAKE,
+                                       None) == cr.CR_ERR_UNSUPPORTED          # 128-dim heads
+    cu = np.array([0, 100, 90], np.int32)
+    assert L.cr_chunk_causal_attention(FAKE, 1024, 16, FAKE, cu.ctypes.data, 2, 90, FAKE,
+                                       None) == cr.CR_ERR_INVALID_ARG          # empty request
