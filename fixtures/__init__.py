@@ -270,6 +270,9 @@ def inv_freq_for(theta: float, dim: int) -> np.ndarray:
     return (theta ** (-2.0 * i / dim)).astype(np.float32)
 
 
+RESIDUAL_SCALE = 0.25
+
+
 def make_weights(rc: Recipe) -> Dict[str, np.ndarray]:
     """Random-init repairer weights: Xavier-uniform matrices (bf16), biases 0, LN identity.
 
@@ -320,7 +323,11 @@ def make_weights(rc: Recipe) -> Dict[str, np.ndarray]:
     w["b_out"] = vec("b_out", D, "bias")
     sig = sigma_stale_for(rc)
     w["sigma_stale"] = sig
-    w["sigma_delta"] = sig.copy()       # residual scale = cache scale: a visible residual
+    # sigma_Delta is the per-coordinate RMS of the joint - stale residual (Sec. 4.2).
+    # The paper measures that residual at about 0.18-0.31 of the joint cache for K
+    # (Sec. 5.3, stale-vs-joint relative RMSE 0.182 interior / 0.310 boundary), so
+    # the synthetic residual scale is a quarter of the cache scale.
+    w["sigma_delta"] = (RESIDUAL_SCALE * sig).astype(np.float32)
     return w
 
 

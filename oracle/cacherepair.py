@@ -52,7 +52,7 @@ __all__ = [
     "reinjection", "layer_norm", "gelu", "rope_rotate_half", "block_causal_mask",
     "block_causal_attention", "repair_block", "repair_backbone", "residual_head",
     "apply_residual", "global_rope_k", "repair_request", "weight_shapes", "param_groups",
-    "cache_payload_bytes", "OracleResult",
+    "cache_payload_bytes", "OracleResult", "repair_inv_freq", "block_weights",
 ]
 
 

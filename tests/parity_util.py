@@ -50,6 +50,17 @@ def assert_close(got, want, rel_rms: float, max_rel: float, what=""):
     return r, m
 
 
+def assert_close_bf16(got, want, rel_rms: float = 3e-3, what=""):
+    """A bf16 output: elementwise |err| <= 2^-8 |want| + 2e-3 RMS(want) (one rounding
+    of the output plus fp32 accumulation order), and relative RMS error <= rel_rms."""
+    g, w = as_f64(got), as_f64(want)
+    rms = np.sqrt(np.mean(w ** 2))
+    bad = np.abs(g - w) > np.abs(w) * 2.0 ** -8 + 2e-3 * rms
+    r, m = rel_errors(got, want)
+    assert not bad.any() and r <= rel_rms, f"{what}: {int(bad.sum())} elements out of bound, rel-RMS {r:.3e}, max/RMS {m:.3e}"
+    return r, m
+
+
 def half_ulp(x: np.ndarray, cache_dtype: str) -> np.ndarray:
     """Half a unit in the last place of x in the cache dtype (normal range)."""
     a = np.abs(x)
