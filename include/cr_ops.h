@@ -79,6 +79,29 @@ cr_status cr_segment_project(const cr_target_dims* target, int32_t d_seg, const 
                              const float* sigma_stale, uint16_t* y, void* workspace,
                              size_t workspace_bytes, void* stream);
 
+/*
+ * cr_segment_project_noalloc - cr_segment_project without a workspace, for
+ * callers that cannot allocate device memory (an engine plugin living inside
+ * a fixed, pre-planned memory budget; a serving loop that must never call
+ * cudaMalloc, which can synchronise the device).  The paper has no
+ * counterpart: this is a deployment variant of the same computation.
+ *
+ * Its scratch (W_seg with 1/sigma_stale folded in, S*d_seg*d_h bf16 values)
+ * is a fixed 4 MiB device array inside the library, present on every GPU that
+ * loads the library until the process exits.  Shapes needing more return
+ * CR_ERR_UNSUPPORTED.  The first call on a device looks up that array's
+ * device address (cudaGetSymbolAddress); make that first call before any
+ * stream capture.  All calls share the one array, so calls whose kernels
+ * overlap on the GPU (different streams, no ordering between them) race on
+ * it; calls on one stream are safe.  Nothing in the array needs clearing:
+ * each call rewrites every element it reads.  Nothing is allocated or freed.
+ * Arguments, layouts and errors otherwise as cr_segment_project.
+ */
+cr_status cr_segment_project_noalloc(const cr_target_dims* target, int32_t d_seg,
+                                     const uint16_t* kv, int64_t n_tokens, const uint16_t* w_seg,
+                                     const float* b_seg, const float* sigma_stale, uint16_t* y,
+                                     void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -27,7 +27,8 @@ ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
           "-diag-suppress", "177",
           "-I" + INCLUDE, "-I" + CSRC]
-SOURCES = ["cr_api.cu", "cr_gemm.cu", "cr_attn.cu", "cr_segproj.cu", "cr_misc.cu"]
+SOURCES = ["cr_api.cu", "cr_gemm.cu", "cr_attn.cu", "cr_segproj.cu", "cr_misc.cu",
+           "cr_noalloc.cu"]
 
 
 def _nvcc() -> str:

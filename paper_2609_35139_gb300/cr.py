@@ -26,6 +26,7 @@ EXPORTED = [
     "cr_workspace_bytes", "cr_assemble_stale", "cr_compress_features", "cr_repair_forward",
     "cr_apply_residual", "cr_get_device_status", "cr_clear_device_status", "cr_status_str",
     "cr_linear", "cr_layernorm", "cr_chunk_causal_attention", "cr_qkv_rope", "cr_segment_project",
+    "cr_segment_project_noalloc",
 ]
 
 
@@ -97,6 +98,7 @@ def lib(build_if_missing: bool = False) -> ctypes.CDLL:
         "cr_qkv_rope": (i32, [vp, vp, vp, vp, i64, i32, i32, c_float, vp, vp]),
         "cr_segment_project": (i32, [P(cr_target_dims), i32, vp, i64, vp, vp, vp, vp, vp, c_size_t,
                                      vp]),
+        "cr_segment_project_noalloc": (i32, [P(cr_target_dims), i32, vp, i64, vp, vp, vp, vp, vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(L, name)
@@ -259,3 +261,10 @@ def cr_segment_project(target, d_seg, kv, w_seg, b_seg, sigma_stale, y, workspac
     _check("cr_segment_project", lib().cr_segment_project(
         ctypes.byref(target), d_seg, _p(kv), kv.shape[0], _p(w_seg), _p(b_seg), _p(sigma_stale),
         _p(y), _p(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def cr_segment_project_noalloc(target, d_seg, kv, w_seg, b_seg, sigma_stale, y, stream=None):
+    """cr_segment_project for callers that cannot allocate: no workspace argument."""
+    _check("cr_segment_project_noalloc", lib().cr_segment_project_noalloc(
+        ctypes.byref(target), d_seg, _p(kv), kv.shape[0], _p(w_seg), _p(b_seg), _p(sigma_stale),
+        _p(y), _stream(stream)))
