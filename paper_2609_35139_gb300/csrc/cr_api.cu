@@ -403,7 +403,7 @@ static cr_status attn_params(const Dims& d, const int32_t* chunk_end,
         if (len < 1) return CR_ERR_INVALID_ARG;
         p->req_start[r] = cu_seqlens_host[r];
         p->tile_prefix[r] = items;
-        items += (len + 127) / 128;
+        items += (len + 255) / 256;       // pairs of 128-query tiles
     }
     p->req_start[n_req] = cu_seqlens_host[n_req];
     p->tile_prefix[n_req] = items;

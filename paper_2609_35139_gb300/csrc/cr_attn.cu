@@ -2,22 +2,27 @@
 //   o_i = sum_{j : c(j) <= c(i)} softmax_j(q_i . k_j / sqrt(d)) v_j
 // inside each request.  Chunk ids are non-decreasing along a request, so the
 // keys visible to query i are exactly j < chunk_end[i]: a prefix.  A query
-// tile [q0, q0+128) therefore needs key tiles 0 .. ceil(max_i chunk_end / 128)
-// and nothing past that; those tiles are never loaded or multiplied.  Inside
-// the last tiles a per-row compare against chunk_end masks the rest.
+// tile therefore needs key tiles 0 .. ceil(max_i chunk_end / 128) - 1 and
+// nothing past that; those tiles are never loaded or multiplied.  Rows whose
+// chunk ends inside a key tile mask the rest of it; fully visible tiles do no
+// masking work at all.
 //
-// CTA = (request, 128-query tile, head).  Warp roles:
-//   warp 0      TMA: Q once, then K_j and V_j per key tile into a 3-deep ring
-//   warp 1      TMEM owner; one lane issues S_j = Q K_j^T (M=128, N=128,
-//               K=d, into one of two 128-column S buffers), and after the
-//               softmax has written P_j, PV_j = P_j V_j (M=128, N=d, K=128,
-//               V read MN-major) into one of two d-column buffers
-//   warps 2..5  one query row per thread: masked online softmax on S_j read
-//               from TMEM, P_j (bf16) written to shared memory in the
-//               128B-swizzled K-major layout the MMA reads, O kept in
-//               registers and updated as O = O * alpha_j + PV_j.
-// S_{j+1} is issued before waiting for P_j, so the tensor core works on the
-// next score tile while the softmax of the current one runs.
+// CTA = (request, head, two consecutive 128-query tiles).  10 warps:
+//   warp 0      TMA: both Q tiles once, then K_j and V_j per key tile into a
+//               3-deep ring shared by the two query tiles
+//   warp 1      TMEM owner; one lane issues, per key tile j and query tile w,
+//               S_w,j = Q_w K_j^T (M=128, N=128, K=d) into S_w, and after
+//               softmax w has written P_w,j, PV_w,j = P_w,j V_j (M=128, N=d,
+//               K=128, V read MN-major) into one of two PV buffers of w
+//   warps 2..5  softmax group 0 (query tile 0), one row per thread
+//   warps 6..9  softmax group 1 (query tile 1)
+// The two groups ping-pong: while group 0 turns S_0,j into P_0,j the tensor
+// core computes S_1,j, PV_0,j-1 and S_0,j+1, and the other way round.  A group
+// reads S_w,j from TMEM (two passes of 32-column loads: row max, then exp2,
+// row sum and bf16 P written to shared memory in the 128B-swizzled K-major
+// layout the MMA reads), then folds the previous tile's PV into its
+// register-resident O: O = O * alpha_{j-1} + PV_{j-1} (between the max pass
+// and the exp pass: PV_{j-1} is issued before S_j, so it is done by then).
 #include <cuda_bf16.h>
 
 #include "cr_internal.h"
@@ -34,14 +39,16 @@ struct AttnCfg {
     static constexpr uint32_t kSwz = (D == 64) ? SWZ_128B : SWZ_64B;
     static constexpr int kStages = 3;
     static constexpr uint32_t kPBytes = 128 * 128 * 2;
-    static constexpr uint32_t kQOff = 0;
-    static constexpr uint32_t kKVOff = kTileBytes;                       // K then V per stage
-    static constexpr uint32_t kPOff = kKVOff + kStages * 2 * kTileBytes;  // 2 P buffers
+    static constexpr uint32_t kQOff = 0;                                  // Q0, Q1
+    static constexpr uint32_t kKVOff = 2 * kTileBytes;                    // K, V per stage
+    static constexpr uint32_t kPOff = kKVOff + kStages * 2 * kTileBytes;  // P0, P1
     static constexpr uint32_t kBarOff = kPOff + 2 * kPBytes;
     static constexpr uint32_t kSmemBytes = 1024 + kBarOff + 256;
-    static constexpr uint32_t kTmemS = 0;      // two 128-column score buffers
-    static constexpr uint32_t kTmemPV = 256;   // two D-column PV buffers
+    static constexpr uint32_t kTmemS = 0;      // S_w at w * 128
+    static constexpr uint32_t kTmemPV = 256;   // PV_w,b at 256 + (2w + b) * D
 };
+
+constexpr int kThreads = 320;
 
 // Byte offset of 16 consecutive keys (c multiple of 16) of row r inside a
 // [128 x 128] bf16 P tile held as two 64-column, 128B-swizzled K-major atoms.
@@ -52,8 +59,14 @@ __device__ __forceinline__ void p_offsets(int r, int c, uint32_t* o0, uint32_t* 
     *o1 = base + (((ch + 1) ^ (r & 7)) << 4);
 }
 
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
 template <int D>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQKV, const __grid_constant__ AttnParams p) {
     using Cfg = AttnCfg<D>;
     constexpr int NS = Cfg::kStages;
@@ -69,24 +82,30 @@ __global__ void __launch_bounds__(192, 1)
     uint64_t* k_full = bars + 1;
     uint64_t* v_full = k_full + NS;
     uint64_t* kv_empty = v_full + NS;
-    uint64_t* s_full = kv_empty + NS;
-    uint64_t* p_full = s_full + 2;
-    uint64_t* pv_full = p_full + 2;
-    uint64_t* drain = pv_full + 2;
+    uint64_t* s_full = kv_empty + NS;     // [2]
+    uint64_t* s_free = s_full + 2;        // [2]
+    uint64_t* p_full = s_free + 2;        // [2]
+    uint64_t* pv_full = p_full + 2;       // [2][2]
+    uint64_t* pv_free = pv_full + 4;      // [2][2]
+    uint64_t* drain = pv_free + 4;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
     int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
-    // ---- work item: heaviest (last) query tiles first
+    // ---- work item: (request, pair of query tiles, head); heaviest pairs first
     const int head = blockIdx.x % p.n_heads;
     const int item = p.n_items - 1 - static_cast<int>(blockIdx.x / p.n_heads);
     int req = 0;
     while (req + 1 < p.n_req && p.tile_prefix[req + 1] <= item) ++req;
-    const int q0 = (item - p.tile_prefix[req]) * 128;
+    const int q0 = (item - p.tile_prefix[req]) * 256;
     const int rs = p.req_start[req];
     const int len = p.req_start[req + 1] - rs;
-    const int last = min(q0 + 127, len - 1);
-    const int kv_extent = __ldg(p.chunk_end + rs + last);      // keys visible to the tile
-    const int n_kv = (kv_extent + 127) / 128;
+    int n_kv[2];
+#pragma unroll
+    for (int w = 0; w < 2; ++w) {
+        const int first = q0 + 128 * w;
+        n_kv[w] = first < len ? (__ldg(p.chunk_end + rs + min(first + 127, len - 1)) + 127) / 128 : 0;
+    }
+    const int n_max = max(n_kv[0], n_kv[1]);
 
     const uint32_t warp = warp_id(), lane = lane_id();
     if (threadIdx.x == 0) {
@@ -96,10 +115,14 @@ __global__ void __launch_bounds__(192, 1)
             mbar_init(&v_full[s], 1);
             mbar_init(&kv_empty[s], 1);
         }
-        for (int s = 0; s < 2; ++s) {
-            mbar_init(&s_full[s], 1);
-            mbar_init(&p_full[s], 128);
-            mbar_init(&pv_full[s], 1);
+        for (int w = 0; w < 2; ++w) {
+            mbar_init(&s_full[w], 1);
+            mbar_init(&s_free[w], 128);
+            mbar_init(&p_full[w], 128);
+            for (int b = 0; b < 2; ++b) {
+                mbar_init(&pv_full[2 * w + b], 1);
+                mbar_init(&pv_free[2 * w + b], 128);
+            }
         }
         mbar_init(drain, 1);
         *abort_flag = 0;
@@ -114,11 +137,14 @@ __global__ void __launch_bounds__(192, 1)
 
     if (warp == 0) {
         if (lane == 0) {
+            // ---------------------------------------------------- TMA producer
             tma_prefetch(&tmQKV);
-            mbar_expect_tx(q_full, Cfg::kTileBytes);
+            mbar_expect_tx(q_full, 2 * Cfg::kTileBytes);
             tma_load_2d(smem + Cfg::kQOff, &tmQKV, q_full, head * D, rs + q0);
+            tma_load_2d(smem + Cfg::kQOff + Cfg::kTileBytes, &tmQKV, q_full, head * D,
+                        rs + q0 + 128);
             bool ok = true;
-            for (int j = 0; j < n_kv; ++j) {
+            for (int j = 0; j < n_max; ++j) {
                 const int st = j % NS;
                 const uint32_t ph = static_cast<uint32_t>(j / NS) & 1u;
                 if (!(ok = mbar_wait(&kv_empty[st], ph ^ 1u, wc, 121))) break;
@@ -137,137 +163,180 @@ __global__ void __launch_bounds__(192, 1)
         }
     } else if (warp == 1) {
         if (lane == 0) {
-            const uint32_t sq = smem_u32(smem + Cfg::kQOff);
-            auto issue_s = [&](int j) -> bool {
+            // ---------------------------------------------------- MMA issuer
+            const uint32_t sq0 = smem_u32(smem + Cfg::kQOff);
+            auto issue_s = [&](int w, int j) -> bool {
                 const int st = j % NS;
-                const uint32_t ph = static_cast<uint32_t>(j / NS) & 1u;
-                if (!mbar_wait(&k_full[st], ph, wc, 222)) return false;
+                if (!mbar_wait(&k_full[st], static_cast<uint32_t>(j / NS) & 1u, wc, 222)) return false;
+                if (j > 0 && !mbar_wait(&s_free[w], static_cast<uint32_t>(j - 1) & 1u, wc, 223))
+                    return false;
                 tc_fence_after();
+                const uint32_t sq = sq0 + w * Cfg::kTileBytes;
                 const uint32_t sk = smem_u32(smem + Cfg::kKVOff + st * 2 * Cfg::kTileBytes);
-                const uint32_t d = tmem_base + Cfg::kTmemS + (j & 1) * 128;
+                const uint32_t d = tmem_base + Cfg::kTmemS + w * 128;
 #pragma unroll
                 for (int k = 0; k < D / 16; ++k)
                     mma_bf16_ss(d, smem_desc(sq + k * 32, 16, Cfg::kAtomBytes, Cfg::kSwz),
                                 smem_desc(sk + k * 32, 16, Cfg::kAtomBytes, Cfg::kSwz), IDESC_S,
                                 k != 0 ? 1u : 0u);
-                mma_commit(&s_full[j & 1]);
+                mma_commit(&s_full[w]);
                 return true;
             };
-            bool ok = mbar_wait(q_full, 0, wc, 221);
-            if (ok) {
-                tc_fence_after();
-                ok = issue_s(0);
-            }
-            for (int j = 0; j < n_kv && ok; ++j) {
-                if (j + 1 < n_kv && !(ok = issue_s(j + 1))) break;
+            auto issue_pv = [&](int w, int j) -> bool {
                 const int st = j % NS;
-                const uint32_t ph = static_cast<uint32_t>(j / NS) & 1u;
-                if (!(ok = mbar_wait(&p_full[j & 1], static_cast<uint32_t>(j >> 1) & 1u, wc, 223)))
-                    break;
-                if (!(ok = mbar_wait(&v_full[st], ph, wc, 224))) break;
+                const int b = j & 1;
+                if (!mbar_wait(&p_full[w], static_cast<uint32_t>(j) & 1u, wc, 224)) return false;
+                if (!mbar_wait(&v_full[st], static_cast<uint32_t>(j / NS) & 1u, wc, 225)) return false;
+                if (j >= 2 &&
+                    !mbar_wait(&pv_free[2 * w + b], static_cast<uint32_t>((j - 2) >> 1) & 1u, wc, 226))
+                    return false;
                 tc_fence_after();
-                const uint32_t sp = smem_u32(smem + Cfg::kPOff + (j & 1) * Cfg::kPBytes);
+                const uint32_t sp = smem_u32(smem + Cfg::kPOff + w * Cfg::kPBytes);
                 const uint32_t sv =
                     smem_u32(smem + Cfg::kKVOff + st * 2 * Cfg::kTileBytes + Cfg::kTileBytes);
-                const uint32_t d = tmem_base + Cfg::kTmemPV + (j & 1) * D;
+                const uint32_t d = tmem_base + Cfg::kTmemPV + (2 * w + b) * D;
 #pragma unroll
                 for (int kk = 0; kk < 8; ++kk) {
                     const uint64_t da =
                         smem_desc(sp + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024, SWZ_128B);
-                    // V: rows = keys (K dimension), D contiguous (MN-major);
-                    // 16 keys = 2 swizzle atoms of 8 rows.
+                    // V: rows = keys (the K dimension), d contiguous (MN-major);
+                    // 16 keys = two 8-row swizzle atoms.
                     const uint64_t db = smem_desc(sv + kk * 16 * Cfg::kRowBytes, Cfg::kTileBytes,
                                                   Cfg::kAtomBytes, Cfg::kSwz);
                     mma_bf16_ss(d, da, db, IDESC_PV, kk != 0 ? 1u : 0u);
                 }
-                mma_commit(&pv_full[j & 1]);
-                mma_commit(&kv_empty[st]);
+                mma_commit(&pv_full[2 * w + b]);
+                return true;
+            };
+            bool ok = mbar_wait(q_full, 0, wc, 221);
+            if (ok) tc_fence_after();
+            for (int w = 0; w < 2 && ok; ++w)
+                if (n_kv[w] > 0) ok = issue_s(w, 0);
+            for (int j = 0; j < n_max && ok; ++j) {
+                for (int w = 0; w < 2 && ok; ++w) {
+                    if (j >= n_kv[w]) continue;
+                    if (!(ok = issue_pv(w, j))) break;
+                    if (j + 1 < n_kv[w]) ok = issue_s(w, j + 1);
+                }
+                if (ok) mma_commit(&kv_empty[j % NS]);
             }
             mma_commit(drain);
-            mbar_wait(drain, 0, wc, 225);
+            mbar_wait(drain, 0, wc, 227);
         }
     } else {
-        // ---------------------------------------------------- softmax (warps 2..5)
+        // ---------------------------------------------------- softmax groups
+        const int w = (warp >= 6) ? 1 : 0;
         const uint32_t quad = warp & 3u;
         const int r = static_cast<int>(quad * 32 + lane);
-        const int qrow = q0 + r;
+        const int qrow = q0 + 128 * w + r;
         const bool valid = qrow < len;
         const int cend = valid ? __ldg(p.chunk_end + rs + qrow) : 1;
         const uint32_t lane_off = (quad * 32u) << 16;
-        float m = NEG_INF, l = 0.0f;
+        const uint32_t ts = tmem_base + lane_off + Cfg::kTmemS + w * 128;
+        const float sc = p.scale_log2;
+        const int n = n_kv[w];
+        uint8_t* pt = smem + Cfg::kPOff + w * Cfg::kPBytes;
+        float m = NEG_INF, l = 0.0f, alpha_prev = 0.0f;
         float o[D];
 #pragma unroll
         for (int i = 0; i < D; ++i) o[i] = 0.0f;
+
+        auto fold = [&](int jj) -> bool {   // O = O * alpha_prev + PV_jj
+            const int b = jj & 1;
+            bool okf = mbar_wait(&pv_full[2 * w + b], static_cast<uint32_t>(jj >> 1) & 1u, wc, 322);
+            if (!__all_sync(0xffffffffu, okf)) return false;
+            tc_fence_after();
+            const uint32_t tp = tmem_base + lane_off + Cfg::kTmemPV + (2 * w + b) * D;
+#pragma unroll
+            for (int c = 0; c < D; c += 32) {
+                float v[32];
+                __syncwarp();
+                tmem_ld32(tp + c, v);
+                tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) o[c + i] = fmaf(o[c + i], alpha_prev, v[i]);
+            }
+            tc_fence_before();
+            mbar_arrive(&pv_free[2 * w + b]);
+            return true;
+        };
+
         bool ok = true;
-        for (int j = 0; j < n_kv; ++j) {
-            ok = mbar_wait(&s_full[j & 1], static_cast<uint32_t>(j >> 1) & 1u, wc, 321);
+        for (int j = 0; j < n; ++j) {
+            ok = mbar_wait(&s_full[w], static_cast<uint32_t>(j) & 1u, wc, 321);
             if (!__all_sync(0xffffffffu, ok)) {
                 ok = false;
                 break;
             }
             tc_fence_after();
             const int k0 = j * 128;
-            const uint32_t ts = tmem_base + lane_off + Cfg::kTmemS + (j & 1) * 128;
-            // pass 1: row max of the scaled, masked scores
+            const bool full_tile = k0 + 128 <= cend;     // all 128 keys visible to this row
+            // pass 1: row max of the (masked) scores
             float mx = NEG_INF;
-            for (int c = 0; c < 128; c += 16) {
-                float v[16];
-                __syncwarp();
-                tmem_ld16(ts + c, v);
-                tmem_wait_ld();
 #pragma unroll
-                for (int i = 0; i < 16; ++i)
-                    if (k0 + c + i < cend) mx = fmaxf(mx, v[i] * p.scale_log2);
-            }
-            const float m_new = fmaxf(m, mx);
-            const float alpha = exp2f(m - m_new);
-            // pass 2: probabilities -> P (bf16, swizzled K-major), row sum
-            float rsum = 0.0f;
-            uint8_t* pt = smem + Cfg::kPOff + (j & 1) * Cfg::kPBytes;
-            for (int c = 0; c < 128; c += 16) {
-                float v[16];
+            for (int c = 0; c < 128; c += 32) {
+                float v[32];
                 __syncwarp();
-                tmem_ld16(ts + c, v);
+                tmem_ld32(ts + c, v);
                 tmem_wait_ld();
+                if (full_tile) {
 #pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    const float e = (k0 + c + i < cend) ? exp2f(v[i] * p.scale_log2 - m_new) : 0.0f;
-                    v[i] = e;
-                    rsum += e;
+                    for (int i = 0; i < 32; ++i) mx = fmaxf(mx, v[i]);
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i)
+                        if (k0 + c + i < cend) mx = fmaxf(mx, v[i]);
                 }
-                uint32_t o0, o1;
-                p_offsets(r, c, &o0, &o1);
-                *reinterpret_cast<uint4*>(pt + o0) =
-                    make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
-                               pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
-                *reinterpret_cast<uint4*>(pt + o1) =
-                    make_uint4(pack_bf16x2(v[8], v[9]), pack_bf16x2(v[10], v[11]),
-                               pack_bf16x2(v[12], v[13]), pack_bf16x2(v[14], v[15]));
             }
-            l = l * alpha + rsum;
-            m = m_new;
-            fence_async_smem();
-            tc_fence_before();
-            mbar_arrive(&p_full[j & 1]);
-            ok = mbar_wait(&pv_full[j & 1], static_cast<uint32_t>(j >> 1) & 1u, wc, 322);
-            if (!__all_sync(0xffffffffu, ok)) {
+            const float m_new = fmaxf(m, mx * sc);
+            const float alpha = ex2(m - m_new);
+            // PV_{j-1} was issued before S_j, so it is complete by now: fold it,
+            // which also frees the P buffer for P_j
+            if (j > 0 && !fold(j - 1)) {
                 ok = false;
                 break;
             }
-            tc_fence_after();
-            const uint32_t tp = tmem_base + lane_off + Cfg::kTmemPV + (j & 1) * D;
+            alpha_prev = alpha;
+            // pass 2: probabilities -> P (bf16, swizzled K-major), row sum
+            float rsum = 0.0f;
 #pragma unroll
-            for (int c = 0; c < D; c += 16) {
-                float v[16];
+            for (int c = 0; c < 128; c += 32) {
+                float v[32];
                 __syncwarp();
-                tmem_ld16(tp + c, v);
+                tmem_ld32(ts + c, v);
                 tmem_wait_ld();
+                uint32_t pk[16];
 #pragma unroll
-                for (int i = 0; i < 16; ++i) o[c + i] = fmaf(o[c + i], alpha, v[i]);
+                for (int i = 0; i < 32; i += 2) {
+                    float e0 = ex2(fmaf(v[i], sc, -m_new));
+                    float e1 = ex2(fmaf(v[i + 1], sc, -m_new));
+                    if (!full_tile) {
+                        if (k0 + c + i >= cend) e0 = 0.0f;
+                        if (k0 + c + i + 1 >= cend) e1 = 0.0f;
+                    }
+                    rsum += e0 + e1;
+                    pk[i >> 1] = pack_bf16x2(e0, e1);
+                }
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    uint32_t o0, o1;
+                    p_offsets(r, c + 16 * h, &o0, &o1);
+                    *reinterpret_cast<uint4*>(pt + o0) =
+                        make_uint4(pk[8 * h], pk[8 * h + 1], pk[8 * h + 2], pk[8 * h + 3]);
+                    *reinterpret_cast<uint4*>(pt + o1) =
+                        make_uint4(pk[8 * h + 4], pk[8 * h + 5], pk[8 * h + 6], pk[8 * h + 7]);
+                }
             }
+            l = l * alpha + rsum;
+            m = m_new;
+            tc_fence_before();
+            mbar_arrive(&s_free[w]);          // S_w may now be overwritten by S_w,j+1
+            fence_async_smem();
+            mbar_arrive(&p_full[w]);
         }
+        if (ok && n > 0) ok = fold(n - 1);
         tc_fence_before();
-        if (ok && valid) {
+        if (ok && valid && n > 0) {
             const float inv = 1.0f / l;
             uint16_t* dst = p.out + static_cast<int64_t>(rs + qrow) * p.d_b + head * D;
 #pragma unroll
@@ -296,7 +365,7 @@ cr_status launch_d(const CUtensorMap& tm, const AttnParams& p, cudaStream_t st) 
     const cr_status sa = ensure_smem_attr(kern, static_cast<int>(Cfg::kSmemBytes), &attr_done);
     if (sa != CR_OK) return sa;
     const int grid = p.n_items * p.n_heads;
-    kern<<<grid, 192, Cfg::kSmemBytes, st>>>(tm, p);
+    kern<<<grid, kThreads, Cfg::kSmemBytes, st>>>(tm, p);
     return cuda_check(cudaGetLastError());
 }
 

@@ -89,11 +89,11 @@ struct AttnParams {
     int32_t d_b;
     int32_t n_heads;
     int32_t n_req;
-    int32_t n_items;         // total (request, q-tile) pairs
+    int32_t n_items;         // total (request, pair of 128-query tiles) items
     float scale_log2;        // log2(e) / sqrt(d)
     unsigned* status;
     int32_t req_start[kMaxReq + 1];   // cu_seqlens
-    int32_t tile_prefix[kMaxReq + 1]; // cumulative q tiles
+    int32_t tile_prefix[kMaxReq + 1]; // cumulative items per request
 };
 
 // ------------------------------------------------------------------ host helpers
