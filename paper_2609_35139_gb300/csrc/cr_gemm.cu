@@ -2,19 +2,22 @@
 //   C[M, N] = A[M, K] * W[N, K]^T + bias, with a fused epilogue.
 //
 // Design (sm_103a, one CTA per SM, persistent):
-//   warp 0      TMA producer: A and W k-slices (64 wide, 128B swizzle) into a
-//               STAGES-deep shared-memory ring; for the residual epilogue also
-//               the stale cache tile [128, BN] of the output.
-//   warp 1      allocates TMEM, one elected lane issues tcgen05.mma
+//   warp 0      TMA producer: per output tile, first the epilogue's inputs —
+//               the bias (and sigma_delta) slice of the tile by bulk copy and,
+//               for in-place epilogues, the output tile itself (the stale cache
+//               tile, or the fp32 residual-stream tile) by TMA — then A and W
+//               k-slices (64 wide, 128B swizzle) into a shared-memory ring.
+//   warp 1      allocates TMEM; one elected lane issues tcgen05.mma
 //               (M = 128, N = BN, K = 16) into a double-buffered fp32
-//               accumulator (2 x BN TMEM columns), commits to mbarriers.
-//   warps 2..5  epilogue: tcgen05.ld 32 lanes x 16 columns, bias, then one of
-//               bf16 store / GELU / fp32 residual add / RoPE on Q,K /
-//               in-place "kv + sigma_delta * z" (+ R_M on K) on the staged
-//               cache tile, written back with TMA stores.
-// Tiles are walked W-tile-major (all M tiles of one N tile back to back), so
-// a W tile is read from HBM once and reused from L2 while the small A
-// operand stays L2-resident.
+//               accumulator (2 x BN TMEM columns) and commits to mbarriers.
+//   warps 2..5  epilogue: tcgen05.ld 32 lanes x 16 columns, bias from shared
+//               memory, then one of: bf16 store, GELU, fp32 store, RoPE on Q/K,
+//               or in place on the staged tile: residual stream x += acc + b,
+//               cache kv = kv + sigma_delta (acc + b) (+ R_M on K); staged
+//               tiles go back with TMA stores.
+// The epilogue of tile i overlaps the MMAs of tile i+1.  Tiles are walked
+// W-tile-major (all M tiles of one N tile back to back), so a W tile is read
+// from HBM once and reused from L2 while the small A operand stays L2-resident.
 #include <cuda_bf16.h>
 
 #include "cr_internal.h"
@@ -26,19 +29,25 @@ namespace {
 constexpr int BM = 128;
 constexpr int BK = 64;
 constexpr uint32_t A_BYTES = BM * BK * 2;
+constexpr uint32_t kSmemLimit = 232448;   // 227 KB opt-in per CTA
 
 template <int BN, int EPI>
 struct GemmCfg {
     static constexpr bool kKV = (EPI == EPI_KV_BF16 || EPI == EPI_KV_F32);
-    static constexpr int kKVEsize = (EPI == EPI_KV_F32) ? 4 : 2;
+    static constexpr bool kInPlace = kKV || EPI == EPI_ADD_F32;
+    static constexpr int kTileEsize = (EPI == EPI_KV_F32 || EPI == EPI_ADD_F32) ? 4 : 2;
+    static constexpr uint32_t kTileBytes = kInPlace ? BM * BN * kTileEsize : 0;
+    static constexpr int kBoxCols = 128 / kTileEsize;          // one 128-byte swizzle row
+    static constexpr int kBoxes = kInPlace ? BN / kBoxCols : 0;
+    static constexpr uint32_t kVecBytes = BN * 4 * (kKV ? 2 : 1);   // bias (+ sigma)
     static constexpr uint32_t kBBytes = BN * BK * 2;
     static constexpr uint32_t kStageBytes = A_BYTES + kBBytes;
-    static constexpr int kStages = kKV ? (BN == 256 ? 3 : 4) : (BN == 256 ? 4 : 6);
-    static constexpr uint32_t kKVBytes = kKV ? BM * BN * kKVEsize : 0;
-    static constexpr int kKVBoxCols = 128 / kKVEsize;          // one 128-byte swizzle row
-    static constexpr int kKVBoxes = kKV ? BN / kKVBoxCols : 0;
+    static constexpr uint32_t kFixed = 1024 + kTileBytes + kVecBytes + 256;
+    static constexpr int kStagesFit = static_cast<int>((kSmemLimit - kFixed) / kStageBytes);
+    static constexpr int kStages = kStagesFit > 6 ? 6 : kStagesFit;
+    static_assert(kStages >= 2, "GEMM tile does not fit in shared memory");
+    static constexpr uint32_t kSmemBytes = kFixed + kStages * kStageBytes;
     static constexpr uint32_t kTmemCols = 2 * BN;
-    static constexpr uint32_t kSmemBytes = 1024 + kStages * kStageBytes + kKVBytes + 256;
 };
 
 __device__ __forceinline__ float gelu_erf(float x) {
@@ -46,8 +55,7 @@ __device__ __forceinline__ float gelu_erf(float x) {
 }
 
 // 16 consecutive bf16 of a [128 x (64*k)] tile stored as 128B-swizzled boxes
-// of 64 columns; col multiple of 16.  Returns the byte offsets of its two
-// 16-byte chunks.
+// of 64 columns; col multiple of 16.  Byte offsets of its two 16-byte chunks.
 __device__ __forceinline__ void swz_offsets_bf16(int row, int col, uint32_t* o0, uint32_t* o1) {
     const int box = col >> 6;
     const int ch = (col & 63) >> 3;
@@ -72,17 +80,11 @@ __device__ __forceinline__ void load16_bf16_smem(const uint8_t* tile, int row, i
 __device__ __forceinline__ void store16_bf16_smem(uint8_t* tile, int row, int col, const float* v) {
     uint32_t o0, o1;
     swz_offsets_bf16(row, col, &o0, &o1);
-    uint4 a, b;
-    a.x = pack_bf16x2(v[0], v[1]);
-    a.y = pack_bf16x2(v[2], v[3]);
-    a.z = pack_bf16x2(v[4], v[5]);
-    a.w = pack_bf16x2(v[6], v[7]);
-    b.x = pack_bf16x2(v[8], v[9]);
-    b.y = pack_bf16x2(v[10], v[11]);
-    b.z = pack_bf16x2(v[12], v[13]);
-    b.w = pack_bf16x2(v[14], v[15]);
-    *reinterpret_cast<uint4*>(tile + o0) = a;
-    *reinterpret_cast<uint4*>(tile + o1) = b;
+    *reinterpret_cast<uint4*>(tile + o0) = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
+                                                      pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
+    *reinterpret_cast<uint4*>(tile + o1) =
+        make_uint4(pack_bf16x2(v[8], v[9]), pack_bf16x2(v[10], v[11]), pack_bf16x2(v[12], v[13]),
+                   pack_bf16x2(v[14], v[15]));
 }
 
 // fp32 tile: boxes of 32 columns (128 B rows), 4 chunks of 4 floats.
@@ -110,24 +112,40 @@ __device__ __forceinline__ void store16_f32_smem(uint8_t* tile, int row, int col
             make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
 }
 
-__device__ __forceinline__ void store16_bf16_global(uint16_t* dst, const float* v) {
-    uint4 a, b;
-    a.x = pack_bf16x2(v[0], v[1]);
-    a.y = pack_bf16x2(v[2], v[3]);
-    a.z = pack_bf16x2(v[4], v[5]);
-    a.w = pack_bf16x2(v[6], v[7]);
-    b.x = pack_bf16x2(v[8], v[9]);
-    b.y = pack_bf16x2(v[10], v[11]);
-    b.z = pack_bf16x2(v[12], v[13]);
-    b.w = pack_bf16x2(v[14], v[15]);
-    reinterpret_cast<uint4*>(dst)[0] = a;
-    reinterpret_cast<uint4*>(dst)[1] = b;
+template <int ES>
+__device__ __forceinline__ void load16_tile(const uint8_t* t, int row, int col, float* v) {
+    if constexpr (ES == 2)
+        load16_bf16_smem(t, row, col, v);
+    else
+        load16_f32_smem(t, row, col, v);
+}
+template <int ES>
+__device__ __forceinline__ void store16_tile(uint8_t* t, int row, int col, const float* v) {
+    if constexpr (ES == 2)
+        store16_bf16_smem(t, row, col, v);
+    else
+        store16_f32_smem(t, row, col, v);
 }
 
-__device__ __forceinline__ void add_bias16(float* v, const float* bias, int col) {
-    if (bias) {
+__device__ __forceinline__ void store16_bf16_global(uint16_t* dst, const float* v) {
+    reinterpret_cast<uint4*>(dst)[0] = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
+                                                  pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
+    reinterpret_cast<uint4*>(dst)[1] =
+        make_uint4(pack_bf16x2(v[8], v[9]), pack_bf16x2(v[10], v[11]), pack_bf16x2(v[12], v[13]),
+                   pack_bf16x2(v[14], v[15]));
+}
+
+// 16 consecutive floats of a shared-memory vector (all lanes read the same
+// addresses: broadcast).
+__device__ __forceinline__ void vec16(const float* v, int col, float* out) {
+    const float4* p4 = reinterpret_cast<const float4*>(v + col);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) v[i] += __ldg(bias + col + i);
+    for (int q = 0; q < 4; ++q) {
+        const float4 x = p4[q];
+        out[4 * q] = x.x;
+        out[4 * q + 1] = x.y;
+        out[4 * q + 2] = x.z;
+        out[4 * q + 3] = x.w;
     }
 }
 
@@ -153,15 +171,16 @@ __global__ void __launch_bounds__(192, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    uint8_t* kv_tile = smem + STAGES * Cfg::kStageBytes;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(kv_tile + Cfg::kKVBytes);
+    uint8_t* tile = smem + STAGES * Cfg::kStageBytes;              // staged output tile
+    float* vec = reinterpret_cast<float*>(tile + Cfg::kTileBytes);  // bias [BN] (+ sigma [BN])
+    uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(vec) + Cfg::kVecBytes);
     uint64_t* full = bars;
     uint64_t* empty = bars + STAGES;
     uint64_t* tfull = bars + 2 * STAGES;
     uint64_t* tempty = tfull + 2;
-    uint64_t* kvfull = tempty + 2;
-    uint64_t* kvempty = kvfull + 1;
-    uint64_t* drain = kvempty + 1;
+    uint64_t* epi_full = tempty + 2;
+    uint64_t* epi_empty = epi_full + 1;
+    uint64_t* drain = epi_empty + 1;
     uint64_t* epi_done = drain + 1;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(epi_done + 1);
     int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
@@ -176,8 +195,8 @@ __global__ void __launch_bounds__(192, 1)
             mbar_init(&tfull[s], 1);
             mbar_init(&tempty[s], 4);
         }
-        mbar_init(kvfull, 1);
-        mbar_init(kvempty, 1);
+        mbar_init(epi_full, 1);
+        mbar_init(epi_empty, 1);
         mbar_init(drain, 1);
         mbar_init(epi_done, 128);
         *abort_flag = 0;
@@ -192,25 +211,35 @@ __global__ void __launch_bounds__(192, 1)
 
     const int total = p.num_m * p.num_n;
     const int num_k = (p.K + BK - 1) / BK;
+    const bool has_bias = p.bias != nullptr;
+    // the epilogue consumes a per-tile load (vectors and/or the staged tile)
+    const bool epi_load = Cfg::kInPlace || has_bias;
 
     if (warp == 0) {
         if (lane == 0) {
             // ------------------------------------------------ TMA producer
             tma_prefetch(&tmA);
             tma_prefetch(&tmB);
-            if constexpr (Cfg::kKV) tma_prefetch(&tmC);
-            uint32_t stage = 0, phase = 0, kv_phase = 0;
+            if constexpr (Cfg::kInPlace) tma_prefetch(&tmC);
+            uint32_t stage = 0, phase = 0, epi_phase = 0;
             bool ok = true;
             for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
                 const int m0 = (t % p.num_m) * BM;
                 const int n0 = (t / p.num_m) * BN;
-                if constexpr (Cfg::kKV) {
-                    if (!(ok = mbar_wait(kvempty, kv_phase ^ 1u, wc, 101))) break;
-                    mbar_expect_tx(kvfull, Cfg::kKVBytes);
-                    for (int b = 0; b < Cfg::kKVBoxes; ++b)
-                        tma_load_2d(kv_tile + b * 16384, &tmC, kvfull, n0 + b * Cfg::kKVBoxCols,
-                                    m0);
-                    kv_phase ^= 1u;
+                if (epi_load) {
+                    if (!(ok = mbar_wait(epi_empty, epi_phase ^ 1u, wc, 101))) break;
+                    const int nb = min(BN, p.N - n0);
+                    const uint32_t vbytes = static_cast<uint32_t>(nb) * 4u;
+                    uint32_t bytes = Cfg::kTileBytes + (has_bias ? vbytes : 0u);
+                    if constexpr (Cfg::kKV) bytes += vbytes;
+                    mbar_expect_tx(epi_full, bytes);
+                    if constexpr (Cfg::kInPlace) {
+                        for (int b = 0; b < Cfg::kBoxes; ++b)
+                            tma_load_2d(tile + b * 16384, &tmC, epi_full, n0 + b * Cfg::kBoxCols, m0);
+                    }
+                    if (has_bias) bulk_load(vec, p.bias + n0, vbytes, epi_full);
+                    if constexpr (Cfg::kKV) bulk_load(vec + BN, p.sigma + n0, vbytes, epi_full);
+                    epi_phase ^= 1u;
                 }
                 for (int kb = 0; kb < num_k; ++kb) {
                     if (!(ok = mbar_wait(&empty[stage], phase ^ 1u, wc, 102))) break;
@@ -269,12 +298,14 @@ __global__ void __launch_bounds__(192, 1)
         // ---------------------------------------------------- epilogue (warps 2..5)
         const uint32_t quad = warp & 3u;
         const int r = static_cast<int>(quad * 32 + lane);     // row inside the tile
-        uint32_t acc = 0, acc_phase = 0, kv_phase = 0;
+        uint32_t acc = 0, acc_phase = 0, epi_phase = 0;
+        const float* vb = vec;             // bias slice of the tile
+        const float* vs = vec + BN;        // sigma_delta slice (KV epilogues)
         for (int t = blockIdx.x; t < total; t += gridDim.x) {
             const int m0 = (t % p.num_m) * BM;
             const int n0 = (t / p.num_m) * BN;
             bool ok = mbar_wait(&tfull[acc], acc_phase, wc, 301);
-            if constexpr (Cfg::kKV) ok = ok && mbar_wait(kvfull, kv_phase, wc, 302);
+            if (epi_load) ok = ok && mbar_wait(epi_full, epi_phase, wc, 302);
             if (!__all_sync(0xffffffffu, ok)) break;
             tc_fence_after();
             const int row = m0 + r;
@@ -288,53 +319,88 @@ __global__ void __launch_bounds__(192, 1)
                 for (int h0 = 0; h0 < BN; h0 += hd) {
                     const bool rot = (n0 + h0) < p.rope_cols;
                     for (int j = 0; j < hd / 2; j += 16) {
-                        float a[16], b[16];
+                        float a[16], b[16], ba[16], bb[16];
+                        __syncwarp();
                         tmem_ld16(taddr + h0 + j, a);
                         tmem_ld16(taddr + h0 + hd / 2 + j, b);
                         tmem_wait_ld();
-                        const int ca = n0 + h0 + j, cb = n0 + h0 + hd / 2 + j;
-                        add_bias16(a, p.bias, ca);
-                        add_bias16(b, p.bias, cb);
+                        const int ta = h0 + j, tb = h0 + hd / 2 + j;
+                        if (has_bias) {
+                            vec16(vb, ta, ba);
+                            vec16(vb, tb, bb);
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) {
+                                a[i] += ba[i];
+                                b[i] += bb[i];
+                            }
+                        }
                         if (rot) rotate16(a, b, pr, p.inv_freq, j);
                         if (row_ok) {
-                            store16_bf16_global(orow + ca, a);
-                            store16_bf16_global(orow + cb, b);
+                            store16_bf16_global(orow + n0 + ta, a);
+                            store16_bf16_global(orow + n0 + tb, b);
                         }
                     }
                 }
-            } else if constexpr (Cfg::kKV) {
-                const int dh = p.rope_dim;
-                const float pr = row_ok ? static_cast<float>(__ldg(p.pos + row)) : 0.0f;
-                for (int s0 = 0; s0 < BN; s0 += dh) {
-                    const int gseg = (n0 + s0) / dh;
-                    const bool rot = p.rope_on && (((gseg / p.n_kv_heads) & 1) == 0);
-                    for (int j = 0; j < dh / 2; j += 16) {
-                        float a[16], b[16], ka[16], kb[16];
-                        tmem_ld16(taddr + s0 + j, a);
-                        tmem_ld16(taddr + s0 + dh / 2 + j, b);
-                        const int ta = s0 + j, tb = s0 + dh / 2 + j;   // tile columns
-                        if constexpr (EPI == EPI_KV_BF16) {
-                            load16_bf16_smem(kv_tile, r, ta, ka);
-                            load16_bf16_smem(kv_tile, r, tb, kb);
+            } else if constexpr (Cfg::kInPlace) {
+                constexpr int ES = Cfg::kTileEsize;
+                if (Cfg::kKV && p.rope_on) {
+                    // R_M pairs (d, d + d_h/2) live inside one d_h-wide segment
+                    const int dh = p.rope_dim;
+                    const float pr = row_ok ? static_cast<float>(__ldg(p.pos + row)) : 0.0f;
+                    for (int s0 = 0; s0 < BN; s0 += dh) {
+                        const int gseg = (n0 + s0) / dh;
+                        const bool rot = ((gseg / p.n_kv_heads) & 1) == 0;
+                        for (int j = 0; j < dh / 2; j += 16) {
+                            float a[16], b[16], ka[16], kb[16], sa_[16], sb_[16], ba[16], bb[16];
+                            const int ta = s0 + j, tb = s0 + dh / 2 + j;
+                            __syncwarp();
+                            tmem_ld16(taddr + ta, a);
+                            tmem_ld16(taddr + tb, b);
+                            load16_tile<ES>(tile, r, ta, ka);
+                            load16_tile<ES>(tile, r, tb, kb);
+                            vec16(vs, ta, sa_);
+                            vec16(vs, tb, sb_);
+                            if (has_bias) {
+                                vec16(vb, ta, ba);
+                                vec16(vb, tb, bb);
+                            } else {
+#pragma unroll
+                                for (int i = 0; i < 16; ++i) ba[i] = bb[i] = 0.0f;
+                            }
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) {
+                                ka[i] = fmaf(sa_[i], a[i] + ba[i], ka[i]);
+                                kb[i] = fmaf(sb_[i], b[i] + bb[i], kb[i]);
+                            }
+                            if (rot) rotate16(ka, kb, pr, p.inv_freq, j);
+                            store16_tile<ES>(tile, r, ta, ka);
+                            store16_tile<ES>(tile, r, tb, kb);
+                        }
+                    }
+                } else {
+                    for (int c = 0; c < BN; c += 16) {
+                        float a[16], k[16], bv[16];
+                        __syncwarp();
+                        tmem_ld16(taddr + c, a);
+                        load16_tile<ES>(tile, r, c, k);
+                        if (has_bias) {
+                            vec16(vb, c, bv);
                         } else {
-                            load16_f32_smem(kv_tile, r, ta, ka);
-                            load16_f32_smem(kv_tile, r, tb, kb);
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) bv[i] = 0.0f;
                         }
                         tmem_wait_ld();
+                        if constexpr (Cfg::kKV) {
+                            float sv[16];
+                            vec16(vs, c, sv);
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) {
-                            const int ga = n0 + ta + i, gb = n0 + tb + i;
-                            ka[i] = fmaf(__ldg(p.sigma + ga), a[i] + __ldg(p.bias + ga), ka[i]);
-                            kb[i] = fmaf(__ldg(p.sigma + gb), b[i] + __ldg(p.bias + gb), kb[i]);
-                        }
-                        if (rot) rotate16(ka, kb, pr, p.inv_freq, j);
-                        if constexpr (EPI == EPI_KV_BF16) {
-                            store16_bf16_smem(kv_tile, r, ta, ka);
-                            store16_bf16_smem(kv_tile, r, tb, kb);
+                            for (int i = 0; i < 16; ++i) k[i] = fmaf(sv[i], a[i] + bv[i], k[i]);
                         } else {
-                            store16_f32_smem(kv_tile, r, ta, ka);
-                            store16_f32_smem(kv_tile, r, tb, kb);
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) k[i] += a[i] + bv[i];
                         }
+                        store16_tile<ES>(tile, r, c, k);
                     }
                 }
             } else {
@@ -345,7 +411,12 @@ __global__ void __launch_bounds__(192, 1)
                     tmem_wait_ld();
                     const int col = n0 + c;
                     if (col >= p.N || !row_ok) continue;
-                    add_bias16(v, p.bias, col);
+                    if (has_bias) {
+                        float bv[16];
+                        vec16(vb, c, bv);
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) v[i] += bv[i];
+                    }
                     if constexpr (EPI == EPI_BF16 || EPI == EPI_GELU_BF16) {
                         if constexpr (EPI == EPI_GELU_BF16) {
 #pragma unroll
@@ -354,19 +425,11 @@ __global__ void __launch_bounds__(192, 1)
                         store16_bf16_global(
                             reinterpret_cast<uint16_t*>(p.out) + static_cast<int64_t>(row) * p.ldo + col, v);
                     } else {
-                        float* o = reinterpret_cast<float*>(p.out) + static_cast<int64_t>(row) * p.ldo + col;
+                        float4* o = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) +
+                                                              static_cast<int64_t>(row) * p.ldo + col);
 #pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            float4 x = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-                            if constexpr (EPI == EPI_ADD_F32) {
-                                const float4 y = reinterpret_cast<const float4*>(o)[q];
-                                x.x += y.x;
-                                x.y += y.y;
-                                x.z += y.z;
-                                x.w += y.w;
-                            }
-                            reinterpret_cast<float4*>(o)[q] = x;
-                        }
+                        for (int q = 0; q < 4; ++q)
+                            o[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
                     }
                 }
             }
@@ -374,32 +437,34 @@ __global__ void __launch_bounds__(192, 1)
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&tempty[acc]);
-            if constexpr (Cfg::kKV) {
-                // every epilogue thread's tile writes -> async proxy; then lane 0
-                // of warp 2, after a bounded wait for all 128 threads, stores the
-                // tile with TMA and hands the buffer back to the producer
+            if (epi_load) {
+                // this thread's reads of the vectors and writes of the staged tile
+                // are done; lane 0 of warp 2 waits (bounded) for all 128, stores
+                // the staged tile with TMA and hands the area back to the producer
                 fence_async_smem();
                 mbar_arrive(epi_done);
                 if (warp == 2) {
                     bool ok2 = true;
                     if (lane == 0) {
-                        ok2 = mbar_wait(epi_done, kv_phase, wc, 303);
+                        ok2 = mbar_wait(epi_done, epi_phase, wc, 303);
                         if (ok2) {
-                            for (int b = 0; b < Cfg::kKVBoxes; ++b)
-                                tma_store_2d(&tmC, kv_tile + b * 16384, n0 + b * Cfg::kKVBoxCols, m0);
-                            tma_store_commit();
-                            tma_store_wait_read0();
-                            mbar_arrive(kvempty);
+                            if constexpr (Cfg::kInPlace) {
+                                for (int b = 0; b < Cfg::kBoxes; ++b)
+                                    tma_store_2d(&tmC, tile + b * 16384, n0 + b * Cfg::kBoxCols, m0);
+                                tma_store_commit();
+                                tma_store_wait_read0();
+                            }
+                            mbar_arrive(epi_empty);
                         }
                     }
                     if (!__shfl_sync(0xffffffffu, ok2 ? 1 : 0, 0)) break;
                 }
-                kv_phase ^= 1u;
+                epi_phase ^= 1u;
             }
             acc ^= 1u;
             if (acc == 0) acc_phase ^= 1u;
         }
-        if constexpr (Cfg::kKV) {
+        if constexpr (Cfg::kInPlace) {
             if (warp == 2 && lane == 0) tma_store_wait0();
         }
     }
@@ -431,8 +496,9 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
                       int64_t K, int epi, GemmParams p, void* kv_base, int64_t ld_kv,
                       cudaStream_t st) {
     const bool kv = (epi == EPI_KV_BF16 || epi == EPI_KV_F32);
+    const bool f32_tile = (epi == EPI_KV_F32 || epi == EPI_ADD_F32);
     int BN;
-    if (epi == EPI_KV_F32)
+    if (f32_tile || epi == EPI_F32)
         BN = 128;
     else if (kv)
         BN = 256;
@@ -440,6 +506,7 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
         BN = (N >= 2048) ? 256 : 128;
     if (kv && (N % BN) != 0) return CR_ERR_UNSUPPORTED;
     if (epi == EPI_QKV_ROPE && (BN % p.rope_dim) != 0) return CR_ERR_UNSUPPORTED;
+    if (p.bias && (N % 4) != 0) return CR_ERR_UNSUPPORTED;   // bias slices are 16-byte bulk copies
     p.M = static_cast<int32_t>(M);
     p.N = static_cast<int32_t>(N);
     p.K = static_cast<int32_t>(K);
@@ -454,10 +521,13 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
         return CR_ERR_INVALID_ARG;
     tc = ta;
     if (kv) {
-        const bool f32 = (epi == EPI_KV_F32);
         if (!make_tmap_2d(&tc, kv_base,
-                          f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
-                          N, M, ld_kv * (f32 ? 4 : 2), f32 ? 32 : 64, BM,
+                          f32_tile ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                          N, M, ld_kv * (f32_tile ? 4 : 2), f32_tile ? 32 : 64, BM,
+                          CU_TENSOR_MAP_SWIZZLE_128B))
+            return CR_ERR_INVALID_ARG;
+    } else if (epi == EPI_ADD_F32) {
+        if (!make_tmap_2d(&tc, p.out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, N, M, p.ldo * 4, 32, BM,
                           CU_TENSOR_MAP_SWIZZLE_128B))
             return CR_ERR_INVALID_ARG;
     }
@@ -469,11 +539,9 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
             return BN == 256 ? launch_bn<256, EPI_GELU_BF16>(ta, tb, tc, p, st)
                              : launch_bn<128, EPI_GELU_BF16>(ta, tb, tc, p, st);
         case EPI_ADD_F32:
-            return BN == 256 ? launch_bn<256, EPI_ADD_F32>(ta, tb, tc, p, st)
-                             : launch_bn<128, EPI_ADD_F32>(ta, tb, tc, p, st);
+            return launch_bn<128, EPI_ADD_F32>(ta, tb, tc, p, st);
         case EPI_F32:
-            return BN == 256 ? launch_bn<256, EPI_F32>(ta, tb, tc, p, st)
-                             : launch_bn<128, EPI_F32>(ta, tb, tc, p, st);
+            return launch_bn<128, EPI_F32>(ta, tb, tc, p, st);
         case EPI_QKV_ROPE:
             return BN == 256 ? launch_bn<256, EPI_QKV_ROPE>(ta, tb, tc, p, st)
                              : launch_bn<128, EPI_QKV_ROPE>(ta, tb, tc, p, st);
