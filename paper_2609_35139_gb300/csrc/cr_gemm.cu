@@ -2,11 +2,12 @@
 //   C[M, N] = A[M, K] * W[N, K]^T + bias, with a fused epilogue.
 //
 // Design (sm_103a, one CTA per SM, persistent):
-//   warp 0      TMA producer: per output tile, first the epilogue's inputs —
-//               the bias (and sigma_delta) slice of the tile by bulk copy and,
-//               for in-place epilogues, the output tile itself (the stale cache
-//               tile, or the fp32 residual-stream tile) by TMA — then A and W
-//               k-slices (64 wide, 128B swizzle) into a shared-memory ring.
+//   warp 0      TMA producer: A and W k-slices (64 wide, 128B swizzle) into a
+//               shared-memory ring, tile after tile without pausing.
+//   warp 6      epilogue-input loader: per tile, the bias (and sigma_delta)
+//               slice by bulk copy and, for in-place epilogues, the output tile
+//               itself (the stale cache tile, or the fp32 residual-stream tile)
+//               by TMA, as soon as the epilogue has released its slot.
 //   warp 1      allocates TMEM; one elected lane issues tcgen05.mma
 //               (M = 128, N = BN, K = 16) into a double-buffered fp32
 //               accumulator (2 x BN TMEM columns) and commits to mbarriers.
@@ -39,10 +40,13 @@ struct GemmCfg {
     static constexpr uint32_t kTileBytes = kInPlace ? BM * BN * kTileEsize : 0;
     static constexpr int kBoxCols = 128 / kTileEsize;          // one 128-byte swizzle row
     static constexpr int kBoxes = kInPlace ? BN / kBoxCols : 0;
-    static constexpr uint32_t kVecBytes = BN * 4 * (kKV ? 2 : 1);   // bias (+ sigma)
+    static constexpr uint32_t kVecBytes = BN * 4 * (kKV ? 2 : 1);   // bias (+ sigma) per slot
+    // epilogue-input slots: the staged in-place tile is single-buffered, bias-only
+    // slots are double-buffered so the next tile's bias lands during this epilogue
+    static constexpr int kEpiSlots = kInPlace ? 1 : 2;
     static constexpr uint32_t kBBytes = BN * BK * 2;
     static constexpr uint32_t kStageBytes = A_BYTES + kBBytes;
-    static constexpr uint32_t kFixed = 1024 + kTileBytes + kVecBytes + 256;
+    static constexpr uint32_t kFixed = 1024 + kTileBytes + kEpiSlots * kVecBytes + 256;
     static constexpr int kStagesFit = static_cast<int>((kSmemLimit - kFixed) / kStageBytes);
     static constexpr int kStages = kStagesFit > 6 ? 6 : kStagesFit;
     static_assert(kStages >= 2, "GEMM tile does not fit in shared memory");
@@ -161,7 +165,7 @@ __device__ __forceinline__ void rotate16(float* a, float* b, float p, const floa
 }
 
 template <int BN, int EPI>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(224, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const __grid_constant__ CUtensorMap tmC, const __grid_constant__ GemmParams p) {
     using Cfg = GemmCfg<BN, EPI>;
@@ -173,14 +177,15 @@ __global__ void __launch_bounds__(192, 1)
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     uint8_t* tile = smem + STAGES * Cfg::kStageBytes;              // staged output tile
     float* vec = reinterpret_cast<float*>(tile + Cfg::kTileBytes);  // bias [BN] (+ sigma [BN])
-    uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(vec) + Cfg::kVecBytes);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(vec) +
+                                                 Cfg::kEpiSlots * Cfg::kVecBytes);
     uint64_t* full = bars;
     uint64_t* empty = bars + STAGES;
     uint64_t* tfull = bars + 2 * STAGES;
     uint64_t* tempty = tfull + 2;
-    uint64_t* epi_full = tempty + 2;
-    uint64_t* epi_empty = epi_full + 1;
-    uint64_t* drain = epi_empty + 1;
+    uint64_t* epi_full = tempty + 2;         // [kEpiSlots]
+    uint64_t* epi_empty = epi_full + 2;      // [kEpiSlots]
+    uint64_t* drain = epi_empty + 2;
     uint64_t* epi_done = drain + 1;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(epi_done + 1);
     int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
@@ -195,8 +200,10 @@ __global__ void __launch_bounds__(192, 1)
             mbar_init(&tfull[s], 1);
             mbar_init(&tempty[s], 4);
         }
-        mbar_init(epi_full, 1);
-        mbar_init(epi_empty, 1);
+        for (int s = 0; s < Cfg::kEpiSlots; ++s) {
+            mbar_init(&epi_full[s], 1);
+            mbar_init(&epi_empty[s], 1);
+        }
         mbar_init(drain, 1);
         mbar_init(epi_done, 128);
         *abort_flag = 0;
@@ -221,26 +228,11 @@ __global__ void __launch_bounds__(192, 1)
             tma_prefetch(&tmA);
             tma_prefetch(&tmB);
             if constexpr (Cfg::kInPlace) tma_prefetch(&tmC);
-            uint32_t stage = 0, phase = 0, epi_phase = 0;
+            uint32_t stage = 0, phase = 0;
             bool ok = true;
             for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
                 const int m0 = (t % p.num_m) * BM;
                 const int n0 = (t / p.num_m) * BN;
-                if (epi_load) {
-                    if (!(ok = mbar_wait(epi_empty, epi_phase ^ 1u, wc, 101))) break;
-                    const int nb = min(BN, p.N - n0);
-                    const uint32_t vbytes = static_cast<uint32_t>(nb) * 4u;
-                    uint32_t bytes = Cfg::kTileBytes + (has_bias ? vbytes : 0u);
-                    if constexpr (Cfg::kKV) bytes += vbytes;
-                    mbar_expect_tx(epi_full, bytes);
-                    if constexpr (Cfg::kInPlace) {
-                        for (int b = 0; b < Cfg::kBoxes; ++b)
-                            tma_load_2d(tile + b * 16384, &tmC, epi_full, n0 + b * Cfg::kBoxCols, m0);
-                    }
-                    if (has_bias) bulk_load(vec, p.bias + n0, vbytes, epi_full);
-                    if constexpr (Cfg::kKV) bulk_load(vec + BN, p.sigma + n0, vbytes, epi_full);
-                    epi_phase ^= 1u;
-                }
                 for (int kb = 0; kb < num_k; ++kb) {
                     if (!(ok = mbar_wait(&empty[stage], phase ^ 1u, wc, 102))) break;
                     uint8_t* sa = smem + stage * Cfg::kStageBytes;
@@ -254,6 +246,40 @@ __global__ void __launch_bounds__(192, 1)
                 }
             }
             if (!ok) {  // let copies already in flight land before the CTA exits
+                const uint64_t t0 = globaltimer();
+                while (globaltimer() - t0 < 50000ull) {
+                }
+            }
+        }
+    } else if (warp == 6) {
+        if (lane == 0 && epi_load) {
+            // ------------------------------------------------ epilogue-input loader:
+            // per tile, the bias (and sigma) slice by bulk copy and, for in-place
+            // epilogues, the output tile by TMA, as soon as the epilogue has
+            // released the slot (independent of the A/B stream of warp 0)
+            if constexpr (Cfg::kInPlace) tma_prefetch(&tmC);
+            bool ok = true;
+            int i = 0;
+            for (int t = blockIdx.x; t < total; t += gridDim.x, ++i) {
+                const int m0 = (t % p.num_m) * BM;
+                const int n0 = (t / p.num_m) * BN;
+                const int slot = i % Cfg::kEpiSlots;
+                const uint32_t ph = static_cast<uint32_t>(i / Cfg::kEpiSlots) & 1u;
+                if (!(ok = mbar_wait(&epi_empty[slot], ph ^ 1u, wc, 101))) break;
+                const int nb = min(BN, p.N - n0);
+                const uint32_t vbytes = static_cast<uint32_t>(nb) * 4u;
+                uint32_t bytes = Cfg::kTileBytes + (has_bias ? vbytes : 0u);
+                if constexpr (Cfg::kKV) bytes += vbytes;
+                float* v = vec + slot * (Cfg::kVecBytes / 4);
+                mbar_expect_tx(&epi_full[slot], bytes);
+                if constexpr (Cfg::kInPlace) {
+                    for (int b = 0; b < Cfg::kBoxes; ++b)
+                        tma_load_2d(tile + b * 16384, &tmC, &epi_full[slot], n0 + b * Cfg::kBoxCols, m0);
+                }
+                if (has_bias) bulk_load(v, p.bias + n0, vbytes, &epi_full[slot]);
+                if constexpr (Cfg::kKV) bulk_load(v + BN, p.sigma + n0, vbytes, &epi_full[slot]);
+            }
+            if (!ok) {
                 const uint64_t t0 = globaltimer();
                 while (globaltimer() - t0 < 50000ull) {
                 }
@@ -298,14 +324,18 @@ __global__ void __launch_bounds__(192, 1)
         // ---------------------------------------------------- epilogue (warps 2..5)
         const uint32_t quad = warp & 3u;
         const int r = static_cast<int>(quad * 32 + lane);     // row inside the tile
-        uint32_t acc = 0, acc_phase = 0, epi_phase = 0;
-        const float* vb = vec;             // bias slice of the tile
-        const float* vs = vec + BN;        // sigma_delta slice (KV epilogues)
-        for (int t = blockIdx.x; t < total; t += gridDim.x) {
+        uint32_t acc = 0, acc_phase = 0, done_phase = 0;
+        int i = 0;
+        for (int t = blockIdx.x; t < total; t += gridDim.x, ++i) {
             const int m0 = (t % p.num_m) * BM;
             const int n0 = (t / p.num_m) * BN;
+            const int slot = i % Cfg::kEpiSlots;
+            const float* vb = vec + slot * (Cfg::kVecBytes / 4);   // bias slice of the tile
+            const float* vs = vb + BN;                               // sigma_delta slice (KV)
             bool ok = mbar_wait(&tfull[acc], acc_phase, wc, 301);
-            if (epi_load) ok = ok && mbar_wait(epi_full, epi_phase, wc, 302);
+            if (epi_load)
+                ok = ok && mbar_wait(&epi_full[slot],
+                                     static_cast<uint32_t>(i / Cfg::kEpiSlots) & 1u, wc, 302);
             if (!__all_sync(0xffffffffu, ok)) break;
             tc_fence_after();
             const int row = m0 + r;
@@ -446,7 +476,7 @@ __global__ void __launch_bounds__(192, 1)
                 if (warp == 2) {
                     bool ok2 = true;
                     if (lane == 0) {
-                        ok2 = mbar_wait(epi_done, epi_phase, wc, 303);
+                        ok2 = mbar_wait(epi_done, done_phase, wc, 303);
                         if (ok2) {
                             if constexpr (Cfg::kInPlace) {
                                 for (int b = 0; b < Cfg::kBoxes; ++b)
@@ -454,12 +484,12 @@ __global__ void __launch_bounds__(192, 1)
                                 tma_store_commit();
                                 tma_store_wait_read0();
                             }
-                            mbar_arrive(epi_empty);
+                            mbar_arrive(&epi_empty[slot]);
                         }
                     }
                     if (!__shfl_sync(0xffffffffu, ok2 ? 1 : 0, 0)) break;
                 }
-                epi_phase ^= 1u;
+                done_phase ^= 1u;
             }
             acc ^= 1u;
             if (acc == 0) acc_phase ^= 1u;
@@ -486,7 +516,7 @@ cr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensor
     if (sa != CR_OK) return sa;
     const int tiles = p.num_m * p.num_n;
     const int grid = tiles < num_sms() ? tiles : num_sms();
-    kern<<<grid, 192, Cfg::kSmemBytes, st>>>(ta, tb, tc, p);
+    kern<<<grid, 224, Cfg::kSmemBytes, st>>>(ta, tb, tc, p);
     return cuda_check(cudaGetLastError());
 }
 
