@@ -220,6 +220,10 @@ cr_status cr_clear_device_status(void);
 
 const char* cr_status_str(cr_status s);
 
+/* Text of the last CUDA error a call of this thread returned CR_ERR_CUDA for
+ * ("no error" if none). */
+const char* cr_last_cuda_error(void);
+
 #ifdef __cplusplus
 }
 #endif

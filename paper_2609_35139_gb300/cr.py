@@ -25,6 +25,7 @@ CR_EPI_BF16, CR_EPI_GELU_BF16, CR_EPI_ADD_F32, CR_EPI_F32 = range(4)
 EXPORTED = [
     "cr_workspace_bytes", "cr_assemble_stale", "cr_compress_features", "cr_repair_forward",
     "cr_apply_residual", "cr_get_device_status", "cr_clear_device_status", "cr_status_str",
+    "cr_last_cuda_error",
     "cr_linear", "cr_layernorm", "cr_chunk_causal_attention", "cr_qkv_rope", "cr_segment_project",
     "cr_segment_project_noalloc",
 ]
@@ -92,6 +93,7 @@ def lib(build_if_missing: bool = False) -> ctypes.CDLL:
         "cr_get_device_status": (i32, [P(c_uint32)]),
         "cr_clear_device_status": (i32, []),
         "cr_status_str": (ctypes.c_char_p, [i32]),
+        "cr_last_cuda_error": (ctypes.c_char_p, []),
         "cr_linear": (i32, [vp, i64, vp, vp, i64, i64, i64, vp, i64, i32, vp]),
         "cr_layernorm": (i32, [vp, vp, i64, vp, vp, vp, c_float, i64, i64, vp, vp]),
         "cr_chunk_causal_attention": (i32, [vp, i32, i32, vp, vp, i32, i64, vp, vp]),
@@ -110,7 +112,10 @@ def lib(build_if_missing: bool = False) -> ctypes.CDLL:
 
 def _check(name: str, status: int):
     if status != CR_OK:
-        raise CrError(name, status, lib().cr_status_str(status).decode())
+        text = lib().cr_status_str(status).decode()
+        if status == CR_ERR_CUDA:
+            text += ": " + lib().cr_last_cuda_error().decode()
+        raise CrError(name, status, text)
 
 
 def _p(t) -> Optional[int]:

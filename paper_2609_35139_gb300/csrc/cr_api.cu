@@ -125,7 +125,15 @@ bool all_aligned(const P* p, R... rest) {
 
 }  // namespace
 
-cr_status cuda_check(cudaError_t e) { return e == cudaSuccess ? CR_OK : CR_ERR_CUDA; }
+namespace {
+thread_local cudaError_t t_last_cuda_error = cudaSuccess;
+}
+
+cr_status cuda_check(cudaError_t e) {
+    if (e == cudaSuccess) return CR_OK;
+    t_last_cuda_error = e;
+    return CR_ERR_CUDA;
+}
 
 int current_device_index() { return current_device(); }
 
@@ -184,6 +192,10 @@ bool make_tmap_2d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, uint
 using namespace cr;
 
 extern "C" {
+
+const char* cr_last_cuda_error(void) {
+    return t_last_cuda_error == cudaSuccess ? "no error" : cudaGetErrorString(t_last_cuda_error);
+}
 
 const char* cr_status_str(cr_status s) {
     switch (s) {

@@ -11,18 +11,21 @@
 //   warp 0      TMA: both Q tiles once, then K_j and V_j per key tile into a
 //               3-deep ring shared by the two query tiles
 //   warp 1      TMEM owner; one lane issues, per key tile j and query tile w,
-//               S_w,j = Q_w K_j^T (M=128, N=128, K=d) into S_w, and after
-//               softmax w has written P_w,j, PV_w,j = P_w,j V_j (M=128, N=d,
-//               K=128, V read MN-major) into one of two PV buffers of w
+//               S_w,j = Q_w K_j^T (M=128, N=128, K=d) into S_w, and, once
+//               softmax w has written P_w,j, O_w += P_w,j V_j (M=128, N=d,
+//               K=128, V read MN-major) accumulating in TMEM
 //   warps 2..5  softmax group 0 (query tile 0), one row per thread
 //   warps 6..9  softmax group 1 (query tile 1)
-// The two groups ping-pong: while group 0 turns S_0,j into P_0,j the tensor
-// core computes S_1,j, PV_0,j-1 and S_0,j+1, and the other way round.  A group
-// reads S_w,j from TMEM (two passes of 32-column loads: row max, then exp2,
-// row sum and bf16 P written to shared memory in the 128B-swizzled K-major
-// layout the MMA reads), then folds the previous tile's PV into its
-// register-resident O: O = O * alpha_{j-1} + PV_{j-1} (between the max pass
-// and the exp pass: PV_{j-1} is issued before S_j, so it is done by then).
+// The two groups ping-pong on the tensor core.  Per key tile a group reads its
+// S row from TMEM twice, 64 columns at a time (the (masked) row max, then the
+// exponentials; 320 threads leave 168 registers each), and writes
+// P = 2^(s*scale*log2e - m) as bf16 into shared memory in the 128B-swizzled
+// K-major layout the MMA reads.  The reference m is the row's running max,
+// updated lazily: only when a tile raises it by more than 2^8 does the group
+// rescale its O row in TMEM (and the row sum l).  Any reference m gives the same
+// softmax (it cancels in O / l), and keeping it at most 8 below the true
+// running max keeps P <= 2^8, so this is exact up to rounding.
+// O_w is read back and divided by l after the last tile.
 #include <cuda_bf16.h>
 
 #include "cr_internal.h"
@@ -45,10 +48,11 @@ struct AttnCfg {
     static constexpr uint32_t kBarOff = kPOff + 2 * kPBytes;
     static constexpr uint32_t kSmemBytes = 1024 + kBarOff + 256;
     static constexpr uint32_t kTmemS = 0;      // S_w at w * 128
-    static constexpr uint32_t kTmemPV = 256;   // PV_w,b at 256 + (2w + b) * D
+    static constexpr uint32_t kTmemO = 256;    // O_w at 256 + w * D
 };
 
 constexpr int kThreads = 320;
+constexpr float kRescaleLog2 = 8.0f;   // lazy-rescale threshold (log2 units)
 
 // Byte offset of 16 consecutive keys (c multiple of 16) of row r inside a
 // [128 x 128] bf16 P tile held as two 64-column, 128B-swizzled K-major atoms.
@@ -83,11 +87,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* v_full = k_full + NS;
     uint64_t* kv_empty = v_full + NS;
     uint64_t* s_full = kv_empty + NS;     // [2]
-    uint64_t* s_free = s_full + 2;        // [2]
-    uint64_t* p_full = s_free + 2;        // [2]
-    uint64_t* pv_full = p_full + 2;       // [2][2]
-    uint64_t* pv_free = pv_full + 4;      // [2][2]
-    uint64_t* drain = pv_free + 4;
+    uint64_t* p_full = s_full + 2;        // [2]
+    uint64_t* o_done = p_full + 2;        // [2]
+    uint64_t* drain = o_done + 2;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
     int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
@@ -117,12 +119,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int w = 0; w < 2; ++w) {
             mbar_init(&s_full[w], 1);
-            mbar_init(&s_free[w], 128);
             mbar_init(&p_full[w], 128);
-            for (int b = 0; b < 2; ++b) {
-                mbar_init(&pv_full[2 * w + b], 1);
-                mbar_init(&pv_free[2 * w + b], 128);
-            }
+            mbar_init(&o_done[w], 1);
         }
         mbar_init(drain, 1);
         *abort_flag = 0;
@@ -164,12 +162,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp == 1) {
         if (lane == 0) {
             // ---------------------------------------------------- MMA issuer
+            // Per query tile w the order is S_0, [P_0] PV_0, S_1, [P_1] PV_1, ...
+            // so the commit after S_j+1 also covers PV_j: when the softmax group
+            // sees S_j+1 its O row is current and its P buffer is free.
             const uint32_t sq0 = smem_u32(smem + Cfg::kQOff);
             auto issue_s = [&](int w, int j) -> bool {
                 const int st = j % NS;
                 if (!mbar_wait(&k_full[st], static_cast<uint32_t>(j / NS) & 1u, wc, 222)) return false;
-                if (j > 0 && !mbar_wait(&s_free[w], static_cast<uint32_t>(j - 1) & 1u, wc, 223))
-                    return false;
                 tc_fence_after();
                 const uint32_t sq = sq0 + w * Cfg::kTileBytes;
                 const uint32_t sk = smem_u32(smem + Cfg::kKVOff + st * 2 * Cfg::kTileBytes);
@@ -184,17 +183,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             };
             auto issue_pv = [&](int w, int j) -> bool {
                 const int st = j % NS;
-                const int b = j & 1;
                 if (!mbar_wait(&p_full[w], static_cast<uint32_t>(j) & 1u, wc, 224)) return false;
                 if (!mbar_wait(&v_full[st], static_cast<uint32_t>(j / NS) & 1u, wc, 225)) return false;
-                if (j >= 2 &&
-                    !mbar_wait(&pv_free[2 * w + b], static_cast<uint32_t>((j - 2) >> 1) & 1u, wc, 226))
-                    return false;
                 tc_fence_after();
                 const uint32_t sp = smem_u32(smem + Cfg::kPOff + w * Cfg::kPBytes);
                 const uint32_t sv =
                     smem_u32(smem + Cfg::kKVOff + st * 2 * Cfg::kTileBytes + Cfg::kTileBytes);
-                const uint32_t d = tmem_base + Cfg::kTmemPV + (2 * w + b) * D;
+                const uint32_t d = tmem_base + Cfg::kTmemO + w * D;
 #pragma unroll
                 for (int kk = 0; kk < 8; ++kk) {
                     const uint64_t da =
@@ -203,9 +198,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // 16 keys = two 8-row swizzle atoms.
                     const uint64_t db = smem_desc(sv + kk * 16 * Cfg::kRowBytes, Cfg::kTileBytes,
                                                   Cfg::kAtomBytes, Cfg::kSwz);
-                    mma_bf16_ss(d, da, db, IDESC_PV, kk != 0 ? 1u : 0u);
+                    mma_bf16_ss(d, da, db, IDESC_PV, (j > 0 || kk != 0) ? 1u : 0u);
                 }
-                mma_commit(&pv_full[2 * w + b]);
                 return true;
             };
             bool ok = mbar_wait(q_full, 0, wc, 221);
@@ -216,7 +210,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int w = 0; w < 2 && ok; ++w) {
                     if (j >= n_kv[w]) continue;
                     if (!(ok = issue_pv(w, j))) break;
-                    if (j + 1 < n_kv[w]) ok = issue_s(w, j + 1);
+                    if (j + 1 < n_kv[w])
+                        ok = issue_s(w, j + 1);
+                    else
+                        mma_commit(&o_done[w]);
                 }
                 if (ok) mma_commit(&kv_empty[j % NS]);
             }
@@ -233,33 +230,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int cend = valid ? __ldg(p.chunk_end + rs + qrow) : 1;
         const uint32_t lane_off = (quad * 32u) << 16;
         const uint32_t ts = tmem_base + lane_off + Cfg::kTmemS + w * 128;
+        const uint32_t to = tmem_base + lane_off + Cfg::kTmemO + w * D;
         const float sc = p.scale_log2;
         const int n = n_kv[w];
         uint8_t* pt = smem + Cfg::kPOff + w * Cfg::kPBytes;
-        float m = NEG_INF, l = 0.0f, alpha_prev = 0.0f;
-        float o[D];
-#pragma unroll
-        for (int i = 0; i < D; ++i) o[i] = 0.0f;
-
-        auto fold = [&](int jj) -> bool {   // O = O * alpha_prev + PV_jj
-            const int b = jj & 1;
-            bool okf = mbar_wait(&pv_full[2 * w + b], static_cast<uint32_t>(jj >> 1) & 1u, wc, 322);
-            if (!__all_sync(0xffffffffu, okf)) return false;
-            tc_fence_after();
-            const uint32_t tp = tmem_base + lane_off + Cfg::kTmemPV + (2 * w + b) * D;
-#pragma unroll
-            for (int c = 0; c < D; c += 32) {
-                float v[32];
-                __syncwarp();
-                tmem_ld32(tp + c, v);
-                tmem_wait_ld();
-#pragma unroll
-                for (int i = 0; i < 32; ++i) o[c + i] = fmaf(o[c + i], alpha_prev, v[i]);
-            }
-            tc_fence_before();
-            mbar_arrive(&pv_free[2 * w + b]);
-            return true;
-        };
+        float m = NEG_INF, l = 0.0f;
 
         bool ok = true;
         for (int j = 0; j < n; ++j) {
@@ -271,83 +246,106 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             const int k0 = j * 128;
             const bool full_tile = k0 + 128 <= cend;     // all 128 keys visible to this row
-            // pass 1: row max of the (masked) scores
+            // pass 1: row max of the (masked) scores, 64 columns at a time
             float mx = NEG_INF;
 #pragma unroll
-            for (int c = 0; c < 128; c += 32) {
-                float v[32];
+            for (int h = 0; h < 128; h += 64) {
+                float s[64];
                 __syncwarp();
-                tmem_ld32(ts + c, v);
+                tmem_ld32(ts + h, s);
+                tmem_ld32(ts + h + 32, s + 32);
                 tmem_wait_ld();
                 if (full_tile) {
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) mx = fmaxf(mx, v[i]);
+                    for (int i = 0; i < 64; ++i) mx = fmaxf(mx, s[i]);
                 } else {
 #pragma unroll
-                    for (int i = 0; i < 32; ++i)
-                        if (k0 + c + i < cend) mx = fmaxf(mx, v[i]);
+                    for (int i = 0; i < 64; ++i)
+                        if (k0 + h + i < cend) mx = fmaxf(mx, s[i]);
                 }
             }
-            const float m_new = fmaxf(m, mx * sc);
-            const float alpha = ex2(m - m_new);
-            // PV_{j-1} was issued before S_j, so it is complete by now: fold it,
-            // which also frees the P buffer for P_j
-            if (j > 0 && !fold(j - 1)) {
-                ok = false;
-                break;
+            mx *= sc;
+            // lazily move the reference max: on the first tile, or when this
+            // tile would push P above 2^8 somewhere in the warp
+            const bool raise = (j == 0) || (mx > m + kRescaleLog2);
+            if (__any_sync(0xffffffffu, raise)) {
+                const float m_new = fmaxf(m, mx);
+                if (j > 0) {
+                    // O holds sum_{k<j} P_k V_k (complete: S_j was issued after PV_{j-1})
+                    const float alpha = ex2(m - m_new);
+#pragma unroll
+                    for (int c = 0; c < D; c += 16) {
+                        float o[16];
+                        tmem_ld16(to + c, o);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) o[i] *= alpha;
+                        tmem_st16(to + c, o);
+                    }
+                    tmem_wait_st();
+                    l *= alpha;
+                }
+                m = m_new;
             }
-            alpha_prev = alpha;
-            // pass 2: probabilities -> P (bf16, swizzled K-major), row sum
+            // pass 2: P = 2^(s*sc - m) -> bf16, swizzled K-major, and the row sum
             float rsum = 0.0f;
 #pragma unroll
-            for (int c = 0; c < 128; c += 32) {
-                float v[32];
+            for (int h = 0; h < 128; h += 64) {
+                float s[64];
                 __syncwarp();
-                tmem_ld32(ts + c, v);
+                tmem_ld32(ts + h, s);
+                tmem_ld32(ts + h + 32, s + 32);
                 tmem_wait_ld();
-                uint32_t pk[16];
 #pragma unroll
-                for (int i = 0; i < 32; i += 2) {
-                    float e0 = ex2(fmaf(v[i], sc, -m_new));
-                    float e1 = ex2(fmaf(v[i + 1], sc, -m_new));
-                    if (!full_tile) {
-                        if (k0 + c + i >= cend) e0 = 0.0f;
-                        if (k0 + c + i + 1 >= cend) e1 = 0.0f;
+                for (int c = 0; c < 64; c += 16) {
+                    uint32_t pk[8];
+#pragma unroll
+                    for (int i = 0; i < 16; i += 2) {
+                        float e0 = ex2(fmaf(s[c + i], sc, -m));
+                        float e1 = ex2(fmaf(s[c + i + 1], sc, -m));
+                        if (!full_tile) {
+                            if (k0 + h + c + i >= cend) e0 = 0.0f;
+                            if (k0 + h + c + i + 1 >= cend) e1 = 0.0f;
+                        }
+                        rsum += e0 + e1;
+                        pk[i >> 1] = pack_bf16x2(e0, e1);
                     }
-                    rsum += e0 + e1;
-                    pk[i >> 1] = pack_bf16x2(e0, e1);
-                }
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
                     uint32_t o0, o1;
-                    p_offsets(r, c + 16 * h, &o0, &o1);
-                    *reinterpret_cast<uint4*>(pt + o0) =
-                        make_uint4(pk[8 * h], pk[8 * h + 1], pk[8 * h + 2], pk[8 * h + 3]);
-                    *reinterpret_cast<uint4*>(pt + o1) =
-                        make_uint4(pk[8 * h + 4], pk[8 * h + 5], pk[8 * h + 6], pk[8 * h + 7]);
+                    p_offsets(r, h + c, &o0, &o1);
+                    *reinterpret_cast<uint4*>(pt + o0) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                    *reinterpret_cast<uint4*>(pt + o1) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
                 }
             }
-            l = l * alpha + rsum;
-            m = m_new;
+            l += rsum;
             tc_fence_before();
-            mbar_arrive(&s_free[w]);          // S_w may now be overwritten by S_w,j+1
             fence_async_smem();
             mbar_arrive(&p_full[w]);
         }
-        if (ok && n > 0) ok = fold(n - 1);
-        tc_fence_before();
-        if (ok && valid && n > 0) {
+        if (ok && n > 0) {
+            ok = mbar_wait(&o_done[w], 0, wc, 322);
+            ok = __all_sync(0xffffffffu, ok);
+        }
+        if (ok && n > 0) {
+            tc_fence_after();
             const float inv = 1.0f / l;
             uint16_t* dst = p.out + static_cast<int64_t>(rs + qrow) * p.d_b + head * D;
 #pragma unroll
-            for (int c = 0; c < D; c += 8) {
-                *reinterpret_cast<uint4*>(dst + c) =
-                    make_uint4(pack_bf16x2(o[c] * inv, o[c + 1] * inv),
-                               pack_bf16x2(o[c + 2] * inv, o[c + 3] * inv),
-                               pack_bf16x2(o[c + 4] * inv, o[c + 5] * inv),
-                               pack_bf16x2(o[c + 6] * inv, o[c + 7] * inv));
+            for (int c = 0; c < D; c += 16) {
+                float o[16];
+                tmem_ld16(to + c, o);
+                tmem_wait_ld();
+                if (valid) {
+                    uint4* d4 = reinterpret_cast<uint4*>(dst + c);
+                    d4[0] = make_uint4(pack_bf16x2(o[0] * inv, o[1] * inv), pack_bf16x2(o[2] * inv, o[3] * inv),
+                                       pack_bf16x2(o[4] * inv, o[5] * inv), pack_bf16x2(o[6] * inv, o[7] * inv));
+                    d4[1] = make_uint4(pack_bf16x2(o[8] * inv, o[9] * inv),
+                                       pack_bf16x2(o[10] * inv, o[11] * inv),
+                                       pack_bf16x2(o[12] * inv, o[13] * inv),
+                                       pack_bf16x2(o[14] * inv, o[15] * inv));
+                }
             }
         }
+        tc_fence_before();
     }
     __syncthreads();
     if (warp == 1) {
