@@ -246,8 +246,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             const int k0 = j * 128;
             const bool full_tile = k0 + 128 <= cend;     // all 128 keys visible to this row
-            // pass 1: row max of the (masked) scores, 64 columns at a time
-            float mx = NEG_INF;
+            // pass 1: row max of the (masked) scores, 64 columns at a time, in
+            // eight independent chains
+            float mxv[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) mxv[q] = NEG_INF;
 #pragma unroll
             for (int h = 0; h < 128; h += 64) {
                 float s[64];
@@ -257,13 +260,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tmem_wait_ld();
                 if (full_tile) {
 #pragma unroll
-                    for (int i = 0; i < 64; ++i) mx = fmaxf(mx, s[i]);
+                    for (int i = 0; i < 64; ++i) mxv[i & 7] = fmaxf(mxv[i & 7], s[i]);
                 } else {
 #pragma unroll
                     for (int i = 0; i < 64; ++i)
-                        if (k0 + h + i < cend) mx = fmaxf(mx, s[i]);
+                        if (k0 + h + i < cend) mxv[i & 7] = fmaxf(mxv[i & 7], s[i]);
                 }
             }
+            float mx = fmaxf(fmaxf(fmaxf(mxv[0], mxv[1]), fmaxf(mxv[2], mxv[3])),
+                             fmaxf(fmaxf(mxv[4], mxv[5]), fmaxf(mxv[6], mxv[7])));
             mx *= sc;
             // lazily move the reference max: on the first tile, or when this
             // tile would push P above 2^8 somewhere in the warp
@@ -287,8 +292,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 m = m_new;
             }
-            // pass 2: P = 2^(s*sc - m) -> bf16, swizzled K-major, and the row sum
-            float rsum = 0.0f;
+            // pass 2: P = 2^(s*sc - m) -> bf16, swizzled K-major, and the row sum.
+            // Fully visible tiles (all tiles of chunk-aligned maps) take a loop
+            // with no per-element masking.
+            float rs8[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) rs8[q] = 0.0f;
+            const int lim = full_tile ? 128 : cend - k0;   // keys < lim are visible
 #pragma unroll
             for (int h = 0; h < 128; h += 64) {
                 float s[64];
@@ -296,18 +306,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tmem_ld32(ts + h, s);
                 tmem_ld32(ts + h + 32, s + 32);
                 tmem_wait_ld();
+                if (!full_tile) {
+#pragma unroll
+                    for (int i = 0; i < 64; ++i) s[i] = (h + i < lim) ? s[i] : NEG_INF;
+                }
 #pragma unroll
                 for (int c = 0; c < 64; c += 16) {
                     uint32_t pk[8];
 #pragma unroll
                     for (int i = 0; i < 16; i += 2) {
-                        float e0 = ex2(fmaf(s[c + i], sc, -m));
-                        float e1 = ex2(fmaf(s[c + i + 1], sc, -m));
-                        if (!full_tile) {
-                            if (k0 + h + c + i >= cend) e0 = 0.0f;
-                            if (k0 + h + c + i + 1 >= cend) e1 = 0.0f;
-                        }
-                        rsum += e0 + e1;
+                        const float e0 = ex2(fmaf(s[c + i], sc, -m));
+                        const float e1 = ex2(fmaf(s[c + i + 1], sc, -m));
+                        rs8[(i >> 1) & 7] += e0 + e1;
                         pk[i >> 1] = pack_bf16x2(e0, e1);
                     }
                     uint32_t o0, o1;
@@ -316,7 +326,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     *reinterpret_cast<uint4*>(pt + o1) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
                 }
             }
-            l += rsum;
+            l += ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
             tc_fence_before();
             fence_async_smem();
             mbar_arrive(&p_full[w]);
