@@ -9,7 +9,7 @@
 //
 // CTA = (request, head, two consecutive 128-query tiles).  10 warps:
 //   warp 0      TMA: both Q tiles once, then K_j and V_j per key tile into a
-//               3-deep ring shared by the two query tiles
+//               5-deep ring shared by the two query tiles
 //   warp 1      TMEM owner; one lane issues, per key tile j and query tile w,
 //               S_w,j = Q_w K_j^T (M=128, N=128, K=d) into S_w, and, once
 //               softmax w has written P_w,j, O_w += P_w,j V_j (M=128, N=d,
@@ -19,8 +19,9 @@
 // The two groups ping-pong on the tensor core.  Per key tile a group reads its
 // S row from TMEM twice, 64 columns at a time (the (masked) row max, then the
 // exponentials; 320 threads leave 168 registers each), and writes
-// P = 2^(s*scale*log2e - m) as bf16 into shared memory in the 128B-swizzled
-// K-major layout the MMA reads.  The reference m is the row's running max,
+// P = 2^(s*scale*log2e - m) as bf16 pairs into its own TMEM columns, from
+// where the PV MMA reads it as the A operand (TMEM holds S_0, S_1, O_0, O_1,
+// P_0, P_1: 512 columns).  The reference m is the row's running max,
 // updated lazily: only when a tile raises it by more than 2^8 does the group
 // rescale its O row in TMEM (and the row sum l).  Any reference m gives the same
 // softmax (it cancels in O / l), and keeping it at most 8 below the true
@@ -40,28 +41,18 @@ struct AttnCfg {
     static constexpr uint32_t kAtomBytes = 8 * kRowBytes;    // swizzle atom (8 rows)
     static constexpr uint32_t kTileBytes = 128 * kRowBytes;
     static constexpr uint32_t kSwz = (D == 64) ? SWZ_128B : SWZ_64B;
-    static constexpr int kStages = 3;
-    static constexpr uint32_t kPBytes = 128 * 128 * 2;
+    static constexpr int kStages = 5;
     static constexpr uint32_t kQOff = 0;                                  // Q0, Q1
     static constexpr uint32_t kKVOff = 2 * kTileBytes;                    // K, V per stage
-    static constexpr uint32_t kPOff = kKVOff + kStages * 2 * kTileBytes;  // P0, P1
-    static constexpr uint32_t kBarOff = kPOff + 2 * kPBytes;
+    static constexpr uint32_t kBarOff = kKVOff + kStages * 2 * kTileBytes;
     static constexpr uint32_t kSmemBytes = 1024 + kBarOff + 256;
-    static constexpr uint32_t kTmemS = 0;      // S_w at w * 128
-    static constexpr uint32_t kTmemO = 256;    // O_w at 256 + w * D
+    static constexpr uint32_t kTmemS = 0;      // S_w at w * 128 (fp32)
+    static constexpr uint32_t kTmemO = 256;    // O_w at 256 + w * D (fp32)
+    static constexpr uint32_t kTmemP = 384;    // P_w at 384 + w * 64 (bf16 pairs)
 };
 
 constexpr int kThreads = 320;
 constexpr float kRescaleLog2 = 8.0f;   // lazy-rescale threshold (log2 units)
-
-// Byte offset of 16 consecutive keys (c multiple of 16) of row r inside a
-// [128 x 128] bf16 P tile held as two 64-column, 128B-swizzled K-major atoms.
-__device__ __forceinline__ void p_offsets(int r, int c, uint32_t* o0, uint32_t* o1) {
-    const uint32_t base = (c >> 6) * 16384 + r * 128;
-    const int ch = (c & 63) >> 3;
-    *o0 = base + ((ch ^ (r & 7)) << 4);
-    *o1 = base + (((ch + 1) ^ (r & 7)) << 4);
-}
 
 __device__ __forceinline__ float ex2(float x) {
     float y;
@@ -186,19 +177,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!mbar_wait(&p_full[w], static_cast<uint32_t>(j) & 1u, wc, 224)) return false;
                 if (!mbar_wait(&v_full[st], static_cast<uint32_t>(j / NS) & 1u, wc, 225)) return false;
                 tc_fence_after();
-                const uint32_t sp = smem_u32(smem + Cfg::kPOff + w * Cfg::kPBytes);
                 const uint32_t sv =
                     smem_u32(smem + Cfg::kKVOff + st * 2 * Cfg::kTileBytes + Cfg::kTileBytes);
                 const uint32_t d = tmem_base + Cfg::kTmemO + w * D;
+                const uint32_t pa = tmem_base + Cfg::kTmemP + w * 64;
 #pragma unroll
                 for (int kk = 0; kk < 8; ++kk) {
-                    const uint64_t da =
-                        smem_desc(sp + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024, SWZ_128B);
-                    // V: rows = keys (the K dimension), d contiguous (MN-major);
-                    // 16 keys = two 8-row swizzle atoms.
+                    // P from TMEM (16 keys = 8 columns); V: rows = keys (the K
+                    // dimension), d contiguous (MN-major); 16 keys = two 8-row atoms.
                     const uint64_t db = smem_desc(sv + kk * 16 * Cfg::kRowBytes, Cfg::kTileBytes,
                                                   Cfg::kAtomBytes, Cfg::kSwz);
-                    mma_bf16_ss(d, da, db, IDESC_PV, (j > 0 || kk != 0) ? 1u : 0u);
+                    mma_bf16_ts(d, pa + kk * 8, db, IDESC_PV, (j > 0 || kk != 0) ? 1u : 0u);
                 }
                 return true;
             };
@@ -233,7 +222,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t to = tmem_base + lane_off + Cfg::kTmemO + w * D;
         const float sc = p.scale_log2;
         const int n = n_kv[w];
-        uint8_t* pt = smem + Cfg::kPOff + w * Cfg::kPBytes;
+        const uint32_t tp = tmem_base + lane_off + Cfg::kTmemP + w * 64;
         float m = NEG_INF, l = 0.0f;
 
         bool ok = true;
@@ -310,25 +299,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int i = 0; i < 64; ++i) s[i] = (h + i < lim) ? s[i] : NEG_INF;
                 }
+                uint32_t pk[32];
 #pragma unroll
-                for (int c = 0; c < 64; c += 16) {
-                    uint32_t pk[8];
-#pragma unroll
-                    for (int i = 0; i < 16; i += 2) {
-                        const float e0 = ex2(fmaf(s[c + i], sc, -m));
-                        const float e1 = ex2(fmaf(s[c + i + 1], sc, -m));
-                        rs8[(i >> 1) & 7] += e0 + e1;
-                        pk[i >> 1] = pack_bf16x2(e0, e1);
-                    }
-                    uint32_t o0, o1;
-                    p_offsets(r, h + c, &o0, &o1);
-                    *reinterpret_cast<uint4*>(pt + o0) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-                    *reinterpret_cast<uint4*>(pt + o1) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+                for (int i = 0; i < 64; i += 2) {
+                    const float e0 = ex2(fmaf(s[i], sc, -m));
+                    const float e1 = ex2(fmaf(s[i + 1], sc, -m));
+                    rs8[(i >> 1) & 7] += e0 + e1;
+                    pk[i >> 1] = pack_bf16x2(e0, e1);
                 }
+                tmem_st32u(tp + h / 2, pk);
             }
             l += ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
+            tmem_wait_st();
             tc_fence_before();
-            fence_async_smem();
             mbar_arrive(&p_full[w]);
         }
         if (ok && n > 0) {
