@@ -81,7 +81,7 @@ cr_status check_repairer(const cr_repairer_dims* r) {
 }
 
 struct WsLayout {
-    size_t wfold, kvb, embb, y, se, x, u, qkv, o, g, total;
+    size_t wfold, kvb, embb, y, se, x, u, qkv, o, g, rope, total;
 };
 
 WsLayout ws_layout(const Dims& d, int64_t n) {
@@ -103,6 +103,7 @@ WsLayout ws_layout(const Dims& d, int64_t n) {
     w.qkv = take(N * 3 * d.db * 2);
     w.o = take(N * d.db * 2);
     w.g = take(N * d.hid * 2);
+    w.rope = take(N * (d.hd / 2) * 8);   // repairer RoPE (cos, sin) per token and pair
     w.total = off;
     return w;
 }
@@ -474,6 +475,16 @@ cr_status cr_repair_forward(const cr_target_dims* target, const cr_repairer_dims
     gq.rope_dim = static_cast<int32_t>(d.hd);
     gq.rope_cols = static_cast<int32_t>(2 * d.db);
     repairer_inv_freq(gq.inv_freq, static_cast<int>(d.hd), rep->rope_theta);
+    // positions are the same for every block: one (cos, sin) table per forward
+    float2* rope = at<float2>(workspace, L.rope);
+    if (d.B > 0) {
+        s = launch_rope_table(pos, N, static_cast<int>(d.hd / 2), gq.inv_freq, rope, st);
+        if (s != CR_OK) {
+            delete ap;
+            return s;
+        }
+        gq.rope_table = rope;
+    }
     GemmParams gr{};
     gr.status = status;
     for (int b = 0; b < d.B && s == CR_OK; ++b) {

@@ -11,11 +11,13 @@
 //   warp 1      allocates TMEM; one elected lane issues tcgen05.mma
 //               (M = 128, N = BN, K = 16) into a double-buffered fp32
 //               accumulator (2 x BN TMEM columns) and commits to mbarriers.
+//   warp 7      TMA store issuer for the staged output.
 //   warps 2..5  epilogue: tcgen05.ld 32 lanes x 16 columns, bias from shared
-//               memory, then one of: bf16 store, GELU, fp32 store, RoPE on Q/K,
-//               or in place on the staged tile: residual stream x += acc + b,
-//               cache kv = kv + sigma_delta (acc + b) (+ R_M on K); staged
-//               tiles go back with TMA stores.
+//               memory, then one of: bf16, GELU, fp32, RoPE on Q/K (into a
+//               128B-swizzled staging buffer, half a tile at a time), or in
+//               place on the staged tile: residual stream x += acc + b, cache
+//               kv = kv + sigma_delta (acc + b) (+ R_M on K).  Staged data goes
+//               out with TMA stores (coalesced, asynchronous).
 // The epilogue of tile i overlaps the MMAs of tile i+1.  Tiles are walked
 // W-tile-major (all M tiles of one N tile back to back), so a W tile is read
 // from HBM once and reused from L2 while the small A operand stays L2-resident.
@@ -35,21 +37,20 @@ constexpr uint32_t kSmemLimit = 232448;   // 227 KB opt-in per CTA
 template <int BN, int EPI>
 struct GemmCfg {
     static constexpr bool kKV = (EPI == EPI_KV_BF16 || EPI == EPI_KV_F32);
-    static constexpr bool kInPlace = kKV || EPI == EPI_ADD_F32;
-    static constexpr int kTileEsize = (EPI == EPI_KV_F32 || EPI == EPI_ADD_F32) ? 4 : 2;
-    static constexpr uint32_t kTileBytes = kInPlace ? BM * BN * kTileEsize : 0;
+    static constexpr bool kInPlace = kKV || EPI == EPI_ADD_F32;   // tile loaded, updated, stored
+    static constexpr int kTileEsize = (EPI == EPI_KV_F32 || EPI == EPI_ADD_F32 || EPI == EPI_F32) ? 4 : 2;
     static constexpr int kBoxCols = 128 / kTileEsize;          // one 128-byte swizzle row
-    static constexpr int kBoxes = kInPlace ? BN / kBoxCols : 0;
-    static constexpr uint32_t kVecBytes = BN * 4 * (kKV ? 2 : 1);   // bias (+ sigma) per slot
-    // epilogue-input slots: the staged in-place tile is single-buffered, bias-only
-    // slots are double-buffered so the next tile's bias lands during this epilogue
-    static constexpr int kEpiSlots = kInPlace ? 1 : 2;
+    // in-place epilogues stage the whole [BM x BN] tile; store-only epilogues
+    // stage one 16 KB box (128 rows x 128 B) at a time, double-buffered
+    static constexpr int kBoxes = BN / kBoxCols;                // boxes per tile
+    static constexpr uint32_t kTileBytes = kInPlace ? BM * BN * kTileEsize : 2 * 16384;
+    static constexpr uint32_t kVecBytes = BN * 4 * (kKV ? 2 : 1);   // bias (+ sigma)
     static constexpr uint32_t kBBytes = BN * BK * 2;
     static constexpr uint32_t kStageBytes = A_BYTES + kBBytes;
-    static constexpr uint32_t kFixed = 1024 + kTileBytes + kEpiSlots * kVecBytes + 256;
+    static constexpr uint32_t kFixed = 1024 + kTileBytes + kVecBytes + 256;
     static constexpr int kStagesFit = static_cast<int>((kSmemLimit - kFixed) / kStageBytes);
     static constexpr int kStages = kStagesFit > 6 ? 6 : kStagesFit;
-    static_assert(kStages >= 2, "GEMM tile does not fit in shared memory");
+    static_assert(kStages >= 3, "GEMM tile does not fit in shared memory");
     static constexpr uint32_t kSmemBytes = kFixed + kStages * kStageBytes;
     static constexpr uint32_t kTmemCols = 2 * BN;
 };
@@ -165,7 +166,7 @@ __device__ __forceinline__ void rotate16(float* a, float* b, float p, const floa
 }
 
 template <int BN, int EPI>
-__global__ void __launch_bounds__(224, 1)
+__global__ void __launch_bounds__(256, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const __grid_constant__ CUtensorMap tmC, const __grid_constant__ GemmParams p) {
     using Cfg = GemmCfg<BN, EPI>;
@@ -175,19 +176,19 @@ __global__ void __launch_bounds__(224, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    uint8_t* tile = smem + STAGES * Cfg::kStageBytes;              // staged output tile
+    uint8_t* tile = smem + STAGES * Cfg::kStageBytes;              // staged output (part)
     float* vec = reinterpret_cast<float*>(tile + Cfg::kTileBytes);  // bias [BN] (+ sigma [BN])
-    uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(vec) +
-                                                 Cfg::kEpiSlots * Cfg::kVecBytes);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(vec) + Cfg::kVecBytes);
     uint64_t* full = bars;
     uint64_t* empty = bars + STAGES;
     uint64_t* tfull = bars + 2 * STAGES;
     uint64_t* tempty = tfull + 2;
-    uint64_t* epi_full = tempty + 2;         // [kEpiSlots]
-    uint64_t* epi_empty = epi_full + 2;      // [kEpiSlots]
-    uint64_t* drain = epi_empty + 2;
-    uint64_t* epi_done = drain + 1;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(epi_done + 1);
+    uint64_t* epi_full = tempty + 2;     // loader -> epilogue: vectors (+ in-place tile) landed
+    uint64_t* epi_empty = epi_full + 1;  // epilogue -> loader: vectors / tile free again
+    uint64_t* drain = epi_empty + 1;
+    uint64_t* epi_done = drain + 1;      // [2] 128 epilogue threads wrote a staged buffer
+    uint64_t* st_free = epi_done + 2;    // [2] the TMA store has read that buffer
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(st_free + 2);
     int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
     const uint32_t warp = warp_id(), lane = lane_id();
@@ -200,12 +201,13 @@ __global__ void __launch_bounds__(224, 1)
             mbar_init(&tfull[s], 1);
             mbar_init(&tempty[s], 4);
         }
-        for (int s = 0; s < Cfg::kEpiSlots; ++s) {
-            mbar_init(&epi_full[s], 1);
-            mbar_init(&epi_empty[s], 1);
+        mbar_init(epi_full, 1);
+        mbar_init(epi_empty, 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&epi_done[b], 128);
+            mbar_init(&st_free[b], 1);
         }
         mbar_init(drain, 1);
-        mbar_init(epi_done, 128);
         *abort_flag = 0;
         fence_barrier_init();
     }
@@ -219,7 +221,7 @@ __global__ void __launch_bounds__(224, 1)
     const int total = p.num_m * p.num_n;
     const int num_k = (p.K + BK - 1) / BK;
     const bool has_bias = p.bias != nullptr;
-    // the epilogue consumes a per-tile load (vectors and/or the staged tile)
+    // the epilogue consumes a per-tile load (vectors and/or the in-place tile)
     const bool epi_load = Cfg::kInPlace || has_bias;
 
     if (warp == 0) {
@@ -253,37 +255,67 @@ __global__ void __launch_bounds__(224, 1)
         }
     } else if (warp == 6) {
         if (lane == 0 && epi_load) {
+            tma_prefetch(&tmC);
             // ------------------------------------------------ epilogue-input loader:
             // per tile, the bias (and sigma) slice by bulk copy and, for in-place
             // epilogues, the output tile by TMA, as soon as the epilogue has
             // released the slot (independent of the A/B stream of warp 0)
-            if constexpr (Cfg::kInPlace) tma_prefetch(&tmC);
             bool ok = true;
             int i = 0;
             for (int t = blockIdx.x; t < total; t += gridDim.x, ++i) {
                 const int m0 = (t % p.num_m) * BM;
                 const int n0 = (t / p.num_m) * BN;
-                const int slot = i % Cfg::kEpiSlots;
-                const uint32_t ph = static_cast<uint32_t>(i / Cfg::kEpiSlots) & 1u;
-                if (!(ok = mbar_wait(&epi_empty[slot], ph ^ 1u, wc, 101))) break;
+                if (!(ok = mbar_wait(epi_empty, (static_cast<uint32_t>(i) & 1u) ^ 1u, wc, 101))) break;
                 const int nb = min(BN, p.N - n0);
                 const uint32_t vbytes = static_cast<uint32_t>(nb) * 4u;
-                uint32_t bytes = Cfg::kTileBytes + (has_bias ? vbytes : 0u);
+                uint32_t bytes = (Cfg::kInPlace ? Cfg::kTileBytes : 0u) + (has_bias ? vbytes : 0u);
                 if constexpr (Cfg::kKV) bytes += vbytes;
-                float* v = vec + slot * (Cfg::kVecBytes / 4);
-                mbar_expect_tx(&epi_full[slot], bytes);
+                mbar_expect_tx(epi_full, bytes);
                 if constexpr (Cfg::kInPlace) {
                     for (int b = 0; b < Cfg::kBoxes; ++b)
-                        tma_load_2d(tile + b * 16384, &tmC, &epi_full[slot], n0 + b * Cfg::kBoxCols, m0);
+                        tma_load_2d(tile + b * 16384, &tmC, epi_full, n0 + b * Cfg::kBoxCols, m0);
                 }
-                if (has_bias) bulk_load(v, p.bias + n0, vbytes, &epi_full[slot]);
-                if constexpr (Cfg::kKV) bulk_load(v + BN, p.sigma + n0, vbytes, &epi_full[slot]);
+                if (has_bias) bulk_load(vec, p.bias + n0, vbytes, epi_full);
+                if constexpr (Cfg::kKV) bulk_load(vec + BN, p.sigma + n0, vbytes, epi_full);
             }
             if (!ok) {
                 const uint64_t t0 = globaltimer();
                 while (globaltimer() - t0 < 50000ull) {
                 }
             }
+        }
+    } else if (warp == 7) {
+        if (lane == 0) {
+            // ------------------------------------------------ TMA store issuer:
+            // writes each staged buffer back once the 128 epilogue threads have
+            // filled it, and hands the buffer (or the in-place tile and the
+            // bias slice) back when TMA has read it
+            bool ok = true;
+            uint32_t pk = 0;   // staged parts so far
+            for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+                const int m0 = (t % p.num_m) * BM;
+                const int n0 = (t / p.num_m) * BN;
+                if constexpr (Cfg::kInPlace) {
+                    if (!(ok = mbar_wait(&epi_done[0], pk & 1u, wc, 401))) break;
+                    for (int b = 0; b < Cfg::kBoxes; ++b)
+                        tma_store_2d(&tmC, tile + b * 16384, n0 + b * Cfg::kBoxCols, m0);
+                    tma_store_commit();
+                    tma_store_wait_read0();
+                    mbar_arrive(epi_empty);
+                    ++pk;
+                } else {
+                    for (int k = 0; k < Cfg::kBoxes; ++k, ++pk) {
+                        const uint32_t b = pk & 1u;
+                        if (!(ok = mbar_wait(&epi_done[b], (pk >> 1) & 1u, wc, 402))) break;
+                        tma_store_2d(&tmC, tile + b * 16384, n0 + k * Cfg::kBoxCols, m0);
+                        tma_store_commit();
+                        tma_store_wait_read0();
+                        mbar_arrive(&st_free[b]);
+                    }
+                    if (ok && epi_load) mbar_arrive(epi_empty);
+                }
+            }
+            tma_store_wait0();
         }
     } else if (warp == 1) {
         if (lane == 0) {
@@ -324,55 +356,27 @@ __global__ void __launch_bounds__(224, 1)
         // ---------------------------------------------------- epilogue (warps 2..5)
         const uint32_t quad = warp & 3u;
         const int r = static_cast<int>(quad * 32 + lane);     // row inside the tile
-        uint32_t acc = 0, acc_phase = 0, done_phase = 0;
+        constexpr int ES = Cfg::kTileEsize;
+        const float* vb = vec;             // bias slice of the tile
+        const float* vs = vec + BN;        // sigma_delta slice (KV epilogues)
+        uint32_t acc = 0, acc_phase = 0, pk = 0;
+        bool ok = true;
         int i = 0;
-        for (int t = blockIdx.x; t < total; t += gridDim.x, ++i) {
+        for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++i) {
             const int m0 = (t % p.num_m) * BM;
             const int n0 = (t / p.num_m) * BN;
-            const int slot = i % Cfg::kEpiSlots;
-            const float* vb = vec + slot * (Cfg::kVecBytes / 4);   // bias slice of the tile
-            const float* vs = vb + BN;                               // sigma_delta slice (KV)
-            bool ok = mbar_wait(&tfull[acc], acc_phase, wc, 301);
-            if (epi_load)
-                ok = ok && mbar_wait(&epi_full[slot],
-                                     static_cast<uint32_t>(i / Cfg::kEpiSlots) & 1u, wc, 302);
-            if (!__all_sync(0xffffffffu, ok)) break;
+            ok = mbar_wait(&tfull[acc], acc_phase, wc, 301);
+            if (epi_load) ok = ok && mbar_wait(epi_full, static_cast<uint32_t>(i) & 1u, wc, 302);
+            if (!__all_sync(0xffffffffu, ok)) {
+                ok = false;
+                break;
+            }
             tc_fence_after();
             const int row = m0 + r;
             const bool row_ok = row < p.M;
             const uint32_t taddr = tmem_base + ((quad * 32u) << 16) + acc * BN;
 
-            if constexpr (EPI == EPI_QKV_ROPE) {
-                const int hd = p.rope_dim;
-                const float pr = row_ok ? static_cast<float>(__ldg(p.pos + row)) : 0.0f;
-                uint16_t* orow = reinterpret_cast<uint16_t*>(p.out) + static_cast<int64_t>(row) * p.ldo;
-                for (int h0 = 0; h0 < BN; h0 += hd) {
-                    const bool rot = (n0 + h0) < p.rope_cols;
-                    for (int j = 0; j < hd / 2; j += 16) {
-                        float a[16], b[16], ba[16], bb[16];
-                        __syncwarp();
-                        tmem_ld16(taddr + h0 + j, a);
-                        tmem_ld16(taddr + h0 + hd / 2 + j, b);
-                        tmem_wait_ld();
-                        const int ta = h0 + j, tb = h0 + hd / 2 + j;
-                        if (has_bias) {
-                            vec16(vb, ta, ba);
-                            vec16(vb, tb, bb);
-#pragma unroll
-                            for (int i = 0; i < 16; ++i) {
-                                a[i] += ba[i];
-                                b[i] += bb[i];
-                            }
-                        }
-                        if (rot) rotate16(a, b, pr, p.inv_freq, j);
-                        if (row_ok) {
-                            store16_bf16_global(orow + n0 + ta, a);
-                            store16_bf16_global(orow + n0 + tb, b);
-                        }
-                    }
-                }
-            } else if constexpr (Cfg::kInPlace) {
-                constexpr int ES = Cfg::kTileEsize;
+            if constexpr (Cfg::kInPlace) {
                 if (Cfg::kKV && p.rope_on) {
                     // R_M pairs (d, d + d_h/2) live inside one d_h-wide segment
                     const int dh = p.rope_dim;
@@ -395,13 +399,13 @@ __global__ void __launch_bounds__(224, 1)
                                 vec16(vb, tb, bb);
                             } else {
 #pragma unroll
-                                for (int i = 0; i < 16; ++i) ba[i] = bb[i] = 0.0f;
+                                for (int q = 0; q < 16; ++q) ba[q] = bb[q] = 0.0f;
                             }
                             tmem_wait_ld();
 #pragma unroll
-                            for (int i = 0; i < 16; ++i) {
-                                ka[i] = fmaf(sa_[i], a[i] + ba[i], ka[i]);
-                                kb[i] = fmaf(sb_[i], b[i] + bb[i], kb[i]);
+                            for (int q = 0; q < 16; ++q) {
+                                ka[q] = fmaf(sa_[q], a[q] + ba[q], ka[q]);
+                                kb[q] = fmaf(sb_[q], b[q] + bb[q], kb[q]);
                             }
                             if (rot) rotate16(ka, kb, pr, p.inv_freq, j);
                             store16_tile<ES>(tile, r, ta, ka);
@@ -418,84 +422,134 @@ __global__ void __launch_bounds__(224, 1)
                             vec16(vb, c, bv);
                         } else {
 #pragma unroll
-                            for (int i = 0; i < 16; ++i) bv[i] = 0.0f;
+                            for (int q = 0; q < 16; ++q) bv[q] = 0.0f;
                         }
                         tmem_wait_ld();
                         if constexpr (Cfg::kKV) {
                             float sv[16];
                             vec16(vs, c, sv);
 #pragma unroll
-                            for (int i = 0; i < 16; ++i) k[i] = fmaf(sv[i], a[i] + bv[i], k[i]);
+                            for (int q = 0; q < 16; ++q) k[q] = fmaf(sv[q], a[q] + bv[q], k[q]);
                         } else {
 #pragma unroll
-                            for (int i = 0; i < 16; ++i) k[i] += a[i] + bv[i];
+                            for (int q = 0; q < 16; ++q) k[q] += a[q] + bv[q];
                         }
                         store16_tile<ES>(tile, r, c, k);
                     }
                 }
-            } else {
-                for (int c = 0; c < BN; c += 16) {
-                    float v[16];
-                    __syncwarp();
-                    tmem_ld16(taddr + c, v);
-                    tmem_wait_ld();
-                    const int col = n0 + c;
-                    if (col >= p.N || !row_ok) continue;
-                    if (has_bias) {
-                        float bv[16];
-                        vec16(vb, c, bv);
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) v[i] += bv[i];
-                    }
-                    if constexpr (EPI == EPI_BF16 || EPI == EPI_GELU_BF16) {
-                        if constexpr (EPI == EPI_GELU_BF16) {
-#pragma unroll
-                            for (int i = 0; i < 16; ++i) v[i] = gelu_erf(v[i]);
-                        }
-                        store16_bf16_global(
-                            reinterpret_cast<uint16_t*>(p.out) + static_cast<int64_t>(row) * p.ldo + col, v);
-                    } else {
-                        float4* o = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) +
-                                                              static_cast<int64_t>(row) * p.ldo + col);
-#pragma unroll
-                        for (int q = 0; q < 4; ++q)
-                            o[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-                    }
-                }
-            }
-            // accumulator buffer free for the MMA warp
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&tempty[acc]);
-            if (epi_load) {
-                // this thread's reads of the vectors and writes of the staged tile
-                // are done; lane 0 of warp 2 waits (bounded) for all 128, stores
-                // the staged tile with TMA and hands the area back to the producer
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&tempty[acc]);
                 fence_async_smem();
-                mbar_arrive(epi_done);
-                if (warp == 2) {
-                    bool ok2 = true;
-                    if (lane == 0) {
-                        ok2 = mbar_wait(epi_done, done_phase, wc, 303);
-                        if (ok2) {
-                            if constexpr (Cfg::kInPlace) {
-                                for (int b = 0; b < Cfg::kBoxes; ++b)
-                                    tma_store_2d(&tmC, tile + b * 16384, n0 + b * Cfg::kBoxCols, m0);
-                                tma_store_commit();
-                                tma_store_wait_read0();
+                mbar_arrive(&epi_done[0]);
+                ++pk;
+            } else {
+                // store-only epilogues: one 128 B-wide box of columns at a time,
+                // into alternating staging buffers
+                constexpr int PC = Cfg::kBoxCols;
+                // QKV: the rotation angles depend on (row, pair index) only, so
+                // cos/sin are computed once per tile for every head in it
+                constexpr int NP = (EPI == EPI_QKV_ROPE) ? 32 : 1;
+                float cs[NP], sn[NP];
+                if constexpr (EPI == EPI_QKV_ROPE) {
+                    if (p.rope_table) {
+                        // precomputed per forward: this row's (cos, sin) pairs
+                        const float4* tr = reinterpret_cast<const float4*>(
+                            p.rope_table + static_cast<int64_t>(row_ok ? row : 0) * (p.rope_dim / 2));
+#pragma unroll
+                        for (int q = 0; q < NP; q += 2) {
+                            if (q < p.rope_dim / 2) {
+                                const float4 v = __ldg(tr + q / 2);
+                                cs[q] = v.x;
+                                sn[q] = v.y;
+                                cs[q + 1] = v.z;
+                                sn[q + 1] = v.w;
                             }
-                            mbar_arrive(&epi_empty[slot]);
+                        }
+                    } else {
+                        const float pr = row_ok ? static_cast<float>(__ldg(p.pos + row)) : 0.0f;
+#pragma unroll
+                        for (int q = 0; q < NP; ++q)
+                            if (q < p.rope_dim / 2) sincos_prod(pr, p.inv_freq[q], &sn[q], &cs[q]);
+                    }
+                }
+                for (int k = 0; k < Cfg::kBoxes && ok; ++k, ++pk) {
+                    const uint32_t bsel = pk & 1u;
+                    if (pk >= 2) {
+                        ok = mbar_wait(&st_free[bsel], ((pk >> 1) - 1) & 1u, wc, 304);
+                        if (!__all_sync(0xffffffffu, ok)) {
+                            ok = false;
+                            break;
                         }
                     }
-                    if (!__shfl_sync(0xffffffffu, ok2 ? 1 : 0, 0)) break;
+                    uint8_t* buf = tile + bsel * 16384;
+                    const int c0 = k * PC;
+                    if constexpr (EPI == EPI_QKV_ROPE) {
+                        const int hd = p.rope_dim;
+#pragma unroll
+                        for (int j = 0; j < NP; j += 16) {
+                            if (j >= hd / 2) break;
+                            for (int h0 = c0; h0 < c0 + PC; h0 += hd) {
+                                const bool rot = (n0 + h0) < p.rope_cols;
+                                float a[16], b[16];
+                                const int ta = h0 + j, tb = h0 + hd / 2 + j;
+                                __syncwarp();
+                                tmem_ld16(taddr + ta, a);
+                                tmem_ld16(taddr + tb, b);
+                                tmem_wait_ld();
+                                if (has_bias) {
+                                    float ba[16], bb[16];
+                                    vec16(vb, ta, ba);
+                                    vec16(vb, tb, bb);
+#pragma unroll
+                                    for (int q = 0; q < 16; ++q) {
+                                        a[q] += ba[q];
+                                        b[q] += bb[q];
+                                    }
+                                }
+                                if (rot) {
+#pragma unroll
+                                    for (int q = 0; q < 16; ++q) {
+                                        const float x = a[q], y = b[q];
+                                        a[q] = x * cs[j + q] - y * sn[j + q];
+                                        b[q] = y * cs[j + q] + x * sn[j + q];
+                                    }
+                                }
+                                store16_tile<ES>(buf, r, ta - c0, a);
+                                store16_tile<ES>(buf, r, tb - c0, b);
+                            }
+                        }
+                    } else {
+                        for (int c = c0; c < c0 + PC; c += 16) {
+                            float v[16];
+                            __syncwarp();
+                            tmem_ld16(taddr + c, v);
+                            tmem_wait_ld();
+                            if (has_bias) {
+                                float bv[16];
+                                vec16(vb, c, bv);
+#pragma unroll
+                                for (int q = 0; q < 16; ++q) v[q] += bv[q];
+                            }
+                            if constexpr (EPI == EPI_GELU_BF16) {
+#pragma unroll
+                                for (int q = 0; q < 16; ++q) v[q] = gelu_erf(v[q]);
+                            }
+                            store16_tile<ES>(buf, r, c - c0, v);
+                        }
+                    }
+                    if (k == Cfg::kBoxes - 1) {
+                        // TMEM buffer fully read
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&tempty[acc]);
+                    }
+                    fence_async_smem();
+                    mbar_arrive(&epi_done[bsel]);
                 }
-                done_phase ^= 1u;
             }
             acc ^= 1u;
             if (acc == 0) acc_phase ^= 1u;
-        }
-        if constexpr (Cfg::kInPlace) {
-            if (warp == 2 && lane == 0) tma_store_wait0();
         }
     }
     __syncthreads();
@@ -516,7 +570,7 @@ cr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensor
     if (sa != CR_OK) return sa;
     const int tiles = p.num_m * p.num_n;
     const int grid = tiles < num_sms() ? tiles : num_sms();
-    kern<<<grid, 224, Cfg::kSmemBytes, st>>>(ta, tb, tc, p);
+    kern<<<grid, 256, Cfg::kSmemBytes, st>>>(ta, tb, tc, p);
     return cuda_check(cudaGetLastError());
 }
 
@@ -549,18 +603,15 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
     if (!make_tmap_2d(&tb, W, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, K, N, K * 2, BK, BN,
                       CU_TENSOR_MAP_SWIZZLE_128B))
         return CR_ERR_INVALID_ARG;
-    tc = ta;
-    if (kv) {
-        if (!make_tmap_2d(&tc, kv_base,
-                          f32_tile ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
-                          N, M, ld_kv * (f32_tile ? 4 : 2), f32_tile ? 32 : 64, BM,
-                          CU_TENSOR_MAP_SWIZZLE_128B))
-            return CR_ERR_INVALID_ARG;
-    } else if (epi == EPI_ADD_F32) {
-        if (!make_tmap_2d(&tc, p.out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, N, M, p.ldo * 4, 32, BM,
-                          CU_TENSOR_MAP_SWIZZLE_128B))
-            return CR_ERR_INVALID_ARG;
-    }
+    // output (staged) tile map: bf16 boxes of 64 or fp32 boxes of 32 columns
+    const bool f32_out = f32_tile || epi == EPI_F32;
+    void* out_base = kv ? kv_base : p.out;
+    const int64_t ld_out = kv ? ld_kv : p.ldo;
+    if (!make_tmap_2d(&tc, out_base,
+                      f32_out ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                      N, M, ld_out * (f32_out ? 4 : 2), f32_out ? 32 : 64, BM,
+                      CU_TENSOR_MAP_SWIZZLE_128B))
+        return CR_ERR_INVALID_ARG;
     switch (epi) {
         case EPI_BF16:
             return BN == 256 ? launch_bn<256, EPI_BF16>(ta, tb, tc, p, st)

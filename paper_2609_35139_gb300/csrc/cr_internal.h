@@ -67,6 +67,7 @@ struct GemmParams {
     int32_t rope_on;         // KV: rotate K segments
     int32_t n_kv_heads;      // KV: segment s is K iff (s / n_kv_heads) is even
     const float* sigma;      // KV: sigma_delta [N]
+    const float2* rope_table;  // QKV: (cos, sin) [M, rope_dim / 2], or null (computed inline)
     unsigned* status;
     float inv_freq[64];      // RoPE frequencies, rope_dim / 2 entries
 };
@@ -131,6 +132,8 @@ cr_status launch_segproj(const uint16_t* kv, int64_t ld_kv, const uint16_t* wfol
 cr_status launch_fold_sigma(const uint16_t* w_seg, const float* sigma, int S, int d_seg,
                             int head_dim, uint16_t* wfold, cudaStream_t st);
 cr_status launch_to_bf16(const float* x, int64_t n, uint16_t* y, cudaStream_t st);
+cr_status launch_rope_table(const int32_t* pos, int64_t n, int half_dim, const float* inv_freq_host,
+                            float2* table, cudaStream_t st);
 cr_status launch_layernorm(const float* x, const uint16_t* add, int64_t ld_add, float* x_out,
                            const float* g, const float* b, float eps, int64_t M, int64_t D,
                            uint16_t* u, cudaStream_t st);

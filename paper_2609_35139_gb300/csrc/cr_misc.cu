@@ -132,7 +132,37 @@ __global__ void to_bf16_kernel(const float* __restrict__ x, int64_t n, uint16_t*
     }
 }
 
+struct InvFreq {
+    float f[64];
+};
+
+// (cos, sin) of pos[t] * inv_freq[i] for every token and pair index, the angle's
+// product rounding folded back in (same arithmetic as the in-epilogue path).
+__global__ void rope_table_kernel(const int32_t* __restrict__ pos, int64_t n, int half,
+                                  const __grid_constant__ InvFreq f, float2* __restrict__ table) {
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n * half;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t t = i / half;
+        const int q = static_cast<int>(i - t * half);
+        float s, c;
+        sincos_prod(static_cast<float>(__ldg(pos + t)), f.f[q], &s, &c);
+        table[i] = make_float2(c, s);
+    }
+}
+
 }  // namespace
+
+cr_status launch_rope_table(const int32_t* pos, int64_t n, int half_dim, const float* inv_freq_host,
+                            float2* table, cudaStream_t st) {
+    if (n <= 0) return CR_OK;
+    if (half_dim < 1 || half_dim > 64) return CR_ERR_UNSUPPORTED;
+    InvFreq f{};
+    for (int i = 0; i < half_dim; ++i) f.f[i] = inv_freq_host[i];
+    int64_t blocks = (n * half_dim + 255) / 256;
+    if (blocks > static_cast<int64_t>(num_sms()) * 8) blocks = static_cast<int64_t>(num_sms()) * 8;
+    rope_table_kernel<<<static_cast<int>(blocks), 256, 0, st>>>(pos, n, half_dim, f, table);
+    return cuda_check(cudaGetLastError());
+}
 
 cr_status launch_gather(const GatherParams& p, cudaStream_t st) {
     if (p.n_tokens <= 0) return CR_OK;
