@@ -7,23 +7,28 @@
 // chunk ends inside a key tile mask the rest of it; fully visible tiles do no
 // masking work at all.
 //
-// CTA = (request, head, two consecutive 128-query tiles).  10 warps:
+// CTA = (request, head, two consecutive 128-query tiles w = 0, 1); three
+// warpgroups, the first of which gives registers to the other two:
 //   warp 0      TMA: both Q tiles once, then K_j and V_j per key tile into a
 //               5-deep ring shared by the two query tiles
-//   warp 1      TMEM owner; one lane issues, per key tile j and query tile w,
-//               S_w,j = Q_w K_j^T (M=128, N=128, K=d) into S_w, and, once
-//               softmax w has written P_w,j, O_w += P_w,j V_j (M=128, N=d,
-//               K=128, V read MN-major) accumulating in TMEM
-//   warps 2..5  softmax group 0 (query tile 0), one row per thread
-//   warps 6..9  softmax group 1 (query tile 1)
-// The two groups ping-pong on the tensor core.  Per key tile a group reads its
-// S row from TMEM twice, 64 columns at a time (the (masked) row max, then the
-// exponentials; 320 threads leave 168 registers each), and writes
-// P = 2^(s*scale*log2e - m) as bf16 pairs into its own TMEM columns, from
+//   warp 1 + w  MMA issue for query tile w (warp 1 also owns TMEM): per key
+//               tile j, S_w,j+1 = Q_w K_j+1^T (M=128, N=128, K=d) as soon as
+//               softmax w has read S_w,j into registers, and O_w += P_w,j V_j
+//               (M=128, N=d, K=128, P read from TMEM, V MN-major from smem)
+//               once softmax w has written P_w,j.  Issue runs in a converged
+//               warp with one elected lane, and each query tile has its own
+//               issuer: the small MMAs of a d <= 64 head are cheap enough that
+//               issue and barrier latency, not the tensor core, set the pace.
+//   warps 4..7  softmax group 0 (query tile 0), one row per thread
+//   warps 8..11 softmax group 1 (query tile 1)
+// Per key tile a softmax thread loads its whole S row (128 fp32) from TMEM in
+// one round trip, masks and takes the row max in registers, and writes
+// P = 2^(s*scale*log2e - m) as bf16 pairs into its group's TMEM columns, from
 // where the PV MMA reads it as the A operand (TMEM holds S_0, S_1, O_0, O_1,
-// P_0, P_1: 512 columns).  The reference m is the row's running max,
-// updated lazily: only when a tile raises it by more than 2^8 does the group
-// rescale its O row in TMEM (and the row sum l).  Any reference m gives the same
+// P_0, P_1: 512 columns).  The two groups overlap each other's exponentials
+// with their MMAs.  The reference m is the row's running max, updated
+// lazily: only when a tile raises it by more than 2^8 does the group rescale
+// its O row in TMEM (and the row sum l).  Any reference m gives the same
 // softmax (it cancels in O / l), and keeping it at most 8 below the true
 // running max keeps P <= 2^8, so this is exact up to rounding.
 // O_w is read back and divided by l after the last tile.
@@ -45,14 +50,47 @@ struct AttnCfg {
     static constexpr uint32_t kQOff = 0;                                  // Q0, Q1
     static constexpr uint32_t kKVOff = 2 * kTileBytes;                    // K, V per stage
     static constexpr uint32_t kBarOff = kKVOff + kStages * 2 * kTileBytes;
-    static constexpr uint32_t kSmemBytes = 1024 + kBarOff + 256;
+    static constexpr uint32_t kSmemBytes = 1024 + kBarOff + 320;
     static constexpr uint32_t kTmemS = 0;      // S_w at w * 128 (fp32)
     static constexpr uint32_t kTmemO = 256;    // O_w at 256 + w * D (fp32)
     static constexpr uint32_t kTmemP = 384;    // P_w at 384 + w * 64 (bf16 pairs)
 };
 
-constexpr int kThreads = 320;
+// Three warpgroups: control (TMA, two MMA issuers, one idle warp) and two
+// softmax groups.
+// At launch each thread gets 65536 / 384 = 168 registers (the host checks
+// this); the control warpgroup gives up most of its share so that the softmax
+// threads can hold a whole S row: 72 * 128 + 2 * 216 * 128 = 168 * 384.
+constexpr int kThreads = 384;
+constexpr uint32_t kRegsLaunch = 168;
+constexpr uint32_t kRegsCtl = 72;
+constexpr uint32_t kRegsSoftmax = 216;
+static_assert(kRegsCtl * 128 + 2 * kRegsSoftmax * 128 <= kRegsLaunch * kThreads,
+              "register split exceeds the launch allocation");
 constexpr float kRescaleLog2 = 8.0f;   // lazy-rescale threshold (log2 units)
+
+// Two fp32 lanes per instruction (Blackwell packed fp32): d = a * b + c, d = a + b.
+__device__ __forceinline__ void ffma2(float& d0, float& d1, float a0, float a1, float b0, float b1,
+                                      float c0, float c1) {
+    asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+        "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d0), "=f"(d1)
+        : "f"(a0), "f"(a1), "f"(b0), "f"(b1), "f"(c0), "f"(c1));
+}
+__device__ __forceinline__ void fadd2(float& d0, float& d1, float a0, float a1, float b0, float b1) {
+    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d0), "=f"(d1)
+        : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
+}
+
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
 
 __device__ __forceinline__ float ex2(float x) {
     float y;
@@ -74,14 +112,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Cfg::kBarOff);
     uint64_t* q_full = bars;
-    uint64_t* k_full = bars + 1;
-    uint64_t* v_full = k_full + NS;
-    uint64_t* kv_empty = v_full + NS;
-    uint64_t* s_full = kv_empty + NS;     // [2]
-    uint64_t* p_full = s_full + 2;        // [2]
-    uint64_t* o_done = p_full + 2;        // [2]
-    uint64_t* drain = o_done + 2;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    uint64_t* kv_full = bars + 1;
+    uint64_t* kv_empty = kv_full + NS;
+    uint64_t* s_full = kv_empty + NS;     // [2] S_w,j in TMEM
+    uint64_t* s_free = s_full + 2;        // [2] S_w,j read into registers
+    uint64_t* p_full = s_free + 2;        // [2] P_w,j in TMEM
+    uint64_t* pv_done = p_full + 2;       // [2] O_w += P_w,j V_j complete
+    uint64_t* drain = pv_done + 2;        // [2]
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 2);
     int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
     // ---- work item: (request, pair of query tiles, head); heaviest pairs first
@@ -104,16 +142,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         mbar_init(q_full, 1);
         for (int s = 0; s < NS; ++s) {
-            mbar_init(&k_full[s], 1);
-            mbar_init(&v_full[s], 1);
-            mbar_init(&kv_empty[s], 1);
+            mbar_init(&kv_full[s], 1);
+            mbar_init(&kv_empty[s], 2);   // both issuers release each stage
         }
         for (int w = 0; w < 2; ++w) {
             mbar_init(&s_full[w], 1);
-            mbar_init(&p_full[w], 128);
-            mbar_init(&o_done[w], 1);
+            mbar_init(&s_free[w], 4);
+            mbar_init(&p_full[w], 4);
+            mbar_init(&pv_done[w], 1);
+            mbar_init(&drain[w], 1);
         }
-        mbar_init(drain, 1);
         *abort_flag = 0;
         fence_barrier_init();
     }
@@ -124,94 +162,127 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem_base = *tmem_slot;
     const WaitCtx wc{abort_flag, p.status};
 
-    if (warp == 0) {
-        if (lane == 0) {
+    if (warp < 4) {
+        setmaxnreg_dec<kRegsCtl>();
+        if (warp == 0) {
             // ---------------------------------------------------- TMA producer
-            tma_prefetch(&tmQKV);
-            mbar_expect_tx(q_full, 2 * Cfg::kTileBytes);
-            tma_load_2d(smem + Cfg::kQOff, &tmQKV, q_full, head * D, rs + q0);
-            tma_load_2d(smem + Cfg::kQOff + Cfg::kTileBytes, &tmQKV, q_full, head * D,
-                        rs + q0 + 128);
+            // (the whole warp runs the loop; one elected lane issues)
+            if (elect_one()) {
+                tma_prefetch(&tmQKV);
+                mbar_expect_tx(q_full, 2 * Cfg::kTileBytes);
+                tma_load_2d(smem + Cfg::kQOff, &tmQKV, q_full, head * D, rs + q0);
+                tma_load_2d(smem + Cfg::kQOff + Cfg::kTileBytes, &tmQKV, q_full, head * D,
+                            rs + q0 + 128);
+            }
+            __syncwarp();
             bool ok = true;
             for (int j = 0; j < n_max; ++j) {
                 const int st = j % NS;
                 const uint32_t ph = static_cast<uint32_t>(j / NS) & 1u;
-                if (!(ok = mbar_wait(&kv_empty[st], ph ^ 1u, wc, 121))) break;
+                if (!(ok = mbar_wait_warp(&kv_empty[st], ph ^ 1u, wc, 121))) break;
                 uint8_t* kt = smem + Cfg::kKVOff + st * 2 * Cfg::kTileBytes;
-                mbar_expect_tx(&k_full[st], Cfg::kTileBytes);
-                tma_load_2d(kt, &tmQKV, &k_full[st], p.d_b + head * D, rs + j * 128);
-                mbar_expect_tx(&v_full[st], Cfg::kTileBytes);
-                tma_load_2d(kt + Cfg::kTileBytes, &tmQKV, &v_full[st], 2 * p.d_b + head * D,
-                            rs + j * 128);
+                if (elect_one()) {
+                    mbar_expect_tx(&kv_full[st], 2 * Cfg::kTileBytes);
+                    tma_load_2d(kt, &tmQKV, &kv_full[st], p.d_b + head * D, rs + j * 128);
+                    tma_load_2d(kt + Cfg::kTileBytes, &tmQKV, &kv_full[st], 2 * p.d_b + head * D,
+                                rs + j * 128);
+                }
+                __syncwarp();
             }
             if (!ok) {
                 const uint64_t t0 = globaltimer();
                 while (globaltimer() - t0 < 50000ull) {
                 }
             }
-        }
-    } else if (warp == 1) {
-        if (lane == 0) {
-            // ---------------------------------------------------- MMA issuer
-            // Per query tile w the order is S_0, [P_0] PV_0, S_1, [P_1] PV_1, ...
-            // so the commit after S_j+1 also covers PV_j: when the softmax group
-            // sees S_j+1 its O row is current and its P buffer is free.
-            const uint32_t sq0 = smem_u32(smem + Cfg::kQOff);
-            auto issue_s = [&](int w, int j) -> bool {
-                const int st = j % NS;
-                if (!mbar_wait(&k_full[st], static_cast<uint32_t>(j / NS) & 1u, wc, 222)) return false;
+        } else if (warp == 1 || warp == 2) {
+            // ---------------------------------------------------- MMA issuers
+            // Warp 1 + w issues for query tile w: per key tile j, S_w,j+1 as
+            // soon as softmax w has read S_w,j out of TMEM, then O_w += P_w,j V_j
+            // once P_w,j is written.  The whole warp runs the loop and computes
+            // the descriptors; one elected lane issues the MMAs and commits.
+            const int w = static_cast<int>(warp) - 1;
+            const int n = n_kv[w];
+            // Descriptors are built once; a K=16 step adds 32 bytes (2 units of
+            // 16 B) to the start address, a stage adds 2 tiles, a V step 16 rows.
+            constexpr uint64_t kStageStep = (2 * Cfg::kTileBytes) >> 4;
+            const uint64_t dq = smem_desc(smem_u32(smem + Cfg::kQOff + w * Cfg::kTileBytes), 16,
+                                          Cfg::kAtomBytes, Cfg::kSwz);
+            const uint64_t dk0 = smem_desc(smem_u32(smem + Cfg::kKVOff), 16, Cfg::kAtomBytes, Cfg::kSwz);
+            const uint64_t dv0 = smem_desc(smem_u32(smem + Cfg::kKVOff + Cfg::kTileBytes),
+                                           Cfg::kTileBytes, Cfg::kAtomBytes, Cfg::kSwz);
+            const uint32_t ds = tmem_base + Cfg::kTmemS + w * 128;
+            const uint32_t dout = tmem_base + Cfg::kTmemO + w * D;
+            const uint32_t pa = tmem_base + Cfg::kTmemP + w * 64;
+            int kv_ready = -1;   // key/value tiles 0..kv_ready are known to be in smem
+            auto ensure_kv = [&](int j) -> bool {
+                if (j <= kv_ready) return true;
+                if (!mbar_wait_warp(&kv_full[j % NS], static_cast<uint32_t>(j / NS) & 1u, wc, 222))
+                    return false;
                 tc_fence_after();
-                const uint32_t sq = sq0 + w * Cfg::kTileBytes;
-                const uint32_t sk = smem_u32(smem + Cfg::kKVOff + st * 2 * Cfg::kTileBytes);
-                const uint32_t d = tmem_base + Cfg::kTmemS + w * 128;
-#pragma unroll
-                for (int k = 0; k < D / 16; ++k)
-                    mma_bf16_ss(d, smem_desc(sq + k * 32, 16, Cfg::kAtomBytes, Cfg::kSwz),
-                                smem_desc(sk + k * 32, 16, Cfg::kAtomBytes, Cfg::kSwz), IDESC_S,
-                                k != 0 ? 1u : 0u);
-                mma_commit(&s_full[w]);
+                kv_ready = j;
                 return true;
             };
-            auto issue_pv = [&](int w, int j) -> bool {
-                const int st = j % NS;
-                if (!mbar_wait(&p_full[w], static_cast<uint32_t>(j) & 1u, wc, 224)) return false;
-                if (!mbar_wait(&v_full[st], static_cast<uint32_t>(j / NS) & 1u, wc, 225)) return false;
-                tc_fence_after();
-                const uint32_t sv =
-                    smem_u32(smem + Cfg::kKVOff + st * 2 * Cfg::kTileBytes + Cfg::kTileBytes);
-                const uint32_t d = tmem_base + Cfg::kTmemO + w * D;
-                const uint32_t pa = tmem_base + Cfg::kTmemP + w * 64;
+            auto issue_s = [&](int j) -> bool {
+                if (!ensure_kv(j)) return false;
+                const uint64_t dk = dk0 + static_cast<uint64_t>(j % NS) * kStageStep;
+                if (elect_one()) {
 #pragma unroll
-                for (int kk = 0; kk < 8; ++kk) {
-                    // P from TMEM (16 keys = 8 columns); V: rows = keys (the K
-                    // dimension), d contiguous (MN-major); 16 keys = two 8-row atoms.
-                    const uint64_t db = smem_desc(sv + kk * 16 * Cfg::kRowBytes, Cfg::kTileBytes,
-                                                  Cfg::kAtomBytes, Cfg::kSwz);
-                    mma_bf16_ts(d, pa + kk * 8, db, IDESC_PV, (j > 0 || kk != 0) ? 1u : 0u);
+                    for (int k = 0; k < D / 16; ++k)
+                        mma_bf16_ss(ds, dq + 2 * k, dk + 2 * k, IDESC_S, k != 0 ? 1u : 0u);
+                    mma_commit(&s_full[w]);
                 }
+                __syncwarp();
                 return true;
             };
-            bool ok = mbar_wait(q_full, 0, wc, 221);
+            auto issue_pv = [&](int j) -> bool {
+                if (!mbar_wait_warp(&p_full[w], static_cast<uint32_t>(j) & 1u, wc, 224)) return false;
+                tc_fence_after();
+                if (!ensure_kv(j)) return false;
+                const uint64_t dv = dv0 + static_cast<uint64_t>(j % NS) * kStageStep;
+                if (elect_one()) {
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) {
+                        // P from TMEM (16 keys = 8 columns); V: rows = keys (the K
+                        // dimension), d contiguous (MN-major); 16 keys = two 8-row atoms.
+                        mma_bf16_ts(dout, pa + kk * 8, dv + kk * ((16 * Cfg::kRowBytes) >> 4), IDESC_PV,
+                                    (j > 0 || kk != 0) ? 1u : 0u);
+                    }
+                    mma_commit(&pv_done[w]);
+                }
+                __syncwarp();
+                return true;
+            };
+            bool ok = mbar_wait_warp(q_full, 0, wc, 221);
             if (ok) tc_fence_after();
-            for (int w = 0; w < 2 && ok; ++w)
-                if (n_kv[w] > 0) ok = issue_s(w, 0);
+            if (ok && n > 0) ok = issue_s(0);
             for (int j = 0; j < n_max && ok; ++j) {
-                for (int w = 0; w < 2 && ok; ++w) {
-                    if (j >= n_kv[w]) continue;
-                    if (!(ok = issue_pv(w, j))) break;
-                    if (j + 1 < n_kv[w])
-                        ok = issue_s(w, j + 1);
-                    else
-                        mma_commit(&o_done[w]);
+                if (j < n) {
+                    if (j + 1 < n) {
+                        ok = mbar_wait_warp(&s_free[w], static_cast<uint32_t>(j) & 1u, wc, 223);
+                        if (ok) {
+                            tc_fence_after();
+                            ok = issue_s(j + 1);
+                        }
+                    }
+                    if (ok) ok = issue_pv(j);
+                } else {
+                    // a tile only the other query tile needs: wait for it so that
+                    // this release lands in the stage's current phase
+                    ok = ensure_kv(j);
                 }
-                if (ok) mma_commit(&kv_empty[j % NS]);
+                if (ok) {
+                    if (elect_one()) mma_commit(&kv_empty[j % NS]);
+                    __syncwarp();
+                }
             }
-            mma_commit(drain);
-            mbar_wait(drain, 0, wc, 227);
+            if (elect_one()) mma_commit(&drain[w]);
+            __syncwarp();
+            mbar_wait_warp(&drain[w], 0, wc, 227);
         }
     } else {
+        setmaxnreg_inc<kRegsSoftmax>();
         // ---------------------------------------------------- softmax groups
-        const int w = (warp >= 6) ? 1 : 0;
+        const int w = (warp >= 8) ? 1 : 0;
         const uint32_t quad = warp & 3u;
         const int r = static_cast<int>(quad * 32 + lane);
         const int qrow = q0 + 128 * w + r;
@@ -233,39 +304,48 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             tc_fence_after();
+            // the whole S row in registers: one TMEM round trip per tile, after
+            // which the tensor core may overwrite S with the next tile's scores
+            float s[128];
+            tmem_ld32(ts, s);
+            tmem_ld32(ts + 32, s + 32);
+            tmem_ld32(ts + 64, s + 64);
+            tmem_ld32(ts + 96, s + 96);
+            tmem_wait_ld();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s_free[w]);
             const int k0 = j * 128;
-            const bool full_tile = k0 + 128 <= cend;     // all 128 keys visible to this row
-            // pass 1: row max of the (masked) scores, 64 columns at a time, in
-            // eight independent chains
+            if (k0 + 128 > cend) {
+                // keys >= cend are masked; fully visible tiles skip this
+                const int lim = cend - k0;
+#pragma unroll
+                for (int i = 0; i < 128; ++i) s[i] = (i < lim) ? s[i] : NEG_INF;
+            }
+            // row max of the (masked) scores in eight independent chains
             float mxv[8];
 #pragma unroll
             for (int q = 0; q < 8; ++q) mxv[q] = NEG_INF;
 #pragma unroll
-            for (int h = 0; h < 128; h += 64) {
-                float s[64];
-                __syncwarp();
-                tmem_ld32(ts + h, s);
-                tmem_ld32(ts + h + 32, s + 32);
-                tmem_wait_ld();
-                if (full_tile) {
-#pragma unroll
-                    for (int i = 0; i < 64; ++i) mxv[i & 7] = fmaxf(mxv[i & 7], s[i]);
-                } else {
-#pragma unroll
-                    for (int i = 0; i < 64; ++i)
-                        if (k0 + h + i < cend) mxv[i & 7] = fmaxf(mxv[i & 7], s[i]);
-                }
-            }
+            for (int i = 0; i < 128; i += 2) mxv[(i >> 1) & 7] = fmax3(mxv[(i >> 1) & 7], s[i], s[i + 1]);
             float mx = fmaxf(fmaxf(fmaxf(mxv[0], mxv[1]), fmaxf(mxv[2], mxv[3])),
                              fmaxf(fmaxf(mxv[4], mxv[5]), fmaxf(mxv[6], mxv[7])));
             mx *= sc;
+            // O_w and P_w are free once PV_w,j-1 has completed
+            if (j > 0) {
+                ok = mbar_wait(&pv_done[w], static_cast<uint32_t>(j - 1) & 1u, wc, 322);
+                if (!__all_sync(0xffffffffu, ok)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+            }
             // lazily move the reference max: on the first tile, or when this
             // tile would push P above 2^8 somewhere in the warp
             const bool raise = (j == 0) || (mx > m + kRescaleLog2);
             if (__any_sync(0xffffffffu, raise)) {
                 const float m_new = fmaxf(m, mx);
                 if (j > 0) {
-                    // O holds sum_{k<j} P_k V_k (complete: S_j was issued after PV_{j-1})
                     const float alpha = ex2(m - m_new);
 #pragma unroll
                     for (int c = 0; c < D; c += 16) {
@@ -276,35 +356,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                         for (int i = 0; i < 16; ++i) o[i] *= alpha;
                         tmem_st16(to + c, o);
                     }
-                    tmem_wait_st();
                     l *= alpha;
                 }
                 m = m_new;
             }
-            // pass 2: P = 2^(s*sc - m) -> bf16, swizzled K-major, and the row sum.
-            // Fully visible tiles (all tiles of chunk-aligned maps) take a loop
-            // with no per-element masking.
+            // P = 2^(s*sc - m) -> bf16 pairs in TMEM, and the row sum
             float rs8[8];
 #pragma unroll
             for (int q = 0; q < 8; ++q) rs8[q] = 0.0f;
-            const int lim = full_tile ? 128 : cend - k0;   // keys < lim are visible
 #pragma unroll
             for (int h = 0; h < 128; h += 64) {
-                float s[64];
-                __syncwarp();
-                tmem_ld32(ts + h, s);
-                tmem_ld32(ts + h + 32, s + 32);
-                tmem_wait_ld();
-                if (!full_tile) {
-#pragma unroll
-                    for (int i = 0; i < 64; ++i) s[i] = (h + i < lim) ? s[i] : NEG_INF;
-                }
                 uint32_t pk[32];
 #pragma unroll
                 for (int i = 0; i < 64; i += 2) {
-                    const float e0 = ex2(fmaf(s[i], sc, -m));
-                    const float e1 = ex2(fmaf(s[i + 1], sc, -m));
-                    rs8[(i >> 1) & 7] += e0 + e1;
+                    float t0, t1;
+                    ffma2(t0, t1, s[h + i], s[h + i + 1], sc, sc, -m, -m);
+                    const float e0 = ex2(t0);
+                    const float e1 = ex2(t1);
+                    const int q = (i >> 1) & 3;       // four pairs of running sums
+                    fadd2(rs8[2 * q], rs8[2 * q + 1], rs8[2 * q], rs8[2 * q + 1], e0, e1);
                     pk[i >> 1] = pack_bf16x2(e0, e1);
                 }
                 tmem_st32u(tp + h / 2, pk);
@@ -312,10 +382,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             l += ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
             tmem_wait_st();
             tc_fence_before();
-            mbar_arrive(&p_full[w]);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&p_full[w]);
         }
         if (ok && n > 0) {
-            ok = mbar_wait(&o_done[w], 0, wc, 322);
+            ok = mbar_wait(&pv_done[w], static_cast<uint32_t>(n - 1) & 1u, wc, 324);
             ok = __all_sync(0xffffffffu, ok);
         }
         if (ok && n > 0) {
@@ -355,6 +426,19 @@ cr_status launch_d(const CUtensorMap& tm, const AttnParams& p, cudaStream_t st) 
     static unsigned long long attr_done = 0;   // one per template instantiation
     const cr_status sa = ensure_smem_attr(kern, static_cast<int>(Cfg::kSmemBytes), &attr_done);
     if (sa != CR_OK) return sa;
+    // The softmax warpgroups raise their register budget inside the kernel;
+    // that only completes if the launch reserved the 168 registers per thread
+    // the split assumes.  Refuse to launch a build that reserves fewer.
+    static int regs_ok = -1;   // per template instantiation; same answer on every device
+    int ok = __atomic_load_n(&regs_ok, __ATOMIC_ACQUIRE);
+    if (ok < 0) {
+        cudaFuncAttributes fa;
+        const cr_status sf = cuda_check(cudaFuncGetAttributes(&fa, kern));
+        if (sf != CR_OK) return sf;
+        ok = (fa.numRegs >= static_cast<int>(kRegsLaunch) && fa.maxThreadsPerBlock >= kThreads) ? 1 : 0;
+        __atomic_store_n(&regs_ok, ok, __ATOMIC_RELEASE);
+    }
+    if (!ok) return CR_ERR_UNSUPPORTED;
     const int grid = p.n_items * p.n_heads;
     kern<<<grid, kThreads, Cfg::kSmemBytes, st>>>(tm, p);
     return cuda_check(cudaGetLastError());

@@ -184,8 +184,8 @@ __global__ void __launch_bounds__(192, 1)
                 const float* bs = p.b_seg + seg * p.d_seg;
                 if (row < p.M) {
                     uint32_t w[8];
-#pragma unroll
                     const int dm = p.d_seg - 1;   // d_seg is 8 or 16; columns >= d_seg are dropped
+#pragma unroll
                     for (int i = 0; i < 8; ++i)
                         w[i] = pack_bf16x2(v[2 * i] + __ldg(bs + ((2 * i) & dm)),
                                            v[2 * i + 1] + __ldg(bs + ((2 * i + 1) & dm)));
