@@ -8,7 +8,8 @@
 //               slice by bulk copy and, for in-place epilogues, the output tile
 //               itself (the stale cache tile, or the fp32 residual-stream tile)
 //               by TMA, as soon as the epilogue has released its slot.
-//   warp 1      allocates TMEM; one elected lane issues tcgen05.mma
+//   warp 1      allocates TMEM; one elected lane of the converged warp issues
+//               tcgen05.mma
 //               (M = 128, N = BN, K = 16) into a double-buffered fp32
 //               accumulator (2 x BN TMEM columns) and commits to mbarriers.
 //   warp 7      TMA store issuer for the staged output.
@@ -224,38 +225,45 @@ __global__ void __launch_bounds__(256, 1)
     // the epilogue consumes a per-tile load (vectors and/or the in-place tile)
     const bool epi_load = Cfg::kInPlace || has_bias;
 
+    // The producer, loader, store and MMA roles each run as a converged warp
+    // (operands stay warp-uniform); one elected lane issues the copies and MMAs.
     if (warp == 0) {
-        if (lane == 0) {
-            // ------------------------------------------------ TMA producer
+        // ---------------------------------------------------- TMA producer
+        if (elect_one()) {
             tma_prefetch(&tmA);
             tma_prefetch(&tmB);
             if constexpr (Cfg::kInPlace) tma_prefetch(&tmC);
-            uint32_t stage = 0, phase = 0;
-            bool ok = true;
-            for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
-                const int m0 = (t % p.num_m) * BM;
-                const int n0 = (t / p.num_m) * BN;
-                for (int kb = 0; kb < num_k; ++kb) {
-                    if (!(ok = mbar_wait(&empty[stage], phase ^ 1u, wc, 102))) break;
-                    uint8_t* sa = smem + stage * Cfg::kStageBytes;
+        }
+        __syncwarp();
+        uint32_t stage = 0, phase = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+            const int m0 = (t % p.num_m) * BM;
+            const int n0 = (t / p.num_m) * BN;
+            for (int kb = 0; kb < num_k; ++kb) {
+                if (!(ok = mbar_wait_warp(&empty[stage], phase ^ 1u, wc, 102))) break;
+                uint8_t* sa = smem + stage * Cfg::kStageBytes;
+                if (elect_one()) {
                     mbar_expect_tx(&full[stage], Cfg::kStageBytes);
                     tma_load_2d(sa, &tmA, &full[stage], kb * BK, m0);
                     tma_load_2d(sa + A_BYTES, &tmB, &full[stage], kb * BK, n0);
-                    if (++stage == STAGES) {
-                        stage = 0;
-                        phase ^= 1u;
-                    }
                 }
-            }
-            if (!ok) {  // let copies already in flight land before the CTA exits
-                const uint64_t t0 = globaltimer();
-                while (globaltimer() - t0 < 50000ull) {
+                __syncwarp();
+                if (++stage == STAGES) {
+                    stage = 0;
+                    phase ^= 1u;
                 }
             }
         }
+        if (!ok) {  // let copies already in flight land before the CTA exits
+            const uint64_t t0 = globaltimer();
+            while (globaltimer() - t0 < 50000ull) {
+            }
+        }
     } else if (warp == 6) {
-        if (lane == 0 && epi_load) {
-            tma_prefetch(&tmC);
+        if (epi_load) {
+            if (elect_one()) tma_prefetch(&tmC);
+            __syncwarp();
             // ------------------------------------------------ epilogue-input loader:
             // per tile, the bias (and sigma) slice by bulk copy and, for in-place
             // epilogues, the output tile by TMA, as soon as the epilogue has
@@ -265,18 +273,22 @@ __global__ void __launch_bounds__(256, 1)
             for (int t = blockIdx.x; t < total; t += gridDim.x, ++i) {
                 const int m0 = (t % p.num_m) * BM;
                 const int n0 = (t / p.num_m) * BN;
-                if (!(ok = mbar_wait(epi_empty, (static_cast<uint32_t>(i) & 1u) ^ 1u, wc, 101))) break;
+                if (!(ok = mbar_wait_warp(epi_empty, (static_cast<uint32_t>(i) & 1u) ^ 1u, wc, 101)))
+                    break;
                 const int nb = min(BN, p.N - n0);
                 const uint32_t vbytes = static_cast<uint32_t>(nb) * 4u;
                 uint32_t bytes = (Cfg::kInPlace ? Cfg::kTileBytes : 0u) + (has_bias ? vbytes : 0u);
                 if constexpr (Cfg::kKV) bytes += vbytes;
-                mbar_expect_tx(epi_full, bytes);
-                if constexpr (Cfg::kInPlace) {
-                    for (int b = 0; b < Cfg::kBoxes; ++b)
-                        tma_load_2d(tile + b * 16384, &tmC, epi_full, n0 + b * Cfg::kBoxCols, m0);
+                if (elect_one()) {
+                    mbar_expect_tx(epi_full, bytes);
+                    if constexpr (Cfg::kInPlace) {
+                        for (int b = 0; b < Cfg::kBoxes; ++b)
+                            tma_load_2d(tile + b * 16384, &tmC, epi_full, n0 + b * Cfg::kBoxCols, m0);
+                    }
+                    if (has_bias) bulk_load(vec, p.bias + n0, vbytes, epi_full);
+                    if constexpr (Cfg::kKV) bulk_load(vec + BN, p.sigma + n0, vbytes, epi_full);
                 }
-                if (has_bias) bulk_load(vec, p.bias + n0, vbytes, epi_full);
-                if constexpr (Cfg::kKV) bulk_load(vec + BN, p.sigma + n0, vbytes, epi_full);
+                __syncwarp();
             }
             if (!ok) {
                 const uint64_t t0 = globaltimer();
@@ -285,73 +297,85 @@ __global__ void __launch_bounds__(256, 1)
             }
         }
     } else if (warp == 7) {
-        if (lane == 0) {
-            // ------------------------------------------------ TMA store issuer:
-            // writes each staged buffer back once the 128 epilogue threads have
-            // filled it, and hands the buffer (or the in-place tile and the
-            // bias slice) back when TMA has read it
-            bool ok = true;
-            uint32_t pk = 0;   // staged parts so far
-            for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
-                const int m0 = (t % p.num_m) * BM;
-                const int n0 = (t / p.num_m) * BN;
-                if constexpr (Cfg::kInPlace) {
-                    if (!(ok = mbar_wait(&epi_done[0], pk & 1u, wc, 401))) break;
+        // ---------------------------------------------------- TMA store issuer:
+        // writes each staged buffer back once the 128 epilogue threads have
+        // filled it, and hands the buffer (or the in-place tile and the bias
+        // slice) back when TMA has read it.  The bulk-group waits belong to the
+        // elected lane that committed the stores.
+        const bool leader = elect_one();
+        bool ok = true;
+        uint32_t pk = 0;   // staged parts so far
+        for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+            const int m0 = (t % p.num_m) * BM;
+            const int n0 = (t / p.num_m) * BN;
+            if constexpr (Cfg::kInPlace) {
+                if (!(ok = mbar_wait_warp(&epi_done[0], pk & 1u, wc, 401))) break;
+                if (leader) {
                     for (int b = 0; b < Cfg::kBoxes; ++b)
                         tma_store_2d(&tmC, tile + b * 16384, n0 + b * Cfg::kBoxCols, m0);
                     tma_store_commit();
                     tma_store_wait_read0();
                     mbar_arrive(epi_empty);
-                    ++pk;
-                } else {
-                    for (int k = 0; k < Cfg::kBoxes; ++k, ++pk) {
-                        const uint32_t b = pk & 1u;
-                        if (!(ok = mbar_wait(&epi_done[b], (pk >> 1) & 1u, wc, 402))) break;
+                }
+                __syncwarp();
+                ++pk;
+            } else {
+                for (int k = 0; k < Cfg::kBoxes; ++k, ++pk) {
+                    const uint32_t b = pk & 1u;
+                    if (!(ok = mbar_wait_warp(&epi_done[b], (pk >> 1) & 1u, wc, 402))) break;
+                    if (leader) {
                         tma_store_2d(&tmC, tile + b * 16384, n0 + k * Cfg::kBoxCols, m0);
                         tma_store_commit();
                         tma_store_wait_read0();
                         mbar_arrive(&st_free[b]);
                     }
-                    if (ok && epi_load) mbar_arrive(epi_empty);
+                    __syncwarp();
                 }
+                if (ok && epi_load && leader) mbar_arrive(epi_empty);
+                __syncwarp();
             }
-            tma_store_wait0();
         }
+        if (leader) tma_store_wait0();
+        __syncwarp();
     } else if (warp == 1) {
-        if (lane == 0) {
-            // ------------------------------------------------ MMA issuer
-            uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
-            bool ok = true;
-            for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
-                if (!(ok = mbar_wait(&tempty[acc], acc_phase ^ 1u, wc, 201))) break;
+        // ---------------------------------------------------- MMA issuer
+        // Stage descriptors: a K=16 step adds 32 bytes (2 units of 16 B) to the
+        // start address, a stage kStageBytes, the W operand A_BYTES.
+        const uint64_t da0 = smem_desc(smem_u32(smem), 16, 1024, SWZ_128B);
+        constexpr uint64_t kStageStep = Cfg::kStageBytes >> 4;
+        constexpr uint64_t kBStep = A_BYTES >> 4;
+        uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+            if (!(ok = mbar_wait_warp(&tempty[acc], acc_phase ^ 1u, wc, 201))) break;
+            tc_fence_after();
+            const uint32_t d = tmem_base + acc * BN;
+            for (int kb = 0; kb < num_k; ++kb) {
+                if (!(ok = mbar_wait_warp(&full[stage], phase, wc, 202))) break;
                 tc_fence_after();
-                const uint32_t d = tmem_base + acc * BN;
-                for (int kb = 0; kb < num_k; ++kb) {
-                    if (!(ok = mbar_wait(&full[stage], phase, wc, 202))) break;
-                    tc_fence_after();
-                    const uint32_t sa = smem_u32(smem + stage * Cfg::kStageBytes);
-                    const uint32_t sb = sa + A_BYTES;
+                const uint64_t da = da0 + stage * kStageStep;
+                if (elect_one()) {
 #pragma unroll
-                    for (int k = 0; k < BK / 16; ++k) {
-                        const uint64_t da = smem_desc(sa + k * 32, 16, 1024, SWZ_128B);
-                        const uint64_t db = smem_desc(sb + k * 32, 16, 1024, SWZ_128B);
-                        mma_bf16_ss(d, da, db, IDESC, (kb | k) != 0 ? 1u : 0u);
-                    }
+                    for (int k = 0; k < BK / 16; ++k)
+                        mma_bf16_ss(d, da + 2 * k, da + kBStep + 2 * k, IDESC, (kb | k) != 0 ? 1u : 0u);
                     mma_commit(&empty[stage]);
-                    if (++stage == STAGES) {
-                        stage = 0;
-                        phase ^= 1u;
-                    }
                 }
-                if (!ok) break;
-                mma_commit(&tfull[acc]);
-                acc ^= 1u;
-                if (acc == 0) acc_phase ^= 1u;
+                __syncwarp();
+                if (++stage == STAGES) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
             }
-            // all MMAs of this thread retire before TMEM can be released
-            mma_commit(drain);
-            mbar_wait(drain, 0, wc, 203);
+            if (!ok) break;
+            if (elect_one()) mma_commit(&tfull[acc]);
+            __syncwarp();
+            acc ^= 1u;
+            if (acc == 0) acc_phase ^= 1u;
         }
+        // all MMAs of this warp retire before TMEM can be released
+        if (elect_one()) mma_commit(drain);
+        __syncwarp();
+        mbar_wait_warp(drain, 0, wc, 203);
     } else {
         // ---------------------------------------------------- epilogue (warps 2..5)
         const uint32_t quad = warp & 3u;

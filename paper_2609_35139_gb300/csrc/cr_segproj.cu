@@ -87,21 +87,25 @@ __global__ void __launch_bounds__(192, 1)
     const WaitCtx wc{abort_flag, p.status};
     const int total = p.num_m * p.num_g;
 
+    // Producer and MMA issuer run as converged warps; one elected lane issues.
     if (warp == 0) {
-        if (lane == 0) {
+        if (elect_one()) {
             tma_prefetch(&tmKV);
             tma_prefetch(&tmW);
-            uint32_t stage = 0, phase = 0;
-            bool ok = true;
-            for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
-                const int m0 = (t % p.num_m) * 128;
-                const int s0 = (t / p.num_m) * SP_G;
-                const int ns = min(SP_G, p.S - s0);
-                for (int g = 0; g < ns; ++g) {
-                    if (!(ok = mbar_wait(&empty[stage], phase ^ 1u, wc, 111))) break;
-                    uint8_t* sa = smem + stage * Cfg::kStageBytes;
-                    uint8_t* sb = sa + Cfg::kABytes;
-                    const int seg = s0 + g;
+        }
+        __syncwarp();
+        uint32_t stage = 0, phase = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+            const int m0 = (t % p.num_m) * 128;
+            const int s0 = (t / p.num_m) * SP_G;
+            const int ns = min(SP_G, p.S - s0);
+            for (int g = 0; g < ns; ++g) {
+                if (!(ok = mbar_wait_warp(&empty[stage], phase ^ 1u, wc, 111))) break;
+                uint8_t* sa = smem + stage * Cfg::kStageBytes;
+                uint8_t* sb = sa + Cfg::kABytes;
+                const int seg = s0 + g;
+                if (elect_one()) {
                     mbar_expect_tx(&full[stage], Cfg::kStageBytes);
 #pragma unroll
                     for (int b = 0; b < Cfg::kBoxes; ++b) {
@@ -109,57 +113,62 @@ __global__ void __launch_bounds__(192, 1)
                         tma_load_2d(sb + b * (SP_N * 128), &tmW, &full[stage], b * 64,
                                     seg * p.d_seg);
                     }
-                    if (++stage == STAGES) {
-                        stage = 0;
-                        phase ^= 1u;
-                    }
+                }
+                __syncwarp();
+                if (++stage == STAGES) {
+                    stage = 0;
+                    phase ^= 1u;
                 }
             }
-            if (!ok) {
-                const uint64_t t0 = globaltimer();
-                while (globaltimer() - t0 < 50000ull) {
-                }
+        }
+        if (!ok) {
+            const uint64_t t0 = globaltimer();
+            while (globaltimer() - t0 < 50000ull) {
             }
         }
     } else if (warp == 1) {
-        if (lane == 0) {
-            uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
-            bool ok = true;
-            for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
-                const int s0 = (t / p.num_m) * SP_G;
-                const int ns = min(SP_G, p.S - s0);
-                if (!(ok = mbar_wait(&tempty[acc], acc_phase ^ 1u, wc, 211))) break;
+        // a K=16 step adds 32 bytes (2 units of 16 B) to a descriptor's start
+        const uint64_t da0 = smem_desc(smem_u32(smem), 16, 1024, SWZ_128B);
+        constexpr uint64_t kStageStep = Cfg::kStageBytes >> 4;
+        uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+            const int s0 = (t / p.num_m) * SP_G;
+            const int ns = min(SP_G, p.S - s0);
+            if (!(ok = mbar_wait_warp(&tempty[acc], acc_phase ^ 1u, wc, 211))) break;
+            tc_fence_after();
+            for (int g = 0; g < ns; ++g) {
+                if (!(ok = mbar_wait_warp(&full[stage], phase, wc, 212))) break;
                 tc_fence_after();
-                for (int g = 0; g < ns; ++g) {
-                    if (!(ok = mbar_wait(&full[stage], phase, wc, 212))) break;
-                    tc_fence_after();
-                    const uint32_t d = tmem_base + acc * 256 + g * SP_N;
-                    const uint32_t sa = smem_u32(smem + stage * Cfg::kStageBytes);
-                    const uint32_t sb = sa + Cfg::kABytes;
+                const uint32_t d = tmem_base + acc * 256 + g * SP_N;
+                const uint64_t da = da0 + stage * kStageStep;
+                const uint64_t db = da + (Cfg::kABytes >> 4);
+                if (elect_one()) {
 #pragma unroll
                     for (int b = 0; b < Cfg::kBoxes; ++b) {
 #pragma unroll
-                        for (int k = 0; k < 4; ++k) {
-                            const uint64_t da = smem_desc(sa + b * 16384 + k * 32, 16, 1024, SWZ_128B);
-                            const uint64_t db =
-                                smem_desc(sb + b * (SP_N * 128) + k * 32, 16, 1024, SWZ_128B);
-                            mma_bf16_ss(d, da, db, IDESC, (b | k) != 0 ? 1u : 0u);
-                        }
+                        for (int k = 0; k < 4; ++k)
+                            mma_bf16_ss(d, da + b * (16384 >> 4) + 2 * k,
+                                        db + b * ((SP_N * 128) >> 4) + 2 * k, IDESC,
+                                        (b | k) != 0 ? 1u : 0u);
                     }
                     mma_commit(&empty[stage]);
-                    if (++stage == STAGES) {
-                        stage = 0;
-                        phase ^= 1u;
-                    }
                 }
-                if (!ok) break;
-                mma_commit(&tfull[acc]);
-                acc ^= 1u;
-                if (acc == 0) acc_phase ^= 1u;
+                __syncwarp();
+                if (++stage == STAGES) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
             }
-            mma_commit(drain);
-            mbar_wait(drain, 0, wc, 213);
+            if (!ok) break;
+            if (elect_one()) mma_commit(&tfull[acc]);
+            __syncwarp();
+            acc ^= 1u;
+            if (acc == 0) acc_phase ^= 1u;
         }
+        if (elect_one()) mma_commit(drain);
+        __syncwarp();
+        mbar_wait_warp(drain, 0, wc, 213);
     } else {
         const uint32_t quad = warp & 3u;
         const int r = static_cast<int>(quad * 32 + lane);
