@@ -35,7 +35,7 @@ constexpr int BK = 64;
 constexpr uint32_t A_BYTES = BM * BK * 2;
 constexpr uint32_t kSmemLimit = 232448;   // 227 KB opt-in per CTA
 
-template <int BN, int EPI>
+template <int BN, int EPI, int CG>
 struct GemmCfg {
     static constexpr bool kKV = (EPI == EPI_KV_BF16 || EPI == EPI_KV_F32);
     static constexpr bool kInPlace = kKV || EPI == EPI_ADD_F32;   // tile loaded, updated, stored
@@ -46,9 +46,9 @@ struct GemmCfg {
     static constexpr int kBoxes = BN / kBoxCols;                // boxes per tile
     static constexpr uint32_t kTileBytes = kInPlace ? BM * BN * kTileEsize : 2 * 16384;
     static constexpr uint32_t kVecBytes = BN * 4 * (kKV ? 2 : 1);   // bias (+ sigma)
-    static constexpr uint32_t kBBytes = BN * BK * 2;
+    static constexpr uint32_t kBBytes = (BN / CG) * BK * 2;      // this CTA's share of W
     static constexpr uint32_t kStageBytes = A_BYTES + kBBytes;
-    static constexpr uint32_t kFixed = 1024 + kTileBytes + kVecBytes + 256;
+    static constexpr uint32_t kFixed = 1024 + kTileBytes + kVecBytes + 320;
     static constexpr int kStagesFit = static_cast<int>((kSmemLimit - kFixed) / kStageBytes);
     static constexpr int kStages = kStagesFit > 6 ? 6 : kStagesFit;
     static_assert(kStages >= 3, "GEMM tile does not fit in shared memory");
@@ -166,13 +166,13 @@ __device__ __forceinline__ void rotate16(float* a, float* b, float p, const floa
     }
 }
 
-template <int BN, int EPI>
+template <int BN, int EPI, int CG>
 __global__ void __launch_bounds__(256, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const __grid_constant__ CUtensorMap tmC, const __grid_constant__ GemmParams p) {
-    using Cfg = GemmCfg<BN, EPI>;
+    using Cfg = GemmCfg<BN, EPI, CG>;
     constexpr int STAGES = Cfg::kStages;
-    constexpr uint32_t IDESC = idesc_bf16(BM, BN, false, false);
+    constexpr uint32_t IDESC = idesc_bf16(BM * CG, BN, false, false);
 
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -193,6 +193,11 @@ __global__ void __launch_bounds__(256, 1)
     int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
     const uint32_t warp = warp_id(), lane = lane_id();
+    // CTA pairs (CG = 2): cluster c computes 256-row tiles; rank r holds rows
+    // 128 r .. 128 r + 127 of each and half of its W tile.
+    const uint32_t rank = (CG == 2) ? cluster_ctarank() : 0u;
+    const int cta0 = static_cast<int>(blockIdx.x) / CG;   // cluster index
+    const int ncta = static_cast<int>(gridDim.x) / CG;    // clusters
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&full[s], 1);
@@ -200,7 +205,7 @@ __global__ void __launch_bounds__(256, 1)
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(&tfull[s], 1);
-            mbar_init(&tempty[s], 4);
+            mbar_init(&tempty[s], 4 * CG);   // the epilogue warps of every CTA of the tile
         }
         mbar_init(epi_full, 1);
         mbar_init(epi_empty, 1);
@@ -212,9 +217,17 @@ __global__ void __launch_bounds__(256, 1)
         *abort_flag = 0;
         fence_barrier_init();
     }
-    if (warp == 1) tmem_alloc(tmem_slot, Cfg::kTmemCols);
+    if (warp == 1) {
+        if constexpr (CG == 2)
+            tmem_alloc2(tmem_slot, Cfg::kTmemCols);
+        else
+            tmem_alloc(tmem_slot, Cfg::kTmemCols);
+    }
     tc_fence_before();
-    __syncthreads();
+    if constexpr (CG == 2)
+        cluster_sync();   // both CTAs' barriers and TMEM exist before any pair traffic
+    else
+        __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
     const WaitCtx wc{abort_flag, p.status};
@@ -237,16 +250,26 @@ __global__ void __launch_bounds__(256, 1)
         __syncwarp();
         uint32_t stage = 0, phase = 0;
         bool ok = true;
-        for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
-            const int m0 = (t % p.num_m) * BM;
+        for (int t = cta0; t < total && ok; t += ncta) {
+            const int m0 = (t % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
             const int n0 = (t / p.num_m) * BN;
             for (int kb = 0; kb < num_k; ++kb) {
                 if (!(ok = mbar_wait_warp(&empty[stage], phase ^ 1u, wc, 102))) break;
                 uint8_t* sa = smem + stage * Cfg::kStageBytes;
                 if (elect_one()) {
-                    mbar_expect_tx(&full[stage], Cfg::kStageBytes);
-                    tma_load_2d(sa, &tmA, &full[stage], kb * BK, m0);
-                    tma_load_2d(sa + A_BYTES, &tmB, &full[stage], kb * BK, n0);
+                    const int nb0 = n0 + static_cast<int>(rank) * (BN / CG);
+                    if (CG == 1) {
+                        mbar_expect_tx(&full[stage], Cfg::kStageBytes);
+                        tma_load_2d(sa, &tmA, &full[stage], kb * BK, m0);
+                        tma_load_2d(sa + A_BYTES, &tmB, &full[stage], kb * BK, nb0);
+                    } else {
+                        // both CTAs' copies count on the even CTA's barrier, which
+                        // expects the pair's bytes (its own arrive is the only one)
+                        const uint32_t fb = mapa_shared(smem_u32(&full[stage]), 0);
+                        if (rank == 0) mbar_expect_tx(&full[stage], CG * Cfg::kStageBytes);
+                        tma_load_2d_pair(sa, &tmA, fb, kb * BK, m0);
+                        tma_load_2d_pair(sa + A_BYTES, &tmB, fb, kb * BK, nb0);
+                    }
                 }
                 __syncwarp();
                 if (++stage == STAGES) {
@@ -270,8 +293,8 @@ __global__ void __launch_bounds__(256, 1)
             // released the slot (independent of the A/B stream of warp 0)
             bool ok = true;
             int i = 0;
-            for (int t = blockIdx.x; t < total; t += gridDim.x, ++i) {
-                const int m0 = (t % p.num_m) * BM;
+            for (int t = cta0; t < total; t += ncta, ++i) {
+                const int m0 = (t % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
                 const int n0 = (t / p.num_m) * BN;
                 if (!(ok = mbar_wait_warp(epi_empty, (static_cast<uint32_t>(i) & 1u) ^ 1u, wc, 101)))
                     break;
@@ -305,13 +328,14 @@ __global__ void __launch_bounds__(256, 1)
         const bool leader = elect_one();
         bool ok = true;
         uint32_t pk = 0;   // staged parts so far
-        for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
-            const int m0 = (t % p.num_m) * BM;
+        for (int t = cta0; t < total && ok; t += ncta) {
+            const int m0 = (t % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
             const int n0 = (t / p.num_m) * BN;
+            const bool rows_in = m0 < p.M;   // a pair tile's second half may lie below M
             if constexpr (Cfg::kInPlace) {
                 if (!(ok = mbar_wait_warp(&epi_done[0], pk & 1u, wc, 401))) break;
                 if (leader) {
-                    for (int b = 0; b < Cfg::kBoxes; ++b)
+                    for (int b = 0; b < Cfg::kBoxes && rows_in; ++b)
                         tma_store_2d(&tmC, tile + b * 16384, n0 + b * Cfg::kBoxCols, m0);
                     tma_store_commit();
                     tma_store_wait_read0();
@@ -324,7 +348,7 @@ __global__ void __launch_bounds__(256, 1)
                     const uint32_t b = pk & 1u;
                     if (!(ok = mbar_wait_warp(&epi_done[b], (pk >> 1) & 1u, wc, 402))) break;
                     if (leader) {
-                        tma_store_2d(&tmC, tile + b * 16384, n0 + k * Cfg::kBoxCols, m0);
+                        if (rows_in) tma_store_2d(&tmC, tile + b * 16384, n0 + k * Cfg::kBoxCols, m0);
                         tma_store_commit();
                         tma_store_wait_read0();
                         mbar_arrive(&st_free[b]);
@@ -337,8 +361,10 @@ __global__ void __launch_bounds__(256, 1)
         }
         if (leader) tma_store_wait0();
         __syncwarp();
-    } else if (warp == 1) {
+    } else if (warp == 1 && (CG == 1 || rank == 0)) {
         // ---------------------------------------------------- MMA issuer
+        // (for a pair: the even CTA, issuing M = 256 MMAs over both CTAs'
+        // shared memory and TMEM, committing to the barriers of both)
         // Stage descriptors: a K=16 step adds 32 bytes (2 units of 16 B) to the
         // start address, a stage kStageBytes, the W operand A_BYTES.
         const uint64_t da0 = smem_desc(smem_u32(smem), 16, 1024, SWZ_128B);
@@ -346,7 +372,7 @@ __global__ void __launch_bounds__(256, 1)
         constexpr uint64_t kBStep = A_BYTES >> 4;
         uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
         bool ok = true;
-        for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+        for (int t = cta0; t < total && ok; t += ncta) {
             if (!(ok = mbar_wait_warp(&tempty[acc], acc_phase ^ 1u, wc, 201))) break;
             tc_fence_after();
             const uint32_t d = tmem_base + acc * BN;
@@ -356,9 +382,16 @@ __global__ void __launch_bounds__(256, 1)
                 const uint64_t da = da0 + stage * kStageStep;
                 if (elect_one()) {
 #pragma unroll
-                    for (int k = 0; k < BK / 16; ++k)
-                        mma_bf16_ss(d, da + 2 * k, da + kBStep + 2 * k, IDESC, (kb | k) != 0 ? 1u : 0u);
-                    mma_commit(&empty[stage]);
+                    for (int k = 0; k < BK / 16; ++k) {
+                        if constexpr (CG == 2)
+                            mma_bf16_ss2(d, da + 2 * k, da + kBStep + 2 * k, IDESC, (kb | k) != 0 ? 1u : 0u);
+                        else
+                            mma_bf16_ss(d, da + 2 * k, da + kBStep + 2 * k, IDESC, (kb | k) != 0 ? 1u : 0u);
+                    }
+                    if constexpr (CG == 2)
+                        mma_commit2_mc(&empty[stage], 0x3);
+                    else
+                        mma_commit(&empty[stage]);
                 }
                 __syncwarp();
                 if (++stage == STAGES) {
@@ -367,15 +400,27 @@ __global__ void __launch_bounds__(256, 1)
                 }
             }
             if (!ok) break;
-            if (elect_one()) mma_commit(&tfull[acc]);
+            if (elect_one()) {
+                if constexpr (CG == 2)
+                    mma_commit2_mc(&tfull[acc], 0x3);
+                else
+                    mma_commit(&tfull[acc]);
+            }
             __syncwarp();
             acc ^= 1u;
             if (acc == 0) acc_phase ^= 1u;
         }
         // all MMAs of this warp retire before TMEM can be released
-        if (elect_one()) mma_commit(drain);
+        if (elect_one()) {
+            if constexpr (CG == 2)
+                mma_commit2(drain);
+            else
+                mma_commit(drain);
+        }
         __syncwarp();
         mbar_wait_warp(drain, 0, wc, 203);
+    } else if (warp == 1) {
+        // pair: the odd CTA's MMA warp only took part in the TMEM allocation
     } else {
         // ---------------------------------------------------- epilogue (warps 2..5)
         const uint32_t quad = warp & 3u;
@@ -383,11 +428,18 @@ __global__ void __launch_bounds__(256, 1)
         constexpr int ES = Cfg::kTileEsize;
         const float* vb = vec;             // bias slice of the tile
         const float* vs = vec + BN;        // sigma_delta slice (KV epilogues)
+        // hand the accumulator buffer back to the issuing CTA's MMA warp
+        auto release_acc = [&](uint64_t* bar) {
+            if (CG == 2 && rank != 0)
+                mbar_arrive_cluster(mapa_shared(smem_u32(bar), 0));
+            else
+                mbar_arrive(bar);
+        };
         uint32_t acc = 0, acc_phase = 0, pk = 0;
         bool ok = true;
         int i = 0;
-        for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++i) {
-            const int m0 = (t % p.num_m) * BM;
+        for (int t = cta0; t < total && ok; t += ncta, ++i) {
+            const int m0 = (t % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
             const int n0 = (t / p.num_m) * BN;
             ok = mbar_wait(&tfull[acc], acc_phase, wc, 301);
             if (epi_load) ok = ok && mbar_wait(epi_full, static_cast<uint32_t>(i) & 1u, wc, 302);
@@ -463,7 +515,7 @@ __global__ void __launch_bounds__(256, 1)
                 }
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&tempty[acc]);
+                if (lane == 0) release_acc(&tempty[acc]);
                 fence_async_smem();
                 mbar_arrive(&epi_done[0]);
                 ++pk;
@@ -566,7 +618,7 @@ __global__ void __launch_bounds__(256, 1)
                         // TMEM buffer fully read
                         tc_fence_before();
                         __syncwarp();
-                        if (lane == 0) mbar_arrive(&tempty[acc]);
+                        if (lane == 0) release_acc(&tempty[acc]);
                     }
                     fence_async_smem();
                     mbar_arrive(&epi_done[bsel]);
@@ -576,27 +628,65 @@ __global__ void __launch_bounds__(256, 1)
             if (acc == 0) acc_phase ^= 1u;
         }
     }
-    __syncthreads();
+    tc_fence_before();
+    if constexpr (CG == 2)
+        cluster_sync();   // no pair traffic (MMAs, remote arrives) is left in flight
+    else
+        __syncthreads();
     if (warp == 1) {
         __syncwarp();
         tc_fence_after();
-        tmem_dealloc(tmem_base, Cfg::kTmemCols);
+        if constexpr (CG == 2)
+            tmem_dealloc2(tmem_base, Cfg::kTmemCols);
+        else
+            tmem_dealloc(tmem_base, Cfg::kTmemCols);
     }
 }
 
-template <int BN, int EPI>
+template <int BN, int EPI, int CG>
 cr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
                     const GemmParams& p, cudaStream_t st) {
-    using Cfg = GemmCfg<BN, EPI>;
-    auto kern = gemm_kernel<BN, EPI>;
+    using Cfg = GemmCfg<BN, EPI, CG>;
+    auto kern = gemm_kernel<BN, EPI, CG>;
     static unsigned long long attr_done = 0;   // one per template instantiation
     const cr_status sa = ensure_smem_attr(kern, static_cast<int>(Cfg::kSmemBytes), &attr_done);
     if (sa != CR_OK) return sa;
     const int tiles = p.num_m * p.num_n;
-    const int grid = tiles < num_sms() ? tiles : num_sms();
-    kern<<<grid, 256, Cfg::kSmemBytes, st>>>(ta, tb, tc, p);
-    return cuda_check(cudaGetLastError());
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    cfg.blockDim = dim3(256, 1, 1);
+    cfg.dynamicSmemBytes = Cfg::kSmemBytes;
+    cfg.stream = st;
+    if constexpr (CG == 2) {
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = 2;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        // persistent: as many pairs as can be resident at once (asked once)
+        static int max_pairs = 0;
+        int mp = __atomic_load_n(&max_pairs, __ATOMIC_ACQUIRE);
+        if (mp <= 0) {
+            cfg.gridDim = dim3(2 * (num_sms() / 2), 1, 1);
+            int n = 0;
+            if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n <= 0) {
+                (void)cudaGetLastError();
+                n = num_sms() / 2;
+            }
+            mp = n;
+            __atomic_store_n(&max_pairs, mp, __ATOMIC_RELEASE);
+        }
+        cfg.gridDim = dim3(2 * (tiles < mp ? tiles : mp), 1, 1);
+    } else {
+        cfg.gridDim = dim3(tiles < num_sms() ? tiles : num_sms(), 1, 1);
+    }
+    return cuda_check(cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, p));
 }
+
+// Every GEMM runs on CTA pairs: 256-row tiles whose MMAs span two SMs, each
+// SM loading its own 128 rows of A and half of the W tile.
+constexpr int kCG = 2;
 
 }  // namespace
 
@@ -618,13 +708,13 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
     p.M = static_cast<int32_t>(M);
     p.N = static_cast<int32_t>(N);
     p.K = static_cast<int32_t>(K);
-    p.num_m = static_cast<int32_t>((M + BM - 1) / BM);
+    p.num_m = static_cast<int32_t>((M + BM * kCG - 1) / (BM * kCG));
     p.num_n = static_cast<int32_t>((N + BN - 1) / BN);
     CUtensorMap ta, tb, tc;
     if (!make_tmap_2d(&ta, A, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, K, M, lda * 2, BK, BM,
                       CU_TENSOR_MAP_SWIZZLE_128B))
         return CR_ERR_INVALID_ARG;
-    if (!make_tmap_2d(&tb, W, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, K, N, K * 2, BK, BN,
+    if (!make_tmap_2d(&tb, W, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, K, N, K * 2, BK, BN / kCG,
                       CU_TENSOR_MAP_SWIZZLE_128B))
         return CR_ERR_INVALID_ARG;
     // output (staged) tile map: bf16 boxes of 64 or fp32 boxes of 32 columns
@@ -638,22 +728,22 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
         return CR_ERR_INVALID_ARG;
     switch (epi) {
         case EPI_BF16:
-            return BN == 256 ? launch_bn<256, EPI_BF16>(ta, tb, tc, p, st)
-                             : launch_bn<128, EPI_BF16>(ta, tb, tc, p, st);
+            return BN == 256 ? launch_bn<256, EPI_BF16, kCG>(ta, tb, tc, p, st)
+                             : launch_bn<128, EPI_BF16, kCG>(ta, tb, tc, p, st);
         case EPI_GELU_BF16:
-            return BN == 256 ? launch_bn<256, EPI_GELU_BF16>(ta, tb, tc, p, st)
-                             : launch_bn<128, EPI_GELU_BF16>(ta, tb, tc, p, st);
+            return BN == 256 ? launch_bn<256, EPI_GELU_BF16, kCG>(ta, tb, tc, p, st)
+                             : launch_bn<128, EPI_GELU_BF16, kCG>(ta, tb, tc, p, st);
         case EPI_ADD_F32:
-            return launch_bn<128, EPI_ADD_F32>(ta, tb, tc, p, st);
+            return launch_bn<128, EPI_ADD_F32, kCG>(ta, tb, tc, p, st);
         case EPI_F32:
-            return launch_bn<128, EPI_F32>(ta, tb, tc, p, st);
+            return launch_bn<128, EPI_F32, kCG>(ta, tb, tc, p, st);
         case EPI_QKV_ROPE:
-            return BN == 256 ? launch_bn<256, EPI_QKV_ROPE>(ta, tb, tc, p, st)
-                             : launch_bn<128, EPI_QKV_ROPE>(ta, tb, tc, p, st);
+            return BN == 256 ? launch_bn<256, EPI_QKV_ROPE, kCG>(ta, tb, tc, p, st)
+                             : launch_bn<128, EPI_QKV_ROPE, kCG>(ta, tb, tc, p, st);
         case EPI_KV_BF16:
-            return launch_bn<256, EPI_KV_BF16>(ta, tb, tc, p, st);
+            return launch_bn<256, EPI_KV_BF16, kCG>(ta, tb, tc, p, st);
         case EPI_KV_F32:
-            return launch_bn<128, EPI_KV_F32>(ta, tb, tc, p, st);
+            return launch_bn<128, EPI_KV_F32, kCG>(ta, tb, tc, p, st);
         default:
             return CR_ERR_INVALID_ARG;
     }
