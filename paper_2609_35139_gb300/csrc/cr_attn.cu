@@ -68,6 +68,11 @@ constexpr uint32_t kRegsSoftmax = 216;
 static_assert(kRegsCtl * 128 + 2 * kRegsSoftmax * 128 <= kRegsLaunch * kThreads,
               "register split exceeds the launch allocation");
 constexpr float kRescaleLog2 = 8.0f;   // lazy-rescale threshold (log2 units)
+// Warp q of softmax group 0 and warp q of group 1 share an SM sub-partition
+// (warps 4 + q and 8 + q) and take turns on the exponentials: while one runs
+// its exp pass, the other waits for its S and PV MMAs, loads S and takes the
+// row max, so the special-function unit stays busy.
+constexpr bool kTurns = true;
 
 // Two fp32 lanes per instruction (Blackwell packed fp32): d = a * b + c, d = a + b.
 __device__ __forceinline__ void ffma2(float& d0, float& d1, float a0, float a1, float b0, float b1,
@@ -116,10 +121,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* kv_empty = kv_full + NS;
     uint64_t* s_full = kv_empty + NS;     // [2] S_w,j in TMEM
     uint64_t* s_free = s_full + 2;        // [2] S_w,j read into registers
-    uint64_t* p_full = s_free + 2;        // [2] P_w,j in TMEM
-    uint64_t* pv_done = p_full + 2;       // [2] O_w += P_w,j V_j complete
+    uint64_t* p_full = s_free + 2;        // [2][2] half h of P_w,j (64 keys) in TMEM
+    uint64_t* pv_done = p_full + 4;       // [2] O_w += P_w,j V_j complete
     uint64_t* drain = pv_done + 2;        // [2]
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 2);
+    uint64_t* turn = drain + 2;           // [2][4]: warp q of group w finished an exp pass
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(turn + 8);
     int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
     // ---- work item: (request, pair of query tiles, head); heaviest pairs first
@@ -148,10 +154,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int w = 0; w < 2; ++w) {
             mbar_init(&s_full[w], 1);
             mbar_init(&s_free[w], 4);
-            mbar_init(&p_full[w], 4);
+            mbar_init(&p_full[2 * w], 4);
+            mbar_init(&p_full[2 * w + 1], 4);
             mbar_init(&pv_done[w], 1);
             mbar_init(&drain[w], 1);
         }
+        for (int t = 0; t < 8; ++t) mbar_init(&turn[t], 1);
         *abort_flag = 0;
         fence_barrier_init();
     }
@@ -234,22 +242,30 @@ __global__ void __launch_bounds__(kThreads, 1)
                 __syncwarp();
                 return true;
             };
+            // PV in two halves of 64 keys, each issued as soon as softmax w has
+            // written that half of P: the first half's MMAs run while the
+            // second half is being exponentiated.
             auto issue_pv = [&](int j) -> bool {
-                if (!mbar_wait_warp(&p_full[w], static_cast<uint32_t>(j) & 1u, wc, 224)) return false;
-                tc_fence_after();
                 if (!ensure_kv(j)) return false;
                 const uint64_t dv = dv0 + static_cast<uint64_t>(j % NS) * kStageStep;
-                if (elect_one()) {
 #pragma unroll
-                    for (int kk = 0; kk < 8; ++kk) {
-                        // P from TMEM (16 keys = 8 columns); V: rows = keys (the K
-                        // dimension), d contiguous (MN-major); 16 keys = two 8-row atoms.
-                        mma_bf16_ts(dout, pa + kk * 8, dv + kk * ((16 * Cfg::kRowBytes) >> 4), IDESC_PV,
-                                    (j > 0 || kk != 0) ? 1u : 0u);
+                for (int h = 0; h < 2; ++h) {
+                    if (!mbar_wait_warp(&p_full[2 * w + h], static_cast<uint32_t>(j) & 1u, wc, 224))
+                        return false;
+                    tc_fence_after();
+                    if (elect_one()) {
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            // P from TMEM (16 keys = 8 columns); V: rows = keys (the K
+                            // dimension), d contiguous (MN-major); 16 keys = two 8-row atoms.
+                            const int kk = 4 * h + q;
+                            mma_bf16_ts(dout, pa + kk * 8, dv + kk * ((16 * Cfg::kRowBytes) >> 4),
+                                        IDESC_PV, (j > 0 || kk != 0) ? 1u : 0u);
+                        }
+                        if (h == 1) mma_commit(&pv_done[w]);
                     }
-                    mma_commit(&pv_done[w]);
+                    __syncwarp();
                 }
-                __syncwarp();
                 return true;
             };
             bool ok = mbar_wait_warp(q_full, 0, wc, 221);
@@ -360,6 +376,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 m = m_new;
             }
+            if (kTurns && (w == 0 ? (j > 0 && j - 1 < n_kv[1]) : (j < n_kv[0]))) {
+                // group 0 goes first on each key tile
+                const int jt = (w == 0) ? j - 1 : j;
+                ok = mbar_wait(&turn[(1 - w) * 4 + quad], static_cast<uint32_t>(jt) & 1u, wc, 323);
+                if (!__all_sync(0xffffffffu, ok)) {
+                    ok = false;
+                    break;
+                }
+            }
             // P = 2^(s*sc - m) -> bf16 pairs in TMEM, and the row sum
             float rs8[8];
 #pragma unroll
@@ -378,12 +403,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                     pk[i >> 1] = pack_bf16x2(e0, e1);
                 }
                 tmem_st32u(tp + h / 2, pk);
+                // hand this half of P to the MMA issuer
+                tmem_wait_st();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&p_full[2 * w + (h >> 6)]);
+            }
+            if (kTurns) {
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&turn[w * 4 + quad]);
             }
             l += ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
-            tmem_wait_st();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&p_full[w]);
         }
         if (ok && n > 0) {
             ok = mbar_wait(&pv_done[w], static_cast<uint32_t>(n - 1) & 1u, wc, 324);

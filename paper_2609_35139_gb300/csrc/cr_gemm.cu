@@ -53,7 +53,8 @@ struct GemmCfg {
     static constexpr int kStages = kStagesFit > 6 ? 6 : kStagesFit;
     static_assert(kStages >= 3, "GEMM tile does not fit in shared memory");
     static constexpr uint32_t kSmemBytes = kFixed + kStages * kStageBytes;
-    static constexpr uint32_t kTmemCols = 2 * BN;
+    // double-buffered accumulator; TMEM is allocated in powers of two
+    static constexpr uint32_t kTmemCols = (2 * BN <= 256) ? 256u : 512u;
 };
 
 __device__ __forceinline__ float gelu_erf(float x) {
@@ -695,13 +696,38 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
                       cudaStream_t st) {
     const bool kv = (epi == EPI_KV_BF16 || epi == EPI_KV_F32);
     const bool f32_tile = (epi == EPI_KV_F32 || epi == EPI_ADD_F32);
+    // Tile width.  Per 64-deep k-block a CTA of a pair moves 32 KB + 128 BN
+    // bytes through shared memory (TMA writes and MMA operand reads of its A
+    // rows and W half) at ~128 B/clock, and its MMAs take 2 BN clocks, so a
+    // tile costs ~(256 + BN) clocks per k-block for BN <= 256; a launch takes
+    // ceil(tiles / pairs) rounds.  Pick the instantiated width with the least
+    // rounds x (256 + BN) (ties: the wider tile).  The width does not change
+    // any output element's K order, so results do not depend on it.
     int BN;
-    if (f32_tile || epi == EPI_F32)
+    if (kv) {
+        BN = (epi == EPI_KV_BF16) ? 256 : 128;
+    } else if (epi == EPI_F32) {
         BN = 128;
-    else if (kv)
-        BN = 256;
-    else
-        BN = (N >= 2048) ? 256 : 128;
+    } else {
+        const int64_t pairs = num_sms() / kCG > 0 ? num_sms() / kCG : 1;
+        const int64_t mt = (M + BM * kCG - 1) / (BM * kCG);
+        static const int kF32W[] = {160, 128};
+        static const int kBf16W[] = {256, 192, 128};
+        const int* cand = f32_tile ? kF32W : kBf16W;
+        const int nc = f32_tile ? 2 : 3;
+        BN = cand[0];
+        int64_t best = -1;
+        for (int i = 0; i < nc; ++i) {
+            const int w = cand[i];
+            if (epi == EPI_QKV_ROPE && (p.rope_dim <= 0 || w % p.rope_dim != 0)) continue;
+            const int64_t tiles = mt * ((N + w - 1) / w);
+            const int64_t cost = ((tiles + pairs - 1) / pairs) * (256 + w);
+            if (best < 0 || cost < best) {
+                best = cost;
+                BN = w;
+            }
+        }
+    }
     if (kv && (N % BN) != 0) return CR_ERR_UNSUPPORTED;
     if (epi == EPI_QKV_ROPE && (BN % p.rope_dim) != 0) return CR_ERR_UNSUPPORTED;
     if (p.bias && (N % 4) != 0) return CR_ERR_UNSUPPORTED;   // bias slices are 16-byte bulk copies
@@ -728,18 +754,22 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
         return CR_ERR_INVALID_ARG;
     switch (epi) {
         case EPI_BF16:
-            return BN == 256 ? launch_bn<256, EPI_BF16, kCG>(ta, tb, tc, p, st)
-                             : launch_bn<128, EPI_BF16, kCG>(ta, tb, tc, p, st);
+            return BN == 256   ? launch_bn<256, EPI_BF16, kCG>(ta, tb, tc, p, st)
+                   : BN == 192 ? launch_bn<192, EPI_BF16, kCG>(ta, tb, tc, p, st)
+                               : launch_bn<128, EPI_BF16, kCG>(ta, tb, tc, p, st);
         case EPI_GELU_BF16:
-            return BN == 256 ? launch_bn<256, EPI_GELU_BF16, kCG>(ta, tb, tc, p, st)
-                             : launch_bn<128, EPI_GELU_BF16, kCG>(ta, tb, tc, p, st);
+            return BN == 256   ? launch_bn<256, EPI_GELU_BF16, kCG>(ta, tb, tc, p, st)
+                   : BN == 192 ? launch_bn<192, EPI_GELU_BF16, kCG>(ta, tb, tc, p, st)
+                               : launch_bn<128, EPI_GELU_BF16, kCG>(ta, tb, tc, p, st);
         case EPI_ADD_F32:
-            return launch_bn<128, EPI_ADD_F32, kCG>(ta, tb, tc, p, st);
+            return BN == 160 ? launch_bn<160, EPI_ADD_F32, kCG>(ta, tb, tc, p, st)
+                             : launch_bn<128, EPI_ADD_F32, kCG>(ta, tb, tc, p, st);
         case EPI_F32:
             return launch_bn<128, EPI_F32, kCG>(ta, tb, tc, p, st);
         case EPI_QKV_ROPE:
-            return BN == 256 ? launch_bn<256, EPI_QKV_ROPE, kCG>(ta, tb, tc, p, st)
-                             : launch_bn<128, EPI_QKV_ROPE, kCG>(ta, tb, tc, p, st);
+            return BN == 256   ? launch_bn<256, EPI_QKV_ROPE, kCG>(ta, tb, tc, p, st)
+                   : BN == 192 ? launch_bn<192, EPI_QKV_ROPE, kCG>(ta, tb, tc, p, st)
+                               : launch_bn<128, EPI_QKV_ROPE, kCG>(ta, tb, tc, p, st);
         case EPI_KV_BF16:
             return launch_bn<256, EPI_KV_BF16, kCG>(ta, tb, tc, p, st);
         case EPI_KV_F32:

@@ -27,8 +27,11 @@ def _bf16(g, shape, scale=1.0):
     return F.f32_to_bf16((g.standard_normal(shape) * scale).astype(np.float32))
 
 
+# the last two shapes make the launcher pick 160-wide (fp32 residual add) and
+# 192-wide (bf16, GELU) tiles with a ragged last column tile
 @pytest.mark.parametrize("M,N,K", [(128, 128, 64), (300, 256, 200), (77, 3072, 1024),
-                                   (513, 1024, 4096), (40, 48, 8), (1000, 512, 8192)])
+                                   (513, 1024, 4096), (40, 48, 8), (1000, 512, 8192),
+                                   (5120, 1008, 320), (5120, 528, 640)])
 @pytest.mark.parametrize("epi", [cr.CR_EPI_BF16, cr.CR_EPI_GELU_BF16, cr.CR_EPI_ADD_F32, cr.CR_EPI_F32])
 def test_linear(M, N, K, epi):
     g = np.random.default_rng(M * 7 + N + K + epi)
