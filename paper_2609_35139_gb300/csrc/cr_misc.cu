@@ -78,16 +78,30 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const float* x,
     const int64_t row = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
     if (row >= M) return;
-    float4 v[VPL];
+    // every load of the row (x, the reinjection term, gamma, beta) is issued
+    // before the first use: one memory round trip per row
+    float4 v[VPL], gg[VPL], bq[VPL];
+    uint2 av[VPL];
     const float4* xr = reinterpret_cast<const float4*>(x + row * D);
+    const float4* g4 = reinterpret_cast<const float4*>(g);
+    const float4* b4 = reinterpret_cast<const float4*>(b);
 #pragma unroll
     for (int k = 0; k < VPL; ++k) v[k] = xr[lane + 32 * k];
     if (add) {
         const uint2* ar = reinterpret_cast<const uint2*>(add + row * ld_add);
+#pragma unroll
+        for (int k = 0; k < VPL; ++k) av[k] = ar[lane + 32 * k];
+    }
+#pragma unroll
+    for (int k = 0; k < VPL; ++k) {
+        gg[k] = __ldg(g4 + lane + 32 * k);
+        bq[k] = __ldg(b4 + lane + 32 * k);
+    }
+    if (add) {
         float4* xo = reinterpret_cast<float4*>(x_out + row * D);
 #pragma unroll
         for (int k = 0; k < VPL; ++k) {
-            const uint2 a = ar[lane + 32 * k];
+            const uint2 a = av[k];
             v[k].x += bf16_lo(a.x);
             v[k].y += bf16_hi(a.x);
             v[k].z += bf16_lo(a.y);
@@ -110,16 +124,14 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const float* x,
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
     const float rstd = rsqrtf(q * (1.0f / D) + eps);
-    const float4* g4 = reinterpret_cast<const float4*>(g);
-    const float4* b4 = reinterpret_cast<const float4*>(b);
     uint2* ur = reinterpret_cast<uint2*>(u + row * D);
 #pragma unroll
     for (int k = 0; k < VPL; ++k) {
-        const float4 gg = __ldg(g4 + lane + 32 * k);
-        const float4 bq = __ldg(b4 + lane + 32 * k);
         uint2 w;
-        w.x = pack_bf16x2((v[k].x - mean) * rstd * gg.x + bq.x, (v[k].y - mean) * rstd * gg.y + bq.y);
-        w.y = pack_bf16x2((v[k].z - mean) * rstd * gg.z + bq.z, (v[k].w - mean) * rstd * gg.w + bq.w);
+        w.x = pack_bf16x2((v[k].x - mean) * rstd * gg[k].x + bq[k].x,
+                          (v[k].y - mean) * rstd * gg[k].y + bq[k].y);
+        w.y = pack_bf16x2((v[k].z - mean) * rstd * gg[k].z + bq[k].z,
+                          (v[k].w - mean) * rstd * gg[k].w + bq[k].w);
         ur[lane + 32 * k] = w;
     }
 }

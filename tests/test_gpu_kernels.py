@@ -55,6 +55,29 @@ def test_linear(M, N, K, epi):
         assert_close_bf16(got, ref, 3e-3, f"linear bf16 {M}x{N}x{K}")
 
 
+def test_gelu_epilogue_tails():
+    """GELU of the GEMM epilogue over [-12, 12]: every row's output equals x, so
+    the epilogue sees each bf16 value of the range; compared with the fp64
+    definition x/2 erfc(-x / sqrt 2) (= x/2 (1 + erf(x / sqrt 2)) without the
+    tail cancellation) after one bf16 rounding."""
+    sp = pytest.importorskip("scipy.special")
+    M, K, N = 4096, 16, 16
+    x = F.f32_to_bf16(np.linspace(-12.0, 12.0, M).astype(np.float32))
+    A = np.zeros((M, K), np.uint16)
+    A[:, 0] = x
+    W = np.zeros((N, K), np.uint16)
+    W[:, 0] = F.f32_to_bf16(np.ones(N, np.float32))
+    out = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
+    cr.cr_linear(to_dev(A), to_dev(W), to_dev(np.zeros(N, np.float32)), out, cr.CR_EPI_GELU_BF16)
+    torch.cuda.synchronize()
+    got = as_f64(to_host(out))
+    xf = as_f64(x)
+    ref = (0.5 * xf * sp.erfc(-xf / np.sqrt(2.0)))[:, None] * np.ones((1, N))
+    # one bf16 rounding (half an ulp, 2^-9 relative) plus float32 evaluation error
+    err = np.abs(got - ref)
+    assert np.all(err <= 2.0 ** -8 * np.abs(ref) + 1e-30), float(np.max(err / (np.abs(ref) + 1e-30)))
+
+
 @pytest.mark.parametrize("D", [128, 512, 1024])
 def test_layernorm_with_reinjection_add(D):
     g = np.random.default_rng(D)
