@@ -1,27 +1,28 @@
 // tcgen05 GEMM for every dense linear of the repair path (Sec. 4.1):
 //   C[M, N] = A[M, K] * W[N, K]^T + bias, with a fused epilogue.
 //
-// Design (sm_103a, one CTA per SM, persistent):
-//   warp 0      TMA producer: A and W k-slices (64 wide, 128B swizzle) into a
-//               shared-memory ring, tile after tile without pausing.
-//   warp 6      epilogue-input loader: per tile, the bias (and sigma_delta)
+// Design (sm_103a, persistent; every launch runs on CTA pairs, clusters of two
+// CTAs on two SMs computing 256-row tiles with tcgen05 cta_group::2 MMAs):
+//   warp 0      TMA producer: this CTA's 128 rows of A and half of the W tile,
+//               64-wide k-slices (128B swizzle) into a shared-memory ring; both
+//               CTAs' copies count on the even CTA's full barrier.
+//   warp 1      TMEM owner (both CTAs); in the even CTA one elected lane of the
+//               converged warp issues the M = 256, N = BN, K = 16 MMAs into a
+//               double-buffered fp32 accumulator and multicasts its commits.
+//   warp 2      epilogue-input loader: per tile, the bias (and sigma_delta)
 //               slice by bulk copy and, for in-place epilogues, the output tile
 //               itself (the stale cache tile, or the fp32 residual-stream tile)
 //               by TMA, as soon as the epilogue has released its slot.
-//   warp 1      allocates TMEM; one elected lane of the converged warp issues
-//               tcgen05.mma
-//               (M = 128, N = BN, K = 16) into a double-buffered fp32
-//               accumulator (2 x BN TMEM columns) and commits to mbarriers.
-//   warp 7      TMA store issuer for the staged output.
-//   warps 2..5  epilogue: tcgen05.ld 32 lanes x 16 columns, bias from shared
-//               memory, then one of: bf16, GELU, fp32, RoPE on Q/K (into a
-//               128B-swizzled staging buffer, half a tile at a time), or in
-//               place on the staged tile: residual stream x += acc + b, cache
-//               kv = kv + sigma_delta (acc + b) (+ R_M on K).  Staged data goes
-//               out with TMA stores (coalesced, asynchronous).
-// The epilogue of tile i overlaps the MMAs of tile i+1.  Tiles are walked
-// W-tile-major (all M tiles of one N tile back to back), so a W tile is read
-// from HBM once and reused from L2 while the small A operand stays L2-resident.
+//   warp 3      TMA store issuer for the staged output.
+//   warps 4..11 epilogue, two groups of four warps (one per TMEM lane
+//               quarter) splitting each tile's columns: tcgen05.ld 32 lanes x
+//               16 columns, bias from shared memory, then one of: bf16, GELU,
+//               fp32, RoPE on Q/K (into 128B-swizzled staging buffers, one box
+//               of 128 B-wide columns at a time, double-buffered per group), or
+//               in place on the staged tile: residual stream x += acc + b,
+//               cache kv = kv + sigma_delta (acc + b) (+ R_M on K).  Staged
+//               data goes out with TMA stores (coalesced, asynchronous).
+// Warps 0..3 give registers to the epilogue warpgroups (setmaxnreg).
 #include <cuda_bf16.h>
 
 #include "cr_internal.h"
@@ -34,6 +35,17 @@ constexpr int BM = 128;
 constexpr int BK = 64;
 constexpr uint32_t A_BYTES = BM * BK * 2;
 constexpr uint32_t kSmemLimit = 232448;   // 227 KB opt-in per CTA
+// 12 warps: 0 TMA producer, 1 MMA issuer (TMEM owner), 2 epilogue-input
+// loader, 3 TMA store issuer, 4..11 epilogue in two groups of four warps that
+// split each tile's columns.  The first warpgroup gives registers to the
+// epilogue warpgroups (launch: 65536 / 384 = 168 per thread, checked on the
+// host): 64 * 128 + 2 * 216 * 128 <= 168 * 384.
+constexpr int kGemmThreads = 384;
+constexpr uint32_t kGemmRegsLaunch = 168;
+constexpr uint32_t kGemmRegsCtl = 64;
+constexpr uint32_t kGemmRegsEpi = 216;
+static_assert(kGemmRegsCtl * 128 + 2 * kGemmRegsEpi * 128 <= kGemmRegsLaunch * kGemmThreads,
+              "register split exceeds the launch allocation");
 
 template <int BN, int EPI, int CG>
 struct GemmCfg {
@@ -42,9 +54,13 @@ struct GemmCfg {
     static constexpr int kTileEsize = (EPI == EPI_KV_F32 || EPI == EPI_ADD_F32 || EPI == EPI_F32) ? 4 : 2;
     static constexpr int kBoxCols = 128 / kTileEsize;          // one 128-byte swizzle row
     // in-place epilogues stage the whole [BM x BN] tile; store-only epilogues
-    // stage one 16 KB box (128 rows x 128 B) at a time, double-buffered
+    // stage one 16 KB box (128 rows x 128 B) at a time per epilogue group
+    // (boxes alternate between the two groups), double-buffered where the
+    // epilogue arithmetic is heavy (GELU, RoPE) and single otherwise, which
+    // leaves room for a deeper operand ring
     static constexpr int kBoxes = BN / kBoxCols;                // boxes per tile
-    static constexpr uint32_t kTileBytes = kInPlace ? BM * BN * kTileEsize : 2 * 16384;
+    static constexpr int kGroupBufs = (EPI == EPI_GELU_BF16 || EPI == EPI_QKV_ROPE) ? 2 : 1;
+    static constexpr uint32_t kTileBytes = kInPlace ? BM * BN * kTileEsize : 2 * kGroupBufs * 16384;
     static constexpr uint32_t kVecBytes = BN * 4 * (kKV ? 2 : 1);   // bias (+ sigma)
     static constexpr uint32_t kBBytes = (BN / CG) * BK * 2;      // this CTA's share of W
     static constexpr uint32_t kStageBytes = A_BYTES + kBBytes;
@@ -189,7 +205,7 @@ __device__ __forceinline__ void rotate16(float* a, float* b, float p, const floa
 }
 
 template <int BN, int EPI, int CG>
-__global__ void __launch_bounds__(256, 1)
+__global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const __grid_constant__ CUtensorMap tmC, const __grid_constant__ GemmParams p) {
     using Cfg = GemmCfg<BN, EPI, CG>;
@@ -209,9 +225,9 @@ __global__ void __launch_bounds__(256, 1)
     uint64_t* epi_full = tempty + 2;     // loader -> epilogue: vectors (+ in-place tile) landed
     uint64_t* epi_empty = epi_full + 1;  // epilogue -> loader: vectors / tile free again
     uint64_t* drain = epi_empty + 1;
-    uint64_t* epi_done = drain + 1;      // [2] 128 epilogue threads wrote a staged buffer
-    uint64_t* st_free = epi_done + 2;    // [2] the TMA store has read that buffer
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(st_free + 2);
+    uint64_t* epi_done = drain + 1;      // [group][buffer]: a staged buffer is written
+    uint64_t* st_free = epi_done + 4;    // [group][buffer]: the TMA store has read that buffer
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(st_free + 4);
     int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
     const uint32_t warp = warp_id(), lane = lane_id();
@@ -227,12 +243,14 @@ __global__ void __launch_bounds__(256, 1)
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(&tfull[s], 1);
-            mbar_init(&tempty[s], 4 * CG);   // the epilogue warps of every CTA of the tile
+            mbar_init(&tempty[s], 8 * CG);   // the epilogue warps of every CTA of the tile
         }
         mbar_init(epi_full, 1);
         mbar_init(epi_empty, 1);
-        for (int b = 0; b < 2; ++b) {
-            mbar_init(&epi_done[b], 128);
+        for (int b = 0; b < 4; ++b) {
+            // in-place: one barrier for all 256 epilogue threads; store-only:
+            // one per group and buffer for that group's 128 threads
+            mbar_init(&epi_done[b], Cfg::kInPlace ? 256 : 128);
             mbar_init(&st_free[b], 1);
         }
         mbar_init(drain, 1);
@@ -262,6 +280,8 @@ __global__ void __launch_bounds__(256, 1)
 
     // The producer, loader, store and MMA roles each run as a converged warp
     // (operands stay warp-uniform); one elected lane issues the copies and MMAs.
+    if (warp < 4) {
+    setmaxnreg_dec<kGemmRegsCtl>();
     if (warp == 0) {
         // ---------------------------------------------------- TMA producer
         if (elect_one()) {
@@ -305,7 +325,7 @@ __global__ void __launch_bounds__(256, 1)
             while (globaltimer() - t0 < 50000ull) {
             }
         }
-    } else if (warp == 6) {
+    } else if (warp == 2) {
         if (epi_load) {
             if (elect_one()) tma_prefetch(&tmC);
             __syncwarp();
@@ -341,7 +361,7 @@ __global__ void __launch_bounds__(256, 1)
                 }
             }
         }
-    } else if (warp == 7) {
+    } else if (warp == 3) {
         // ---------------------------------------------------- TMA store issuer:
         // writes each staged buffer back once the 128 epilogue threads have
         // filled it, and hands the buffer (or the in-place tile and the bias
@@ -349,7 +369,8 @@ __global__ void __launch_bounds__(256, 1)
         // elected lane that committed the stores.
         const bool leader = elect_one();
         bool ok = true;
-        uint32_t pk = 0;   // staged parts so far
+        uint32_t pk = 0;               // in-place tiles so far
+        uint32_t pkg[2] = {0u, 0u};    // boxes of each epilogue group so far
         for (int t = cta0; t < total && ok; t += ncta) {
             const int m0 = (t % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
             const int n0 = (t / p.num_m) * BN;
@@ -366,9 +387,12 @@ __global__ void __launch_bounds__(256, 1)
                 __syncwarp();
                 ++pk;
             } else {
-                for (int k = 0; k < Cfg::kBoxes; ++k, ++pk) {
-                    const uint32_t b = pk & 1u;
-                    if (!(ok = mbar_wait_warp(&epi_done[b], (pk >> 1) & 1u, wc, 402))) break;
+                for (int k = 0; k < Cfg::kBoxes; ++k) {
+                    // box k was staged by epilogue group k & 1 in its buffer pkg & 1
+                    constexpr uint32_t GB = Cfg::kGroupBufs;
+                    const int g = k & 1;
+                    const uint32_t b = static_cast<uint32_t>(g) * GB + (pkg[g] % GB);
+                    if (!(ok = mbar_wait_warp(&epi_done[b], (pkg[g] / GB) & 1u, wc, 402))) break;
                     if (leader) {
                         if (rows_in) tma_store_2d(&tmC, tile + b * 16384, n0 + k * Cfg::kBoxCols, m0);
                         tma_store_commit();
@@ -376,6 +400,7 @@ __global__ void __launch_bounds__(256, 1)
                         mbar_arrive(&st_free[b]);
                     }
                     __syncwarp();
+                    ++pkg[g];
                 }
                 if (ok && epi_load && leader) mbar_arrive(epi_empty);
                 __syncwarp();
@@ -443,9 +468,12 @@ __global__ void __launch_bounds__(256, 1)
         mbar_wait_warp(drain, 0, wc, 203);
     } else if (warp == 1) {
         // pair: the odd CTA's MMA warp only took part in the TMEM allocation
+    }
     } else {
-        // ---------------------------------------------------- epilogue (warps 2..5)
-        const uint32_t quad = warp & 3u;
+        setmaxnreg_inc<kGemmRegsEpi>();
+        // ---------------------------------------------------- epilogue (warps 4..11)
+        const uint32_t quad = warp & 3u;                       // TMEM lanes 32 quad ..
+        const int eg = (static_cast<int>(warp) - 4) >> 2;      // column group 0 / 1
         const int r = static_cast<int>(quad * 32 + lane);     // row inside the tile
         constexpr int ES = Cfg::kTileEsize;
         const float* vb = vec;             // bias slice of the tile
@@ -479,7 +507,8 @@ __global__ void __launch_bounds__(256, 1)
                     // R_M pairs (d, d + d_h/2) live inside one d_h-wide segment
                     const int dh = p.rope_dim;
                     const float pr = row_ok ? static_cast<float>(__ldg(p.pos + row)) : 0.0f;
-                    for (int s0 = 0; s0 < BN; s0 += dh) {
+                    // d_h-wide segments alternate between the two groups
+                    for (int s0 = eg * dh; s0 < BN; s0 += 2 * dh) {
                         const int gseg = (n0 + s0) / dh;
                         const bool rot = ((gseg / p.n_kv_heads) & 1) == 0;
                         for (int j = 0; j < dh / 2; j += 16) {
@@ -511,7 +540,8 @@ __global__ void __launch_bounds__(256, 1)
                         }
                     }
                 } else {
-                    for (int c = 0; c < BN; c += 16) {
+                    // 16-column chunks alternate between the two groups
+                    for (int c = eg * 16; c < BN; c += 32) {
                         float a[16], k[16], bv[16];
                         __syncwarp();
                         tmem_ld16(taddr + c, a);
@@ -571,10 +601,13 @@ __global__ void __launch_bounds__(256, 1)
                             if (q < p.rope_dim / 2) sincos_prod(pr, p.inv_freq[q], &sn[q], &cs[q]);
                     }
                 }
-                for (int k = 0; k < Cfg::kBoxes && ok; ++k, ++pk) {
-                    const uint32_t bsel = pk & 1u;
-                    if (pk >= 2) {
-                        ok = mbar_wait(&st_free[bsel], ((pk >> 1) - 1) & 1u, wc, 304);
+                // boxes alternate between the groups; each group cycles its own
+                // kGroupBufs staging buffers (pk counts this group's boxes)
+                for (int k = eg; k < Cfg::kBoxes && ok; k += 2, ++pk) {
+                    constexpr uint32_t GB = Cfg::kGroupBufs;
+                    const uint32_t bsel = static_cast<uint32_t>(eg) * GB + (pk % GB);
+                    if (pk >= GB) {
+                        ok = mbar_wait(&st_free[bsel], ((pk / GB) - 1) & 1u, wc, 304);
                         if (!__all_sync(0xffffffffu, ok)) {
                             ok = false;
                             break;
@@ -636,15 +669,13 @@ __global__ void __launch_bounds__(256, 1)
                             store16_tile<ES>(buf, r, c - c0, v);
                         }
                     }
-                    if (k == Cfg::kBoxes - 1) {
-                        // TMEM buffer fully read
-                        tc_fence_before();
-                        __syncwarp();
-                        if (lane == 0) release_acc(&tempty[acc]);
-                    }
                     fence_async_smem();
                     mbar_arrive(&epi_done[bsel]);
                 }
+                // this group has read its columns of the TMEM buffer
+                tc_fence_before();
+                __syncwarp();
+                if (ok && lane == 0) release_acc(&tempty[acc]);
             }
             acc ^= 1u;
             if (acc == 0) acc_phase ^= 1u;
@@ -674,9 +705,22 @@ cr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensor
     const cr_status sa = ensure_smem_attr(kern, static_cast<int>(Cfg::kSmemBytes), &attr_done);
     if (sa != CR_OK) return sa;
     const int tiles = p.num_m * p.num_n;
+    // the epilogue warpgroups raise their register budget inside the kernel,
+    // which only completes if the launch reserved the 168 per thread assumed
+    static int regs_ok = -1;
+    int rok = __atomic_load_n(&regs_ok, __ATOMIC_ACQUIRE);
+    if (rok < 0) {
+        cudaFuncAttributes fa;
+        const cr_status sf = cuda_check(cudaFuncGetAttributes(&fa, kern));
+        if (sf != CR_OK) return sf;
+        rok = (fa.numRegs >= static_cast<int>(kGemmRegsLaunch) && fa.maxThreadsPerBlock >= kGemmThreads)
+                  ? 1 : 0;
+        __atomic_store_n(&regs_ok, rok, __ATOMIC_RELEASE);
+    }
+    if (!rok) return CR_ERR_UNSUPPORTED;
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
-    cfg.blockDim = dim3(256, 1, 1);
+    cfg.blockDim = dim3(kGemmThreads, 1, 1);
     cfg.dynamicSmemBytes = Cfg::kSmemBytes;
     cfg.stream = st;
     if constexpr (CG == 2) {
