@@ -107,15 +107,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int q0 = (item - p.tile_prefix[req]) * 256;
     const int rs = p.req_start[req];
     const int len = p.req_start[req + 1] - rs;
-    int n_kv[2];
-#pragma unroll
-    for (int w = 0; w < 2; ++w) {
-        const int first = q0 + 128 * w;
-        n_kv[w] = first < len ? (__ldg(p.chunk_end + rs + min(first + 127, len - 1)) + 127) / 128 : 0;
-    }
-    const int n_max = max(n_kv[0], n_kv[1]);
 
     const uint32_t warp = warp_id(), lane = lane_id();
+    pdl_launch_dependents();
     if (threadIdx.x == 0) {
         mbar_init(q_full, 1);
         for (int s = 0; s < NS; ++s) {
@@ -138,6 +132,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    pdl_wait();   // qkv and the chunk map come from earlier kernels
+    int n_kv[2];
+#pragma unroll
+    for (int w = 0; w < 2; ++w) {
+        const int first = q0 + 128 * w;
+        n_kv[w] = first < len ? (__ldg(p.chunk_end + rs + min(first + 127, len - 1)) + 127) / 128 : 0;
+    }
+    const int n_max = max(n_kv[0], n_kv[1]);
     const uint32_t tmem_base = *tmem_slot;
     const WaitCtx wc{abort_flag, p.status};
 
@@ -441,8 +443,7 @@ cr_status launch_d(const CUtensorMap& tm, const AttnParams& p, cudaStream_t st) 
     }
     if (!ok) return CR_ERR_UNSUPPORTED;
     const int grid = p.n_items * p.n_heads;
-    kern<<<grid, kThreads, Cfg::kSmemBytes, st>>>(tm, p);
-    return cuda_check(cudaGetLastError());
+    return launch_pdl(kern, dim3(grid), dim3(kThreads), Cfg::kSmemBytes, st, tm, p);
 }
 
 }  // namespace

@@ -231,6 +231,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
     const uint32_t warp = warp_id(), lane = lane_id();
+    pdl_launch_dependents();
     // CTA pairs (CG = 2): cluster c computes 256-row tiles; rank r holds rows
     // 128 r .. 128 r + 127 of each and half of its W tile.
     const uint32_t rank = (CG == 2) ? cluster_ctarank() : 0u;
@@ -269,6 +270,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     else
         __syncthreads();
     tc_fence_after();
+    pdl_wait();   // operands, the in-place tile and positions come from earlier kernels
     const uint32_t tmem_base = *tmem_slot;
     const WaitCtx wc{abort_flag, p.status};
 
@@ -719,17 +721,20 @@ cr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensor
     }
     if (!rok) return CR_ERR_UNSUPPORTED;
     cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     cfg.blockDim = dim3(kGemmThreads, 1, 1);
     cfg.dynamicSmemBytes = Cfg::kSmemBytes;
     cfg.stream = st;
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // see launch_pdl
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
     if constexpr (CG == 2) {
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = 2;
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
+        attr[1].id = cudaLaunchAttributeClusterDimension;
+        attr[1].val.clusterDim.x = 2;
+        attr[1].val.clusterDim.y = 1;
+        attr[1].val.clusterDim.z = 1;
+        cfg.numAttrs = 2;
         // persistent: as many pairs as can be resident at once (asked once)
         static int max_pairs = 0;
         int mp = __atomic_load_n(&max_pairs, __ATOMIC_ACQUIRE);

@@ -110,6 +110,26 @@ inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 
 // uncaptured call does it, so later calls can be captured into CUDA graphs).
 int current_device_index();
 // `done` must be a static owned by the caller's kernel-specific code (one per kernel).
+// Launch with programmatic dependent launch allowed: the kernel may start (and
+// run its prologue) while the previous kernel in the stream finishes; every
+// kernel of the library executes griddepcontrol.wait before its first global
+// memory access, so it sees all of the previous kernel's writes.
+template <typename... P, typename... A>
+cr_status launch_pdl(void (*kern)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                     A&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cuda_check(cudaLaunchKernelEx(&cfg, kern, static_cast<A&&>(args)...));
+}
+
 template <typename K>
 cr_status ensure_smem_attr(K kern, int bytes, unsigned long long* done) {
     const int d = current_device_index();

@@ -17,6 +17,8 @@ namespace {
 // values plus its d_model embedding values, each copied with 16-byte vectors,
 // four loads in flight per thread before the matching stores.
 __global__ void __launch_bounds__(512) gather_kernel(const __grid_constant__ GatherParams p) {
+    pdl_launch_dependents();
+    pdl_wait();
     for (int64_t t = blockIdx.x; t < p.n_tokens; t += gridDim.x) {
         int lo = 0, hi = p.n_seg - 1;
         while (lo < hi) {
@@ -75,6 +77,8 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const float* x,
                                                         const float* __restrict__ b, float eps,
                                                         int64_t M, uint16_t* __restrict__ u) {
     constexpr int D = VPL * 128;
+    pdl_launch_dependents();
+    pdl_wait();
     const int64_t row = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
     if (row >= M) return;
@@ -137,6 +141,8 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const float* x,
 }
 
 __global__ void to_bf16_kernel(const float* __restrict__ x, int64_t n, uint16_t* __restrict__ y) {
+    pdl_launch_dependents();
+    pdl_wait();
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const __nv_bfloat16 b = __float2bfloat16_rn(x[i]);
@@ -152,6 +158,8 @@ struct InvFreq {
 // product rounding folded back in (same arithmetic as the in-epilogue path).
 __global__ void rope_table_kernel(const int32_t* __restrict__ pos, int64_t n, int half,
                                   const __grid_constant__ InvFreq f, float2* __restrict__ table) {
+    pdl_launch_dependents();
+    pdl_wait();
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n * half;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const int64_t t = i / half;
@@ -172,16 +180,15 @@ cr_status launch_rope_table(const int32_t* pos, int64_t n, int half_dim, const f
     for (int i = 0; i < half_dim; ++i) f.f[i] = inv_freq_host[i];
     int64_t blocks = (n * half_dim + 255) / 256;
     if (blocks > static_cast<int64_t>(num_sms()) * 8) blocks = static_cast<int64_t>(num_sms()) * 8;
-    rope_table_kernel<<<static_cast<int>(blocks), 256, 0, st>>>(pos, n, half_dim, f, table);
-    return cuda_check(cudaGetLastError());
+    return launch_pdl(rope_table_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st, pos, n,
+                      half_dim, f, table);
 }
 
 cr_status launch_gather(const GatherParams& p, cudaStream_t st) {
     if (p.n_tokens <= 0) return CR_OK;
     int64_t grid = static_cast<int64_t>(num_sms()) * 4;
     if (grid > p.n_tokens) grid = p.n_tokens;
-    gather_kernel<<<static_cast<int>(grid), 512, 0, st>>>(p);
-    return cuda_check(cudaGetLastError());
+    return launch_pdl(gather_kernel, dim3(static_cast<unsigned>(grid)), dim3(512), 0, st, p);
 }
 
 cr_status launch_layernorm(const float* x, const uint16_t* add, int64_t ld_add, float* x_out,
@@ -193,8 +200,8 @@ cr_status launch_layernorm(const float* x, const uint16_t* add, int64_t ld_add, 
     switch (D) {
 #define CR_LN_CASE(V)                                                                       \
     case V * 128:                                                                           \
-        layernorm_kernel<V><<<grid, 256, 0, st>>>(x, add, ld_add, x_out, g, b, eps, M, u); \
-        break;
+        return launch_pdl(layernorm_kernel<V>, dim3(grid), dim3(256), 0, st, x, add, ld_add, \
+                          x_out, g, b, eps, M, u);
         CR_LN_CASE(1)
         CR_LN_CASE(2)
         CR_LN_CASE(3)
@@ -207,15 +214,13 @@ cr_status launch_layernorm(const float* x, const uint16_t* add, int64_t ld_add, 
         default:
             return CR_ERR_UNSUPPORTED;
     }
-    return cuda_check(cudaGetLastError());
 }
 
 cr_status launch_to_bf16(const float* x, int64_t n, uint16_t* y, cudaStream_t st) {
     if (n <= 0) return CR_OK;
     int64_t blocks = (n + 255) / 256;
     if (blocks > static_cast<int64_t>(num_sms()) * 16) blocks = static_cast<int64_t>(num_sms()) * 16;
-    to_bf16_kernel<<<static_cast<int>(blocks), 256, 0, st>>>(x, n, y);
-    return cuda_check(cudaGetLastError());
+    return launch_pdl(to_bf16_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st, x, n, y);
 }
 
 }  // namespace cr

@@ -31,6 +31,15 @@ __device__ __forceinline__ uint64_t globaltimer() {
 __device__ __forceinline__ uint32_t warp_id() { return threadIdx.x >> 5; }
 __device__ __forceinline__ uint32_t lane_id() { return threadIdx.x & 31; }
 
+// ----------------------------------------------------------------- dependent launch
+// Let the next kernel of the stream start its prologue (no-op unless it was
+// launched with programmatic serialization), and wait until the previous
+// kernel has completed and its writes are visible (no-op without it).
+__device__ __forceinline__ void pdl_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // ----------------------------------------------------------------- status word
 // status[0]: first error code (CR_DEV_*); status[1]: site; status[2]: block.
 __device__ __forceinline__ void report(unsigned* status, unsigned code, unsigned site) {

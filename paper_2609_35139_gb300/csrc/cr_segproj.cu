@@ -33,6 +33,8 @@ struct SegCfg {
 
 __global__ void fold_sigma_kernel(const uint16_t* __restrict__ w, const float* __restrict__ sigma,
                                   int64_t n, int d_seg, int dh, uint16_t* __restrict__ out) {
+    pdl_launch_dependents();
+    pdl_wait();
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const int64_t d = i % dh;
@@ -66,6 +68,7 @@ __global__ void __launch_bounds__(192, 1)
     int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
     const uint32_t warp = warp_id(), lane = lane_id();
+    pdl_launch_dependents();
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&full[s], 1);
@@ -83,6 +86,7 @@ __global__ void __launch_bounds__(192, 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    pdl_wait();   // the cache and the folded weights come from earlier kernels
     const uint32_t tmem_base = *tmem_slot;
     const WaitCtx wc{abort_flag, p.status};
     const int total = p.num_m * p.num_g;
@@ -228,8 +232,7 @@ cr_status launch_dh(const CUtensorMap& tk, const CUtensorMap& tw, const SegParam
     if (sa != CR_OK) return sa;
     const int items = p.num_m * p.num_g;
     const int grid = items < num_sms() ? items : num_sms();
-    kern<<<grid, 192, Cfg::kSmemBytes, st>>>(tk, tw, p);
-    return cuda_check(cudaGetLastError());
+    return launch_pdl(kern, dim3(grid), dim3(192), Cfg::kSmemBytes, st, tk, tw, p);
 }
 
 }  // namespace
@@ -240,9 +243,8 @@ cr_status launch_fold_sigma(const uint16_t* w_seg, const float* sigma, int S, in
     const int threads = 256;
     int64_t blocks = (n + threads - 1) / threads;
     if (blocks > 4 * 1024) blocks = 4 * 1024;
-    fold_sigma_kernel<<<static_cast<int>(blocks), threads, 0, st>>>(w_seg, sigma, n, d_seg,
-                                                                     head_dim, wfold);
-    return cuda_check(cudaGetLastError());
+    return launch_pdl(fold_sigma_kernel, dim3(static_cast<unsigned>(blocks)), dim3(threads), 0, st,
+                      w_seg, sigma, n, d_seg, head_dim, wfold);
 }
 
 cr_status launch_segproj(const uint16_t* kv, int64_t ld_kv, const uint16_t* wfold, int head_dim,
