@@ -110,3 +110,83 @@ def dims_from(target, repairer):
                          repairer.n_heads, repairer.mlp_hidden, repairer.ln_eps,
                          repairer.rope_theta)
     return t, r
+
+
+class RepairPipeline:
+    """Serving loop that hides host<->device transfers behind the repair.
+
+    Requests arrive as chunk caches in pinned host memory and leave as repaired
+    caches in pinned host memory.  Two slots (each a RepairSession plus a device
+    staging pool) alternate: while one slot repairs request i on the compute
+    stream, request i+1's chunks are copied into the other slot's staging pool
+    on a host-to-device stream and request i-1's repaired cache is copied back
+    on a device-to-host stream.  A slot is reused only after its previous repair
+    has consumed the staging pool and its previous result has been read back,
+    so the per-request time approaches the slower of the link and the repair.
+    This is the copy-stream overlap of the serving integration the paper names
+    as future work (Sec. 6); the paged target-cache write is not part of it.
+
+    Only stream/event plumbing lives here: the copies are cudaMemcpyAsync calls
+    (torch ``copy_``) and every step of the repair runs in the library's kernels.
+    """
+
+    def __init__(self, target: cr.cr_target_dims, rep: cr.cr_repairer_dims,
+                 weights: cr.PackedWeights, max_tokens: int, device="cuda"):
+        self.device = torch.device(device)
+        self.slots = [RepairSession(target, rep, weights, max_tokens, device) for _ in range(2)]
+        dt = _dtype(target.cache_dtype)
+        d_kv = self.slots[0].d_kv
+        self.stage_kv = [torch.empty(max_tokens, d_kv, dtype=dt, device=self.device) for _ in range(2)]
+        self.stage_emb = [torch.empty(max_tokens, target.d_model, dtype=dt, device=self.device)
+                          for _ in range(2)]
+        self.compute = torch.cuda.Stream(self.device)
+        self.h2d = torch.cuda.Stream(self.device)
+        self.d2h = torch.cuda.Stream(self.device)
+        self.ev_h2d = [torch.cuda.Event() for _ in range(2)]
+        self.ev_comp = [torch.cuda.Event() for _ in range(2)]
+        self.ev_d2h = [torch.cuda.Event() for _ in range(2)]
+        self.max_tokens = max_tokens
+        self.n_submitted = 0
+
+    def submit(self, kv_host: torch.Tensor, emb_host: torch.Tensor, chunk_start, chunk_len,
+               out_host: torch.Tensor, inv_freq_target=None, rope_mode=cr.CR_ROPE_NONE):
+        """Queue one request: the chunks ``[chunk_start[k], chunk_start[k] + chunk_len[k])``
+        of the pinned host pool, in document order.  Returns an event that completes
+        when ``out_host[:n_tokens]`` holds the repaired cache (``out_host`` pinned,
+        not reused by the caller before then).  Nothing here waits on the GPU."""
+        starts = np.asarray(chunk_start, np.int64)
+        lens = np.asarray(chunk_len, np.int64)
+        n = int(lens.sum())
+        if n < 1 or n > self.max_tokens:
+            raise ValueError(f"request of {n} tokens: the pipeline holds 1..{self.max_tokens}")
+        s = self.n_submitted % 2
+        sess, skv, semb = self.slots[s], self.stage_kv[s], self.stage_emb[s]
+        dst = np.concatenate([[0], np.cumsum(lens)[:-1]]).astype(np.int64)
+        # this slot's staging pool is free once its previous repair has run
+        self.h2d.wait_event(self.ev_comp[s])
+        with torch.cuda.stream(self.h2d):
+            for a, m, d in zip(starts.tolist(), lens.tolist(), dst.tolist()):
+                skv[d:d + m].copy_(kv_host[a:a + m], non_blocking=True)
+                semb[d:d + m].copy_(emb_host[a:a + m], non_blocking=True)
+            self.ev_h2d[s].record(self.h2d)
+        # the chunks have landed, and the slot's previous result has been read back
+        self.compute.wait_event(self.ev_h2d[s])
+        self.compute.wait_event(self.ev_d2h[s])
+        idx = np.arange(len(lens), dtype=np.int32)
+        cu = np.array([0, len(lens)], np.int32)
+        with torch.cuda.stream(self.compute):
+            sess.repair(skv, semb, dst, lens.astype(np.int32), idx, cu, inv_freq_target, rope_mode,
+                        stream=self.compute)
+            self.ev_comp[s].record(self.compute)
+        self.d2h.wait_event(self.ev_comp[s])
+        with torch.cuda.stream(self.d2h):
+            out_host[:n].copy_(sess.kv[:n], non_blocking=True)
+            self.ev_d2h[s].record(self.d2h)
+        self.n_submitted += 1
+        return self.ev_d2h[s]
+
+    def drain(self):
+        """Make the current stream wait for everything submitted so far."""
+        cur = torch.cuda.current_stream(self.device)
+        for s in range(2):
+            cur.wait_event(self.ev_d2h[s])
