@@ -36,7 +36,7 @@ METRIC = "repaired doc tokens/s and p50 repair latency per request (1 GB300, % r
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="llama8b")
@@ -67,21 +67,41 @@ def workload_desc(case):
 
 
 def sample_clocks(dev_index):
+    """Start nvidia-smi sampling every 50 ms and wait (up to 10 s) for its first
+    sample, so that the timed region that follows is covered."""
     path = tempfile.mktemp(prefix="cr_clocks_", suffix=".csv")
-    q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    q = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
     try:
         f = open(path, "w")
         p = subprocess.Popen(["nvidia-smi", f"--query-gpu={q}", "--format=csv,noheader,nounits",
-                              "-lms", "200", "-i", str(dev_index)], stdout=f,
+                              "-lms", "50", "-i", str(dev_index)], stdout=f,
                              stderr=subprocess.DEVNULL)
-        return p, f, path
     except Exception:
         return None, None, path
+    t0 = time.time()
+    while time.time() - t0 < 10.0:
+        f.flush()
+        if os.path.getsize(path) > 0:
+            break
+        time.sleep(0.05)
+    return p, f, path
 
 
-def stop_clocks(handle):
+def _smi_time(stamp):
+    import datetime
+    for fmt in ("%Y/%m/%d %H:%M:%S.%f", "%Y/%m/%d %H:%M:%S"):
+        try:
+            return datetime.datetime.strptime(stamp, fmt).timestamp()
+        except ValueError:
+            pass
+    return None
+
+
+def stop_clocks(handle, t_begin=None, t_end=None):
+    """Samples taken between t_begin and t_end (host wall clock); all samples if
+    none of them carries a usable timestamp."""
     p, f, path = handle
     if p is None:
         return None
@@ -95,23 +115,29 @@ def stop_clocks(handle):
     with open(path) as fh:
         for line in fh:
             parts = [x.strip() for x in line.split(",")]
-            if len(parts) >= 9 and parts[1].replace(".", "").isdigit():
+            if len(parts) >= 10 and parts[2].replace(".", "").isdigit():
                 rows.append(parts)
     os.unlink(path)
     if not rows:
         return None
-    sm = [float(r[1]) for r in rows]
+    window, in_region = rows, False
+    if t_begin is not None and t_end is not None:
+        inside = [r for r in rows if (lambda ts: ts is not None and t_begin - 0.05 <= ts <= t_end + 0.05)(
+            _smi_time(r[0]))]
+        if inside:
+            window, in_region = inside, True
+    sm = [float(r[2]) for r in window]
     names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-    reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
-    return {"sm_mhz": statistics.median(sm), "sm_max_mhz": float(rows[0][2]),
-            "power_w_max": max(float(r[3]) for r in rows if r[3].replace(".", "").isdigit())
-            if any(r[3].replace(".", "").isdigit() for r in rows) else None,
-            "reasons": reasons, "samples": len(rows)}
+    reasons = sorted({names[i] for r in window for i in range(4) if r[6 + i].lower() == "active"})
+    pw = [float(r[4]) for r in window if r[4].replace(".", "").isdigit()]
+    return {"sm_mhz": statistics.median(sm), "sm_max_mhz": float(window[0][3]),
+            "power_w_max": max(pw) if pw else None, "reasons": reasons, "samples": len(window),
+            "samples_in_timed_region": in_region}
 
 
-def oracle_sample(case, n_chunks):
-    """Run the oracle on the first n_chunks of request 0 (a document prefix); returns
-    (tokens, seconds)."""
+def oracle_sample(case, n_chunks, max_tokens=None):
+    """Run the oracle on the first n_chunks of request 0 (a document prefix), cut to
+    max_tokens tokens if given; returns (tokens, seconds)."""
     import numpy as np
     import oracle as O
     p = case.plan
@@ -124,6 +150,8 @@ def oracle_sample(case, n_chunks):
     kv, emb = np.concatenate(kvs), np.concatenate(embs)
     lens = p.chunk_len[sel]
     cid = np.concatenate([np.full(l, i, np.int32) for i, l in enumerate(lens)])
+    if max_tokens is not None and max_tokens < len(cid):
+        kv, emb, cid = kv[:max_tokens], emb[:max_tokens], cid[:max_tokens]
     pos = np.arange(len(cid), dtype=np.int32)
     t, r = case.target, case.repairer
     t0 = time.perf_counter()
@@ -140,16 +168,19 @@ def run_reference(args):
     import fixtures as F
     case = F.make_case(args.workload)
     n_chunks = 1
+    # each step repairs a prefix of the first chunk, sized so that the K timed
+    # steps take about a minute of host time at any K
+    cap = max(32, min(512, 25600 // max(args.steps, 1)))
     times, toks = [], 0
     for i in range(args.warmup + args.steps):
-        n, s = oracle_sample(case, n_chunks)
+        n, s = oracle_sample(case, n_chunks, cap)
         if i >= args.warmup:
             times.append(s)
             toks = n
     total = sum(times)
     value = toks * len(times) / total
     cores = os.cpu_count()
-    sample = f"first {n_chunks} chunk ({toks} tokens) of the request, full repair incl. head"
+    sample = f"first {toks} tokens of the request's first chunk, full repair incl. head"
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
@@ -238,15 +269,17 @@ def run_ours(args):
     torch.cuda.synchronize()
     clk = sample_clocks(local)
     evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    t_begin = time.time()
     evs[0].record(stream)
     for i in range(args.steps):
         run()
         evs[i + 1].record(stream)
     torch.cuda.synchronize()
+    t_end = time.time()
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
-    clocks = stop_clocks(clk)
+    clocks = stop_clocks(clk, t_begin, t_end)
     per_step = [evs[i].elapsed_time(evs[i + 1]) for i in range(args.steps)]
     total_ms = evs[0].elapsed_time(evs[-1])
     if world > 1:
