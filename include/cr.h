@@ -212,6 +212,35 @@ cr_status cr_apply_residual(const cr_target_dims* target, const cr_repairer_dims
                             void* kv_inout, const int32_t* pos, const float* inv_freq_host,
                             int32_t rope_mode, void* stream);
 
+/*
+ * cr_apply_residual_paged - the same head and residual add, with the repaired
+ * cache written into a paged, layer-major target cache instead of in place:
+ * the KV write of the serving integration the paper leaves to future work
+ * (Sec. 6 and App. I: pipelining H2D transfer, repair and KV writes; the
+ * "KV write" column of the repair-latency table of Sec. 5).  The stale
+ * cache is read once and each repaired row is written once, straight from the
+ * head GEMM's epilogue, so no separate scatter pass runs.
+ *   paged[(2l + kv) * num_slots + slot_mapping[t]][h * d_h + d]
+ *       = round(kv_stale[t][((2l + kv) * H_kv + h) * d_h + d] + sigma_delta * z_t)
+ * (R_M on K as in cr_apply_residual).  The layout is, per layer and K|V, a
+ * [num_slots][H_kv * d_h] array, i.e. [num_blocks][block_size][H_kv][d_h] with
+ * slot = block * block_size + offset, planes ordered (layer 0 K, layer 0 V,
+ * layer 1 K, ...).  Tokens whose slot is negative are not written (e.g. the
+ * tokens after the last complete 16-token block, which the target recomputes
+ * with the query); a slot >= num_slots is recorded as a device index error
+ * and not written.  Slots of the tokens written must be distinct.
+ * yf [N, d_b] bf16; kv_stale [N, D_KV] bf16, read only; pos [N] device int32;
+ * slot_mapping [N] device int64; paged_cache [2 L * num_slots * H_kv * d_h]
+ * bf16, device; inv_freq_host as in cr_apply_residual.
+ * bf16 caches with H_kv * d_h a multiple of 256 only (else CR_ERR_UNSUPPORTED).
+ */
+cr_status cr_apply_residual_paged(const cr_target_dims* target, const cr_repairer_dims* rep,
+                                  const cr_weights* w, const uint16_t* yf, int64_t n_tokens,
+                                  const void* kv_stale, const int32_t* pos,
+                                  const float* inv_freq_host, int32_t rope_mode,
+                                  const int64_t* slot_mapping, void* paged_cache, int64_t num_slots,
+                                  void* stream);
+
 /* Device status word: out[0] = first error (0 none, 1 wait timeout, 2 device
  * index out of range), out[1] = site, out[2] = block.  Synchronises the
  * device.  cr_clear_device_status() resets it to zero. */

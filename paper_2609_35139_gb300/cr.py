@@ -24,8 +24,8 @@ CR_EPI_BF16, CR_EPI_GELU_BF16, CR_EPI_ADD_F32, CR_EPI_F32 = range(4)
 
 EXPORTED = [
     "cr_workspace_bytes", "cr_assemble_stale", "cr_compress_features", "cr_repair_forward",
-    "cr_apply_residual", "cr_get_device_status", "cr_clear_device_status", "cr_status_str",
-    "cr_last_cuda_error",
+    "cr_apply_residual", "cr_apply_residual_paged", "cr_get_device_status",
+    "cr_clear_device_status", "cr_status_str", "cr_last_cuda_error",
     "cr_linear", "cr_layernorm", "cr_chunk_causal_attention", "cr_qkv_rope", "cr_segment_project",
     "cr_segment_project_noalloc",
 ]
@@ -90,6 +90,8 @@ def lib(build_if_missing: bool = False) -> ctypes.CDLL:
                                     vp, vp, vp, i32, i64, vp, vp, c_size_t, vp]),
         "cr_apply_residual": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp, i64,
                                     vp, vp, vp, i32, vp]),
+        "cr_apply_residual_paged": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp,
+                                          i64, vp, vp, vp, i32, vp, vp, i64, vp]),
         "cr_get_device_status": (i32, [P(c_uint32)]),
         "cr_clear_device_status": (i32, []),
         "cr_status_str": (ctypes.c_char_p, [i32]),
@@ -220,6 +222,18 @@ def cr_apply_residual(target, rep, weights: PackedWeights, yf, n_tokens, kv_inou
         ctypes.byref(target), ctypes.byref(rep), ctypes.byref(weights.struct), _p(yf), n_tokens,
         _p(kv_inout), _p(pos), None if f is None else f.ctypes.data, rope_mode, _stream(stream))
     _check("cr_apply_residual", st)
+
+
+def cr_apply_residual_paged(target, rep, weights: PackedWeights, yf, n_tokens, kv_stale, pos,
+                            slot_mapping, paged_cache, num_slots, inv_freq_host=None,
+                            rope_mode=CR_ROPE_NONE, stream=None):
+    """Head + residual add, repaired rows written to paged_cache[(2l+kv)*num_slots + slot]."""
+    f = None if inv_freq_host is None else _host_arr(inv_freq_host, np.float32)
+    st = lib().cr_apply_residual_paged(
+        ctypes.byref(target), ctypes.byref(rep), ctypes.byref(weights.struct), _p(yf), n_tokens,
+        _p(kv_stale), _p(pos), None if f is None else f.ctypes.data, rope_mode, _p(slot_mapping),
+        _p(paged_cache), num_slots, _stream(stream))
+    _check("cr_apply_residual_paged", st)
 
 
 def cr_get_device_status():

@@ -554,6 +554,46 @@ cr_status cr_apply_residual(const cr_target_dims* target, const cr_repairer_dims
                        gp, kv_inout, d.D, static_cast<cudaStream_t>(stream));
 }
 
+cr_status cr_apply_residual_paged(const cr_target_dims* target, const cr_repairer_dims* rep,
+                                  const cr_weights* w, const uint16_t* yf, int64_t n_tokens,
+                                  const void* kv_stale, const int32_t* pos,
+                                  const float* inv_freq_host, int32_t rope_mode,
+                                  const int64_t* slot_mapping, void* paged_cache, int64_t num_slots,
+                                  void* stream) {
+    cr_status s = check_target(target);
+    if (s == CR_OK) s = check_repairer(rep);
+    if (s != CR_OK) return s;
+    const Dims d = dims_of(target, rep);
+    if (!w || n_tokens < 1 || n_tokens > INT32_MAX / 2 || num_slots < 1) return CR_ERR_INVALID_ARG;
+    if (rope_mode != CR_ROPE_NONE && rope_mode != CR_ROPE_GLOBAL) return CR_ERR_INVALID_ARG;
+    if (!all_aligned(yf, kv_stale, pos, slot_mapping, paged_cache, w->w_out, w->b_out,
+                     w->sigma_delta))
+        return CR_ERR_INVALID_ARG;
+    if (rope_mode == CR_ROPE_GLOBAL && !inv_freq_host) return CR_ERR_INVALID_ARG;
+    const int64_t plane = static_cast<int64_t>(d.H) * d.dh;   // one (layer, K|V) row
+    if (d.f32 || plane % 256 != 0 || d.D % 256 != 0) return CR_ERR_UNSUPPORTED;
+    if (num_slots > INT64_MAX / (2 * static_cast<int64_t>(d.L) * plane)) return CR_ERR_INVALID_ARG;
+    unsigned* status = device_status_ptr();
+    if (!status) return CR_ERR_CUDA;
+    GemmParams gp{};
+    gp.status = status;
+    gp.bias = w->b_out;
+    gp.sigma = w->sigma_delta;
+    gp.pos = pos;
+    gp.rope_dim = static_cast<int32_t>(d.dh);
+    gp.rope_on = rope_mode == CR_ROPE_GLOBAL ? 1 : 0;
+    gp.n_kv_heads = static_cast<int32_t>(d.H);
+    if (gp.rope_on)
+        for (int i = 0; i < d.dh / 2; ++i) gp.inv_freq[i] = inv_freq_host[i];
+    gp.slot = slot_mapping;
+    gp.paged = static_cast<uint16_t*>(paged_cache);
+    gp.num_slots = num_slots;
+    gp.seg_width = static_cast<int32_t>(plane);
+    // the stale tile is read through the same tensor map as the in-place update
+    return launch_gemm(yf, d.db, w->w_out, n_tokens, d.D, d.db, EPI_KV_PAGED, gp,
+                       const_cast<void*>(kv_stale), d.D, static_cast<cudaStream_t>(stream));
+}
+
 // ------------------------------------------------------------------ cr_ops.h
 cr_status cr_linear(const uint16_t* A, int64_t lda, const uint16_t* W, const float* bias,
                     int64_t M, int64_t N, int64_t K, void* out, int64_t ldo, int32_t epi,

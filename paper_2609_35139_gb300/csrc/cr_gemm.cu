@@ -49,7 +49,10 @@ static_assert(kGemmRegsCtl * 128 + 2 * kGemmRegsEpi * 128 <= kGemmRegsLaunch * k
 
 template <int BN, int EPI, int CG>
 struct GemmCfg {
-    static constexpr bool kKV = (EPI == EPI_KV_BF16 || EPI == EPI_KV_F32);
+    static constexpr bool kKV = (EPI == EPI_KV_BF16 || EPI == EPI_KV_F32 || EPI == EPI_KV_PAGED);
+    // the stale tile is staged as for the in-place update, but the repaired rows
+    // go straight from registers to the paged target cache (no TMA store)
+    static constexpr bool kPaged = (EPI == EPI_KV_PAGED);
     static constexpr bool kInPlace = kKV || EPI == EPI_ADD_F32;   // tile loaded, updated, stored
     static constexpr int kTileEsize = (EPI == EPI_KV_F32 || EPI == EPI_ADD_F32 || EPI == EPI_F32) ? 4 : 2;
     static constexpr int kBoxCols = 128 / kTileEsize;          // one 128-byte swizzle row
@@ -380,7 +383,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if constexpr (Cfg::kInPlace) {
                 if (!(ok = mbar_wait_warp(&epi_done[0], pk & 1u, wc, 401))) break;
                 if (leader) {
-                    for (int b = 0; b < Cfg::kBoxes && rows_in; ++b)
+                    for (int b = 0; b < Cfg::kBoxes && rows_in && !Cfg::kPaged; ++b)
                         tma_store_2d(&tmC, tile + b * 16384, n0 + b * Cfg::kBoxCols, m0);
                     tma_store_commit();
                     tma_store_wait_read0();
@@ -505,6 +508,27 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             const uint32_t taddr = tmem_base + ((quad * 32u) << 16) + acc * BN;
 
             if constexpr (Cfg::kInPlace) {
+                // where a repaired 16-column chunk goes: back into the staged tile
+                // (stored in place by TMA), or straight to the token's row of its
+                // (layer, K|V) plane in the paged target cache
+                uint16_t* prow = nullptr;
+                if constexpr (Cfg::kPaged) {
+                    const int64_t slot = row_ok ? __ldg(p.slot + row) : -1;
+                    if (slot >= 0 && slot < p.num_slots) {
+                        const int plane = n0 / p.seg_width;
+                        prow = p.paged + (static_cast<int64_t>(plane) * p.num_slots + slot) * p.seg_width +
+                               (n0 - plane * p.seg_width);
+                    } else if (slot >= p.num_slots) {
+                        report(p.status, CR_DEV_INDEX, 410);
+                    }
+                }
+                auto put16 = [&](int col, const float* v) {
+                    if constexpr (Cfg::kPaged) {
+                        if (prow) store16_bf16_global(prow + col, v);
+                    } else {
+                        store16_tile<ES>(tile, r, col, v);
+                    }
+                };
                 if (Cfg::kKV && p.rope_on) {
                     // R_M pairs (d, d + d_h/2) live inside one d_h-wide segment
                     const int dh = p.rope_dim;
@@ -537,8 +561,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                                 kb[q] = fmaf(sb_[q], b[q] + bb[q], kb[q]);
                             }
                             if (rot) rotate16(ka, kb, pr, p.inv_freq, j);
-                            store16_tile<ES>(tile, r, ta, ka);
-                            store16_tile<ES>(tile, r, tb, kb);
+                            put16(ta, ka);
+                            put16(tb, kb);
                         }
                     }
                 } else {
@@ -564,7 +588,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 #pragma unroll
                             for (int q = 0; q < 16; ++q) k[q] += a[q] + bv[q];
                         }
-                        store16_tile<ES>(tile, r, c, k);
+                        put16(c, k);
                     }
                 }
                 tc_fence_before();
@@ -764,7 +788,7 @@ constexpr int kCG = 2;
 cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t M, int64_t N,
                       int64_t K, int epi, GemmParams p, void* kv_base, int64_t ld_kv,
                       cudaStream_t st) {
-    const bool kv = (epi == EPI_KV_BF16 || epi == EPI_KV_F32);
+    const bool kv = (epi == EPI_KV_BF16 || epi == EPI_KV_F32 || epi == EPI_KV_PAGED);
     const bool f32_tile = (epi == EPI_KV_F32 || epi == EPI_ADD_F32);
     // Tile width.  Per 64-deep k-block a CTA of a pair moves 32 KB + 128 BN
     // bytes through shared memory (TMA writes and MMA operand reads of its A
@@ -775,7 +799,7 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
     // any output element's K order, so results do not depend on it.
     int BN;
     if (kv) {
-        BN = (epi == EPI_KV_BF16) ? 256 : 128;
+        BN = (epi == EPI_KV_F32) ? 128 : 256;
     } else if (epi == EPI_F32) {
         BN = 128;
     } else {
@@ -844,6 +868,9 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
             return launch_bn<256, EPI_KV_BF16, kCG>(ta, tb, tc, p, st);
         case EPI_KV_F32:
             return launch_bn<128, EPI_KV_F32, kCG>(ta, tb, tc, p, st);
+        case EPI_KV_PAGED:
+            if (p.seg_width <= 0 || p.seg_width % 256 != 0 || p.num_slots < 1) return CR_ERR_UNSUPPORTED;
+            return launch_bn<256, EPI_KV_PAGED, kCG>(ta, tb, tc, p, st);
         default:
             return CR_ERR_INVALID_ARG;
     }

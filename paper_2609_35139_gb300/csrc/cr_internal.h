@@ -52,7 +52,9 @@ enum GemmEpi : int {
     EPI_F32 = 3,
     EPI_QKV_ROPE = 4,   // bf16 out, repairer RoPE on columns < rope_cols
     EPI_KV_BF16 = 5,    // in-place residual add on a bf16 cache tile (+ global RoPE on K)
-    EPI_KV_F32 = 6      // same for an fp32 cache
+    EPI_KV_F32 = 6,     // same for an fp32 cache
+    EPI_KV_PAGED = 7    // bf16 cache: stale tile read token-major, repaired rows written
+                        // to a paged, layer-major target cache through a slot mapping
 };
 
 struct GemmParams {
@@ -68,6 +70,10 @@ struct GemmParams {
     int32_t n_kv_heads;      // KV: segment s is K iff (s / n_kv_heads) is even
     const float* sigma;      // KV: sigma_delta [N]
     const float2* rope_table;  // QKV: (cos, sin) [M, rope_dim / 2], or null (computed inline)
+    const int64_t* slot;     // KV_PAGED: destination slot of each token, < 0 = not written
+    uint16_t* paged;         // KV_PAGED: [N / seg_width][num_slots][seg_width] bf16
+    int64_t num_slots;       // KV_PAGED: slots per (layer, K|V) plane
+    int32_t seg_width;       // KV_PAGED: H_kv * d_h, the columns of one (layer, K|V) plane
     unsigned* status;
     float inv_freq[64];      // RoPE frequencies, rope_dim / 2 entries
 };

@@ -72,6 +72,14 @@ class RepairSession:
         cr.cr_apply_residual(self.target, self.rep, self.weights, self.yf, a.n_tokens, self.kv,
                              self.pos, inv_freq_target, rope_mode, stream)
 
+    def apply_paged(self, a: Assembled, slot_mapping: torch.Tensor, paged_cache: torch.Tensor,
+                    num_slots: int, inv_freq_target=None, rope_mode=cr.CR_ROPE_NONE, stream=None):
+        """Head and residual add with the repaired rows written to a paged target cache
+        ([2 L, num_slots, H_kv d_h] bf16) at slot_mapping[t] (int64, < 0 = skip); kv stays stale."""
+        cr.cr_apply_residual_paged(self.target, self.rep, self.weights, self.yf, a.n_tokens, self.kv,
+                                   self.pos, slot_mapping, paged_cache, num_slots, inv_freq_target,
+                                   rope_mode, stream)
+
     def repair(self, kv_pool, emb_pool, chunk_start, chunk_len, chunk_idx, cu_chunks,
                inv_freq_target=None, rope_mode=cr.CR_ROPE_NONE, stream=None) -> Assembled:
         """Assemble, compress, run the blocks and apply the residual; kv holds the result."""

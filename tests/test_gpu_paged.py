@@ -1,0 +1,99 @@
+"""cr_apply_residual_paged: the repaired rows written into a paged, layer-major
+target cache equal, bit for bit, the rows cr_apply_residual repairs in place
+(whose values the parity tests pin to the oracle); tokens with a negative slot
+and unused slots are left alone, the stale cache is not modified, and a slot out
+of range is reported on the device and not written (the report makes the
+kernel's other roles stop, as for any device-detected index error)."""
+import numpy as np
+import pytest
+import torch
+
+import fixtures as F
+from paper_2609_35139_gb300 import RepairSession, cr, dims_from, pack_host_weights
+from parity_util import to_dev, to_host
+
+pytestmark = pytest.mark.gpu
+
+SENTINEL = 0x7F7F   # a bf16 bit pattern the repair never produces here (about 3.4e38)
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2609_35139_gb300 import build
+    build.build()
+    cr.lib()
+    cr.cr_clear_device_status()
+    yield
+    st, word = cr.cr_get_device_status()
+    assert st == cr.CR_OK, f"device status {word}"
+
+
+def _prepared(name="small"):
+    case = F.make_case(name)
+    t, r = dims_from(case.target, case.repairer)
+    pw = pack_host_weights(case.weights, case.repairer.n_blocks)
+    kvp, embp = case.pool()
+    p = case.plan
+    sess = RepairSession(t, r, pw, max_tokens=p.n_tokens)
+    a = sess.assemble(to_dev(kvp), to_dev(embp), p.chunk_start, p.chunk_len, p.chunk_idx, p.cu_chunks)
+    sess.compress(a)
+    sess.forward(a)
+    return case, sess, a
+
+
+@pytest.mark.parametrize("rope_mode", [cr.CR_ROPE_NONE, cr.CR_ROPE_GLOBAL])
+def test_paged_write_equals_in_place_repair(rope_mode):
+    case, sess, a = _prepared()
+    n = a.n_tokens
+    tg = case.target
+    plane = tg.n_kv_heads * tg.head_dim
+    planes = 2 * tg.n_layers
+    stale = sess.kv[:n].clone()
+    inv = case.inv_freq_target if rope_mode == cr.CR_ROPE_GLOBAL else None
+
+    # blocks of 16 tokens in a shuffled order with spare blocks; the tail after
+    # the last complete block is not written
+    full = (n // 16) * 16
+    n_blocks = n // 16 + 7
+    order = np.random.default_rng(5).permutation(n_blocks)[: (n + 15) // 16]
+    slots = np.full(n, -1, np.int64)
+    tok = np.arange(full)
+    slots[:full] = order[tok // 16] * 16 + tok % 16
+    num_slots = n_blocks * 16
+    paged = torch.full((planes, num_slots, plane), 0, dtype=torch.int16, device="cuda")
+    paged.fill_(SENTINEL)
+    paged = paged.view(torch.bfloat16)
+    sess.apply_paged(a, to_dev(slots), paged, num_slots, inv, rope_mode)
+
+    # reference: the in-place repair of a copy of the same stale rows
+    ref = stale.clone()
+    cr.cr_apply_residual(sess.target, sess.rep, sess.weights, sess.yf, n, ref, sess.pos, inv, rope_mode)
+    torch.cuda.synchronize()
+    assert torch.equal(sess.kv[:n], stale), "the stale cache must stay untouched"
+    got = to_host(paged).reshape(planes, num_slots, plane)
+    want = to_host(ref).reshape(n, planes, plane)
+    written = np.zeros(num_slots, bool)
+    written[slots[:full]] = True
+    for pl in range(planes):
+        assert np.array_equal(got[pl, slots[:full]], want[:full, pl]), f"plane {pl}"
+        assert np.all(got[pl, ~written] == SENTINEL), f"plane {pl}: a slot not mapped was written"
+
+
+def test_paged_slot_out_of_range_is_reported_and_skipped():
+    case, sess, a = _prepared()
+    n = a.n_tokens
+    tg = case.target
+    plane = tg.n_kv_heads * tg.head_dim
+    num_slots = n
+    slots = np.arange(n, dtype=np.int64)
+    slots[3] = num_slots + 5
+    paged = torch.empty((2 * tg.n_layers, num_slots, plane), dtype=torch.int16, device="cuda")
+    paged.fill_(SENTINEL)
+    sess.apply_paged(a, to_dev(slots), paged.view(torch.bfloat16), num_slots)
+    st, word = cr.cr_get_device_status()
+    cr.cr_clear_device_status()
+    assert st == cr.CR_ERR_DEVICE_INDEX, word
+    got = to_host(paged)
+    assert np.all(got[:, 3] == SENTINEL)            # slot 3 belonged to the bad token only

@@ -116,3 +116,19 @@ def test_other_calls_reject_bad_inputs_on_host(L):
     cu = np.array([0, 100, 90], np.int32)
     assert L.cr_chunk_causal_attention(FAKE, 1024, 16, FAKE, cu.ctypes.data, 2, 90, FAKE,
                                        None) == cr.CR_ERR_INVALID_ARG          # empty request
+
+
+def test_paged_residual_rejects_bad_inputs_on_host(L):
+    c, (t, r) = _dims()
+    w = cr.cr_weights()
+    w.w_out = w.b_out = w.sigma_delta = FAKE
+    call = lambda tt, n=10, slots=64, paged=FAKE: L.cr_apply_residual_paged(
+        ctypes.byref(tt), ctypes.byref(r), ctypes.byref(w), FAKE, n, FAKE, FAKE, None, 0, FAKE, paged,
+        slots, None)
+    assert call(t, slots=0) == cr.CR_ERR_INVALID_ARG          # no slots
+    assert call(t, n=0) == cr.CR_ERR_INVALID_ARG              # no tokens
+    assert call(t, paged=FAKE + 8) == cr.CR_ERR_INVALID_ARG   # misaligned cache
+    f32 = cr.target_dims(4, 2, 128, 512, "f32")
+    assert call(f32) == cr.CR_ERR_UNSUPPORTED                 # bf16 caches only
+    narrow = cr.target_dims(4, 1, 128, 512, "bf16")           # H_kv d_h = 128: not a multiple of 256
+    assert call(narrow) == cr.CR_ERR_UNSUPPORTED
