@@ -6,3 +6,4 @@ product path (``paper_2609_35139_gb300``) never imports it and shares no code
 with it.
 """
 from .cacherepair import *  # noqa: F401,F403
+from .offline import *  # noqa: F401,F403
