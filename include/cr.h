@@ -241,6 +241,44 @@ cr_status cr_apply_residual_paged(const cr_target_dims* target, const cr_repaire
                                   const int64_t* slot_mapping, void* paged_cache, int64_t num_slots,
                                   void* stream);
 
+/* ---------------------------------------------------------------- offline
+ * Preparation that runs once per chunk or once per corpus, not per request.
+ *
+ * cr_canonicalize_chunks - canonical chunk caches (Sec. 4.1, "Chunk-cache
+ * preparation"): each chunk is prefilled alone, and its K is stored without
+ * its local rotary encoding,
+ *     K^c_t = R_M(q_t)^{-1} K_t,   V^c_t = V_t,
+ * q_t the token's position inside its chunk.  In place on kv_inout [N, D_KV]
+ * (cache dtype; only K segments are written), pos [N] device int32 = q_t,
+ * inv_freq_host [head_dim/2] HOST fp32 (the target's R_M frequencies).  Each
+ * rotate-half pair (d, d + d_h/2) of every K segment is rotated by -q_t f_d
+ * and rounded once to the cache dtype.
+ */
+cr_status cr_canonicalize_chunks(const cr_target_dims* target, void* kv_inout, int64_t n_tokens,
+                                 const int32_t* pos, const float* inv_freq_host, void* stream);
+
+/*
+ * sigma statistics (Sec. 4.2, "Normalization and objective"): one RMS per
+ * D_KV coordinate (layer, KV head, K|V, head coordinate) over corpus document
+ * tokens; sigma_stale over stale caches, sigma_Delta over the residual targets
+ * KV_joint^c - KV_stale^c.  Streamed over the corpus:
+ *   cr_sigma_accumulate adds, for every coordinate j, the sum over the call's
+ *     n_tokens rows of a[t][j]^2 (or (a[t][j] - b[t][j])^2 when b is not NULL)
+ *     to sumsq[j] (device fp64 [D_KV], zeroed by the caller before the first
+ *     call); a, b [n_tokens, D_KV] device, cache dtype.  The sum is formed in
+ *     a fixed order (fp32 over 64-token slices, fp64 across slices), so equal
+ *     inputs give equal bits.  workspace: cr_sigma_workspace_bytes(target,
+ *     n_tokens) device bytes, 16-byte aligned.
+ *   cr_sigma_finalize writes sigma_out[j] = sqrt(sumsq[j] / count) (fp32
+ *     [D_KV], device), count = all rows accumulated.
+ */
+size_t cr_sigma_workspace_bytes(const cr_target_dims* target, int64_t n_tokens);
+cr_status cr_sigma_accumulate(const cr_target_dims* target, const void* a, const void* b,
+                              int64_t n_tokens, double* sumsq, void* workspace,
+                              size_t workspace_bytes, void* stream);
+cr_status cr_sigma_finalize(const cr_target_dims* target, const double* sumsq, int64_t count,
+                            float* sigma_out, void* stream);
+
 /* Device status word: out[0] = first error (0 none, 1 wait timeout, 2 device
  * index out of range), out[1] = site, out[2] = block.  Synchronises the
  * device.  cr_clear_device_status() resets it to zero. */

@@ -24,7 +24,8 @@ CR_EPI_BF16, CR_EPI_GELU_BF16, CR_EPI_ADD_F32, CR_EPI_F32 = range(4)
 
 EXPORTED = [
     "cr_workspace_bytes", "cr_assemble_stale", "cr_compress_features", "cr_repair_forward",
-    "cr_apply_residual", "cr_apply_residual_paged", "cr_get_device_status",
+    "cr_apply_residual", "cr_apply_residual_paged", "cr_canonicalize_chunks",
+    "cr_sigma_workspace_bytes", "cr_sigma_accumulate", "cr_sigma_finalize", "cr_get_device_status",
     "cr_clear_device_status", "cr_status_str", "cr_last_cuda_error",
     "cr_linear", "cr_layernorm", "cr_chunk_causal_attention", "cr_qkv_rope", "cr_segment_project",
     "cr_segment_project_noalloc",
@@ -92,6 +93,10 @@ def lib(build_if_missing: bool = False) -> ctypes.CDLL:
                                     vp, vp, vp, i32, vp]),
         "cr_apply_residual_paged": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp,
                                           i64, vp, vp, vp, i32, vp, vp, i64, vp]),
+        "cr_canonicalize_chunks": (i32, [P(cr_target_dims), vp, i64, vp, vp, vp]),
+        "cr_sigma_workspace_bytes": (ctypes.c_size_t, [P(cr_target_dims), i64]),
+        "cr_sigma_accumulate": (i32, [P(cr_target_dims), vp, vp, i64, vp, vp, ctypes.c_size_t, vp]),
+        "cr_sigma_finalize": (i32, [P(cr_target_dims), vp, i64, vp, vp]),
         "cr_get_device_status": (i32, [P(c_uint32)]),
         "cr_clear_device_status": (i32, []),
         "cr_status_str": (ctypes.c_char_p, [i32]),
@@ -234,6 +239,27 @@ def cr_apply_residual_paged(target, rep, weights: PackedWeights, yf, n_tokens, k
         _p(kv_stale), _p(pos), None if f is None else f.ctypes.data, rope_mode, _p(slot_mapping),
         _p(paged_cache), num_slots, _stream(stream))
     _check("cr_apply_residual_paged", st)
+
+
+def cr_canonicalize_chunks(target, kv_inout, n_tokens, pos, inv_freq_host, stream=None):
+    f = _host_arr(inv_freq_host, np.float32)
+    _check("cr_canonicalize_chunks", lib().cr_canonicalize_chunks(
+        ctypes.byref(target), _p(kv_inout), n_tokens, _p(pos), f.ctypes.data, _stream(stream)))
+
+
+def cr_sigma_workspace_bytes(target, n_tokens) -> int:
+    return int(lib().cr_sigma_workspace_bytes(ctypes.byref(target), n_tokens))
+
+
+def cr_sigma_accumulate(target, a, b, n_tokens, sumsq, workspace, stream=None):
+    _check("cr_sigma_accumulate", lib().cr_sigma_accumulate(
+        ctypes.byref(target), _p(a), _p(b), n_tokens, _p(sumsq), _p(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def cr_sigma_finalize(target, sumsq, count, sigma_out, stream=None):
+    _check("cr_sigma_finalize", lib().cr_sigma_finalize(
+        ctypes.byref(target), _p(sumsq), count, _p(sigma_out), _stream(stream)))
 
 
 def cr_get_device_status():

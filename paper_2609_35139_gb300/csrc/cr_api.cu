@@ -594,6 +594,48 @@ cr_status cr_apply_residual_paged(const cr_target_dims* target, const cr_repaire
                        const_cast<void*>(kv_stale), d.D, static_cast<cudaStream_t>(stream));
 }
 
+// ------------------------------------------------------------------ offline preparation
+cr_status cr_canonicalize_chunks(const cr_target_dims* target, void* kv_inout, int64_t n_tokens,
+                                 const int32_t* pos, const float* inv_freq_host, void* stream) {
+    const cr_status s = check_target(target);
+    if (s != CR_OK) return s;
+    if (n_tokens < 1 || !inv_freq_host || !all_aligned(kv_inout, pos)) return CR_ERR_INVALID_ARG;
+    const Dims d = dims_of(target, nullptr);
+    if (n_tokens > INT64_MAX / (d.D * 4)) return CR_ERR_INVALID_ARG;
+    return launch_canonicalize(kv_inout, d.f32, n_tokens, pos, static_cast<int>(d.L),
+                               static_cast<int>(d.H), static_cast<int>(d.dh), inv_freq_host,
+                               static_cast<cudaStream_t>(stream));
+}
+
+size_t cr_sigma_workspace_bytes(const cr_target_dims* target, int64_t n_tokens) {
+    if (check_target(target) != CR_OK || n_tokens < 1) return 0;
+    const Dims d = dims_of(target, nullptr);
+    const int64_t slices = (n_tokens + kSigmaSlice - 1) / kSigmaSlice;
+    return align256(static_cast<size_t>(slices) * static_cast<size_t>(d.D) * sizeof(float));
+}
+
+cr_status cr_sigma_accumulate(const cr_target_dims* target, const void* a, const void* b,
+                              int64_t n_tokens, double* sumsq, void* workspace,
+                              size_t workspace_bytes, void* stream) {
+    const cr_status s = check_target(target);
+    if (s != CR_OK) return s;
+    if (n_tokens < 1 || !all_aligned(a, sumsq, workspace) || (b && !aligned16(b)))
+        return CR_ERR_INVALID_ARG;
+    if (workspace_bytes < cr_sigma_workspace_bytes(target, n_tokens)) return CR_ERR_INVALID_ARG;
+    const Dims d = dims_of(target, nullptr);
+    return launch_sigma_accumulate(a, b, d.f32, n_tokens, d.D, static_cast<float*>(workspace), sumsq,
+                                   static_cast<cudaStream_t>(stream));
+}
+
+cr_status cr_sigma_finalize(const cr_target_dims* target, const double* sumsq, int64_t count,
+                            float* sigma_out, void* stream) {
+    const cr_status s = check_target(target);
+    if (s != CR_OK) return s;
+    if (count < 1 || !all_aligned(sumsq, sigma_out)) return CR_ERR_INVALID_ARG;
+    const Dims d = dims_of(target, nullptr);
+    return launch_sigma_finalize(sumsq, d.D, count, sigma_out, static_cast<cudaStream_t>(stream));
+}
+
 // ------------------------------------------------------------------ cr_ops.h
 cr_status cr_linear(const uint16_t* A, int64_t lda, const uint16_t* W, const float* bias,
                     int64_t M, int64_t N, int64_t K, void* out, int64_t ldo, int32_t epi,

@@ -148,8 +148,17 @@ cr_status ensure_smem_attr(K kern, int bytes, unsigned long long* done) {
     return CR_OK;
 }
 
+// Offline preparation: tokens per partial sum of the sigma statistics.
+constexpr int64_t kSigmaSlice = 64;
+
 // Launchers (validated arguments).
 cr_status launch_gather(const GatherParams& p, cudaStream_t st);
+cr_status launch_canonicalize(void* kv, bool f32, int64_t n, const int32_t* pos, int L, int H, int dh,
+                              const float* inv_freq_host, cudaStream_t st);
+cr_status launch_sigma_accumulate(const void* a, const void* b, bool f32, int64_t n, int64_t D,
+                                  float* part, double* sumsq, cudaStream_t st);
+cr_status launch_sigma_finalize(const double* sumsq, int64_t D, int64_t count, float* sigma,
+                                cudaStream_t st);
 cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t M, int64_t N,
                       int64_t K, int epi, GemmParams p, void* kv_base, int64_t ld_kv,
                       cudaStream_t st);
