@@ -37,6 +37,9 @@ Readings where the paper is silent (each repeated in the design doc):
       pairs within each K segment, frequencies supplied by the caller.
   R11 The repaired value is formed exactly, then rounded once to the cache
       dtype (round to nearest even for bf16).
+  R18 The attention-topology variants of App. F change only the mask:
+      A1 "strict token-causal" is j <= i (self included, as in R7), A2 is
+      every token of the request, A3 "block-diagonal" is c(j) == c(i).
 """
 from __future__ import annotations
 
@@ -53,6 +56,7 @@ __all__ = [
     "block_causal_attention", "repair_block", "repair_backbone", "residual_head",
     "apply_residual", "global_rope_k", "repair_request", "weight_shapes", "param_groups",
     "cache_payload_bytes", "OracleResult", "repair_inv_freq", "block_weights",
+    "MASK_MODES", "attention_mask", "masked_attention",
 ]
 
 
@@ -254,16 +258,64 @@ def block_causal_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray,
     return out
 
 
+MASK_MODES = ("block_causal", "token_causal", "bidirectional", "block_diagonal")
+
+
+def attention_mask(chunk_id: np.ndarray, mode: str) -> np.ndarray:
+    """A[i, j] = True iff query i attends to key j, one request.
+
+    block_causal   c(j) <= c(i)   the method's mask (Sec. 4.1), ablation A0
+    token_causal   j <= i         ablation A1 (App. F, R18)
+    bidirectional  every j        ablation A2 (App. F)
+    block_diagonal c(j) == c(i)   ablation A3 (App. F, R18)
+    """
+    n = len(chunk_id)
+    ci, cj = chunk_id[:, None], chunk_id[None, :]
+    i, j = np.arange(n)[:, None], np.arange(n)[None, :]
+    if mode == "block_causal":
+        return cj <= ci
+    if mode == "token_causal":
+        return j <= i
+    if mode == "bidirectional":
+        return np.ones((n, n), bool)
+    if mode == "block_diagonal":
+        return cj == ci
+    raise ValueError(f"unknown mask mode {mode!r}")
+
+
+def masked_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, mask: np.ndarray) -> np.ndarray:
+    """Multi-head softmax attention of one request under an explicit mask.
+
+    q, k, v: [N, n_heads, d_head]; mask: [N, N] bool, every row with at least
+    one True.  Per head, the full score matrix q k^T / sqrt(d_head) is formed,
+    entries outside the mask are set to -inf, and each row's softmax
+    (max-subtracted) weights the values.
+    """
+    n, nh, dh = q.shape
+    assert mask.shape == (n, n) and mask.any(axis=1).all(), "every query needs a visible key"
+    out = np.empty_like(q)
+    for h in range(nh):
+        sc = (q[:, h, :] @ k[:, h, :].T) / math.sqrt(dh)
+        sc = np.where(mask, sc, -np.inf)
+        sc = sc - sc.max(axis=1, keepdims=True)
+        p = np.exp(sc)
+        p = p / p.sum(axis=1, keepdims=True)
+        out[:, h, :] = p @ v[:, h, :]
+    return out
+
+
 def repair_inv_freq(head_dim: int, theta: float) -> np.ndarray:
     i = np.arange(head_dim // 2, dtype=np.float64)
     return theta ** (-2.0 * i / head_dim)
 
 
 def repair_block(x: np.ndarray, blk: Dict[str, np.ndarray], chunk_id: np.ndarray,
-                 pos: np.ndarray, n_heads: int, eps: float, rope_theta: float) -> np.ndarray:
+                 pos: np.ndarray, n_heads: int, eps: float, rope_theta: float,
+                 mask_mode: str = "block_causal") -> np.ndarray:
     """One Repair Block: attention then MLP, pre-LN residual form (Sec. 4.1, R4).
 
-    x is the block input h^{b-1} + P_b(s).
+    x is the block input h^{b-1} + P_b(s).  `mask_mode` selects the attention
+    topology (App. F); the default is the method's block-causal mask.
     """
     n, db = x.shape
     dh = db // n_heads
@@ -274,7 +326,10 @@ def repair_block(x: np.ndarray, blk: Dict[str, np.ndarray], chunk_id: np.ndarray
     v = qkv[:, 2 * db:].reshape(n, n_heads, dh)
     f = repair_inv_freq(dh, rope_theta)
     q, k = rope_rotate_half(q, pos, f), rope_rotate_half(k, pos, f)
-    a = block_causal_attention(q, k, v, chunk_id).reshape(n, db)
+    if mask_mode == "block_causal":
+        a = block_causal_attention(q, k, v, chunk_id).reshape(n, db)
+    else:
+        a = masked_attention(q, k, v, attention_mask(chunk_id, mask_mode)).reshape(n, db)
     x = x + (a @ _bf16_mat(blk["w_o"]).T + _vec(blk["b_o"]))
     u = layer_norm(x, blk["ln2_g"], blk["ln2_b"], eps)
     g = gelu(u @ _bf16_mat(blk["w_fc1"]).T + _vec(blk["b_fc1"]))
@@ -288,12 +343,14 @@ def block_weights(w: Dict[str, np.ndarray], b: int) -> Dict[str, np.ndarray]:
 
 def repair_backbone(h0: np.ndarray, s: np.ndarray, w: Dict[str, np.ndarray],
                     chunk_id: np.ndarray, pos: np.ndarray, n_heads: int, eps: float,
-                    rope_theta: float, keep: Optional[List] = None) -> np.ndarray:
+                    rope_theta: float, keep: Optional[List] = None,
+                    mask_mode: str = "block_causal") -> np.ndarray:
     """h^b = RepairBlock_b(h^{b-1} + P_b(s); A, p), b = 1..B  (Sec. 4.1)."""
     h = h0
     for b in range(w["w_rein"].shape[0]):
         h = repair_block(h + reinjection(s, w["w_rein"][b], w["b_rein"][b]),
-                         block_weights(w, b), chunk_id, pos, n_heads, eps, rope_theta)
+                         block_weights(w, b), chunk_id, pos, n_heads, eps, rope_theta,
+                         mask_mode=mask_mode)
         if keep is not None:
             keep.append(h)
     return h
@@ -343,7 +400,8 @@ def repair_request(kv: np.ndarray, emb: np.ndarray, chunk_id: np.ndarray, pos: n
                    w: Dict[str, np.ndarray], *, cache_dtype: str, n_layers: int, n_kv_heads: int,
                    head_dim: int, n_heads: int, eps: float = 1e-5, rope_theta: float = 1e4,
                    inv_freq_target: Optional[np.ndarray] = None, with_head: bool = True,
-                   head_cols: Optional[np.ndarray] = None) -> OracleResult:
+                   head_cols: Optional[np.ndarray] = None,
+                   mask_mode: str = "block_causal") -> OracleResult:
     """The full repair forward of one request (Sec. 4.1), all in float64.
 
     kv/emb are the assembled stale cache and embeddings in their stored
@@ -357,7 +415,8 @@ def repair_request(kv: np.ndarray, emb: np.ndarray, chunk_id: np.ndarray, pos: n
     h0 = token_fusion(s, emb64, w["w_tok"], w["b_tok"], w["w_fuse"], w["b_fuse"])
     rein = [reinjection(s, w["w_rein"][b], w["b_rein"][b]) for b in range(w["w_rein"].shape[0])]
     blocks: List[np.ndarray] = []
-    hB = repair_backbone(h0, s, w, chunk_id, pos, n_heads, eps, rope_theta, keep=blocks)
+    hB = repair_backbone(h0, s, w, chunk_id, pos, n_heads, eps, rope_theta, keep=blocks,
+                         mask_mode=mask_mode)
     yf = layer_norm(hB, w["lnf_g"], w["lnf_b"], eps)
     z = rep = rot = None
     if with_head:
