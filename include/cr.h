@@ -66,6 +66,16 @@ typedef enum cr_dtype { CR_F32 = 0, CR_BF16 = 1 } cr_dtype;
 /* Global RoPE on repaired K: none (canonical K out) or R_M(p_t) (Sec. 4.1). */
 typedef enum cr_rope_mode { CR_ROPE_NONE = 0, CR_ROPE_GLOBAL = 1 } cr_rope_mode;
 
+/* Attention mask of the Repair Blocks inside one request: the method's
+ * block-causal mask (Sec. 4.1) and the attention-topology ablations of
+ * App. F.  c(i) is token i's chunk index in the request. */
+typedef enum cr_mask_mode {
+    CR_MASK_BLOCK_CAUSAL = 0,    /* A0: query i sees key j iff c(j) <= c(i) */
+    CR_MASK_TOKEN_CAUSAL = 1,    /* A1: iff j <= i */
+    CR_MASK_BIDIRECTIONAL = 2,   /* A2: every key of the request */
+    CR_MASK_BLOCK_DIAGONAL = 3   /* A3: iff c(j) == c(i) */
+} cr_mask_mode;
+
 /* Frozen target LLM cache shape (Sec. 4.1: S = 2 L H_KV segments of d_h). */
 typedef struct cr_target_dims {
     int32_t n_layers;     /* L_M */
@@ -196,6 +206,23 @@ cr_status cr_repair_forward(const cr_target_dims* target, const cr_repairer_dims
                             const int32_t* cu_seqlens_host, int32_t n_req, int64_t n_tokens,
                             uint16_t* yf_out, void* workspace, size_t workspace_bytes,
                             void* stream);
+
+/*
+ * cr_repair_forward_masked - cr_repair_forward under any mask of
+ * cr_mask_mode: the method's block-causal mask (CR_MASK_BLOCK_CAUSAL, the
+ * same computation as cr_repair_forward) or one of the attention-topology
+ * ablations A1-A3 of App. F, which change only which keys each query sees.
+ * Same arguments and buffers as cr_repair_forward; chunk_end is read for
+ * CR_MASK_BLOCK_CAUSAL and CR_MASK_BLOCK_DIAGONAL (for the latter the
+ * workspace also receives each token's chunk start).  An unknown mode returns
+ * CR_ERR_INVALID_ARG before any launch.
+ */
+cr_status cr_repair_forward_masked(const cr_target_dims* target, const cr_repairer_dims* rep,
+                                   const cr_weights* w, const float* h0, const uint16_t* rein,
+                                   const int32_t* chunk_end, const int32_t* pos,
+                                   const int32_t* cu_seqlens_host, int32_t n_req,
+                                   int64_t n_tokens, int32_t mask_mode, uint16_t* yf_out,
+                                   void* workspace, size_t workspace_bytes, void* stream);
 
 /*
  * cr_apply_residual - KV residual head and residual add, in place (Sec. 4.1):

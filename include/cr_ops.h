@@ -58,6 +58,30 @@ cr_status cr_chunk_causal_attention(const uint16_t* qkv, int32_t d_b, int32_t n_
                                     void* stream);
 
 /*
+ * cr_masked_attention - the same attention under any cr_mask_mode (Sec. 4.1
+ * for A0, App. F for the ablations A1-A3).  Arguments as in
+ * cr_chunk_causal_attention, plus: chunk_end is read for
+ * CR_MASK_BLOCK_CAUSAL and CR_MASK_BLOCK_DIAGONAL (may be NULL otherwise);
+ * chunk_start [N] int32 (request-local start of each token's chunk, as
+ * written by cr_chunk_starts) is read for CR_MASK_BLOCK_DIAGONAL only (may be
+ * NULL otherwise).  Every query sees at least itself in every mode.
+ */
+cr_status cr_masked_attention(const uint16_t* qkv, int32_t d_b, int32_t n_heads,
+                              int32_t mask_mode, const int32_t* chunk_end,
+                              const int32_t* chunk_start, const int32_t* cu_seqlens_host,
+                              int32_t n_req, int64_t n_tokens, uint16_t* out, void* stream);
+
+/*
+ * cr_chunk_starts - chunk_start[t] = request-local index of the first token
+ * of t's chunk, from the chunk map of cr_assemble_stale: the smallest u with
+ * chunk_end[u] > t inside t's request (chunk_end is non-decreasing there).
+ * chunk_end, chunk_start [N] int32 device; cu_seqlens_host [n_req+1] HOST.
+ * Integer work, exact.
+ */
+cr_status cr_chunk_starts(const int32_t* chunk_end, const int32_t* cu_seqlens_host, int32_t n_req,
+                          int64_t n_tokens, int32_t* chunk_start, void* stream);
+
+/*
  * cr_qkv_rope - the repair block's QKV linear with the repairer RoPE fused
  * into its epilogue: qkv = u W_qkv^T + b_qkv, then Q and K of every head
  * rotated (rotate-half pairs, angle pos[t] * theta^(-2i/d)).

@@ -24,10 +24,11 @@ CR_EPI_BF16, CR_EPI_GELU_BF16, CR_EPI_ADD_F32, CR_EPI_F32 = range(4)
 
 EXPORTED = [
     "cr_workspace_bytes", "cr_assemble_stale", "cr_compress_features", "cr_repair_forward",
-    "cr_apply_residual", "cr_apply_residual_paged", "cr_canonicalize_chunks",
+    "cr_repair_forward_masked", "cr_apply_residual", "cr_apply_residual_paged", "cr_canonicalize_chunks",
     "cr_sigma_workspace_bytes", "cr_sigma_accumulate", "cr_sigma_finalize", "cr_get_device_status",
     "cr_clear_device_status", "cr_status_str", "cr_last_cuda_error",
-    "cr_linear", "cr_layernorm", "cr_chunk_causal_attention", "cr_qkv_rope", "cr_segment_project",
+    "cr_linear", "cr_layernorm", "cr_chunk_causal_attention", "cr_masked_attention",
+    "cr_chunk_starts", "cr_qkv_rope", "cr_segment_project",
     "cr_segment_project_noalloc",
 ]
 
@@ -89,6 +90,9 @@ def lib(build_if_missing: bool = False) -> ctypes.CDLL:
                                        vp, i64, vp, vp, vp, c_size_t, vp]),
         "cr_repair_forward": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp, vp,
                                     vp, vp, vp, i32, i64, vp, vp, c_size_t, vp]),
+        "cr_repair_forward_masked": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights),
+                                           vp, vp, vp, vp, vp, i32, i64, i32, vp, vp, c_size_t,
+                                           vp]),
         "cr_apply_residual": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp, i64,
                                     vp, vp, vp, i32, vp]),
         "cr_apply_residual_paged": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp,
@@ -104,6 +108,8 @@ def lib(build_if_missing: bool = False) -> ctypes.CDLL:
         "cr_linear": (i32, [vp, i64, vp, vp, i64, i64, i64, vp, i64, i32, vp]),
         "cr_layernorm": (i32, [vp, vp, i64, vp, vp, vp, c_float, i64, i64, vp, vp]),
         "cr_chunk_causal_attention": (i32, [vp, i32, i32, vp, vp, i32, i64, vp, vp]),
+        "cr_masked_attention": (i32, [vp, i32, i32, i32, vp, vp, vp, i32, i64, vp, vp]),
+        "cr_chunk_starts": (i32, [vp, vp, i32, i64, vp, vp]),
         "cr_qkv_rope": (i32, [vp, vp, vp, vp, i64, i32, i32, c_float, vp, vp]),
         "cr_segment_project": (i32, [P(cr_target_dims), i32, vp, i64, vp, vp, vp, vp, vp, c_size_t,
                                      vp]),
@@ -220,6 +226,25 @@ def cr_repair_forward(target, rep, weights: PackedWeights, h0, rein, chunk_end, 
     _check("cr_repair_forward", st)
 
 
+CR_MASK_BLOCK_CAUSAL, CR_MASK_TOKEN_CAUSAL, CR_MASK_BIDIRECTIONAL, CR_MASK_BLOCK_DIAGONAL = 0, 1, 2, 3
+MASK_MODES = {"block_causal": CR_MASK_BLOCK_CAUSAL, "token_causal": CR_MASK_TOKEN_CAUSAL,
+              "bidirectional": CR_MASK_BIDIRECTIONAL, "block_diagonal": CR_MASK_BLOCK_DIAGONAL}
+
+
+def _mask_mode(mode):
+    return MASK_MODES[mode] if isinstance(mode, str) else int(mode)
+
+
+def cr_repair_forward_masked(target, rep, weights: PackedWeights, h0, rein, chunk_end, pos,
+                             cu_seqlens_host, n_tokens, mask_mode, yf_out, workspace, stream=None):
+    cu = _host_arr(cu_seqlens_host, np.int32)
+    st = lib().cr_repair_forward_masked(
+        ctypes.byref(target), ctypes.byref(rep), ctypes.byref(weights.struct), _p(h0), _p(rein),
+        _p(chunk_end), _p(pos), cu.ctypes.data, len(cu) - 1, n_tokens, _mask_mode(mask_mode),
+        _p(yf_out), _p(workspace), workspace.numel() * workspace.element_size(), _stream(stream))
+    _check("cr_repair_forward_masked", st)
+
+
 def cr_apply_residual(target, rep, weights: PackedWeights, yf, n_tokens, kv_inout, pos,
                       inv_freq_host=None, rope_mode=CR_ROPE_NONE, stream=None):
     f = None if inv_freq_host is None else _host_arr(inv_freq_host, np.float32)
@@ -295,6 +320,20 @@ def cr_chunk_causal_attention(qkv, d_b, n_heads, chunk_end, cu_seqlens_host, out
     _check("cr_chunk_causal_attention", lib().cr_chunk_causal_attention(
         _p(qkv), d_b, n_heads, _p(chunk_end), cu.ctypes.data, len(cu) - 1, qkv.shape[0], _p(out),
         _stream(stream)))
+
+
+def cr_masked_attention(qkv, d_b, n_heads, mask_mode, chunk_end, chunk_start, cu_seqlens_host, out,
+                        stream=None):
+    cu = _host_arr(cu_seqlens_host, np.int32)
+    _check("cr_masked_attention", lib().cr_masked_attention(
+        _p(qkv), d_b, n_heads, _mask_mode(mask_mode), _p(chunk_end), _p(chunk_start), cu.ctypes.data,
+        len(cu) - 1, qkv.shape[0], _p(out), _stream(stream)))
+
+
+def cr_chunk_starts(chunk_end, cu_seqlens_host, n_tokens, chunk_start, stream=None):
+    cu = _host_arr(cu_seqlens_host, np.int32)
+    _check("cr_chunk_starts", lib().cr_chunk_starts(
+        _p(chunk_end), cu.ctypes.data, len(cu) - 1, n_tokens, _p(chunk_start), _stream(stream)))
 
 
 def cr_qkv_rope(u, w_qkv, b_qkv, pos, d_b, n_heads, rope_theta, qkv, stream=None):

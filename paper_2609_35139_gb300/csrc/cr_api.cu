@@ -81,7 +81,7 @@ cr_status check_repairer(const cr_repairer_dims* r) {
 }
 
 struct WsLayout {
-    size_t wfold, kvb, embb, y, se, x, u, qkv, o, g, rope, total;
+    size_t wfold, kvb, embb, y, se, x, u, qkv, o, g, rope, kstart, total;
 };
 
 WsLayout ws_layout(const Dims& d, int64_t n) {
@@ -104,6 +104,7 @@ WsLayout ws_layout(const Dims& d, int64_t n) {
     w.o = take(N * d.db * 2);
     w.g = take(N * d.hid * 2);
     w.rope = take(N * (d.hd / 2) * 8);   // repairer RoPE (cos, sin) per token and pair
+    w.kstart = take(N * 4);              // chunk start per token (block-diagonal mask)
     w.total = off;
     return w;
 }
@@ -404,10 +405,20 @@ cr_status cr_compress_features(const cr_target_dims* target, const cr_repairer_d
     return CR_OK;
 }
 
-static cr_status attn_params(const Dims& d, const int32_t* chunk_end,
-                             const int32_t* cu_seqlens_host, int n_req, int64_t N, uint16_t* out,
-                             unsigned* status, AttnParams* p) {
+static bool valid_mask_mode(int32_t m) {
+    return m == CR_MASK_BLOCK_CAUSAL || m == CR_MASK_TOKEN_CAUSAL || m == CR_MASK_BIDIRECTIONAL ||
+           m == CR_MASK_BLOCK_DIAGONAL;
+}
+
+static cr_status attn_params(const Dims& d, int32_t mask_mode, const int32_t* chunk_end,
+                             const int32_t* chunk_start, const int32_t* cu_seqlens_host, int n_req,
+                             int64_t N, uint16_t* out, unsigned* status, AttnParams* p) {
     if (!cu_seqlens_host || n_req < 1 || n_req > kMaxReq) return CR_ERR_INVALID_ARG;
+    if (!valid_mask_mode(mask_mode)) return CR_ERR_INVALID_ARG;
+    if ((mask_mode == CR_MASK_BLOCK_CAUSAL || mask_mode == CR_MASK_BLOCK_DIAGONAL) &&
+        !all_aligned(chunk_end))
+        return CR_ERR_INVALID_ARG;
+    if (mask_mode == CR_MASK_BLOCK_DIAGONAL && !all_aligned(chunk_start)) return CR_ERR_INVALID_ARG;
     if (cu_seqlens_host[0] != 0 || cu_seqlens_host[n_req] != N) return CR_ERR_INVALID_ARG;
     memset(p, 0, sizeof(*p));
     int items = 0;
@@ -421,6 +432,8 @@ static cr_status attn_params(const Dims& d, const int32_t* chunk_end,
     p->req_start[n_req] = cu_seqlens_host[n_req];
     p->tile_prefix[n_req] = items;
     p->chunk_end = chunk_end;
+    p->chunk_start = chunk_start;
+    p->mask_mode = mask_mode;
     p->out = out;
     p->d_b = static_cast<int32_t>(d.db);
     p->n_heads = static_cast<int32_t>(d.nh);
@@ -437,6 +450,17 @@ cr_status cr_repair_forward(const cr_target_dims* target, const cr_repairer_dims
                             const int32_t* cu_seqlens_host, int32_t n_req, int64_t n_tokens,
                             uint16_t* yf_out, void* workspace, size_t workspace_bytes,
                             void* stream) {
+    return cr_repair_forward_masked(target, rep, w, h0, rein, chunk_end, pos, cu_seqlens_host,
+                                    n_req, n_tokens, CR_MASK_BLOCK_CAUSAL, yf_out, workspace,
+                                    workspace_bytes, stream);
+}
+
+cr_status cr_repair_forward_masked(const cr_target_dims* target, const cr_repairer_dims* rep,
+                                   const cr_weights* w, const float* h0, const uint16_t* rein,
+                                   const int32_t* chunk_end, const int32_t* pos,
+                                   const int32_t* cu_seqlens_host, int32_t n_req,
+                                   int64_t n_tokens, int32_t mask_mode, uint16_t* yf_out,
+                                   void* workspace, size_t workspace_bytes, void* stream) {
     cr_status s = check_target(target);
     if (s == CR_OK) s = check_repairer(rep);
     if (s != CR_OK) return s;
@@ -444,6 +468,7 @@ cr_status cr_repair_forward(const cr_target_dims* target, const cr_repairer_dims
     if (!w || n_tokens < 1 || n_tokens > INT32_MAX / 2) return CR_ERR_INVALID_ARG;
     if (!all_aligned(h0, chunk_end, pos, yf_out, workspace, w->lnf_g, w->lnf_b))
         return CR_ERR_INVALID_ARG;
+    if (!valid_mask_mode(mask_mode)) return CR_ERR_INVALID_ARG;
     if (d.B > 0 && (!w->blocks || !all_aligned(rein))) return CR_ERR_INVALID_ARG;
     for (int b = 0; b < d.B; ++b) {
         const cr_block_weights& k = w->blocks[b];
@@ -459,8 +484,9 @@ cr_status cr_repair_forward(const cr_target_dims* target, const cr_repairer_dims
     uint16_t* qkv = at<uint16_t>(workspace, L.qkv);
     uint16_t* o = at<uint16_t>(workspace, L.o);
     uint16_t* g = at<uint16_t>(workspace, L.g);
+    int32_t* kstart = at<int32_t>(workspace, L.kstart);
     AttnParams* ap = new AttnParams();
-    s = attn_params(d, chunk_end, cu_seqlens_host, n_req, N, o, nullptr, ap);
+    s = attn_params(d, mask_mode, chunk_end, kstart, cu_seqlens_host, n_req, N, o, nullptr, ap);
     unsigned* status = (s == CR_OK) ? device_status_ptr() : nullptr;
     if (s == CR_OK && !status) s = CR_ERR_CUDA;
     if (s != CR_OK) {
@@ -469,6 +495,14 @@ cr_status cr_repair_forward(const cr_target_dims* target, const cr_repairer_dims
     }
     ap->status = status;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
+    // the block-diagonal mask also needs each token's chunk start: once per forward
+    if (mask_mode == CR_MASK_BLOCK_DIAGONAL && d.B > 0) {
+        s = launch_chunk_starts(chunk_end, *ap, N, kstart, st);
+        if (s != CR_OK) {
+            delete ap;
+            return s;
+        }
+    }
     GemmParams gq{};
     gq.status = status;
     gq.pos = pos;
@@ -684,12 +718,55 @@ cr_status cr_chunk_causal_attention(const uint16_t* qkv, int32_t d_b, int32_t n_
     d.nh = n_heads;
     d.hd = hd;
     AttnParams* ap = new AttnParams();
-    cr_status s = attn_params(d, chunk_end, cu_seqlens_host, n_req, n_tokens, out, nullptr, ap);
+    cr_status s = attn_params(d, CR_MASK_BLOCK_CAUSAL, chunk_end, nullptr, cu_seqlens_host, n_req,
+                              n_tokens, out, nullptr, ap);
     if (s == CR_OK) {
         ap->status = device_status_ptr();
         s = ap->status ? launch_attention(qkv, n_tokens, hd, *ap, static_cast<cudaStream_t>(stream))
                        : CR_ERR_CUDA;
     }
+    delete ap;
+    return s;
+}
+
+cr_status cr_masked_attention(const uint16_t* qkv, int32_t d_b, int32_t n_heads,
+                              int32_t mask_mode, const int32_t* chunk_end,
+                              const int32_t* chunk_start, const int32_t* cu_seqlens_host,
+                              int32_t n_req, int64_t n_tokens, uint16_t* out, void* stream) {
+    if (n_heads < 1 || d_b < 1 || d_b % n_heads != 0 || n_tokens < 1 || n_tokens > INT32_MAX / 2)
+        return CR_ERR_INVALID_ARG;
+    const int hd = d_b / n_heads;
+    if (hd != 32 && hd != 64) return CR_ERR_UNSUPPORTED;
+    if (!all_aligned(qkv, out)) return CR_ERR_INVALID_ARG;
+    Dims d{};
+    d.db = d_b;
+    d.nh = n_heads;
+    d.hd = hd;
+    AttnParams* ap = new AttnParams();
+    cr_status s = attn_params(d, mask_mode, chunk_end, chunk_start, cu_seqlens_host, n_req,
+                              n_tokens, out, nullptr, ap);
+    if (s == CR_OK) {
+        ap->status = device_status_ptr();
+        s = ap->status ? launch_attention(qkv, n_tokens, hd, *ap, static_cast<cudaStream_t>(stream))
+                       : CR_ERR_CUDA;
+    }
+    delete ap;
+    return s;
+}
+
+cr_status cr_chunk_starts(const int32_t* chunk_end, const int32_t* cu_seqlens_host, int32_t n_req,
+                          int64_t n_tokens, int32_t* chunk_start, void* stream) {
+    if (n_tokens < 1 || n_tokens > INT32_MAX / 2 || !all_aligned(chunk_end, chunk_start))
+        return CR_ERR_INVALID_ARG;
+    Dims d{};
+    d.db = 64;
+    d.nh = 1;
+    d.hd = 64;
+    AttnParams* ap = new AttnParams();
+    cr_status s = attn_params(d, CR_MASK_BLOCK_DIAGONAL, chunk_end, chunk_start, cu_seqlens_host,
+                              n_req, n_tokens, nullptr, nullptr, ap);
+    if (s == CR_OK) s = launch_chunk_starts(chunk_end, *ap, n_tokens, chunk_start,
+                                            static_cast<cudaStream_t>(stream));
     delete ap;
     return s;
 }

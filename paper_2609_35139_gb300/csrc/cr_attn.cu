@@ -1,11 +1,16 @@
 // Chunk-block-causal attention of the Repair Blocks (Sec. 4.1):
 //   o_i = sum_{j : c(j) <= c(i)} softmax_j(q_i . k_j / sqrt(d)) v_j
 // inside each request.  Chunk ids are non-decreasing along a request, so the
-// keys visible to query i are exactly j < chunk_end[i]: a prefix.  A query
-// tile therefore needs key tiles 0 .. ceil(max_i chunk_end / 128) - 1 and
-// nothing past that; those tiles are never loaded or multiplied.  Rows whose
-// chunk ends inside a key tile mask the rest of it; fully visible tiles do no
-// masking work at all.
+// keys visible to query i are exactly j < chunk_end[i]: a prefix.  The
+// attention-topology ablations of App. F keep that shape: with A1 (token-
+// causal) the keys are j <= i, with A2 (bidirectional) the whole request, with
+// A3 (block-diagonal) j in [chunk_start[i], chunk_end[i]).  In every mode the
+// visible keys of row i are one interval [lo(i), hi(i)) whose ends never
+// decrease with i, so a query tile needs key tiles
+// floor(lo(first row) / 128) .. ceil(hi(last row) / 128) - 1 and nothing
+// else; other tiles are never loaded or multiplied.  Rows whose interval ends
+// inside a key tile mask the rest of it; fully visible tiles do no masking
+// work at all.
 //
 // CTA = (request, head, two consecutive 128-query tiles w = 0, 1); three
 // warpgroups, the first of which gives registers to the other two:
@@ -74,6 +79,16 @@ constexpr float kRescaleLog2 = 8.0f;   // lazy-rescale threshold (log2 units)
 // row max, so the special-function unit stays busy.
 constexpr bool kTurns = true;
 
+// Exclusive end and start of the visible keys of request-local row i.
+__device__ __forceinline__ int key_hi(const AttnParams& p, int rs, int len, int i) {
+    if (p.mask_mode == CR_MASK_TOKEN_CAUSAL) return i + 1;
+    if (p.mask_mode == CR_MASK_BIDIRECTIONAL) return len;
+    return __ldg(p.chunk_end + rs + i);
+}
+__device__ __forceinline__ int key_lo(const AttnParams& p, int rs, int i) {
+    return p.mask_mode == CR_MASK_BLOCK_DIAGONAL ? __ldg(p.chunk_start + rs + i) : 0;
+}
+
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQKV, const __grid_constant__ AttnParams p) {
@@ -133,11 +148,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
     pdl_wait();   // qkv and the chunk map come from earlier kernels
+    // Both query tiles start at the key tile of the pair's first visible key,
+    // kbase = 128 * floor(lo(q0) / 128): every issuer and softmax group then
+    // takes the ring's tiles in order from its first slot use, which keeps
+    // each parity wait within one phase of its barrier.  (Under the
+    // block-diagonal mask the second tile's rows may start later; their
+    // leading key tiles are fully masked and contribute exact zeros.)  Tile j
+    // below is key tile kbase / 128 + j; query tile w needs j in [0, n_kv[w]),
+    // an empty second tile (past the request's end) none.
+    const int kbase = key_lo(p, rs, q0) & ~127;
     int n_kv[2];
 #pragma unroll
     for (int w = 0; w < 2; ++w) {
         const int first = q0 + 128 * w;
-        n_kv[w] = first < len ? (__ldg(p.chunk_end + rs + min(first + 127, len - 1)) + 127) / 128 : 0;
+        n_kv[w] = first < len ? (key_hi(p, rs, len, min(first + 127, len - 1)) - kbase + 127) / 128 : 0;
     }
     const int n_max = max(n_kv[0], n_kv[1]);
     const uint32_t tmem_base = *tmem_slot;
@@ -164,9 +188,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 uint8_t* kt = smem + Cfg::kKVOff + st * 2 * Cfg::kTileBytes;
                 if (elect_one()) {
                     mbar_expect_tx(&kv_full[st], 2 * Cfg::kTileBytes);
-                    tma_load_2d(kt, &tmQKV, &kv_full[st], p.d_b + head * D, rs + j * 128);
+                    tma_load_2d(kt, &tmQKV, &kv_full[st], p.d_b + head * D, rs + kbase + j * 128);
                     tma_load_2d(kt + Cfg::kTileBytes, &tmQKV, &kv_full[st], 2 * p.d_b + head * D,
-                                rs + j * 128);
+                                rs + kbase + j * 128);
+                    // the stage is free once both issuers release it; an issuer
+                    // whose query tile ends before tile j is released for here
+                    // (its partner's release, after its MMAs, completes the phase)
+                    if (j >= n_kv[0]) mbar_arrive(&kv_empty[st]);
+                    if (j >= n_kv[1]) mbar_arrive(&kv_empty[st]);
                 }
                 __syncwarp();
             }
@@ -182,6 +211,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             // once P_w,j is written.  The whole warp runs the loop and computes
             // the descriptors; one elected lane issues the MMAs and commits.
             const int w = static_cast<int>(warp) - 1;
+            constexpr int jl = 0;
             const int n = n_kv[w];
             // Descriptors are built once; a K=16 step adds 32 bytes (2 units of
             // 16 B) to the start address, a stage adds 2 tiles, a V step 16 rows.
@@ -223,7 +253,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint64_t dv = dv0 + static_cast<uint64_t>(j % NS) * kStageStep;
 #pragma unroll
                 for (int h = 0; h < 2; ++h) {
-                    if (!mbar_wait_warp(&p_full[2 * w + h], static_cast<uint32_t>(j) & 1u, wc, 224))
+                    if (!mbar_wait_warp(&p_full[2 * w + h], static_cast<uint32_t>(j - jl) & 1u, wc, 224))
                         return false;
                     tc_fence_after();
                     if (elect_one()) {
@@ -233,7 +263,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                             // dimension), d contiguous (MN-major); 16 keys = two 8-row atoms.
                             const int kk = 4 * h + q;
                             mma_bf16_ts(dout, pa + kk * 8, dv + kk * ((16 * Cfg::kRowBytes) >> 4),
-                                        IDESC_PV, (j > 0 || kk != 0) ? 1u : 0u);
+                                        IDESC_PV, (j > jl || kk != 0) ? 1u : 0u);
                         }
                         if (h == 1) mma_commit(&pv_done[w]);
                     }
@@ -243,22 +273,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             };
             bool ok = mbar_wait_warp(q_full, 0, wc, 221);
             if (ok) tc_fence_after();
-            if (ok && n > 0) ok = issue_s(0);
-            for (int j = 0; j < n_max && ok; ++j) {
-                if (j < n) {
-                    if (j + 1 < n) {
-                        ok = mbar_wait_warp(&s_free[w], static_cast<uint32_t>(j) & 1u, wc, 223);
-                        if (ok) {
-                            tc_fence_after();
-                            ok = issue_s(j + 1);
-                        }
+            // only the tiles of [jl, n): the producer releases the others
+            if (ok && n > jl) ok = issue_s(jl);
+            for (int j = jl; j < n && ok; ++j) {
+                if (j + 1 < n) {
+                    ok = mbar_wait_warp(&s_free[w], static_cast<uint32_t>(j - jl) & 1u, wc, 223);
+                    if (ok) {
+                        tc_fence_after();
+                        ok = issue_s(j + 1);
                     }
-                    if (ok) ok = issue_pv(j);
-                } else {
-                    // a tile only the other query tile needs: wait for it so that
-                    // this release lands in the stage's current phase
-                    ok = ensure_kv(j);
                 }
+                if (ok) ok = issue_pv(j);
                 if (ok) {
                     if (elect_one()) mma_commit(&kv_empty[j % NS]);
                     __syncwarp();
@@ -276,18 +301,27 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int r = static_cast<int>(quad * 32 + lane);
         const int qrow = q0 + 128 * w + r;
         const bool valid = qrow < len;
-        const int cend = valid ? __ldg(p.chunk_end + rs + qrow) : 1;
+        // visible keys of this row, relative to kbase
+        const int cend = (valid ? key_hi(p, rs, len, qrow) : 1) - kbase;
+        const int cbeg = (valid ? key_lo(p, rs, qrow) : 0) - kbase;
         const uint32_t lane_off = (quad * 32u) << 16;
         const uint32_t ts = tmem_base + lane_off + Cfg::kTmemS + w * 128;
         const uint32_t to = tmem_base + lane_off + Cfg::kTmemO + w * D;
         const float sc = p.scale_log2;
+        constexpr int jl = 0;
         const int n = n_kv[w];
+        // exp-pass turns: tile j of group 0 waits for group 1's tile j - 1, tile
+        // j of group 1 for group 0's tile j, when the other group has that tile;
+        // jt = j - turn_lo is the waited-for pass of the other group
+        const int turn_lo = (w == 0) ? 1 : 0;
+        const int turn_hi = (w == 0) ? n_kv[1] + 1 : n_kv[0];
         const uint32_t tp = tmem_base + lane_off + Cfg::kTmemP + w * 64;
         float m = NEG_INF, l = 0.0f;
 
         bool ok = true;
-        for (int j = 0; j < n; ++j) {
-            ok = mbar_wait(&s_full[w], static_cast<uint32_t>(j) & 1u, wc, 321);
+        for (int j = jl; j < n; ++j) {
+            const uint32_t it = static_cast<uint32_t>(j - jl);   // tiles done by this group
+            ok = mbar_wait(&s_full[w], it & 1u, wc, 321);
             if (!__all_sync(0xffffffffu, ok)) {
                 ok = false;
                 break;
@@ -305,11 +339,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive(&s_free[w]);
             const int k0 = j * 128;
-            if (k0 + 128 > cend) {
-                // keys >= cend are masked; fully visible tiles skip this
-                const int lim = cend - k0;
+            if (k0 + 128 > cend || k0 < cbeg) {
+                // keys outside [cbeg, cend) are masked; fully visible tiles skip this
+                const int hi = cend - k0, lo = cbeg - k0;
 #pragma unroll
-                for (int i = 0; i < 128; ++i) s[i] = (i < lim) ? s[i] : NEG_INF;
+                for (int i = 0; i < 128; ++i) s[i] = (i < hi && i >= lo) ? s[i] : NEG_INF;
             }
             // row max of the (masked) scores in eight independent chains
             float mxv[8];
@@ -321,8 +355,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                              fmaxf(fmaxf(mxv[4], mxv[5]), fmaxf(mxv[6], mxv[7])));
             mx *= sc;
             // O_w and P_w are free once PV_w,j-1 has completed
-            if (j > 0) {
-                ok = mbar_wait(&pv_done[w], static_cast<uint32_t>(j - 1) & 1u, wc, 322);
+            if (j > jl) {
+                ok = mbar_wait(&pv_done[w], (it - 1u) & 1u, wc, 322);
                 if (!__all_sync(0xffffffffu, ok)) {
                     ok = false;
                     break;
@@ -330,12 +364,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_after();
             }
             // lazily move the reference max: on the first tile, or when this
-            // tile would push P above 2^8 somewhere in the warp
-            const bool raise = (j == 0) || (mx > m + kRescaleLog2);
+            // tile would push P above 2^8 somewhere in the warp.  A row whose
+            // visible keys start in a later tile (block-diagonal mask) keeps
+            // m = -inf until then: its P is 0 (exponent taken against 0) and
+            // its first rescale multiplies the zero O and l by 0.
+            const bool raise = (j == jl) || (mx > m + kRescaleLog2);
             if (__any_sync(0xffffffffu, raise)) {
                 const float m_new = fmaxf(m, mx);
-                if (j > 0) {
-                    const float alpha = ex2(m - m_new);
+                if (j > jl) {
+                    const float alpha = (m == m_new) ? 1.0f : ex2(m - m_new);
 #pragma unroll
                     for (int c = 0; c < D; c += 16) {
                         float o[16];
@@ -349,9 +386,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 m = m_new;
             }
-            if (kTurns && (w == 0 ? (j > 0 && j - 1 < n_kv[1]) : (j < n_kv[0]))) {
+            if (kTurns && j >= turn_lo && j < turn_hi) {
                 // group 0 goes first on each key tile
-                const int jt = (w == 0) ? j - 1 : j;
+                const int jt = j - turn_lo;
                 ok = mbar_wait(&turn[(1 - w) * 4 + quad], static_cast<uint32_t>(jt) & 1u, wc, 323);
                 if (!__all_sync(0xffffffffu, ok)) {
                     ok = false;
@@ -359,6 +396,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             // P = 2^(s*sc - m) -> bf16 pairs in TMEM, and the row sum
+            const float m_ref = (m == NEG_INF) ? 0.0f : m;
             float rs8[8];
 #pragma unroll
             for (int q = 0; q < 8; ++q) rs8[q] = 0.0f;
@@ -368,7 +406,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int i = 0; i < 64; i += 2) {
                     float t0, t1;
-                    ffma2(t0, t1, s[h + i], s[h + i + 1], sc, sc, -m, -m);
+                    ffma2(t0, t1, s[h + i], s[h + i + 1], sc, sc, -m_ref, -m_ref);
                     const float e0 = ex2(t0);
                     const float e1 = ex2(t1);
                     const int q = (i >> 1) & 3;       // four pairs of running sums
@@ -388,11 +426,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             l += ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
         }
-        if (ok && n > 0) {
-            ok = mbar_wait(&pv_done[w], static_cast<uint32_t>(n - 1) & 1u, wc, 324);
+        if (ok && n > jl) {
+            ok = mbar_wait(&pv_done[w], static_cast<uint32_t>(n - 1 - jl) & 1u, wc, 324);
             ok = __all_sync(0xffffffffu, ok);
         }
-        if (ok && n > 0) {
+        if (ok && n > jl) {
             tc_fence_after();
             const float inv = 1.0f / l;
             uint16_t* dst = p.out + static_cast<int64_t>(rs + qrow) * p.d_b + head * D;
@@ -446,7 +484,45 @@ cr_status launch_d(const CUtensorMap& tm, const AttnParams& p, cudaStream_t st) 
     return launch_pdl(kern, dim3(grid), dim3(kThreads), Cfg::kSmemBytes, st, tm, p);
 }
 
+// chunk_start[t] = the request-local index of the first token of t's chunk:
+// the smallest u with chunk_end[u] > i, i = t's request-local index (tokens of
+// earlier chunks have chunk_end <= their chunk's end <= i, tokens of i's chunk
+// have chunk_end > i).  One thread per token, binary searches over the
+// request starts and over the request's non-decreasing chunk_end; the result
+// lies in [0, i] whatever the map holds.
+__global__ void __launch_bounds__(256)
+    chunk_start_kernel(const int32_t* __restrict__ chunk_end, int32_t* __restrict__ chunk_start,
+                       const __grid_constant__ AttnParams p, int n_tokens) {
+    pdl_launch_dependents();
+    pdl_wait();   // the chunk map comes from an earlier kernel
+    const int t = static_cast<int>(blockIdx.x * blockDim.x + threadIdx.x);
+    if (t >= n_tokens) return;
+    int r0 = 0, r1 = p.n_req - 1;       // the request r with req_start[r] <= t
+    while (r0 < r1) {
+        const int mid = (r0 + r1 + 1) >> 1;
+        if (p.req_start[mid] <= t) r0 = mid;
+        else r1 = mid - 1;
+    }
+    const int rs = p.req_start[r0];
+    const int i = t - rs;
+    int a = 0, b = i;
+    while (a < b) {
+        const int mid = (a + b) >> 1;
+        if (__ldg(chunk_end + rs + mid) > i) b = mid;
+        else a = mid + 1;
+    }
+    chunk_start[t] = a;
+}
+
 }  // namespace
+
+cr_status launch_chunk_starts(const int32_t* chunk_end, const AttnParams& p, int64_t n_tokens,
+                              int32_t* chunk_start, cudaStream_t st) {
+    if (n_tokens < 1) return CR_OK;
+    const int grid = static_cast<int>((n_tokens + 255) / 256);
+    return launch_pdl(chunk_start_kernel, dim3(grid), dim3(256), 0, st, chunk_end, chunk_start, p,
+                      static_cast<int>(n_tokens));
+}
 
 cr_status launch_attention(const uint16_t* qkv, int64_t n_tokens, int head_dim,
                            const AttnParams& p, cudaStream_t st) {

@@ -91,7 +91,9 @@ struct SegParams {
 
 // ------------------------------------------------------------------ attention
 struct AttnParams {
-    const int32_t* chunk_end;
+    const int32_t* chunk_end;    // [N] request-local visible-key end (A0, A3)
+    const int32_t* chunk_start;  // [N] request-local chunk start (A3 only)
+    int32_t mask_mode;           // cr_mask_mode
     uint16_t* out;           // [N, d_b]
     int32_t d_b;
     int32_t n_heads;
@@ -172,6 +174,8 @@ cr_status launch_rope_table(const int32_t* pos, int64_t n, int half_dim, const f
 cr_status launch_layernorm(const float* x, const uint16_t* add, int64_t ld_add, float* x_out,
                            const float* g, const float* b, float eps, int64_t M, int64_t D,
                            uint16_t* u, cudaStream_t st);
+cr_status launch_chunk_starts(const int32_t* chunk_end, const AttnParams& p, int64_t n_tokens,
+                              int32_t* chunk_start, cudaStream_t st);
 cr_status launch_attention(const uint16_t* qkv, int64_t n_tokens, int head_dim,
                            const AttnParams& p, cudaStream_t st);
 

@@ -63,10 +63,17 @@ class RepairSession:
         cr.cr_compress_features(self.target, self.rep, self.weights, self.kv, self.emb, a.n_tokens,
                                 self.h0, self.rein, self.workspace, stream)
 
-    def forward(self, a: Assembled, stream=None):
-        cr.cr_repair_forward(self.target, self.rep, self.weights, self.h0, self.rein,
-                             self.chunk_end, self.pos, a.cu_seqlens, a.n_tokens, self.yf,
-                             self.workspace, stream)
+    def forward(self, a: Assembled, stream=None, mask_mode="block_causal"):
+        """The Repair Blocks and LN_f; mask_mode picks the attention mask (the method's
+        block-causal mask, or an App. F ablation: token_causal, bidirectional, block_diagonal)."""
+        if mask_mode in ("block_causal", cr.CR_MASK_BLOCK_CAUSAL):
+            cr.cr_repair_forward(self.target, self.rep, self.weights, self.h0, self.rein,
+                                 self.chunk_end, self.pos, a.cu_seqlens, a.n_tokens, self.yf,
+                                 self.workspace, stream)
+        else:
+            cr.cr_repair_forward_masked(self.target, self.rep, self.weights, self.h0, self.rein,
+                                        self.chunk_end, self.pos, a.cu_seqlens, a.n_tokens,
+                                        mask_mode, self.yf, self.workspace, stream)
 
     def apply(self, a: Assembled, inv_freq_target=None, rope_mode=cr.CR_ROPE_NONE, stream=None):
         cr.cr_apply_residual(self.target, self.rep, self.weights, self.yf, a.n_tokens, self.kv,

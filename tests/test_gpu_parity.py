@@ -35,7 +35,8 @@ def lib():
 class GpuRun:
     """One pass of the repair chain on a case, keeping the intermediates on the host."""
 
-    def __init__(self, case, rope_mode=cr.CR_ROPE_NONE, weights=None, pool=None, patch=None):
+    def __init__(self, case, rope_mode=cr.CR_ROPE_NONE, weights=None, pool=None, patch=None,
+                 mask_mode="block_causal"):
         t, r = dims_from(case.target, case.repairer)
         w = weights if weights is not None else case.weights
         self.pw = pack_host_weights(w, case.repairer.n_blocks)
@@ -56,7 +57,7 @@ class GpuRun:
         if patch is not None:
             patch(s, n)
         s.compress(self.a)
-        s.forward(self.a)
+        s.forward(self.a, mask_mode=mask_mode)
         s.apply(self.a, case.inv_freq_target, rope_mode)
         torch.cuda.synchronize()
         self.h0 = to_host(s.h0[:n])
@@ -65,7 +66,7 @@ class GpuRun:
         self.kv = to_host(s.kv[:n])
 
 
-def oracle_request(case, assembled, r, rows=None, rope=False, weights=None):
+def oracle_request(case, assembled, r, rows=None, rope=False, weights=None, mask_mode="block_causal"):
     """Oracle pass over request r; head only on `rows` (request-local) if given."""
     t, rp = case.target, case.repairer
     w = weights if weights is not None else case.weights
@@ -75,7 +76,7 @@ def oracle_request(case, assembled, r, rows=None, rope=False, weights=None):
                            cache_dtype=t.cache_dtype, n_layers=t.n_layers,
                            n_kv_heads=t.n_kv_heads, head_dim=t.head_dim, n_heads=rp.n_heads,
                            inv_freq_target=case.inv_freq_target if rope else None,
-                           with_head=rows is None)
+                           with_head=rows is None, mask_mode=mask_mode)
     if rows is not None:
         z = O.residual_head(res.blocks[-1][rows] if res.blocks else res.h0[rows], w["lnf_g"],
                             w["lnf_b"], w["w_out"], w["b_out"], rp.ln_eps)

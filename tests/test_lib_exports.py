@@ -60,10 +60,10 @@ def test_workspace_bytes_host_logic(L):
     w1 = cr.cr_workspace_bytes(t, r, 1)
     w2 = cr.cr_workspace_bytes(t, r, 5120)
     assert 0 < w1 < w2
-    # dominated by per-token buffers: y, s|e, x, u, qkv, o, g (bf16 / fp32 x) and the
-    # repairer RoPE table (32 (cos, sin) pairs per token)
+    # dominated by per-token buffers: y, s|e, x, u, qkv, o, g (bf16 / fp32 x), the
+    # repairer RoPE table (32 (cos, sin) pairs per token) and the chunk start (int32)
     per_tok = (512 * 16 * 2 + 2 * 512 * 2 + 1024 * 4 + 1024 * 2 + 3 * 1024 * 2 + 1024 * 2
-               + 4096 * 2 + 32 * 8)
+               + 4096 * 2 + 32 * 8 + 4)
     assert abs((w2 - w1) - 5119 * per_tok) < 64 * 256
     bad = cr.repairer_dims(16, 512, 1000, 6, 16, 4096)   # d_b not a multiple of 128
     assert cr.cr_workspace_bytes(t, bad, 10) == 0
@@ -116,6 +116,28 @@ def test_other_calls_reject_bad_inputs_on_host(L):
     cu = np.array([0, 100, 90], np.int32)
     assert L.cr_chunk_causal_attention(FAKE, 1024, 16, FAKE, cu.ctypes.data, 2, 90, FAKE,
                                        None) == cr.CR_ERR_INVALID_ARG          # empty request
+
+
+def test_mask_calls_reject_bad_inputs_on_host(L):
+    cu = np.array([0, 100], np.int32)
+    att = lambda mode, cend=FAKE, cstart=FAKE, cuv=cu: L.cr_masked_attention(
+        FAKE, 512, 8, mode, cend, cstart, cuv.ctypes.data, 1, 100, FAKE, None)
+    assert att(7) == cr.CR_ERR_INVALID_ARG                                 # unknown mask
+    assert att(-1) == cr.CR_ERR_INVALID_ARG
+    assert att(cr.CR_MASK_BLOCK_DIAGONAL, cstart=None) == cr.CR_ERR_INVALID_ARG   # needs starts
+    assert att(cr.CR_MASK_BLOCK_CAUSAL, cend=None) == cr.CR_ERR_INVALID_ARG       # needs ends
+    assert att(cr.CR_MASK_BLOCK_CAUSAL, cuv=np.array([0, 99], np.int32)) == cr.CR_ERR_INVALID_ARG
+    assert L.cr_masked_attention(FAKE, 1024, 8, 1, None, None, cu.ctypes.data, 1, 100, FAKE,
+                                 None) == cr.CR_ERR_UNSUPPORTED             # 128-dim heads
+    assert L.cr_chunk_starts(FAKE, np.array([0, 99], np.int32).ctypes.data, 1, 100, FAKE,
+                             None) == cr.CR_ERR_INVALID_ARG
+    assert L.cr_chunk_starts(FAKE + 4, cu.ctypes.data, 1, 100, FAKE, None) == cr.CR_ERR_INVALID_ARG
+    c, (t, r) = _dims()
+    w = cr.cr_weights()
+    w.lnf_g = w.lnf_b = FAKE
+    assert L.cr_repair_forward_masked(ctypes.byref(t), ctypes.byref(r), ctypes.byref(w), FAKE, FAKE,
+                                      FAKE, FAKE, cu.ctypes.data, 1, 100, 9, FAKE, FAKE, 1 << 30,
+                                      None) == cr.CR_ERR_INVALID_ARG
 
 
 def test_paged_residual_rejects_bad_inputs_on_host(L):
