@@ -76,6 +76,15 @@ typedef enum cr_mask_mode {
     CR_MASK_BLOCK_DIAGONAL = 3   /* A3: iff c(j) == c(i) */
 } cr_mask_mode;
 
+/* Output choices of App. F ("Applying the predicted K and V", ablation A5):
+ * which cache components receive the predicted correction, and what it is
+ * added to. */
+typedef enum cr_apply_component { CR_APPLY_K = 1, CR_APPLY_V = 2, CR_APPLY_KV = 3 } cr_apply_component;
+typedef enum cr_apply_offset {
+    CR_OFFSET_STALE = 0,   /* KV_stale + sigma_Delta z: the method (Sec. 4.1) */
+    CR_OFFSET_ZERO = 1     /* sigma_Delta z alone: A5, the head predicts the joint cache */
+} cr_apply_offset;
+
 /* Frozen target LLM cache shape (Sec. 4.1: S = 2 L H_KV segments of d_h). */
 typedef struct cr_target_dims {
     int32_t n_layers;     /* L_M */
@@ -238,6 +247,41 @@ cr_status cr_apply_residual(const cr_target_dims* target, const cr_repairer_dims
                             const cr_weights* w, const uint16_t* yf, int64_t n_tokens,
                             void* kv_inout, const int32_t* pos, const float* inv_freq_host,
                             int32_t rope_mode, void* stream);
+
+/*
+ * cr_apply_residual_select - cr_apply_residual under an output choice of
+ * App. F.  components: the coordinates that receive the correction
+ * (CR_APPLY_K, CR_APPLY_V or both); every other coordinate keeps its stale
+ * value bit for bit.  offset: CR_OFFSET_STALE (the method) or CR_OFFSET_ZERO
+ * (A5: the repaired value is round(sigma_delta * z)).  keep_chunk_id: NULL, or
+ * the chunk map chunk_id [N] device int32 of cr_assemble_stale, in which case
+ * the rows of each request's first chunk (chunk_id == 0) keep their stale
+ * cache ("keep first chunk").  With CR_ROPE_GLOBAL every K segment leaves
+ * rotated by R_M(p_t), repaired or not (an unrepaired K is the stale cache's
+ * K, which is rotated to its request position, Sec. 2.2).  A single-component
+ * choice needs H_kv * d_h to be a multiple of the head's tile width (256 for
+ * bf16 caches, 128 for fp32), else CR_ERR_UNSUPPORTED.  Other arguments as
+ * in cr_apply_residual; CR_APPLY_KV with CR_OFFSET_STALE and no kept rows is
+ * cr_apply_residual.  Unknown components or offsets: CR_ERR_INVALID_ARG.
+ */
+cr_status cr_apply_residual_select(const cr_target_dims* target, const cr_repairer_dims* rep,
+                                   const cr_weights* w, const uint16_t* yf, int64_t n_tokens,
+                                   void* kv_inout, const int32_t* pos, const float* inv_freq_host,
+                                   int32_t rope_mode, int32_t components, int32_t offset,
+                                   const int32_t* keep_chunk_id, void* stream);
+
+/*
+ * cr_rotate_k - K_t <- R_M(p_t) K_t on every K segment, V unchanged, in place:
+ * the re-rotation that aligns canonical chunk caches to their request
+ * positions in the stale cache (Sec. 2.2; the inverse of
+ * cr_canonicalize_chunks).  Assembly followed by this call gives the stale
+ * cache KV_stale of independent reuse (the "Stale KV" comparison point).
+ * kv_inout [N, D_KV] cache dtype; pos [N] device int32; inv_freq_host
+ * [head_dim/2] HOST fp32.  Each rotate-half pair is rotated by p_t f_d and
+ * rounded once to the cache dtype.
+ */
+cr_status cr_rotate_k(const cr_target_dims* target, void* kv_inout, int64_t n_tokens,
+                      const int32_t* pos, const float* inv_freq_host, void* stream);
 
 /*
  * cr_apply_residual_paged - the same head and residual add, with the repaired

@@ -24,7 +24,8 @@ CR_EPI_BF16, CR_EPI_GELU_BF16, CR_EPI_ADD_F32, CR_EPI_F32 = range(4)
 
 EXPORTED = [
     "cr_workspace_bytes", "cr_assemble_stale", "cr_compress_features", "cr_repair_forward",
-    "cr_repair_forward_masked", "cr_apply_residual", "cr_apply_residual_paged", "cr_canonicalize_chunks",
+    "cr_repair_forward_masked", "cr_apply_residual", "cr_apply_residual_select", "cr_rotate_k",
+    "cr_apply_residual_paged", "cr_canonicalize_chunks",
     "cr_sigma_workspace_bytes", "cr_sigma_accumulate", "cr_sigma_finalize", "cr_get_device_status",
     "cr_clear_device_status", "cr_status_str", "cr_last_cuda_error",
     "cr_linear", "cr_layernorm", "cr_chunk_causal_attention", "cr_masked_attention",
@@ -98,6 +99,9 @@ def lib(build_if_missing: bool = False) -> ctypes.CDLL:
         "cr_apply_residual_paged": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp,
                                           i64, vp, vp, vp, i32, vp, vp, i64, vp]),
         "cr_canonicalize_chunks": (i32, [P(cr_target_dims), vp, i64, vp, vp, vp]),
+        "cr_rotate_k": (i32, [P(cr_target_dims), vp, i64, vp, vp, vp]),
+        "cr_apply_residual_select": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp,
+                                           i64, vp, vp, vp, i32, i32, i32, vp, vp]),
         "cr_sigma_workspace_bytes": (ctypes.c_size_t, [P(cr_target_dims), i64]),
         "cr_sigma_accumulate": (i32, [P(cr_target_dims), vp, vp, i64, vp, vp, ctypes.c_size_t, vp]),
         "cr_sigma_finalize": (i32, [P(cr_target_dims), vp, i64, vp, vp]),
@@ -252,6 +256,34 @@ def cr_apply_residual(target, rep, weights: PackedWeights, yf, n_tokens, kv_inou
         ctypes.byref(target), ctypes.byref(rep), ctypes.byref(weights.struct), _p(yf), n_tokens,
         _p(kv_inout), _p(pos), None if f is None else f.ctypes.data, rope_mode, _stream(stream))
     _check("cr_apply_residual", st)
+
+
+CR_APPLY_K, CR_APPLY_V, CR_APPLY_KV = 1, 2, 3
+CR_OFFSET_STALE, CR_OFFSET_ZERO = 0, 1
+COMPONENTS = {"k": CR_APPLY_K, "v": CR_APPLY_V, "kv": CR_APPLY_KV}
+OFFSETS = {"stale": CR_OFFSET_STALE, "zero": CR_OFFSET_ZERO}
+
+
+def cr_apply_residual_select(target, rep, weights: PackedWeights, yf, n_tokens, kv_inout, pos,
+                             inv_freq_host=None, rope_mode=CR_ROPE_NONE, component="kv",
+                             offset="stale", keep_chunk_id=None, stream=None):
+    """Head + residual add under an output choice (K only / V only, zero offset,
+    first chunk kept stale when keep_chunk_id is the chunk map)."""
+    f = None if inv_freq_host is None else _host_arr(inv_freq_host, np.float32)
+    comp = COMPONENTS[component] if isinstance(component, str) else int(component)
+    off = OFFSETS[offset] if isinstance(offset, str) else int(offset)
+    st = lib().cr_apply_residual_select(
+        ctypes.byref(target), ctypes.byref(rep), ctypes.byref(weights.struct), _p(yf), n_tokens,
+        _p(kv_inout), _p(pos), None if f is None else f.ctypes.data, rope_mode, comp, off,
+        _p(keep_chunk_id), _stream(stream))
+    _check("cr_apply_residual_select", st)
+
+
+def cr_rotate_k(target, kv_inout, n_tokens, pos, inv_freq_host, stream=None):
+    """K <- R_M(pos) K in place (the stale cache's re-rotation of canonical K)."""
+    f = _host_arr(inv_freq_host, np.float32)
+    _check("cr_rotate_k", lib().cr_rotate_k(
+        ctypes.byref(target), _p(kv_inout), n_tokens, _p(pos), f.ctypes.data, _stream(stream)))
 
 
 def cr_apply_residual_paged(target, rep, weights: PackedWeights, yf, n_tokens, kv_stale, pos,

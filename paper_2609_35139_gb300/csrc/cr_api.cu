@@ -561,6 +561,15 @@ cr_status cr_apply_residual(const cr_target_dims* target, const cr_repairer_dims
                             const cr_weights* w, const uint16_t* yf, int64_t n_tokens,
                             void* kv_inout, const int32_t* pos, const float* inv_freq_host,
                             int32_t rope_mode, void* stream) {
+    return cr_apply_residual_select(target, rep, w, yf, n_tokens, kv_inout, pos, inv_freq_host,
+                                    rope_mode, CR_APPLY_KV, CR_OFFSET_STALE, nullptr, stream);
+}
+
+cr_status cr_apply_residual_select(const cr_target_dims* target, const cr_repairer_dims* rep,
+                                   const cr_weights* w, const uint16_t* yf, int64_t n_tokens,
+                                   void* kv_inout, const int32_t* pos, const float* inv_freq_host,
+                                   int32_t rope_mode, int32_t components, int32_t offset,
+                                   const int32_t* keep_chunk_id, void* stream) {
     cr_status s = check_target(target);
     if (s == CR_OK) s = check_repairer(rep);
     if (s != CR_OK) return s;
@@ -570,8 +579,14 @@ cr_status cr_apply_residual(const cr_target_dims* target, const cr_repairer_dims
     if (!all_aligned(yf, kv_inout, pos, w->w_out, w->b_out, w->sigma_delta))
         return CR_ERR_INVALID_ARG;
     if (rope_mode == CR_ROPE_GLOBAL && !inv_freq_host) return CR_ERR_INVALID_ARG;
+    if (components != CR_APPLY_K && components != CR_APPLY_V && components != CR_APPLY_KV)
+        return CR_ERR_INVALID_ARG;
+    if (offset != CR_OFFSET_STALE && offset != CR_OFFSET_ZERO) return CR_ERR_INVALID_ARG;
+    if (keep_chunk_id && !all_aligned(keep_chunk_id)) return CR_ERR_INVALID_ARG;
     const int bn = d.f32 ? 128 : 256;
     if (d.D % bn != 0) return CR_ERR_UNSUPPORTED;
+    const int64_t plane = static_cast<int64_t>(d.H) * d.dh;   // one (layer, K|V) block
+    if (components != CR_APPLY_KV && plane % bn != 0) return CR_ERR_UNSUPPORTED;
     unsigned* status = device_status_ptr();
     if (!status) return CR_ERR_CUDA;
     GemmParams gp{};
@@ -584,8 +599,34 @@ cr_status cr_apply_residual(const cr_target_dims* target, const cr_repairer_dims
     gp.n_kv_heads = static_cast<int32_t>(d.H);
     if (gp.rope_on)
         for (int i = 0; i < d.dh / 2; ++i) gp.inv_freq[i] = inv_freq_host[i];
-    return launch_gemm(yf, d.db, w->w_out, n_tokens, d.D, d.db, d.f32 ? EPI_KV_F32 : EPI_KV_BF16,
-                       gp, kv_inout, d.D, static_cast<cudaStream_t>(stream));
+    if (components != CR_APPLY_KV) {
+        gp.col_block = static_cast<int32_t>(plane);
+        gp.col_phase = components == CR_APPLY_K ? 0 : 1;
+    }
+    gp.kv_zero = offset == CR_OFFSET_ZERO ? 1 : 0;
+    gp.keep_chunk = keep_chunk_id;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    s = launch_gemm(yf, d.db, w->w_out, n_tokens, d.D, d.db, d.f32 ? EPI_KV_F32 : EPI_KV_BF16, gp,
+                    kv_inout, d.D, st);
+    // V-only under the target's R_M: the K segments the head did not visit are
+    // still rotated to their request positions
+    if (s == CR_OK && gp.rope_on && components == CR_APPLY_V)
+        s = launch_canonicalize(kv_inout, d.f32, n_tokens, pos, static_cast<int>(d.L),
+                                static_cast<int>(d.H), static_cast<int>(d.dh), inv_freq_host, st,
+                                -1.0f);
+    return s;
+}
+
+cr_status cr_rotate_k(const cr_target_dims* target, void* kv_inout, int64_t n_tokens,
+                      const int32_t* pos, const float* inv_freq_host, void* stream) {
+    const cr_status s = check_target(target);
+    if (s != CR_OK) return s;
+    if (n_tokens < 1 || !inv_freq_host || !all_aligned(kv_inout, pos)) return CR_ERR_INVALID_ARG;
+    const Dims d = dims_of(target, nullptr);
+    if (n_tokens > INT64_MAX / (d.D * 4)) return CR_ERR_INVALID_ARG;
+    return launch_canonicalize(kv_inout, d.f32, n_tokens, pos, static_cast<int>(d.L),
+                               static_cast<int>(d.H), static_cast<int>(d.dh), inv_freq_host,
+                               static_cast<cudaStream_t>(stream), -1.0f);
 }
 
 cr_status cr_apply_residual_paged(const cr_target_dims* target, const cr_repairer_dims* rep,

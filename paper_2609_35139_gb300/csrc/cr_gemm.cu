@@ -196,6 +196,22 @@ __device__ __forceinline__ void vec16(const float* v, int col, float* out) {
     }
 }
 
+// First output column of tile t.  Tiles are walked W-tile-major (t / num_m is
+// the column tile); under an output choice (KV epilogues with col_block > 0)
+// only the K or only the V column blocks are walked.
+template <int BN, bool KV>
+__device__ __forceinline__ int tile_n0(const GemmParams& p, int t) {
+    const int c = t / p.num_m;
+    if constexpr (KV) {
+        if (p.col_block > 0) {
+            const int per = p.col_block / BN;   // column tiles per block
+            const int blk = c / per;
+            return (2 * blk + p.col_phase) * p.col_block + (c - blk * per) * BN;
+        }
+    }
+    return c * BN;
+}
+
 __device__ __forceinline__ void rotate16(float* a, float* b, float p, const float* inv_freq, int j0) {
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
@@ -282,6 +298,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const bool has_bias = p.bias != nullptr;
     // the epilogue consumes a per-tile load (vectors and/or the in-place tile)
     const bool epi_load = Cfg::kInPlace || has_bias;
+    // the in-place tile is read unless a zero output offset makes every row's
+    // stale value unused (no kept rows)
+    const bool load_tile = Cfg::kInPlace && !(Cfg::kKV && p.kv_zero && p.keep_chunk == nullptr);
 
     // The producer, loader, store and MMA roles each run as a converged warp
     // (operands stay warp-uniform); one elected lane issues the copies and MMAs.
@@ -299,7 +318,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         bool ok = true;
         for (int t = cta0; t < total && ok; t += ncta) {
             const int m0 = (t % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-            const int n0 = (t / p.num_m) * BN;
+            const int n0 = tile_n0<BN, Cfg::kKV>(p, t);
             for (int kb = 0; kb < num_k; ++kb) {
                 if (!(ok = mbar_wait_warp(&empty[stage], phase ^ 1u, wc, 102))) break;
                 uint8_t* sa = smem + stage * Cfg::kStageBytes;
@@ -342,16 +361,16 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             int i = 0;
             for (int t = cta0; t < total; t += ncta, ++i) {
                 const int m0 = (t % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-                const int n0 = (t / p.num_m) * BN;
+                const int n0 = tile_n0<BN, Cfg::kKV>(p, t);
                 if (!(ok = mbar_wait_warp(epi_empty, (static_cast<uint32_t>(i) & 1u) ^ 1u, wc, 101)))
                     break;
                 const int nb = min(BN, p.N - n0);
                 const uint32_t vbytes = static_cast<uint32_t>(nb) * 4u;
-                uint32_t bytes = (Cfg::kInPlace ? Cfg::kTileBytes : 0u) + (has_bias ? vbytes : 0u);
+                uint32_t bytes = (load_tile ? Cfg::kTileBytes : 0u) + (has_bias ? vbytes : 0u);
                 if constexpr (Cfg::kKV) bytes += vbytes;
                 if (elect_one()) {
                     mbar_expect_tx(epi_full, bytes);
-                    if constexpr (Cfg::kInPlace) {
+                    if (load_tile) {
                         for (int b = 0; b < Cfg::kBoxes; ++b)
                             tma_load_2d(tile + b * 16384, &tmC, epi_full, n0 + b * Cfg::kBoxCols, m0);
                     }
@@ -378,7 +397,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         uint32_t pkg[2] = {0u, 0u};    // boxes of each epilogue group so far
         for (int t = cta0; t < total && ok; t += ncta) {
             const int m0 = (t % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-            const int n0 = (t / p.num_m) * BN;
+            const int n0 = tile_n0<BN, Cfg::kKV>(p, t);
             const bool rows_in = m0 < p.M;   // a pair tile's second half may lie below M
             if constexpr (Cfg::kInPlace) {
                 if (!(ok = mbar_wait_warp(&epi_done[0], pk & 1u, wc, 401))) break;
@@ -495,7 +514,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         int i = 0;
         for (int t = cta0; t < total && ok; t += ncta, ++i) {
             const int m0 = (t % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-            const int n0 = (t / p.num_m) * BN;
+            const int n0 = tile_n0<BN, Cfg::kKV>(p, t);
             ok = mbar_wait(&tfull[acc], acc_phase, wc, 301);
             if (epi_load) ok = ok && mbar_wait(epi_full, static_cast<uint32_t>(i) & 1u, wc, 302);
             if (!__all_sync(0xffffffffu, ok)) {
@@ -508,6 +527,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             const uint32_t taddr = tmem_base + ((quad * 32u) << 16) + acc * BN;
 
             if constexpr (Cfg::kInPlace) {
+                // output choices: a kept row (first chunk) leaves its stale value,
+                // a zero output offset drops the stale value from the sum
+                bool keep = false, zero = false;
+                if constexpr (Cfg::kKV) {
+                    keep = p.keep_chunk != nullptr && row_ok && __ldg(p.keep_chunk + row) == 0;
+                    zero = p.kv_zero != 0 && !keep;
+                }
                 // where a repaired 16-column chunk goes: back into the staged tile
                 // (stored in place by TMA), or straight to the token's row of its
                 // (layer, K|V) plane in the paged target cache
@@ -543,8 +569,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                             __syncwarp();
                             tmem_ld16(taddr + ta, a);
                             tmem_ld16(taddr + tb, b);
-                            load16_tile<ES>(tile, r, ta, ka);
-                            load16_tile<ES>(tile, r, tb, kb);
+                            if (zero) {
+#pragma unroll
+                                for (int q = 0; q < 16; ++q) ka[q] = kb[q] = 0.0f;
+                            } else {
+                                load16_tile<ES>(tile, r, ta, ka);
+                                load16_tile<ES>(tile, r, tb, kb);
+                            }
                             vec16(vs, ta, sa_);
                             vec16(vs, tb, sb_);
                             if (has_bias) {
@@ -555,10 +586,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                                 for (int q = 0; q < 16; ++q) ba[q] = bb[q] = 0.0f;
                             }
                             tmem_wait_ld();
+                            if (!keep) {
 #pragma unroll
-                            for (int q = 0; q < 16; ++q) {
-                                ka[q] = fmaf(sa_[q], a[q] + ba[q], ka[q]);
-                                kb[q] = fmaf(sb_[q], b[q] + bb[q], kb[q]);
+                                for (int q = 0; q < 16; ++q) {
+                                    ka[q] = fmaf(sa_[q], a[q] + ba[q], ka[q]);
+                                    kb[q] = fmaf(sb_[q], b[q] + bb[q], kb[q]);
+                                }
                             }
                             if (rot) rotate16(ka, kb, pr, p.inv_freq, j);
                             put16(ta, ka);
@@ -571,7 +604,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                         float a[16], k[16], bv[16];
                         __syncwarp();
                         tmem_ld16(taddr + c, a);
-                        load16_tile<ES>(tile, r, c, k);
+                        if (zero) {
+#pragma unroll
+                            for (int q = 0; q < 16; ++q) k[q] = 0.0f;
+                        } else {
+                            load16_tile<ES>(tile, r, c, k);
+                        }
                         if (has_bias) {
                             vec16(vb, c, bv);
                         } else {
@@ -580,10 +618,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                         }
                         tmem_wait_ld();
                         if constexpr (Cfg::kKV) {
-                            float sv[16];
-                            vec16(vs, c, sv);
+                            if (!keep) {
+                                float sv[16];
+                                vec16(vs, c, sv);
 #pragma unroll
-                            for (int q = 0; q < 16; ++q) k[q] = fmaf(sv[q], a[q] + bv[q], k[q]);
+                                for (int q = 0; q < 16; ++q) k[q] = fmaf(sv[q], a[q] + bv[q], k[q]);
+                            }
                         } else {
 #pragma unroll
                             for (int q = 0; q < 16; ++q) k[q] += a[q] + bv[q];
@@ -830,6 +870,14 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
     p.K = static_cast<int32_t>(K);
     p.num_m = static_cast<int32_t>((M + BM * kCG - 1) / (BM * kCG));
     p.num_n = static_cast<int32_t>((N + BN - 1) / BN);
+    if (kv && p.col_block > 0) {
+        // output choice: half of the column blocks, each a whole number of tiles
+        if (p.col_block % BN != 0 || N % (2 * static_cast<int64_t>(p.col_block)) != 0)
+            return CR_ERR_UNSUPPORTED;
+        p.num_n = static_cast<int32_t>(N / 2 / BN);
+    } else {
+        p.col_block = 0;
+    }
     CUtensorMap ta, tb, tc;
     if (!make_tmap_2d(&ta, A, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, K, M, lda * 2, BK, BM,
                       CU_TENSOR_MAP_SWIZZLE_128B))

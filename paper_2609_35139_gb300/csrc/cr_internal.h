@@ -74,6 +74,15 @@ struct GemmParams {
     uint16_t* paged;         // KV_PAGED: [N / seg_width][num_slots][seg_width] bf16
     int64_t num_slots;       // KV_PAGED: slots per (layer, K|V) plane
     int32_t seg_width;       // KV_PAGED: H_kv * d_h, the columns of one (layer, K|V) plane
+    // KV output choices (App. F): only the column blocks [b w, (b + 1) w), w =
+    // col_block, with b % 2 == col_phase (0: K, 1: V) are visited, or every
+    // column if col_block == 0; kv_zero: zero output offset (A5), sigma (z + b)
+    // replaces kv + sigma (z + b); rows t with keep_chunk[t] == 0 (the first
+    // chunk) keep their stale value, if keep_chunk is given.
+    int32_t col_block;
+    int32_t col_phase;
+    int32_t kv_zero;
+    const int32_t* keep_chunk;
     unsigned* status;
     float inv_freq[64];      // RoPE frequencies, rope_dim / 2 entries
 };
@@ -155,8 +164,10 @@ constexpr int64_t kSigmaSlice = 64;
 
 // Launchers (validated arguments).
 cr_status launch_gather(const GatherParams& p, cudaStream_t st);
+// K segments rotated in place by R_M(dir * (-pos)): dir = +1 canonicalises
+// (R_M(q)^{-1}), dir = -1 applies R_M(p).
 cr_status launch_canonicalize(void* kv, bool f32, int64_t n, const int32_t* pos, int L, int H, int dh,
-                              const float* inv_freq_host, cudaStream_t st);
+                              const float* inv_freq_host, cudaStream_t st, float dir = 1.0f);
 cr_status launch_sigma_accumulate(const void* a, const void* b, bool f32, int64_t n, int64_t D,
                                   float* part, double* sumsq, cudaStream_t st);
 cr_status launch_sigma_finalize(const double* sumsq, int64_t D, int64_t count, float* sigma,

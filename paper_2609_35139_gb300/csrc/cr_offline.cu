@@ -43,12 +43,14 @@ __device__ __forceinline__ void store8(float* p, const float* v) {
 // 8 angles q_t * f_d are computed once and applied to that group in the K
 // segments of the thread's layers (rotate-half pairs (d, d + d_h/2) inside
 // each d_h-wide segment, by -q_t f_d: (a, b) -> (a cos + b sin, b cos - a sin)),
-// one rounding to the cache dtype.  Two segments are loaded before either is
+// one rounding to the cache dtype.  With dir = -1 the sine changes sign and the
+// rotation is by +q_t f_d, R_M itself (the stale cache's re-rotation of K to
+// request positions, Sec. 2.2).  Two segments are loaded before either is
 // rotated, for memory-level parallelism.
 template <typename T>
 __global__ void __launch_bounds__(256) canon_kernel(T* kv, int64_t n, const int32_t* __restrict__ pos,
                                                     int L, int H, int dh,
-                                                    const __grid_constant__ Freq f) {
+                                                    const __grid_constant__ Freq f, float dir) {
     pdl_launch_dependents();
     pdl_wait();
     const int groups = dh / 16;
@@ -64,7 +66,10 @@ __global__ void __launch_bounds__(256) canon_kernel(T* kv, int64_t n, const int3
         const float q = static_cast<float>(__ldg(pos + t));
         float c[8], s[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) sincos_prod(q, f.f[g * 8 + i], &s[i], &c[i]);
+        for (int i = 0; i < 8; ++i) {
+            sincos_prod(q, f.f[g * 8 + i], &s[i], &c[i]);
+            s[i] *= dir;
+        }
         T* row = kv + t * D;
         // the K segments (layer l, head h) of this part, l in [l0, l1)
         const int l0 = part * L / kParts, l1 = (part + 1) * L / kParts;
@@ -168,7 +173,7 @@ __global__ void __launch_bounds__(256) sigma_finalize_kernel(const double* __res
 }  // namespace
 
 cr_status launch_canonicalize(void* kv, bool f32, int64_t n, const int32_t* pos, int L, int H, int dh,
-                              const float* inv_freq_host, cudaStream_t st) {
+                              const float* inv_freq_host, cudaStream_t st, float dir) {
     if (n <= 0) return CR_OK;
     if (dh != 64 && dh != 128) return CR_ERR_UNSUPPORTED;
     Freq f{};
@@ -179,9 +184,9 @@ cr_status launch_canonicalize(void* kv, bool f32, int64_t n, const int32_t* pos,
     const dim3 grid(static_cast<unsigned>(blocks)), block(256);
     if (f32)
         return launch_pdl(canon_kernel<float>, grid, block, 0, st, static_cast<float*>(kv), n, pos, L, H,
-                          dh, f);
+                          dh, f, dir);
     return launch_pdl(canon_kernel<uint16_t>, grid, block, 0, st, static_cast<uint16_t*>(kv), n, pos, L,
-                      H, dh, f);
+                      H, dh, f, dir);
 }
 
 cr_status launch_sigma_accumulate(const void* a, const void* b, bool f32, int64_t n, int64_t D,

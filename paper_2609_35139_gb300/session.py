@@ -75,9 +75,23 @@ class RepairSession:
                                         self.chunk_end, self.pos, a.cu_seqlens, a.n_tokens,
                                         mask_mode, self.yf, self.workspace, stream)
 
-    def apply(self, a: Assembled, inv_freq_target=None, rope_mode=cr.CR_ROPE_NONE, stream=None):
-        cr.cr_apply_residual(self.target, self.rep, self.weights, self.yf, a.n_tokens, self.kv,
-                             self.pos, inv_freq_target, rope_mode, stream)
+    def apply(self, a: Assembled, inv_freq_target=None, rope_mode=cr.CR_ROPE_NONE, stream=None,
+              component="kv", offset="stale", keep_first_chunk=False):
+        """Head and residual add in place on kv.  The defaults are the method; the
+        output choices (App. F) repair only K or only V, drop the stale offset (A5),
+        or keep each request's first chunk stale."""
+        if component == "kv" and offset == "stale" and not keep_first_chunk:
+            cr.cr_apply_residual(self.target, self.rep, self.weights, self.yf, a.n_tokens, self.kv,
+                                 self.pos, inv_freq_target, rope_mode, stream)
+        else:
+            cr.cr_apply_residual_select(self.target, self.rep, self.weights, self.yf, a.n_tokens,
+                                        self.kv, self.pos, inv_freq_target, rope_mode, component,
+                                        offset, self.chunk_id if keep_first_chunk else None, stream)
+
+    def stale_kv(self, a: Assembled, inv_freq_target, stream=None):
+        """The stale cache of independent reuse: the assembled canonical cache with K
+        rotated to its request positions (no repair), in place on kv."""
+        cr.cr_rotate_k(self.target, self.kv, a.n_tokens, self.pos, inv_freq_target, stream)
 
     def apply_paged(self, a: Assembled, slot_mapping: torch.Tensor, paged_cache: torch.Tensor,
                     num_slots: int, inv_freq_target=None, rope_mode=cr.CR_ROPE_NONE, stream=None):

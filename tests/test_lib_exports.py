@@ -140,6 +140,26 @@ def test_mask_calls_reject_bad_inputs_on_host(L):
                                       None) == cr.CR_ERR_INVALID_ARG
 
 
+def test_output_choice_calls_reject_bad_inputs_on_host(L):
+    c, (t, r) = _dims()
+    w = cr.cr_weights()
+    w.w_out = w.b_out = w.sigma_delta = FAKE
+    sel = lambda tt, comp=3, off=0, keep=None, rope=0, freq=None: L.cr_apply_residual_select(
+        ctypes.byref(tt), ctypes.byref(r), ctypes.byref(w), FAKE, 10, FAKE, FAKE, freq, rope, comp,
+        off, keep, None)
+    for comp in (0, 4, -1):
+        assert sel(t, comp=comp) == cr.CR_ERR_INVALID_ARG
+    assert sel(t, off=2) == cr.CR_ERR_INVALID_ARG
+    assert sel(t, keep=FAKE + 4) == cr.CR_ERR_INVALID_ARG                 # misaligned chunk map
+    assert sel(t, rope=cr.CR_ROPE_GLOBAL) == cr.CR_ERR_INVALID_ARG         # R_M needs frequencies
+    one_head = cr.target_dims(4, 1, 128, 512, "bf16")                      # H d_h = 128 < 256
+    assert sel(one_head, comp=cr.CR_APPLY_K) == cr.CR_ERR_UNSUPPORTED
+    f = np.ones(64, np.float32)
+    assert L.cr_rotate_k(ctypes.byref(t), FAKE, 10, FAKE, None, None) == cr.CR_ERR_INVALID_ARG
+    assert L.cr_rotate_k(ctypes.byref(t), FAKE + 8, 10, FAKE, f.ctypes.data, None) == cr.CR_ERR_INVALID_ARG
+    assert L.cr_rotate_k(ctypes.byref(t), FAKE, 0, FAKE, f.ctypes.data, None) == cr.CR_ERR_INVALID_ARG
+
+
 def test_paged_residual_rejects_bad_inputs_on_host(L):
     c, (t, r) = _dims()
     w = cr.cr_weights()
