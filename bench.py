@@ -11,6 +11,12 @@ pool (1 GiB) and the assembled cache (0.67 GB) exceed the 129 MB L2, so no
 explicit L2 flush is needed between steps.
 
     python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+                    [--mask MODE] [--component kv|k|v] [--offset stale|zero]
+                    [--keep-first-chunk] [--rope]
+
+The last options time the attention-mask and output variants of App. F (and
+the target's R_M on K) in place of the method's defaults; a variant run
+names itself in config.variant and reports no e2e figure.
 
 For N > 1 (torchrun, one process per GPU) every rank repairs its own request
 stream with a weight replica: requests never interact, so there is no
@@ -40,10 +46,33 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="llama8b")
+    ap.add_argument("--chunks", type=int, default=None,
+                    help="request of this many chunks instead of the workload's (same shapes; "
+                         "a smaller case for profiling)")
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    return ap.parse_args()
+    ap.add_argument("--mask", default="block_causal",
+                    choices=["block_causal", "token_causal", "bidirectional", "block_diagonal"])
+    ap.add_argument("--component", default="kv", choices=["kv", "k", "v"])
+    ap.add_argument("--offset", default="stale", choices=["stale", "zero"])
+    ap.add_argument("--keep-first-chunk", action="store_true")
+    ap.add_argument("--rope", action="store_true", help="apply the target's R_M to K after repair")
+    args = ap.parse_args()
+    args.variant = {k: v for k, v in (("mask", args.mask), ("component", args.component),
+                                      ("offset", args.offset))
+                    if v != {"mask": "block_causal", "component": "kv", "offset": "stale"}[k]}
+    if args.keep_first_chunk:
+        args.variant["keep_first_chunk"] = True
+    if args.rope:
+        args.variant["target_rope"] = True
+    return args
+
+
+def make_workload(F, args):
+    if args.chunks is None:
+        return F.make_case(args.workload)
+    return F.make_case(args.workload, n_req_chunks=args.chunks, requests=None, batched=None)
 
 
 def load_peaks():
@@ -135,7 +164,7 @@ def stop_clocks(handle, t_begin=None, t_end=None):
             "samples_in_timed_region": in_region}
 
 
-def oracle_sample(case, n_chunks, max_tokens=None):
+def oracle_sample(case, n_chunks, max_tokens=None, mask="block_causal"):
     """Run the oracle on the first n_chunks of request 0 (a document prefix), cut to
     max_tokens tokens if given; returns (tokens, seconds)."""
     import numpy as np
@@ -157,7 +186,7 @@ def oracle_sample(case, n_chunks, max_tokens=None):
     t0 = time.perf_counter()
     O.repair_request(kv, emb, cid, pos, case.weights, cache_dtype=t.cache_dtype,
                      n_layers=t.n_layers, n_kv_heads=t.n_kv_heads, head_dim=t.head_dim,
-                     n_heads=r.n_heads)
+                     n_heads=r.n_heads, mask_mode=mask)
     return len(cid), time.perf_counter() - t0
 
 
@@ -166,14 +195,14 @@ def run_reference(args):
     if rank != 0:
         return
     import fixtures as F
-    case = F.make_case(args.workload)
+    case = make_workload(F, args)
     n_chunks = 1
     # each step repairs a prefix of the first chunk, sized so that the K timed
     # steps take about a minute of host time at any K
     cap = max(32, min(512, 25600 // max(args.steps, 1)))
     times, toks = [], 0
     for i in range(args.warmup + args.steps):
-        n, s = oracle_sample(case, n_chunks, cap)
+        n, s = oracle_sample(case, n_chunks, cap, args.mask)
         if i >= args.warmup:
             times.append(s)
             toks = n
@@ -213,7 +242,7 @@ def run_ours(args):
     cr.lib()
     cr.cr_clear_device_status()
 
-    case = F.make_case(args.workload)
+    case = make_workload(F, args)
     t, r = dims_from(case.target, case.repairer)
     pw = pack_host_weights(case.weights, case.repairer.n_blocks)
     p = case.plan
@@ -225,16 +254,21 @@ def run_ours(args):
     sess = RepairSession(t, r, pw, max_tokens=N)
     stream = torch.cuda.current_stream()
 
+    rope_mode = cr.CR_ROPE_GLOBAL if args.rope else cr.CR_ROPE_NONE
+    freq = case.inv_freq_target if args.rope else None
+    choice = dict(component=args.component, offset=args.offset, keep_first_chunk=args.keep_first_chunk)
+
     def step():
-        sess.repair(kvp, embp, p.chunk_start, p.chunk_len, p.chunk_idx, p.cu_chunks)
+        sess.repair(kvp, embp, p.chunk_start, p.chunk_len, p.chunk_idx, p.cu_chunks, freq, rope_mode,
+                    mask_mode=args.mask, **choice)
 
     # ---- per-call timing (eager), for the stage breakdown and the roofline
     a = sess.assemble(kvp, embp, p.chunk_start, p.chunk_len, p.chunk_idx, p.cu_chunks)
     calls = [("assemble", lambda: sess.assemble(kvp, embp, p.chunk_start, p.chunk_len,
                                                 p.chunk_idx, p.cu_chunks)),
              ("compress", lambda: sess.compress(a)),
-             ("forward", lambda: sess.forward(a)),
-             ("apply", lambda: sess.apply(a))]
+             ("forward", lambda: sess.forward(a, mask_mode=args.mask)),
+             ("apply", lambda: sess.apply(a, freq, rope_mode, **choice))]
     for _ in range(3):
         for _, fn in calls:
             fn()
@@ -293,32 +327,37 @@ def run_ours(args):
 
     # ---- end to end through the public API with host buffers
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and not args.variant:
         e2e = run_e2e(case, sess, kvp_h, embp_h, args, world)
 
     # ---- per-kernel rooflines; the one with the most time per step is reported
     hbm, tf_burst, tf_sus, src = load_peaks()
     tg, rp = case.target, case.repairer
     es = 2 if tg.cache_dtype == "bf16" else 4
-    head_flops = 2.0 * N * rp.d_b * tg.d_kv
-    head_ms = stages["apply"]                       # cr_apply_residual is one kernel launch
-    attn_flops, attn_ms = attention_timing(case, sess, a)
+    head_cols = tg.d_kv if args.component == "kv" else tg.d_kv // 2
+    head_flops = 2.0 * N * rp.d_b * head_cols
+    # cr_apply_residual is one kernel launch (a V-only choice under R_M adds the K rotation)
+    head_ms = stages["apply"]
+    attn_flops, attn_ms = attention_timing(case, sess, a, args.mask)
     gather_bytes = 2.0 * N * (tg.d_kv + tg.d_model) * es
     kernels = {
-        "attn_kernel": dict(name="attn_kernel (block-causal flash attention)", launches=rp.n_blocks,
+        "attn_kernel": dict(name=f"attn_kernel ({args.mask.replace('_', '-')} flash attention)",
+                            launches=rp.n_blocks,
                             ms=attn_ms, flops=attn_flops,
                             algorithmic=f"4*d_b per visible (query, key) pair = {attn_flops:.3e} "
                                         f"flop per launch"),
         "gemm_kernel<256,KV>": dict(name="cr_apply_residual (KV residual head GEMM + residual add)",
                                     launches=1, ms=head_ms, flops=head_flops,
-                                    algorithmic=f"2*N*d_b*D_KV = {head_flops:.3e} flop per launch"),
+                                    algorithmic=f"2*N*d_b*(columns visited) = {head_flops:.3e} "
+                                                f"flop per launch"),
     }
     dom_key = max(kernels, key=lambda k: kernels[k]["launches"] * kernels[k]["ms"])
     dom = kernels[dom_key]
     achieved = dom["flops"] / (dom["ms"] * 1e-3) / 1e12
     roofline = {"kernel": dom["name"], "bound": "tensor", "achieved": achieved, "peak": tf_sus,
                 "unit": "TFLOP/s", "frac": achieved / tf_sus,
-                "traffic": traffic_from_profiles(dom_key),
+                # DRAM counters were taken on the method's workload, not on a variant
+                "traffic": None if args.variant else traffic_from_profiles(dom_key),
                 "peak_source": f"{src} bf16_tflops_sustained (kernel timed inside the step loop)",
                 "algorithmic": dom["algorithmic"], "launch_ms": dom["ms"],
                 "launches_per_step": dom["launches"]}
@@ -332,10 +371,12 @@ def run_ours(args):
     }
     launches_per_step = 1 + (2 + 4 + (2 if tg.cache_dtype == "f32" else 0) - (1 if rp.n_blocks == 0 else 0)) \
         + 7 * rp.n_blocks + 1 + 1
+    launches_per_step += 1 if (args.mask == "block_diagonal" and rp.n_blocks > 0) else 0
+    launches_per_step += 1 if (args.rope and args.component == "v") else 0
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         n_chunks = 2
-        ntok, secs = oracle_sample(case, n_chunks)
+        ntok, secs = oracle_sample(case, n_chunks, mask=args.mask)
         cpu = {"value": ntok / secs, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
                "sample": f"first {n_chunks} chunks ({ntok} tokens) of the request, full repair "
                          f"incl. head, float64 numpy, {secs:.1f} s"}
@@ -349,7 +390,8 @@ def run_ours(args):
             "data": "synthetic (seeded caches, embeddings, chunk map; random-init Xavier repairer)",
             "config": {"workload": workload_desc(case), "n_tokens": N, "cuda_graph": use_graph,
                        "l2": "no flush: pool 1 GiB and assembled cache 0.67 GB exceed L2",
-                       "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+                       "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                       **({"variant": args.variant} if args.variant else {})},
             "roofline": roofline, "stage_roofline": stage_roofline,
             "stages_ms": stages, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": launches_per_step * args.steps, "clocks": clocks,
@@ -359,10 +401,10 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
-def attention_timing(case, sess, a, iters=10):
-    """Per-launch time of the block-causal attention kernel at this workload's shapes
-    (same chunk map, same launch configuration as inside cr_repair_forward) and its
-    algorithmic flops: 4 d_b per visible (query, key) pair."""
+def attention_timing(case, sess, a, mask="block_causal", iters=10):
+    """Per-launch time of the attention kernel at this workload's shapes (same chunk
+    map, mask and launch configuration as inside the forward) and its algorithmic
+    flops: 4 d_b per visible (query, key) pair."""
     import numpy as np
     import torch
     from paper_2609_35139_gb300 import cr
@@ -370,7 +412,10 @@ def attention_timing(case, sess, a, iters=10):
     N = a.n_tokens
     qkv = torch.randn(N, 3 * rp.d_b, device="cuda").to(torch.bfloat16)
     out = torch.empty(N, rp.d_b, device="cuda", dtype=torch.bfloat16)
-    run = lambda: cr.cr_chunk_causal_attention(qkv, rp.d_b, rp.n_heads, sess.chunk_end, a.cu_seqlens, out)
+    starts = torch.empty(N, dtype=torch.int32, device="cuda")
+    cr.cr_chunk_starts(sess.chunk_end, a.cu_seqlens, N, starts)
+    run = lambda: cr.cr_masked_attention(qkv, rp.d_b, rp.n_heads, mask, sess.chunk_end, starts,
+                                         a.cu_seqlens, out)
     for _ in range(3):
         run()
     torch.cuda.synchronize()
@@ -381,8 +426,14 @@ def attention_timing(case, sess, a, iters=10):
         run()
     e1.record(stream)
     torch.cuda.synchronize()
-    visible = int(sess.chunk_end[:N].to(torch.int64).sum().item())   # sum_i chunk_end(i)
-    return 4.0 * rp.d_b * visible, e0.elapsed_time(e1) / iters
+    cend = sess.chunk_end[:N].to(torch.int64).cpu().numpy()
+    cstart = starts[:N].to(torch.int64).cpu().numpy()
+    cu = np.asarray(a.cu_seqlens, np.int64)
+    local = np.arange(N) - np.repeat(cu[:-1], np.diff(cu))
+    lens = np.repeat(np.diff(cu), np.diff(cu))
+    visible = {"block_causal": cend, "token_causal": local + 1, "bidirectional": lens,
+               "block_diagonal": cend - cstart}[mask]
+    return 4.0 * rp.d_b * float(visible.sum()), e0.elapsed_time(e1) / iters
 
 
 def traffic_from_profiles(kernel_key):

@@ -102,12 +102,16 @@ class RepairSession:
                                    rope_mode, stream)
 
     def repair(self, kv_pool, emb_pool, chunk_start, chunk_len, chunk_idx, cu_chunks,
-               inv_freq_target=None, rope_mode=cr.CR_ROPE_NONE, stream=None) -> Assembled:
-        """Assemble, compress, run the blocks and apply the residual; kv holds the result."""
+               inv_freq_target=None, rope_mode=cr.CR_ROPE_NONE, stream=None,
+               mask_mode="block_causal", component="kv", offset="stale",
+               keep_first_chunk=False) -> Assembled:
+        """Assemble, compress, run the blocks and apply the residual; kv holds the result.
+        The keyword options select the App. F mask and output variants (defaults: the method)."""
         a = self.assemble(kv_pool, emb_pool, chunk_start, chunk_len, chunk_idx, cu_chunks, stream)
         self.compress(a, stream)
-        self.forward(a, stream)
-        self.apply(a, inv_freq_target, rope_mode, stream)
+        self.forward(a, stream, mask_mode=mask_mode)
+        self.apply(a, inv_freq_target, rope_mode, stream, component=component, offset=offset,
+                   keep_first_chunk=keep_first_chunk)
         return a
 
 
