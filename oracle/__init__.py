@@ -8,3 +8,4 @@ with it.
 from .cacherepair import *  # noqa: F401,F403
 from .offline import *  # noqa: F401,F403
 from .variants import *  # noqa: F401,F403
+from .training import *  # noqa: F401,F403
