@@ -12,11 +12,12 @@ explicit L2 flush is needed between steps.
 
     python bench.py [--gpus N --steps K --warmup W] [--impl reference]
                     [--mask MODE] [--component kv|k|v] [--offset stale|zero]
-                    [--keep-first-chunk] [--rope]
+                    [--keep-first-chunk] [--rope] [--train]
 
 The last options time the attention-mask and output variants of App. F (and
 the target's R_M on K) in place of the method's defaults; a variant run
-names itself in config.variant and reports no e2e figure.
+names itself in config.variant and reports no e2e figure.  --train times one
+AdamW update of the repair network per step instead (Sec. 4.2, App. A).
 
 For N > 1 (torchrun, one process per GPU) every rank repairs its own request
 stream with a weight replica: requests never interact, so there is no
@@ -58,6 +59,8 @@ def parse():
     ap.add_argument("--offset", default="stale", choices=["stale", "zero"])
     ap.add_argument("--keep-first-chunk", action="store_true")
     ap.add_argument("--rope", action="store_true", help="apply the target's R_M to K after repair")
+    ap.add_argument("--train", action="store_true",
+                    help="time one training update (forward, objective, backward, AdamW) per step")
     args = ap.parse_args()
     args.variant = {k: v for k, v in (("mask", args.mask), ("component", args.component),
                                       ("offset", args.offset))
@@ -505,10 +508,108 @@ def run_e2e(case, sess, kvp_h, embp_h, args, world):
                     "two slots, transfers overlapped with the neighbouring requests' repairs"}
 
 
+def train_flops(case, visible_pairs):
+    """Algorithmic flops of one update: the forward's linears, head, segment projection and
+    attention (visible pairs only), and the backward's two products per linear (dX, dW; the
+    segment projection needs dW only), the FC1 recompute and 2.5x the attention's work
+    (S again, dV, dP, dQ, dK against S and PV forward)."""
+    t, r = case.target, case.repairer
+    N = case.plan.n_tokens
+    S = 2 * t.n_layers * t.n_kv_heads
+    dc, db, B, hid = r.d_c, r.d_b, r.n_blocks, r.mlp_hidden
+    lin = 2.0 * N * (S * r.d_seg * dc + t.d_model * dc + 2 * dc * db + B * dc * db
+                     + B * (4 * db * db + 2 * hid * db))
+    head = 2.0 * N * db * t.d_kv
+    seg = 2.0 * N * t.d_kv * r.d_seg
+    attn = B * 4.0 * db * visible_pairs
+    return 3 * lin + 3 * head + 2 * seg + 2.0 * N * db * hid * B + 3.5 * attn
+
+
+def run_train(args):
+    """One AdamW update of the repair network per step (Sec. 4.2, App. A) on the
+    workload's request against a seeded synthetic joint cache (stale + sigma_Delta noise),
+    through cr_train_step: eager launches, the backward's plain GEMMs in cuBLAS."""
+    import numpy as np
+    import torch
+
+    import fixtures as F
+    from paper_2609_35139_gb300 import RepairSession, TrainSession, build, cr, dims_from, pack_host_weights
+
+    if int(os.environ.get("WORLD_SIZE", "1")) > 1:
+        raise SystemExit("--train runs on one GPU: data-parallel training would need a gradient "
+                         "all-reduce, which is not built")
+    torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+    build.build()
+    cr.lib()
+    cr.cr_clear_device_status()
+    case = make_workload(F, args)
+    t, r = dims_from(case.target, case.repairer)
+    p = case.plan
+    kvp_h, embp_h = case.pool()
+    to_dev = lambda a: (torch.from_numpy(a.view(np.int16)).view(torch.bfloat16)
+                        if a.dtype == np.uint16 else torch.from_numpy(a)).cuda()
+    N = p.n_tokens
+    sess = RepairSession(t, r, pack_host_weights(case.weights, case.repairer.n_blocks), max_tokens=N)
+    a = sess.assemble(to_dev(kvp_h), to_dev(embp_h), p.chunk_start, p.chunk_len, p.chunk_idx, p.cu_chunks)
+    kv = sess.kv[:N]
+    g = torch.Generator(device="cuda").manual_seed(7)
+    sd = torch.from_numpy(case.weights["sigma_delta"]).cuda()
+    joint = (kv.float() + sd[None] * torch.randn(kv.shape, device="cuda", generator=g)).to(torch.bfloat16)
+    lens = np.diff(a.cu_seqlens)
+    ts = TrainSession(t, r, case.weights, N, int(lens.max()))
+    del sess.h0, sess.rein, sess.yf, sess.workspace
+    step = lambda: ts.step(kv, joint, sess.emb[:N], sess.chunk_end[:N], sess.pos[:N], a.cu_seqlens, N, 3e-4)
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    loss0 = float(ts.stats[0].item())
+    stream = torch.cuda.current_stream()
+    clk = sample_clocks(int(os.environ.get("LOCAL_RANK", "0")))
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    t_begin = time.time()
+    evs[0].record(stream)
+    for i in range(args.steps):
+        step()
+        evs[i + 1].record(stream)
+    torch.cuda.synchronize()
+    t_end = time.time()
+    clocks = stop_clocks(clk, t_begin, t_end)
+    per = [evs[i].elapsed_time(evs[i + 1]) for i in range(args.steps)]
+    total_ms = evs[0].elapsed_time(evs[-1])
+    st, word = cr.cr_get_device_status()
+    if st != cr.CR_OK:
+        raise RuntimeError(f"device status {word}")
+    cend = sess.chunk_end[:N].to(torch.int64).cpu().numpy()
+    flops = train_flops(case, float(cend.sum()))
+    hbm, tf_burst, tf_sus, src = load_peaks()
+    achieved = flops / (total_ms / args.steps * 1e-3) / 1e12
+    B = case.repairer.n_blocks
+    launches = 35 + B * (36 + 2 * (len(a.cu_seqlens) - 1)) if B > 0 else 0
+    print(json.dumps({
+        "metric": "trained doc tokens/s (one AdamW update of the repair network per step, 1 GB300)",
+        "value": N * args.steps / (total_ms / 1e3), "unit": "tokens/s", "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
+        "p50_ms": statistics.median(per), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16 GEMM operands, fp32 accumulation and master weights",
+        "data": "synthetic (seeded caches, embeddings, joint = stale + sigma_Delta noise; random-init repairer)",
+        "config": {"workload": workload_desc(case), "n_tokens": N, "variant": {"train": True},
+                   "l2": "no flush: the cache, joint cache and residual buffers exceed L2",
+                   "optimizer": "AdamW (0.9, 0.95), wd 0.01, clip 1.0, lr 3e-4"},
+        "roofline": {"kernel": "whole update (forward, objective, backward, AdamW)", "bound": "tensor",
+                     "achieved": achieved, "peak": tf_sus, "unit": "TFLOP/s", "frac": achieved / tf_sus,
+                     "traffic": None, "algorithmic": f"{flops:.3e} flop per update",
+                     "peak_source": f"{src} bf16_tflops_sustained"},
+        "loss_first_timed": loss0, "loss_last": float(ts.stats[0].item()),
+        "gpu_launches": launches * args.steps, "clocks": clocks,
+    }))
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         run_reference(args)
+    elif args.train:
+        run_train(args)
     else:
         run_ours(args)
 

@@ -350,6 +350,69 @@ cr_status cr_sigma_accumulate(const cr_target_dims* target, const void* a, const
 cr_status cr_sigma_finalize(const cr_target_dims* target, const double* sumsq, int64_t count,
                             float* sigma_out, void* stream);
 
+/* ---------------------------------------------------------------- training
+ * One update of the repair network (Sec. 4.2 "Paired cache supervision" and
+ * "Normalization and objective"; App. A "Optimization").
+ *
+ * Parameters live in one flat vector: the trained tensors in this order,
+ *   w_seg [S][d_seg][d_h], b_seg [S][d_seg], w_map [d_c][S d_seg], b_map [d_c],
+ *   w_tok [d_c][d_model], b_tok [d_c], w_fuse [d_b][2 d_c], b_fuse [d_b],
+ *   w_rein [B][d_b][d_c], b_rein [B][d_b],
+ *   per block: ln1_g, ln1_b [d_b], w_qkv [3 d_b][d_b], b_qkv [3 d_b],
+ *              w_o [d_b][d_b], b_o [d_b], ln2_g, ln2_b [d_b],
+ *              w_fc1 [hidden][d_b], b_fc1 [hidden], w_fc2 [d_b][hidden], b_fc2 [d_b],
+ *   lnf_g, lnf_b [d_b], w_out [D_KV][d_b], b_out [D_KV],
+ * each starting at a multiple of 8 elements (gaps are zero and stay zero).
+ * cr_param_layout writes the n_tensors + 1 offsets (the last is the total
+ * count) and returns CR_ERR_INVALID_ARG if `max_offsets` is too small; the
+ * tensor count is 14 + 12 B.  Row-major [out][in] matrices as elsewhere.
+ */
+cr_status cr_param_layout(const cr_target_dims* target, const cr_repairer_dims* rep,
+                          int64_t* offsets, int32_t max_offsets);
+
+typedef struct cr_adamw {
+    float lr;                 /* learning rate of this update */
+    float beta1, beta2;       /* (0.9, 0.95) in App. A */
+    float eps;                /* 1e-8 */
+    float weight_decay;       /* 0.01, decoupled, on every parameter */
+    float max_grad_norm;      /* 1: "unit gradient clipping" of the global L2 norm */
+    int32_t step;             /* 1-based update count, for the bias corrections */
+} cr_adamw;
+
+/* Workspace bytes of cr_train_step for batches of up to max_tokens tokens in
+ * total whose longest request has max_request_tokens tokens; 0 if the
+ * dimensions are invalid. */
+size_t cr_train_workspace_bytes(const cr_target_dims* target, const cr_repairer_dims* rep,
+                                int64_t max_tokens, int64_t max_request_tokens);
+
+/*
+ * cr_train_step - forward, objective, backward, clipping and AdamW for one
+ * batch of requests (the method's block-causal mask, bf16 caches only):
+ *   L = mean over requests of 1/(N_r D_KV) sum_t || z_t - (KV_joint,t - KV_stale,t) / sigma_Delta ||^2,
+ *   g = dL/dtheta over every trained tensor; g <- g min(1, max_norm / (||g|| + 1e-6));
+ *   theta <- theta (1 - lr wd) - lr (m / (1 - b1^t)) / (sqrt(v / (1 - b2^t)) + eps)
+ * with m, v the AdamW moments.  params [P] fp32 masters (updated in place);
+ * params_bf16 [P] their bf16 copies, read by the forward's matrices and
+ * rewritten after the update; adam_m, adam_v [P] fp32 (updated); grads [P]
+ * fp32, written with the unclipped gradient; sigma_stale, sigma_delta [D_KV]
+ * fp32 (fixed statistics, not trained).  kv_stale, kv_joint [N, D_KV] bf16
+ * (canonical K), emb [N, d_model] bf16, chunk_end, pos [N] int32 as written by
+ * cr_assemble_stale; cu_seqlens_host [n_req + 1] HOST.  stats_out: device
+ * fp32 [4] = loss, gradient norm before clipping, clipping coefficient, 0.
+ * The forward computes as cr_compress_features + cr_repair_forward; the
+ * backward's plain matrix products run in cuBLAS (bf16 operands, fp32
+ * accumulation; the attention backward in TF32 on fp32 operands), using a
+ * part of the workspace as cuBLAS's workspace.  All device buffers 16-byte
+ * aligned; P = the last offset of cr_param_layout.
+ */
+cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* rep, float* params,
+                        uint16_t* params_bf16, float* adam_m, float* adam_v, float* grads,
+                        const float* sigma_stale, const float* sigma_delta, const void* kv_stale,
+                        const void* kv_joint, const void* emb, const int32_t* chunk_end,
+                        const int32_t* pos, const int32_t* cu_seqlens_host, int32_t n_req,
+                        int64_t n_tokens, const cr_adamw* hp, float* stats_out, void* workspace,
+                        size_t workspace_bytes, void* stream);
+
 /* Device status word: out[0] = first error (0 none, 1 wait timeout, 2 device
  * index out of range), out[1] = site, out[2] = block.  Synchronises the
  * device.  cr_clear_device_status() resets it to zero. */

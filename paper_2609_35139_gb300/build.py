@@ -28,7 +28,9 @@ CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relax
           "-diag-suppress", "177",
           "-I" + INCLUDE, "-I" + CSRC]
 SOURCES = ["cr_api.cu", "cr_gemm.cu", "cr_attn.cu", "cr_segproj.cu", "cr_misc.cu",
-           "cr_noalloc.cu", "cr_offline.cu"]
+           "cr_noalloc.cu", "cr_offline.cu", "cr_train.cu"]
+# the training step's plain (unfused) backward GEMMs go through cuBLAS
+LIBS = ["-lcublas"]
 
 
 def _nvcc() -> str:
@@ -45,7 +47,7 @@ def _digest(extra) -> str:
             if f.endswith((".cu", ".cuh", ".h")):
                 with open(os.path.join(d, f), "rb") as fh:
                     h.update(f.encode() + b"\0" + fh.read())
-    h.update(" ".join(ARCH + CFLAGS + list(extra)).encode())
+    h.update(" ".join(ARCH + CFLAGS + LIBS + list(extra)).encode())
     return h.hexdigest()
 
 
@@ -75,7 +77,7 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
     with ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
         objs = list(ex.map(compile_one, SOURCES))
     tmp = LIB_PATH + f".tmp{os.getpid()}"
-    cmd = [nvcc, *ARCH, "-shared", "-o", tmp, *objs]
+    cmd = [nvcc, *ARCH, "-shared", "-o", tmp, *objs, *LIBS]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")

@@ -30,7 +30,7 @@ EXPORTED = [
     "cr_clear_device_status", "cr_status_str", "cr_last_cuda_error",
     "cr_linear", "cr_layernorm", "cr_chunk_causal_attention", "cr_masked_attention",
     "cr_chunk_starts", "cr_qkv_rope", "cr_segment_project",
-    "cr_segment_project_noalloc",
+    "cr_segment_project_noalloc", "cr_param_layout", "cr_train_workspace_bytes", "cr_train_step",
 ]
 
 
@@ -64,6 +64,11 @@ class cr_block_weights(ctypes.Structure):
 
 class cr_weights(ctypes.Structure):
     _fields_ = [(f, c_void_p) for f in _WEIGHT_FIELDS]
+
+
+class cr_adamw(ctypes.Structure):
+    _fields_ = [("lr", c_float), ("beta1", c_float), ("beta2", c_float), ("eps", c_float),
+                ("weight_decay", c_float), ("max_grad_norm", c_float), ("step", c_int32)]
 
 
 _lib_handle = None
@@ -112,6 +117,10 @@ def lib(build_if_missing: bool = False) -> ctypes.CDLL:
         "cr_linear": (i32, [vp, i64, vp, vp, i64, i64, i64, vp, i64, i32, vp]),
         "cr_layernorm": (i32, [vp, vp, i64, vp, vp, vp, c_float, i64, i64, vp, vp]),
         "cr_chunk_causal_attention": (i32, [vp, i32, i32, vp, vp, i32, i64, vp, vp]),
+        "cr_param_layout": (i32, [P(cr_target_dims), P(cr_repairer_dims), vp, i32]),
+        "cr_train_workspace_bytes": (c_size_t, [P(cr_target_dims), P(cr_repairer_dims), i64, i64]),
+        "cr_train_step": (i32, [P(cr_target_dims), P(cr_repairer_dims), vp, vp, vp, vp, vp, vp, vp, vp, vp,
+                                vp, vp, vp, vp, i32, i64, P(cr_adamw), vp, vp, c_size_t, vp]),
         "cr_masked_attention": (i32, [vp, i32, i32, i32, vp, vp, vp, i32, i64, vp, vp]),
         "cr_chunk_starts": (i32, [vp, vp, i32, i64, vp, vp]),
         "cr_qkv_rope": (i32, [vp, vp, vp, vp, i64, i32, i32, c_float, vp, vp]),
@@ -352,6 +361,30 @@ def cr_chunk_causal_attention(qkv, d_b, n_heads, chunk_end, cu_seqlens_host, out
     _check("cr_chunk_causal_attention", lib().cr_chunk_causal_attention(
         _p(qkv), d_b, n_heads, _p(chunk_end), cu.ctypes.data, len(cu) - 1, qkv.shape[0], _p(out),
         _stream(stream)))
+
+
+def cr_param_layout(target, rep) -> np.ndarray:
+    """Offsets of the trained tensors in the flat parameter vector (last entry: the total)."""
+    off = np.zeros(14 + 12 * 64 + 1, np.int64)
+    _check("cr_param_layout", lib().cr_param_layout(ctypes.byref(target), ctypes.byref(rep),
+                                                    off.ctypes.data, len(off)))
+    return off[:14 + 12 * rep.n_blocks + 1].copy()
+
+
+def cr_train_workspace_bytes(target, rep, max_tokens, max_request_tokens) -> int:
+    return int(lib().cr_train_workspace_bytes(ctypes.byref(target), ctypes.byref(rep), max_tokens,
+                                              max_request_tokens))
+
+
+def cr_train_step(target, rep, params, params_bf16, adam_m, adam_v, grads, sigma_stale, sigma_delta,
+                  kv_stale, kv_joint, emb, chunk_end, pos, cu_seqlens_host, n_tokens, hp: "cr_adamw",
+                  stats_out, workspace, stream=None):
+    cu = _host_arr(cu_seqlens_host, np.int32)
+    _check("cr_train_step", lib().cr_train_step(
+        ctypes.byref(target), ctypes.byref(rep), _p(params), _p(params_bf16), _p(adam_m), _p(adam_v),
+        _p(grads), _p(sigma_stale), _p(sigma_delta), _p(kv_stale), _p(kv_joint), _p(emb), _p(chunk_end),
+        _p(pos), cu.ctypes.data, len(cu) - 1, n_tokens, ctypes.byref(hp), _p(stats_out), _p(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
 def cr_masked_attention(qkv, d_b, n_heads, mask_mode, chunk_end, chunk_start, cu_seqlens_host, out,

@@ -4,7 +4,9 @@
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 #include <math.h>
+#include <algorithm>
 #include <mutex>
+#include <vector>
 #include <string.h>
 
 #include "cr_internal.h"
@@ -862,6 +864,490 @@ cr_status cr_segment_project(const cr_target_dims* target, int32_t d_seg, const 
     sp.y = y;
     sp.status = status;
     return launch_segproj(kv, d.D, wfold, static_cast<int>(d.dh), sp, st);
+}
+
+// ------------------------------------------------------------------ training step
+// Flat parameter layout (include/cr.h): the trained tensors in a fixed order,
+// each starting at a multiple of 8 elements so that every tensor's fp32 and
+// bf16 copies are 16-byte aligned.
+static int train_tensor_sizes(const Dims& d, int64_t* sz, int max) {
+    const int n = 14 + 12 * static_cast<int>(d.B);
+    if (n > max) return -1;
+    int k = 0;
+    sz[k++] = d.S * d.dseg * d.dh;      // w_seg
+    sz[k++] = d.S * d.dseg;             // b_seg
+    sz[k++] = d.dc * d.S * d.dseg;      // w_map
+    sz[k++] = d.dc;                     // b_map
+    sz[k++] = d.dc * d.dmodel;          // w_tok
+    sz[k++] = d.dc;                     // b_tok
+    sz[k++] = d.db * 2 * d.dc;          // w_fuse
+    sz[k++] = d.db;                     // b_fuse
+    sz[k++] = d.B * d.db * d.dc;        // w_rein
+    sz[k++] = d.B * d.db;               // b_rein
+    for (int64_t b = 0; b < d.B; ++b) {
+        sz[k++] = d.db;                 // ln1_g
+        sz[k++] = d.db;                 // ln1_b
+        sz[k++] = 3 * d.db * d.db;      // w_qkv
+        sz[k++] = 3 * d.db;             // b_qkv
+        sz[k++] = d.db * d.db;          // w_o
+        sz[k++] = d.db;                 // b_o
+        sz[k++] = d.db;                 // ln2_g
+        sz[k++] = d.db;                 // ln2_b
+        sz[k++] = d.hid * d.db;         // w_fc1
+        sz[k++] = d.hid;                // b_fc1
+        sz[k++] = d.db * d.hid;         // w_fc2
+        sz[k++] = d.db;                 // b_fc2
+    }
+    sz[k++] = d.db;                     // lnf_g
+    sz[k++] = d.db;                     // lnf_b
+    sz[k++] = d.D * d.db;               // w_out
+    sz[k++] = d.D;                      // b_out
+    return k;
+}
+
+static int train_offsets(const Dims& d, int64_t* off, int max) {
+    int64_t sz[14 + 12 * 64];
+    const int n = train_tensor_sizes(d, sz, 14 + 12 * 64);
+    if (n < 0 || n + 1 > max) return -1;
+    int64_t o = 0;
+    for (int i = 0; i < n; ++i) {
+        off[i] = o;
+        o += (sz[i] + 7) / 8 * 8;
+    }
+    off[n] = o;
+    return n;
+}
+
+cr_status cr_param_layout(const cr_target_dims* target, const cr_repairer_dims* rep, int64_t* offsets,
+                          int32_t max_offsets) {
+    cr_status s = check_target(target);
+    if (s == CR_OK) s = check_repairer(rep);
+    if (s != CR_OK) return s;
+    if (!offsets) return CR_ERR_INVALID_ARG;
+    return train_offsets(dims_of(target, rep), offsets, max_offsets) < 0 ? CR_ERR_INVALID_ARG : CR_OK;
+}
+
+namespace {
+struct TrainLayout {
+    size_t inf, h0, rein, blk, blk_stride, hbuf, yf, rope, ones, r, dz, rowsq, perreq, stats_pad, dh, dxm,
+        du, dtmp, pre, gprod, sig16, qkv32, dqkv, da, sbuf, dpbuf, dse, dy, colsum, norm, blas, total;
+    size_t x_in, x_mid, u1, u2, qkv, o, g;   // offsets inside one block's region
+};
+constexpr size_t kBlasBytes = 32ull << 20;
+
+TrainLayout train_layout(const Dims& d, int64_t n, int64_t nmax) {
+    TrainLayout L{};
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        const size_t o = off;
+        off += align256(bytes);
+        return o;
+    };
+    const size_t N = static_cast<size_t>(n);
+    L.inf = take(ws_layout(d, n).total);
+    L.h0 = take(N * d.db * 4);
+    L.rein = take(N * (d.B > 0 ? d.B : 1) * d.db * 2);
+    // per block: x_in, x_mid (fp32), u1, u2 (bf16), qkv (bf16), o (bf16), g (bf16)
+    size_t bo = 0;
+    auto btake = [&](size_t bytes) {
+        const size_t o = bo;
+        bo += align256(bytes);
+        return o;
+    };
+    L.x_in = btake(N * d.db * 4);
+    L.x_mid = btake(N * d.db * 4);
+    L.u1 = btake(N * d.db * 2);
+    L.u2 = btake(N * d.db * 2);
+    L.qkv = btake(N * 3 * d.db * 2);
+    L.o = btake(N * d.db * 2);
+    L.g = btake(N * d.hid * 2);
+    L.blk_stride = bo;
+    L.blk = take(bo * (d.B > 0 ? d.B : 1));
+    L.hbuf = take(N * d.db * 4);
+    L.yf = take(N * d.db * 2);
+    L.rope = take(N * (d.hd / 2) * 8);
+    L.ones = take(d.D * 4);
+    L.r = take(N * d.D * 4);
+    L.dz = take(N * d.D * 2);
+    L.rowsq = take(N * 4);
+    L.perreq = take(kMaxReq * 8);
+    L.dh = take(N * d.db * 4);
+    L.dxm = take(N * d.db * 4);
+    L.du = take(N * d.db * 4);
+    const int64_t wide = std::max(std::max(d.hid, 3 * d.db), std::max(2 * d.dc, d.S * d.dseg));
+    L.dtmp = take(N * d.hid * 4);
+    L.pre = take(N * d.hid * 4);
+    L.gprod = take(N * d.db * 4);
+    L.sig16 = take(N * wide * 2);
+    L.qkv32 = take(N * 3 * d.db * 4);
+    L.dqkv = take(N * 3 * d.db * 4);
+    L.da = take(N * d.db * 4);
+    L.sbuf = take(static_cast<size_t>(d.nh) * nmax * nmax * 4);
+    L.dpbuf = take(static_cast<size_t>(d.nh) * nmax * nmax * 4);
+    L.dse = take(N * 2 * d.dc * 4);
+    L.dy = take(N * d.S * d.dseg * 4);
+    L.colsum = take(colsum_scratch_floats(n, std::max(d.D, wide)) * 4);
+    L.norm = take(sqnorm_scratch_doubles() * 8);
+    L.blas = take(kBlasBytes);
+    L.total = off;
+    return L;
+}
+}  // namespace
+
+size_t cr_train_workspace_bytes(const cr_target_dims* target, const cr_repairer_dims* rep,
+                                int64_t max_tokens, int64_t max_request_tokens) {
+    if (check_target(target) != CR_OK || check_repairer(rep) != CR_OK) return 0;
+    if (max_tokens < 1 || max_request_tokens < 1 || max_request_tokens > max_tokens ||
+        max_tokens > INT32_MAX / 2)
+        return 0;
+    return train_layout(dims_of(target, rep), max_tokens, max_request_tokens).total;
+}
+
+cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* rep, float* params,
+                        uint16_t* params_bf16, float* adam_m, float* adam_v, float* grads,
+                        const float* sigma_stale, const float* sigma_delta, const void* kv_stale,
+                        const void* kv_joint, const void* emb, const int32_t* chunk_end,
+                        const int32_t* pos, const int32_t* cu_seqlens_host, int32_t n_req,
+                        int64_t n_tokens, const cr_adamw* hp, float* stats_out, void* workspace,
+                        size_t workspace_bytes, void* stream) {
+    cr_status s = check_target(target);
+    if (s == CR_OK) s = check_repairer(rep);
+    if (s != CR_OK) return s;
+    const Dims d = dims_of(target, rep);
+    if (d.f32) return CR_ERR_UNSUPPORTED;
+    if (!hp || !cu_seqlens_host || n_req < 1 || n_req > kMaxReq || n_tokens < 1 ||
+        n_tokens > INT32_MAX / 2)
+        return CR_ERR_INVALID_ARG;
+    if (!(hp->lr >= 0.0f) || !(hp->beta1 >= 0.0f && hp->beta1 < 1.0f) ||
+        !(hp->beta2 >= 0.0f && hp->beta2 < 1.0f) || !(hp->eps > 0.0f) || !(hp->weight_decay >= 0.0f) ||
+        !(hp->max_grad_norm > 0.0f) || hp->step < 1)
+        return CR_ERR_INVALID_ARG;
+    if (!all_aligned(params, params_bf16, adam_m, adam_v, grads, sigma_stale, sigma_delta, kv_stale,
+                     kv_joint, emb, chunk_end, pos, stats_out, workspace))
+        return CR_ERR_INVALID_ARG;
+    if (cu_seqlens_host[0] != 0 || cu_seqlens_host[n_req] != n_tokens) return CR_ERR_INVALID_ARG;
+    int64_t nmax = 0;
+    for (int r = 0; r < n_req; ++r) {
+        const int64_t len = cu_seqlens_host[r + 1] - cu_seqlens_host[r];
+        if (len < 1) return CR_ERR_INVALID_ARG;
+        nmax = std::max(nmax, len);
+    }
+    const int64_t N = n_tokens;
+    const TrainLayout L = train_layout(d, N, nmax);
+    if (workspace_bytes < L.total) return CR_ERR_INVALID_ARG;
+    int64_t off[14 + 12 * 64 + 1];
+    const int nt = train_offsets(d, off, 14 + 12 * 64 + 1);
+    if (nt < 0) return CR_ERR_INVALID_ARG;
+    const int64_t P = off[nt];
+    unsigned* status = device_status_ptr();
+    if (!status) return CR_ERR_CUDA;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const float eps = rep->ln_eps;
+    const int64_t B = d.B, db = d.db, dc = d.dc, hid = d.hid, hd = d.hd, D = d.D;
+
+    // tensor k of the flat vector: fp32 master, bf16 copy, gradient
+    auto pf = [&](int k) { return params + off[k]; };
+    auto pb = [&](int k) { return params_bf16 + off[k]; };
+    auto gk = [&](int k) { return grads + off[k]; };
+    enum { W_SEG, B_SEG, W_MAP, B_MAP, W_TOK, B_TOK, W_FUSE, B_FUSE, W_REIN, B_REIN, BLK0 };
+    enum { LN1G, LN1B, WQKV, BQKV, WO, BO, LN2G, LN2B, WFC1, BFC1, WFC2, BFC2 };
+    auto bk = [&](int64_t b, int j) { return BLK0 + static_cast<int>(12 * b) + j; };
+    const int LNFG = BLK0 + static_cast<int>(12 * B), LNFB = LNFG + 1, W_OUT = LNFG + 2, B_OUT = LNFG + 3;
+
+    // the forward's weights: matrices from the bf16 copy, vectors from the masters
+    std::vector<cr_block_weights> blocks(static_cast<size_t>(std::max<int64_t>(B, 1)));
+    for (int64_t b = 0; b < B; ++b) {
+        cr_block_weights& k = blocks[static_cast<size_t>(b)];
+        k.ln1_g = pf(bk(b, LN1G));
+        k.ln1_b = pf(bk(b, LN1B));
+        k.w_qkv = pb(bk(b, WQKV));
+        k.b_qkv = pf(bk(b, BQKV));
+        k.w_o = pb(bk(b, WO));
+        k.b_o = pf(bk(b, BO));
+        k.ln2_g = pf(bk(b, LN2G));
+        k.ln2_b = pf(bk(b, LN2B));
+        k.w_fc1 = pb(bk(b, WFC1));
+        k.b_fc1 = pf(bk(b, BFC1));
+        k.w_fc2 = pb(bk(b, WFC2));
+        k.b_fc2 = pf(bk(b, BFC2));
+    }
+    cr_weights w{};
+    w.w_seg = pb(W_SEG);
+    w.b_seg = pf(B_SEG);
+    w.w_map = pb(W_MAP);
+    w.b_map = pf(B_MAP);
+    w.w_tok = pb(W_TOK);
+    w.b_tok = pf(B_TOK);
+    w.w_fuse = pb(W_FUSE);
+    w.b_fuse = pf(B_FUSE);
+    w.w_rein = pb(W_REIN);
+    w.b_rein = pf(B_REIN);
+    w.blocks = blocks.data();
+    w.lnf_g = pf(LNFG);
+    w.lnf_b = pf(LNFB);
+    w.w_out = pb(W_OUT);
+    w.b_out = pf(B_OUT);
+    w.sigma_stale = sigma_stale;
+    w.sigma_delta = sigma_delta;
+
+    // ---- workspace
+    uint8_t* base = static_cast<uint8_t*>(workspace);
+    void* inf = base + L.inf;
+    const WsLayout IL = ws_layout(d, N);
+    const uint16_t* y = at<uint16_t>(inf, IL.y);      // [N, S d_seg] after compress
+    const uint16_t* se = at<uint16_t>(inf, IL.se);    // [N, 2 d_c] = [s ; e]
+    float* h0 = at<float>(base, L.h0);
+    uint16_t* rein = at<uint16_t>(base, L.rein);
+    auto blk = [&](int64_t b, size_t o) { return base + L.blk + static_cast<size_t>(b) * L.blk_stride + o; };
+    float* H = at<float>(base, L.hbuf);
+    uint16_t* yf = at<uint16_t>(base, L.yf);
+    float2* rope = at<float2>(base, L.rope);
+    float* ones = at<float>(base, L.ones);
+    float* R = at<float>(base, L.r);
+    uint16_t* DZ = at<uint16_t>(base, L.dz);
+    float* ROWSQ = at<float>(base, L.rowsq);
+    double* PERREQ = at<double>(base, L.perreq);
+    float* DH = at<float>(base, L.dh);
+    float* DXM = at<float>(base, L.dxm);
+    float* DU = at<float>(base, L.du);
+    float* DTMP = at<float>(base, L.dtmp);
+    float* PRE = at<float>(base, L.pre);
+    float* GPROD = at<float>(base, L.gprod);
+    uint16_t* SIG = at<uint16_t>(base, L.sig16);
+    float* QKV32 = at<float>(base, L.qkv32);
+    float* DQKV = at<float>(base, L.dqkv);
+    float* DA = at<float>(base, L.da);
+    float* SB = at<float>(base, L.sbuf);
+    float* DPB = at<float>(base, L.dpbuf);
+    float* DSE = at<float>(base, L.dse);
+    float* DY = at<float>(base, L.dy);
+    float* CS = at<float>(base, L.colsum);
+    double* NRM = at<double>(base, L.norm);
+
+    // ---- forward (Sec. 4.1), keeping what the backward needs
+    s = cr_compress_features(target, rep, &w, kv_stale, emb, N, h0, rein, inf, IL.total, stream);
+    if (s != CR_OK) return s;
+    AttnParams* ap = new AttnParams();
+    s = attn_params(d, CR_MASK_BLOCK_CAUSAL, chunk_end, nullptr, cu_seqlens_host, n_req, N, nullptr,
+                    status, ap);
+    GemmParams gq{};
+    gq.status = status;
+    gq.pos = pos;
+    gq.rope_dim = static_cast<int32_t>(hd);
+    gq.rope_cols = static_cast<int32_t>(2 * db);
+    repairer_inv_freq(gq.inv_freq, static_cast<int>(hd), rep->rope_theta);
+    if (s == CR_OK && B > 0) s = launch_rope_table(pos, N, static_cast<int>(hd / 2), gq.inv_freq, rope, st);
+    gq.rope_table = rope;
+    GemmParams gr{};
+    gr.status = status;
+    for (int64_t b = 0; b < B && s == CR_OK; ++b) {
+        const cr_block_weights& k = blocks[static_cast<size_t>(b)];
+        float* x_in = reinterpret_cast<float*>(blk(b, L.x_in));
+        float* x_mid = reinterpret_cast<float*>(blk(b, L.x_mid));
+        uint16_t* u1 = reinterpret_cast<uint16_t*>(blk(b, L.u1));
+        uint16_t* u2 = reinterpret_cast<uint16_t*>(blk(b, L.u2));
+        uint16_t* qkv = reinterpret_cast<uint16_t*>(blk(b, L.qkv));
+        uint16_t* o = reinterpret_cast<uint16_t*>(blk(b, L.o));
+        uint16_t* g = reinterpret_cast<uint16_t*>(blk(b, L.g));
+        if ((s = launch_layernorm(b == 0 ? h0 : H, rein + b * db, B * db, x_in, k.ln1_g, k.ln1_b, eps, N, db,
+                                  u1, st)) != CR_OK)
+            break;
+        gq.bias = k.b_qkv;
+        gq.out = qkv;
+        gq.ldo = 3 * db;
+        if ((s = launch_gemm(u1, db, k.w_qkv, N, 3 * db, db, EPI_QKV_ROPE, gq, nullptr, 0, st)) != CR_OK) break;
+        ap->out = o;
+        if ((s = launch_attention(qkv, N, static_cast<int>(hd), *ap, st)) != CR_OK) break;
+        if ((s = cuda_check(cudaMemcpyAsync(x_mid, x_in, static_cast<size_t>(N * db) * 4,
+                                            cudaMemcpyDeviceToDevice, st))) != CR_OK)
+            break;
+        gr.bias = k.b_o;
+        gr.out = x_mid;
+        gr.ldo = db;
+        if ((s = launch_gemm(o, db, k.w_o, N, db, db, EPI_ADD_F32, gr, nullptr, 0, st)) != CR_OK) break;
+        if ((s = launch_layernorm(x_mid, nullptr, 0, nullptr, k.ln2_g, k.ln2_b, eps, N, db, u2, st)) != CR_OK)
+            break;
+        gr.bias = k.b_fc1;
+        gr.out = g;
+        gr.ldo = hid;
+        if ((s = launch_gemm(u2, db, k.w_fc1, N, hid, db, EPI_GELU_BF16, gr, nullptr, 0, st)) != CR_OK) break;
+        if ((s = cuda_check(cudaMemcpyAsync(H, x_mid, static_cast<size_t>(N * db) * 4,
+                                            cudaMemcpyDeviceToDevice, st))) != CR_OK)
+            break;
+        gr.bias = k.b_fc2;
+        gr.out = H;
+        gr.ldo = db;
+        if ((s = launch_gemm(g, hid, k.w_fc2, N, db, hid, EPI_ADD_F32, gr, nullptr, 0, st)) != CR_OK) break;
+    }
+    delete ap;
+    if (s != CR_OK) return s;
+    if (B == 0 && (s = cuda_check(cudaMemcpyAsync(H, h0, static_cast<size_t>(N * db) * 4,
+                                                  cudaMemcpyDeviceToDevice, st))) != CR_OK)
+        return s;
+    if ((s = launch_layernorm(H, nullptr, 0, nullptr, w.lnf_g, w.lnf_b, eps, N, db, yf, st)) != CR_OK) return s;
+
+    // ---- objective (Sec. 4.2): the head writes r = z - (joint - stale) / sigma_Delta
+    if ((s = launch_target(kv_stale, kv_joint, false, sigma_delta, N, D, R, st)) != CR_OK) return s;
+    if ((s = launch_fill(ones, D, 1.0f, st)) != CR_OK) return s;
+    GemmParams gh{};
+    gh.status = status;
+    gh.bias = w.b_out;
+    gh.sigma = ones;
+    gh.pos = pos;
+    gh.rope_dim = static_cast<int32_t>(d.dh);
+    gh.n_kv_heads = static_cast<int32_t>(d.H);
+    if ((s = launch_gemm(yf, db, w.w_out, N, D, db, EPI_KV_F32, gh, R, D, st)) != CR_OK) return s;
+    LossParams* lp = new LossParams();
+    lp->n_req = n_req;
+    for (int r = 0; r <= n_req; ++r) lp->req_start[r] = cu_seqlens_host[r];
+    for (int r = 0; r < n_req; ++r)
+        lp->scale[r] = static_cast<float>(
+            2.0 / (static_cast<double>(cu_seqlens_host[r + 1] - cu_seqlens_host[r]) * D * n_req));
+    s = launch_loss(R, N, D, *lp, DZ, ROWSQ, stats_out, PERREQ, st);
+    delete lp;
+    if (s != CR_OK) return s;
+
+    // ---- backward: the chain rule in reverse, gradients straight into `grads`
+    cublasHandle_t hb;
+    if ((s = blas_handle(st, base + L.blas, kBlasBytes, &hb)) != CR_OK) return s;
+    if ((s = cuda_check(cudaMemsetAsync(grads, 0, static_cast<size_t>(P) * 4, st))) != CR_OK) return s;
+    const cudaDataType_t BF = CUDA_R_16BF, F32 = CUDA_R_32F;
+    auto colsum = [&](const void* a, bool bf16, int64_t cols, int64_t lda, float* out) {
+        return launch_colsum(a, bf16, N, cols, lda, out, false, CS, st);
+    };
+    auto to16 = [&](const float* a, int64_t n, uint16_t* out) { return launch_to_bf16(a, n, out, st); };
+#define CR_TRY(x)                   \
+    do {                            \
+        if ((s = (x)) != CR_OK) return s; \
+    } while (0)
+    // head: dW_out = dz^T y_f, db_out = sum_t dz, dy_f = dz W_out
+    CR_TRY(gemm_rm(hb, true, false, D, db, N, 1.0f, DZ, BF, D, yf, BF, db, 0.0f, gk(W_OUT), F32, db));
+    CR_TRY(colsum(DZ, true, D, D, gk(B_OUT)));
+    CR_TRY(gemm_rm(hb, false, false, N, db, D, 1.0f, DZ, BF, D, pb(W_OUT), BF, db, 0.0f, DU, F32, db));
+    CR_TRY(launch_ln_backward(H, w.lnf_g, DU, nullptr, eps, N, static_cast<int>(db), DH, GPROD, st));
+    CR_TRY(colsum(GPROD, false, db, db, gk(LNFG)));
+    CR_TRY(colsum(DU, false, db, db, gk(LNFB)));
+    CR_TRY(cuda_check(cudaMemsetAsync(DSE, 0, static_cast<size_t>(N * 2 * dc) * 4, st)));
+    const float scale = static_cast<float>(1.0 / sqrt(static_cast<double>(hd)));
+    for (int64_t b = B - 1; b >= 0; --b) {
+        const float* x_in = reinterpret_cast<const float*>(blk(b, L.x_in));
+        const float* x_mid = reinterpret_cast<const float*>(blk(b, L.x_mid));
+        const uint16_t* u1 = reinterpret_cast<const uint16_t*>(blk(b, L.u1));
+        const uint16_t* u2 = reinterpret_cast<const uint16_t*>(blk(b, L.u2));
+        const uint16_t* qkv = reinterpret_cast<const uint16_t*>(blk(b, L.qkv));
+        const uint16_t* o = reinterpret_cast<const uint16_t*>(blk(b, L.o));
+        const uint16_t* g = reinterpret_cast<const uint16_t*>(blk(b, L.g));
+        // h = x_mid + W_fc2 g + b_fc2
+        CR_TRY(to16(DH, N * db, SIG));
+        CR_TRY(gemm_rm(hb, true, false, db, hid, N, 1.0f, SIG, BF, db, g, BF, hid, 0.0f, gk(bk(b, WFC2)), F32, hid));
+        CR_TRY(colsum(DH, false, db, db, gk(bk(b, BFC2))));
+        CR_TRY(gemm_rm(hb, false, false, N, hid, db, 1.0f, SIG, BF, db, pb(bk(b, WFC2)), BF, hid, 0.0f, DTMP, F32,
+                       hid));
+        // g = GELU(pre), pre = W_fc1 u2 + b_fc1 (recomputed in fp32)
+        GemmParams gp{};
+        gp.status = status;
+        gp.bias = pf(bk(b, BFC1));
+        gp.out = PRE;
+        gp.ldo = hid;
+        CR_TRY(launch_gemm(u2, db, pb(bk(b, WFC1)), N, hid, db, EPI_F32, gp, nullptr, 0, st));
+        CR_TRY(launch_gelu_backward(DTMP, PRE, N * hid, st));
+        CR_TRY(to16(DTMP, N * hid, SIG));
+        CR_TRY(gemm_rm(hb, true, false, hid, db, N, 1.0f, SIG, BF, hid, u2, BF, db, 0.0f, gk(bk(b, WFC1)), F32, db));
+        CR_TRY(colsum(DTMP, false, hid, hid, gk(bk(b, BFC1))));
+        CR_TRY(gemm_rm(hb, false, false, N, db, hid, 1.0f, SIG, BF, hid, pb(bk(b, WFC1)), BF, db, 0.0f, DU, F32,
+                       db));
+        // u2 = LN2(x_mid): dx_mid = dh + LN2 backward
+        CR_TRY(launch_ln_backward(x_mid, pf(bk(b, LN2G)), DU, DH, eps, N, static_cast<int>(db), DXM, GPROD, st));
+        CR_TRY(colsum(GPROD, false, db, db, gk(bk(b, LN2G))));
+        CR_TRY(colsum(DU, false, db, db, gk(bk(b, LN2B))));
+        // x_mid = x_in + W_o a + b_o
+        CR_TRY(to16(DXM, N * db, SIG));
+        CR_TRY(gemm_rm(hb, true, false, db, db, N, 1.0f, SIG, BF, db, o, BF, db, 0.0f, gk(bk(b, WO)), F32, db));
+        CR_TRY(colsum(DXM, false, db, db, gk(bk(b, BO))));
+        CR_TRY(gemm_rm(hb, false, false, N, db, db, 1.0f, SIG, BF, db, pb(bk(b, WO)), BF, db, 0.0f, DA, F32, db));
+        // attention, per request, heads batched: S = Q K^T scale; P = softmax;
+        // dV = P^T dA; dP = dA V^T; dS = P (dP - rowsum(P dP)); dQ = dS K scale; dK = dS^T Q scale
+        CR_TRY(launch_f32_from_bf16(qkv, N * 3 * db, QKV32, st));
+        for (int r = 0; r < n_req; ++r) {
+            const int64_t lo = cu_seqlens_host[r], n = cu_seqlens_host[r + 1] - lo;
+            const float* Q = QKV32 + lo * 3 * db;
+            const float* K = Q + db;
+            const float* V = Q + 2 * db;
+            const float* dA = DA + lo * db;
+            float* dQ = DQKV + lo * 3 * db;
+            const int64_t nn = n * n;
+            CR_TRY(gemm_rm(hb, false, true, n, n, hd, scale, Q, F32, 3 * db, K, F32, 3 * db, 0.0f, SB, F32, n,
+                           d.nh, hd, hd, nn));
+            SoftmaxParams sp{};
+            sp.n = static_cast<int32_t>(n);
+            sp.heads = static_cast<int32_t>(d.nh);
+            sp.mask_mode = CR_MASK_BLOCK_CAUSAL;
+            sp.chunk_end = chunk_end + lo;
+            CR_TRY(launch_softmax_rows(SB, sp, st));
+            CR_TRY(gemm_rm(hb, true, false, n, hd, n, 1.0f, SB, F32, n, dA, F32, db, 0.0f, dQ + 2 * db, F32,
+                           3 * db, d.nh, nn, hd, hd));
+            CR_TRY(gemm_rm(hb, false, true, n, n, hd, 1.0f, dA, F32, db, V, F32, 3 * db, 0.0f, DPB, F32, n, d.nh,
+                           hd, hd, nn));
+            CR_TRY(launch_softmax_bwd(SB, DPB, sp, st));
+            CR_TRY(gemm_rm(hb, false, false, n, hd, n, scale, DPB, F32, n, K, F32, 3 * db, 0.0f, dQ, F32, 3 * db,
+                           d.nh, nn, hd, hd));
+            CR_TRY(gemm_rm(hb, true, false, n, hd, n, scale, DPB, F32, n, Q, F32, 3 * db, 0.0f, dQ + db, F32,
+                           3 * db, d.nh, nn, hd, hd));
+        }
+        CR_TRY(launch_rope_backward(DQKV, rope, N, static_cast<int>(db), static_cast<int>(hd), st));
+        // qkv = W_qkv u1 + b_qkv;  u1 = LN1(x_in): dx_in = dx_mid + LN1 backward
+        CR_TRY(to16(DQKV, N * 3 * db, SIG));
+        CR_TRY(gemm_rm(hb, true, false, 3 * db, db, N, 1.0f, SIG, BF, 3 * db, u1, BF, db, 0.0f, gk(bk(b, WQKV)),
+                       F32, db));
+        CR_TRY(colsum(DQKV, false, 3 * db, 3 * db, gk(bk(b, BQKV))));
+        CR_TRY(gemm_rm(hb, false, false, N, db, 3 * db, 1.0f, SIG, BF, 3 * db, pb(bk(b, WQKV)), BF, db, 0.0f, DU,
+                       F32, db));
+        CR_TRY(launch_ln_backward(x_in, pf(bk(b, LN1G)), DU, DXM, eps, N, static_cast<int>(db), DH, GPROD, st));
+        CR_TRY(colsum(GPROD, false, db, db, gk(bk(b, LN1G))));
+        CR_TRY(colsum(DU, false, db, db, gk(bk(b, LN1B))));
+        // x_in = h^{b-1} + W_rein,b s + b_rein,b: ds += dx_in W_rein,b
+        CR_TRY(to16(DH, N * db, SIG));
+        CR_TRY(gemm_rm(hb, true, false, db, dc, N, 1.0f, SIG, BF, db, se, BF, 2 * dc, 0.0f, gk(W_REIN) + b * db * dc,
+                       F32, dc));
+        CR_TRY(colsum(DH, false, db, db, gk(B_REIN) + b * db));
+        CR_TRY(gemm_rm(hb, false, false, N, dc, db, 1.0f, SIG, BF, db, pb(W_REIN) + b * db * dc, BF, dc, 1.0f, DSE,
+                       F32, 2 * dc));
+    }
+    // h0 = W_fuse [s; e] + b_fuse
+    CR_TRY(to16(DH, N * db, SIG));
+    CR_TRY(gemm_rm(hb, true, false, db, 2 * dc, N, 1.0f, SIG, BF, db, se, BF, 2 * dc, 0.0f, gk(W_FUSE), F32, 2 * dc));
+    CR_TRY(colsum(DH, false, db, db, gk(B_FUSE)));
+    CR_TRY(gemm_rm(hb, false, false, N, 2 * dc, db, 1.0f, SIG, BF, db, pb(W_FUSE), BF, 2 * dc, 1.0f, DSE, F32,
+                   2 * dc));
+    // e = W_tok emb + b_tok;  s = W_map y + b_map
+    CR_TRY(to16(DSE, N * 2 * dc, SIG));
+    CR_TRY(gemm_rm(hb, true, false, dc, d.dmodel, N, 1.0f, SIG + dc, BF, 2 * dc, emb, BF, d.dmodel, 0.0f, gk(W_TOK),
+                   F32, d.dmodel));
+    CR_TRY(colsum(DSE + dc, false, dc, 2 * dc, gk(B_TOK)));
+    const int64_t Sd = d.S * d.dseg;
+    CR_TRY(gemm_rm(hb, true, false, dc, Sd, N, 1.0f, SIG, BF, 2 * dc, y, BF, Sd, 0.0f, gk(W_MAP), F32, Sd));
+    CR_TRY(colsum(DSE, false, dc, 2 * dc, gk(B_MAP)));
+    CR_TRY(gemm_rm(hb, false, false, N, Sd, dc, 1.0f, SIG, BF, 2 * dc, pb(W_MAP), BF, Sd, 0.0f, DY, F32, Sd));
+    // y_{t,s} = (W_seg,s / sigma_stale) kv_{t,s} + b_seg,s: per segment dy^T kv, then / sigma_stale
+    CR_TRY(to16(DY, N * Sd, SIG));
+    CR_TRY(gemm_rm(hb, true, false, d.dseg, d.dh, N, 1.0f, SIG, BF, Sd, kv_stale, BF, D, 0.0f, gk(W_SEG), F32, d.dh,
+                   d.S, d.dseg, d.dh, d.dseg * d.dh));
+    CR_TRY(launch_scale_seg_grad(gk(W_SEG), d.S, d.dseg, d.dh, sigma_stale, st));
+    CR_TRY(colsum(DY, false, Sd, Sd, gk(B_SEG)));
+
+    // ---- clipping and AdamW (App. A)
+    AdamWParams ah{};
+    ah.lr = hp->lr;
+    ah.b1 = hp->beta1;
+    ah.b2 = hp->beta2;
+    ah.eps = hp->eps;
+    ah.wd = hp->weight_decay;
+    ah.bc1 = static_cast<float>(1.0 - pow(static_cast<double>(hp->beta1), hp->step));
+    ah.bc2 = static_cast<float>(1.0 - pow(static_cast<double>(hp->beta2), hp->step));
+    CR_TRY(launch_clip_adamw(params, adam_m, adam_v, grads, params_bf16, P, ah, hp->max_grad_norm, NRM, stats_out,
+                             st));
+#undef CR_TRY
+    return CR_OK;
 }
 
 }  // extern "C"

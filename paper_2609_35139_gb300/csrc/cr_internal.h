@@ -4,6 +4,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <cublas_v2.h>
+
 #include "cr.h"
 #include "cr_ops.h"
 
@@ -114,6 +116,21 @@ struct AttnParams {
     int32_t tile_prefix[kMaxReq + 1]; // cumulative items per request
 };
 
+// ------------------------------------------------------------------ training step
+struct LossParams {
+    int32_t n_req;
+    int32_t req_start[kMaxReq + 1];
+    float scale[kMaxReq];     // dL/dr factor of each request: 2 / (N_r D_KV n_req)
+};
+struct SoftmaxParams {
+    int32_t n, heads, mask_mode;
+    const int32_t* chunk_end;     // request-local
+    const int32_t* chunk_start;   // request-local (block-diagonal mask only)
+};
+struct AdamWParams {
+    float lr, b1, b2, eps, wd, bc1, bc2;
+};
+
 // ------------------------------------------------------------------ host helpers
 unsigned* device_status_ptr();          // per current device, nullptr on failure
 int num_sms();                          // SMs of the current device
@@ -189,5 +206,33 @@ cr_status launch_chunk_starts(const int32_t* chunk_end, const AttnParams& p, int
                               int32_t* chunk_start, cudaStream_t st);
 cr_status launch_attention(const uint16_t* qkv, int64_t n_tokens, int head_dim,
                            const AttnParams& p, cudaStream_t st);
+
+// training step (cr_train.cu)
+cr_status launch_fill(float* p, int64_t n, float v, cudaStream_t st);
+cr_status launch_target(const void* stale, const void* joint, bool f32, const float* sd, int64_t n,
+                        int64_t D, float* out, cudaStream_t st);
+cr_status launch_loss(const float* r, int64_t N, int64_t D, const LossParams& p, uint16_t* dz, float* rowsq,
+                      float* loss_out, double* per_req, cudaStream_t st);
+size_t colsum_scratch_floats(int64_t rows, int64_t cols);
+cr_status launch_colsum(const void* a, bool bf16, int64_t rows, int64_t cols, int64_t lda, float* out,
+                        bool accumulate, float* scratch, cudaStream_t st);
+cr_status launch_ln_backward(const float* x, const float* gamma, const float* dy, const float* add, float eps,
+                             int64_t N, int D, float* dx, float* gprod, cudaStream_t st);
+cr_status launch_gelu_backward(float* dg, const float* pre, int64_t n, cudaStream_t st);
+cr_status launch_rope_backward(float* dqkv, const float2* table, int64_t N, int db, int hd, cudaStream_t st);
+cr_status launch_softmax_rows(float* S, const SoftmaxParams& p, cudaStream_t st);
+cr_status launch_softmax_bwd(const float* P, float* dP, const SoftmaxParams& p, cudaStream_t st);
+cr_status launch_scale_seg_grad(float* g, int64_t S, int64_t dseg, int64_t dh, const float* sigma,
+                                cudaStream_t st);
+cr_status launch_f32_from_bf16(const uint16_t* a, int64_t n, float* out, cudaStream_t st);
+size_t sqnorm_scratch_doubles();
+cr_status launch_clip_adamw(float* p, float* m, float* v, const float* g, uint16_t* pb, int64_t n,
+                            const AdamWParams& hp, float max_norm, double* scratch, float* stats,
+                            cudaStream_t st);
+cr_status blas_handle(cudaStream_t st, void* ws, size_t ws_bytes, cublasHandle_t* out);
+cr_status gemm_rm(cublasHandle_t h, bool tA, bool tB, int64_t M, int64_t N, int64_t K, float alpha,
+                  const void* A, cudaDataType_t ta, int64_t lda, const void* B, cudaDataType_t tb, int64_t ldb,
+                  float beta, void* C, cudaDataType_t tc, int64_t ldc, int64_t batch = 1, int64_t sA = 0,
+                  int64_t sB = 0, int64_t sC = 0);
 
 }  // namespace cr

@@ -1,0 +1,572 @@
+// Training-step kernels (Sec. 4.2, App. A): the bandwidth-bound pieces of the
+// backward pass and of the optimizer, plus the row-major GEMM helpers over
+// cuBLAS that the backward's plain (unfused) matrix products use.
+//   target_kernel        -(KV_joint - KV_stale) / sigma_Delta, the head's in-place
+//                        input, so that the head epilogue writes r = z - target
+//   loss_grad_kernel     per row: sum of r^2, and dz = c_request * r (bf16)
+//   loss_reduce_kernel   per request, rows summed in order (fp64): the loss
+//   colsum_*             column sums in a fixed order (bias, LayerNorm grads)
+//   ln_backward_kernel   LayerNorm backward per row, plus dy * x_hat per element
+//   gelu_backward_kernel dpre = dg * (Phi(pre) + pre phi(pre))
+//   rope_backward_kernel the repairer RoPE's transpose on dQ, dK
+//   softmax_rows_kernel  masked row softmax of the score matrix, in place
+//   softmax_bwd_kernel   dS = P (dP - rowsum(P dP)), in place on dP
+//   sqnorm_*             squared L2 norm of the gradient (fp64, fixed order)
+//   adamw_kernel         clipping coefficient, AdamW, bf16 mirror of the weights
+#include <cublas_v2.h>
+#include <cuda_bf16.h>
+
+#include "cr_internal.h"
+#include "cr_ptx.cuh"
+
+namespace cr {
+namespace {
+
+__device__ __forceinline__ float bf16_to_f32(uint16_t b) { return __uint_as_float(static_cast<uint32_t>(b) << 16); }
+__device__ __forceinline__ uint16_t f32_to_bf16(float x) {
+    return __bfloat16_as_ushort(__float2bfloat16_rn(x));
+}
+template <typename T>
+__device__ __forceinline__ float ld(const T* p, int64_t i);
+template <>
+__device__ __forceinline__ float ld<uint16_t>(const uint16_t* p, int64_t i) { return bf16_to_f32(p[i]); }
+template <>
+__device__ __forceinline__ float ld<float>(const float* p, int64_t i) { return p[i]; }
+
+// the request of row t: req_start[r] <= t < req_start[r + 1]
+__device__ __forceinline__ int request_of(const LossParams& p, int64_t t) {
+    int r0 = 0, r1 = p.n_req - 1;
+    while (r0 < r1) {
+        const int mid = (r0 + r1 + 1) >> 1;
+        if (p.req_start[mid] <= t) r0 = mid;
+        else r1 = mid - 1;
+    }
+    return r0;
+}
+
+// bf16 caches, 8 values per thread (D_KV is a multiple of 8): 16-byte loads and
+// two 16-byte stores
+__global__ void __launch_bounds__(256)
+    target_kernel(const uint16_t* __restrict__ stale, const uint16_t* __restrict__ joint,
+                  const float* __restrict__ sd, int64_t n, int64_t D, float* __restrict__ out) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int64_t groups = n * D / 8;
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < groups;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t c = (i * 8) % D;
+        const uint4 a = reinterpret_cast<const uint4*>(stale)[i];
+        const uint4 b = reinterpret_cast<const uint4*>(joint)[i];
+        const float4 s0 = __ldg(reinterpret_cast<const float4*>(sd + c));
+        const float4 s1 = __ldg(reinterpret_cast<const float4*>(sd + c + 4));
+        const uint32_t ua[4] = {a.x, a.y, a.z, a.w}, ub[4] = {b.x, b.y, b.z, b.w};
+        const float sv[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+        float o[8];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float a0 = __uint_as_float(ua[k] << 16), a1 = __uint_as_float(ua[k] & 0xFFFF0000u);
+            const float b0 = __uint_as_float(ub[k] << 16), b1 = __uint_as_float(ub[k] & 0xFFFF0000u);
+            o[2 * k] = -(b0 - a0) / sv[2 * k];
+            o[2 * k + 1] = -(b1 - a1) / sv[2 * k + 1];
+        }
+        float4* dst = reinterpret_cast<float4*>(out + i * 8);
+        dst[0] = make_float4(o[0], o[1], o[2], o[3]);
+        dst[1] = make_float4(o[4], o[5], o[6], o[7]);
+    }
+}
+
+// One CTA per row: the row's sum of squares of r (fixed-order tree), and
+// dz = scale(request) * r rounded to bf16.
+__global__ void __launch_bounds__(256)
+    loss_grad_kernel(const float* __restrict__ r, int64_t D, const __grid_constant__ LossParams p,
+                     uint16_t* __restrict__ dz, float* __restrict__ rowsq) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int64_t t = blockIdx.x;
+    const float c = p.scale[request_of(p, t)];
+    const float* row = r + t * D;
+    uint16_t* drow = dz + t * D;
+    float acc = 0.0f;
+    for (int64_t j = threadIdx.x; j < D; j += blockDim.x) {
+        const float v = row[j];
+        acc = fmaf(v, v, acc);
+        drow[j] = f32_to_bf16(c * v);
+    }
+    __shared__ float red[256];
+    red[threadIdx.x] = acc;
+    __syncthreads();
+    for (int s = 128; s > 0; s >>= 1) {
+        if (static_cast<int>(threadIdx.x) < s) red[threadIdx.x] += red[threadIdx.x + s];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) rowsq[t] = red[0];
+}
+
+// One block per request: each thread sums a fixed stride of the request's rows
+// (fp64), then a fixed tree; the result divided by N_r D n_req (the mean over
+// requests).  loss_total_kernel adds the requests in order.
+__global__ void __launch_bounds__(256)
+    loss_reduce_kernel(const float* __restrict__ rowsq, const __grid_constant__ LossParams p, int64_t D,
+                       double* __restrict__ per_req) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int r = blockIdx.x;
+    double s = 0.0;
+    for (int64_t t = p.req_start[r] + threadIdx.x; t < p.req_start[r + 1]; t += blockDim.x)
+        s += static_cast<double>(rowsq[t]);
+    __shared__ double red[256];
+    red[threadIdx.x] = s;
+    __syncthreads();
+    for (int k = 128; k > 0; k >>= 1) {
+        if (static_cast<int>(threadIdx.x) < k) red[threadIdx.x] += red[threadIdx.x + k];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0)
+        per_req[r] = red[0] / (static_cast<double>(p.req_start[r + 1] - p.req_start[r]) * D * p.n_req);
+}
+
+__global__ void loss_total_kernel(const double* __restrict__ per_req, int n_req, float* __restrict__ loss_out) {
+    pdl_launch_dependents();
+    pdl_wait();
+    if (threadIdx.x != 0 || blockIdx.x != 0) return;
+    double l = 0.0;
+    for (int r = 0; r < n_req; ++r) l += per_req[r];
+    loss_out[0] = static_cast<float>(l);
+}
+
+// Column sums in a fixed order: slice y of kColSlice rows per block row,
+// partial[y][c]; then the slices in order.
+constexpr int kColSlice = 64;
+template <typename T>
+__global__ void __launch_bounds__(256)
+    colsum_partial_kernel(const T* __restrict__ a, int64_t rows, int64_t cols, int64_t lda,
+                          float* __restrict__ part) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int64_t c = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
+    if (c >= cols) return;
+    const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kColSlice;
+    const int64_t r1 = min(rows, r0 + kColSlice);
+    float s = 0.0f;
+    for (int64_t r = r0; r < r1; ++r) s += ld(a, r * lda + c);
+    part[static_cast<int64_t>(blockIdx.y) * cols + c] = s;
+}
+
+__global__ void __launch_bounds__(256)
+    colsum_reduce_kernel(const float* __restrict__ part, int64_t slices, int64_t cols, float* __restrict__ out,
+                         int accumulate) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int64_t c = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
+    if (c >= cols) return;
+    float s = 0.0f;
+    for (int64_t y = 0; y < slices; ++y) s += part[y * cols + c];
+    out[c] = accumulate ? out[c] + s : s;
+}
+
+// LayerNorm backward, one warp per row of D (a multiple of 32, at most 1024)
+// values: with x_hat = (x - mean) rstd and g = dy gamma,
+//   dx = rstd (g - mean(g) - x_hat mean(g x_hat))  (+ add, if given)
+// and gprod = dy x_hat per element (its column sums are dgamma).
+__global__ void __launch_bounds__(256)
+    ln_backward_kernel(const float* __restrict__ x, const float* __restrict__ gamma,
+                       const float* __restrict__ dy, const float* __restrict__ add, float eps, int64_t N,
+                       int D, float* __restrict__ dx, float* __restrict__ gprod) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int lane = threadIdx.x & 31;
+    const int64_t row = blockIdx.x * static_cast<int64_t>(blockDim.x / 32) + (threadIdx.x >> 5);
+    if (row >= N) return;
+    const float* xr = x + row * D;
+    const float* dr = dy + row * D;
+    const int per = D / 32;   // <= 32
+    float xv[32], gv[32];
+    float s = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+        if (i < per) {
+            xv[i] = xr[i * 32 + lane];
+            s += xv[i];
+        }
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    const float mean = s / D;
+    float v = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+        if (i < per) {
+            const float d = xv[i] - mean;
+            v = fmaf(d, d, v);
+        }
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    const float rstd = rsqrtf(v / D + eps);
+    float sg = 0.0f, sgx = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+        if (i < per) {
+            const int c = i * 32 + lane;
+            const float dyv = dr[c];
+            xv[i] = (xv[i] - mean) * rstd;
+            gv[i] = dyv * __ldg(gamma + c);
+            sg += gv[i];
+            sgx = fmaf(gv[i], xv[i], sgx);
+            gprod[row * D + c] = dyv * xv[i];
+        }
+    for (int o = 16; o > 0; o >>= 1) {
+        sg += __shfl_xor_sync(0xffffffffu, sg, o);
+        sgx += __shfl_xor_sync(0xffffffffu, sgx, o);
+    }
+    const float mg = sg / D, mgx = sgx / D;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+        if (i < per) {
+            const int64_t k = row * D + i * 32 + lane;
+            float d = rstd * (gv[i] - mg - xv[i] * mgx);
+            if (add) d += add[k];
+            dx[k] = d;
+        }
+}
+
+// dpre = dg * GELU'(pre), GELU'(x) = Phi(x) + x phi(x), in place on dg.
+__global__ void __launch_bounds__(256)
+    gelu_backward_kernel(float* __restrict__ dg, const float* __restrict__ pre, int64_t n) {
+    pdl_launch_dependents();
+    pdl_wait();
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const float x = pre[i];
+        const float Phi = 0.5f * erfcf(-x * 0.70710678118654752f);
+        const float phi = 0.39894228040143268f * expf(-0.5f * x * x);
+        dg[i] *= fmaf(x, phi, Phi);
+    }
+}
+
+// The repairer RoPE rotated q and k of every head by angle p_t f_i (pairs
+// (i, i + d/2)); its transpose rotates the gradients back:
+//   (a, b) -> (a cos + b sin, b cos - a sin).  dqkv [N, 3 d_b] fp32, Q and K
+// columns [0, 2 d_b); table [N, d/2] (cos, sin) of the forward.
+__global__ void __launch_bounds__(256)
+    rope_backward_kernel(float* __restrict__ dqkv, const float2* __restrict__ table, int64_t N, int db,
+                         int hd) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int half = hd / 2;
+    const int64_t pairs_per_row = static_cast<int64_t>(2 * db / hd) * half;   // Q and K heads
+    const int64_t total = N * pairs_per_row;
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t t = i / pairs_per_row;
+        const int64_t rem = i - t * pairs_per_row;
+        const int64_t h = rem / half;
+        const int j = static_cast<int>(rem - h * half);
+        const float2 cs = table[t * half + j];
+        float* base = dqkv + t * 3 * db + h * hd;
+        const float a = base[j], b = base[j + half];
+        base[j] = a * cs.x + b * cs.y;
+        base[j + half] = b * cs.x - a * cs.y;
+    }
+}
+
+// Masked softmax of each score row in place, one warp per (head, row): S
+// [heads, n, n] fp32 already scaled; key j visible to row i iff
+// lo(i) <= j < hi(i) (the mask modes of the attention kernel).
+__device__ __forceinline__ void visible_keys(const SoftmaxParams& p, int i, int* lo, int* hi) {
+    int a = (p.mask_mode == CR_MASK_BLOCK_DIAGONAL) ? p.chunk_start[i] : 0;
+    int b = (p.mask_mode == CR_MASK_TOKEN_CAUSAL) ? i + 1
+            : (p.mask_mode == CR_MASK_BIDIRECTIONAL) ? p.n
+                                                     : p.chunk_end[i];
+    b = min(max(b, 0), p.n);   // stay inside the row whatever the map holds
+    *lo = min(max(a, 0), b);
+    *hi = b;
+}
+
+__global__ void __launch_bounds__(256) softmax_rows_kernel(float* __restrict__ S, const __grid_constant__ SoftmaxParams p) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int lane = threadIdx.x & 31;
+    const int64_t w = blockIdx.x * static_cast<int64_t>(blockDim.x / 32) + (threadIdx.x >> 5);
+    if (w >= static_cast<int64_t>(p.heads) * p.n) return;
+    const int i = static_cast<int>(w % p.n);
+    float* row = S + w * p.n;
+    int lo, hi;
+    visible_keys(p, i, &lo, &hi);
+    float mx = -INFINITY;
+    for (int j = lo + lane; j < hi; j += 32) mx = fmaxf(mx, row[j]);
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    float sum = 0.0f;
+    for (int j = lo + lane; j < hi; j += 32) {
+        const float e = expf(row[j] - mx);
+        row[j] = e;
+        sum += e;
+    }
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    const float inv = 1.0f / sum;
+    for (int j = lane; j < p.n; j += 32) row[j] = (j >= lo && j < hi) ? row[j] * inv : 0.0f;
+}
+
+// dS = P (dP - sum_j P dP) per row, in place on dP (masked entries have P = 0).
+__global__ void __launch_bounds__(256)
+    softmax_bwd_kernel(const float* __restrict__ P, float* __restrict__ dP, const __grid_constant__ SoftmaxParams p) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int lane = threadIdx.x & 31;
+    const int64_t w = blockIdx.x * static_cast<int64_t>(blockDim.x / 32) + (threadIdx.x >> 5);
+    if (w >= static_cast<int64_t>(p.heads) * p.n) return;
+    const float* pr = P + w * p.n;
+    float* dr = dP + w * p.n;
+    float s = 0.0f;
+    for (int j = lane; j < p.n; j += 32) s = fmaf(pr[j], dr[j], s);
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    for (int j = lane; j < p.n; j += 32) dr[j] = pr[j] * (dr[j] - s);
+}
+
+// out[i] = in[i] * scale[i % cols] (dW_seg: the cache's 1 / sigma_stale per column)
+__global__ void __launch_bounds__(256)
+    scale_cols_kernel(float* __restrict__ a, int64_t n, const float* __restrict__ sigma, int64_t period,
+                      int64_t seg_cols, int64_t d_seg) {
+    pdl_launch_dependents();
+    pdl_wait();
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        // a = [S][d_seg][d_h]: element (s, ., j) divides by sigma[s d_h + j]
+        const int64_t s = i / period;
+        const int64_t j = i % seg_cols;
+        (void)d_seg;
+        a[i] /= __ldg(sigma + s * seg_cols + j);
+    }
+}
+
+__global__ void __launch_bounds__(256)
+    f32_from_bf16_kernel(const uint16_t* __restrict__ a, int64_t n, float* __restrict__ out) {
+    pdl_launch_dependents();
+    pdl_wait();
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x)
+        out[i] = bf16_to_f32(a[i]);
+}
+
+// Squared norm of the flat gradient: fp64 partial per CTA over a fixed range,
+// then the partials in order.  coef = min(1, max_norm / (norm + 1e-6)).
+constexpr int kNormCtas = 1024;
+__global__ void __launch_bounds__(256)
+    sqnorm_partial_kernel(const float* __restrict__ g, int64_t n, double* __restrict__ part) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int64_t per = (n + gridDim.x - 1) / gridDim.x;
+    const int64_t a = blockIdx.x * per, b = min(n, a + per);
+    float s = 0.0f;
+    for (int64_t i = a + threadIdx.x; i < b; i += blockDim.x) s = fmaf(g[i], g[i], s);
+    __shared__ double red[256];
+    red[threadIdx.x] = static_cast<double>(s);
+    __syncthreads();
+    for (int k = 128; k > 0; k >>= 1) {
+        if (static_cast<int>(threadIdx.x) < k) red[threadIdx.x] += red[threadIdx.x + k];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) part[blockIdx.x] = red[0];
+}
+
+__global__ void sqnorm_reduce_kernel(const double* __restrict__ part, int n_part, float max_norm,
+                                     float* __restrict__ stats) {
+    pdl_launch_dependents();
+    pdl_wait();
+    if (threadIdx.x != 0 || blockIdx.x != 0) return;
+    double s = 0.0;
+    for (int i = 0; i < n_part; ++i) s += part[i];
+    const double norm = sqrt(s);
+    stats[1] = static_cast<float>(norm);
+    stats[2] = static_cast<float>(fmin(1.0, static_cast<double>(max_norm) / (norm + 1e-6)));
+    stats[3] = 0.0f;
+}
+
+// AdamW on the flat parameter vector with the clipped gradient coef * g:
+//   theta <- theta (1 - lr wd); m <- b1 m + (1 - b1) g; v <- b2 v + (1 - b2) g^2;
+//   theta <- theta - lr (m / bc1) / (sqrt(v / bc2) + eps);  bf16 mirror rewritten.
+__global__ void __launch_bounds__(256)
+    adamw_kernel(float* __restrict__ p, float* __restrict__ m, float* __restrict__ v, const float* __restrict__ g,
+                 uint16_t* __restrict__ pb, int64_t n, const __grid_constant__ AdamWParams hp,
+                 const float* __restrict__ stats) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const float coef = stats[2];
+    for (int64_t q = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; q < n / 4;
+         q += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        float4 P4 = reinterpret_cast<float4*>(p)[q], M4 = reinterpret_cast<float4*>(m)[q];
+        float4 V4 = reinterpret_cast<float4*>(v)[q];
+        const float4 G4 = reinterpret_cast<const float4*>(g)[q];
+        float* pp = &P4.x;
+        float* mm = &M4.x;
+        float* vv = &V4.x;
+        const float* gg = &G4.x;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float gi = gg[k] * coef;
+            const float th = pp[k] * (1.0f - hp.lr * hp.wd);
+            mm[k] = hp.b1 * mm[k] + (1.0f - hp.b1) * gi;
+            vv[k] = hp.b2 * vv[k] + (1.0f - hp.b2) * gi * gi;
+            const float upd = (mm[k] / hp.bc1) / (sqrtf(vv[k] / hp.bc2) + hp.eps);
+            pp[k] = th - hp.lr * upd;
+        }
+        reinterpret_cast<float4*>(p)[q] = P4;
+        reinterpret_cast<float4*>(m)[q] = M4;
+        reinterpret_cast<float4*>(v)[q] = V4;
+        reinterpret_cast<uint2*>(pb)[q] = make_uint2(
+            static_cast<uint32_t>(f32_to_bf16(P4.x)) | (static_cast<uint32_t>(f32_to_bf16(P4.y)) << 16),
+            static_cast<uint32_t>(f32_to_bf16(P4.z)) | (static_cast<uint32_t>(f32_to_bf16(P4.w)) << 16));
+    }
+}
+
+__global__ void __launch_bounds__(256) fill_kernel(float* __restrict__ p, int64_t n, float v) {
+    pdl_launch_dependents();
+    pdl_wait();
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x)
+        p[i] = v;
+}
+
+dim3 grid_for(int64_t n, int64_t cap_per_sm = 16) {
+    int64_t b = (n + 255) / 256;
+    const int64_t cap = static_cast<int64_t>(num_sms()) * cap_per_sm;
+    if (b > cap) b = cap;
+    if (b < 1) b = 1;
+    return dim3(static_cast<unsigned>(b));
+}
+
+}  // namespace
+
+cr_status launch_fill(float* p, int64_t n, float v, cudaStream_t st) {
+    return launch_pdl(fill_kernel, grid_for(n), dim3(256), 0, st, p, n, v);
+}
+
+cr_status launch_target(const void* stale, const void* joint, bool f32, const float* sd, int64_t n,
+                        int64_t D, float* out, cudaStream_t st) {
+    if (f32 || D % 8 != 0) return CR_ERR_UNSUPPORTED;
+    return launch_pdl(target_kernel, grid_for(n * D / 8), dim3(256), 0, st,
+                      static_cast<const uint16_t*>(stale), static_cast<const uint16_t*>(joint), sd, n, D, out);
+}
+
+cr_status launch_loss(const float* r, int64_t N, int64_t D, const LossParams& p, uint16_t* dz, float* rowsq,
+                      float* loss_out, double* per_req, cudaStream_t st) {
+    cr_status s = launch_pdl(loss_grad_kernel, dim3(static_cast<unsigned>(N)), dim3(256), 0, st, r, D, p,
+                             dz, rowsq);
+    if (s != CR_OK) return s;
+    s = launch_pdl(loss_reduce_kernel, dim3(static_cast<unsigned>(p.n_req)), dim3(256), 0, st, rowsq, p, D,
+                   per_req);
+    if (s != CR_OK) return s;
+    return launch_pdl(loss_total_kernel, dim3(1), dim3(32), 0, st, static_cast<const double*>(per_req), p.n_req,
+                      loss_out);
+}
+
+size_t colsum_scratch_floats(int64_t rows, int64_t cols) {
+    return static_cast<size_t>((rows + kColSlice - 1) / kColSlice) * static_cast<size_t>(cols);
+}
+
+cr_status launch_colsum(const void* a, bool bf16, int64_t rows, int64_t cols, int64_t lda, float* out,
+                        bool accumulate, float* scratch, cudaStream_t st) {
+    const int64_t slices = (rows + kColSlice - 1) / kColSlice;
+    const dim3 g1(static_cast<unsigned>((cols + 255) / 256), static_cast<unsigned>(slices));
+    cr_status s = bf16 ? launch_pdl(colsum_partial_kernel<uint16_t>, g1, dim3(256), 0, st,
+                                    static_cast<const uint16_t*>(a), rows, cols, lda, scratch)
+                       : launch_pdl(colsum_partial_kernel<float>, g1, dim3(256), 0, st,
+                                    static_cast<const float*>(a), rows, cols, lda, scratch);
+    if (s != CR_OK) return s;
+    return launch_pdl(colsum_reduce_kernel, dim3(static_cast<unsigned>((cols + 255) / 256)), dim3(256), 0, st,
+                      static_cast<const float*>(scratch), slices, cols, out, accumulate ? 1 : 0);
+}
+
+cr_status launch_ln_backward(const float* x, const float* gamma, const float* dy, const float* add, float eps,
+                             int64_t N, int D, float* dx, float* gprod, cudaStream_t st) {
+    if (D % 32 != 0 || D > 1024) return CR_ERR_UNSUPPORTED;
+    return launch_pdl(ln_backward_kernel, dim3(static_cast<unsigned>((N + 7) / 8)), dim3(256), 0, st, x, gamma,
+                      dy, add, eps, N, D, dx, gprod);
+}
+
+cr_status launch_gelu_backward(float* dg, const float* pre, int64_t n, cudaStream_t st) {
+    return launch_pdl(gelu_backward_kernel, grid_for(n), dim3(256), 0, st, dg, pre, n);
+}
+
+cr_status launch_rope_backward(float* dqkv, const float2* table, int64_t N, int db, int hd, cudaStream_t st) {
+    return launch_pdl(rope_backward_kernel, grid_for(N * db), dim3(256), 0, st, dqkv, table, N, db, hd);
+}
+
+cr_status launch_softmax_rows(float* S, const SoftmaxParams& p, cudaStream_t st) {
+    const int64_t warps = static_cast<int64_t>(p.heads) * p.n;
+    return launch_pdl(softmax_rows_kernel, dim3(static_cast<unsigned>((warps + 7) / 8)), dim3(256), 0, st, S, p);
+}
+
+cr_status launch_softmax_bwd(const float* P, float* dP, const SoftmaxParams& p, cudaStream_t st) {
+    const int64_t warps = static_cast<int64_t>(p.heads) * p.n;
+    return launch_pdl(softmax_bwd_kernel, dim3(static_cast<unsigned>((warps + 7) / 8)), dim3(256), 0, st, P, dP, p);
+}
+
+cr_status launch_scale_seg_grad(float* g, int64_t S, int64_t dseg, int64_t dh, const float* sigma,
+                                cudaStream_t st) {
+    const int64_t n = S * dseg * dh;
+    return launch_pdl(scale_cols_kernel, grid_for(n), dim3(256), 0, st, g, n, sigma, dseg * dh, dh, dseg);
+}
+
+cr_status launch_f32_from_bf16(const uint16_t* a, int64_t n, float* out, cudaStream_t st) {
+    return launch_pdl(f32_from_bf16_kernel, grid_for(n), dim3(256), 0, st, a, n, out);
+}
+
+size_t sqnorm_scratch_doubles() { return kNormCtas; }
+
+cr_status launch_clip_adamw(float* p, float* m, float* v, const float* g, uint16_t* pb, int64_t n,
+                            const AdamWParams& hp, float max_norm, double* scratch, float* stats,
+                            cudaStream_t st) {
+    cr_status s = launch_pdl(sqnorm_partial_kernel, dim3(kNormCtas), dim3(256), 0, st, g, n, scratch);
+    if (s != CR_OK) return s;
+    s = launch_pdl(sqnorm_reduce_kernel, dim3(1), dim3(32), 0, st, static_cast<const double*>(scratch),
+                   kNormCtas, max_norm, stats);
+    if (s != CR_OK) return s;
+    if (n % 4 != 0) return CR_ERR_UNSUPPORTED;
+    return launch_pdl(adamw_kernel, grid_for(n / 4), dim3(256), 0, st, p, m, v, g, pb, n, hp,
+                      static_cast<const float*>(stats));
+}
+
+// ------------------------------------------------------------------ cuBLAS, row-major
+// One handle per device, created on first use; its workspace is set to a
+// caller-provided region before every call, so cuBLAS allocates nothing per call.
+namespace {
+cublasHandle_t g_blas[64];
+}
+
+cr_status blas_handle(cudaStream_t st, void* ws, size_t ws_bytes, cublasHandle_t* out) {
+    const int d = current_device_index();
+    if (d < 0 || d >= 64) return CR_ERR_CUDA;
+    if (!g_blas[d]) {
+        cublasHandle_t h;
+        if (cublasCreate(&h) != CUBLAS_STATUS_SUCCESS) return CR_ERR_CUDA;
+        cublasHandle_t expected = nullptr;
+        if (!__atomic_compare_exchange_n(&g_blas[d], &expected, h, false, __ATOMIC_ACQ_REL, __ATOMIC_ACQUIRE))
+            cublasDestroy(h);
+    }
+    cublasHandle_t h = g_blas[d];
+    if (cublasSetStream(h, st) != CUBLAS_STATUS_SUCCESS) return CR_ERR_CUDA;
+    if (cublasSetWorkspace(h, ws, ws_bytes) != CUBLAS_STATUS_SUCCESS) return CR_ERR_CUDA;
+    *out = h;
+    return CR_OK;
+}
+
+// Row-major C[M, N] = alpha op(A) op(B) + beta C, op(A) [M, K], op(B) [K, N];
+// tA: A is stored [K, M] (op(A) = A^T); tB: B is stored [N, K].  In cuBLAS's
+// column-major terms this is C^T = op(B)^T op(A)^T on the same memory.
+cr_status gemm_rm(cublasHandle_t h, bool tA, bool tB, int64_t M, int64_t N, int64_t K, float alpha,
+                  const void* A, cudaDataType_t ta, int64_t lda, const void* B, cudaDataType_t tb, int64_t ldb,
+                  float beta, void* C, cudaDataType_t tc, int64_t ldc, int64_t batch, int64_t sA, int64_t sB,
+                  int64_t sC) {
+    const cublasComputeType_t ct = (ta == CUDA_R_32F) ? CUBLAS_COMPUTE_32F_FAST_TF32 : CUBLAS_COMPUTE_32F;
+    cublasStatus_t e;
+    if (batch <= 1)
+        e = cublasGemmEx(h, tB ? CUBLAS_OP_T : CUBLAS_OP_N, tA ? CUBLAS_OP_T : CUBLAS_OP_N, static_cast<int>(N),
+                         static_cast<int>(M), static_cast<int>(K), &alpha, B, tb, static_cast<int>(ldb), A, ta,
+                         static_cast<int>(lda), &beta, C, tc, static_cast<int>(ldc), ct, CUBLAS_GEMM_DEFAULT);
+    else
+        e = cublasGemmStridedBatchedEx(h, tB ? CUBLAS_OP_T : CUBLAS_OP_N, tA ? CUBLAS_OP_T : CUBLAS_OP_N,
+                                       static_cast<int>(N), static_cast<int>(M), static_cast<int>(K), &alpha, B,
+                                       tb, static_cast<int>(ldb), sB, A, ta, static_cast<int>(lda), sA, &beta, C,
+                                       tc, static_cast<int>(ldc), sC, static_cast<int>(batch), ct,
+                                       CUBLAS_GEMM_DEFAULT);
+    return e == CUBLAS_STATUS_SUCCESS ? CR_OK : CR_ERR_CUDA;
+}
+
+}  // namespace cr

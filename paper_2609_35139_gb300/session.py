@@ -223,3 +223,62 @@ class RepairPipeline:
         cur = torch.cuda.current_stream(self.device)
         for s in range(2):
             cur.wait_event(self.ev_d2h[s])
+
+
+# ------------------------------------------------------------------ training (Sec. 4.2, App. A)
+_TRAIN_TOP = ["w_seg", "b_seg", "w_map", "b_map", "w_tok", "b_tok", "w_fuse", "b_fuse", "w_rein", "b_rein"]
+_TRAIN_BLOCK = ["ln1_g", "ln1_b", "w_qkv", "b_qkv", "w_o", "b_o", "ln2_g", "ln2_b", "w_fc1", "b_fc1",
+                "w_fc2", "b_fc2"]
+_TRAIN_END = ["lnf_g", "lnf_b", "w_out", "b_out"]
+
+
+def trained_tensor_names(n_blocks: int):
+    """The trained tensors in the order of the flat parameter vector (include/cr.h)."""
+    return _TRAIN_TOP + [f"blk{b}.{k}" for b in range(n_blocks) for k in _TRAIN_BLOCK] + _TRAIN_END
+
+
+class TrainSession:
+    """Training state of the repair network on one GPU: the flat fp32 master weights and
+    their bf16 copy, the AdamW moments, the last gradient and the workspace; `step` runs
+    one update (forward, objective, backward, clipping, AdamW) through cr_train_step."""
+
+    def __init__(self, target: cr.cr_target_dims, rep: cr.cr_repairer_dims, w: Dict[str, np.ndarray],
+                 max_tokens: int, max_request_tokens: int, device="cuda"):
+        self.target, self.rep = target, rep
+        self.device = torch.device(device)
+        self.names = trained_tensor_names(rep.n_blocks)
+        self.offsets = cr.cr_param_layout(target, rep)
+        P = int(self.offsets[-1])
+        flat = np.zeros(P, np.float32)
+        for k, name in enumerate(self.names):
+            a = np.asarray(w[name])
+            a = (a.astype(np.uint32) << 16).view(np.float32) if a.dtype == np.uint16 else a.astype(np.float32)
+            flat[self.offsets[k]:self.offsets[k] + a.size] = a.ravel()
+        self.params = torch.from_numpy(flat).to(self.device)
+        self.params_bf16 = self.params.to(torch.bfloat16)
+        self.adam_m = torch.zeros_like(self.params)
+        self.adam_v = torch.zeros_like(self.params)
+        self.grads = torch.zeros_like(self.params)
+        self.sigma_stale = torch.from_numpy(np.asarray(w["sigma_stale"], np.float32)).to(self.device)
+        self.sigma_delta = torch.from_numpy(np.asarray(w["sigma_delta"], np.float32)).to(self.device)
+        self.stats = torch.zeros(4, dtype=torch.float32, device=self.device)
+        ws = cr.cr_train_workspace_bytes(target, rep, max_tokens, max_request_tokens)
+        if ws == 0:
+            raise cr.CrError("cr_train_workspace_bytes", cr.CR_ERR_INVALID_ARG, "invalid dimensions")
+        self.workspace = torch.empty((ws + 15) // 16 * 16, dtype=torch.uint8, device=self.device)
+        self.n_steps = 0
+
+    def view(self, t: torch.Tensor, name: str) -> torch.Tensor:
+        k = self.names.index(name)
+        a, b = int(self.offsets[k]), int(self.offsets[k + 1])
+        return t[a:b]
+
+    def step(self, kv_stale, kv_joint, emb, chunk_end, pos, cu_seqlens_host, n_tokens, lr, *,
+             beta1=0.9, beta2=0.95, eps=1e-8, weight_decay=0.01, max_grad_norm=1.0, stream=None):
+        """One AdamW update; returns the device stats tensor (loss, grad norm, clip coef, 0)."""
+        self.n_steps += 1
+        hp = cr.cr_adamw(lr, beta1, beta2, eps, weight_decay, max_grad_norm, self.n_steps)
+        cr.cr_train_step(self.target, self.rep, self.params, self.params_bf16, self.adam_m, self.adam_v,
+                         self.grads, self.sigma_stale, self.sigma_delta, kv_stale, kv_joint, emb, chunk_end,
+                         pos, cu_seqlens_host, n_tokens, hp, self.stats, self.workspace, stream)
+        return self.stats
