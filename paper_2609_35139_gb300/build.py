@@ -28,7 +28,7 @@ CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relax
           "-diag-suppress", "177",
           "-I" + INCLUDE, "-I" + CSRC]
 SOURCES = ["cr_api.cu", "cr_gemm.cu", "cr_attn.cu", "cr_segproj.cu", "cr_misc.cu",
-           "cr_noalloc.cu", "cr_offline.cu", "cr_train.cu"]
+           "cr_noalloc.cu", "cr_offline.cu", "cr_train.cu", "cr_attn_bwd.cu"]
 # the training step's plain (unfused) backward GEMMs go through cuBLAS
 LIBS = ["-lcublas"]
 

@@ -5,6 +5,7 @@
 #include <cuda_runtime.h>
 #include <math.h>
 #include <algorithm>
+#include <memory>
 #include <mutex>
 #include <vector>
 #include <string.h>
@@ -930,12 +931,12 @@ cr_status cr_param_layout(const cr_target_dims* target, const cr_repairer_dims* 
 namespace {
 struct TrainLayout {
     size_t inf, h0, rein, blk, blk_stride, hbuf, yf, rope, ones, r, dz, rowsq, perreq, stats_pad, dh, dxm,
-        du, dtmp, pre, gprod, sig16, qkv32, dqkv, da, sbuf, dpbuf, dse, dy, colsum, norm, blas, total;
+        du, dtmp, pre, gprod, sig16, dqkv, da, lse, dvec, cstart, dse, dy, colsum, norm, blas, total;
     size_t x_in, x_mid, u1, u2, qkv, o, g;   // offsets inside one block's region
 };
 constexpr size_t kBlasBytes = 32ull << 20;
 
-TrainLayout train_layout(const Dims& d, int64_t n, int64_t nmax) {
+TrainLayout train_layout(const Dims& d, int64_t n) {
     TrainLayout L{};
     size_t off = 0;
     auto take = [&](size_t bytes) {
@@ -979,11 +980,11 @@ TrainLayout train_layout(const Dims& d, int64_t n, int64_t nmax) {
     L.pre = take(N * d.hid * 4);
     L.gprod = take(N * d.db * 4);
     L.sig16 = take(N * wide * 2);
-    L.qkv32 = take(N * 3 * d.db * 4);
     L.dqkv = take(N * 3 * d.db * 4);
     L.da = take(N * d.db * 4);
-    L.sbuf = take(static_cast<size_t>(d.nh) * nmax * nmax * 4);
-    L.dpbuf = take(static_cast<size_t>(d.nh) * nmax * nmax * 4);
+    L.lse = take(static_cast<size_t>(d.B > 0 ? d.B : 1) * d.nh * N * 4);   // per block [heads][N]
+    L.dvec = take(static_cast<size_t>(d.nh) * N * 4);
+    L.cstart = take(N * 4);
     L.dse = take(N * 2 * d.dc * 4);
     L.dy = take(N * d.S * d.dseg * 4);
     L.colsum = take(colsum_scratch_floats(n, std::max(d.D, wide)) * 4);
@@ -1000,7 +1001,7 @@ size_t cr_train_workspace_bytes(const cr_target_dims* target, const cr_repairer_
     if (max_tokens < 1 || max_request_tokens < 1 || max_request_tokens > max_tokens ||
         max_tokens > INT32_MAX / 2)
         return 0;
-    return train_layout(dims_of(target, rep), max_tokens, max_request_tokens).total;
+    return train_layout(dims_of(target, rep), max_tokens).total;
 }
 
 cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* rep, float* params,
@@ -1033,7 +1034,7 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
         nmax = std::max(nmax, len);
     }
     const int64_t N = n_tokens;
-    const TrainLayout L = train_layout(d, N, nmax);
+    const TrainLayout L = train_layout(d, N);
     if (workspace_bytes < L.total) return CR_ERR_INVALID_ARG;
     int64_t off[14 + 12 * 64 + 1];
     const int nt = train_offsets(d, off, 14 + 12 * 64 + 1);
@@ -1114,11 +1115,11 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
     float* PRE = at<float>(base, L.pre);
     float* GPROD = at<float>(base, L.gprod);
     uint16_t* SIG = at<uint16_t>(base, L.sig16);
-    float* QKV32 = at<float>(base, L.qkv32);
     float* DQKV = at<float>(base, L.dqkv);
     float* DA = at<float>(base, L.da);
-    float* SB = at<float>(base, L.sbuf);
-    float* DPB = at<float>(base, L.dpbuf);
+    float* LSE = at<float>(base, L.lse);
+    float* DVEC = at<float>(base, L.dvec);
+    int32_t* CSTART = at<int32_t>(base, L.cstart);
     float* DSE = at<float>(base, L.dse);
     float* DY = at<float>(base, L.dy);
     float* CS = at<float>(base, L.colsum);
@@ -1137,6 +1138,26 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
     gq.rope_cols = static_cast<int32_t>(2 * db);
     repairer_inv_freq(gq.inv_freq, static_cast<int>(hd), rep->rope_theta);
     if (s == CR_OK && B > 0) s = launch_rope_table(pos, N, static_cast<int>(hd / 2), gq.inv_freq, rope, st);
+    // chunk starts, for the attention backward's walk of each key tile's queries
+    if (s == CR_OK && B > 0) s = launch_chunk_starts(chunk_end, *ap, N, CSTART, st);
+    std::unique_ptr<AttnBwdParams> bp_own(new AttnBwdParams());
+    AttnBwdParams* bp = bp_own.get();
+    bp->chunk_end = chunk_end;
+    bp->chunk_start = CSTART;
+    bp->d_b = static_cast<int32_t>(db);
+    bp->n_heads = static_cast<int32_t>(d.nh);
+    bp->n_req = n_req;
+    bp->mask_mode = CR_MASK_BLOCK_CAUSAL;
+    bp->scale_log2 = ap->scale_log2;
+    bp->scale = static_cast<float>(1.0 / sqrt(static_cast<double>(hd)));
+    bp->status = status;
+    for (int r = 0; r < n_req; ++r) {
+        bp->req_start[r] = cu_seqlens_host[r];
+        bp->tile_prefix[r] = bp->n_items;
+        bp->n_items += (cu_seqlens_host[r + 1] - cu_seqlens_host[r] + 127) / 128;
+    }
+    bp->req_start[n_req] = cu_seqlens_host[n_req];
+    bp->tile_prefix[n_req] = bp->n_items;
     gq.rope_table = rope;
     GemmParams gr{};
     gr.status = status;
@@ -1157,6 +1178,7 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
         gq.ldo = 3 * db;
         if ((s = launch_gemm(u1, db, k.w_qkv, N, 3 * db, db, EPI_QKV_ROPE, gq, nullptr, 0, st)) != CR_OK) break;
         ap->out = o;
+        ap->lse = LSE + b * d.nh * N;
         if ((s = launch_attention(qkv, N, static_cast<int>(hd), *ap, st)) != CR_OK) break;
         if ((s = cuda_check(cudaMemcpyAsync(x_mid, x_in, static_cast<size_t>(N * db) * 4,
                                             cudaMemcpyDeviceToDevice, st))) != CR_OK)
@@ -1228,7 +1250,6 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
     CR_TRY(colsum(GPROD, false, db, db, gk(LNFG)));
     CR_TRY(colsum(DU, false, db, db, gk(LNFB)));
     CR_TRY(cuda_check(cudaMemsetAsync(DSE, 0, static_cast<size_t>(N * 2 * dc) * 4, st)));
-    const float scale = static_cast<float>(1.0 / sqrt(static_cast<double>(hd)));
     for (int64_t b = B - 1; b >= 0; --b) {
         const float* x_in = reinterpret_cast<const float*>(blk(b, L.x_in));
         const float* x_mid = reinterpret_cast<const float*>(blk(b, L.x_mid));
@@ -1265,35 +1286,12 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
         CR_TRY(gemm_rm(hb, true, false, db, db, N, 1.0f, SIG, BF, db, o, BF, db, 0.0f, gk(bk(b, WO)), F32, db));
         CR_TRY(colsum(DXM, false, db, db, gk(bk(b, BO))));
         CR_TRY(gemm_rm(hb, false, false, N, db, db, 1.0f, SIG, BF, db, pb(bk(b, WO)), BF, db, 0.0f, DA, F32, db));
-        // attention, per request, heads batched: S = Q K^T scale; P = softmax;
-        // dV = P^T dA; dP = dA V^T; dS = P (dP - rowsum(P dP)); dQ = dS K scale; dK = dS^T Q scale
-        CR_TRY(launch_f32_from_bf16(qkv, N * 3 * db, QKV32, st));
-        for (int r = 0; r < n_req; ++r) {
-            const int64_t lo = cu_seqlens_host[r], n = cu_seqlens_host[r + 1] - lo;
-            const float* Q = QKV32 + lo * 3 * db;
-            const float* K = Q + db;
-            const float* V = Q + 2 * db;
-            const float* dA = DA + lo * db;
-            float* dQ = DQKV + lo * 3 * db;
-            const int64_t nn = n * n;
-            CR_TRY(gemm_rm(hb, false, true, n, n, hd, scale, Q, F32, 3 * db, K, F32, 3 * db, 0.0f, SB, F32, n,
-                           d.nh, hd, hd, nn));
-            SoftmaxParams sp{};
-            sp.n = static_cast<int32_t>(n);
-            sp.heads = static_cast<int32_t>(d.nh);
-            sp.mask_mode = CR_MASK_BLOCK_CAUSAL;
-            sp.chunk_end = chunk_end + lo;
-            CR_TRY(launch_softmax_rows(SB, sp, st));
-            CR_TRY(gemm_rm(hb, true, false, n, hd, n, 1.0f, SB, F32, n, dA, F32, db, 0.0f, dQ + 2 * db, F32,
-                           3 * db, d.nh, nn, hd, hd));
-            CR_TRY(gemm_rm(hb, false, true, n, n, hd, 1.0f, dA, F32, db, V, F32, 3 * db, 0.0f, DPB, F32, n, d.nh,
-                           hd, hd, nn));
-            CR_TRY(launch_softmax_bwd(SB, DPB, sp, st));
-            CR_TRY(gemm_rm(hb, false, false, n, hd, n, scale, DPB, F32, n, K, F32, 3 * db, 0.0f, dQ, F32, 3 * db,
-                           d.nh, nn, hd, hd));
-            CR_TRY(gemm_rm(hb, true, false, n, hd, n, scale, DPB, F32, n, Q, F32, 3 * db, 0.0f, dQ + db, F32,
-                           3 * db, d.nh, nn, hd, hd));
-        }
+        // attention: the fused backward (P recomputed from the forward's log-sum-exp,
+        // dQ, dK, dV into dqkv), dO in bf16 for its MMAs
+        CR_TRY(to16(DA, N * db, SIG));
+        bp->lse = LSE + b * d.nh * N;
+        bp->dqkv = DQKV;
+        CR_TRY(launch_attention_backward(qkv, SIG, DA, o, N, static_cast<int>(hd), *bp, DVEC, st));
         CR_TRY(launch_rope_backward(DQKV, rope, N, static_cast<int>(db), static_cast<int>(hd), st));
         // qkv = W_qkv u1 + b_qkv;  u1 = LN1(x_in): dx_in = dx_mid + LN1 backward
         CR_TRY(to16(DQKV, N * 3 * db, SIG));

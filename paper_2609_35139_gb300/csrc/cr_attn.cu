@@ -89,7 +89,9 @@ __device__ __forceinline__ int key_lo(const AttnParams& p, int rs, int i) {
     return p.mask_mode == CR_MASK_BLOCK_DIAGONAL ? __ldg(p.chunk_start + rs + i) : 0;
 }
 
-template <int D>
+// kLse: also write each row's log-sum-exp (for the training step's backward);
+// the inference forward's instantiation has none of that code.
+template <int D, bool kLse>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQKV, const __grid_constant__ AttnParams p) {
     using Cfg = AttnCfg<D>;
@@ -433,6 +435,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (ok && n > jl) {
             tc_fence_after();
             const float inv = 1.0f / l;
+            // the row's log-sum-exp for a backward pass: P = 2^(s sc - (m + log2 l))
+            if (kLse && valid)
+                p.lse[static_cast<int64_t>(head) * p.req_start[p.n_req] + rs + qrow] = m + log2f(l);
             uint16_t* dst = p.out + static_cast<int64_t>(rs + qrow) * p.d_b + head * D;
 #pragma unroll
             for (int c = 0; c < D; c += 16) {
@@ -460,10 +465,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-template <int D>
+template <int D, bool kLse>
 cr_status launch_d(const CUtensorMap& tm, const AttnParams& p, cudaStream_t st) {
     using Cfg = AttnCfg<D>;
-    auto kern = attn_kernel<D>;
+    auto kern = attn_kernel<D, kLse>;
     static unsigned long long attr_done = 0;   // one per template instantiation
     const cr_status sa = ensure_smem_attr(kern, static_cast<int>(Cfg::kSmemBytes), &attr_done);
     if (sa != CR_OK) return sa;
@@ -533,7 +538,8 @@ cr_status launch_attention(const uint16_t* qkv, int64_t n_tokens, int head_dim,
                       3ull * p.d_b * 2, head_dim, 128,
                       head_dim == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B))
         return CR_ERR_INVALID_ARG;
-    return head_dim == 64 ? launch_d<64>(tm, p, st) : launch_d<32>(tm, p, st);
+    if (p.lse) return head_dim == 64 ? launch_d<64, true>(tm, p, st) : launch_d<32, true>(tm, p, st);
+    return head_dim == 64 ? launch_d<64, false>(tm, p, st) : launch_d<32, false>(tm, p, st);
 }
 
 }  // namespace cr

@@ -114,6 +114,22 @@ struct AttnParams {
     unsigned* status;
     int32_t req_start[kMaxReq + 1];   // cu_seqlens
     int32_t tile_prefix[kMaxReq + 1]; // cumulative items per request
+    float* lse;                  // [heads][N] or null: log2-unit log-sum-exp of each row (training)
+};
+
+// attention backward (training step)
+struct AttnBwdParams {
+    const int32_t* chunk_end;     // [N] request-local
+    const int32_t* chunk_start;   // [N] request-local
+    const float* lse;             // [heads][N] the forward's log-sum-exp (log2 units, scale folded in)
+    const float* dvec;            // [heads][N] sum_d dO O
+    float* dqkv;                  // [N, 3 d_b] fp32: dQ, dK, dV
+    int32_t d_b, n_heads, n_req, n_items, mask_mode;
+    float scale_log2;             // log2(e) / sqrt(d)
+    float scale;                  // 1 / sqrt(d)
+    unsigned* status;
+    int32_t req_start[kMaxReq + 1];
+    int32_t tile_prefix[kMaxReq + 1];   // cumulative 128-row tiles per request
 };
 
 // ------------------------------------------------------------------ training step
@@ -121,11 +137,6 @@ struct LossParams {
     int32_t n_req;
     int32_t req_start[kMaxReq + 1];
     float scale[kMaxReq];     // dL/dr factor of each request: 2 / (N_r D_KV n_req)
-};
-struct SoftmaxParams {
-    int32_t n, heads, mask_mode;
-    const int32_t* chunk_end;     // request-local
-    const int32_t* chunk_start;   // request-local (block-diagonal mask only)
 };
 struct AdamWParams {
     float lr, b1, b2, eps, wd, bc1, bc2;
@@ -207,6 +218,9 @@ cr_status launch_chunk_starts(const int32_t* chunk_end, const AttnParams& p, int
 cr_status launch_attention(const uint16_t* qkv, int64_t n_tokens, int head_dim,
                            const AttnParams& p, cudaStream_t st);
 
+cr_status launch_attention_backward(const uint16_t* qkv, const uint16_t* dO16, const float* dO, const uint16_t* O,
+                                    int64_t n_tokens, int head_dim, AttnBwdParams& p, float* dvec, cudaStream_t st);
+
 // training step (cr_train.cu)
 cr_status launch_fill(float* p, int64_t n, float v, cudaStream_t st);
 cr_status launch_target(const void* stale, const void* joint, bool f32, const float* sd, int64_t n,
@@ -220,11 +234,8 @@ cr_status launch_ln_backward(const float* x, const float* gamma, const float* dy
                              int64_t N, int D, float* dx, float* gprod, cudaStream_t st);
 cr_status launch_gelu_backward(float* dg, const float* pre, int64_t n, cudaStream_t st);
 cr_status launch_rope_backward(float* dqkv, const float2* table, int64_t N, int db, int hd, cudaStream_t st);
-cr_status launch_softmax_rows(float* S, const SoftmaxParams& p, cudaStream_t st);
-cr_status launch_softmax_bwd(const float* P, float* dP, const SoftmaxParams& p, cudaStream_t st);
 cr_status launch_scale_seg_grad(float* g, int64_t S, int64_t dseg, int64_t dh, const float* sigma,
                                 cudaStream_t st);
-cr_status launch_f32_from_bf16(const uint16_t* a, int64_t n, float* out, cudaStream_t st);
 size_t sqnorm_scratch_doubles();
 cr_status launch_clip_adamw(float* p, float* m, float* v, const float* g, uint16_t* pb, int64_t n,
                             const AdamWParams& hp, float max_norm, double* scratch, float* stats,

@@ -9,8 +9,6 @@
 //   ln_backward_kernel   LayerNorm backward per row, plus dy * x_hat per element
 //   gelu_backward_kernel dpre = dg * (Phi(pre) + pre phi(pre))
 //   rope_backward_kernel the repairer RoPE's transpose on dQ, dK
-//   softmax_rows_kernel  masked row softmax of the score matrix, in place
-//   softmax_bwd_kernel   dS = P (dP - rowsum(P dP)), in place on dP
 //   sqnorm_*             squared L2 norm of the gradient (fp64, fixed order)
 //   adamw_kernel         clipping coefficient, AdamW, bf16 mirror of the weights
 #include <cublas_v2.h>
@@ -266,59 +264,6 @@ __global__ void __launch_bounds__(256)
     }
 }
 
-// Masked softmax of each score row in place, one warp per (head, row): S
-// [heads, n, n] fp32 already scaled; key j visible to row i iff
-// lo(i) <= j < hi(i) (the mask modes of the attention kernel).
-__device__ __forceinline__ void visible_keys(const SoftmaxParams& p, int i, int* lo, int* hi) {
-    int a = (p.mask_mode == CR_MASK_BLOCK_DIAGONAL) ? p.chunk_start[i] : 0;
-    int b = (p.mask_mode == CR_MASK_TOKEN_CAUSAL) ? i + 1
-            : (p.mask_mode == CR_MASK_BIDIRECTIONAL) ? p.n
-                                                     : p.chunk_end[i];
-    b = min(max(b, 0), p.n);   // stay inside the row whatever the map holds
-    *lo = min(max(a, 0), b);
-    *hi = b;
-}
-
-__global__ void __launch_bounds__(256) softmax_rows_kernel(float* __restrict__ S, const __grid_constant__ SoftmaxParams p) {
-    pdl_launch_dependents();
-    pdl_wait();
-    const int lane = threadIdx.x & 31;
-    const int64_t w = blockIdx.x * static_cast<int64_t>(blockDim.x / 32) + (threadIdx.x >> 5);
-    if (w >= static_cast<int64_t>(p.heads) * p.n) return;
-    const int i = static_cast<int>(w % p.n);
-    float* row = S + w * p.n;
-    int lo, hi;
-    visible_keys(p, i, &lo, &hi);
-    float mx = -INFINITY;
-    for (int j = lo + lane; j < hi; j += 32) mx = fmaxf(mx, row[j]);
-    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    float sum = 0.0f;
-    for (int j = lo + lane; j < hi; j += 32) {
-        const float e = expf(row[j] - mx);
-        row[j] = e;
-        sum += e;
-    }
-    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-    const float inv = 1.0f / sum;
-    for (int j = lane; j < p.n; j += 32) row[j] = (j >= lo && j < hi) ? row[j] * inv : 0.0f;
-}
-
-// dS = P (dP - sum_j P dP) per row, in place on dP (masked entries have P = 0).
-__global__ void __launch_bounds__(256)
-    softmax_bwd_kernel(const float* __restrict__ P, float* __restrict__ dP, const __grid_constant__ SoftmaxParams p) {
-    pdl_launch_dependents();
-    pdl_wait();
-    const int lane = threadIdx.x & 31;
-    const int64_t w = blockIdx.x * static_cast<int64_t>(blockDim.x / 32) + (threadIdx.x >> 5);
-    if (w >= static_cast<int64_t>(p.heads) * p.n) return;
-    const float* pr = P + w * p.n;
-    float* dr = dP + w * p.n;
-    float s = 0.0f;
-    for (int j = lane; j < p.n; j += 32) s = fmaf(pr[j], dr[j], s);
-    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    for (int j = lane; j < p.n; j += 32) dr[j] = pr[j] * (dr[j] - s);
-}
-
 // out[i] = in[i] * scale[i % cols] (dW_seg: the cache's 1 / sigma_stale per column)
 __global__ void __launch_bounds__(256)
     scale_cols_kernel(float* __restrict__ a, int64_t n, const float* __restrict__ sigma, int64_t period,
@@ -333,15 +278,6 @@ __global__ void __launch_bounds__(256)
         (void)d_seg;
         a[i] /= __ldg(sigma + s * seg_cols + j);
     }
-}
-
-__global__ void __launch_bounds__(256)
-    f32_from_bf16_kernel(const uint16_t* __restrict__ a, int64_t n, float* __restrict__ out) {
-    pdl_launch_dependents();
-    pdl_wait();
-    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
-         i += static_cast<int64_t>(gridDim.x) * blockDim.x)
-        out[i] = bf16_to_f32(a[i]);
 }
 
 // Squared norm of the flat gradient: fp64 partial per CTA over a fixed range,
@@ -488,24 +424,10 @@ cr_status launch_rope_backward(float* dqkv, const float2* table, int64_t N, int 
     return launch_pdl(rope_backward_kernel, grid_for(N * db), dim3(256), 0, st, dqkv, table, N, db, hd);
 }
 
-cr_status launch_softmax_rows(float* S, const SoftmaxParams& p, cudaStream_t st) {
-    const int64_t warps = static_cast<int64_t>(p.heads) * p.n;
-    return launch_pdl(softmax_rows_kernel, dim3(static_cast<unsigned>((warps + 7) / 8)), dim3(256), 0, st, S, p);
-}
-
-cr_status launch_softmax_bwd(const float* P, float* dP, const SoftmaxParams& p, cudaStream_t st) {
-    const int64_t warps = static_cast<int64_t>(p.heads) * p.n;
-    return launch_pdl(softmax_bwd_kernel, dim3(static_cast<unsigned>((warps + 7) / 8)), dim3(256), 0, st, P, dP, p);
-}
-
 cr_status launch_scale_seg_grad(float* g, int64_t S, int64_t dseg, int64_t dh, const float* sigma,
                                 cudaStream_t st) {
     const int64_t n = S * dseg * dh;
     return launch_pdl(scale_cols_kernel, grid_for(n), dim3(256), 0, st, g, n, sigma, dseg * dh, dh, dseg);
-}
-
-cr_status launch_f32_from_bf16(const uint16_t* a, int64_t n, float* out, cudaStream_t st) {
-    return launch_pdl(f32_from_bf16_kernel, grid_for(n), dim3(256), 0, st, a, n, out);
 }
 
 size_t sqnorm_scratch_doubles() { return kNormCtas; }
