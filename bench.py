@@ -558,7 +558,8 @@ def run_train(args):
     lens = np.diff(a.cu_seqlens)
     ts = TrainSession(t, r, case.weights, N, int(lens.max()))
     del sess.h0, sess.rein, sess.yf, sess.workspace
-    step = lambda: ts.step(kv, joint, sess.emb[:N], sess.chunk_end[:N], sess.pos[:N], a.cu_seqlens, N, 3e-4)
+    step = lambda: ts.step(kv, joint, sess.emb[:N], sess.chunk_end[:N], sess.pos[:N], a.cu_seqlens, N, 3e-4,
+                           mask_mode=args.mask)
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
@@ -580,11 +581,19 @@ def run_train(args):
     if st != cr.CR_OK:
         raise RuntimeError(f"device status {word}")
     cend = sess.chunk_end[:N].to(torch.int64).cpu().numpy()
-    flops = train_flops(case, float(cend.sum()))
+    cid = sess.chunk_id[:N].to(torch.int64).cpu().numpy()
+    local = np.arange(N) - np.repeat(a.cu_seqlens[:-1], lens)
+    starts = np.array([np.searchsorted(cid[a.cu_seqlens[q]:a.cu_seqlens[q + 1]], cid[t], "left")
+                       for q in range(len(lens)) for t in range(a.cu_seqlens[q], a.cu_seqlens[q + 1])])
+    visible = {"block_causal": cend, "token_causal": local + 1, "bidirectional": np.repeat(lens, lens),
+               "block_diagonal": cend - starts}[args.mask]
+    flops = train_flops(case, float(visible.sum()))
     hbm, tf_burst, tf_sus, src = load_peaks()
     achieved = flops / (total_ms / args.steps * 1e-3) / 1e12
     B = case.repairer.n_blocks
-    launches = 35 + B * (36 + 2 * (len(a.cu_seqlens) - 1)) if B > 0 else 0
+    # this library's launches per update: forward 9 + 7 B, objective 6, head backward 7,
+    # 33 per block backward, encoder backward 12, clipping and AdamW 3
+    launches = 37 + 40 * B if B > 0 else 0
     print(json.dumps({
         "metric": "trained doc tokens/s (one AdamW update of the repair network per step, 1 GB300)",
         "value": N * args.steps / (total_ms / 1e3), "unit": "tokens/s", "n_gpus": 1,
@@ -592,7 +601,7 @@ def run_train(args):
         "p50_ms": statistics.median(per), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16 GEMM operands, fp32 accumulation and master weights",
         "data": "synthetic (seeded caches, embeddings, joint = stale + sigma_Delta noise; random-init repairer)",
-        "config": {"workload": workload_desc(case), "n_tokens": N, "variant": {"train": True},
+        "config": {"workload": workload_desc(case), "n_tokens": N, "variant": {"train": True, **args.variant},
                    "l2": "no flush: the cache, joint cache and residual buffers exceed L2",
                    "optimizer": "AdamW (0.9, 0.95), wd 0.01, clip 1.0, lr 3e-4"},
         "roofline": {"kernel": "whole update (forward, objective, backward, AdamW)", "bound": "tensor",

@@ -387,7 +387,9 @@ size_t cr_train_workspace_bytes(const cr_target_dims* target, const cr_repairer_
 
 /*
  * cr_train_step - forward, objective, backward, clipping and AdamW for one
- * batch of requests (the method's block-causal mask, bf16 caches only):
+ * batch of requests (bf16 caches only) under mask_mode, the method's
+ * block-causal mask or an attention ablation of App. F (each trained with its
+ * own mask there):
  *   L = mean over requests of 1/(N_r D_KV) sum_t || z_t - (KV_joint,t - KV_stale,t) / sigma_Delta ||^2,
  *   g = dL/dtheta over every trained tensor; g <- g min(1, max_norm / (||g|| + 1e-6));
  *   theta <- theta (1 - lr wd) - lr (m / (1 - b1^t)) / (sqrt(v / (1 - b2^t)) + eps)
@@ -410,8 +412,8 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
                         const float* sigma_stale, const float* sigma_delta, const void* kv_stale,
                         const void* kv_joint, const void* emb, const int32_t* chunk_end,
                         const int32_t* pos, const int32_t* cu_seqlens_host, int32_t n_req,
-                        int64_t n_tokens, const cr_adamw* hp, float* stats_out, void* workspace,
-                        size_t workspace_bytes, void* stream);
+                        int64_t n_tokens, int32_t mask_mode, const cr_adamw* hp, float* stats_out,
+                        void* workspace, size_t workspace_bytes, void* stream);
 
 /* Device status word: out[0] = first error (0 none, 1 wait timeout, 2 device
  * index out of range), out[1] = site, out[2] = block.  Synchronises the

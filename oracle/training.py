@@ -330,7 +330,7 @@ def lr_schedule(step: int, *, peak: float = 3e-4, final: float = 3e-5, warmup: i
 
 def train_step(params, m, v, step: int, lr: float, batch: Dict[str, np.ndarray], *, sigma_stale,
                sigma_delta, cache_dtype: str, head_dim: int, n_heads: int, hp: AdamWHyper = AdamWHyper(),
-               eps: float = 1e-5, rope_theta: float = 1e4):
+               eps: float = 1e-5, rope_theta: float = 1e4, mask_mode: str = "block_causal"):
     """Forward, loss, backward, clipping and AdamW: one update.  batch holds the
     assembled stale cache, the joint cache, embeddings, chunk_id, pos and cu_seqlens.
     Returns (loss, grad norm, raw grads, new params, new m, new v)."""
@@ -338,7 +338,7 @@ def train_step(params, m, v, step: int, lr: float, batch: Dict[str, np.ndarray],
     wf["sigma_stale"], wf["sigma_delta"] = sigma_stale, sigma_delta
     c = train_forward(batch["kv"], batch["emb"], batch["chunk_id"], batch["pos"], batch["cu_seqlens"],
                       wf, cache_dtype=cache_dtype, head_dim=head_dim, n_heads=n_heads, eps=eps,
-                      rope_theta=rope_theta)
+                      rope_theta=rope_theta, mask_mode=mask_mode)
     loss, dz = train_loss(c.z, batch["kv"], batch["kv_joint"], sigma_delta, batch["cu_seqlens"],
                           cache_dtype)
     grads = train_backward(c, dz, wf, batch["pos"], batch["cu_seqlens"],

@@ -120,7 +120,7 @@ def lib(build_if_missing: bool = False) -> ctypes.CDLL:
         "cr_param_layout": (i32, [P(cr_target_dims), P(cr_repairer_dims), vp, i32]),
         "cr_train_workspace_bytes": (c_size_t, [P(cr_target_dims), P(cr_repairer_dims), i64, i64]),
         "cr_train_step": (i32, [P(cr_target_dims), P(cr_repairer_dims), vp, vp, vp, vp, vp, vp, vp, vp, vp,
-                                vp, vp, vp, vp, i32, i64, P(cr_adamw), vp, vp, c_size_t, vp]),
+                                vp, vp, vp, vp, i32, i64, i32, P(cr_adamw), vp, vp, c_size_t, vp]),
         "cr_masked_attention": (i32, [vp, i32, i32, i32, vp, vp, vp, i32, i64, vp, vp]),
         "cr_chunk_starts": (i32, [vp, vp, i32, i64, vp, vp]),
         "cr_qkv_rope": (i32, [vp, vp, vp, vp, i64, i32, i32, c_float, vp, vp]),
@@ -378,12 +378,13 @@ def cr_train_workspace_bytes(target, rep, max_tokens, max_request_tokens) -> int
 
 def cr_train_step(target, rep, params, params_bf16, adam_m, adam_v, grads, sigma_stale, sigma_delta,
                   kv_stale, kv_joint, emb, chunk_end, pos, cu_seqlens_host, n_tokens, hp: "cr_adamw",
-                  stats_out, workspace, stream=None):
+                  stats_out, workspace, stream=None, mask_mode="block_causal"):
     cu = _host_arr(cu_seqlens_host, np.int32)
     _check("cr_train_step", lib().cr_train_step(
         ctypes.byref(target), ctypes.byref(rep), _p(params), _p(params_bf16), _p(adam_m), _p(adam_v),
         _p(grads), _p(sigma_stale), _p(sigma_delta), _p(kv_stale), _p(kv_joint), _p(emb), _p(chunk_end),
-        _p(pos), cu.ctypes.data, len(cu) - 1, n_tokens, ctypes.byref(hp), _p(stats_out), _p(workspace),
+        _p(pos), cu.ctypes.data, len(cu) - 1, n_tokens, _mask_mode(mask_mode), ctypes.byref(hp),
+        _p(stats_out), _p(workspace),
         workspace.numel() * workspace.element_size(), _stream(stream)))
 
 

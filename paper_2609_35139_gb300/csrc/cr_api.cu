@@ -1009,15 +1009,15 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
                         const float* sigma_stale, const float* sigma_delta, const void* kv_stale,
                         const void* kv_joint, const void* emb, const int32_t* chunk_end,
                         const int32_t* pos, const int32_t* cu_seqlens_host, int32_t n_req,
-                        int64_t n_tokens, const cr_adamw* hp, float* stats_out, void* workspace,
-                        size_t workspace_bytes, void* stream) {
+                        int64_t n_tokens, int32_t mask_mode, const cr_adamw* hp, float* stats_out,
+                        void* workspace, size_t workspace_bytes, void* stream) {
     cr_status s = check_target(target);
     if (s == CR_OK) s = check_repairer(rep);
     if (s != CR_OK) return s;
     const Dims d = dims_of(target, rep);
     if (d.f32) return CR_ERR_UNSUPPORTED;
     if (!hp || !cu_seqlens_host || n_req < 1 || n_req > kMaxReq || n_tokens < 1 ||
-        n_tokens > INT32_MAX / 2)
+        n_tokens > INT32_MAX / 2 || !valid_mask_mode(mask_mode))
         return CR_ERR_INVALID_ARG;
     if (!(hp->lr >= 0.0f) || !(hp->beta1 >= 0.0f && hp->beta1 < 1.0f) ||
         !(hp->beta2 >= 0.0f && hp->beta2 < 1.0f) || !(hp->eps > 0.0f) || !(hp->weight_decay >= 0.0f) ||
@@ -1129,8 +1129,7 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
     s = cr_compress_features(target, rep, &w, kv_stale, emb, N, h0, rein, inf, IL.total, stream);
     if (s != CR_OK) return s;
     AttnParams* ap = new AttnParams();
-    s = attn_params(d, CR_MASK_BLOCK_CAUSAL, chunk_end, nullptr, cu_seqlens_host, n_req, N, nullptr,
-                    status, ap);
+    s = attn_params(d, mask_mode, chunk_end, CSTART, cu_seqlens_host, n_req, N, nullptr, status, ap);
     GemmParams gq{};
     gq.status = status;
     gq.pos = pos;
@@ -1147,7 +1146,7 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
     bp->d_b = static_cast<int32_t>(db);
     bp->n_heads = static_cast<int32_t>(d.nh);
     bp->n_req = n_req;
-    bp->mask_mode = CR_MASK_BLOCK_CAUSAL;
+    bp->mask_mode = mask_mode;
     bp->scale_log2 = ap->scale_log2;
     bp->scale = static_cast<float>(1.0 / sqrt(static_cast<double>(hd)));
     bp->status = status;

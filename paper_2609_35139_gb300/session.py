@@ -274,11 +274,14 @@ class TrainSession:
         return t[a:b]
 
     def step(self, kv_stale, kv_joint, emb, chunk_end, pos, cu_seqlens_host, n_tokens, lr, *,
-             beta1=0.9, beta2=0.95, eps=1e-8, weight_decay=0.01, max_grad_norm=1.0, stream=None):
-        """One AdamW update; returns the device stats tensor (loss, grad norm, clip coef, 0)."""
+             beta1=0.9, beta2=0.95, eps=1e-8, weight_decay=0.01, max_grad_norm=1.0, stream=None,
+             mask_mode="block_causal"):
+        """One AdamW update under mask_mode (the method's mask or an App. F ablation);
+        returns the device stats tensor (loss, grad norm, clip coef, 0)."""
         self.n_steps += 1
         hp = cr.cr_adamw(lr, beta1, beta2, eps, weight_decay, max_grad_norm, self.n_steps)
         cr.cr_train_step(self.target, self.rep, self.params, self.params_bf16, self.adam_m, self.adam_v,
                          self.grads, self.sigma_stale, self.sigma_delta, kv_stale, kv_joint, emb, chunk_end,
-                         pos, cu_seqlens_host, n_tokens, hp, self.stats, self.workspace, stream)
+                         pos, cu_seqlens_host, n_tokens, hp, self.stats, self.workspace, stream,
+                         mask_mode)
         return self.stats

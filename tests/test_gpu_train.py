@@ -39,8 +39,9 @@ def _session(case, a):
     return ts, dev, n
 
 
-def _step(ts, dev, a, n, lr):
-    st = ts.step(dev["kv"], dev["kj"], dev["emb"], dev["ce"], dev["pos"], a["cu_seqlens"], n, lr)
+def _step(ts, dev, a, n, lr, mask="block_causal"):
+    st = ts.step(dev["kv"], dev["kj"], dev["emb"], dev["ce"], dev["pos"], a["cu_seqlens"], n, lr,
+                 mask_mode=mask)
     torch.cuda.synchronize()
     return st.cpu().numpy().copy()
 
@@ -49,8 +50,10 @@ def _tensor(ts, flat, name, shape):
     return ts.view(flat, name)[:int(np.prod(shape))].cpu().numpy().astype(np.float64).reshape(shape)
 
 
-@pytest.mark.parametrize("name", ["small", "small_multi"])
-def test_train_step_matches_oracle(name):
+@pytest.mark.parametrize("name,mask", [("small", "block_causal"), ("small_multi", "block_causal"),
+                                       ("small_multi", "token_causal"), ("small_multi", "bidirectional"),
+                                       ("small_multi", "block_diagonal")])
+def test_train_step_matches_oracle(name, mask):
     case = F.make_case(name)
     a = _batch(case)
     t, r = case.target, case.repairer
@@ -62,11 +65,11 @@ def test_train_step_matches_oracle(name):
     loss, norm, grads, _, _, _ = T.train_step(params, zeros, zeros, 1, lr, a,
                                               sigma_stale=case.weights["sigma_stale"],
                                               sigma_delta=case.weights["sigma_delta"], cache_dtype="bf16",
-                                              head_dim=t.head_dim, n_heads=r.n_heads, hp=hp)
+                                              head_dim=t.head_dim, n_heads=r.n_heads, hp=hp, mask_mode=mask)
     ts, dev, n = _session(case, a)
-    stats = _step(ts, dev, a, n, lr)
+    stats = _step(ts, dev, a, n, lr, mask)
     g_loss, g_norm, g_coef = float(stats[0]), float(stats[1]), float(stats[2])
-    print(name, "loss", g_loss, loss, "norm", g_norm, norm)
+    print(name, mask, "loss", g_loss, loss, "norm", g_norm, norm)
     assert abs(g_loss - loss) <= 1e-3 * loss
     assert abs(g_norm - norm) <= 5e-3 * norm
     # The gradient, tensor by tensor.  The GPU rounds every GEMM operand (stored

@@ -42,18 +42,18 @@ def setup():
     return case, a, names, params, wf
 
 
-def _loss(case, a, wf):
+def _loss(case, a, wf, mask="block_causal"):
     t, r = case.target, case.repairer
     c = T.train_forward(a["kv"], a["emb"], a["chunk_id"], a["pos"], a["cu_seqlens"], wf,
-                        cache_dtype=t.cache_dtype, head_dim=t.head_dim, n_heads=r.n_heads)
+                        cache_dtype=t.cache_dtype, head_dim=t.head_dim, n_heads=r.n_heads, mask_mode=mask)
     loss, dz = T.train_loss(c.z, a["kv"], a["kv_joint"], wf["sigma_delta"], a["cu_seqlens"],
                             t.cache_dtype)
     return loss, dz, c
 
 
-def _grads(case, a, wf):
+def _grads(case, a, wf, mask="block_causal"):
     t, r = case.target, case.repairer
-    loss, dz, c = _loss(case, a, wf)
+    loss, dz, c = _loss(case, a, wf, mask)
     g = T.train_backward(c, dz, wf, a["pos"], a["cu_seqlens"], O.dtype_to_f64(a["emb"], t.cache_dtype),
                          head_dim=t.head_dim, n_heads=r.n_heads)
     return loss, g
@@ -96,7 +96,7 @@ def test_backward_matches_finite_differences(setup):
             assert abs(fd - an) <= 1e-6 * max(1e-3, abs(fd)) + 1e-9, (k, idx, fd, an)
 
 
-def _torch_loss(case, a, wt):
+def _torch_loss(case, a, wt, mask="block_causal"):
     """The same objective stated with torch ops (float64), for autograd."""
     t, r = case.target, case.repairer
     n = a["kv"].shape[0]
@@ -130,7 +130,7 @@ def _torch_loss(case, a, wt):
         outs = []
         for rq in range(len(a["cu_seqlens"]) - 1):
             lo, hi = a["cu_seqlens"][rq], a["cu_seqlens"][rq + 1]
-            m = torch.from_numpy(O.attention_mask(a["chunk_id"][lo:hi], "block_causal"))
+            m = torch.from_numpy(O.attention_mask(a["chunk_id"][lo:hi], mask))
             o = torch.nn.functional.scaled_dot_product_attention(
                 q[lo:hi].transpose(0, 1), k[lo:hi].transpose(0, 1), v[lo:hi].transpose(0, 1), attn_mask=m)
             outs.append(o.transpose(0, 1))
@@ -150,11 +150,13 @@ def _torch_loss(case, a, wt):
     return total
 
 
-def test_backward_matches_torch_autograd(setup):
+@pytest.mark.parametrize("mask", O.MASK_MODES)
+def test_backward_matches_torch_autograd(setup, mask):
+    """Every attention mask (the method's and the App. F ablations) through the same backward."""
     case, a, names, params, wf = setup
-    loss, g = _grads(case, a, wf)
+    loss, g = _grads(case, a, wf, mask)
     wt = {k: torch.tensor(wf[k], dtype=torch.float64, requires_grad=True) for k in names}
-    tl = _torch_loss(case, a, wt)
+    tl = _torch_loss(case, a, wt, mask)
     tl.backward()
     assert abs(float(tl.detach()) - loss) <= 1e-12 * abs(loss)
     for k in names:
