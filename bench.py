@@ -378,7 +378,8 @@ def run_ours(args):
     launches_per_step += 1 if (args.rope and args.component == "v") else 0
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        n_chunks = 2
+        # the whole first request: about 10-30 s of oracle work on the host cores
+        n_chunks = int(case.plan.cu_chunks[1] - case.plan.cu_chunks[0])
         ntok, secs = oracle_sample(case, n_chunks, mask=args.mask)
         cpu = {"value": ntok / secs, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
                "sample": f"first {n_chunks} chunks ({ntok} tokens) of the request, full repair "
