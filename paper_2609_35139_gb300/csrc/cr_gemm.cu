@@ -65,9 +65,12 @@ struct GemmCfg {
     static constexpr int kGroupBufs = (EPI == EPI_GELU_BF16 || EPI == EPI_QKV_ROPE) ? 2 : 1;
     static constexpr uint32_t kTileBytes = kInPlace ? BM * BN * kTileEsize : 2 * kGroupBufs * 16384;
     static constexpr uint32_t kVecBytes = BN * 4 * (kKV ? 2 : 1);   // bias (+ sigma)
+    // in-place epilogues recycle the staged tile box by box, so the next tile's
+    // vectors may land while this tile is still being finished: two buffers
+    static constexpr int kVecBufs = kInPlace ? 2 : 1;
     static constexpr uint32_t kBBytes = (BN / CG) * BK * 2;      // this CTA's share of W
     static constexpr uint32_t kStageBytes = A_BYTES + kBBytes;
-    static constexpr uint32_t kFixed = 1024 + kTileBytes + kVecBytes + 320;
+    static constexpr uint32_t kFixed = 1024 + kTileBytes + kVecBufs * kVecBytes + 512;
     static constexpr int kStagesFit = static_cast<int>((kSmemLimit - kFixed) / kStageBytes);
     static constexpr int kStages = kStagesFit > 6 ? 6 : kStagesFit;
     static_assert(kStages >= 3, "GEMM tile does not fit in shared memory");
@@ -235,17 +238,20 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     uint8_t* tile = smem + STAGES * Cfg::kStageBytes;              // staged output (part)
-    float* vec = reinterpret_cast<float*>(tile + Cfg::kTileBytes);  // bias [BN] (+ sigma [BN])
-    uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(vec) + Cfg::kVecBytes);
+    float* vec = reinterpret_cast<float*>(tile + Cfg::kTileBytes);  // [buffer] bias [BN] (+ sigma [BN])
+    uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(vec) +
+                                                 Cfg::kVecBufs * Cfg::kVecBytes);
     uint64_t* full = bars;
     uint64_t* empty = bars + STAGES;
     uint64_t* tfull = bars + 2 * STAGES;
     uint64_t* tempty = tfull + 2;
-    uint64_t* epi_full = tempty + 2;     // loader -> epilogue: vectors (+ in-place tile) landed
-    uint64_t* epi_empty = epi_full + 1;  // epilogue -> loader: vectors / tile free again
-    uint64_t* drain = epi_empty + 1;
-    uint64_t* epi_done = drain + 1;      // [group][buffer]: a staged buffer is written
-    uint64_t* st_free = epi_done + 4;    // [group][buffer]: the TMA store has read that buffer
+    // loader -> epilogue: the vectors (+ box b of the in-place tile) landed; in-place
+    // epilogues use one per box (box 0 also carries the vectors), the others only [0]
+    uint64_t* epi_full = tempty + 2;     // [8]
+    uint64_t* epi_empty = epi_full + 8;  // [8] back to the loader: box b (and the vectors) free
+    uint64_t* drain = epi_empty + 8;
+    uint64_t* epi_done = drain + 1;      // [8] in-place: box b written; else [group][buffer]
+    uint64_t* st_free = epi_done + 8;    // [group][buffer]: the TMA store has read that buffer
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(st_free + 4);
     int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
@@ -265,14 +271,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             mbar_init(&tfull[s], 1);
             mbar_init(&tempty[s], 8 * CG);   // the epilogue warps of every CTA of the tile
         }
-        mbar_init(epi_full, 1);
-        mbar_init(epi_empty, 1);
-        for (int b = 0; b < 4; ++b) {
-            // in-place: one barrier for all 256 epilogue threads; store-only:
-            // one per group and buffer for that group's 128 threads
+        for (int b = 0; b < 8; ++b) {
+            mbar_init(&epi_full[b], 1);
+            mbar_init(&epi_empty[b], 1);
+            // in-place: one barrier per box for all 256 epilogue threads;
+            // store-only: one per group and buffer for that group's 128 threads
             mbar_init(&epi_done[b], Cfg::kInPlace ? 256 : 128);
-            mbar_init(&st_free[b], 1);
         }
+        for (int b = 0; b < 4; ++b) mbar_init(&st_free[b], 1);
         mbar_init(drain, 1);
         *abort_flag = 0;
         fence_barrier_init();
@@ -359,25 +365,41 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             // released the slot (independent of the A/B stream of warp 0)
             bool ok = true;
             int i = 0;
-            for (int t = cta0; t < total; t += ncta, ++i) {
+            for (int t = cta0; t < total && ok; t += ncta, ++i) {
                 const int m0 = (t % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
                 const int n0 = tile_n0<BN, Cfg::kKV>(p, t);
-                if (!(ok = mbar_wait_warp(epi_empty, (static_cast<uint32_t>(i) & 1u) ^ 1u, wc, 101)))
-                    break;
                 const int nb = min(BN, p.N - n0);
                 const uint32_t vbytes = static_cast<uint32_t>(nb) * 4u;
-                uint32_t bytes = (load_tile ? Cfg::kTileBytes : 0u) + (has_bias ? vbytes : 0u);
-                if constexpr (Cfg::kKV) bytes += vbytes;
-                if (elect_one()) {
-                    mbar_expect_tx(epi_full, bytes);
-                    if (load_tile) {
-                        for (int b = 0; b < Cfg::kBoxes; ++b)
-                            tma_load_2d(tile + b * 16384, &tmC, epi_full, n0 + b * Cfg::kBoxCols, m0);
+                if constexpr (Cfg::kInPlace) {
+                    // box by box, each as soon as the previous tile's copy of it has
+                    // been stored; box 0 also brings this tile's vectors (buffer i & 1)
+                    float* vdst = vec + (i & 1) * (Cfg::kVecBytes / 4);
+                    for (int b = 0; b < Cfg::kBoxes; ++b) {
+                        if (!(ok = mbar_wait_warp(&epi_empty[b], (static_cast<uint32_t>(i) & 1u) ^ 1u, wc, 101)))
+                            break;
+                        uint32_t bytes = load_tile ? 16384u : 0u;
+                        if (b == 0) bytes += (has_bias ? vbytes : 0u) + (Cfg::kKV ? vbytes : 0u);
+                        if (elect_one()) {
+                            if (bytes) mbar_expect_tx(&epi_full[b], bytes);
+                            else mbar_arrive(&epi_full[b]);
+                            if (load_tile)
+                                tma_load_2d(tile + b * 16384, &tmC, &epi_full[b], n0 + b * Cfg::kBoxCols, m0);
+                            if (b == 0) {
+                                if (has_bias) bulk_load(vdst, p.bias + n0, vbytes, &epi_full[0]);
+                                if constexpr (Cfg::kKV) bulk_load(vdst + BN, p.sigma + n0, vbytes, &epi_full[0]);
+                            }
+                        }
+                        __syncwarp();
                     }
-                    if (has_bias) bulk_load(vec, p.bias + n0, vbytes, epi_full);
-                    if constexpr (Cfg::kKV) bulk_load(vec + BN, p.sigma + n0, vbytes, epi_full);
+                } else {
+                    if (!(ok = mbar_wait_warp(epi_empty, (static_cast<uint32_t>(i) & 1u) ^ 1u, wc, 101)))
+                        break;
+                    if (elect_one()) {
+                        mbar_expect_tx(epi_full, vbytes);
+                        bulk_load(vec, p.bias + n0, vbytes, epi_full);
+                    }
+                    __syncwarp();
                 }
-                __syncwarp();
             }
             if (!ok) {
                 const uint64_t t0 = globaltimer();
@@ -400,15 +422,20 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             const int n0 = tile_n0<BN, Cfg::kKV>(p, t);
             const bool rows_in = m0 < p.M;   // a pair tile's second half may lie below M
             if constexpr (Cfg::kInPlace) {
-                if (!(ok = mbar_wait_warp(&epi_done[0], pk & 1u, wc, 401))) break;
-                if (leader) {
-                    for (int b = 0; b < Cfg::kBoxes && rows_in && !Cfg::kPaged; ++b)
-                        tma_store_2d(&tmC, tile + b * 16384, n0 + b * Cfg::kBoxCols, m0);
-                    tma_store_commit();
-                    tma_store_wait_read0();
-                    mbar_arrive(epi_empty);
+                // each box as soon as the epilogue has written it; once TMA has read
+                // it, the loader may bring the next tile's copy of that box
+                for (int b = 0; b < Cfg::kBoxes && ok; ++b) {
+                    if (!(ok = mbar_wait_warp(&epi_done[b], pk & 1u, wc, 401))) break;
+                    if (leader) {
+                        if (rows_in && !Cfg::kPaged) {
+                            tma_store_2d(&tmC, tile + b * 16384, n0 + b * Cfg::kBoxCols, m0);
+                            tma_store_commit();
+                            tma_store_wait_read0();
+                        }
+                        mbar_arrive(&epi_empty[b]);
+                    }
+                    __syncwarp();
                 }
-                __syncwarp();
                 ++pk;
             } else {
                 for (int k = 0; k < Cfg::kBoxes; ++k) {
@@ -516,7 +543,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             const int m0 = (t % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
             const int n0 = tile_n0<BN, Cfg::kKV>(p, t);
             ok = mbar_wait(&tfull[acc], acc_phase, wc, 301);
-            if (epi_load) ok = ok && mbar_wait(epi_full, static_cast<uint32_t>(i) & 1u, wc, 302);
+            // in-place epilogues wait box by box below
+            if (epi_load && !Cfg::kInPlace) ok = ok && mbar_wait(epi_full, static_cast<uint32_t>(i) & 1u, wc, 302);
             if (!__all_sync(0xffffffffu, ok)) {
                 ok = false;
                 break;
@@ -555,15 +583,32 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                         store16_tile<ES>(tile, r, col, v);
                     }
                 };
+                // this tile's vectors, and the per-box hand-over: box b of the
+                // staged tile is waited for before it is read and released to the
+                // store as soon as both groups have written their part of it
+                const float* vbt = vb + (i & 1) * (Cfg::kVecBytes / 4);
+                const float* vst = vbt + BN;
+                auto wait_box = [&](int b) -> bool {
+                    const bool w = mbar_wait(&epi_full[b], static_cast<uint32_t>(i) & 1u, wc, 302);
+                    return __all_sync(0xffffffffu, w);
+                };
+                auto done_box = [&](int b) {
+                    fence_async_smem();
+                    mbar_arrive(&epi_done[b]);
+                };
                 if (Cfg::kKV && p.rope_on) {
-                    // R_M pairs (d, d + d_h/2) live inside one d_h-wide segment
+                    // R_M pairs (d, d + d_h/2) live inside one d_h-wide segment, which
+                    // spans d_h / kBoxCols boxes; each group takes half of its pairs
                     const int dh = p.rope_dim;
+                    const int nbx = dh / Cfg::kBoxCols;
                     const float pr = row_ok ? static_cast<float>(__ldg(p.pos + row)) : 0.0f;
-                    // d_h-wide segments alternate between the two groups
-                    for (int s0 = eg * dh; s0 < BN; s0 += 2 * dh) {
+                    for (int s0 = 0; s0 < BN && ok; s0 += dh) {
+                        const int bx0 = s0 / Cfg::kBoxCols;
+                        for (int b = bx0; b < bx0 + nbx && ok; ++b) ok = wait_box(b);
+                        if (!ok) break;
                         const int gseg = (n0 + s0) / dh;
                         const bool rot = ((gseg / p.n_kv_heads) & 1) == 0;
-                        for (int j = 0; j < dh / 2; j += 16) {
+                        for (int j = eg * (dh / 4); j < (eg + 1) * (dh / 4); j += 16) {
                             float a[16], b[16], ka[16], kb[16], sa_[16], sb_[16], ba[16], bb[16];
                             const int ta = s0 + j, tb = s0 + dh / 2 + j;
                             __syncwarp();
@@ -576,11 +621,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                                 load16_tile<ES>(tile, r, ta, ka);
                                 load16_tile<ES>(tile, r, tb, kb);
                             }
-                            vec16(vs, ta, sa_);
-                            vec16(vs, tb, sb_);
+                            vec16(vst, ta, sa_);
+                            vec16(vst, tb, sb_);
                             if (has_bias) {
-                                vec16(vb, ta, ba);
-                                vec16(vb, tb, bb);
+                                vec16(vbt, ta, ba);
+                                vec16(vbt, tb, bb);
                             } else {
 #pragma unroll
                                 for (int q = 0; q < 16; ++q) ba[q] = bb[q] = 0.0f;
@@ -597,10 +642,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                             put16(ta, ka);
                             put16(tb, kb);
                         }
+                        for (int b = bx0; b < bx0 + nbx; ++b) done_box(b);
                     }
                 } else {
-                    // 16-column chunks alternate between the two groups
-                    for (int c = eg * 16; c < BN; c += 32) {
+                    // box by box; each group takes one half of the box's columns
+                    constexpr int HALF = Cfg::kBoxCols / 2;
+                    for (int bx = 0; bx < Cfg::kBoxes && ok; ++bx) {
+                      if (!(ok = wait_box(bx))) break;
+                      for (int c = bx * Cfg::kBoxCols + eg * HALF; c < bx * Cfg::kBoxCols + (eg + 1) * HALF;
+                           c += 16) {
                         float a[16], k[16], bv[16];
                         __syncwarp();
                         tmem_ld16(taddr + c, a);
@@ -611,7 +661,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                             load16_tile<ES>(tile, r, c, k);
                         }
                         if (has_bias) {
-                            vec16(vb, c, bv);
+                            vec16(vbt, c, bv);
                         } else {
 #pragma unroll
                             for (int q = 0; q < 16; ++q) bv[q] = 0.0f;
@@ -620,7 +670,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                         if constexpr (Cfg::kKV) {
                             if (!keep) {
                                 float sv[16];
-                                vec16(vs, c, sv);
+                                vec16(vst, c, sv);
 #pragma unroll
                                 for (int q = 0; q < 16; ++q) k[q] = fmaf(sv[q], a[q] + bv[q], k[q]);
                             }
@@ -629,13 +679,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                             for (int q = 0; q < 16; ++q) k[q] += a[q] + bv[q];
                         }
                         put16(c, k);
+                      }
+                      done_box(bx);
                     }
                 }
+                if (!ok) break;
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) release_acc(&tempty[acc]);
-                fence_async_smem();
-                mbar_arrive(&epi_done[0]);
                 ++pk;
             } else {
                 // store-only epilogues: one 128 B-wide box of columns at a time,
