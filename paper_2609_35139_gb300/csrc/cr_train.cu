@@ -301,14 +301,23 @@ __global__ void __launch_bounds__(256)
     if (threadIdx.x == 0) part[blockIdx.x] = red[0];
 }
 
-__global__ void sqnorm_reduce_kernel(const double* __restrict__ part, int n_part, float max_norm,
-                                     float* __restrict__ stats) {
+__global__ void __launch_bounds__(256)
+    sqnorm_reduce_kernel(const double* __restrict__ part, int n_part, float max_norm,
+                         float* __restrict__ stats) {
     pdl_launch_dependents();
     pdl_wait();
-    if (threadIdx.x != 0 || blockIdx.x != 0) return;
-    double s = 0.0;
-    for (int i = 0; i < n_part; ++i) s += part[i];
-    const double norm = sqrt(s);
+    // a fixed-order tree over the partials (each thread a fixed stride of them)
+    __shared__ double red[256];
+    double t = 0.0;
+    for (int i = threadIdx.x; i < n_part; i += blockDim.x) t += part[i];
+    red[threadIdx.x] = t;
+    __syncthreads();
+    for (int k = 128; k > 0; k >>= 1) {
+        if (static_cast<int>(threadIdx.x) < k) red[threadIdx.x] += red[threadIdx.x + k];
+        __syncthreads();
+    }
+    if (threadIdx.x != 0) return;
+    const double norm = sqrt(red[0]);
     stats[1] = static_cast<float>(norm);
     stats[2] = static_cast<float>(fmin(1.0, static_cast<double>(max_norm) / (norm + 1e-6)));
     stats[3] = 0.0f;
@@ -437,7 +446,7 @@ cr_status launch_clip_adamw(float* p, float* m, float* v, const float* g, uint16
                             cudaStream_t st) {
     cr_status s = launch_pdl(sqnorm_partial_kernel, dim3(kNormCtas), dim3(256), 0, st, g, n, scratch);
     if (s != CR_OK) return s;
-    s = launch_pdl(sqnorm_reduce_kernel, dim3(1), dim3(32), 0, st, static_cast<const double*>(scratch),
+    s = launch_pdl(sqnorm_reduce_kernel, dim3(1), dim3(256), 0, st, static_cast<const double*>(scratch),
                    kNormCtas, max_norm, stats);
     if (s != CR_OK) return s;
     if (n % 4 != 0) return CR_ERR_UNSUPPORTED;

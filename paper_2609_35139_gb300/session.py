@@ -164,20 +164,21 @@ class RepairPipeline:
     """
 
     def __init__(self, target: cr.cr_target_dims, rep: cr.cr_repairer_dims,
-                 weights: cr.PackedWeights, max_tokens: int, device="cuda"):
+                 weights: cr.PackedWeights, max_tokens: int, device="cuda", n_slots: int = 2):
         self.device = torch.device(device)
-        self.slots = [RepairSession(target, rep, weights, max_tokens, device) for _ in range(2)]
+        self.n_slots = n_slots
+        self.slots = [RepairSession(target, rep, weights, max_tokens, device) for _ in range(n_slots)]
         dt = _dtype(target.cache_dtype)
         d_kv = self.slots[0].d_kv
-        self.stage_kv = [torch.empty(max_tokens, d_kv, dtype=dt, device=self.device) for _ in range(2)]
+        self.stage_kv = [torch.empty(max_tokens, d_kv, dtype=dt, device=self.device) for _ in range(n_slots)]
         self.stage_emb = [torch.empty(max_tokens, target.d_model, dtype=dt, device=self.device)
-                          for _ in range(2)]
+                          for _ in range(n_slots)]
         self.compute = torch.cuda.Stream(self.device)
         self.h2d = torch.cuda.Stream(self.device)
         self.d2h = torch.cuda.Stream(self.device)
-        self.ev_h2d = [torch.cuda.Event() for _ in range(2)]
-        self.ev_comp = [torch.cuda.Event() for _ in range(2)]
-        self.ev_d2h = [torch.cuda.Event() for _ in range(2)]
+        self.ev_h2d = [torch.cuda.Event() for _ in range(n_slots)]
+        self.ev_comp = [torch.cuda.Event() for _ in range(n_slots)]
+        self.ev_d2h = [torch.cuda.Event() for _ in range(n_slots)]
         self.max_tokens = max_tokens
         self.n_submitted = 0
 
@@ -192,7 +193,7 @@ class RepairPipeline:
         n = int(lens.sum())
         if n < 1 or n > self.max_tokens:
             raise ValueError(f"request of {n} tokens: the pipeline holds 1..{self.max_tokens}")
-        s = self.n_submitted % 2
+        s = self.n_submitted % self.n_slots
         sess, skv, semb = self.slots[s], self.stage_kv[s], self.stage_emb[s]
         dst = np.concatenate([[0], np.cumsum(lens)[:-1]]).astype(np.int64)
         # this slot's staging pool is free once its previous repair has run
@@ -221,7 +222,7 @@ class RepairPipeline:
     def drain(self):
         """Make the current stream wait for everything submitted so far."""
         cur = torch.cuda.current_stream(self.device)
-        for s in range(2):
+        for s in range(self.n_slots):
             cur.wait_event(self.ev_d2h[s])
 
 

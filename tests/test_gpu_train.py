@@ -52,9 +52,12 @@ def _tensor(ts, flat, name, shape):
 
 @pytest.mark.parametrize("name,mask", [("small", "block_causal"), ("small_multi", "block_causal"),
                                        ("small_multi", "token_causal"), ("small_multi", "bidirectional"),
-                                       ("small_multi", "block_diagonal")])
+                                       ("small_multi", "block_diagonal"), ("small_heads32", "block_causal")])
 def test_train_step_matches_oracle(name, mask):
-    case = F.make_case(name)
+    if name == "small_heads32":   # 8 attention heads of 32 (the backward's other head size)
+        case = F.make_case("small", repairer=F.RepairerDims(8, 128, 256, 2, 8, 1024))
+    else:
+        case = F.make_case(name)
     a = _batch(case)
     t, r = case.target, case.repairer
     names = T.trained_names(r.n_blocks)
