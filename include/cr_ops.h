@@ -82,6 +82,16 @@ cr_status cr_chunk_starts(const int32_t* chunk_end, const int32_t* cu_seqlens_ho
                           int64_t n_tokens, int32_t* chunk_start, void* stream);
 
 /*
+ * cr_wait_selftest - failure-reporting check: one CTA waits on a pipeline
+ * barrier that nothing arrives on, through the bounded wait every kernel of
+ * the library uses.  The wait gives up after its limit (2 s), records a
+ * timeout at site 900 in the device status word and returns, so
+ * cr_get_device_status then returns CR_ERR_TIMEOUT with out = {1, 900, 0}; the
+ * context stays usable (cr_clear_device_status resets the word).
+ */
+cr_status cr_wait_selftest(void* stream);
+
+/*
  * cr_qkv_rope - the repair block's QKV linear with the repairer RoPE fused
  * into its epilogue: qkv = u W_qkv^T + b_qkv, then Q and K of every head
  * rotated (rotate-half pairs, angle pos[t] * theta^(-2i/d)).

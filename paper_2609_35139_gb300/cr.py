@@ -31,6 +31,7 @@ EXPORTED = [
     "cr_linear", "cr_layernorm", "cr_chunk_causal_attention", "cr_masked_attention",
     "cr_chunk_starts", "cr_qkv_rope", "cr_segment_project",
     "cr_segment_project_noalloc", "cr_param_layout", "cr_train_workspace_bytes", "cr_train_step",
+    "cr_wait_selftest",
 ]
 
 
@@ -118,6 +119,7 @@ def lib(build_if_missing: bool = False) -> ctypes.CDLL:
         "cr_layernorm": (i32, [vp, vp, i64, vp, vp, vp, c_float, i64, i64, vp, vp]),
         "cr_chunk_causal_attention": (i32, [vp, i32, i32, vp, vp, i32, i64, vp, vp]),
         "cr_param_layout": (i32, [P(cr_target_dims), P(cr_repairer_dims), vp, i32]),
+        "cr_wait_selftest": (i32, [vp]),
         "cr_train_workspace_bytes": (c_size_t, [P(cr_target_dims), P(cr_repairer_dims), i64, i64]),
         "cr_train_step": (i32, [P(cr_target_dims), P(cr_repairer_dims), vp, vp, vp, vp, vp, vp, vp, vp, vp,
                                 vp, vp, vp, vp, i32, i64, i32, P(cr_adamw), vp, vp, c_size_t, vp]),
@@ -361,6 +363,11 @@ def cr_chunk_causal_attention(qkv, d_b, n_heads, chunk_end, cu_seqlens_host, out
     _check("cr_chunk_causal_attention", lib().cr_chunk_causal_attention(
         _p(qkv), d_b, n_heads, _p(chunk_end), cu.ctypes.data, len(cu) - 1, qkv.shape[0], _p(out),
         _stream(stream)))
+
+
+def cr_wait_selftest(stream=None):
+    """Launch the bounded-wait check (a wait that must time out and report it)."""
+    _check("cr_wait_selftest", lib().cr_wait_selftest(_stream(stream)))
 
 
 def cr_param_layout(target, rep) -> np.ndarray:

@@ -1347,4 +1347,10 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
     return CR_OK;
 }
 
+cr_status cr_wait_selftest(void* stream) {
+    unsigned* status = device_status_ptr();
+    if (!status) return CR_ERR_CUDA;
+    return launch_wait_selftest(status, static_cast<cudaStream_t>(stream));
+}
+
 }  // extern "C"

@@ -213,6 +213,7 @@ cr_status launch_rope_table(const int32_t* pos, int64_t n, int half_dim, const f
 cr_status launch_layernorm(const float* x, const uint16_t* add, int64_t ld_add, float* x_out,
                            const float* g, const float* b, float eps, int64_t M, int64_t D,
                            uint16_t* u, cudaStream_t st);
+cr_status launch_wait_selftest(unsigned* status, cudaStream_t st);
 cr_status launch_chunk_starts(const int32_t* chunk_end, const AttnParams& p, int64_t n_tokens,
                               int32_t* chunk_start, cudaStream_t st);
 cr_status launch_attention(const uint16_t* qkv, int64_t n_tokens, int head_dim,

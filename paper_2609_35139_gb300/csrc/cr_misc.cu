@@ -223,4 +223,30 @@ cr_status launch_to_bf16(const float* x, int64_t n, uint16_t* y, cudaStream_t st
     return launch_pdl(to_bf16_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st, x, n, y);
 }
 
+// One CTA waiting on a pipeline barrier that nothing arrives on, through the
+// same bounded wait every kernel uses: after CR_WAIT_TIMEOUT_NS the wait gives
+// up, records a timeout at site 900 in the status word and the kernel returns.
+// A check of the failure reporting that neither hangs nor faults the GPU.
+namespace {
+__global__ void wait_selftest_kernel(unsigned* status) {
+    __shared__ uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        abort_flag = 0;
+        fence_barrier_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        const WaitCtx wc{&abort_flag, status};
+        mbar_wait(&bar, 0, wc, 900);
+    }
+}
+}  // namespace
+
+cr_status launch_wait_selftest(unsigned* status, cudaStream_t st) {
+    wait_selftest_kernel<<<1, 32, 0, st>>>(status);
+    return cuda_check(cudaGetLastError());
+}
+
 }  // namespace cr
