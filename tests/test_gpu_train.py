@@ -101,6 +101,35 @@ def test_train_step_matches_oracle(name, mask):
     assert torch.equal(ts.params_bf16, ts.params.to(torch.bfloat16))
 
 
+@pytest.mark.slow
+def test_train_step_matches_oracle_8b_shapes():
+    """The 8B shapes (D_KV 65536, d_b 1024, 6 blocks, 16 heads of 64) on a two-chunk
+    request (1024 tokens): loss, norm and every gradient tensor against the oracle."""
+    case = F.make_case("llama8b", n_req_chunks=2, requests=None)
+    a = _batch(case)
+    t, r = case.target, case.repairer
+    names = T.trained_names(r.n_blocks)
+    params = {k: (O.dtype_to_f64(case.weights[k], "bf16") if case.weights[k].dtype == np.uint16
+                  else case.weights[k].astype(np.float64)) for k in names}
+    zeros = {k: np.zeros_like(v) for k, v in params.items()}
+    lr = 1e-4
+    loss, norm, grads, _, _, _ = T.train_step(params, zeros, zeros, 1, lr, a,
+                                              sigma_stale=case.weights["sigma_stale"],
+                                              sigma_delta=case.weights["sigma_delta"], cache_dtype="bf16",
+                                              head_dim=t.head_dim, n_heads=r.n_heads)
+    ts, dev, n = _session(case, a)
+    stats = _step(ts, dev, a, n, lr)
+    print("8b shapes loss", stats[0], loss, "norm", stats[1], norm)
+    assert abs(float(stats[0]) - loss) <= 1e-3 * loss
+    assert abs(float(stats[1]) - norm) <= 5e-3 * norm
+    for k in names:
+        gg, ref = _tensor(ts, ts.grads, k, params[k].shape), grads[k]
+        cos = float((gg * ref).sum() / np.sqrt((gg ** 2).sum() * (ref ** 2).sum()))
+        rel = float(np.sqrt(np.mean((gg - ref) ** 2)) / np.sqrt(np.mean(ref ** 2)))
+        print(f"  {k:14s} cos {cos:.6f} rel-RMS {rel:.3e}")
+        assert cos >= 0.9999 and rel <= 1.5e-2, (k, cos, rel)
+
+
 def test_train_steps_lower_the_loss():
     case = F.make_case("small_multi")
     a = _batch(case)
