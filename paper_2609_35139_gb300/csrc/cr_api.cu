@@ -931,7 +931,7 @@ cr_status cr_param_layout(const cr_target_dims* target, const cr_repairer_dims* 
 namespace {
 struct TrainLayout {
     size_t inf, h0, rein, blk, blk_stride, hbuf, yf, rope, ones, r, dz, rowsq, perreq, stats_pad, dh, dxm,
-        du, dtmp, pre, gprod, sig16, dqkv, da, lse, dvec, cstart, dse, dy, colsum, norm, blas, total;
+        du, dtmp, pre, gprod, sig16, dqkv, da, lse, dvec, cstart, dse, dy, colsum, colcnt, norm, blas, total;
     size_t x_in, x_mid, u1, u2, qkv, o, g;   // offsets inside one block's region
 };
 constexpr size_t kBlasBytes = 32ull << 20;
@@ -988,6 +988,7 @@ TrainLayout train_layout(const Dims& d, int64_t n) {
     L.dse = take(N * 2 * d.dc * 4);
     L.dy = take(N * d.S * d.dseg * 4);
     L.colsum = take(colsum_scratch_floats(n, std::max(d.D, wide)) * 4);
+    L.colcnt = take(colsum_counters(std::max(d.D, wide)) * 4);
     L.norm = take(sqnorm_scratch_doubles() * 8);
     L.blas = take(kBlasBytes);
     L.total = off;
@@ -1123,6 +1124,7 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
     float* DSE = at<float>(base, L.dse);
     float* DY = at<float>(base, L.dy);
     float* CS = at<float>(base, L.colsum);
+    unsigned* CCNT = at<unsigned>(base, L.colcnt);
     double* NRM = at<double>(base, L.norm);
 
     // ---- forward (Sec. 4.1), keeping what the backward needs
@@ -1232,9 +1234,15 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
     cublasHandle_t hb;
     if ((s = blas_handle(st, base + L.blas, kBlasBytes, &hb)) != CR_OK) return s;
     if ((s = cuda_check(cudaMemsetAsync(grads, 0, static_cast<size_t>(P) * 4, st))) != CR_OK) return s;
+    // column-sum election counters start at zero (each use leaves them at zero)
+    if ((s = cuda_check(cudaMemsetAsync(CCNT, 0, colsum_counters(std::max(d.D, std::max(std::max(d.hid, 3 * d.db),
+                                                                           std::max(2 * d.dc, d.S * d.dseg)))) *
+                                                     4,
+                                        st))) != CR_OK)
+        return s;
     const cudaDataType_t BF = CUDA_R_16BF, F32 = CUDA_R_32F;
     auto colsum = [&](const void* a, bool bf16, int64_t cols, int64_t lda, float* out) {
-        return launch_colsum(a, bf16, N, cols, lda, out, false, CS, st);
+        return launch_colsum(a, bf16, N, cols, lda, out, false, CS, CCNT, st);
     };
     auto to16 = [&](const float* a, int64_t n, uint16_t* out) { return launch_to_bf16(a, n, out, st); };
 #define CR_TRY(x)                   \

@@ -229,8 +229,9 @@ cr_status launch_target(const void* stale, const void* joint, bool f32, const fl
 cr_status launch_loss(const float* r, int64_t N, int64_t D, const LossParams& p, uint16_t* dz, float* rowsq,
                       float* loss_out, double* per_req, cudaStream_t st);
 size_t colsum_scratch_floats(int64_t rows, int64_t cols);
+size_t colsum_counters(int64_t cols);
 cr_status launch_colsum(const void* a, bool bf16, int64_t rows, int64_t cols, int64_t lda, float* out,
-                        bool accumulate, float* scratch, cudaStream_t st);
+                        bool accumulate, float* scratch, unsigned* counters, cudaStream_t st);
 cr_status launch_ln_backward(const float* x, const float* gamma, const float* dy, const float* add, float eps,
                              int64_t N, int D, float* dx, float* gprod, cudaStream_t st);
 cr_status launch_gelu_backward(float* dg, const float* pre, int64_t n, cudaStream_t st);

@@ -5,7 +5,7 @@
 //                        input, so that the head epilogue writes r = z - target
 //   loss_grad_kernel     per row: sum of r^2, and dz = c_request * r (bf16)
 //   loss_reduce_kernel   per request, rows summed in order (fp64): the loss
-//   colsum_*             column sums in a fixed order (bias, LayerNorm grads)
+//   colsum_kernel        column sums in a fixed order (bias, LayerNorm grads)
 //   ln_backward_kernel   LayerNorm backward per row, plus dy * x_hat per element
 //   gelu_backward_kernel dpre = dg * (Phi(pre) + pre phi(pre))
 //   rope_backward_kernel the repairer RoPE's transpose on dQ, dK
@@ -132,34 +132,38 @@ __global__ void loss_total_kernel(const double* __restrict__ per_req, int n_req,
     loss_out[0] = static_cast<float>(l);
 }
 
-// Column sums in a fixed order: slice y of kColSlice rows per block row,
-// partial[y][c]; then the slices in order.
+// Column sums in a fixed order, one launch: block (x, y) sums slice y (kColSlice
+// rows) of 256 columns into partial[y][c]; the last block of column block x to
+// finish (elected by a counter, after a fence) adds the slices in order and
+// resets the counter.  The order of the additions never depends on timing.
 constexpr int kColSlice = 64;
 template <typename T>
 __global__ void __launch_bounds__(256)
-    colsum_partial_kernel(const T* __restrict__ a, int64_t rows, int64_t cols, int64_t lda,
-                          float* __restrict__ part) {
+    colsum_kernel(const T* __restrict__ a, int64_t rows, int64_t cols, int64_t lda, float* part,
+                  float* __restrict__ out, int accumulate, unsigned* __restrict__ counters) {
     pdl_launch_dependents();
     pdl_wait();
     const int64_t c = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
-    if (c >= cols) return;
-    const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kColSlice;
-    const int64_t r1 = min(rows, r0 + kColSlice);
-    float s = 0.0f;
-    for (int64_t r = r0; r < r1; ++r) s += ld(a, r * lda + c);
-    part[static_cast<int64_t>(blockIdx.y) * cols + c] = s;
-}
-
-__global__ void __launch_bounds__(256)
-    colsum_reduce_kernel(const float* __restrict__ part, int64_t slices, int64_t cols, float* __restrict__ out,
-                         int accumulate) {
-    pdl_launch_dependents();
-    pdl_wait();
-    const int64_t c = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
-    if (c >= cols) return;
-    float s = 0.0f;
-    for (int64_t y = 0; y < slices; ++y) s += part[y * cols + c];
-    out[c] = accumulate ? out[c] + s : s;
+    if (c < cols) {
+        const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kColSlice;
+        const int64_t r1 = min(rows, r0 + kColSlice);
+        float s = 0.0f;
+        for (int64_t r = r0; r < r1; ++r) s += ld(a, r * lda + c);
+        part[static_cast<int64_t>(blockIdx.y) * cols + c] = s;
+    }
+    __threadfence();
+    __syncthreads();
+    __shared__ bool last;
+    if (threadIdx.x == 0) last = atomicAdd(&counters[blockIdx.x], 1u) == gridDim.y - 1;
+    __syncthreads();
+    if (!last) return;
+    __threadfence();
+    if (c < cols) {
+        float s = 0.0f;
+        for (int64_t y = 0; y < gridDim.y; ++y) s += __ldcg(part + y * cols + c);
+        out[c] = accumulate ? out[c] + s : s;
+    }
+    if (threadIdx.x == 0) counters[blockIdx.x] = 0u;
 }
 
 // LayerNorm backward, one warp per row of D (a multiple of 32, at most 1024)
@@ -405,17 +409,17 @@ size_t colsum_scratch_floats(int64_t rows, int64_t cols) {
     return static_cast<size_t>((rows + kColSlice - 1) / kColSlice) * static_cast<size_t>(cols);
 }
 
+size_t colsum_counters(int64_t cols) { return static_cast<size_t>((cols + 255) / 256); }
+
 cr_status launch_colsum(const void* a, bool bf16, int64_t rows, int64_t cols, int64_t lda, float* out,
-                        bool accumulate, float* scratch, cudaStream_t st) {
+                        bool accumulate, float* scratch, unsigned* counters, cudaStream_t st) {
     const int64_t slices = (rows + kColSlice - 1) / kColSlice;
+    if (slices > 65535) return CR_ERR_UNSUPPORTED;
     const dim3 g1(static_cast<unsigned>((cols + 255) / 256), static_cast<unsigned>(slices));
-    cr_status s = bf16 ? launch_pdl(colsum_partial_kernel<uint16_t>, g1, dim3(256), 0, st,
-                                    static_cast<const uint16_t*>(a), rows, cols, lda, scratch)
-                       : launch_pdl(colsum_partial_kernel<float>, g1, dim3(256), 0, st,
-                                    static_cast<const float*>(a), rows, cols, lda, scratch);
-    if (s != CR_OK) return s;
-    return launch_pdl(colsum_reduce_kernel, dim3(static_cast<unsigned>((cols + 255) / 256)), dim3(256), 0, st,
-                      static_cast<const float*>(scratch), slices, cols, out, accumulate ? 1 : 0);
+    return bf16 ? launch_pdl(colsum_kernel<uint16_t>, g1, dim3(256), 0, st, static_cast<const uint16_t*>(a),
+                             rows, cols, lda, scratch, out, accumulate ? 1 : 0, counters)
+                : launch_pdl(colsum_kernel<float>, g1, dim3(256), 0, st, static_cast<const float*>(a), rows,
+                             cols, lda, scratch, out, accumulate ? 1 : 0, counters);
 }
 
 cr_status launch_ln_backward(const float* x, const float* gamma, const float* dy, const float* add, float eps,
