@@ -380,8 +380,9 @@ typedef struct cr_adamw {
 } cr_adamw;
 
 /* Workspace bytes of cr_train_step for batches of up to max_tokens tokens in
- * total whose longest request has max_request_tokens tokens; 0 if the
- * dimensions are invalid. */
+ * total (max_request_tokens, the longest request, must lie in
+ * [1, max_tokens]; the fused attention backward needs no per-request
+ * scratch); 0 if the dimensions are invalid. */
 size_t cr_train_workspace_bytes(const cr_target_dims* target, const cr_repairer_dims* rep,
                                 int64_t max_tokens, int64_t max_request_tokens);
 
@@ -401,11 +402,13 @@ size_t cr_train_workspace_bytes(const cr_target_dims* target, const cr_repairer_
  * (canonical K), emb [N, d_model] bf16, chunk_end, pos [N] int32 as written by
  * cr_assemble_stale; cu_seqlens_host [n_req + 1] HOST.  stats_out: device
  * fp32 [4] = loss, gradient norm before clipping, clipping coefficient, 0.
- * The forward computes as cr_compress_features + cr_repair_forward; the
- * backward's plain matrix products run in cuBLAS (bf16 operands, fp32
- * accumulation; the attention backward in TF32 on fp32 operands), using a
- * part of the workspace as cuBLAS's workspace.  All device buffers 16-byte
- * aligned; P = the last offset of cr_param_layout.
+ * The forward computes as cr_compress_features + cr_repair_forward (its
+ * attention also keeps each row's log-sum-exp); the attention backward is
+ * fused (P recomputed tile by tile, no score matrix in memory); the backward's
+ * plain matrix products (weight and input gradients) run in cuBLAS (bf16
+ * operands, fp32 accumulation), using a part of the workspace as cuBLAS's
+ * workspace.  All device buffers 16-byte aligned; P = the last offset of
+ * cr_param_layout.
  */
 cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* rep, float* params,
                         uint16_t* params_bf16, float* adam_m, float* adam_v, float* grads,

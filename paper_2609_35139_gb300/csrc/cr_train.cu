@@ -482,7 +482,8 @@ cr_status blas_handle(cudaStream_t st, void* ws, size_t ws_bytes, cublasHandle_t
     return CR_OK;
 }
 
-// Row-major C[M, N] = alpha op(A) op(B) + beta C, op(A) [M, K], op(B) [K, N];
+// Row-major C[M, N] = alpha op(A) op(B) + beta C, op(A) [M, K], op(B) [K, N]
+// (bf16 operands with fp32 accumulation; fp32 operands would run in TF32);
 // tA: A is stored [K, M] (op(A) = A^T); tB: B is stored [N, K].  In cuBLAS's
 // column-major terms this is C^T = op(B)^T op(A)^T on the same memory.
 cr_status gemm_rm(cublasHandle_t h, bool tA, bool tB, int64_t M, int64_t N, int64_t K, float alpha,
