@@ -15,8 +15,10 @@
 //       walks the key tiles it sees (as the forward); S = Q K^T, dP = dO V^T,
 //       dS into TMEM, dQ += dS K.
 // Warp 0 loads by TMA (the CTA's own two tiles once, the walked tiles' pairs
-// into a 2-stage ring), warp 1 issues the MMAs and owns TMEM, warps 4-7 do
-// the exponentials (32 columns at a time).  Every wait is bounded.
+// into a 2-stage ring), warp 1 issues the MMAs and owns TMEM, warps 4-7 and
+// 8-11 do the exponentials on the same rows (TMEM lanes), the first group the
+// low 64 columns of each tile and the second the high 64, 32 at a time, so two
+// warps share each SM sub-partition.  Every wait is bounded.
 #include <cuda_bf16.h>
 
 #include "cr_internal.h"
@@ -41,7 +43,7 @@ struct BwdCfg {
     static constexpr uint32_t kTmemP = 384, kTmemDS = 448;
 };
 
-constexpr int kBwdThreads = 256;
+constexpr int kBwdThreads = 384;
 
 __device__ __forceinline__ int bwd_hi(const AttnBwdParams& p, int rs, int len, int q) {
     if (p.mask_mode == CR_MASK_TOKEN_CAUSAL) return q + 1;
@@ -97,12 +99,12 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
             mbar_init(&kv_empty[s], 1);
         }
         mbar_init(s_full, 1);
-        mbar_init(s_free, 4);
-        mbar_init(p_full, 4);
+        mbar_init(s_free, 8);
+        mbar_init(p_full, 8);
         mbar_init(pv_done, 1);
         mbar_init(drain, 1);
-        mbar_init(&vec_full[0], 128);
-        mbar_init(&vec_full[1], 128);
+        mbar_init(&vec_full[0], 256);
+        mbar_init(&vec_full[1], 256);
         *abort_flag = 0;
         fence_barrier_init();
     }
@@ -244,6 +246,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
     } else if (warp >= 4) {
         // ---------------------------------------------------- elementwise warps
         const uint32_t quad = warp & 3u;
+        const int eg = (static_cast<int>(warp) - 4) >> 2;   // column half 0 / 1
         const int r = static_cast<int>(quad * 32 + lane);
         const int own = t0 + r;                  // this thread's row of the own tile
         const bool own_ok = own < len;
@@ -267,17 +270,20 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
             const int wrow0 = (w0 + j) * 128;    // walked tile's first row (request-local)
             float* vb = vec + (j & 1) * 4 * 128;
             if constexpr (KV) {
-                // the walked query tile's lse, D and visible-key bounds, one per thread
-                const int q = wrow0 + r;
-                const bool qv = q < len;
-                reinterpret_cast<float2*>(vb)[r] =
-                    qv ? make_float2(__ldg(p.lse + static_cast<int64_t>(head) * total + rs + q),
-                                     __ldg(p.dvec + static_cast<int64_t>(head) * total + rs + q))
-                       : make_float2(0.0f, 0.0f);
-                vb[256 + r] = __int_as_float(qv ? bwd_hi(p, rs, len, q) : 0);
-                vb[384 + r] = __int_as_float(qv ? bwd_lo(p, rs, q) : 0);
-                // all 128 entries written (a buffer is rewritten two tiles later, after
-                // every thread has passed the tile in between)
+                // the walked query tile's lse, D and visible-key bounds, one per
+                // thread of the first group; both groups arrive, so a buffer is
+                // rewritten (two tiles later) only after both have passed the tile
+                // in between
+                if (eg == 0) {
+                    const int q = wrow0 + r;
+                    const bool qv = q < len;
+                    reinterpret_cast<float2*>(vb)[r] =
+                        qv ? make_float2(__ldg(p.lse + static_cast<int64_t>(head) * total + rs + q),
+                                         __ldg(p.dvec + static_cast<int64_t>(head) * total + rs + q))
+                           : make_float2(0.0f, 0.0f);
+                    vb[256 + r] = __int_as_float(qv ? bwd_hi(p, rs, len, q) : 0);
+                    vb[384 + r] = __int_as_float(qv ? bwd_lo(p, rs, q) : 0);
+                }
                 mbar_arrive(&vec_full[j & 1]);
                 ok = mbar_wait(&vec_full[j & 1], static_cast<uint32_t>(j >> 1) & 1u, wc, 330);
                 if (!__all_sync(0xffffffffu, ok)) {
@@ -297,12 +303,12 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
             if constexpr (KV)
                 full = own_ok && wrow0 + 127 < len && own < __float_as_int(vb[256]) &&
                        own >= __float_as_int(vb[384 + 127]);
-            for (int c0 = 0; c0 < 128; c0 += 32) {
+            for (int c0 = eg * 64; c0 < eg * 64 + 64; c0 += 32) {
                 float s[32], dp[32];
                 tmem_ld32(tS + c0, s);
                 tmem_ld32(tDP + c0, dp);
                 tmem_wait_ld();
-                if (c0 == 96) {   // S and dP fully read: the next tile's MMAs may overwrite them
+                if (c0 == eg * 64 + 32) {   // this half of S and dP read: the next tile's MMAs may overwrite them
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(s_free);
@@ -346,7 +352,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
                     pk[i] = pack_bf16x2(pv[2 * i], pv[2 * i + 1]);
                     dk[i] = pack_bf16x2(dsv[2 * i], dsv[2 * i + 1]);
                 }
-                if (c0 == 0 && j > 0) {   // the previous tile's TS products read P and dS
+                if (c0 == eg * 64 && j > 0) {   // the previous tile's TS products read P and dS
                     ok = mbar_wait(pv_done, static_cast<uint32_t>(j - 1) & 1u, wc, 332);
                     if (!__all_sync(0xffffffffu, ok)) {
                         ok = false;
@@ -384,7 +390,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
                 const float f = (KV && a == 0) ? 1.0f : p.scale;
                 float* dst = row + (KV ? (a == 0 ? 2 * p.d_b : p.d_b) : 0) + head * D;
 #pragma unroll
-                for (int c = 0; c < D; c += 16) {
+                for (int c = eg * (D / 2); c < (eg + 1) * (D / 2); c += 16) {
                     float v[16];
                     if (nw > 0) {
                         tmem_ld16(ta + c, v);
