@@ -15,6 +15,9 @@
  *   cr_apply_residual     KV residual head, in-place residual add,
  *                         optional global RoPE on K               (Sec. 4.1)
  *
+ * (cr_assemble_compress runs the first two as one call, with one fewer pass
+ * over the cache.)
+ *
  * Conventions shared by every call
  * --------------------------------
  * Ownership: the caller owns and allocates every buffer (device memory
@@ -198,6 +201,27 @@ cr_status cr_assemble_stale(const cr_target_dims* target, const void* kv_pool,
 cr_status cr_compress_features(const cr_target_dims* target, const cr_repairer_dims* rep,
                                const cr_weights* w, const void* kv, const void* emb,
                                int64_t n_tokens, float* h0_out, uint16_t* rein_out,
+                               void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * cr_assemble_compress - cr_assemble_stale followed by cr_compress_features
+ * in one call, with the same arguments and the same results bit for bit
+ * (Sec. 4.1, "Chunk-cache preparation" and the StaleEncoder).  For a bf16
+ * cache the segment projection reads its cache tiles straight from kv_pool
+ * and writes each tile it reads into kv_out, so the assembly costs one read
+ * and one write of the cache instead of two reads and a write; fp32 caches
+ * take the two-call path.  The caller sizes kv_out, emb_out and the
+ * workspace (cr_workspace_bytes(.., max_tokens)) for max_tokens rows.
+ * Errors: those of the two calls, checked before any launch.
+ */
+cr_status cr_assemble_compress(const cr_target_dims* target, const cr_repairer_dims* rep,
+                               const cr_weights* w, const void* kv_pool, const void* emb_pool,
+                               int64_t n_pool_tokens, const int64_t* chunk_start,
+                               const int32_t* chunk_len, int32_t n_pool_chunks,
+                               const int32_t* chunk_idx, const int32_t* cu_chunks, int32_t n_req,
+                               void* kv_out, void* emb_out, int64_t max_tokens, int32_t* chunk_id,
+                               int32_t* chunk_end, int32_t* pos, int32_t* cu_seqlens_dev,
+                               int32_t* cu_seqlens_host, float* h0_out, uint16_t* rein_out,
                                void* workspace, size_t workspace_bytes, void* stream);
 
 /*

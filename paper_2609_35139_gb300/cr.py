@@ -23,7 +23,8 @@ CR_ROPE_NONE, CR_ROPE_GLOBAL = 0, 1
 CR_EPI_BF16, CR_EPI_GELU_BF16, CR_EPI_ADD_F32, CR_EPI_F32 = range(4)
 
 EXPORTED = [
-    "cr_workspace_bytes", "cr_assemble_stale", "cr_compress_features", "cr_repair_forward",
+    "cr_workspace_bytes", "cr_assemble_stale", "cr_compress_features", "cr_assemble_compress",
+    "cr_repair_forward",
     "cr_repair_forward_masked", "cr_apply_residual", "cr_apply_residual_select", "cr_rotate_k",
     "cr_apply_residual_paged", "cr_canonicalize_chunks",
     "cr_sigma_workspace_bytes", "cr_sigma_accumulate", "cr_sigma_finalize", "cr_get_device_status",
@@ -95,6 +96,9 @@ def lib(build_if_missing: bool = False) -> ctypes.CDLL:
                                     vp, i64, vp, vp, vp, vp, vp, vp]),
         "cr_compress_features": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp,
                                        vp, i64, vp, vp, vp, c_size_t, vp]),
+        "cr_assemble_compress": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp,
+                                       vp, i64, vp, vp, i32, vp, vp, i32, vp, vp, i64, vp, vp, vp,
+                                       vp, vp, vp, vp, vp, c_size_t, vp]),
         "cr_repair_forward": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp, vp,
                                     vp, vp, vp, i32, i64, vp, vp, c_size_t, vp]),
         "cr_repair_forward_masked": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights),
@@ -229,6 +233,26 @@ def cr_compress_features(target, rep, weights: PackedWeights, kv, emb, n_tokens,
         n_tokens, _p(h0_out), _p(rein_out), _p(workspace), workspace.numel() * workspace.element_size(),
         _stream(stream))
     _check("cr_compress_features", st)
+
+
+def cr_assemble_compress(target, rep, weights: PackedWeights, kv_pool, emb_pool, chunk_start,
+                         chunk_len, chunk_idx, cu_chunks, kv_out, emb_out, chunk_id, chunk_end, pos,
+                         cu_seqlens_dev, h0_out, rein_out, workspace, stream=None):
+    """cr_assemble_stale + cr_compress_features in one call; returns (n_tokens, cu_seqlens_host)."""
+    cs = _host_arr(chunk_start, np.int64)
+    cl = _host_arr(chunk_len, np.int32)
+    ci = _host_arr(chunk_idx, np.int32)
+    cu = _host_arr(cu_chunks, np.int32)
+    n_req = len(cu) - 1
+    cu_host = np.zeros(max(n_req + 1, 1), np.int32)
+    st = lib().cr_assemble_compress(
+        ctypes.byref(target), ctypes.byref(rep), ctypes.byref(weights.struct), _p(kv_pool),
+        _p(emb_pool), kv_pool.shape[0], cs.ctypes.data, cl.ctypes.data, len(cl), ci.ctypes.data,
+        cu.ctypes.data, n_req, _p(kv_out), _p(emb_out), kv_out.shape[0], _p(chunk_id),
+        _p(chunk_end), _p(pos), _p(cu_seqlens_dev), cu_host.ctypes.data, _p(h0_out), _p(rein_out),
+        _p(workspace), workspace.numel() * workspace.element_size(), _stream(stream))
+    _check("cr_assemble_compress", st)
+    return int(cu_host[-1]), cu_host
 
 
 def cr_repair_forward(target, rep, weights: PackedWeights, h0, rein, chunk_end, pos,

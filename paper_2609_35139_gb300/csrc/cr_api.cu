@@ -239,51 +239,35 @@ size_t cr_workspace_bytes(const cr_target_dims* target, const cr_repairer_dims* 
     return ws_layout(dims_of(target, rep), max_tokens).total;
 }
 
-cr_status cr_assemble_stale(const cr_target_dims* target, const void* kv_pool,
-                            const void* emb_pool, int64_t n_pool_tokens,
-                            const int64_t* chunk_start, const int32_t* chunk_len,
-                            int32_t n_pool_chunks, const int32_t* chunk_idx,
-                            const int32_t* cu_chunks, int32_t n_req, void* kv_out,
-                            void* emb_out, int64_t max_tokens, int32_t* chunk_id,
-                            int32_t* chunk_end, int32_t* pos, int32_t* cu_seqlens_dev,
-                            int32_t* cu_seqlens_host, void* stream) {
-    cr_status s = check_target(target);
-    if (s != CR_OK) return s;
-    if (!chunk_start || !chunk_len || !chunk_idx || !cu_chunks || !cu_seqlens_host)
-        return CR_ERR_INVALID_ARG;
+// The gather table of one assembly call from the HOST chunk map (validated):
+// every selected chunk's pool rows, output rows and request-local position.
+static cr_status build_gather(const Dims& d, const void* kv_pool, const void* emb_pool,
+                              int64_t n_pool_tokens, const int64_t* chunk_start,
+                              const int32_t* chunk_len, int32_t n_pool_chunks,
+                              const int32_t* chunk_idx, const int32_t* cu_chunks, int32_t n_req,
+                              void* kv_out, void* emb_out, int64_t max_tokens, int32_t* chunk_id,
+                              int32_t* chunk_end, int32_t* pos, int32_t* cu_seqlens_dev,
+                              GatherParams* p) {
+    if (!chunk_start || !chunk_len || !chunk_idx || !cu_chunks) return CR_ERR_INVALID_ARG;
     if (n_req < 1 || n_req > kMaxReq || n_pool_chunks < 1 || n_pool_tokens < 1)
         return CR_ERR_INVALID_ARG;
     if (!all_aligned(kv_pool, emb_pool, kv_out, emb_out, chunk_id, chunk_end, pos, cu_seqlens_dev))
         return CR_ERR_INVALID_ARG;
-    const Dims d = dims_of(target, nullptr);
+    if (cu_chunks[0] != 0) return CR_ERR_INVALID_ARG;
     const int64_t es = d.f32 ? 4 : 2;
-    GatherParams* p = new GatherParams();   // ~17 KB: keep it off the caller's stack
     memset(p, 0, sizeof(*p));
-    if (cu_chunks[0] != 0) {
-        delete p;
-        return CR_ERR_INVALID_ARG;
-    }
     int64_t t = 0;
     int n_seg = 0;
     p->cu_seqlens_host[0] = 0;
     for (int r = 0; r < n_req; ++r) {
         const int a = cu_chunks[r], b = cu_chunks[r + 1];
-        if (b <= a || b - a > kMaxSegs) {
-            delete p;
-            return CR_ERR_INVALID_ARG;
-        }
+        if (b <= a || b - a > kMaxSegs) return CR_ERR_INVALID_ARG;
         int64_t local = 0;
         for (int k = a; k < b; ++k) {
             const int c = chunk_idx[k];
-            if (c < 0 || c >= n_pool_chunks || n_seg >= kMaxSegs) {
-                delete p;
-                return CR_ERR_INVALID_ARG;
-            }
+            if (c < 0 || c >= n_pool_chunks || n_seg >= kMaxSegs) return CR_ERR_INVALID_ARG;
             const int64_t st = chunk_start[c], ln = chunk_len[c];
-            if (ln < 1 || st < 0 || st + ln > n_pool_tokens) {
-                delete p;
-                return CR_ERR_INVALID_ARG;
-            }
+            if (ln < 1 || st < 0 || st + ln > n_pool_tokens) return CR_ERR_INVALID_ARG;
             GatherSeg& g = p->seg[n_seg++];
             g.src_row = st;
             g.dst_row = t;
@@ -292,17 +276,11 @@ cr_status cr_assemble_stale(const cr_target_dims* target, const void* kv_pool,
             g.local_start = static_cast<int32_t>(local);
             local += ln;
             t += ln;
-            if (local > INT32_MAX / 2) {
-                delete p;
-                return CR_ERR_INVALID_ARG;
-            }
+            if (local > INT32_MAX / 2) return CR_ERR_INVALID_ARG;
         }
         p->cu_seqlens_host[r + 1] = static_cast<int32_t>(t);
     }
-    if (t > max_tokens || t > INT32_MAX / 2) {
-        delete p;
-        return CR_ERR_INVALID_ARG;
-    }
+    if (t > max_tokens || t > INT32_MAX / 2) return CR_ERR_INVALID_ARG;
     p->kv_pool = static_cast<const uint8_t*>(kv_pool);
     p->emb_pool = static_cast<const uint8_t*>(emb_pool);
     p->kv_out = static_cast<uint8_t*>(kv_out);
@@ -318,8 +296,29 @@ cr_status cr_assemble_stale(const cr_target_dims* target, const void* kv_pool,
     p->n_seg = n_seg;
     p->n_req = n_req;
     p->status = device_status_ptr();
-    for (int r = 0; r <= n_req; ++r) cu_seqlens_host[r] = p->cu_seqlens_host[r];
-    s = p->status ? launch_gather(*p, static_cast<cudaStream_t>(stream)) : CR_ERR_CUDA;
+    return p->status ? CR_OK : CR_ERR_CUDA;
+}
+
+cr_status cr_assemble_stale(const cr_target_dims* target, const void* kv_pool,
+                            const void* emb_pool, int64_t n_pool_tokens,
+                            const int64_t* chunk_start, const int32_t* chunk_len,
+                            int32_t n_pool_chunks, const int32_t* chunk_idx,
+                            const int32_t* cu_chunks, int32_t n_req, void* kv_out,
+                            void* emb_out, int64_t max_tokens, int32_t* chunk_id,
+                            int32_t* chunk_end, int32_t* pos, int32_t* cu_seqlens_dev,
+                            int32_t* cu_seqlens_host, void* stream) {
+    cr_status s = check_target(target);
+    if (s != CR_OK) return s;
+    if (!cu_seqlens_host) return CR_ERR_INVALID_ARG;
+    const Dims d = dims_of(target, nullptr);
+    GatherParams* p = new GatherParams();   // ~17 KB: keep it off the caller's stack
+    s = build_gather(d, kv_pool, emb_pool, n_pool_tokens, chunk_start, chunk_len, n_pool_chunks,
+                     chunk_idx, cu_chunks, n_req, kv_out, emb_out, max_tokens, chunk_id, chunk_end,
+                     pos, cu_seqlens_dev, p);
+    if (s == CR_OK) {
+        for (int r = 0; r <= n_req; ++r) cu_seqlens_host[r] = p->cu_seqlens_host[r];
+        s = launch_gather(*p, static_cast<cudaStream_t>(stream));
+    }
     delete p;
     return s;
 }
@@ -333,50 +332,13 @@ static cr_status check_weights_compress(const Dims& d, const cr_weights* w) {
     return CR_OK;
 }
 
-cr_status cr_compress_features(const cr_target_dims* target, const cr_repairer_dims* rep,
-                               const cr_weights* w, const void* kv, const void* emb,
-                               int64_t n_tokens, float* h0_out, uint16_t* rein_out,
-                               void* workspace, size_t workspace_bytes, void* stream) {
-    cr_status s = check_target(target);
-    if (s == CR_OK) s = check_repairer(rep);
-    if (s != CR_OK) return s;
-    const Dims d = dims_of(target, rep);
-    if (n_tokens < 1 || n_tokens > INT32_MAX / 2) return CR_ERR_INVALID_ARG;
-    if ((s = check_weights_compress(d, w)) != CR_OK) return s;
-    if (!all_aligned(kv, emb, h0_out, workspace)) return CR_ERR_INVALID_ARG;
-    if (d.B > 0 && !all_aligned(rein_out)) return CR_ERR_INVALID_ARG;
-    const WsLayout L = ws_layout(d, n_tokens);
-    if (workspace_bytes < L.total) return CR_ERR_INVALID_ARG;
-    unsigned* status = device_status_ptr();
-    if (!status) return CR_ERR_CUDA;
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    const int64_t N = n_tokens;
-
-    uint16_t* wfold = at<uint16_t>(workspace, L.wfold);
-    if ((s = launch_fold_sigma(w->w_seg, w->sigma_stale, static_cast<int>(d.S),
-                               static_cast<int>(d.dseg), static_cast<int>(d.dh), wfold, st)) != CR_OK)
-        return s;
-    const uint16_t* kvb = static_cast<const uint16_t*>(kv);
-    const uint16_t* embb = static_cast<const uint16_t*>(emb);
-    if (d.f32) {
-        uint16_t* k2 = at<uint16_t>(workspace, L.kvb);
-        uint16_t* e2 = at<uint16_t>(workspace, L.embb);
-        if ((s = launch_to_bf16(static_cast<const float*>(kv), N * d.D, k2, st)) != CR_OK) return s;
-        if ((s = launch_to_bf16(static_cast<const float*>(emb), N * d.dmodel, e2, st)) != CR_OK)
-            return s;
-        kvb = k2;
-        embb = e2;
-    }
-    uint16_t* y = at<uint16_t>(workspace, L.y);
-    SegParams sp{};
-    sp.M = static_cast<int32_t>(N);
-    sp.S = static_cast<int32_t>(d.S);
-    sp.d_seg = static_cast<int32_t>(d.dseg);
-    sp.b_seg = w->b_seg;
-    sp.y = y;
-    sp.status = status;
-    if ((s = launch_segproj(kvb, d.D, wfold, static_cast<int>(d.dh), sp, st)) != CR_OK) return s;
-
+// Stage 2 and token fusion of the encoder (Sec. 4.1): s = W_map y + b_map,
+// [s ; P_tok E] -> h^0 = F(.), and the reinjection terms P_b(s).
+static cr_status compress_stage2(const Dims& d, const cr_weights* w, const uint16_t* y,
+                                 const uint16_t* embb, int64_t N, float* h0_out,
+                                 uint16_t* rein_out, void* workspace, const WsLayout& L,
+                                 unsigned* status, cudaStream_t st) {
+    cr_status s;
     uint16_t* se = at<uint16_t>(workspace, L.se);   // [N, 2 d_c] = [s ; P_tok E]
     GemmParams gp{};
     gp.status = status;
@@ -406,6 +368,135 @@ cr_status cr_compress_features(const cr_target_dims* target, const cr_repairer_d
             return s;
     }
     return CR_OK;
+}
+
+static SegParams seg_params(const Dims& d, const cr_weights* w, int64_t N, uint16_t* y,
+                            unsigned* status) {
+    SegParams sp{};
+    sp.M = static_cast<int32_t>(N);
+    sp.S = static_cast<int32_t>(d.S);
+    sp.d_seg = static_cast<int32_t>(d.dseg);
+    sp.b_seg = w->b_seg;
+    sp.y = y;
+    sp.status = status;
+    return sp;
+}
+
+// Argument checks shared by the encoder entry points; fills the workspace layout.
+static cr_status check_compress(const cr_target_dims* target, const cr_repairer_dims* rep,
+                                const cr_weights* w, int64_t max_tokens, float* h0_out,
+                                uint16_t* rein_out, void* workspace, size_t workspace_bytes,
+                                Dims* d, WsLayout* L) {
+    cr_status s = check_target(target);
+    if (s == CR_OK) s = check_repairer(rep);
+    if (s != CR_OK) return s;
+    *d = dims_of(target, rep);
+    if (max_tokens < 1 || max_tokens > INT32_MAX / 2) return CR_ERR_INVALID_ARG;
+    if ((s = check_weights_compress(*d, w)) != CR_OK) return s;
+    if (!all_aligned(h0_out, workspace)) return CR_ERR_INVALID_ARG;
+    if (d->B > 0 && !all_aligned(rein_out)) return CR_ERR_INVALID_ARG;
+    *L = ws_layout(*d, max_tokens);
+    if (workspace_bytes < L->total) return CR_ERR_INVALID_ARG;
+    return CR_OK;
+}
+
+cr_status cr_compress_features(const cr_target_dims* target, const cr_repairer_dims* rep,
+                               const cr_weights* w, const void* kv, const void* emb,
+                               int64_t n_tokens, float* h0_out, uint16_t* rein_out,
+                               void* workspace, size_t workspace_bytes, void* stream) {
+    Dims d;
+    WsLayout L;
+    cr_status s = check_compress(target, rep, w, n_tokens, h0_out, rein_out, workspace,
+                                 workspace_bytes, &d, &L);
+    if (s != CR_OK) return s;
+    if (!all_aligned(kv, emb)) return CR_ERR_INVALID_ARG;
+    unsigned* status = device_status_ptr();
+    if (!status) return CR_ERR_CUDA;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int64_t N = n_tokens;
+
+    uint16_t* wfold = at<uint16_t>(workspace, L.wfold);
+    if ((s = launch_fold_sigma(w->w_seg, w->sigma_stale, static_cast<int>(d.S),
+                               static_cast<int>(d.dseg), static_cast<int>(d.dh), wfold, st)) != CR_OK)
+        return s;
+    const uint16_t* kvb = static_cast<const uint16_t*>(kv);
+    const uint16_t* embb = static_cast<const uint16_t*>(emb);
+    if (d.f32) {
+        uint16_t* k2 = at<uint16_t>(workspace, L.kvb);
+        uint16_t* e2 = at<uint16_t>(workspace, L.embb);
+        if ((s = launch_to_bf16(static_cast<const float*>(kv), N * d.D, k2, st)) != CR_OK) return s;
+        if ((s = launch_to_bf16(static_cast<const float*>(emb), N * d.dmodel, e2, st)) != CR_OK)
+            return s;
+        kvb = k2;
+        embb = e2;
+    }
+    uint16_t* y = at<uint16_t>(workspace, L.y);
+    const SegParams sp = seg_params(d, w, N, y, status);
+    if ((s = launch_segproj(kvb, d.D, wfold, static_cast<int>(d.dh), sp, st)) != CR_OK) return s;
+    return compress_stage2(d, w, y, embb, N, h0_out, rein_out, workspace, L, status, st);
+}
+
+cr_status cr_assemble_compress(const cr_target_dims* target, const cr_repairer_dims* rep,
+                               const cr_weights* w, const void* kv_pool, const void* emb_pool,
+                               int64_t n_pool_tokens, const int64_t* chunk_start,
+                               const int32_t* chunk_len, int32_t n_pool_chunks,
+                               const int32_t* chunk_idx, const int32_t* cu_chunks, int32_t n_req,
+                               void* kv_out, void* emb_out, int64_t max_tokens, int32_t* chunk_id,
+                               int32_t* chunk_end, int32_t* pos, int32_t* cu_seqlens_dev,
+                               int32_t* cu_seqlens_host, float* h0_out, uint16_t* rein_out,
+                               void* workspace, size_t workspace_bytes, void* stream) {
+    Dims d;
+    WsLayout L;
+    cr_status s = check_compress(target, rep, w, max_tokens, h0_out, rein_out, workspace,
+                                 workspace_bytes, &d, &L);
+    if (s != CR_OK) return s;
+    if (!cu_seqlens_host) return CR_ERR_INVALID_ARG;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    GatherParams* p = new GatherParams();
+    s = build_gather(d, kv_pool, emb_pool, n_pool_tokens, chunk_start, chunk_len, n_pool_chunks,
+                     chunk_idx, cu_chunks, n_req, kv_out, emb_out, max_tokens, chunk_id, chunk_end,
+                     pos, cu_seqlens_dev, p);
+    const int64_t N = p->n_tokens;
+    if (s == CR_OK && (d.f32 || n_pool_tokens > INT32_MAX)) {
+        // fp32 caches go through the bf16 conversion of the two-call form
+        for (int r = 0; r <= n_req; ++r) cu_seqlens_host[r] = p->cu_seqlens_host[r];
+        s = launch_gather(*p, st);
+        delete p;
+        if (s != CR_OK) return s;
+        return cr_compress_features(target, rep, w, kv_out, emb_out, N, h0_out, rein_out,
+                                    workspace, workspace_bytes, stream);
+    }
+    SegTiles* tl = (s == CR_OK) ? new SegTiles() : nullptr;
+    if (s == CR_OK) {
+        for (int r = 0; r <= n_req; ++r) cu_seqlens_host[r] = p->cu_seqlens_host[r];
+        tl->n_seg = p->n_seg;
+        tl->tile_prefix[0] = 0;
+        for (int i = 0; i < p->n_seg; ++i) {
+            const GatherSeg& g = p->seg[i];
+            tl->src_row[i] = g.src_row;
+            tl->dst_row[i] = static_cast<int32_t>(g.dst_row);
+            tl->len[i] = g.len;
+            tl->tile_prefix[i + 1] = tl->tile_prefix[i] + (g.len + 127) / 128;
+        }
+        // the embeddings and the chunk map here; the cache rows go with the projection
+        p->kv_row_bytes = 0;
+        s = launch_gather(*p, st);
+    }
+    unsigned* status = p->status;
+    delete p;
+    uint16_t* wfold = at<uint16_t>(workspace, L.wfold);
+    if (s == CR_OK)
+        s = launch_fold_sigma(w->w_seg, w->sigma_stale, static_cast<int>(d.S),
+                              static_cast<int>(d.dseg), static_cast<int>(d.dh), wfold, st);
+    uint16_t* y = at<uint16_t>(workspace, L.y);
+    if (s == CR_OK)
+        s = launch_segproj_pool(static_cast<const uint16_t*>(kv_pool), n_pool_tokens,
+                                static_cast<uint16_t*>(kv_out), wfold, static_cast<int>(d.dh),
+                                seg_params(d, w, N, y, status), *tl, st);
+    delete tl;
+    if (s != CR_OK) return s;
+    return compress_stage2(d, w, y, static_cast<const uint16_t*>(emb_out), N, h0_out, rein_out,
+                           workspace, L, status, st);
 }
 
 static bool valid_mask_mode(int32_t m) {

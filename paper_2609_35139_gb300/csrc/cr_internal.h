@@ -98,6 +98,18 @@ struct SegParams {
     const float* b_seg;  // [S, d_seg]
     uint16_t* y;         // [M, S * d_seg]
     unsigned* status;
+    uint16_t* kv_out;    // pool variant: assembled cache [M, ld_out]
+    int64_t ld_out;
+};
+// Row map of the pool-reading segment projection: selected chunk i covers
+// assembled rows [dst_row[i], dst_row[i] + len[i]), read from pool rows
+// starting at src_row[i]; its 128-row tiles are numbered from tile_prefix[i].
+struct SegTiles {
+    int32_t n_seg;
+    int32_t tile_prefix[kMaxSegs + 1];
+    int32_t dst_row[kMaxSegs];
+    int32_t len[kMaxSegs];
+    int64_t src_row[kMaxSegs];
 };
 
 // ------------------------------------------------------------------ attention
@@ -205,6 +217,12 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
                       cudaStream_t st);
 cr_status launch_segproj(const uint16_t* kv, int64_t ld_kv, const uint16_t* wfold, int head_dim,
                          SegParams p, cudaStream_t st);
+// The same projection reading the cache tiles straight from the pool (rows
+// mapped by `tiles`) and storing each tile, as read, into kv_out [M, D_KV]:
+// the stale-cache assembly and stage 1 of the encoder in one pass (bf16).
+cr_status launch_segproj_pool(const uint16_t* kv_pool, int64_t n_pool_tokens, uint16_t* kv_out,
+                              const uint16_t* wfold, int head_dim, SegParams p,
+                              const SegTiles& tiles, cudaStream_t st);
 cr_status launch_fold_sigma(const uint16_t* w_seg, const float* sigma, int S, int d_seg,
                             int head_dim, uint16_t* wfold, cudaStream_t st);
 cr_status launch_to_bf16(const float* x, int64_t n, uint16_t* y, cudaStream_t st);

@@ -12,6 +12,16 @@
 // bias and store d_seg bf16 values per segment.  For d_seg = 8 the weight box
 // still spans 16 rows (the next segment's rows, or TMA zero fill past the
 // end); those 8 extra output columns are computed and discarded.
+//
+// Pool variant (kPool): the same projection reads its cache tiles straight
+// from the chunk pool, each 128-row tile inside one selected chunk, and warp 6
+// stores every tile it has loaded into the assembled cache (TMA store from the
+// same shared-memory stage, or plain stores for a chunk's last, shorter tile).
+// The assembly of Sec. 4.1 then costs one read and one write of the cache
+// instead of two reads and a write.  Rows of a shorter tile past its chunk
+// end are loaded (the pool's next rows, or zero fill) but neither projected
+// into y nor stored.
+#include <type_traits>
 #include "cr_internal.h"
 #include "cr_ptx.cuh"
 
@@ -46,10 +56,37 @@ __global__ void fold_sigma_kernel(const uint16_t* __restrict__ w, const float* _
     }
 }
 
-template <int DH>
-__global__ void __launch_bounds__(192, 1)
+struct NoTiles {};
+
+// Rows of M tile mt: its first source row, first output row and row count.
+struct TileRows {
+    int64_t src;
+    int32_t dst;
+    int32_t rows;
+};
+__device__ __forceinline__ TileRows tile_rows(const NoTiles&, const SegParams& p, int mt) {
+    const int r0 = mt * 128;
+    return TileRows{r0, r0, min(128, p.M - r0)};
+}
+__device__ __forceinline__ TileRows tile_rows(const SegTiles& tm, const SegParams&, int mt) {
+    int lo = 0, hi = tm.n_seg - 1;   // last chunk whose first tile is <= mt
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (tm.tile_prefix[mid] <= mt)
+            lo = mid;
+        else
+            hi = mid - 1;
+    }
+    const int k = (mt - tm.tile_prefix[lo]) * 128;
+    return TileRows{tm.src_row[lo] + k, tm.dst_row[lo] + k, min(128, tm.len[lo] - k)};
+}
+
+
+template <int DH, bool kPool>
+__global__ void __launch_bounds__(224, 1)
     segproj_kernel(const __grid_constant__ CUtensorMap tmKV, const __grid_constant__ CUtensorMap tmW,
-                   const __grid_constant__ SegParams p) {
+                   const __grid_constant__ CUtensorMap tmOut, const __grid_constant__ SegParams p,
+                   const __grid_constant__ std::conditional_t<kPool, SegTiles, NoTiles> tiles) {
     using Cfg = SegCfg<DH>;
     constexpr int STAGES = Cfg::kStages;
     constexpr uint32_t IDESC = idesc_bf16(128, SP_N, false, false);
@@ -72,7 +109,7 @@ __global__ void __launch_bounds__(192, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&full[s], 1);
-            mbar_init(&empty[s], 1);
+            mbar_init(&empty[s], kPool ? 2 : 1);   // the MMA's commit (+ the tile store)
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(&tfull[s], 1);
@@ -101,7 +138,7 @@ __global__ void __launch_bounds__(192, 1)
         uint32_t stage = 0, phase = 0;
         bool ok = true;
         for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
-            const int m0 = (t % p.num_m) * 128;
+            const int src0 = static_cast<int>(tile_rows(tiles, p, t % p.num_m).src);
             const int s0 = (t / p.num_m) * SP_G;
             const int ns = min(SP_G, p.S - s0);
             for (int g = 0; g < ns; ++g) {
@@ -113,7 +150,7 @@ __global__ void __launch_bounds__(192, 1)
                     mbar_expect_tx(&full[stage], Cfg::kStageBytes);
 #pragma unroll
                     for (int b = 0; b < Cfg::kBoxes; ++b) {
-                        tma_load_2d(sa + b * 16384, &tmKV, &full[stage], seg * DH + b * 64, m0);
+                        tma_load_2d(sa + b * 16384, &tmKV, &full[stage], seg * DH + b * 64, src0);
                         tma_load_2d(sb + b * (SP_N * 128), &tmW, &full[stage], b * 64,
                                     seg * p.d_seg);
                     }
@@ -173,19 +210,99 @@ __global__ void __launch_bounds__(192, 1)
         if (elect_one()) mma_commit(drain);
         __syncwarp();
         mbar_wait_warp(drain, 0, wc, 213);
+    } else if (warp == 6) {
+        if constexpr (kPool) {
+            // tile store: a whole tile goes out by TMA from the stage it was
+            // loaded into, and the stage is released once the store has read
+            // it (two younger stores stay in flight: q0, q1 are the stages whose
+            // stores may still be reading, oldest first); a chunk's shorter
+            // last tile is copied row by row with plain stores
+            uint32_t stage = 0, phase = 0, q0 = 0, q1 = 0;
+            int npend = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+                const TileRows tr = tile_rows(tiles, p, t % p.num_m);
+                const int s0 = (t / p.num_m) * SP_G;
+                const int ns = min(SP_G, p.S - s0);
+                for (int g = 0; g < ns; ++g) {
+                    if (!(ok = mbar_wait_warp(&full[stage], phase, wc, 114))) break;
+                    const uint8_t* sa = smem + stage * Cfg::kStageBytes;
+                    const int col = (s0 + g) * DH;
+                    if (tr.rows == 128) {
+                        if (lane == 0) {
+                            fence_async_smem();
+#pragma unroll
+                            for (int b = 0; b < Cfg::kBoxes; ++b)
+                                tma_store_2d(&tmOut, sa + b * 16384, col + b * 64, tr.dst);
+                            tma_store_commit();
+                        }
+                        if (npend == 2) {
+                            // q0's store is done reading once at most two groups remain
+                            if (lane == 0) tma_store_wait_read<2>();
+                            __syncwarp();
+                            if (lane == 0) mbar_arrive(&empty[q0]);
+                            q0 = q1;
+                            q1 = stage;
+                        } else if (npend == 1) {
+                            q1 = stage;
+                            npend = 2;
+                        } else {
+                            q0 = stage;
+                            npend = 1;
+                        }
+                    } else {
+                        // release the held stages first: a held stage may be at most
+                        // two uses old, or the producer, which refills in ring order,
+                        // would wait for it while this warp waits for the producer
+                        if (npend > 0) {
+                            if (lane == 0) tma_store_wait_read<0>();
+                            __syncwarp();
+                            if (lane == 0) mbar_arrive(&empty[q0]);
+                            if (lane == 0 && npend > 1) mbar_arrive(&empty[q1]);
+                            npend = 0;
+                        }
+                        // 16-byte chunk c of row r sits at r*128 + ((c ^ (r & 7)) << 4)
+                        // in each 128B-swizzled box of 64 columns
+                        const int n16 = tr.rows * 8;
+                        for (int b = 0; b < Cfg::kBoxes; ++b) {
+                            for (int i = static_cast<int>(lane); i < n16; i += 32) {
+                                const int r = i >> 3, c = i & 7;
+                                const uint4 v = *reinterpret_cast<const uint4*>(
+                                    sa + b * 16384 + r * 128 + ((c ^ (r & 7)) << 4));
+                                *reinterpret_cast<uint4*>(p.kv_out + static_cast<int64_t>(tr.dst + r) * p.ld_out +
+                                                          col + b * 64 + c * 8) = v;
+                            }
+                        }
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&empty[stage]);
+                    }
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+            }
+            // every store has finished reading (and, before exit, writing)
+            if (lane == 0) tma_store_wait_read<0>();
+            __syncwarp();
+            if (lane == 0 && npend > 0) mbar_arrive(&empty[q0]);
+            if (lane == 0 && npend > 1) mbar_arrive(&empty[q1]);
+            if (lane == 0) tma_store_wait0();
+            __syncwarp();
+        }
     } else {
         const uint32_t quad = warp & 3u;
         const int r = static_cast<int>(quad * 32 + lane);
         const int ldy = p.S * p.d_seg;
         uint32_t acc = 0, acc_phase = 0;
         for (int t = blockIdx.x; t < total; t += gridDim.x) {
-            const int m0 = (t % p.num_m) * 128;
+            const TileRows tr = tile_rows(tiles, p, t % p.num_m);
             const int s0 = (t / p.num_m) * SP_G;
             const int ns = min(SP_G, p.S - s0);
             const bool ok = mbar_wait(&tfull[acc], acc_phase, wc, 311);
             if (!__all_sync(0xffffffffu, ok)) break;
             tc_fence_after();
-            const int row = m0 + r;
+            const int row = tr.dst + r;
             const uint32_t taddr = tmem_base + ((quad * 32u) << 16) + acc * 256;
             uint16_t* yrow = p.y + static_cast<int64_t>(row) * ldy;
             for (int g = 0; g < ns; ++g) {
@@ -195,7 +312,7 @@ __global__ void __launch_bounds__(192, 1)
                 tmem_wait_ld();
                 const int seg = s0 + g;
                 const float* bs = p.b_seg + seg * p.d_seg;
-                if (row < p.M) {
+                if (r < tr.rows) {
                     uint32_t w[8];
                     const int dm = p.d_seg - 1;   // d_seg is 8 or 16; columns >= d_seg are dropped
 #pragma unroll
@@ -222,17 +339,18 @@ __global__ void __launch_bounds__(192, 1)
     }
 }
 
-template <int DH>
-cr_status launch_dh(const CUtensorMap& tk, const CUtensorMap& tw, const SegParams& p,
-                    cudaStream_t st) {
+template <int DH, bool kPool, class Tiles>
+cr_status launch_dh(const CUtensorMap& tk, const CUtensorMap& tw, const CUtensorMap& to,
+                    const SegParams& p, const Tiles& tiles, cudaStream_t st) {
     using Cfg = SegCfg<DH>;
-    auto kern = segproj_kernel<DH>;
+    auto kern = segproj_kernel<DH, kPool>;
     static unsigned long long attr_done = 0;   // one per template instantiation
     const cr_status sa = ensure_smem_attr(kern, static_cast<int>(Cfg::kSmemBytes), &attr_done);
     if (sa != CR_OK) return sa;
     const int items = p.num_m * p.num_g;
     const int grid = items < num_sms() ? items : num_sms();
-    return launch_pdl(kern, dim3(grid), dim3(192), Cfg::kSmemBytes, st, tk, tw, p);
+    return launch_pdl(kern, dim3(grid), dim3(kPool ? 224 : 192), Cfg::kSmemBytes, st, tk, tw, to, p,
+                      tiles);
 }
 
 }  // namespace
@@ -262,7 +380,35 @@ cr_status launch_segproj(const uint16_t* kv, int64_t ld_kv, const uint16_t* wfol
                       static_cast<uint64_t>(p.S) * p.d_seg, head_dim * 2, 64, SP_N,
                       CU_TENSOR_MAP_SWIZZLE_128B))
         return CR_ERR_INVALID_ARG;
-    return head_dim == 128 ? launch_dh<128>(tk, tw, p, st) : launch_dh<64>(tk, tw, p, st);
+    const NoTiles none{};
+    return head_dim == 128 ? launch_dh<128, false>(tk, tw, tk, p, none, st)
+                           : launch_dh<64, false>(tk, tw, tk, p, none, st);
+}
+
+cr_status launch_segproj_pool(const uint16_t* kv_pool, int64_t n_pool_tokens, uint16_t* kv_out,
+                              const uint16_t* wfold, int head_dim, SegParams p,
+                              const SegTiles& tiles, cudaStream_t st) {
+    if (head_dim != 64 && head_dim != 128) return CR_ERR_UNSUPPORTED;
+    if (p.d_seg != 8 && p.d_seg != 16) return CR_ERR_UNSUPPORTED;
+    if (tiles.n_seg < 1 || tiles.n_seg > kMaxSegs || n_pool_tokens > INT32_MAX) return CR_ERR_INVALID_ARG;
+    p.num_m = tiles.tile_prefix[tiles.n_seg];
+    p.num_g = (p.S + SP_G - 1) / SP_G;
+    const uint64_t dkv = static_cast<uint64_t>(p.S) * head_dim;
+    p.kv_out = kv_out;
+    p.ld_out = static_cast<int64_t>(dkv);
+    CUtensorMap tk, tw, to;
+    if (!make_tmap_2d(&tk, kv_pool, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dkv, n_pool_tokens, dkv * 2, 64,
+                      128, CU_TENSOR_MAP_SWIZZLE_128B))
+        return CR_ERR_INVALID_ARG;
+    if (!make_tmap_2d(&tw, wfold, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, head_dim,
+                      static_cast<uint64_t>(p.S) * p.d_seg, head_dim * 2, 64, SP_N,
+                      CU_TENSOR_MAP_SWIZZLE_128B))
+        return CR_ERR_INVALID_ARG;
+    if (!make_tmap_2d(&to, kv_out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dkv, p.M, dkv * 2, 64, 128,
+                      CU_TENSOR_MAP_SWIZZLE_128B))
+        return CR_ERR_INVALID_ARG;
+    return head_dim == 128 ? launch_dh<128, true>(tk, tw, to, p, tiles, st)
+                           : launch_dh<64, true>(tk, tw, to, p, tiles, st);
 }
 
 }  // namespace cr

@@ -63,6 +63,16 @@ class RepairSession:
         cr.cr_compress_features(self.target, self.rep, self.weights, self.kv, self.emb, a.n_tokens,
                                 self.h0, self.rein, self.workspace, stream)
 
+    def assemble_compress(self, kv_pool: torch.Tensor, emb_pool: torch.Tensor, chunk_start,
+                          chunk_len, chunk_idx, cu_chunks, stream=None) -> Assembled:
+        """assemble + compress as one call: the segment projection reads the pool and
+        writes the assembled cache as it goes (same results, one cache read fewer)."""
+        n, cu = cr.cr_assemble_compress(self.target, self.rep, self.weights, kv_pool, emb_pool,
+                                        chunk_start, chunk_len, chunk_idx, cu_chunks, self.kv,
+                                        self.emb, self.chunk_id, self.chunk_end, self.pos,
+                                        self.cu_seqlens, self.h0, self.rein, self.workspace, stream)
+        return Assembled(n, cu)
+
     def forward(self, a: Assembled, stream=None, mask_mode="block_causal"):
         """The Repair Blocks and LN_f; mask_mode picks the attention mask (the method's
         block-causal mask, or an App. F ablation: token_causal, bidirectional, block_diagonal)."""
@@ -107,8 +117,8 @@ class RepairSession:
                keep_first_chunk=False) -> Assembled:
         """Assemble, compress, run the blocks and apply the residual; kv holds the result.
         The keyword options select the App. F mask and output variants (defaults: the method)."""
-        a = self.assemble(kv_pool, emb_pool, chunk_start, chunk_len, chunk_idx, cu_chunks, stream)
-        self.compress(a, stream)
+        a = self.assemble_compress(kv_pool, emb_pool, chunk_start, chunk_len, chunk_idx, cu_chunks,
+                                   stream)
         self.forward(a, stream, mask_mode=mask_mode)
         self.apply(a, inv_freq_target, rope_mode, stream, component=component, offset=offset,
                    keep_first_chunk=keep_first_chunk)

@@ -174,3 +174,40 @@ def test_paged_residual_rejects_bad_inputs_on_host(L):
     assert call(f32) == cr.CR_ERR_UNSUPPORTED                 # bf16 caches only
     narrow = cr.target_dims(4, 1, 128, 512, "bf16")           # H_kv d_h = 128: not a multiple of 256
     assert call(narrow) == cr.CR_ERR_UNSUPPORTED
+
+
+def test_fused_front_rejects_bad_inputs_on_host(L):
+    """cr_assemble_compress checks the chunk map, weights and workspace before any launch."""
+    c, (t, r) = _dims()
+    w = cr.cr_weights()
+    for f in ("w_seg", "b_seg", "w_map", "b_map", "w_tok", "b_tok", "w_fuse", "b_fuse", "w_rein",
+              "b_rein", "sigma_stale"):
+        setattr(w, f, FAKE)
+    ws = cr.cr_workspace_bytes(t, r, 1000)
+
+    def call(chunk_idx, cu, chunk_len=(10, 20, 30), n_pool=60, max_tokens=1000, ptr=FAKE,
+             weights=w, ws_bytes=ws):
+        cs = np.array([0, 10, 30], np.int64)
+        cl = np.array(chunk_len, np.int32)
+        ci = np.array(chunk_idx, np.int32)
+        cc = np.array(cu, np.int32)
+        cuh = np.zeros(len(cc), np.int32)
+        return L.cr_assemble_compress(ctypes.byref(t), ctypes.byref(r), ctypes.byref(weights), ptr,
+                                      ptr, n_pool, cs.ctypes.data, cl.ctypes.data, len(cl),
+                                      ci.ctypes.data, cc.ctypes.data, len(cc) - 1, ptr, ptr,
+                                      max_tokens, ptr, ptr, ptr, ptr, cuh.ctypes.data, FAKE, FAKE,
+                                      FAKE, ws_bytes, None)
+
+    assert call([0, 5], [0, 2]) == cr.CR_ERR_INVALID_ARG          # chunk id out of range
+    assert call([0, 1], [0, 0, 2]) == cr.CR_ERR_INVALID_ARG       # empty request
+    assert call([0, 2], [0, 2], n_pool=50) == cr.CR_ERR_INVALID_ARG   # chunk past the pool
+    assert call([0, 1], [0, 2], chunk_len=(10, 0, 30)) == cr.CR_ERR_INVALID_ARG
+    assert call([2, 1], [0, 2], max_tokens=40) == cr.CR_ERR_INVALID_ARG
+    assert call([0, 1], [0, 2], ptr=FAKE + 8) == cr.CR_ERR_INVALID_ARG   # misaligned
+    assert call([0, 1], [0, 2], weights=cr.cr_weights()) == cr.CR_ERR_INVALID_ARG   # no weights
+    assert call([0, 1], [0, 2], ws_bytes=ws - 256) == cr.CR_ERR_INVALID_ARG    # workspace short
+    bad = cr.repairer_dims(12, 128, 256, 2, 4, 1024)    # d_seg 12: unsupported
+    assert L.cr_assemble_compress(ctypes.byref(t), ctypes.byref(bad), ctypes.byref(w), *([FAKE] * 2),
+                                  60, None, None, 3, None, None, 1, *([FAKE] * 2), 100,
+                                  *([FAKE] * 4), None, FAKE, FAKE, FAKE, ws, None) == \
+        cr.CR_ERR_UNSUPPORTED
