@@ -104,6 +104,32 @@ __device__ __forceinline__ void gelu2(float& a, float& b) {
     b = b < 0.0f ? hb : b - hb;
 }
 
+// This row's (cos, sin) for every pair index q of the repairer RoPE: from the
+// angle-major table (entry q * M + row: a warp's 32 rows read 256 contiguous
+// bytes per q), or computed in place when no table is given.
+template <int NP>
+__device__ __forceinline__ void rope_angles(const GemmParams& p, int row, float (&cs)[NP],
+                                            float (&sn)[NP]) {
+    const bool in = row < p.M;
+    const int half = p.rope_dim / 2;
+    if (p.rope_table) {
+        const float2* tb = p.rope_table + (in ? row : 0);
+#pragma unroll
+        for (int q = 0; q < NP; ++q) {
+            if (q < half) {
+                const float2 v = __ldg(tb + static_cast<int64_t>(q) * p.M);
+                cs[q] = v.x;
+                sn[q] = v.y;
+            }
+        }
+    } else {
+        const float pr = in ? static_cast<float>(__ldg(p.pos + row)) : 0.0f;
+#pragma unroll
+        for (int q = 0; q < NP; ++q)
+            if (q < half) sincos_prod(pr, p.inv_freq[q], &sn[q], &cs[q]);
+    }
+}
+
 // 16 consecutive bf16 of a [128 x (64*k)] tile stored as 128B-swizzled boxes
 // of 64 columns; col multiple of 16.  Byte offsets of its two 16-byte chunks.
 __device__ __forceinline__ void swz_offsets_bf16(int row, int col, uint32_t* o0, uint32_t* o1) {
@@ -542,6 +568,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         for (int t = cta0; t < total && ok; t += ncta, ++i) {
             const int m0 = (t % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
             const int n0 = tile_n0<BN, Cfg::kKV>(p, t);
+            // QKV: the rotation angles depend on (row, pair index) only: cos/sin
+            // for every head of the tile, fetched while the MMAs still run
+            constexpr int NP = (EPI == EPI_QKV_ROPE) ? 32 : 1;
+            float cs[NP], sn[NP];
+            if constexpr (EPI == EPI_QKV_ROPE) rope_angles<NP>(p, m0 + r, cs, sn);
             ok = mbar_wait(&tfull[acc], acc_phase, wc, 301);
             // in-place epilogues wait box by box below
             if (epi_load && !Cfg::kInPlace) ok = ok && mbar_wait(epi_full, static_cast<uint32_t>(i) & 1u, wc, 302);
@@ -692,32 +723,6 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 // store-only epilogues: one 128 B-wide box of columns at a time,
                 // into alternating staging buffers
                 constexpr int PC = Cfg::kBoxCols;
-                // QKV: the rotation angles depend on (row, pair index) only, so
-                // cos/sin are computed once per tile for every head in it
-                constexpr int NP = (EPI == EPI_QKV_ROPE) ? 32 : 1;
-                float cs[NP], sn[NP];
-                if constexpr (EPI == EPI_QKV_ROPE) {
-                    if (p.rope_table) {
-                        // precomputed per forward: this row's (cos, sin) pairs
-                        const float4* tr = reinterpret_cast<const float4*>(
-                            p.rope_table + static_cast<int64_t>(row_ok ? row : 0) * (p.rope_dim / 2));
-#pragma unroll
-                        for (int q = 0; q < NP; q += 2) {
-                            if (q < p.rope_dim / 2) {
-                                const float4 v = __ldg(tr + q / 2);
-                                cs[q] = v.x;
-                                sn[q] = v.y;
-                                cs[q + 1] = v.z;
-                                sn[q + 1] = v.w;
-                            }
-                        }
-                    } else {
-                        const float pr = row_ok ? static_cast<float>(__ldg(p.pos + row)) : 0.0f;
-#pragma unroll
-                        for (int q = 0; q < NP; ++q)
-                            if (q < p.rope_dim / 2) sincos_prod(pr, p.inv_freq[q], &sn[q], &cs[q]);
-                    }
-                }
                 // boxes alternate between the groups; each group cycles its own
                 // kGroupBufs staging buffers (pk counts this group's boxes)
                 for (int k = eg; k < Cfg::kBoxes && ok; k += 2, ++pk) {

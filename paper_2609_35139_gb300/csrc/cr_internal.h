@@ -71,7 +71,7 @@ struct GemmParams {
     int32_t rope_on;         // KV: rotate K segments
     int32_t n_kv_heads;      // KV: segment s is K iff (s / n_kv_heads) is even
     const float* sigma;      // KV: sigma_delta [N]
-    const float2* rope_table;  // QKV: (cos, sin) [M, rope_dim / 2], or null (computed inline)
+    const float2* rope_table;  // QKV: (cos, sin) [rope_dim / 2, M] angle-major, or null (computed inline)
     const int64_t* slot;     // KV_PAGED: destination slot of each token, < 0 = not written
     uint16_t* paged;         // KV_PAGED: [N / seg_width][num_slots][seg_width] bf16
     int64_t num_slots;       // KV_PAGED: slots per (layer, K|V) plane

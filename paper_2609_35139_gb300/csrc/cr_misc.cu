@@ -154,16 +154,17 @@ struct InvFreq {
     float f[64];
 };
 
-// (cos, sin) of pos[t] * inv_freq[i] for every token and pair index, the angle's
+// (cos, sin) of pos[t] * inv_freq[q] for every token and pair index, the angle's
 // product rounding folded back in (same arithmetic as the in-epilogue path).
+// Angle-major: entry q * n + t, so that the rows of a tile read it coalesced.
 __global__ void rope_table_kernel(const int32_t* __restrict__ pos, int64_t n, int half,
                                   const __grid_constant__ InvFreq f, float2* __restrict__ table) {
     pdl_launch_dependents();
     pdl_wait();
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n * half;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const int64_t t = i / half;
-        const int q = static_cast<int>(i - t * half);
+        const int q = static_cast<int>(i / n);
+        const int64_t t = i - static_cast<int64_t>(q) * n;
         float s, c;
         sincos_prod(static_cast<float>(__ldg(pos + t)), f.f[q], &s, &c);
         table[i] = make_float2(c, s);

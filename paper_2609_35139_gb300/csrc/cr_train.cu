@@ -245,7 +245,7 @@ __global__ void __launch_bounds__(256)
 // The repairer RoPE rotated q and k of every head by angle p_t f_i (pairs
 // (i, i + d/2)); its transpose rotates the gradients back:
 //   (a, b) -> (a cos + b sin, b cos - a sin).  dqkv [N, 3 d_b] fp32, Q and K
-// columns [0, 2 d_b); table [N, d/2] (cos, sin) of the forward.
+// columns [0, 2 d_b); table [d/2, N] (cos, sin) of the forward, angle-major.
 __global__ void __launch_bounds__(256)
     rope_backward_kernel(float* __restrict__ dqkv, const float2* __restrict__ table, int64_t N, int db,
                          int hd) {
@@ -260,7 +260,7 @@ __global__ void __launch_bounds__(256)
         const int64_t rem = i - t * pairs_per_row;
         const int64_t h = rem / half;
         const int j = static_cast<int>(rem - h * half);
-        const float2 cs = table[t * half + j];
+        const float2 cs = table[static_cast<int64_t>(j) * N + t];
         float* base = dqkv + t * 3 * db + h * hd;
         const float a = base[j], b = base[j + half];
         base[j] = a * cs.x + b * cs.y;
