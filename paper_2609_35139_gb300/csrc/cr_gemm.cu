@@ -79,29 +79,26 @@ struct GemmCfg {
     static constexpr uint32_t kTmemCols = (2 * BN <= 256) ? 256u : 512u;
 };
 
-// GELU(x) = x/2 (1 + erf(x / sqrt 2)) for a pair of values, branch-free.
-// With z = |x| / sqrt 2 and t = 1 / (1 + z/2), erfc(z) = t exp(f(t) - z^2) where
-// f is a degree-9 polynomial fitted by gelu_erfc_fit.py in this directory
-// (relative error of erfc <= 1.1e-7 in float64; the form of the Chebyshev erfc
-// of Numerical Recipes, Sec. 6.2).  Then GELU(x) = x/2 erfc(z) for x < 0 and
-// x - x/2 erfc(z) otherwise.  One reciprocal and one exponential on the
-// special-function unit and nine packed FMAs per pair.
-__device__ constexpr float kErfcC[10] = {-1.265512225e+00f, 1.000023680e+00f, 3.740919597e-01f,
-                              9.678418949e-02f,  -1.862880617e-01f, 2.788680845e-01f,
-                              -1.135204000e+00f, 1.488515889e+00f,  -8.221522344e-01f,
-                              1.708727777e-01f};
+// GELU(x) = x Phi(x) for a pair of values, branch-free.  Phi is written as a
+// logistic function of its log2-odds: Phi(x) = 1 / (1 + 2^(x H(x^2))), with H a
+// degree-6 polynomial fitted by gelu_sigmoid_fit.py in this directory (GELU's
+// absolute error <= 8.3e-8 on [-12, 12] in float64; beyond the fitted range
+// |x H| >= 34, so Phi is 0 or 1 to within 2^-34 there as the exact Phi is).
+// Per pair: a packed square, six packed FMAs, a packed multiply, two 2^y, a
+// packed add, two reciprocals and a packed multiply.
+__device__ constexpr float kGeluH[7] = {-2.302209146e+00f, -1.048354083e-01f, 9.409242776e-05f,
+                                        1.596513719e-04f, -1.146683675e-05f,
+                                        3.847686963e-07f, -5.180393528e-09f};
 __device__ __forceinline__ void gelu2(float& a, float& b) {
-    const float za = fabsf(a) * 0.70710678118654752f, zb = fabsf(b) * 0.70710678118654752f;
-    const float ta = rcp_approx(fmaf(0.5f, za, 1.0f)), tb = rcp_approx(fmaf(0.5f, zb, 1.0f));
-    float fa = kErfcC[9], fb = kErfcC[9];
+    float sa, sb;
+    fmul2(sa, sb, a, b, a, b);
+    float ha = kGeluH[6], hb = kGeluH[6];
 #pragma unroll
-    for (int i = 8; i >= 0; --i) ffma2(fa, fb, fa, fb, ta, tb, kErfcC[i], kErfcC[i]);
-    // exp(f - z^2) = 2^((f - z^2) log2 e)
-    const float ea = ex2(fmaf(-za, za, fa) * 1.4426950408889634f);
-    const float eb = ex2(fmaf(-zb, zb, fb) * 1.4426950408889634f);
-    const float ha = 0.5f * a * (ta * ea), hb = 0.5f * b * (tb * eb);
-    a = a < 0.0f ? ha : a - ha;
-    b = b < 0.0f ? hb : b - hb;
+    for (int i = 5; i >= 0; --i) ffma2(ha, hb, ha, hb, sa, sb, kGeluH[i], kGeluH[i]);
+    fmul2(ha, hb, ha, hb, a, b);                        // -log2 odds of Phi
+    float da, db;
+    fadd2(da, db, ex2(ha), ex2(hb), 1.0f, 1.0f);        // 1 / Phi
+    fmul2(a, b, a, b, rcp_approx(da), rcp_approx(db));
 }
 
 // This row's (cos, sin) for every pair index q of the repairer RoPE: from the
