@@ -503,16 +503,23 @@ def run_e2e(case, sess, kvp_h, embp_h, args, world):
     run(args.warmup)
     torch.cuda.synchronize()
     stream = torch.cuda.current_stream()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    run(args.steps)
-    e1.record(stream)
-    torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1) / args.steps
+    # three timed batches of K requests, the median reported: the host link is
+    # shared with the machine's other GPUs and one batch can catch a burst of
+    # their traffic
+    batches = []
+    for _ in range(3):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        run(args.steps)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        batches.append(e0.elapsed_time(e1) / args.steps)
+    ms = statistics.median(batches)
     es = kv_h.element_size()
     return {"value": world * N / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
             "h2d_bytes_per_step": int(N * (kv_h.shape[1] + emb_h.shape[1]) * es),
             "d2h_bytes_per_step": int(N * kv_h.shape[1] * es),
+            "batches_ms_per_step": batches,
             "path": "RepairPipeline: pinned host chunks -> device staging (H2D stream) -> four "
                     "C-ABI calls (compute stream) -> pinned host repaired cache (D2H stream); "
                     "two slots, transfers overlapped with the neighbouring requests' repairs"}

@@ -2,6 +2,7 @@
 //   gather_kernel     stale-cache assembly (Sec. 4.1, "Chunk-cache
 //                     preparation": canonical chunk caches concatenated in
 //                     document order; a pure copy, K is not rotated)
+//   gather_emb_kernel the same for the embeddings and chunk map alone
 //   layernorm_kernel  LayerNorm of the residual stream (optionally adding the
 //                     block's reinjection P_b(s) first, Sec. 4.1 eq. for h^b)
 //   to_bf16_kernel    fp32 cache/embedding -> bf16 operands for the tensor cores
@@ -62,6 +63,59 @@ __global__ void __launch_bounds__(512) gather_kernel(const __grid_constant__ Gat
     }
     if (blockIdx.x == 0 && static_cast<int>(threadIdx.x) <= p.n_req)
         p.cu_seqlens[threadIdx.x] = p.cu_seqlens_host[threadIdx.x];
+}
+
+// The same assembly without the cache rows (they go with the segment
+// projection, which reads them from the pool): embedding rows and the chunk
+// map, one warp per output row, eight 16-byte loads in flight per lane before
+// the stores.
+__global__ void __launch_bounds__(256) gather_emb_kernel(const __grid_constant__ GatherParams p) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int wpb = static_cast<int>(blockDim.x >> 5);
+    const int lane = static_cast<int>(threadIdx.x & 31);
+    for (int64_t t = static_cast<int64_t>(blockIdx.x) * wpb + (threadIdx.x >> 5); t < p.n_tokens;
+         t += static_cast<int64_t>(gridDim.x) * wpb) {
+        int lo = 0, hi = p.n_seg - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (p.seg[mid].dst_row <= t)
+                lo = mid;
+            else
+                hi = mid - 1;
+        }
+        const GatherSeg& sg = p.seg[lo];
+        const int64_t off = t - sg.dst_row;
+        const int64_t src = sg.src_row + off;
+        if (off < 0 || off >= sg.len || src < 0 || src >= p.n_pool_tokens) {
+            if (lane == 0) report(p.status, CR_DEV_INDEX, 2);
+            continue;
+        }
+        if (lane == 0) {
+            p.chunk_id[t] = sg.chunk_local;
+            p.pos[t] = static_cast<int32_t>(sg.local_start + off);
+            p.chunk_end[t] = sg.local_start + sg.len;
+        }
+        const uint4* s = reinterpret_cast<const uint4*>(p.emb_pool + src * p.emb_row_bytes);
+        uint4* d = reinterpret_cast<uint4*>(p.emb_out + t * p.emb_row_bytes);
+        const int64_t nv = p.emb_row_bytes >> 4;
+        for (int64_t base = lane; base < nv; base += 8 * 32) {
+            uint4 v[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int64_t i = base + u * 32;
+                if (i < nv) v[u] = __ldcs(s + i);
+            }
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int64_t i = base + u * 32;
+                if (i < nv) d[i] = v[u];
+            }
+        }
+    }
+    if (blockIdx.x == 0)
+        for (int i = static_cast<int>(threadIdx.x); i <= p.n_req; i += static_cast<int>(blockDim.x))
+            p.cu_seqlens[i] = p.cu_seqlens_host[i];
 }
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
@@ -187,6 +241,11 @@ cr_status launch_rope_table(const int32_t* pos, int64_t n, int half_dim, const f
 
 cr_status launch_gather(const GatherParams& p, cudaStream_t st) {
     if (p.n_tokens <= 0) return CR_OK;
+    if (p.kv_row_bytes == 0) {
+        // no cache rows: every row's embedding copy in flight at once (8 rows per block)
+        const int64_t grid = (p.n_tokens + 7) / 8;
+        return launch_pdl(gather_emb_kernel, dim3(static_cast<unsigned>(grid)), dim3(256), 0, st, p);
+    }
     int64_t grid = static_cast<int64_t>(num_sms()) * 4;
     if (grid > p.n_tokens) grid = p.n_tokens;
     return launch_pdl(gather_kernel, dim3(static_cast<unsigned>(grid)), dim3(512), 0, st, p);

@@ -6,7 +6,7 @@ The fused call must give every output of cr_assemble_stale + cr_compress_feature
 bit for bit: the assembled cache (written by the projection kernel's tile
 stores), embeddings, chunk map, h^0 and the reinjection terms.  Chunk layouts
 cover 128-row tiles with ragged tails, a 1-token chunk, a chunk that ends the
-pool (its last tile reads past the pool, zero fill), several requests, 64- and
+pool (its last tile reads past the pool, zero fill), up to 256 requests, 64- and
 128-dim target heads, d_seg 8 and 16, and the fp32 cache (two-call path).
 """
 from dataclasses import replace
@@ -32,6 +32,8 @@ def _case(name):
         return F.make_case(rc)
     if name == "small_tail":   # the request ends with the pool's last (33-token) chunk
         return F.make_case("small_multi", requests=[[7], [4, 7, 3]])
+    if name == "small_256req":   # the most requests one call takes
+        return F.make_case("small_multi", requests=[[i % 8, (3 * i + 1) % 8] for i in range(256)])
     return F.make_case(name)
 
 
@@ -41,8 +43,8 @@ def _outputs(s, n, n_req):
                 cu=s.cu_seqlens[:n_req + 1].clone(), h0=s.h0[:n].clone(), rein=s.rein[:n].clone())
 
 
-@pytest.mark.parametrize("name", ["small", "small_multi", "small_tail", "small_dh64", "tiny",
-                                  "qwen3b", "qwen7b", "llama8b"])
+@pytest.mark.parametrize("name", ["small", "small_multi", "small_tail", "small_dh64", "small_256req",
+                                  "tiny", "qwen3b", "qwen7b", "llama8b"])
 def test_fused_matches_two_calls(name):
     case = _case(name)
     t, r = dims_from(case.target, case.repairer)
