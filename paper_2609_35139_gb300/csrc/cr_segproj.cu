@@ -41,18 +41,31 @@ struct SegCfg {
     static constexpr uint32_t kSmemBytes = 1024 + kStages * kStageBytes + 256;
 };
 
+// W_seg / sigma_stale per input coordinate, rounded to bf16; eight weights
+// (16 bytes) per thread.  n and d_h are multiples of 8.
 __global__ void fold_sigma_kernel(const uint16_t* __restrict__ w, const float* __restrict__ sigma,
                                   int64_t n, int d_seg, int dh, uint16_t* __restrict__ out) {
     pdl_launch_dependents();
     pdl_wait();
-    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
-         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t n8 = n >> 3;
+    for (int64_t i8 = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i8 < n8;
+         i8 += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t i = i8 << 3;
         const int64_t d = i % dh;
         const int64_t s = i / (static_cast<int64_t>(d_seg) * dh);
-        const float wv = __uint_as_float(static_cast<uint32_t>(w[i]) << 16);
-        const float v = wv / sigma[s * dh + d];
-        const __nv_bfloat16 b = __float2bfloat16_rn(v);
-        out[i] = *reinterpret_cast<const uint16_t*>(&b);
+        const uint4 wv = __ldg(reinterpret_cast<const uint4*>(w) + i8);
+        const float4* sp = reinterpret_cast<const float4*>(sigma + s * dh + d);
+        const float4 s0 = __ldg(sp), s1 = __ldg(sp + 1);
+        const uint32_t in[4] = {wv.x, wv.y, wv.z, wv.w};
+        const float sg[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+        uint32_t o[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float lo = __uint_as_float(in[k] << 16) / sg[2 * k];
+            const float hi = __uint_as_float(in[k] & 0xFFFF0000u) / sg[2 * k + 1];
+            o[k] = pack_bf16x2(lo, hi);
+        }
+        reinterpret_cast<uint4*>(out)[i8] = make_uint4(o[0], o[1], o[2], o[3]);
     }
 }
 
@@ -359,7 +372,7 @@ cr_status launch_fold_sigma(const uint16_t* w_seg, const float* sigma, int S, in
                             int head_dim, uint16_t* wfold, cudaStream_t st) {
     const int64_t n = static_cast<int64_t>(S) * d_seg * head_dim;
     const int threads = 256;
-    int64_t blocks = (n + threads - 1) / threads;
+    int64_t blocks = (n / 8 + threads - 1) / threads;
     if (blocks > 4 * 1024) blocks = 4 * 1024;
     return launch_pdl(fold_sigma_kernel, dim3(static_cast<unsigned>(blocks)), dim3(threads), 0, st,
                       w_seg, sigma, n, d_seg, head_dim, wfold);
