@@ -2,8 +2,9 @@
 """Benchmark of the GB300 repair path: repaired document tokens/s and p50 repair
 latency per request, with the roofline fraction of the dominant kernel.
 
-One step = one request through all four C-ABI calls (assemble, compress,
-forward, apply) on one stream, captured once into a CUDA graph and replayed.
+One step = one request through RepairSession.repair on one stream: the C-ABI
+calls cr_assemble_compress (assembly fused with the encoder), cr_repair_forward
+and cr_apply_residual, captured once into a CUDA graph and replayed.
 Default workload: the Llama-3.1-8B-shaped cache (32 layers, 8 KV heads,
 head_dim 128, d_model 4096) with the d_c 512 / d_b 1024 / 6-block repairer,
 one request of 10 chunks x 512 tokens.  Inputs are seeded and synthetic; the
@@ -381,8 +382,11 @@ def run_ours(args):
         "head_tensor_frac": head_flops / (head_ms * 1e-3) / 1e12 / tf_sus,
         "head_ms": head_ms,
     }
+    # front: gather (embeddings + chunk map), sigma fold, projection, four encoder
+    # GEMMs (fp32 caches: the two-call path with its two bf16 conversions);
+    # forward: RoPE table, 7 kernels per block, final LayerNorm; head
     launches_per_step = 1 + (2 + 4 + (2 if tg.cache_dtype == "f32" else 0) - (1 if rp.n_blocks == 0 else 0)) \
-        + 7 * rp.n_blocks + 1 + 1
+        + (1 if rp.n_blocks > 0 else 0) + 7 * rp.n_blocks + 1 + 1
     launches_per_step += 1 if (args.mask == "block_diagonal" and rp.n_blocks > 0) else 0
     launches_per_step += 1 if (args.rope and args.component == "v") else 0
     cpu = None
@@ -520,8 +524,9 @@ def run_e2e(case, sess, kvp_h, embp_h, args, world):
             "h2d_bytes_per_step": int(N * (kv_h.shape[1] + emb_h.shape[1]) * es),
             "d2h_bytes_per_step": int(N * kv_h.shape[1] * es),
             "batches_ms_per_step": batches,
-            "path": "RepairPipeline: pinned host chunks -> device staging (H2D stream) -> four "
-                    "C-ABI calls (compute stream) -> pinned host repaired cache (D2H stream); "
+            "path": "RepairPipeline: pinned host chunks -> device staging (H2D stream) -> three "
+                    "C-ABI calls (compute stream: fused assembly + encoder, repair blocks, head) "
+                    "-> pinned host repaired cache (D2H stream); "
                     "two slots, transfers overlapped with the neighbouring requests' repairs"}
 
 
