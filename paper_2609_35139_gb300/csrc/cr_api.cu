@@ -1336,6 +1336,10 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
         return launch_colsum(a, bf16, N, cols, lda, out, false, CS, CCNT, st);
     };
     auto to16 = [&](const float* a, int64_t n, uint16_t* out) { return launch_to_bf16(a, n, out, st); };
+    // a bias gradient and the bf16 copy of the same fp32 signal, in one pass
+    auto colsum16 = [&](const float* a, int64_t cols, uint16_t* a16, float* out) {
+        return launch_colsum_bf16(a, N, cols, a16, out, CS, CCNT, st);
+    };
 #define CR_TRY(x)                   \
     do {                            \
         if ((s = (x)) != CR_OK) return s; \
@@ -1357,9 +1361,8 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
         const uint16_t* o = reinterpret_cast<const uint16_t*>(blk(b, L.o));
         const uint16_t* g = reinterpret_cast<const uint16_t*>(blk(b, L.g));
         // h = x_mid + W_fc2 g + b_fc2
-        CR_TRY(to16(DH, N * db, SIG));
+        CR_TRY(colsum16(DH, db, SIG, gk(bk(b, BFC2))));
         CR_TRY(gemm_rm(hb, true, false, db, hid, N, 1.0f, SIG, BF, db, g, BF, hid, 0.0f, gk(bk(b, WFC2)), F32, hid));
-        CR_TRY(colsum(DH, false, db, db, gk(bk(b, BFC2))));
         CR_TRY(gemm_rm(hb, false, false, N, hid, db, 1.0f, SIG, BF, db, pb(bk(b, WFC2)), BF, hid, 0.0f, DTMP, F32,
                        hid));
         // g = GELU(pre), pre = W_fc1 u2 + b_fc1 (recomputed in fp32)
@@ -1370,9 +1373,8 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
         gp.ldo = hid;
         CR_TRY(launch_gemm(u2, db, pb(bk(b, WFC1)), N, hid, db, EPI_F32, gp, nullptr, 0, st));
         CR_TRY(launch_gelu_backward(DTMP, PRE, N * hid, st));
-        CR_TRY(to16(DTMP, N * hid, SIG));
+        CR_TRY(colsum16(DTMP, hid, SIG, gk(bk(b, BFC1))));
         CR_TRY(gemm_rm(hb, true, false, hid, db, N, 1.0f, SIG, BF, hid, u2, BF, db, 0.0f, gk(bk(b, WFC1)), F32, db));
-        CR_TRY(colsum(DTMP, false, hid, hid, gk(bk(b, BFC1))));
         CR_TRY(gemm_rm(hb, false, false, N, db, hid, 1.0f, SIG, BF, hid, pb(bk(b, WFC1)), BF, db, 0.0f, DU, F32,
                        db));
         // u2 = LN2(x_mid): dx_mid = dh + LN2 backward
@@ -1380,9 +1382,8 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
         CR_TRY(colsum(GPROD, false, db, db, gk(bk(b, LN2G))));
         CR_TRY(colsum(DU, false, db, db, gk(bk(b, LN2B))));
         // x_mid = x_in + W_o a + b_o
-        CR_TRY(to16(DXM, N * db, SIG));
+        CR_TRY(colsum16(DXM, db, SIG, gk(bk(b, BO))));
         CR_TRY(gemm_rm(hb, true, false, db, db, N, 1.0f, SIG, BF, db, o, BF, db, 0.0f, gk(bk(b, WO)), F32, db));
-        CR_TRY(colsum(DXM, false, db, db, gk(bk(b, BO))));
         CR_TRY(gemm_rm(hb, false, false, N, db, db, 1.0f, SIG, BF, db, pb(bk(b, WO)), BF, db, 0.0f, DA, F32, db));
         // attention: the fused backward (P recomputed from the forward's log-sum-exp,
         // dQ, dK, dV into dqkv), dO in bf16 for its MMAs
@@ -1392,27 +1393,24 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
         CR_TRY(launch_attention_backward(qkv, SIG, DA, o, N, static_cast<int>(hd), *bp, DVEC, st));
         CR_TRY(launch_rope_backward(DQKV, rope, N, static_cast<int>(db), static_cast<int>(hd), st));
         // qkv = W_qkv u1 + b_qkv;  u1 = LN1(x_in): dx_in = dx_mid + LN1 backward
-        CR_TRY(to16(DQKV, N * 3 * db, SIG));
+        CR_TRY(colsum16(DQKV, 3 * db, SIG, gk(bk(b, BQKV))));
         CR_TRY(gemm_rm(hb, true, false, 3 * db, db, N, 1.0f, SIG, BF, 3 * db, u1, BF, db, 0.0f, gk(bk(b, WQKV)),
                        F32, db));
-        CR_TRY(colsum(DQKV, false, 3 * db, 3 * db, gk(bk(b, BQKV))));
         CR_TRY(gemm_rm(hb, false, false, N, db, 3 * db, 1.0f, SIG, BF, 3 * db, pb(bk(b, WQKV)), BF, db, 0.0f, DU,
                        F32, db));
         CR_TRY(launch_ln_backward(x_in, pf(bk(b, LN1G)), DU, DXM, eps, N, static_cast<int>(db), DH, GPROD, st));
         CR_TRY(colsum(GPROD, false, db, db, gk(bk(b, LN1G))));
         CR_TRY(colsum(DU, false, db, db, gk(bk(b, LN1B))));
         // x_in = h^{b-1} + W_rein,b s + b_rein,b: ds += dx_in W_rein,b
-        CR_TRY(to16(DH, N * db, SIG));
+        CR_TRY(colsum16(DH, db, SIG, gk(B_REIN) + b * db));
         CR_TRY(gemm_rm(hb, true, false, db, dc, N, 1.0f, SIG, BF, db, se, BF, 2 * dc, 0.0f, gk(W_REIN) + b * db * dc,
                        F32, dc));
-        CR_TRY(colsum(DH, false, db, db, gk(B_REIN) + b * db));
         CR_TRY(gemm_rm(hb, false, false, N, dc, db, 1.0f, SIG, BF, db, pb(W_REIN) + b * db * dc, BF, dc, 1.0f, DSE,
                        F32, 2 * dc));
     }
     // h0 = W_fuse [s; e] + b_fuse
-    CR_TRY(to16(DH, N * db, SIG));
+    CR_TRY(colsum16(DH, db, SIG, gk(B_FUSE)));
     CR_TRY(gemm_rm(hb, true, false, db, 2 * dc, N, 1.0f, SIG, BF, db, se, BF, 2 * dc, 0.0f, gk(W_FUSE), F32, 2 * dc));
-    CR_TRY(colsum(DH, false, db, db, gk(B_FUSE)));
     CR_TRY(gemm_rm(hb, false, false, N, 2 * dc, db, 1.0f, SIG, BF, db, pb(W_FUSE), BF, 2 * dc, 1.0f, DSE, F32,
                    2 * dc));
     // e = W_tok emb + b_tok;  s = W_map y + b_map
@@ -1425,11 +1423,10 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
     CR_TRY(colsum(DSE, false, dc, 2 * dc, gk(B_MAP)));
     CR_TRY(gemm_rm(hb, false, false, N, Sd, dc, 1.0f, SIG, BF, 2 * dc, pb(W_MAP), BF, Sd, 0.0f, DY, F32, Sd));
     // y_{t,s} = (W_seg,s / sigma_stale) kv_{t,s} + b_seg,s: per segment dy^T kv, then / sigma_stale
-    CR_TRY(to16(DY, N * Sd, SIG));
+    CR_TRY(colsum16(DY, Sd, SIG, gk(B_SEG)));
     CR_TRY(gemm_rm(hb, true, false, d.dseg, d.dh, N, 1.0f, SIG, BF, Sd, kv_stale, BF, D, 0.0f, gk(W_SEG), F32, d.dh,
                    d.S, d.dseg, d.dh, d.dseg * d.dh));
     CR_TRY(launch_scale_seg_grad(gk(W_SEG), d.S, d.dseg, d.dh, sigma_stale, st));
-    CR_TRY(colsum(DY, false, Sd, Sd, gk(B_SEG)));
 
     // ---- clipping and AdamW (App. A)
     AdamWParams ah{};

@@ -248,6 +248,10 @@ cr_status launch_loss(const float* r, int64_t N, int64_t D, const LossParams& p,
                       float* loss_out, double* per_req, cudaStream_t st);
 size_t colsum_scratch_floats(int64_t rows, int64_t cols);
 size_t colsum_counters(int64_t cols);
+// Column sums of a contiguous fp32 [rows, cols] matrix (the order of
+// launch_colsum) that also write it rounded to bf16 into a16 [rows, cols].
+cr_status launch_colsum_bf16(const float* a, int64_t rows, int64_t cols, uint16_t* a16, float* out,
+                             float* scratch, unsigned* counters, cudaStream_t st);
 cr_status launch_colsum(const void* a, bool bf16, int64_t rows, int64_t cols, int64_t lda, float* out,
                         bool accumulate, float* scratch, unsigned* counters, cudaStream_t st);
 cr_status launch_ln_backward(const float* x, const float* gamma, const float* dy, const float* add, float eps,

@@ -132,24 +132,56 @@ __global__ void loss_total_kernel(const double* __restrict__ per_req, int n_req,
     loss_out[0] = static_cast<float>(l);
 }
 
-// Column sums in a fixed order, one launch: block (x, y) sums slice y (kColSlice
-// rows) of 256 columns into partial[y][c]; the last block of column block x to
-// finish (elected by a counter, after a fence) adds the slices in order and
-// resets the counter.  The order of the additions never depends on timing.
-constexpr int kColSlice = 64;
-template <typename T>
+// Column sums in a fixed order, one launch: block (x, y) sums rows
+// [kColSlice y, kColSlice (y + 1)) of the 64 columns [64 x, 64 x + 64), two
+// adjacent columns per lane: warp w of 8 adds rows w, w + 8, ... in row order
+// (eight loads in flight), the warps' sums are added in warp order into
+// partial[y][c], and the last block of column block x to finish (elected by a
+// counter, after a fence) adds the slices in order and resets the counter.
+// The order of the additions never depends on timing.  kOut16: an fp32 input
+// is also written rounded to bf16 (round to nearest even) into a16 [rows,
+// cols], the operand of the backward's GEMMs, from the same read.  cols and
+// lda are even.
+constexpr int kColSlice = 256;
+__device__ __forceinline__ float2 ld2(const float* p, int64_t i) {
+    return *reinterpret_cast<const float2*>(p + i);
+}
+__device__ __forceinline__ float2 ld2(const uint16_t* p, int64_t i) {
+    const uint32_t v = *reinterpret_cast<const uint32_t*>(p + i);
+    return make_float2(__uint_as_float(v << 16), __uint_as_float(v & 0xFFFF0000u));
+}
+template <typename T, bool kOut16>
 __global__ void __launch_bounds__(256)
-    colsum_kernel(const T* __restrict__ a, int64_t rows, int64_t cols, int64_t lda, float* part,
-                  float* __restrict__ out, int accumulate, unsigned* __restrict__ counters) {
+    colsum_kernel(const T* __restrict__ a, int64_t rows, int64_t cols, int64_t lda,
+                  uint16_t* __restrict__ a16, float* part, float* __restrict__ out, int accumulate,
+                  unsigned* __restrict__ counters) {
     pdl_launch_dependents();
     pdl_wait();
-    const int64_t c = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
+    const int lane = static_cast<int>(threadIdx.x & 31), w = static_cast<int>(threadIdx.x >> 5);
+    const int64_t c = static_cast<int64_t>(blockIdx.x) * 64 + 2 * lane;
+    const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kColSlice;
+    const int64_t r1 = min(rows, r0 + kColSlice);
+    float s0 = 0.0f, s1 = 0.0f;
     if (c < cols) {
-        const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kColSlice;
-        const int64_t r1 = min(rows, r0 + kColSlice);
-        float s = 0.0f;
-        for (int64_t r = r0; r < r1; ++r) s += ld(a, r * lda + c);
-        part[static_cast<int64_t>(blockIdx.y) * cols + c] = s;
+#pragma unroll 8
+        for (int64_t r = r0 + w; r < r1; r += 8) {
+            const float2 v = ld2(a, r * lda + c);
+            s0 += v.x;
+            s1 += v.y;
+            if constexpr (kOut16) *reinterpret_cast<uint32_t*>(a16 + r * cols + c) = pack_bf16x2(v.x, v.y);
+        }
+    }
+    __shared__ float2 red[8][32];
+    red[w][lane] = make_float2(s0, s1);
+    __syncthreads();
+    if (w == 0 && c < cols) {
+        float t0 = 0.0f, t1 = 0.0f;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            t0 += red[k][lane].x;
+            t1 += red[k][lane].y;
+        }
+        *reinterpret_cast<float2*>(part + static_cast<int64_t>(blockIdx.y) * cols + c) = make_float2(t0, t1);
     }
     __threadfence();
     __syncthreads();
@@ -158,10 +190,15 @@ __global__ void __launch_bounds__(256)
     __syncthreads();
     if (!last) return;
     __threadfence();
-    if (c < cols) {
-        float s = 0.0f;
-        for (int64_t y = 0; y < gridDim.y; ++y) s += __ldcg(part + y * cols + c);
-        out[c] = accumulate ? out[c] + s : s;
+    if (w == 0 && c < cols) {
+        float t0 = 0.0f, t1 = 0.0f;
+        for (int64_t y = 0; y < gridDim.y; ++y) {
+            const float2 v = __ldcg(reinterpret_cast<const float2*>(part + y * cols + c));
+            t0 += v.x;
+            t1 += v.y;
+        }
+        out[c] = accumulate ? out[c] + t0 : t0;
+        out[c + 1] = accumulate ? out[c + 1] + t1 : t1;
     }
     if (threadIdx.x == 0) counters[blockIdx.x] = 0u;
 }
@@ -409,17 +446,30 @@ size_t colsum_scratch_floats(int64_t rows, int64_t cols) {
     return static_cast<size_t>((rows + kColSlice - 1) / kColSlice) * static_cast<size_t>(cols);
 }
 
-size_t colsum_counters(int64_t cols) { return static_cast<size_t>((cols + 255) / 256); }
+size_t colsum_counters(int64_t cols) { return static_cast<size_t>((cols + 31) / 32); }
+
+cr_status launch_colsum_bf16(const float* a, int64_t rows, int64_t cols, uint16_t* a16, float* out,
+                             float* scratch, unsigned* counters, cudaStream_t st) {
+    const int64_t slices = (rows + kColSlice - 1) / kColSlice;
+    if (slices > 65535) return CR_ERR_UNSUPPORTED;
+    if ((cols & 1) != 0) return CR_ERR_UNSUPPORTED;
+    const dim3 g1(static_cast<unsigned>((cols + 63) / 64), static_cast<unsigned>(slices));
+    return launch_pdl(colsum_kernel<float, true>, g1, dim3(256), 0, st, a, rows, cols, cols, a16, scratch, out,
+                      0, counters);
+}
 
 cr_status launch_colsum(const void* a, bool bf16, int64_t rows, int64_t cols, int64_t lda, float* out,
                         bool accumulate, float* scratch, unsigned* counters, cudaStream_t st) {
     const int64_t slices = (rows + kColSlice - 1) / kColSlice;
     if (slices > 65535) return CR_ERR_UNSUPPORTED;
-    const dim3 g1(static_cast<unsigned>((cols + 255) / 256), static_cast<unsigned>(slices));
-    return bf16 ? launch_pdl(colsum_kernel<uint16_t>, g1, dim3(256), 0, st, static_cast<const uint16_t*>(a),
-                             rows, cols, lda, scratch, out, accumulate ? 1 : 0, counters)
-                : launch_pdl(colsum_kernel<float>, g1, dim3(256), 0, st, static_cast<const float*>(a), rows,
-                             cols, lda, scratch, out, accumulate ? 1 : 0, counters);
+    if ((cols & 1) != 0 || (lda & 1) != 0) return CR_ERR_UNSUPPORTED;
+    const dim3 g1(static_cast<unsigned>((cols + 63) / 64), static_cast<unsigned>(slices));
+    uint16_t* none = nullptr;
+    return bf16 ? launch_pdl(colsum_kernel<uint16_t, false>, g1, dim3(256), 0, st,
+                             static_cast<const uint16_t*>(a), rows, cols, lda, none, scratch, out,
+                             accumulate ? 1 : 0, counters)
+                : launch_pdl(colsum_kernel<float, false>, g1, dim3(256), 0, st, static_cast<const float*>(a),
+                             rows, cols, lda, none, scratch, out, accumulate ? 1 : 0, counters);
 }
 
 cr_status launch_ln_backward(const float* x, const float* gamma, const float* dy, const float* add, float eps,
