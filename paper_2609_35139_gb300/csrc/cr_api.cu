@@ -1021,8 +1021,9 @@ cr_status cr_param_layout(const cr_target_dims* target, const cr_repairer_dims* 
 
 namespace {
 struct TrainLayout {
-    size_t inf, h0, rein, blk, blk_stride, hbuf, yf, rope, ones, r, dz, rowsq, perreq, stats_pad, dh, dxm,
-        du, dtmp, pre, gprod, sig16, dqkv, da, lse, dvec, cstart, dse, dy, colsum, colcnt, norm, blas, total;
+    size_t inf, h0, rein, blk, blk_stride, hbuf, yf, rope, ones, r, dz, rowsq, rowscale, losspart, perreq,
+        stats_pad, dh, dxm, du, dtmp, pre, gprod, sig16, dqkv, da, lse, dvec, cstart, dse, dy, colsum, colcnt,
+        norm, blas, total;
     size_t x_in, x_mid, u1, u2, qkv, o, g;   // offsets inside one block's region
 };
 constexpr size_t kBlasBytes = 32ull << 20;
@@ -1062,6 +1063,8 @@ TrainLayout train_layout(const Dims& d, int64_t n) {
     L.r = take(N * d.D * 4);
     L.dz = take(N * d.D * 2);
     L.rowsq = take(N * 4);
+    L.rowscale = take(N * 4);
+    L.losspart = take(N * static_cast<size_t>(2 * (d.D / 128)) * 4);   // r^2 per (row, column tile, group)
     L.perreq = take(kMaxReq * 8);
     L.dh = take(N * d.db * 4);
     L.dxm = take(N * d.db * 4);
@@ -1300,24 +1303,20 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
         return s;
     if ((s = launch_layernorm(H, nullptr, 0, nullptr, w.lnf_g, w.lnf_b, eps, N, db, yf, st)) != CR_OK) return s;
 
-    // ---- objective (Sec. 4.2): the head writes r = z - (joint - stale) / sigma_Delta
+    // ---- objective (Sec. 4.2): r = z - (joint - stale) / sigma_Delta in the head's
+    // epilogue, which writes dz = c r and the rows' r^2 sums
     if ((s = launch_target(kv_stale, kv_joint, false, sigma_delta, N, D, R, st)) != CR_OK) return s;
     if ((s = launch_fill(ones, D, 1.0f, st)) != CR_OK) return s;
-    GemmParams gh{};
-    gh.status = status;
-    gh.bias = w.b_out;
-    gh.sigma = ones;
-    gh.pos = pos;
-    gh.rope_dim = static_cast<int32_t>(d.dh);
-    gh.n_kv_heads = static_cast<int32_t>(d.H);
-    if ((s = launch_gemm(yf, db, w.w_out, N, D, db, EPI_KV_F32, gh, R, D, st)) != CR_OK) return s;
     LossParams* lp = new LossParams();
     lp->n_req = n_req;
     for (int r = 0; r <= n_req; ++r) lp->req_start[r] = cu_seqlens_host[r];
     for (int r = 0; r < n_req; ++r)
         lp->scale[r] = static_cast<float>(
             2.0 / (static_cast<double>(cu_seqlens_host[r + 1] - cu_seqlens_host[r]) * D * n_req));
-    s = launch_loss(R, N, D, *lp, DZ, ROWSQ, stats_out, PERREQ, st);
+    // the head writes dz and the loss straight from r, which is never stored
+    s = launch_loss_head(yf, w.w_out, w.b_out, ones, R, N, D, db, *lp, DZ,
+                         reinterpret_cast<float*>(base + L.rowscale), reinterpret_cast<float*>(base + L.losspart),
+                         ROWSQ, stats_out, PERREQ, status, st);
     delete lp;
     if (s != CR_OK) return s;
 

@@ -49,12 +49,18 @@ static_assert(kGemmRegsCtl * 128 + 2 * kGemmRegsEpi * 128 <= kGemmRegsLaunch * k
 
 template <int BN, int EPI, int CG>
 struct GemmCfg {
-    static constexpr bool kKV = (EPI == EPI_KV_BF16 || EPI == EPI_KV_F32 || EPI == EPI_KV_PAGED);
+    static constexpr bool kKV =
+        (EPI == EPI_KV_BF16 || EPI == EPI_KV_F32 || EPI == EPI_KV_PAGED || EPI == EPI_KV_LOSS);
     // the stale tile is staged as for the in-place update, but the repaired rows
     // go straight from registers to the paged target cache (no TMA store)
     static constexpr bool kPaged = (EPI == EPI_KV_PAGED);
+    // training head: the residual r goes out as the bf16 gradient dz and row sums
+    // of r^2, from registers (no TMA store)
+    static constexpr bool kLoss = (EPI == EPI_KV_LOSS);
+    static constexpr bool kDirect = kPaged || kLoss;
     static constexpr bool kInPlace = kKV || EPI == EPI_ADD_F32;   // tile loaded, updated, stored
-    static constexpr int kTileEsize = (EPI == EPI_KV_F32 || EPI == EPI_ADD_F32 || EPI == EPI_F32) ? 4 : 2;
+    static constexpr int kTileEsize =
+        (EPI == EPI_KV_F32 || EPI == EPI_KV_LOSS || EPI == EPI_ADD_F32 || EPI == EPI_F32) ? 4 : 2;
     static constexpr int kBoxCols = 128 / kTileEsize;          // one 128-byte swizzle row
     // in-place epilogues stage the whole [BM x BN] tile; store-only epilogues
     // stage one 16 KB box (128 rows x 128 B) at a time per epilogue group
@@ -450,7 +456,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 for (int b = 0; b < Cfg::kBoxes && ok; ++b) {
                     if (!(ok = mbar_wait_warp(&epi_done[b], pk & 1u, wc, 401))) break;
                     if (leader) {
-                        if (rows_in && !Cfg::kPaged) {
+                        if (rows_in && !Cfg::kDirect) {
                             tma_store_2d(&tmC, tile + b * 16384, n0 + b * Cfg::kBoxCols, m0);
                             tma_store_commit();
                             tma_store_wait_read0();
@@ -604,9 +610,29 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                         report(p.status, CR_DEV_INDEX, 410);
                     }
                 }
+                // training head: this row's gradient row, loss weight and r^2 sum
+                // over this group's columns of the tile (chunks in column order)
+                uint16_t* dzrow = nullptr;
+                float lsc = 0.0f, lsq = 0.0f;
+                if constexpr (Cfg::kLoss) {
+                    if (row_ok) {
+                        dzrow = p.loss_dz + static_cast<int64_t>(row) * p.N + n0;
+                        lsc = __ldg(p.row_scale + row);
+                    }
+                }
                 auto put16 = [&](int col, const float* v) {
                     if constexpr (Cfg::kPaged) {
                         if (prow) store16_bf16_global(prow + col, v);
+                    } else if constexpr (Cfg::kLoss) {
+                        if (dzrow) {
+                            float d[16];
+#pragma unroll
+                            for (int q = 0; q < 16; ++q) {
+                                lsq = fmaf(v[q], v[q], lsq);
+                                d[q] = lsc * v[q];
+                            }
+                            store16_bf16_global(dzrow + col, d);
+                        }
                     } else {
                         store16_tile<ES>(tile, r, col, v);
                     }
@@ -712,6 +738,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     }
                 }
                 if (!ok) break;
+                if constexpr (Cfg::kLoss) {
+                    if (row_ok) p.loss_part[static_cast<int64_t>((n0 / BN) * 2 + eg) * p.M + row] = lsq;
+                }
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) release_acc(&tempty[acc]);
@@ -881,8 +910,8 @@ constexpr int kCG = 2;
 cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t M, int64_t N,
                       int64_t K, int epi, GemmParams p, void* kv_base, int64_t ld_kv,
                       cudaStream_t st) {
-    const bool kv = (epi == EPI_KV_BF16 || epi == EPI_KV_F32 || epi == EPI_KV_PAGED);
-    const bool f32_tile = (epi == EPI_KV_F32 || epi == EPI_ADD_F32);
+    const bool kv = (epi == EPI_KV_BF16 || epi == EPI_KV_F32 || epi == EPI_KV_PAGED || epi == EPI_KV_LOSS);
+    const bool f32_tile = (epi == EPI_KV_F32 || epi == EPI_KV_LOSS || epi == EPI_ADD_F32);
     // Tile width.  Per 64-deep k-block a CTA of a pair moves 32 KB + 128 BN
     // bytes through shared memory (TMA writes and MMA operand reads of its A
     // rows and W half) at ~128 B/clock, and its MMAs take 2 BN clocks, so a
@@ -892,7 +921,7 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
     // any output element's K order, so results do not depend on it.
     int BN;
     if (kv) {
-        BN = (epi == EPI_KV_F32) ? 128 : 256;
+        BN = (epi == EPI_KV_F32 || epi == EPI_KV_LOSS) ? 128 : 256;
     } else if (epi == EPI_F32) {
         BN = 128;
     } else {
@@ -969,6 +998,9 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
             return launch_bn<256, EPI_KV_BF16, kCG>(ta, tb, tc, p, st);
         case EPI_KV_F32:
             return launch_bn<128, EPI_KV_F32, kCG>(ta, tb, tc, p, st);
+        case EPI_KV_LOSS:
+            if (!p.loss_dz || !p.row_scale || !p.loss_part) return CR_ERR_INVALID_ARG;
+            return launch_bn<128, EPI_KV_LOSS, kCG>(ta, tb, tc, p, st);
         case EPI_KV_PAGED:
             if (p.seg_width <= 0 || p.seg_width % 256 != 0 || p.num_slots < 1) return CR_ERR_UNSUPPORTED;
             return launch_bn<256, EPI_KV_PAGED, kCG>(ta, tb, tc, p, st);

@@ -4,6 +4,8 @@
 //   target_kernel        -(KV_joint - KV_stale) / sigma_Delta, the head's in-place
 //                        input, so that the head epilogue writes r = z - target
 //   loss_grad_kernel     per row: sum of r^2, and dz = c_request * r (bf16)
+//   row_scale_kernel     c_request of every row, for the loss head's epilogue
+//   rowsq_kernel         per row: the loss head's partial sums of r^2 in order
 //   loss_reduce_kernel   per request, rows summed in order (fp64): the loss
 //   colsum_kernel        column sums in a fixed order (bias, LayerNorm grads)
 //   ln_backward_kernel   LayerNorm backward per row, plus dy * x_hat per element
@@ -70,6 +72,43 @@ __global__ void __launch_bounds__(256)
         float4* dst = reinterpret_cast<float4*>(out + i * 8);
         dst[0] = make_float4(o[0], o[1], o[2], o[3]);
         dst[1] = make_float4(o[4], o[5], o[6], o[7]);
+    }
+}
+
+// The loss weight c of each row's request: dL/dr = c r.
+__global__ void row_scale_kernel(const __grid_constant__ LossParams p, int64_t n, float* __restrict__ out) {
+    pdl_launch_dependents();
+    pdl_wait();
+    for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < n;
+         t += static_cast<int64_t>(gridDim.x) * blockDim.x)
+        out[t] = p.scale[request_of(p, t)];
+}
+
+// Per row, the loss head's nparts partial sums of r^2 (part[j][row], one per
+// column tile and epilogue column group) added in a fixed order: block of 8
+// warps over 32 rows (a lane per row), warp w adds parts [w P/8, (w+1) P/8) in
+// order, eight loads in flight, then the warps' sums in warp order.
+__global__ void __launch_bounds__(256)
+    rowsq_kernel(const float* __restrict__ part, int64_t rows, int nparts, float* __restrict__ rowsq) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int lane = static_cast<int>(threadIdx.x & 31), w = static_cast<int>(threadIdx.x >> 5);
+    const int64_t t = static_cast<int64_t>(blockIdx.x) * 32 + lane;
+    const int per = (nparts + 7) / 8;
+    const int j0 = w * per, j1 = min(nparts, j0 + per);
+    float s = 0.0f;
+    if (t < rows) {
+#pragma unroll 8
+        for (int j = j0; j < j1; ++j) s += part[static_cast<int64_t>(j) * rows + t];
+    }
+    __shared__ float red[8][32];
+    red[w][lane] = s;
+    __syncthreads();
+    if (w == 0 && t < rows) {
+        float a = 0.0f;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) a += red[k][lane];
+        rowsq[t] = a;
     }
 }
 
@@ -428,6 +467,31 @@ cr_status launch_target(const void* stale, const void* joint, bool f32, const fl
     if (f32 || D % 8 != 0) return CR_ERR_UNSUPPORTED;
     return launch_pdl(target_kernel, grid_for(n * D / 8), dim3(256), 0, st,
                       static_cast<const uint16_t*>(stale), static_cast<const uint16_t*>(joint), sd, n, D, out);
+}
+
+cr_status launch_loss_head(const uint16_t* yf, const uint16_t* w_out, const float* b_out, const float* ones,
+                           float* neg_target, int64_t N, int64_t D, int64_t db, const LossParams& p,
+                           uint16_t* dz, float* row_scale, float* part, float* rowsq, float* loss_out,
+                           double* per_req, unsigned* status, cudaStream_t st) {
+    cr_status s = launch_pdl(row_scale_kernel, grid_for(N), dim3(256), 0, st, p, N, row_scale);
+    if (s != CR_OK) return s;
+    GemmParams gh{};
+    gh.status = status;
+    gh.bias = b_out;
+    gh.sigma = ones;
+    gh.loss_dz = dz;
+    gh.row_scale = row_scale;
+    gh.loss_part = part;
+    if ((s = launch_gemm(yf, db, w_out, N, D, db, EPI_KV_LOSS, gh, neg_target, D, st)) != CR_OK) return s;
+    const int nparts = static_cast<int>(2 * (D / 128));
+    s = launch_pdl(rowsq_kernel, dim3(static_cast<unsigned>((N + 31) / 32)), dim3(256), 0, st,
+                   static_cast<const float*>(part), N, nparts, rowsq);
+    if (s != CR_OK) return s;
+    s = launch_pdl(loss_reduce_kernel, dim3(static_cast<unsigned>(p.n_req)), dim3(256), 0, st,
+                   static_cast<const float*>(rowsq), p, D, per_req);
+    if (s != CR_OK) return s;
+    return launch_pdl(loss_total_kernel, dim3(1), dim3(32), 0, st, static_cast<const double*>(per_req), p.n_req,
+                      loss_out);
 }
 
 cr_status launch_loss(const float* r, int64_t N, int64_t D, const LossParams& p, uint16_t* dz, float* rowsq,
