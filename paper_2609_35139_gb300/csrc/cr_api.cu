@@ -1021,7 +1021,7 @@ cr_status cr_param_layout(const cr_target_dims* target, const cr_repairer_dims* 
 
 namespace {
 struct TrainLayout {
-    size_t inf, h0, rein, blk, blk_stride, hbuf, yf, rope, ones, r, dz, rowsq, rowscale, losspart, perreq,
+    size_t inf, h0, rein, blk, blk_stride, hbuf, yf, rope, dz, rowsq, rowscale, losspart, perreq,
         stats_pad, dh, dxm, du, dtmp, pre, gprod, sig16, dqkv, da, lse, dvec, cstart, dse, dy, colsum, colcnt,
         norm, blas, total;
     size_t x_in, x_mid, u1, u2, qkv, o, g;   // offsets inside one block's region
@@ -1059,8 +1059,6 @@ TrainLayout train_layout(const Dims& d, int64_t n) {
     L.hbuf = take(N * d.db * 4);
     L.yf = take(N * d.db * 2);
     L.rope = take(N * (d.hd / 2) * 8);
-    L.ones = take(d.D * 4);
-    L.r = take(N * d.D * 4);
     L.dz = take(N * d.D * 2);
     L.rowsq = take(N * 4);
     L.rowscale = take(N * 4);
@@ -1198,8 +1196,6 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
     float* H = at<float>(base, L.hbuf);
     uint16_t* yf = at<uint16_t>(base, L.yf);
     float2* rope = at<float2>(base, L.rope);
-    float* ones = at<float>(base, L.ones);
-    float* R = at<float>(base, L.r);
     uint16_t* DZ = at<uint16_t>(base, L.dz);
     float* ROWSQ = at<float>(base, L.rowsq);
     double* PERREQ = at<double>(base, L.perreq);
@@ -1305,8 +1301,6 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
 
     // ---- objective (Sec. 4.2): r = z - (joint - stale) / sigma_Delta in the head's
     // epilogue, which writes dz = c r and the rows' r^2 sums
-    if ((s = launch_target(kv_stale, kv_joint, false, sigma_delta, N, D, R, st)) != CR_OK) return s;
-    if ((s = launch_fill(ones, D, 1.0f, st)) != CR_OK) return s;
     LossParams* lp = new LossParams();
     lp->n_req = n_req;
     for (int r = 0; r <= n_req; ++r) lp->req_start[r] = cu_seqlens_host[r];
@@ -1314,7 +1308,8 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
         lp->scale[r] = static_cast<float>(
             2.0 / (static_cast<double>(cu_seqlens_host[r + 1] - cu_seqlens_host[r]) * D * n_req));
     // the head writes dz and the loss straight from r, which is never stored
-    s = launch_loss_head(yf, w.w_out, w.b_out, ones, R, N, D, db, *lp, DZ,
+    s = launch_loss_head(yf, w.w_out, w.b_out, sigma_delta, static_cast<const uint16_t*>(kv_stale),
+                         static_cast<const uint16_t*>(kv_joint), N, D, db, *lp, DZ,
                          reinterpret_cast<float*>(base + L.rowscale), reinterpret_cast<float*>(base + L.losspart),
                          ROWSQ, stats_out, PERREQ, status, st);
     delete lp;

@@ -59,8 +59,7 @@ struct GemmCfg {
     static constexpr bool kLoss = (EPI == EPI_KV_LOSS);
     static constexpr bool kDirect = kPaged || kLoss;
     static constexpr bool kInPlace = kKV || EPI == EPI_ADD_F32;   // tile loaded, updated, stored
-    static constexpr int kTileEsize =
-        (EPI == EPI_KV_F32 || EPI == EPI_KV_LOSS || EPI == EPI_ADD_F32 || EPI == EPI_F32) ? 4 : 2;
+    static constexpr int kTileEsize = (EPI == EPI_KV_F32 || EPI == EPI_ADD_F32 || EPI == EPI_F32) ? 4 : 2;
     static constexpr int kBoxCols = 128 / kTileEsize;          // one 128-byte swizzle row
     // in-place epilogues stage the whole [BM x BN] tile; store-only epilogues
     // stage one 16 KB box (128 rows x 128 B) at a time per epilogue group
@@ -69,7 +68,10 @@ struct GemmCfg {
     // leaves room for a deeper operand ring
     static constexpr int kBoxes = BN / kBoxCols;                // boxes per tile
     static constexpr int kGroupBufs = (EPI == EPI_GELU_BF16 || EPI == EPI_QKV_ROPE) ? 2 : 1;
-    static constexpr uint32_t kTileBytes = kInPlace ? BM * BN * kTileEsize : 2 * kGroupBufs * 16384;
+    // (the loss head stages two bf16 tiles: stale in the even, joint in the odd
+    // 16 KB boxes, column box b at boxes 2 b and 2 b + 1)
+    static constexpr uint32_t kTileBytes =
+        kInPlace ? BM * BN * kTileEsize * (kLoss ? 2 : 1) : 2 * kGroupBufs * 16384;
     static constexpr uint32_t kVecBytes = BN * 4 * (kKV ? 2 : 1);   // bias (+ sigma)
     // in-place epilogues recycle the staged tile box by box, so the next tile's
     // vectors may land while this tile is still being finished: two buffers
@@ -406,13 +408,20 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     for (int b = 0; b < Cfg::kBoxes; ++b) {
                         if (!(ok = mbar_wait_warp(&epi_empty[b], (static_cast<uint32_t>(i) & 1u) ^ 1u, wc, 101)))
                             break;
-                        uint32_t bytes = load_tile ? 16384u : 0u;
+                        uint32_t bytes = load_tile ? (Cfg::kLoss ? 32768u : 16384u) : 0u;
                         if (b == 0) bytes += (has_bias ? vbytes : 0u) + (Cfg::kKV ? vbytes : 0u);
                         if (elect_one()) {
                             if (bytes) mbar_expect_tx(&epi_full[b], bytes);
                             else mbar_arrive(&epi_full[b]);
-                            if (load_tile)
-                                tma_load_2d(tile + b * 16384, &tmC, &epi_full[b], n0 + b * Cfg::kBoxCols, m0);
+                            if (load_tile) {
+                                if constexpr (Cfg::kLoss) {
+                                    tma_load_2d(tile + 2 * b * 16384, &tmC, &epi_full[b], n0 + b * Cfg::kBoxCols, m0);
+                                    tma_load_2d(tile + (2 * b + 1) * 16384, &p.tm_joint, &epi_full[b],
+                                                n0 + b * Cfg::kBoxCols, m0);
+                                } else {
+                                    tma_load_2d(tile + b * 16384, &tmC, &epi_full[b], n0 + b * Cfg::kBoxCols, m0);
+                                }
+                            }
                             if (b == 0) {
                                 if (has_bias) bulk_load(vdst, p.bias + n0, vbytes, &epi_full[0]);
                                 if constexpr (Cfg::kKV) bulk_load(vdst + BN, p.sigma + n0, vbytes, &epi_full[0]);
@@ -650,7 +659,39 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     fence_async_smem();
                     mbar_arrive(&epi_done[b]);
                 };
-                if (Cfg::kKV && p.rope_on) {
+                if constexpr (Cfg::kLoss) {
+                    // r = z + b - (joint - stale) / sigma_Delta, the stale and joint
+                    // values from column box bx's two staged bf16 boxes; each group
+                    // takes one half of the box's columns
+                    constexpr int HALF = Cfg::kBoxCols / 2;
+                    for (int bx = 0; bx < Cfg::kBoxes && ok; ++bx) {
+                        if (!(ok = wait_box(bx))) break;
+                        const uint8_t* sbox = tile + 2 * bx * 16384;
+                        for (int c = bx * Cfg::kBoxCols + eg * HALF; c < bx * Cfg::kBoxCols + (eg + 1) * HALF;
+                             c += 16) {
+                            float a[16], st16[16], jt16[16], bv[16], sd[16];
+                            __syncwarp();
+                            tmem_ld16(taddr + c, a);
+                            load16_bf16_smem(sbox, r, c - bx * Cfg::kBoxCols, st16);
+                            load16_bf16_smem(sbox + 16384, r, c - bx * Cfg::kBoxCols, jt16);
+                            if (has_bias) {
+                                vec16(vbt, c, bv);
+                            } else {
+#pragma unroll
+                                for (int q = 0; q < 16; ++q) bv[q] = 0.0f;
+                            }
+                            vec16(vst, c, sd);
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int q = 0; q < 16; ++q) {
+                                const float nt = -(jt16[q] - st16[q]) / sd[q];
+                                a[q] = (a[q] + bv[q]) + nt;
+                            }
+                            put16(c, a);
+                        }
+                        done_box(bx);
+                    }
+                } else if (Cfg::kKV && p.rope_on) {
                     // R_M pairs (d, d + d_h/2) live inside one d_h-wide segment, which
                     // spans d_h / kBoxCols boxes; each group takes half of its pairs
                     const int dh = p.rope_dim;
@@ -911,7 +952,7 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
                       int64_t K, int epi, GemmParams p, void* kv_base, int64_t ld_kv,
                       cudaStream_t st) {
     const bool kv = (epi == EPI_KV_BF16 || epi == EPI_KV_F32 || epi == EPI_KV_PAGED || epi == EPI_KV_LOSS);
-    const bool f32_tile = (epi == EPI_KV_F32 || epi == EPI_KV_LOSS || epi == EPI_ADD_F32);
+    const bool f32_tile = (epi == EPI_KV_F32 || epi == EPI_ADD_F32);
     // Tile width.  Per 64-deep k-block a CTA of a pair moves 32 KB + 128 BN
     // bytes through shared memory (TMA writes and MMA operand reads of its A
     // rows and W half) at ~128 B/clock, and its MMAs take 2 BN clocks, so a
@@ -999,7 +1040,10 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
         case EPI_KV_F32:
             return launch_bn<128, EPI_KV_F32, kCG>(ta, tb, tc, p, st);
         case EPI_KV_LOSS:
-            if (!p.loss_dz || !p.row_scale || !p.loss_part) return CR_ERR_INVALID_ARG;
+            if (!p.loss_dz || !p.row_scale || !p.loss_part || !p.loss_joint || !p.sigma) return CR_ERR_INVALID_ARG;
+            if (!make_tmap_2d(&p.tm_joint, p.loss_joint, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, N, M, ld_kv * 2, 64,
+                              BM, CU_TENSOR_MAP_SWIZZLE_128B))
+                return CR_ERR_INVALID_ARG;
             return launch_bn<128, EPI_KV_LOSS, kCG>(ta, tb, tc, p, st);
         case EPI_KV_PAGED:
             if (p.seg_width <= 0 || p.seg_width % 256 != 0 || p.num_slots < 1) return CR_ERR_UNSUPPORTED;

@@ -57,9 +57,9 @@ enum GemmEpi : int {
     EPI_KV_F32 = 6,     // same for an fp32 cache
     EPI_KV_PAGED = 7,   // bf16 cache: stale tile read token-major, repaired rows written
                         // to a paged, layer-major target cache through a slot mapping
-    EPI_KV_LOSS = 8     // training head: r = z + b + tile (the fp32 tile holds -target,
-                        // sigma = 1); writes dz = row_scale[t] r (bf16) and per-row
-                        // partial sums of r^2 instead of storing r
+    EPI_KV_LOSS = 8     // training head: r = z + b - (joint - stale) / sigma from the staged
+                        // bf16 stale and joint tiles; writes dz = row_scale[t] r (bf16)
+                        // and per-row partial sums of r^2 instead of storing r
 };
 
 struct GemmParams {
@@ -88,13 +88,17 @@ struct GemmParams {
     int32_t col_phase;
     int32_t kv_zero;
     const int32_t* keep_chunk;
-    // EPI_KV_LOSS: dz [M, N] bf16; row_scale [M]; loss_part [2 num_n][M], the sum of
-    // r^2 over each (column tile, epilogue column group) of a row
+    // EPI_KV_LOSS: the stale cache is the in-place tile, the joint cache [M, N] bf16
+    // (same row stride) comes in through tm_joint, sigma holds sigma_Delta; dz [M, N]
+    // bf16; row_scale [M]; loss_part [2 num_n][M], the sum of r^2 over each
+    // (column tile, epilogue column group) of a row
+    const uint16_t* loss_joint;
     uint16_t* loss_dz;
     const float* row_scale;
     float* loss_part;
     unsigned* status;
     float inv_freq[64];      // RoPE frequencies, rope_dim / 2 entries
+    alignas(64) CUtensorMap tm_joint;   // EPI_KV_LOSS (set by launch_gemm)
 };
 
 // ------------------------------------------------------------------ segment projection
@@ -249,19 +253,15 @@ cr_status launch_attention_backward(const uint16_t* qkv, const uint16_t* dO16, c
                                     int64_t n_tokens, int head_dim, AttnBwdParams& p, float* dvec, cudaStream_t st);
 
 // training step (cr_train.cu)
-cr_status launch_fill(float* p, int64_t n, float v, cudaStream_t st);
-cr_status launch_target(const void* stale, const void* joint, bool f32, const float* sd, int64_t n,
-                        int64_t D, float* out, cudaStream_t st);
-// The training head and objective in one pass over the cache: r = W_out y_f +
-// b_out - target, with neg_target [N, D] fp32 holding -target; writes dz =
-// c_request r (bf16) and the per-request loss, never r itself.  row_scale [N]
-// and part [2 D / 128][N] fp32 are scratch.
-cr_status launch_loss_head(const uint16_t* yf, const uint16_t* w_out, const float* b_out, const float* ones,
-                           float* neg_target, int64_t N, int64_t D, int64_t db, const LossParams& p,
-                           uint16_t* dz, float* row_scale, float* part, float* rowsq, float* loss_out,
-                           double* per_req, unsigned* status, cudaStream_t st);
-cr_status launch_loss(const float* r, int64_t N, int64_t D, const LossParams& p, uint16_t* dz, float* rowsq,
-                      float* loss_out, double* per_req, cudaStream_t st);
+// The training head and objective in one pass over the caches: r = W_out y_f +
+// b_out - (joint - stale) / sigma_delta from the bf16 stale and joint caches
+// [N, D]; writes dz = c_request r (bf16) and the per-request loss, never r or
+// the target.  row_scale [N] and part [2 D / 128][N] fp32 are scratch.
+cr_status launch_loss_head(const uint16_t* yf, const uint16_t* w_out, const float* b_out,
+                           const float* sigma_delta, const uint16_t* stale, const uint16_t* joint, int64_t N,
+                           int64_t D, int64_t db, const LossParams& p, uint16_t* dz, float* row_scale,
+                           float* part, float* rowsq, float* loss_out, double* per_req, unsigned* status,
+                           cudaStream_t st);
 size_t colsum_scratch_floats(int64_t rows, int64_t cols);
 size_t colsum_counters(int64_t cols);
 // Column sums of a contiguous fp32 [rows, cols] matrix (the order of

@@ -1,9 +1,6 @@
 // Training-step kernels (Sec. 4.2, App. A): the bandwidth-bound pieces of the
 // backward pass and of the optimizer, plus the row-major GEMM helpers over
 // cuBLAS that the backward's plain (unfused) matrix products use.
-//   target_kernel        -(KV_joint - KV_stale) / sigma_Delta, the head's in-place
-//                        input, so that the head epilogue writes r = z - target
-//   loss_grad_kernel     per row: sum of r^2, and dz = c_request * r (bf16)
 //   row_scale_kernel     c_request of every row, for the loss head's epilogue
 //   rowsq_kernel         per row: the loss head's partial sums of r^2 in order
 //   loss_reduce_kernel   per request, rows summed in order (fp64): the loss
@@ -44,36 +41,6 @@ __device__ __forceinline__ int request_of(const LossParams& p, int64_t t) {
     return r0;
 }
 
-// bf16 caches, 8 values per thread (D_KV is a multiple of 8): 16-byte loads and
-// two 16-byte stores
-__global__ void __launch_bounds__(256)
-    target_kernel(const uint16_t* __restrict__ stale, const uint16_t* __restrict__ joint,
-                  const float* __restrict__ sd, int64_t n, int64_t D, float* __restrict__ out) {
-    pdl_launch_dependents();
-    pdl_wait();
-    const int64_t groups = n * D / 8;
-    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < groups;
-         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const int64_t c = (i * 8) % D;
-        const uint4 a = reinterpret_cast<const uint4*>(stale)[i];
-        const uint4 b = reinterpret_cast<const uint4*>(joint)[i];
-        const float4 s0 = __ldg(reinterpret_cast<const float4*>(sd + c));
-        const float4 s1 = __ldg(reinterpret_cast<const float4*>(sd + c + 4));
-        const uint32_t ua[4] = {a.x, a.y, a.z, a.w}, ub[4] = {b.x, b.y, b.z, b.w};
-        const float sv[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
-        float o[8];
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const float a0 = __uint_as_float(ua[k] << 16), a1 = __uint_as_float(ua[k] & 0xFFFF0000u);
-            const float b0 = __uint_as_float(ub[k] << 16), b1 = __uint_as_float(ub[k] & 0xFFFF0000u);
-            o[2 * k] = -(b0 - a0) / sv[2 * k];
-            o[2 * k + 1] = -(b1 - a1) / sv[2 * k + 1];
-        }
-        float4* dst = reinterpret_cast<float4*>(out + i * 8);
-        dst[0] = make_float4(o[0], o[1], o[2], o[3]);
-        dst[1] = make_float4(o[4], o[5], o[6], o[7]);
-    }
-}
 
 // The loss weight c of each row's request: dL/dr = c r.
 __global__ void row_scale_kernel(const __grid_constant__ LossParams p, int64_t n, float* __restrict__ out) {
@@ -112,32 +79,6 @@ __global__ void __launch_bounds__(256)
     }
 }
 
-// One CTA per row: the row's sum of squares of r (fixed-order tree), and
-// dz = scale(request) * r rounded to bf16.
-__global__ void __launch_bounds__(256)
-    loss_grad_kernel(const float* __restrict__ r, int64_t D, const __grid_constant__ LossParams p,
-                     uint16_t* __restrict__ dz, float* __restrict__ rowsq) {
-    pdl_launch_dependents();
-    pdl_wait();
-    const int64_t t = blockIdx.x;
-    const float c = p.scale[request_of(p, t)];
-    const float* row = r + t * D;
-    uint16_t* drow = dz + t * D;
-    float acc = 0.0f;
-    for (int64_t j = threadIdx.x; j < D; j += blockDim.x) {
-        const float v = row[j];
-        acc = fmaf(v, v, acc);
-        drow[j] = f32_to_bf16(c * v);
-    }
-    __shared__ float red[256];
-    red[threadIdx.x] = acc;
-    __syncthreads();
-    for (int s = 128; s > 0; s >>= 1) {
-        if (static_cast<int>(threadIdx.x) < s) red[threadIdx.x] += red[threadIdx.x + s];
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) rowsq[t] = red[0];
-}
 
 // One block per request: each thread sums a fixed stride of the request's rows
 // (fp64), then a fixed tree; the result divided by N_r D n_req (the mean over
@@ -440,13 +381,6 @@ __global__ void __launch_bounds__(256)
     }
 }
 
-__global__ void __launch_bounds__(256) fill_kernel(float* __restrict__ p, int64_t n, float v) {
-    pdl_launch_dependents();
-    pdl_wait();
-    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
-         i += static_cast<int64_t>(gridDim.x) * blockDim.x)
-        p[i] = v;
-}
 
 dim3 grid_for(int64_t n, int64_t cap_per_sm = 16) {
     int64_t b = (n + 255) / 256;
@@ -458,49 +392,29 @@ dim3 grid_for(int64_t n, int64_t cap_per_sm = 16) {
 
 }  // namespace
 
-cr_status launch_fill(float* p, int64_t n, float v, cudaStream_t st) {
-    return launch_pdl(fill_kernel, grid_for(n), dim3(256), 0, st, p, n, v);
-}
-
-cr_status launch_target(const void* stale, const void* joint, bool f32, const float* sd, int64_t n,
-                        int64_t D, float* out, cudaStream_t st) {
-    if (f32 || D % 8 != 0) return CR_ERR_UNSUPPORTED;
-    return launch_pdl(target_kernel, grid_for(n * D / 8), dim3(256), 0, st,
-                      static_cast<const uint16_t*>(stale), static_cast<const uint16_t*>(joint), sd, n, D, out);
-}
-
-cr_status launch_loss_head(const uint16_t* yf, const uint16_t* w_out, const float* b_out, const float* ones,
-                           float* neg_target, int64_t N, int64_t D, int64_t db, const LossParams& p,
-                           uint16_t* dz, float* row_scale, float* part, float* rowsq, float* loss_out,
-                           double* per_req, unsigned* status, cudaStream_t st) {
+cr_status launch_loss_head(const uint16_t* yf, const uint16_t* w_out, const float* b_out,
+                           const float* sigma_delta, const uint16_t* stale, const uint16_t* joint, int64_t N,
+                           int64_t D, int64_t db, const LossParams& p, uint16_t* dz, float* row_scale,
+                           float* part, float* rowsq, float* loss_out, double* per_req, unsigned* status,
+                           cudaStream_t st) {
     cr_status s = launch_pdl(row_scale_kernel, grid_for(N), dim3(256), 0, st, p, N, row_scale);
     if (s != CR_OK) return s;
     GemmParams gh{};
     gh.status = status;
     gh.bias = b_out;
-    gh.sigma = ones;
+    gh.sigma = sigma_delta;
+    gh.loss_joint = joint;
     gh.loss_dz = dz;
     gh.row_scale = row_scale;
     gh.loss_part = part;
-    if ((s = launch_gemm(yf, db, w_out, N, D, db, EPI_KV_LOSS, gh, neg_target, D, st)) != CR_OK) return s;
+    if ((s = launch_gemm(yf, db, w_out, N, D, db, EPI_KV_LOSS, gh, const_cast<uint16_t*>(stale), D, st)) != CR_OK)
+        return s;
     const int nparts = static_cast<int>(2 * (D / 128));
     s = launch_pdl(rowsq_kernel, dim3(static_cast<unsigned>((N + 31) / 32)), dim3(256), 0, st,
                    static_cast<const float*>(part), N, nparts, rowsq);
     if (s != CR_OK) return s;
     s = launch_pdl(loss_reduce_kernel, dim3(static_cast<unsigned>(p.n_req)), dim3(256), 0, st,
                    static_cast<const float*>(rowsq), p, D, per_req);
-    if (s != CR_OK) return s;
-    return launch_pdl(loss_total_kernel, dim3(1), dim3(32), 0, st, static_cast<const double*>(per_req), p.n_req,
-                      loss_out);
-}
-
-cr_status launch_loss(const float* r, int64_t N, int64_t D, const LossParams& p, uint16_t* dz, float* rowsq,
-                      float* loss_out, double* per_req, cudaStream_t st) {
-    cr_status s = launch_pdl(loss_grad_kernel, dim3(static_cast<unsigned>(N)), dim3(256), 0, st, r, D, p,
-                             dz, rowsq);
-    if (s != CR_OK) return s;
-    s = launch_pdl(loss_reduce_kernel, dim3(static_cast<unsigned>(p.n_req)), dim3(256), 0, st, rowsq, p, D,
-                   per_req);
     if (s != CR_OK) return s;
     return launch_pdl(loss_total_kernel, dim3(1), dim3(32), 0, st, static_cast<const double*>(per_req), p.n_req,
                       loss_out);
