@@ -11,8 +11,9 @@
 //               double-buffered fp32 accumulator and multicasts its commits.
 //   warp 2      epilogue-input loader: per tile, the bias (and sigma_delta)
 //               slice by bulk copy and, for in-place epilogues, the output tile
-//               itself (the stale cache tile, or the fp32 residual-stream tile)
-//               by TMA, as soon as the epilogue has released its slot.
+//               itself (the stale cache tile, the fp32 residual-stream tile, or
+//               for the training loss head the stale and joint cache tiles) by
+//               TMA, as soon as the epilogue has released its slot.
 //   warp 3      TMA store issuer for the staged output.
 //   warps 4..11 epilogue, two groups of four warps (one per TMEM lane
 //               quarter) splitting each tile's columns: tcgen05.ld 32 lanes x
@@ -21,7 +22,11 @@
 //               of 128 B-wide columns at a time, double-buffered per group), or
 //               in place on the staged tile: residual stream x += acc + b,
 //               cache kv = kv + sigma_delta (acc + b) (+ R_M on K).  Staged
-//               data goes out with TMA stores (coalesced, asynchronous).
+//               data goes out with TMA stores (coalesced, asynchronous).  The
+//               paged head and the loss head write from registers instead: the
+//               repaired rows into the paged target cache, or the training
+//               gradient dz = c (acc + b - (joint - stale) / sigma_delta) in
+//               bf16 with each row's sum of squares of the residual.
 // Warps 0..3 give registers to the epilogue warpgroups (setmaxnreg).
 #include <cuda_bf16.h>
 
