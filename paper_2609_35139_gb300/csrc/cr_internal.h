@@ -98,7 +98,7 @@ struct GemmParams {
     float* loss_part;
     unsigned* status;
     float inv_freq[64];      // RoPE frequencies, rope_dim / 2 entries
-    alignas(64) CUtensorMap tm_joint;   // EPI_KV_LOSS (set by launch_gemm)
+    CUtensorMap tm_joint;    // EPI_KV_LOSS (set by launch_gemm; the type carries its alignment)
 };
 
 // ------------------------------------------------------------------ segment projection

@@ -19,16 +19,9 @@
 namespace cr {
 namespace {
 
-__device__ __forceinline__ float bf16_to_f32(uint16_t b) { return __uint_as_float(static_cast<uint32_t>(b) << 16); }
 __device__ __forceinline__ uint16_t f32_to_bf16(float x) {
     return __bfloat16_as_ushort(__float2bfloat16_rn(x));
 }
-template <typename T>
-__device__ __forceinline__ float ld(const T* p, int64_t i);
-template <>
-__device__ __forceinline__ float ld<uint16_t>(const uint16_t* p, int64_t i) { return bf16_to_f32(p[i]); }
-template <>
-__device__ __forceinline__ float ld<float>(const float* p, int64_t i) { return p[i]; }
 
 // the request of row t: req_start[r] <= t < req_start[r + 1]
 __device__ __forceinline__ int request_of(const LossParams& p, int64_t t) {
