@@ -408,7 +408,7 @@ def _recipes() -> Dict[str, Recipe]:
 
 
 RECIPES: Dict[str, Recipe] = _recipes()
-BASELINE_CONFIGS = ["tiny", "qwen3b", "llama8b", "qwen7b", "batched"]
+WORKLOAD_CONFIGS = ["tiny", "qwen3b", "llama8b", "qwen7b", "batched"]
 
 
 def make_case(name_or_recipe, **overrides) -> Case:

@@ -19,7 +19,7 @@ Cache Fusion" (arxiv 2609.35139).  Section references are to that paper:
             is affine, b + col(W_out).
   App. I    Cache payload 2 N D_KV bytes (bf16).
 
-Readings where the paper is silent (each repeated in the design doc):
+Readings where the paper is silent:
   R1  Widths: the StaleEncoder and P_tok output width d_c; F: 2 d_c -> d_b;
       P_b: d_c -> d_b; backbone and head at d_b.  With d_c = d_b this is the
       paper's single width.

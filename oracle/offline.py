@@ -12,7 +12,7 @@ tests; the product path never imports it.
             per D_KV coordinate.  sigma_stale is taken over stale caches,
             sigma_Delta over the residual targets KV_joint^c - KV_stale^c.
 
-Reading (R17, also in the design doc): the inverse rotation is the same
+Reading (R17): the inverse rotation is the same
 rotate-half rotation as R_M (R10) with the angle negated, computed exactly
 and rounded once to the cache dtype (R11); the RMS is sqrt(mean of squares)
 over all tokens given, without centring.

@@ -20,7 +20,7 @@ written out by hand step by step in reverse order.  Matrices enter the
 forward as the bf16 rounding of their fp32 masters (the GPU's mixed
 precision); the gradient is taken with respect to those values.
 
-Readings (each repeated in the design doc):
+Readings:
   R21 A batch of several requests is trained on the mean of the per-request
       losses (each normalised by its own N D_KV).
   R22 Unit gradient clipping is clipping of the global L2 norm over all

@@ -15,7 +15,7 @@ tests; the product path never imports it.
             (zero output offset), whose normalised target is
             KV^c_joint / sigma_Delta.
 
-Readings (each repeated in the design doc):
+Readings:
   R19 Under an output choice, every coordinate that is not repaired keeps its
       stale value exactly; with the target's R_M every K segment still leaves
       rotated, repaired or not (the other component's "stale value" is that of
