@@ -194,6 +194,24 @@ def oracle_sample(case, n_chunks, max_tokens=None, mask="block_causal"):
     return len(cid), time.perf_counter() - t0
 
 
+def max_over_ranks(ms, device):
+    """The slowest rank's time: every rank of the process group passes its own and
+    gets the maximum (no process group, or one rank: the value itself)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(ms)
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world, tokens_per_rank, steps, total_ms):
+    """Weak scaling: every rank repairs its own tokens_per_rank per step; the rate is
+    all ranks' tokens over the slowest rank's time."""
+    return world * tokens_per_rank * steps / (total_ms / 1e3)
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -324,12 +342,8 @@ def run_ours(args):
     torch.cuda.synchronize()
     clocks = stop_clocks(clk, t_begin, t_end)
     per_step = [evs[i].elapsed_time(evs[i + 1]) for i in range(args.steps)]
-    total_ms = evs[0].elapsed_time(evs[-1])
-    if world > 1:
-        tt = torch.tensor([total_ms], device="cuda")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms = float(tt.item())
-    value = world * N * args.steps / (total_ms / 1e3)
+    total_ms = max_over_ranks(evs[0].elapsed_time(evs[-1]), "cuda")
+    value = whole_job_rate(world, N, args.steps, total_ms)
     st, word = cr.cr_get_device_status()
     if st != cr.CR_OK:
         raise RuntimeError(f"device status {word}")
