@@ -427,7 +427,10 @@ size_t cr_train_workspace_bytes(const cr_target_dims* target, const cr_repairer_
  * cr_assemble_stale; cu_seqlens_host [n_req + 1] HOST.  stats_out: device
  * fp32 [4] = loss, gradient norm before clipping, clipping coefficient, 0.
  * The forward computes as cr_compress_features + cr_repair_forward (its
- * attention also keeps each row's log-sum-exp); the attention backward is
+ * attention also keeps each row's log-sum-exp); the head and the objective
+ * are one GEMM whose epilogue forms the residual from the staged kv_stale and
+ * kv_joint tiles and writes dL/dz (bf16) and the rows' squared residuals,
+ * never the residual itself; the attention backward is
  * fused (P recomputed tile by tile, no score matrix in memory); the backward's
  * plain matrix products (weight and input gradients) run in cuBLAS (bf16
  * operands, fp32 accumulation), using a part of the workspace as cuBLAS's
