@@ -39,6 +39,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "repaired doc tokens/s and p50 repair latency per request (1 GB300, % roofline)"
+L2_BYTES = 129 * 1000 * 1000
 
 
 def parse():
@@ -328,22 +329,37 @@ def run_ours(args):
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
+    # Inputs smaller than twice the L2 (129 MB): a 512 MB buffer is written between
+    # steps, outside each step's events, so every step starts from a cold L2.
+    es_c = 2 if case.target.cache_dtype == "bf16" else 4
+    cache_bytes = N * case.target.d_kv * es_c
+    flush = None
+    if cache_bytes < 2 * L2_BYTES:
+        flush = torch.empty(4 * L2_BYTES, dtype=torch.uint8, device="cuda")
     clk = sample_clocks(local)
-    evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    ev0 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ev1 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     t_begin = time.time()
-    evs[0].record(stream)
     for i in range(args.steps):
+        if flush is not None:
+            flush.zero_()
+        ev0[i].record(stream)
         run()
-        evs[i + 1].record(stream)
+        ev1[i].record(stream)
     torch.cuda.synchronize()
     t_end = time.time()
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
     clocks = stop_clocks(clk, t_begin, t_end)
-    per_step = [evs[i].elapsed_time(evs[i + 1]) for i in range(args.steps)]
-    total_ms = max_over_ranks(evs[0].elapsed_time(evs[-1]), "cuda")
+    per_step = [ev0[i].elapsed_time(ev1[i]) for i in range(args.steps)]
+    total_ms = max_over_ranks(sum(per_step), "cuda")
     value = whole_job_rate(world, N, args.steps, total_ms)
+    l2_note = (f"L2 flushed between steps (512 MB written outside the timed events): the "
+               f"assembled cache ({cache_bytes / 1e6:.0f} MB) is under twice the 129 MB L2"
+               if flush is not None else
+               f"no flush: the assembled cache ({cache_bytes / 1e6:.0f} MB) and the pool exceed the "
+               f"129 MB L2")
     st, word = cr.cr_get_device_status()
     if st != cr.CR_OK:
         raise RuntimeError(f"device status {word}")
@@ -377,11 +393,13 @@ def run_ours(args):
     dom_key = max(kernels, key=lambda k: kernels[k]["launches"] * kernels[k]["ms"])
     dom = kernels[dom_key]
     achieved = dom["flops"] / (dom["ms"] * 1e-3) / 1e12
-    roofline = {"kernel": dom["name"], "bound": "tensor", "achieved": achieved, "peak": tf_sus,
-                "unit": "TFLOP/s", "frac": achieved / tf_sus,
+    # the kernel is timed in isolated calls (ten eager launches, CUDA events): the
+    # burst peak applies
+    roofline = {"kernel": dom["name"], "bound": "tensor", "achieved": achieved, "peak": tf_burst,
+                "unit": "TFLOP/s", "frac": achieved / tf_burst,
                 # DRAM counters were taken on the method's workload, not on a variant
                 "traffic": None if args.variant else traffic_from_profiles(dom_key),
-                "peak_source": f"{src} bf16_tflops_sustained (kernel timed inside the step loop)",
+                "peak_source": f"{src} bf16_tflops (burst: the kernel timed in isolated calls)",
                 "algorithmic": dom["algorithmic"], "launch_ms": dom["ms"],
                 "launches_per_step": dom["launches"]}
     stage_roofline = {
@@ -391,9 +409,10 @@ def run_ours(args):
         # encoder's small GEMMs, over the whole call
         "front_hbm_frac": gather_bytes / (stages["assemble_compress"] * 1e-3) / 1e9 / hbm,
         "front_ms": stages["assemble_compress"],
-        "attention_tensor_frac": attn_flops / (attn_ms * 1e-3) / 1e12 / tf_sus,
+        "attention_tensor_frac": attn_flops / (attn_ms * 1e-3) / 1e12 / tf_burst,
         "attention_ms_per_launch": attn_ms,
-        "head_tensor_frac": head_flops / (head_ms * 1e-3) / 1e12 / tf_sus,
+        "head_tensor_frac": head_flops / (head_ms * 1e-3) / 1e12 / tf_burst,
+        "peaks": f"{src}: HBM {hbm} GB/s, bf16 {tf_burst} TF/s burst for isolated kernels",
         "head_ms": head_ms,
     }
     # front: gather (embeddings + chunk map), sigma fold, projection, four encoder
@@ -420,7 +439,7 @@ def run_ours(args):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded caches, embeddings, chunk map; random-init Xavier repairer)",
             "config": {"workload": workload_desc(case), "n_tokens": N, "cuda_graph": use_graph,
-                       "l2": "no flush: pool 1 GiB and assembled cache 0.67 GB exceed L2",
+                       "l2": l2_note,
                        "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                        **({"variant": args.variant} if args.variant else {})},
             "roofline": roofline, "stage_roofline": stage_roofline,

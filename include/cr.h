@@ -195,12 +195,18 @@ cr_status cr_assemble_stale(const cr_target_dims* target, const void* kv_pool,
  *   r_b   = P_b(s)  for every block b (stale-feature reinjection)
  * kv [N, D_KV], emb [N, d_model] (cache dtype, from cr_assemble_stale).
  * h0_out   [N, d_b] fp32  backbone input h^0.
- * rein_out [N, B d_b] bf16  P_b(s_t) at columns b*d_b .. (b+1)*d_b.
+ * rein_out [N, B d_b] fp32  P_b(s_t) at columns b*d_b .. (b+1)*d_b.
+ * Precision: the tensor cores take bf16 operands; the intermediate features
+ * (the segment outputs, s and the embedding projection) enter the next
+ * linear as two bf16 terms (value = hi + lo, about 16 significant bits), and
+ * W_seg / sigma_stale likewise, so that no bf16 rounding of the encoder's
+ * features reaches h^0 or the P_b(s), which every block adds into its
+ * residual stream.
  * workspace: cr_workspace_bytes(.., max_tokens >= N) bytes, 256-B aligned.
  */
 cr_status cr_compress_features(const cr_target_dims* target, const cr_repairer_dims* rep,
                                const cr_weights* w, const void* kv, const void* emb,
-                               int64_t n_tokens, float* h0_out, uint16_t* rein_out,
+                               int64_t n_tokens, float* h0_out, float* rein_out,
                                void* workspace, size_t workspace_bytes, void* stream);
 
 /*
@@ -221,7 +227,7 @@ cr_status cr_assemble_compress(const cr_target_dims* target, const cr_repairer_d
                                const int32_t* chunk_idx, const int32_t* cu_chunks, int32_t n_req,
                                void* kv_out, void* emb_out, int64_t max_tokens, int32_t* chunk_id,
                                int32_t* chunk_end, int32_t* pos, int32_t* cu_seqlens_dev,
-                               int32_t* cu_seqlens_host, float* h0_out, uint16_t* rein_out,
+                               int32_t* cu_seqlens_host, float* h0_out, float* rein_out,
                                void* workspace, size_t workspace_bytes, void* stream);
 
 /*
@@ -229,12 +235,12 @@ cr_status cr_assemble_compress(const cr_target_dims* target, const cr_repairer_d
  *   h^b = RepairBlock_b(h^{b-1} + P_b(s); A, p),   y_f = LN(h^B)
  * with the block-causal mask A_ij = 1[c(j) <= c(i)] inside each request and
  * the repairer's RoPE on Q, K at positions p.
- * h0 [N, d_b] fp32 and rein [N, B d_b] bf16 from cr_compress_features;
+ * h0 [N, d_b] fp32 and rein [N, B d_b] fp32 from cr_compress_features;
  * chunk_end, pos [N] from cr_assemble_stale; cu_seqlens_host [n_req+1] HOST.
  * yf_out [N, d_b] bf16.
  */
 cr_status cr_repair_forward(const cr_target_dims* target, const cr_repairer_dims* rep,
-                            const cr_weights* w, const float* h0, const uint16_t* rein,
+                            const cr_weights* w, const float* h0, const float* rein,
                             const int32_t* chunk_end, const int32_t* pos,
                             const int32_t* cu_seqlens_host, int32_t n_req, int64_t n_tokens,
                             uint16_t* yf_out, void* workspace, size_t workspace_bytes,
@@ -251,7 +257,7 @@ cr_status cr_repair_forward(const cr_target_dims* target, const cr_repairer_dims
  * CR_ERR_INVALID_ARG before any launch.
  */
 cr_status cr_repair_forward_masked(const cr_target_dims* target, const cr_repairer_dims* rep,
-                                   const cr_weights* w, const float* h0, const uint16_t* rein,
+                                   const cr_weights* w, const float* h0, const float* rein,
                                    const int32_t* chunk_end, const int32_t* pos,
                                    const int32_t* cu_seqlens_host, int32_t n_req,
                                    int64_t n_tokens, int32_t mask_mode, uint16_t* yf_out,

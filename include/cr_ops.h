@@ -35,11 +35,11 @@ cr_status cr_linear(const uint16_t* A, int64_t lda, const uint16_t* W, const flo
 /*
  * cr_layernorm - u = LN(x + add) * gamma + beta per row (biased variance,
  * eps), fp32 statistics (R4).  x [M, D] fp32 (row stride D).  If `add` is
- * non-NULL ([M, D] bf16, row stride ld_add), x + add is also written to
- * x_out ([M, D] fp32; may equal x).  u [M, D] bf16.  D a multiple of 128,
- * at most 1024.
+ * non-NULL ([M, D] fp32, row stride ld_add, a multiple of 4), x + add is also
+ * written to x_out ([M, D] fp32; may equal x).  u [M, D] bf16.  D a multiple
+ * of 128, at most 1024.
  */
-cr_status cr_layernorm(const float* x, const uint16_t* add, int64_t ld_add, float* x_out,
+cr_status cr_layernorm(const float* x, const float* add, int64_t ld_add, float* x_out,
                        const float* gamma, const float* beta, float eps, int64_t M, int64_t D,
                        uint16_t* u, void* stream);
 
@@ -105,8 +105,9 @@ cr_status cr_qkv_rope(const uint16_t* u, const uint16_t* w_qkv, const float* b_q
  * cr_segment_project - StaleEncoder stage 1 (Sec. 4.1):
  *   y[t, s*d_seg + k] = sum_d W_seg[s,k,d] kv[t, s*d_h + d] / sigma_stale[s*d_h + d]
  *                       + b_seg[s,k]
- * kv [N, D_KV] bf16; y [N, S*d_seg] bf16.  workspace: at least
- * S*d_seg*d_h*2 bytes (holds W_seg with 1/sigma folded in).
+ * kv [N, D_KV] bf16; y [N, S*d_seg] bf16 (fp32 sums rounded once).  workspace:
+ * at least S*d_seg*d_h*4 bytes (holds W_seg with 1/sigma folded in, as two
+ * bf16 terms per weight).
  */
 cr_status cr_segment_project(const cr_target_dims* target, int32_t d_seg, const uint16_t* kv,
                              int64_t n_tokens, const uint16_t* w_seg, const float* b_seg,
@@ -120,10 +121,11 @@ cr_status cr_segment_project(const cr_target_dims* target, int32_t d_seg, const 
  * cudaMalloc, which can synchronise the device).  The paper has no
  * counterpart: this is a deployment variant of the same computation.
  *
- * Its scratch (W_seg with 1/sigma_stale folded in, S*d_seg*d_h bf16 values)
- * is a fixed 4 MiB device array inside the library, present on every GPU that
- * loads the library until the process exits.  Shapes needing more return
- * CR_ERR_UNSUPPORTED.  The first call on a device looks up that array's
+ * Its scratch (W_seg with 1/sigma_stale folded in, two bf16 terms for each of
+ * the S*d_seg*d_h weights) is a fixed 8 MiB device array inside the library,
+ * present on every GPU that loads the library until the process exits: at
+ * most S*d_seg*d_h = 2 Mi weights (the 8B-shape target has 1 Mi).  Larger
+ * shapes return CR_ERR_UNSUPPORTED.  The first call on a device looks up that array's
  * device address (cudaGetSymbolAddress); make that first call before any
  * stream capture.  All calls share the one array, so calls whose kernels
  * overlap on the GPU (different streams, no ordering between them) race on

@@ -9,3 +9,4 @@ from .cacherepair import *  # noqa: F401,F403
 from .offline import *  # noqa: F401,F403
 from .variants import *  # noqa: F401,F403
 from .training import *  # noqa: F401,F403
+from .serving import *  # noqa: F401,F403

@@ -60,6 +60,8 @@ Dims dims_of(const cr_target_dims* t, const cr_repairer_dims* r) {
     return d;
 }
 
+}  // namespace
+
 cr_status check_target(const cr_target_dims* t) {
     if (!t) return CR_ERR_INVALID_ARG;
     if (t->n_layers < 1 || t->n_kv_heads < 1 || t->d_model < 8 || (t->d_model % 8) != 0)
@@ -68,6 +70,8 @@ cr_status check_target(const cr_target_dims* t) {
     if (t->head_dim != 64 && t->head_dim != 128) return CR_ERR_UNSUPPORTED;
     return CR_OK;
 }
+
+namespace {
 
 cr_status check_repairer(const cr_repairer_dims* r) {
     if (!r) return CR_ERR_INVALID_ARG;
@@ -84,7 +88,7 @@ cr_status check_repairer(const cr_repairer_dims* r) {
 }
 
 struct WsLayout {
-    size_t wfold, kvb, embb, y, se, x, u, qkv, o, g, rope, kstart, total;
+    size_t wfold, kvb, embb, y, se32, se2, x, u, qkv, o, g, rope, kstart, total;
 };
 
 WsLayout ws_layout(const Dims& d, int64_t n) {
@@ -96,11 +100,12 @@ WsLayout ws_layout(const Dims& d, int64_t n) {
         return o;
     };
     const size_t N = static_cast<size_t>(n);
-    w.wfold = take(static_cast<size_t>(d.S * d.dseg * d.dh) * 2);
+    w.wfold = take(static_cast<size_t>(d.S * d.dseg * d.dh) * 2 * 2);   // hi and lo terms
     w.kvb = take(d.f32 ? N * d.D * 2 : 0);
     w.embb = take(d.f32 ? N * d.dmodel * 2 : 0);
-    w.y = take(N * d.S * d.dseg * 2);
-    w.se = take(N * 2 * d.dc * 2);
+    w.y = take(N * d.S * d.dseg * 2 * 2);   // per row [y_hi | y_lo]
+    w.se32 = take(N * 2 * d.dc * 4);        // per row [s ; e] fp32
+    w.se2 = take(N * 4 * d.dc * 2);         // per row [s_hi e_hi | s_lo e_lo]
     w.x = take(N * d.db * 4);
     w.u = take(N * d.db * 2);
     w.qkv = take(N * 3 * d.db * 2);
@@ -333,38 +338,46 @@ static cr_status check_weights_compress(const Dims& d, const cr_weights* w) {
 }
 
 // Stage 2 and token fusion of the encoder (Sec. 4.1): s = W_map y + b_map,
-// [s ; P_tok E] -> h^0 = F(.), and the reinjection terms P_b(s).
+// e = P_tok E + b_tok, h^0 = F([s ; e]) + b_fuse, and the reinjection terms
+// P_b(s) + b_rein.  The encoder's outputs feed the whole residual stream (h^0
+// and one P_b(s) per block), so no bf16 rounding is taken there: y comes in
+// as two bf16 terms per row ([y_hi | y_lo], from the segment projection); s
+// and e are formed in fp32 and split into two terms per row ([s_hi e_hi |
+// s_lo e_lo]) for F and the P_b, whose outputs h^0 and P_b(s) stay fp32.
 static cr_status compress_stage2(const Dims& d, const cr_weights* w, const uint16_t* y,
                                  const uint16_t* embb, int64_t N, float* h0_out,
-                                 uint16_t* rein_out, void* workspace, const WsLayout& L,
+                                 float* rein_out, void* workspace, const WsLayout& L,
                                  unsigned* status, cudaStream_t st) {
     cr_status s;
-    uint16_t* se = at<uint16_t>(workspace, L.se);   // [N, 2 d_c] = [s ; P_tok E]
+    float* se32 = at<float>(workspace, L.se32);      // [N, 2 d_c] = [s ; P_tok E]
+    uint16_t* se2 = at<uint16_t>(workspace, L.se2);  // [N, 4 d_c] two-term bf16
+    const int64_t Sd = d.S * d.dseg;
     GemmParams gp{};
     gp.status = status;
     gp.bias = w->b_map;
-    gp.out = se;
+    gp.out = se32;
     gp.ldo = 2 * d.dc;
-    if ((s = launch_gemm(y, d.S * d.dseg, w->w_map, N, d.dc, d.S * d.dseg, EPI_BF16, gp, nullptr,
-                         0, st)) != CR_OK)
+    if ((s = launch_gemm(y, 2 * Sd, w->w_map, N, d.dc, Sd, EPI_F32, gp, nullptr, 0, st,
+                         y + Sd)) != CR_OK)
         return s;
     gp.bias = w->b_tok;
-    gp.out = se + d.dc;
-    if ((s = launch_gemm(embb, d.dmodel, w->w_tok, N, d.dc, d.dmodel, EPI_BF16, gp, nullptr, 0,
+    gp.out = se32 + d.dc;
+    if ((s = launch_gemm(embb, d.dmodel, w->w_tok, N, d.dc, d.dmodel, EPI_F32, gp, nullptr, 0,
                          st)) != CR_OK)
         return s;
+    if ((s = launch_split_bf16(se32, N, 2 * d.dc, se2, st)) != CR_OK) return s;
     gp.bias = w->b_fuse;
     gp.out = h0_out;
     gp.ldo = d.db;
-    if ((s = launch_gemm(se, 2 * d.dc, w->w_fuse, N, d.db, 2 * d.dc, EPI_F32, gp, nullptr, 0,
-                         st)) != CR_OK)
+    if ((s = launch_gemm(se2, 4 * d.dc, w->w_fuse, N, d.db, 2 * d.dc, EPI_F32, gp, nullptr, 0,
+                         st, se2 + 2 * d.dc)) != CR_OK)
         return s;
     if (d.B > 0) {
         gp.bias = w->b_rein;
         gp.out = rein_out;
         gp.ldo = d.B * d.db;
-        if ((s = launch_gemm(se, 2 * d.dc, w->w_rein, N, d.B * d.db, d.dc, EPI_BF16, gp, nullptr,
-                             0, st)) != CR_OK)
+        if ((s = launch_gemm(se2, 4 * d.dc, w->w_rein, N, d.B * d.db, d.dc, EPI_F32, gp, nullptr,
+                             0, st, se2 + 2 * d.dc)) != CR_OK)
             return s;
     }
     return CR_OK;
@@ -377,7 +390,9 @@ static SegParams seg_params(const Dims& d, const cr_weights* w, int64_t N, uint1
     sp.S = static_cast<int32_t>(d.S);
     sp.d_seg = static_cast<int32_t>(d.dseg);
     sp.b_seg = w->b_seg;
-    sp.y = y;
+    sp.y = y;                     // per row [y_hi | y_lo]
+    sp.y_lo = y + d.S * d.dseg;
+    sp.ldy = 2 * d.S * d.dseg;
     sp.status = status;
     return sp;
 }
@@ -385,7 +400,7 @@ static SegParams seg_params(const Dims& d, const cr_weights* w, int64_t N, uint1
 // Argument checks shared by the encoder entry points; fills the workspace layout.
 static cr_status check_compress(const cr_target_dims* target, const cr_repairer_dims* rep,
                                 const cr_weights* w, int64_t max_tokens, float* h0_out,
-                                uint16_t* rein_out, void* workspace, size_t workspace_bytes,
+                                float* rein_out, void* workspace, size_t workspace_bytes,
                                 Dims* d, WsLayout* L) {
     cr_status s = check_target(target);
     if (s == CR_OK) s = check_repairer(rep);
@@ -402,7 +417,7 @@ static cr_status check_compress(const cr_target_dims* target, const cr_repairer_
 
 cr_status cr_compress_features(const cr_target_dims* target, const cr_repairer_dims* rep,
                                const cr_weights* w, const void* kv, const void* emb,
-                               int64_t n_tokens, float* h0_out, uint16_t* rein_out,
+                               int64_t n_tokens, float* h0_out, float* rein_out,
                                void* workspace, size_t workspace_bytes, void* stream) {
     Dims d;
     WsLayout L;
@@ -443,7 +458,7 @@ cr_status cr_assemble_compress(const cr_target_dims* target, const cr_repairer_d
                                const int32_t* chunk_idx, const int32_t* cu_chunks, int32_t n_req,
                                void* kv_out, void* emb_out, int64_t max_tokens, int32_t* chunk_id,
                                int32_t* chunk_end, int32_t* pos, int32_t* cu_seqlens_dev,
-                               int32_t* cu_seqlens_host, float* h0_out, uint16_t* rein_out,
+                               int32_t* cu_seqlens_host, float* h0_out, float* rein_out,
                                void* workspace, size_t workspace_bytes, void* stream) {
     Dims d;
     WsLayout L;
@@ -539,7 +554,7 @@ static cr_status attn_params(const Dims& d, int32_t mask_mode, const int32_t* ch
 }
 
 cr_status cr_repair_forward(const cr_target_dims* target, const cr_repairer_dims* rep,
-                            const cr_weights* w, const float* h0, const uint16_t* rein,
+                            const cr_weights* w, const float* h0, const float* rein,
                             const int32_t* chunk_end, const int32_t* pos,
                             const int32_t* cu_seqlens_host, int32_t n_req, int64_t n_tokens,
                             uint16_t* yf_out, void* workspace, size_t workspace_bytes,
@@ -550,7 +565,7 @@ cr_status cr_repair_forward(const cr_target_dims* target, const cr_repairer_dims
 }
 
 cr_status cr_repair_forward_masked(const cr_target_dims* target, const cr_repairer_dims* rep,
-                                   const cr_weights* w, const float* h0, const uint16_t* rein,
+                                   const cr_weights* w, const float* h0, const float* rein,
                                    const int32_t* chunk_end, const int32_t* pos,
                                    const int32_t* cu_seqlens_host, int32_t n_req,
                                    int64_t n_tokens, int32_t mask_mode, uint16_t* yf_out,
@@ -828,12 +843,12 @@ cr_status cr_linear(const uint16_t* A, int64_t lda, const uint16_t* W, const flo
                        static_cast<cudaStream_t>(stream));
 }
 
-cr_status cr_layernorm(const float* x, const uint16_t* add, int64_t ld_add, float* x_out,
+cr_status cr_layernorm(const float* x, const float* add, int64_t ld_add, float* x_out,
                        const float* gamma, const float* beta, float eps, int64_t M, int64_t D,
                        uint16_t* u, void* stream) {
     if (M < 1 || D < 128 || D > 1024 || (D % 128) != 0 || !(eps > 0.0f)) return CR_ERR_INVALID_ARG;
     if (!all_aligned(x, gamma, beta, u)) return CR_ERR_INVALID_ARG;
-    if (add && (!all_aligned(add, x_out) || ld_add < D || (ld_add % 8) != 0))
+    if (add && (!all_aligned(add, x_out) || ld_add < D || (ld_add % 4) != 0))
         return CR_ERR_INVALID_ARG;
     return launch_layernorm(x, add, ld_add, x_out, gamma, beta, eps, M, D, u,
                             static_cast<cudaStream_t>(stream));
@@ -940,7 +955,7 @@ cr_status cr_segment_project(const cr_target_dims* target, int32_t d_seg, const 
     if (n_tokens < 1 || n_tokens > INT32_MAX / 2) return CR_ERR_INVALID_ARG;
     if (!all_aligned(kv, w_seg, b_seg, sigma_stale, y, workspace)) return CR_ERR_INVALID_ARG;
     const Dims d = dims_of(target, nullptr);
-    if (workspace_bytes < static_cast<size_t>(d.S * d_seg * d.dh) * 2) return CR_ERR_INVALID_ARG;
+    if (workspace_bytes < static_cast<size_t>(d.S * d_seg * d.dh) * 4) return CR_ERR_INVALID_ARG;
     unsigned* status = device_status_ptr();
     if (!status) return CR_ERR_CUDA;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -954,6 +969,7 @@ cr_status cr_segment_project(const cr_target_dims* target, int32_t d_seg, const 
     sp.d_seg = d_seg;
     sp.b_seg = b_seg;
     sp.y = y;
+    sp.ldy = d.S * d_seg;
     sp.status = status;
     return launch_segproj(kv, d.D, wfold, static_cast<int>(d.dh), sp, st);
 }
@@ -1039,7 +1055,7 @@ TrainLayout train_layout(const Dims& d, int64_t n) {
     const size_t N = static_cast<size_t>(n);
     L.inf = take(ws_layout(d, n).total);
     L.h0 = take(N * d.db * 4);
-    L.rein = take(N * (d.B > 0 ? d.B : 1) * d.db * 2);
+    L.rein = take(N * (d.B > 0 ? d.B : 1) * d.db * 4);
     // per block: x_in, x_mid (fp32), u1, u2 (bf16), qkv (bf16), o (bf16), g (bf16)
     size_t bo = 0;
     auto btake = [&](size_t bytes) {
@@ -1188,10 +1204,12 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
     uint8_t* base = static_cast<uint8_t*>(workspace);
     void* inf = base + L.inf;
     const WsLayout IL = ws_layout(d, N);
-    const uint16_t* y = at<uint16_t>(inf, IL.y);      // [N, S d_seg] after compress
-    const uint16_t* se = at<uint16_t>(inf, IL.se);    // [N, 2 d_c] = [s ; e]
+    // after compress: y rows [y_hi | y_lo], se rows [s_hi e_hi | s_lo e_lo]; the
+    // weight gradients take the hi terms as their bf16 operands
+    const uint16_t* y = at<uint16_t>(inf, IL.y);
+    const uint16_t* se = at<uint16_t>(inf, IL.se2);
     float* h0 = at<float>(base, L.h0);
-    uint16_t* rein = at<uint16_t>(base, L.rein);
+    float* rein = at<float>(base, L.rein);
     auto blk = [&](int64_t b, size_t o) { return base + L.blk + static_cast<size_t>(b) * L.blk_stride + o; };
     float* H = at<float>(base, L.hbuf);
     uint16_t* yf = at<uint16_t>(base, L.yf);
@@ -1397,14 +1415,14 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
         CR_TRY(colsum(DU, false, db, db, gk(bk(b, LN1B))));
         // x_in = h^{b-1} + W_rein,b s + b_rein,b: ds += dx_in W_rein,b
         CR_TRY(colsum16(DH, db, SIG, gk(B_REIN) + b * db));
-        CR_TRY(gemm_rm(hb, true, false, db, dc, N, 1.0f, SIG, BF, db, se, BF, 2 * dc, 0.0f, gk(W_REIN) + b * db * dc,
+        CR_TRY(gemm_rm(hb, true, false, db, dc, N, 1.0f, SIG, BF, db, se, BF, 4 * dc, 0.0f, gk(W_REIN) + b * db * dc,
                        F32, dc));
         CR_TRY(gemm_rm(hb, false, false, N, dc, db, 1.0f, SIG, BF, db, pb(W_REIN) + b * db * dc, BF, dc, 1.0f, DSE,
                        F32, 2 * dc));
     }
     // h0 = W_fuse [s; e] + b_fuse
     CR_TRY(colsum16(DH, db, SIG, gk(B_FUSE)));
-    CR_TRY(gemm_rm(hb, true, false, db, 2 * dc, N, 1.0f, SIG, BF, db, se, BF, 2 * dc, 0.0f, gk(W_FUSE), F32, 2 * dc));
+    CR_TRY(gemm_rm(hb, true, false, db, 2 * dc, N, 1.0f, SIG, BF, db, se, BF, 4 * dc, 0.0f, gk(W_FUSE), F32, 2 * dc));
     CR_TRY(gemm_rm(hb, false, false, N, 2 * dc, db, 1.0f, SIG, BF, db, pb(W_FUSE), BF, 2 * dc, 1.0f, DSE, F32,
                    2 * dc));
     // e = W_tok emb + b_tok;  s = W_map y + b_map
@@ -1413,7 +1431,7 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
                    F32, d.dmodel));
     CR_TRY(colsum(DSE + dc, false, dc, 2 * dc, gk(B_TOK)));
     const int64_t Sd = d.S * d.dseg;
-    CR_TRY(gemm_rm(hb, true, false, dc, Sd, N, 1.0f, SIG, BF, 2 * dc, y, BF, Sd, 0.0f, gk(W_MAP), F32, Sd));
+    CR_TRY(gemm_rm(hb, true, false, dc, Sd, N, 1.0f, SIG, BF, 2 * dc, y, BF, 2 * Sd, 0.0f, gk(W_MAP), F32, Sd));
     CR_TRY(colsum(DSE, false, dc, 2 * dc, gk(B_MAP)));
     CR_TRY(gemm_rm(hb, false, false, N, Sd, dc, 1.0f, SIG, BF, 2 * dc, pb(W_MAP), BF, Sd, 0.0f, DY, F32, Sd));
     // y_{t,s} = (W_seg,s / sigma_stale) kv_{t,s} + b_seg,s: per segment dy^T kv, then / sigma_stale

@@ -336,7 +336,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const WaitCtx wc{abort_flag, p.status};
 
     const int total = p.num_m * p.num_n;
-    const int num_k = (p.K + BK - 1) / BK;
+    // a two-term A runs the W k-blocks twice: first against A_hi, then A_lo
+    const int num_k = p.split_kb > 0 ? 2 * p.split_kb : (p.K + BK - 1) / BK;
     const bool has_bias = p.bias != nullptr;
     // the epilogue consumes a per-tile load (vectors and/or the in-place tile)
     const bool epi_load = Cfg::kInPlace || has_bias;
@@ -353,6 +354,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         if (elect_one()) {
             tma_prefetch(&tmA);
             tma_prefetch(&tmB);
+            if (p.split_kb > 0) tma_prefetch(&p.tm_alo);
             if constexpr (Cfg::kInPlace) tma_prefetch(&tmC);
         }
         __syncwarp();
@@ -366,17 +368,20 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 uint8_t* sa = smem + stage * Cfg::kStageBytes;
                 if (elect_one()) {
                     const int nb0 = n0 + static_cast<int>(rank) * (BN / CG);
+                    const bool lo = p.split_kb > 0 && kb >= p.split_kb;
+                    const CUtensorMap* ma = lo ? &p.tm_alo : &tmA;
+                    const int ka = (lo ? kb - p.split_kb : kb) * BK;   // A and W column
                     if (CG == 1) {
                         mbar_expect_tx(&full[stage], Cfg::kStageBytes);
-                        tma_load_2d(sa, &tmA, &full[stage], kb * BK, m0);
-                        tma_load_2d(sa + A_BYTES, &tmB, &full[stage], kb * BK, nb0);
+                        tma_load_2d(sa, ma, &full[stage], ka, m0);
+                        tma_load_2d(sa + A_BYTES, &tmB, &full[stage], ka, nb0);
                     } else {
                         // both CTAs' copies count on the even CTA's barrier, which
                         // expects the pair's bytes (its own arrive is the only one)
                         const uint32_t fb = mapa_shared(smem_u32(&full[stage]), 0);
                         if (rank == 0) mbar_expect_tx(&full[stage], CG * Cfg::kStageBytes);
-                        tma_load_2d_pair(sa, &tmA, fb, kb * BK, m0);
-                        tma_load_2d_pair(sa + A_BYTES, &tmB, fb, kb * BK, nb0);
+                        tma_load_2d_pair(sa, ma, fb, ka, m0);
+                        tma_load_2d_pair(sa + A_BYTES, &tmB, fb, ka, nb0);
                     }
                 }
                 __syncwarp();
@@ -955,7 +960,7 @@ constexpr int kCG = 2;
 
 cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t M, int64_t N,
                       int64_t K, int epi, GemmParams p, void* kv_base, int64_t ld_kv,
-                      cudaStream_t st) {
+                      cudaStream_t st, const uint16_t* A_lo) {
     const bool kv = (epi == EPI_KV_BF16 || epi == EPI_KV_F32 || epi == EPI_KV_PAGED || epi == EPI_KV_LOSS);
     const bool f32_tile = (epi == EPI_KV_F32 || epi == EPI_ADD_F32);
     // Tile width.  Per 64-deep k-block a CTA of a pair moves 32 KB + 128 BN
@@ -968,8 +973,6 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
     int BN;
     if (kv) {
         BN = (epi == EPI_KV_F32 || epi == EPI_KV_LOSS) ? 128 : 256;
-    } else if (epi == EPI_F32) {
-        BN = 128;
     } else {
         const int64_t pairs = num_sms() / kCG > 0 ? num_sms() / kCG : 1;
         const int64_t mt = (M + BM * kCG - 1) / (BM * kCG);
@@ -1010,6 +1013,15 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
     if (!make_tmap_2d(&ta, A, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, K, M, lda * 2, BK, BM,
                       CU_TENSOR_MAP_SWIZZLE_128B))
         return CR_ERR_INVALID_ARG;
+    p.split_kb = 0;
+    if (A_lo) {
+        // columns past K read as zeros in both terms (TMA bounds), so the two
+        // k-loops line up with the same W k-blocks
+        if (!make_tmap_2d(&p.tm_alo, A_lo, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, K, M, lda * 2, BK, BM,
+                          CU_TENSOR_MAP_SWIZZLE_128B))
+            return CR_ERR_INVALID_ARG;
+        p.split_kb = static_cast<int32_t>((K + BK - 1) / BK);
+    }
     if (!make_tmap_2d(&tb, W, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, K, N, K * 2, BK, BN / kCG,
                       CU_TENSOR_MAP_SWIZZLE_128B))
         return CR_ERR_INVALID_ARG;
@@ -1035,7 +1047,9 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
             return BN == 160 ? launch_bn<160, EPI_ADD_F32, kCG>(ta, tb, tc, p, st)
                              : launch_bn<128, EPI_ADD_F32, kCG>(ta, tb, tc, p, st);
         case EPI_F32:
-            return launch_bn<128, EPI_F32, kCG>(ta, tb, tc, p, st);
+            return BN == 256   ? launch_bn<256, EPI_F32, kCG>(ta, tb, tc, p, st)
+                   : BN == 192 ? launch_bn<192, EPI_F32, kCG>(ta, tb, tc, p, st)
+                               : launch_bn<128, EPI_F32, kCG>(ta, tb, tc, p, st);
         case EPI_QKV_ROPE:
             return BN == 256   ? launch_bn<256, EPI_QKV_ROPE, kCG>(ta, tb, tc, p, st)
                    : BN == 192 ? launch_bn<192, EPI_QKV_ROPE, kCG>(ta, tb, tc, p, st)

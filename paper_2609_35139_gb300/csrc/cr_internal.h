@@ -97,8 +97,14 @@ struct GemmParams {
     const float* row_scale;
     float* loss_part;
     unsigned* status;
+    // two-term A (set by launch_gemm when A_lo is given): A = A_hi + A_lo, both
+    // bf16 [M, K]; the k-loop runs over the split_kb k-blocks of A_hi, then the
+    // same k-blocks of A_lo (tm_alo) against the same W columns, into one
+    // accumulator: A at about 16 significant bits for twice the MMAs.  0 = plain A.
+    int32_t split_kb;
     float inv_freq[64];      // RoPE frequencies, rope_dim / 2 entries
     CUtensorMap tm_joint;    // EPI_KV_LOSS (set by launch_gemm; the type carries its alignment)
+    CUtensorMap tm_alo;      // two-term A: the A_lo operand
 };
 
 // ------------------------------------------------------------------ segment projection
@@ -108,7 +114,9 @@ struct SegParams {
     int32_t d_seg;       // 8 or 16
     int32_t num_m, num_g;
     const float* b_seg;  // [S, d_seg]
-    uint16_t* y;         // [M, S * d_seg]
+    uint16_t* y;         // [M, S * d_seg] bf16 (row stride ldy)
+    uint16_t* y_lo;      // [M, S * d_seg] remainder y - bf16(y) (row stride ldy), or null
+    int64_t ldy;
     unsigned* status;
     uint16_t* kv_out;    // pool variant: assembled cache [M, ld_out]
     int64_t ld_out;
@@ -167,6 +175,8 @@ struct AdamWParams {
 };
 
 // ------------------------------------------------------------------ host helpers
+// Target-shape validation shared by every entry point that takes cr_target_dims.
+cr_status check_target(const cr_target_dims* t);
 unsigned* device_status_ptr();          // per current device, nullptr on failure
 int num_sms();                          // SMs of the current device
 cr_status cuda_check(cudaError_t e);
@@ -224,9 +234,11 @@ cr_status launch_sigma_accumulate(const void* a, const void* b, bool f32, int64_
                                   float* part, double* sumsq, cudaStream_t st);
 cr_status launch_sigma_finalize(const double* sumsq, int64_t D, int64_t count, float* sigma,
                                 cudaStream_t st);
+// A_lo (optional): the second term of a two-term A operand (same shape and
+// row stride as A); the product is then (A + A_lo) W^T.
 cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t M, int64_t N,
                       int64_t K, int epi, GemmParams p, void* kv_base, int64_t ld_kv,
-                      cudaStream_t st);
+                      cudaStream_t st, const uint16_t* A_lo = nullptr);
 cr_status launch_segproj(const uint16_t* kv, int64_t ld_kv, const uint16_t* wfold, int head_dim,
                          SegParams p, cudaStream_t st);
 // The same projection reading the cache tiles straight from the pool (rows
@@ -238,9 +250,13 @@ cr_status launch_segproj_pool(const uint16_t* kv_pool, int64_t n_pool_tokens, ui
 cr_status launch_fold_sigma(const uint16_t* w_seg, const float* sigma, int S, int d_seg,
                             int head_dim, uint16_t* wfold, cudaStream_t st);
 cr_status launch_to_bf16(const float* x, int64_t n, uint16_t* y, cudaStream_t st);
+// x [rows, cols] fp32 -> out [rows, 2 cols] bf16: each row's hi = rn(x) terms,
+// then its lo = rn(x - hi) terms (a two-term A operand for launch_gemm).
+cr_status launch_split_bf16(const float* x, int64_t rows, int64_t cols, uint16_t* out,
+                            cudaStream_t st);
 cr_status launch_rope_table(const int32_t* pos, int64_t n, int half_dim, const float* inv_freq_host,
                             float2* table, cudaStream_t st);
-cr_status launch_layernorm(const float* x, const uint16_t* add, int64_t ld_add, float* x_out,
+cr_status launch_layernorm(const float* x, const float* add, int64_t ld_add, float* x_out,
                            const float* g, const float* b, float eps, int64_t M, int64_t D,
                            uint16_t* u, cudaStream_t st);
 cr_status launch_wait_selftest(unsigned* status, cudaStream_t st);

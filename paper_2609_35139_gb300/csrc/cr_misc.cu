@@ -6,6 +6,7 @@
 //   layernorm_kernel  LayerNorm of the residual stream (optionally adding the
 //                     block's reinjection P_b(s) first, Sec. 4.1 eq. for h^b)
 //   to_bf16_kernel    fp32 cache/embedding -> bf16 operands for the tensor cores
+//   split_bf16_kernel fp32 -> two-term bf16 operand (hi, lo) for the tensor cores
 #include <cuda_bf16.h>
 
 #include "cr_internal.h"
@@ -118,14 +119,12 @@ __global__ void __launch_bounds__(256) gather_emb_kernel(const __grid_constant__
             p.cu_seqlens[i] = p.cu_seqlens_host[i];
 }
 
-__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
 // One warp per row, VPL float4 per lane (D = 128 * VPL); two-pass statistics
 // from registers (mean, then mean squared deviation: biased variance).
 template <int VPL>
 __global__ void __launch_bounds__(256) layernorm_kernel(const float* x,
-                                                        const uint16_t* __restrict__ add,
+                                                        const float* __restrict__ add,
                                                         int64_t ld_add, float* x_out,
                                                         const float* __restrict__ g,
                                                         const float* __restrict__ b, float eps,
@@ -138,15 +137,14 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const float* x,
     if (row >= M) return;
     // every load of the row (x, the reinjection term, gamma, beta) is issued
     // before the first use: one memory round trip per row
-    float4 v[VPL], gg[VPL], bq[VPL];
-    uint2 av[VPL];
+    float4 v[VPL], gg[VPL], bq[VPL], av[VPL];
     const float4* xr = reinterpret_cast<const float4*>(x + row * D);
     const float4* g4 = reinterpret_cast<const float4*>(g);
     const float4* b4 = reinterpret_cast<const float4*>(b);
 #pragma unroll
     for (int k = 0; k < VPL; ++k) v[k] = xr[lane + 32 * k];
     if (add) {
-        const uint2* ar = reinterpret_cast<const uint2*>(add + row * ld_add);
+        const float4* ar = reinterpret_cast<const float4*>(add + row * ld_add);
 #pragma unroll
         for (int k = 0; k < VPL; ++k) av[k] = ar[lane + 32 * k];
     }
@@ -159,11 +157,10 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const float* x,
         float4* xo = reinterpret_cast<float4*>(x_out + row * D);
 #pragma unroll
         for (int k = 0; k < VPL; ++k) {
-            const uint2 a = av[k];
-            v[k].x += bf16_lo(a.x);
-            v[k].y += bf16_hi(a.x);
-            v[k].z += bf16_lo(a.y);
-            v[k].w += bf16_hi(a.y);
+            v[k].x += av[k].x;
+            v[k].y += av[k].y;
+            v[k].z += av[k].z;
+            v[k].w += av[k].w;
             xo[lane + 32 * k] = v[k];
         }
     }
@@ -201,6 +198,31 @@ __global__ void to_bf16_kernel(const float* __restrict__ x, int64_t n, uint16_t*
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const __nv_bfloat16 b = __float2bfloat16_rn(x[i]);
         y[i] = *reinterpret_cast<const uint16_t*>(&b);
+    }
+}
+
+// Two-term bf16 operand of an fp32 matrix: x [rows, cols] fp32 (contiguous)
+// -> out row r = [hi (cols) | lo (cols)], hi = rn(x), lo = rn(x - hi); eight
+// values per thread.  cols is a multiple of 8.
+__global__ void split_bf16_kernel(const float* __restrict__ x, int64_t rows, int64_t cols,
+                                  uint16_t* __restrict__ out) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int64_t c8 = cols >> 3;
+    const int64_t n8 = rows * c8;
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n8;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t r = i / c8, c = (i - r * c8) << 3;
+        const float4* src = reinterpret_cast<const float4*>(x + r * cols + c);
+        const float4 a = src[0], b = src[1];
+        uint32_t h[4], l[4];
+        split_bf16x2(a.x, a.y, &h[0], &l[0]);
+        split_bf16x2(a.z, a.w, &h[1], &l[1]);
+        split_bf16x2(b.x, b.y, &h[2], &l[2]);
+        split_bf16x2(b.z, b.w, &h[3], &l[3]);
+        uint16_t* o = out + r * 2 * cols + c;
+        *reinterpret_cast<uint4*>(o) = make_uint4(h[0], h[1], h[2], h[3]);
+        *reinterpret_cast<uint4*>(o + cols) = make_uint4(l[0], l[1], l[2], l[3]);
     }
 }
 
@@ -251,7 +273,7 @@ cr_status launch_gather(const GatherParams& p, cudaStream_t st) {
     return launch_pdl(gather_kernel, dim3(static_cast<unsigned>(grid)), dim3(512), 0, st, p);
 }
 
-cr_status launch_layernorm(const float* x, const uint16_t* add, int64_t ld_add, float* x_out,
+cr_status launch_layernorm(const float* x, const float* add, int64_t ld_add, float* x_out,
                            const float* g, const float* b, float eps, int64_t M, int64_t D,
                            uint16_t* u, cudaStream_t st) {
     if (M <= 0) return CR_OK;
@@ -274,6 +296,17 @@ cr_status launch_layernorm(const float* x, const uint16_t* add, int64_t ld_add, 
         default:
             return CR_ERR_UNSUPPORTED;
     }
+}
+
+cr_status launch_split_bf16(const float* x, int64_t rows, int64_t cols, uint16_t* out,
+                            cudaStream_t st) {
+    if (rows <= 0) return CR_OK;
+    if ((cols % 8) != 0) return CR_ERR_UNSUPPORTED;
+    const int64_t n8 = rows * (cols / 8);
+    int64_t blocks = (n8 + 255) / 256;
+    if (blocks > 8 * 1024) blocks = 8 * 1024;
+    return launch_pdl(split_bf16_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st, x,
+                      rows, cols, out);
 }
 
 cr_status launch_to_bf16(const float* x, int64_t n, uint16_t* y, cudaStream_t st) {

@@ -6,18 +6,18 @@
 // budget, a real-time serving loop that must never call cudaMalloc (it can
 // synchronise the device and stall every stream), or code running where the
 // allocator is unavailable.  This entry point needs no workspace: its only
-// scratch, the weight copy with 1/sigma_stale folded in, lives in a file-scope
-// device array of fixed size that every GPU loading the library holds until the
-// process exits.
+// scratch, the weight copy with 1/sigma_stale folded in (two bf16 terms per
+// weight), lives in a file-scope device array of fixed size that every GPU
+// loading the library holds until the process exits.
 #include <mutex>
 
 #include "cr_internal.h"
 
-// Largest folded weight copy this entry point accepts: S * d_seg * d_h bf16
-// values, 4 MiB (the 8B-shape target needs 2 MiB).
+// Largest weight this entry point accepts: S * d_seg * d_h values (the 8B-shape
+// target has 1 Mi).  The folded copy keeps two bf16 terms per value: 8 MiB.
 #define CR_NOALLOC_SCRATCH_ELEMS (2u * 1024u * 1024u)
 
-static __device__ __align__(256) uint16_t g_noalloc_scratch[CR_NOALLOC_SCRATCH_ELEMS];
+static __device__ __align__(256) uint16_t g_noalloc_scratch[2u * CR_NOALLOC_SCRATCH_ELEMS];
 
 namespace {
 std::mutex g_noalloc_mu;
@@ -50,19 +50,18 @@ extern "C" cr_status cr_segment_project_noalloc(const cr_target_dims* target, in
                                                 const float* sigma_stale, uint16_t* y,
                                                 void* stream) {
     using namespace cr;
-    if (!target) return CR_ERR_INVALID_ARG;
-    if (target->n_layers < 1 || target->n_kv_heads < 1) return CR_ERR_INVALID_ARG;
-    if (target->head_dim != 64 && target->head_dim != 128) return CR_ERR_UNSUPPORTED;
+    cr_status err = check_target(target);
+    if (err != CR_OK) return err;
     if (d_seg != 8 && d_seg != 16) return CR_ERR_UNSUPPORTED;
     if (n_tokens < 1 || n_tokens > INT32_MAX / 2) return CR_ERR_INVALID_ARG;
     if (!kv || !w_seg || !b_seg || !sigma_stale || !y) return CR_ERR_INVALID_ARG;
     if (!aligned16(kv) || !aligned16(w_seg) || !aligned16(b_seg) || !aligned16(sigma_stale) ||
         !aligned16(y))
         return CR_ERR_INVALID_ARG;
+    // S is bounded before the product so that the size check cannot wrap
     const int64_t S = 2ll * target->n_layers * target->n_kv_heads;
-    const int64_t elems = S * d_seg * target->head_dim;
-    if (elems > static_cast<int64_t>(CR_NOALLOC_SCRATCH_ELEMS)) return CR_ERR_UNSUPPORTED;
-    cr_status err = CR_OK;
+    const int64_t per_seg = static_cast<int64_t>(d_seg) * target->head_dim;
+    if (S > static_cast<int64_t>(CR_NOALLOC_SCRATCH_ELEMS) / per_seg) return CR_ERR_UNSUPPORTED;
     uint16_t* scratch = scratch_for_current_device(&err);
     if (!scratch) return err;
     unsigned* status = device_status_ptr();
@@ -79,6 +78,7 @@ extern "C" cr_status cr_segment_project_noalloc(const cr_target_dims* target, in
     sp.d_seg = d_seg;
     sp.b_seg = b_seg;
     sp.y = y;
+    sp.ldy = S * d_seg;
     sp.status = status;
     return launch_segproj(kv, S * target->head_dim, scratch, target->head_dim, sp, st);
 }

@@ -444,6 +444,14 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// Two-term bf16 split of a pair: hi = rn(a), lo = rn(a - hi) (and so for b);
+// hi + lo carries a to about 16 significant bits.
+__device__ __forceinline__ void split_bf16x2(float a, float b, uint32_t* hi, uint32_t* lo) {
+    const uint32_t h = pack_bf16x2(a, b);
+    *hi = h;
+    *lo = pack_bf16x2(a - __uint_as_float(h << 16), b - __uint_as_float(h & 0xFFFF0000u));
+}
+
 // cos/sin of (p * f) with the product's rounding error folded back in:
 // a = fl(p*f), e = p*f - a exactly (FMA), then rotate (cos a, sin a) by e.
 __device__ __forceinline__ void sincos_prod(float p, float f, float* s, float* c) {

@@ -6,12 +6,17 @@
 //
 // Work item: 128 tokens x G = 16 consecutive segments.  Warp 0 streams, per
 // segment, the [128 x d_h] cache slice (TMA, 128B swizzle) and the segment's
-// [16 x d_h] weight rows (1/sigma already folded in) through a ring of
-// shared-memory stages; warp 1 issues one M=128, N=16 MMA chain per segment
-// into its own 16 TMEM columns (two 256-column buffers); warps 2..5 add the
-// bias and store d_seg bf16 values per segment.  For d_seg = 8 the weight box
-// still spans 16 rows (the next segment's rows, or TMA zero fill past the
-// end); those 8 extra output columns are computed and discarded.
+// [16 x d_h] weight rows through a ring of shared-memory stages.  The weights
+// W_seg / sigma_stale come as two bf16 terms (hi + lo, folded once per call),
+// so the folded weight carries about 16 significant bits, not 8; warp 1
+// issues, per segment, one M=128, N=16 MMA chain over both terms into the
+// segment's own 16 TMEM columns (two 256-column buffers).  The MMAs are idle
+// most of the time either way: the doubled chain costs no time.  Warps 2..5
+// add the bias and store d_seg values per segment, as bf16 (y) and, when
+// asked, as the bf16 remainder y - bf16(y) too (y_lo), so that the next
+// linear can take y to about 16 bits.  For d_seg = 8 the weight box still
+// spans 16 rows (the next segment's rows, or TMA zero fill past the end);
+// those 8 extra output columns are computed and discarded.
 //
 // Pool variant (kPool): the same projection reads its cache tiles straight
 // from the chunk pool, each 128-row tile inside one selected chunk, and warp 6
@@ -35,14 +40,15 @@ template <int DH>
 struct SegCfg {
     static constexpr int kBoxes = DH / 64;                 // 64-column swizzle boxes per slice
     static constexpr uint32_t kABytes = 128 * DH * 2;
-    static constexpr uint32_t kBBytes = SP_N * DH * 2;
-    static constexpr uint32_t kStageBytes = kABytes + kBBytes;
+    static constexpr uint32_t kBBytes = SP_N * DH * 2;         // one weight term
+    static constexpr uint32_t kStageBytes = kABytes + 2 * kBBytes;
     static constexpr int kStages = (DH == 128) ? 5 : 8;
     static constexpr uint32_t kSmemBytes = 1024 + kStages * kStageBytes + 256;
 };
 
-// W_seg / sigma_stale per input coordinate, rounded to bf16; eight weights
-// (16 bytes) per thread.  n and d_h are multiples of 8.
+// W_seg / sigma_stale per input coordinate as two bf16 terms: out[i] = hi =
+// rn(w / sigma), out[n + i] = lo = rn(w / sigma - hi); eight weights (16 bytes)
+// per thread.  n and d_h are multiples of 8.
 __global__ void fold_sigma_kernel(const uint16_t* __restrict__ w, const float* __restrict__ sigma,
                                   int64_t n, int d_seg, int dh, uint16_t* __restrict__ out) {
     pdl_launch_dependents();
@@ -58,14 +64,15 @@ __global__ void fold_sigma_kernel(const uint16_t* __restrict__ w, const float* _
         const float4 s0 = __ldg(sp), s1 = __ldg(sp + 1);
         const uint32_t in[4] = {wv.x, wv.y, wv.z, wv.w};
         const float sg[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
-        uint32_t o[4];
+        uint32_t oh[4], ol[4];
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-            const float lo = __uint_as_float(in[k] << 16) / sg[2 * k];
-            const float hi = __uint_as_float(in[k] & 0xFFFF0000u) / sg[2 * k + 1];
-            o[k] = pack_bf16x2(lo, hi);
+            const float a = __uint_as_float(in[k] << 16) / sg[2 * k];
+            const float b = __uint_as_float(in[k] & 0xFFFF0000u) / sg[2 * k + 1];
+            split_bf16x2(a, b, &oh[k], &ol[k]);
         }
-        reinterpret_cast<uint4*>(out)[i8] = make_uint4(o[0], o[1], o[2], o[3]);
+        reinterpret_cast<uint4*>(out)[i8] = make_uint4(oh[0], oh[1], oh[2], oh[3]);
+        reinterpret_cast<uint4*>(out + n)[i8] = make_uint4(ol[0], ol[1], ol[2], ol[3]);
     }
 }
 
@@ -164,8 +171,11 @@ __global__ void __launch_bounds__(224, 1)
 #pragma unroll
                     for (int b = 0; b < Cfg::kBoxes; ++b) {
                         tma_load_2d(sa + b * 16384, &tmKV, &full[stage], seg * DH + b * 64, src0);
+                        // hi term rows [0, S d_seg), lo term rows [S d_seg, 2 S d_seg)
                         tma_load_2d(sb + b * (SP_N * 128), &tmW, &full[stage], b * 64,
                                     seg * p.d_seg);
+                        tma_load_2d(sb + Cfg::kBBytes + b * (SP_N * 128), &tmW, &full[stage], b * 64,
+                                    (p.S + seg) * p.d_seg);
                     }
                 }
                 __syncwarp();
@@ -201,10 +211,12 @@ __global__ void __launch_bounds__(224, 1)
 #pragma unroll
                     for (int b = 0; b < Cfg::kBoxes; ++b) {
 #pragma unroll
-                        for (int k = 0; k < 4; ++k)
-                            mma_bf16_ss(d, da + b * (16384 >> 4) + 2 * k,
-                                        db + b * ((SP_N * 128) >> 4) + 2 * k, IDESC,
-                                        (b | k) != 0 ? 1u : 0u);
+                        for (int k = 0; k < 4; ++k) {
+                            const uint64_t a = da + b * (16384 >> 4) + 2 * k;
+                            const uint64_t w = db + b * ((SP_N * 128) >> 4) + 2 * k;
+                            mma_bf16_ss(d, a, w, IDESC, (b | k) != 0 ? 1u : 0u);
+                            mma_bf16_ss(d, a, w + (Cfg::kBBytes >> 4), IDESC, 1u);
+                        }
                     }
                     mma_commit(&empty[stage]);
                 }
@@ -306,7 +318,7 @@ __global__ void __launch_bounds__(224, 1)
     } else {
         const uint32_t quad = warp & 3u;
         const int r = static_cast<int>(quad * 32 + lane);
-        const int ldy = p.S * p.d_seg;
+        const int64_t ldy = p.ldy;
         uint32_t acc = 0, acc_phase = 0;
         for (int t = blockIdx.x; t < total; t += gridDim.x) {
             const TileRows tr = tile_rows(tiles, p, t % p.num_m);
@@ -318,6 +330,7 @@ __global__ void __launch_bounds__(224, 1)
             const int row = tr.dst + r;
             const uint32_t taddr = tmem_base + ((quad * 32u) << 16) + acc * 256;
             uint16_t* yrow = p.y + static_cast<int64_t>(row) * ldy;
+            uint16_t* ylrow = p.y_lo ? p.y_lo + static_cast<int64_t>(row) * ldy : nullptr;
             for (int g = 0; g < ns; ++g) {
                 float v[16];
                 __syncwarp();
@@ -326,15 +339,20 @@ __global__ void __launch_bounds__(224, 1)
                 const int seg = s0 + g;
                 const float* bs = p.b_seg + seg * p.d_seg;
                 if (r < tr.rows) {
-                    uint32_t w[8];
+                    uint32_t w[8], wl[8];
                     const int dm = p.d_seg - 1;   // d_seg is 8 or 16; columns >= d_seg are dropped
 #pragma unroll
                     for (int i = 0; i < 8; ++i)
-                        w[i] = pack_bf16x2(v[2 * i] + __ldg(bs + ((2 * i) & dm)),
-                                           v[2 * i + 1] + __ldg(bs + ((2 * i + 1) & dm)));
+                        split_bf16x2(v[2 * i] + __ldg(bs + ((2 * i) & dm)),
+                                     v[2 * i + 1] + __ldg(bs + ((2 * i + 1) & dm)), &w[i], &wl[i]);
                     uint4* dst = reinterpret_cast<uint4*>(yrow + seg * p.d_seg);
                     dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
                     if (p.d_seg == 16) dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
+                    if (ylrow) {
+                        uint4* dl = reinterpret_cast<uint4*>(ylrow + seg * p.d_seg);
+                        dl[0] = make_uint4(wl[0], wl[1], wl[2], wl[3]);
+                        if (p.d_seg == 16) dl[1] = make_uint4(wl[4], wl[5], wl[6], wl[7]);
+                    }
                 }
             }
             tc_fence_before();
@@ -390,7 +408,7 @@ cr_status launch_segproj(const uint16_t* kv, int64_t ld_kv, const uint16_t* wfol
                       CU_TENSOR_MAP_SWIZZLE_128B))
         return CR_ERR_INVALID_ARG;
     if (!make_tmap_2d(&tw, wfold, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, head_dim,
-                      static_cast<uint64_t>(p.S) * p.d_seg, head_dim * 2, 64, SP_N,
+                      2 * static_cast<uint64_t>(p.S) * p.d_seg, head_dim * 2, 64, SP_N,
                       CU_TENSOR_MAP_SWIZZLE_128B))
         return CR_ERR_INVALID_ARG;
     const NoTiles none{};
@@ -414,7 +432,7 @@ cr_status launch_segproj_pool(const uint16_t* kv_pool, int64_t n_pool_tokens, ui
                       128, CU_TENSOR_MAP_SWIZZLE_128B))
         return CR_ERR_INVALID_ARG;
     if (!make_tmap_2d(&tw, wfold, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, head_dim,
-                      static_cast<uint64_t>(p.S) * p.d_seg, head_dim * 2, 64, SP_N,
+                      2 * static_cast<uint64_t>(p.S) * p.d_seg, head_dim * 2, 64, SP_N,
                       CU_TENSOR_MAP_SWIZZLE_128B))
         return CR_ERR_INVALID_ARG;
     if (!make_tmap_2d(&to, kv_out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dkv, p.M, dkv * 2, 64, 128,

@@ -43,7 +43,7 @@ class RepairSession:
         self.pos = z(n, dtype=torch.int32)
         self.cu_seqlens = z(257, dtype=torch.int32)
         self.h0 = z(n, rep.d_b, dtype=torch.float32)
-        self.rein = z(n, max(rep.n_blocks, 1) * rep.d_b, dtype=torch.bfloat16)
+        self.rein = z(n, max(rep.n_blocks, 1) * rep.d_b, dtype=torch.float32)
         self.yf = z(n, rep.d_b, dtype=torch.bfloat16)
         ws = cr.cr_workspace_bytes(target, rep, n)
         if ws == 0:

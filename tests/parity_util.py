@@ -70,25 +70,46 @@ def half_ulp(x: np.ndarray, cache_dtype: str) -> np.ndarray:
 
 
 def check_repaired_cache(got: np.ndarray, exact: np.ndarray, target, cache_dtype: str,
-                         max_tol=2e-2, cos_tol=0.999):
-    """The repaired-cache tolerance per (layer, K|V) group; returns the worst figures."""
+                         max_tol=2e-2, cos_tol=0.999, stale=None, resid_cos_tol=0.999):
+    """The repaired-cache tolerance per (layer, K|V) group.
+
+    Every group is measured before any assertion, so a failure reports the whole
+    table.  With `stale` given (the un-repaired cache, canonical K), the residual
+    alone (repaired - stale) is compared as well: its cosine per group must reach
+    resid_cos_tol, which catches a wrong but small correction that the cache
+    tolerance cannot see.  Returns (worst max err / RMS, worst cosine, worst
+    residual cosine or None, rows), rows = (layer, 'K'|'V', err, cos, resid_cos).
+    """
     g = as_f64(got) if cache_dtype == "bf16" else got.astype(np.float64)
     n = g.shape[0]
     L, H, dh = target.n_layers, target.n_kv_heads, target.head_dim
     g5 = g.reshape(n, L, 2, H * dh)
     e5 = exact.reshape(n, L, 2, H * dh)
     hu5 = half_ulp(exact, cache_dtype).reshape(n, L, 2, H * dh)
-    worst_max, worst_cos = 0.0, 1.0
+    s5 = None
+    if stale is not None:
+        s5 = (as_f64(stale) if cache_dtype == "bf16" else stale.astype(np.float64)).reshape(n, L, 2, H * dh)
+    rows = []
     for l in range(L):
         for kv in range(2):
             gg, ee, hu = g5[:, l, kv], e5[:, l, kv], hu5[:, l, kv]
             rms = np.sqrt(np.mean(ee ** 2))
-            err = np.maximum(np.abs(gg - ee) - hu, 0.0).max() / rms
+            err = float(np.maximum(np.abs(gg - ee) - hu, 0.0).max() / rms)
             cos = float((gg * ee).sum() / np.sqrt((gg ** 2).sum() * (ee ** 2).sum()))
-            worst_max, worst_cos = max(worst_max, err), min(worst_cos, cos)
-            assert err <= max_tol, f"layer {l} {'KV'[kv]}: max err {err:.3e} x RMS > {max_tol}"
-            assert cos >= cos_tol, f"layer {l} {'KV'[kv]}: cosine {cos:.6f} < {cos_tol}"
-    return worst_max, worst_cos
+            rc = None
+            if s5 is not None:
+                dg, de = gg - s5[:, l, kv], ee - s5[:, l, kv]
+                rc = float((dg * de).sum() / np.sqrt((dg ** 2).sum() * (de ** 2).sum()))
+            rows.append((l, "KV"[kv], err, cos, rc))
+    worst_max = max(r[2] for r in rows)
+    worst_cos = min(r[3] for r in rows)
+    worst_rc = min(r[4] for r in rows) if s5 is not None else None
+    for l, kv, err, cos, rc in rows:
+        assert err <= max_tol, f"layer {l} {kv}: max err {err:.3e} x RMS > {max_tol} (worst {worst_max:.3e})"
+        assert cos >= cos_tol, f"layer {l} {kv}: cosine {cos:.6f} < {cos_tol}"
+        assert rc is None or rc >= resid_cos_tol, \
+            f"layer {l} {kv}: residual cosine {rc:.6f} < {resid_cos_tol} (worst {worst_rc:.6f})"
+    return worst_max, worst_cos, worst_rc, rows
 
 
 def residual_cosine(got: np.ndarray, stale: np.ndarray, exact: np.ndarray, cache_dtype: str) -> float:

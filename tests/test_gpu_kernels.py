@@ -89,7 +89,7 @@ def test_layernorm_with_reinjection_add(D):
     g = np.random.default_rng(D)
     M = 301
     x = (g.standard_normal((M, D)) * 3 + 0.5).astype(np.float32)
-    add = _bf16(g, (M, 2 * D))          # strided slice of a wider matrix, like P_b(s)
+    add = g.standard_normal((M, 2 * D)).astype(np.float32)   # strided slice, like P_b(s)
     gam = (1 + 0.2 * g.standard_normal(D)).astype(np.float32)
     bet = (0.1 * g.standard_normal(D)).astype(np.float32)
     xd = to_dev(x)
@@ -107,19 +107,12 @@ def _chunk_ids(lens):
     return np.concatenate([np.full(n, i, np.int32) for i, n in enumerate(lens)])
 
 
-@pytest.mark.parametrize("hd", [32, 64])
-@pytest.mark.parametrize("reqs", [
-    [[64, 64]],                      # two chunks, one tile
-    [[300]],                          # single chunk: bidirectional, ragged tail
-    [[1] * 150],                      # unit chunks: token-causal
-    [[130, 77, 200, 1, 95]],          # ragged chunk map across several tiles
-    [[129, 40], [5], [300, 256, 3]],  # several requests (varlen)
-])
-def test_chunk_causal_attention(hd, reqs):
-    g = np.random.default_rng(hd + sum(map(sum, reqs)))
-    nh = 4 if hd == 32 else 8
+def _attention_check(reqs, hd, nh, seed, what):
+    """cr_chunk_causal_attention on random bf16 Q, K, V for requests of the given
+    chunk lengths, every output against the oracle's block-causal attention."""
+    g = np.random.default_rng(seed)
     db = nh * hd
-    lens = [sum(r) for r in reqs]
+    lens = [int(sum(r)) for r in reqs]
     N = sum(lens)
     qkv = _bf16(g, (N, 3 * db))
     cend = []
@@ -148,8 +141,34 @@ def test_chunk_causal_attention(hd, reqs):
     # the output is rounded once to bf16: |err| <= 2^-9 mag + 2^-9 |o|; 2x margin.
     bound = 2.0 ** -8 * mag + 2.0 ** -8 * np.abs(want) + 1e-5
     worst = float((np.abs(g - want) / bound).max())
-    assert worst <= 1.0, f"attention hd={hd} {reqs}: error / bound = {worst:.3f}"
-    assert_close(got, want, 8e-3, 1.0, f"attention hd={hd} {reqs}")
+    print(f"attention {what}: N {N}, error / bound = {worst:.3f}")
+    assert worst <= 1.0, f"attention {what}: error / bound = {worst:.3f}"
+    assert_close(got, want, 8e-3, 1.0, f"attention {what}")
+
+
+@pytest.mark.parametrize("hd", [32, 64])
+@pytest.mark.parametrize("reqs", [
+    [[64, 64]],                      # two chunks, one tile
+    [[300]],                          # single chunk: bidirectional, ragged tail
+    [[1] * 150],                      # unit chunks: token-causal
+    [[130, 77, 200, 1, 95]],          # ragged chunk map across several tiles
+    [[129, 40], [5], [300, 256, 3]],  # several requests (varlen)
+])
+def test_chunk_causal_attention(hd, reqs):
+    _attention_check(reqs, hd, 4 if hd == 32 else 8, hd + sum(map(sum, reqs)), f"hd={hd} {reqs}")
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("name", ["llama8b", "qwen7b"])
+def test_chunk_causal_attention_full_size(name):
+    """A whole request of a workload, every row checked: the 8B shape's 5120 tokens
+    in ten 512-token chunks (20 query-tile pairs per head, many passes around the
+    kernel's K/V ring) and the 7B shape's ragged 20-chunk map (chunk ends inside
+    tiles), both with the workloads' 16 heads of 64."""
+    c = F.make_case(name)
+    p = c.plan
+    lens = [int(x) for x in p.chunk_len[p.chunk_idx[p.cu_chunks[0]:p.cu_chunks[1]]]]
+    _attention_check([lens], c.repairer.head_dim, c.repairer.n_heads, 17, name)
 
 
 @pytest.mark.parametrize("db,nh", [(128, 4), (512, 8), (1024, 16)])
@@ -184,7 +203,7 @@ def test_segment_projection(name):
     from paper_2609_35139_gb300 import dims_from
     td, _ = dims_from(t, r)
     y = torch.empty(rows, t.n_segments * r.d_seg, dtype=torch.bfloat16, device="cuda")
-    ws = torch.empty(t.n_segments * r.d_seg * t.head_dim * 2, dtype=torch.uint8, device="cuda")
+    ws = torch.empty(t.n_segments * r.d_seg * t.head_dim * 4, dtype=torch.uint8, device="cuda")
     cr.cr_segment_project(td, r.d_seg, to_dev(kv), to_dev(w["w_seg"]), to_dev(w["b_seg"]),
                           to_dev(w["sigma_stale"]), y, ws)
     torch.cuda.synchronize()

@@ -106,7 +106,7 @@ def test_forward_parity_masked(name, mode):
     check_assembly(g, a)
     for r in range(len(a["cu_seqlens"]) - 1):
         res = oracle_request(case, a, r, mask_mode=mode)
-        print(name, mode, r, check_request(case, g, a, r, res))
+        print(name, mode, r, check_request(case, g, a, r, res, tag=f"{name} mask={mode}"))
 
 
 def test_block_diagonal_chunks_independent_on_gpu():
@@ -137,4 +137,4 @@ def test_forward_parity_masked_full_size(mode):
     a = oracle_assemble(case)
     rows = _sample_rows(a["chunk_id"], 96)
     res = oracle_request(case, a, 0, rows=rows, mask_mode=mode)
-    print(mode, check_request(case, g, a, 0, res, rows=rows))
+    print(mode, check_request(case, g, a, 0, res, rows=rows, tag=f"{case.recipe.name} mask={mode}"))

@@ -1,16 +1,19 @@
 """cr_apply_residual_paged: the repaired rows written into a paged, layer-major
-target cache equal, bit for bit, the rows cr_apply_residual repairs in place
-(whose values the parity tests pin to the oracle); tokens with a negative slot
-and unused slots are left alone, the stale cache is not modified, and a slot out
-of range is reported on the device and not written (the report makes the
-kernel's other roles stop, as for any device-detected index error)."""
+target cache match the oracle's repaired cache placed by the oracle's paged
+scatter (App. A serving setup: loaded through the last complete 16-token block)
+within the repaired-cache tolerance, and equal, bit for bit, the rows
+cr_apply_residual repairs in place; tokens with a negative slot and unused slots
+are left alone, the stale cache is not modified, and a slot out of range is
+reported on the device and not written (the report makes the kernel's other
+roles stop, as for any device-detected index error)."""
 import numpy as np
 import pytest
 import torch
 
 import fixtures as F
+import oracle as O
 from paper_2609_35139_gb300 import RepairSession, cr, dims_from, pack_host_weights
-from parity_util import to_dev, to_host
+from parity_util import as_f64, half_ulp, to_dev, to_host
 
 pytestmark = pytest.mark.gpu
 
@@ -97,3 +100,48 @@ def test_paged_slot_out_of_range_is_reported_and_skipped():
     assert st == cr.CR_ERR_DEVICE_INDEX, word
     got = to_host(paged)
     assert np.all(got[:, 3] == SENTINEL)            # slot 3 belonged to the bad token only
+
+
+@pytest.mark.parametrize("rope_mode", [cr.CR_ROPE_NONE, cr.CR_ROPE_GLOBAL])
+def test_paged_write_matches_oracle(rope_mode):
+    case, sess, a = _prepared()
+    n = a.n_tokens
+    tg = case.target
+    L, H, dh = tg.n_layers, tg.n_kv_heads, tg.head_dim
+    plane, planes = H * dh, 2 * L
+    rope = rope_mode == cr.CR_ROPE_GLOBAL
+    inv = case.inv_freq_target if rope else None
+    # the request's blocks in a shuffled physical order among spare blocks
+    n_phys = n // 16 + 9
+    table = np.random.default_rng(11).permutation(n_phys)[: (n + 15) // 16]
+    slots = O.paged_slot_mapping(n, table)
+    num_slots = n_phys * 16
+    paged = torch.empty((planes, num_slots, plane), dtype=torch.int16, device="cuda")
+    paged.fill_(SENTINEL)
+    sess.apply_paged(a, to_dev(slots), paged.view(torch.bfloat16), num_slots, inv, rope_mode)
+    torch.cuda.synchronize()
+    got = to_host(paged.view(torch.bfloat16)).reshape(planes, num_slots, plane)
+
+    kvp, embp = case.pool()
+    p = case.plan
+    asm = O.assemble_stale(kvp, embp, p.chunk_start, p.chunk_len, p.chunk_idx, p.cu_chunks)
+    res = O.repair_request(asm["kv"], asm["emb"], asm["chunk_id"], asm["pos"], case.weights,
+                           cache_dtype="bf16", n_layers=L, n_kv_heads=H, head_dim=dh,
+                           n_heads=case.repairer.n_heads,
+                           inv_freq_target=case.inv_freq_target if rope else None)
+    exact = res.repaired_rot if rope else res.repaired
+    want = O.paged_scatter(exact, slots, np.full((planes, num_slots, plane), np.nan), L, H, dh)
+    written = ~np.isnan(want[:, :, 0])
+    assert int(written[0].sum()) == (n // 16) * 16
+    g64 = as_f64(got)
+    worst = 0.0
+    for pl in range(planes):
+        w = written[pl]
+        assert np.all(got[pl, ~w] == SENTINEL), f"plane {pl}: a slot outside the mapping was written"
+        e, gg = want[pl, w], g64[pl, w]
+        rms = np.sqrt(np.mean(e ** 2))
+        err = float(np.maximum(np.abs(gg - e) - half_ulp(e, "bf16"), 0.0).max() / rms)
+        cos = float((gg * e).sum() / np.sqrt((gg ** 2).sum() * (e ** 2).sum()))
+        worst = max(worst, err)
+        assert err <= 2e-2 and cos >= 0.999, f"plane {pl}: max err {err:.3e} x RMS, cosine {cos:.6f}"
+    print(f"paged write vs oracle (rope={rope}): worst max err {worst:.3e} x RMS")

@@ -6,6 +6,8 @@ every output; the full-size ones on every intermediate and on a sample of
 repaired rows (all D_KV coordinates of each sampled token) that the oracle's
 head computes one by one.
 """
+import json
+
 import numpy as np
 import pytest
 import torch
@@ -103,27 +105,58 @@ def check_assembly(g: GpuRun, a):
     assert np.array_equal(g.cu_dev, a["cu_seqlens"])
 
 
-def check_request(case, g: GpuRun, a, r, res, rows=None, rope=False):
+# Gates of the intermediate activations (relative RMS error, max error / RMS):
+# the largest figures measured over every workload and test shape on a GB300,
+# times about three; the repaired cache's own tolerance is the stated one
+# (parity_util).  h^0 and the P_b(s) come from the two-term encoder (no bf16
+# rounding of its features: measured at most 2.9e-5 / 1.7e-4 on bf16 caches).
+# An fp32 cache enters the tensor cores rounded once to bf16, which bounds h^0
+# and the P_b(s) there (measured 1.6e-3 / 8.4e-3).  y_f carries the bf16
+# operands of the blocks' linears and attention (measured 2.5e-3 / 1.7e-2).
+GATE_H0 = {"bf16": (1e-4, 5e-4), "f32": (5e-3, 2.5e-2)}
+GATE_REIN = GATE_H0
+GATE_YF = (6e-3, 4e-2)
+
+
+def check_request(case, g: GpuRun, a, r, res, rows=None, rope=False, tag=None):
+    """Every intermediate and the repaired cache of request r against the oracle.
+    All figures are measured and printed (one PARITY line, the per-(layer, K|V)
+    table included) before any gate is asserted."""
     t = case.target
     lo, hi = a["cu_seqlens"][r], a["cu_seqlens"][r + 1]
-    report = {}
-    report["h0"] = assert_close(g.h0[lo:hi], res.h0, 1e-2, 6e-2, "h0 (compress)")
     B = case.repairer.n_blocks
     db = case.repairer.d_b
+    inter = {"h0": (rel_errors(g.h0[lo:hi], res.h0), GATE_H0[t.cache_dtype])}
     for b in range(B):
-        report[f"rein{b}"] = assert_close(g.rein[lo:hi, b * db:(b + 1) * db], res.rein[b], 1e-2,
-                                          6e-2, f"P_{b}(s)")
-    report["yf"] = assert_close(g.yf[lo:hi], res.yf, 2.5e-2, 0.2, "y_f (forward)")
+        inter[f"rein{b}"] = (rel_errors(g.rein[lo:hi, b * db:(b + 1) * db], res.rein[b]),
+                             GATE_REIN[t.cache_dtype])
+    inter["yf"] = (rel_errors(g.yf[lo:hi], res.yf), GATE_YF)
     sel = np.arange(hi - lo) if rows is None else rows
     got = g.kv[lo:hi][sel]
     exact = res.repaired if rows is not None else (res.repaired_rot if rope else res.repaired)
     if rope and rows is None:
         exact = res.repaired_rot
-    report["cache"] = check_repaired_cache(got, exact, t, t.cache_dtype)
-    if not rope:
-        report["resid_cos"] = residual_cosine(got, g.kv_stale[lo:hi][sel], exact, t.cache_dtype)
-        assert report["resid_cos"] >= 0.99, report
-    return report
+    stale = None if rope else g.kv_stale[lo:hi][sel]
+    cache_err = None
+    try:
+        worst = check_repaired_cache(got, exact, t, t.cache_dtype, stale=stale)
+    except AssertionError as e:
+        cache_err = e
+        worst = check_repaired_cache(got, exact, t, t.cache_dtype, stale=stale, max_tol=np.inf,
+                                     cos_tol=-1.0, resid_cos_tol=-1.0)
+    worst_max, worst_cos, worst_rc, table = worst
+    rein = [v[0] for k, v in inter.items() if k.startswith("rein")]
+    # one line per request: the per-(layer, K|V) parity table
+    print("PARITY " + json.dumps({
+        "case": tag or case.recipe.name, "request": int(r), "rope": bool(rope), "rows": int(len(sel)),
+        "h0": inter["h0"][0], "yf": inter["yf"][0],
+        "rein_worst": [max(x[0] for x in rein), max(x[1] for x in rein)] if rein else None,
+        "cache_worst": [worst_max, worst_cos, worst_rc], "groups": table}))
+    for name, ((rr, mm), (gr, gm)) in inter.items():
+        assert rr <= gr and mm <= gm, f"{name}: rel-RMS {rr:.3e} (<= {gr}), max/RMS {mm:.3e} (<= {gm})"
+    if cache_err is not None:
+        raise cache_err
+    return {"cache": (worst_max, worst_cos, worst_rc), **{k: v[0] for k, v in inter.items()}}
 
 
 # ------------------------------------------------------------------ small workloads, every output
@@ -294,4 +327,4 @@ def test_parity_batched_sampled_requests():
         g = type("G", (), {})()
         g.h0, g.rein = to_host(sess.h0[lo:hi]), to_host(sess.rein[lo:hi])
         g.yf, g.kv, g.kv_stale = to_host(sess.yf[lo:hi]), to_host(sess.kv[lo:hi]), stale_rows[r][0]
-        print("batched", r, check_request(case, g, asm_r, 0, res, rows=rows))
+        print("batched", r, check_request(case, g, asm_r, 0, res, rows=rows, tag=f"batched request {r}"))

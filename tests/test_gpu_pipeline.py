@@ -1,13 +1,15 @@
 """RepairPipeline (host transfers overlapped with repair on two slots) returns
 exactly what a plain RepairSession returns for each request, through several
-reuses of each slot."""
+reuses of each slot, and each request's repaired cache, read back into host
+memory, matches the oracle's within the repaired-cache tolerance."""
 import numpy as np
 import pytest
 import torch
 
 import fixtures as F
+import oracle as O
 from paper_2609_35139_gb300 import RepairPipeline, RepairSession, cr, dims_from, pack_host_weights
-from parity_util import to_dev, to_host
+from parity_util import check_repaired_cache, to_dev, to_host
 
 pytestmark = pytest.mark.gpu
 
@@ -66,6 +68,18 @@ def test_pipeline_matches_session_per_request():
         got = outs[k][:lens[i]].view(torch.int16).numpy().view(np.uint16) \
             if kv_h.dtype == torch.bfloat16 else outs[k][:lens[i]].numpy()
         assert np.array_equal(got.view(np.uint8), ref[i].view(np.uint8)), f"request {i} (submission {k})"
+    # every request's host copy against the oracle (first submission of each)
+    tg = case.target
+    for i, sel in enumerate(reqs):
+        k = order.index(i)
+        got = outs[k][:lens[i]].view(torch.int16).numpy().view(np.uint16)
+        kv_r = np.concatenate([kvp[p.chunk_start[c]:p.chunk_start[c] + p.chunk_len[c]] for c in sel])
+        emb_r = np.concatenate([embp[p.chunk_start[c]:p.chunk_start[c] + p.chunk_len[c]] for c in sel])
+        cid = np.concatenate([np.full(p.chunk_len[c], j, np.int32) for j, c in enumerate(sel)])
+        res = O.repair_request(kv_r, emb_r, cid, np.arange(lens[i], dtype=np.int32), case.weights,
+                               cache_dtype="bf16", n_layers=tg.n_layers, n_kv_heads=tg.n_kv_heads,
+                               head_dim=tg.head_dim, n_heads=case.repairer.n_heads)
+        check_repaired_cache(got, res.repaired, tg, "bf16", stale=kv_r)
 
 
 def test_pipeline_rejects_oversize_request():

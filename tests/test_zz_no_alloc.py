@@ -29,7 +29,7 @@ def test_noalloc_segment_projection_matches_workspace_version():
         args = (to_dev(kv), to_dev(w["w_seg"]), to_dev(w["b_seg"]), to_dev(w["sigma_stale"]))
         width = t.n_segments * r.d_seg
         y_ws = torch.empty(600, width, dtype=torch.bfloat16, device="cuda")
-        ws = torch.empty(t.n_segments * r.d_seg * t.head_dim * 2, dtype=torch.uint8, device="cuda")
+        ws = torch.empty(t.n_segments * r.d_seg * t.head_dim * 4, dtype=torch.uint8, device="cuda")
         cr.cr_segment_project(td, r.d_seg, *args, y_ws, ws)
         y_na = torch.full((600, width), float("nan"), dtype=torch.bfloat16, device="cuda")
         cr.cr_segment_project_noalloc(td, r.d_seg, *args, y_na)
@@ -41,11 +41,22 @@ def test_noalloc_segment_projection_matches_workspace_version():
 
 
 def test_noalloc_rejects_oversized_shapes():
-    """Shapes whose folded weights exceed the fixed 4 MiB scratch are refused on the host."""
+    """Shapes whose weights exceed the fixed scratch (2 Mi weights, two bf16 terms each:
+    8 MiB) are refused on the host, including L * H_kv so large that S * d_seg * d_h
+    would not fit in 64 bits; target dimensions are checked as cr_segment_project
+    checks them."""
     build.build()
-    t = cr.target_dims(80, 16, 128, 8192, "bf16")    # S * 16 * 128 * 2 B = 10 MiB
     FAKE = 0x10000
     L = cr.lib()
     import ctypes
-    assert L.cr_segment_project_noalloc(ctypes.byref(t), 16, FAKE, 10, FAKE, FAKE, FAKE, FAKE,
-                                        None) == cr.CR_ERR_UNSUPPORTED
+
+    def call(t, d_seg=16):
+        return L.cr_segment_project_noalloc(ctypes.byref(t), d_seg, FAKE, 10, FAKE, FAKE, FAKE, FAKE,
+                                            None)
+
+    assert call(cr.target_dims(80, 16, 128, 8192, "bf16")) == cr.CR_ERR_UNSUPPORTED   # 5 Mi weights
+    assert call(cr.target_dims(2 ** 30, 2 ** 30, 128, 8192, "bf16")) == cr.CR_ERR_UNSUPPORTED
+    assert call(cr.target_dims(4, 2, 128, 0, "bf16")) == cr.CR_ERR_INVALID_ARG       # d_model
+    assert call(cr.target_dims(4, 2, 128, 4096, 7)) == cr.CR_ERR_INVALID_ARG         # cache dtype
+    assert call(cr.target_dims(4, 2, 96, 4096, "bf16")) == cr.CR_ERR_UNSUPPORTED     # head dim
+    assert call(cr.target_dims(4, 2, 128, 4096, "bf16"), d_seg=12) == cr.CR_ERR_UNSUPPORTED
