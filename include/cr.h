@@ -272,11 +272,20 @@ cr_status cr_repair_forward_masked(const cr_target_dims* target, const cr_repair
  * yf [N, d_b] bf16; kv_inout [N, D_KV] cache dtype; pos [N] device int32;
  * inv_freq_host [head_dim/2] HOST fp32, the target's RoPE frequencies
  * (may be NULL for CR_ROPE_NONE).
+ * workspace: NULL, or at least N * head_dim * 4 bytes (16-byte aligned; the
+ * cr_workspace_bytes workspace of the other calls is always enough), whose
+ * first N * head_dim * 4 bytes are overwritten.  Under CR_ROPE_GLOBAL the call
+ * writes R_M's (cos, sin) for every token and rotation pair there once, and
+ * the head reads each row's angles from it instead of evaluating them for
+ * every K segment of the row; with NULL it evaluates them in the epilogue
+ * (the same formula: results agree to one rounding of the cache dtype; more
+ * time).  Unused for CR_ROPE_NONE.
  */
 cr_status cr_apply_residual(const cr_target_dims* target, const cr_repairer_dims* rep,
                             const cr_weights* w, const uint16_t* yf, int64_t n_tokens,
                             void* kv_inout, const int32_t* pos, const float* inv_freq_host,
-                            int32_t rope_mode, void* stream);
+                            int32_t rope_mode, void* workspace, size_t workspace_bytes,
+                            void* stream);
 
 /*
  * cr_apply_residual_select - cr_apply_residual under an output choice of
@@ -298,7 +307,8 @@ cr_status cr_apply_residual_select(const cr_target_dims* target, const cr_repair
                                    const cr_weights* w, const uint16_t* yf, int64_t n_tokens,
                                    void* kv_inout, const int32_t* pos, const float* inv_freq_host,
                                    int32_t rope_mode, int32_t components, int32_t offset,
-                                   const int32_t* keep_chunk_id, void* stream);
+                                   const int32_t* keep_chunk_id, void* workspace,
+                                   size_t workspace_bytes, void* stream);
 
 /*
  * cr_rotate_k - K_t <- R_M(p_t) K_t on every K segment, V unchanged, in place:
@@ -332,7 +342,7 @@ cr_status cr_rotate_k(const cr_target_dims* target, void* kv_inout, int64_t n_to
  * and not written.  Slots of the tokens written must be distinct.
  * yf [N, d_b] bf16; kv_stale [N, D_KV] bf16, read only; pos [N] device int32;
  * slot_mapping [N] device int64; paged_cache [2 L * num_slots * H_kv * d_h]
- * bf16, device; inv_freq_host as in cr_apply_residual.
+ * bf16, device; inv_freq_host and workspace as in cr_apply_residual.
  * bf16 caches with H_kv * d_h a multiple of 256 only (else CR_ERR_UNSUPPORTED).
  */
 cr_status cr_apply_residual_paged(const cr_target_dims* target, const cr_repairer_dims* rep,
@@ -340,7 +350,7 @@ cr_status cr_apply_residual_paged(const cr_target_dims* target, const cr_repaire
                                   const void* kv_stale, const int32_t* pos,
                                   const float* inv_freq_host, int32_t rope_mode,
                                   const int64_t* slot_mapping, void* paged_cache, int64_t num_slots,
-                                  void* stream);
+                                  void* workspace, size_t workspace_bytes, void* stream);
 
 /* ---------------------------------------------------------------- offline
  * Preparation that runs once per chunk or once per corpus, not per request.
@@ -438,10 +448,12 @@ size_t cr_train_workspace_bytes(const cr_target_dims* target, const cr_repairer_
  * kv_joint tiles and writes dL/dz (bf16) and the rows' squared residuals,
  * never the residual itself; the attention backward is
  * fused (P recomputed tile by tile, no score matrix in memory); the backward's
- * plain matrix products (weight and input gradients) run in cuBLAS (bf16
- * operands, fp32 accumulation), using a part of the workspace as cuBLAS's
- * workspace.  All device buffers 16-byte aligned; P = the last offset of
- * cr_param_layout.
+ * plain matrix products (weight and input gradients) run in the library's
+ * tcgen05 GEMM with operands read in their stored layouts (cr_matmul), bf16
+ * operands and fp32 accumulation; the W_seg gradient is one grouped product
+ * over all segments.  The backward's products need d_c, d_model, mlp_hidden
+ * and S d_seg to be multiples of 64 (else CR_ERR_UNSUPPORTED).  All device
+ * buffers 16-byte aligned; P = the last offset of cr_param_layout.
  */
 cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* rep, float* params,
                         uint16_t* params_bf16, float* adam_m, float* adam_v, float* grads,

@@ -33,6 +33,26 @@ cr_status cr_linear(const uint16_t* A, int64_t lda, const uint16_t* W, const flo
                     void* stream);
 
 /*
+ * cr_matmul - the matrix products of the training step's backward pass
+ * (Sec. 4.2; App. A optimisation): dX = dY W and dW = dY^T X, on the tcgen05
+ * tensor cores with bf16 operands and fp32 accumulation:
+ *   C = op(A) B,  or  C += op(A) B  if accumulate != 0.
+ * B [K, N] bf16, row stride ldb (N contiguous).  op(A) [M, K]: A stored
+ * [M, K] (a_trans = 0) or A stored [K, M] and transposed (a_trans = 1), row
+ * stride lda.  C [M, N] fp32, row stride ldc.  N must be a multiple of 64, and
+ * so must M when a_trans; lda and ldb multiples of 8, ldc of 4; pointers
+ * 16-byte aligned.  workspace: NULL, or fp32 scratch of workspace_bytes (16-byte
+ * aligned) that lets a product whose tiles fill the GPU poorly run as up to 8
+ * k-parts (each written to the scratch, then summed in a fixed order into C:
+ * deterministic, a different rounding order than one k-loop).  Errors:
+ * CR_ERR_INVALID_ARG for non-positive sizes, bad strides or pointers;
+ * CR_ERR_UNSUPPORTED for widths that are not whole 64-column blocks.
+ */
+cr_status cr_matmul(const uint16_t* A, int64_t lda, int32_t a_trans, const uint16_t* B, int64_t ldb,
+                    int64_t M, int64_t N, int64_t K, float* C, int64_t ldc, int32_t accumulate,
+                    void* workspace, size_t workspace_bytes, void* stream);
+
+/*
  * cr_layernorm - u = LN(x + add) * gamma + beta per row (biased variance,
  * eps), fp32 statistics (R4).  x [M, D] fp32 (row stride D).  If `add` is
  * non-NULL ([M, D] fp32, row stride ld_add, a multiple of 4), x + add is also

@@ -29,8 +29,8 @@ CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relax
           "-I" + INCLUDE, "-I" + CSRC]
 SOURCES = ["cr_api.cu", "cr_gemm.cu", "cr_attn.cu", "cr_segproj.cu", "cr_misc.cu",
            "cr_noalloc.cu", "cr_offline.cu", "cr_train.cu", "cr_attn_bwd.cu"]
-# the training step's plain (unfused) backward GEMMs go through cuBLAS
-LIBS = ["-lcublas"]
+# every kernel is this library's own: no vendor math library is linked
+LIBS = []
 
 
 def _nvcc() -> str:

@@ -29,7 +29,7 @@ EXPORTED = [
     "cr_apply_residual_paged", "cr_canonicalize_chunks",
     "cr_sigma_workspace_bytes", "cr_sigma_accumulate", "cr_sigma_finalize", "cr_get_device_status",
     "cr_clear_device_status", "cr_status_str", "cr_last_cuda_error",
-    "cr_linear", "cr_layernorm", "cr_chunk_causal_attention", "cr_masked_attention",
+    "cr_linear", "cr_matmul", "cr_layernorm", "cr_chunk_causal_attention", "cr_masked_attention",
     "cr_chunk_starts", "cr_qkv_rope", "cr_segment_project",
     "cr_segment_project_noalloc", "cr_param_layout", "cr_train_workspace_bytes", "cr_train_step",
     "cr_wait_selftest",
@@ -105,13 +105,13 @@ def lib(build_if_missing: bool = False) -> ctypes.CDLL:
                                            vp, vp, vp, vp, vp, i32, i64, i32, vp, vp, c_size_t,
                                            vp]),
         "cr_apply_residual": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp, i64,
-                                    vp, vp, vp, i32, vp]),
+                                    vp, vp, vp, i32, vp, c_size_t, vp]),
         "cr_apply_residual_paged": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp,
-                                          i64, vp, vp, vp, i32, vp, vp, i64, vp]),
+                                          i64, vp, vp, vp, i32, vp, vp, i64, vp, c_size_t, vp]),
         "cr_canonicalize_chunks": (i32, [P(cr_target_dims), vp, i64, vp, vp, vp]),
         "cr_rotate_k": (i32, [P(cr_target_dims), vp, i64, vp, vp, vp]),
         "cr_apply_residual_select": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp,
-                                           i64, vp, vp, vp, i32, i32, i32, vp, vp]),
+                                           i64, vp, vp, vp, i32, i32, i32, vp, vp, c_size_t, vp]),
         "cr_sigma_workspace_bytes": (ctypes.c_size_t, [P(cr_target_dims), i64]),
         "cr_sigma_accumulate": (i32, [P(cr_target_dims), vp, vp, i64, vp, vp, ctypes.c_size_t, vp]),
         "cr_sigma_finalize": (i32, [P(cr_target_dims), vp, i64, vp, vp]),
@@ -120,6 +120,7 @@ def lib(build_if_missing: bool = False) -> ctypes.CDLL:
         "cr_status_str": (ctypes.c_char_p, [i32]),
         "cr_last_cuda_error": (ctypes.c_char_p, []),
         "cr_linear": (i32, [vp, i64, vp, vp, i64, i64, i64, vp, i64, i32, vp]),
+        "cr_matmul": (i32, [vp, i64, i32, vp, i64, i64, i64, i64, vp, i64, i32, vp, c_size_t, vp]),
         "cr_layernorm": (i32, [vp, vp, i64, vp, vp, vp, c_float, i64, i64, vp, vp]),
         "cr_chunk_causal_attention": (i32, [vp, i32, i32, vp, vp, i32, i64, vp, vp]),
         "cr_param_layout": (i32, [P(cr_target_dims), P(cr_repairer_dims), vp, i32]),
@@ -284,12 +285,17 @@ def cr_repair_forward_masked(target, rep, weights: PackedWeights, h0, rein, chun
     _check("cr_repair_forward_masked", st)
 
 
+def _ws(workspace):
+    return (None, 0) if workspace is None else (_p(workspace), workspace.numel() * workspace.element_size())
+
+
 def cr_apply_residual(target, rep, weights: PackedWeights, yf, n_tokens, kv_inout, pos,
-                      inv_freq_host=None, rope_mode=CR_ROPE_NONE, stream=None):
+                      inv_freq_host=None, rope_mode=CR_ROPE_NONE, workspace=None, stream=None):
     f = None if inv_freq_host is None else _host_arr(inv_freq_host, np.float32)
     st = lib().cr_apply_residual(
         ctypes.byref(target), ctypes.byref(rep), ctypes.byref(weights.struct), _p(yf), n_tokens,
-        _p(kv_inout), _p(pos), None if f is None else f.ctypes.data, rope_mode, _stream(stream))
+        _p(kv_inout), _p(pos), None if f is None else f.ctypes.data, rope_mode, *_ws(workspace),
+        _stream(stream))
     _check("cr_apply_residual", st)
 
 
@@ -301,7 +307,7 @@ OFFSETS = {"stale": CR_OFFSET_STALE, "zero": CR_OFFSET_ZERO}
 
 def cr_apply_residual_select(target, rep, weights: PackedWeights, yf, n_tokens, kv_inout, pos,
                              inv_freq_host=None, rope_mode=CR_ROPE_NONE, component="kv",
-                             offset="stale", keep_chunk_id=None, stream=None):
+                             offset="stale", keep_chunk_id=None, workspace=None, stream=None):
     """Head + residual add under an output choice (K only / V only, zero offset,
     first chunk kept stale when keep_chunk_id is the chunk map)."""
     f = None if inv_freq_host is None else _host_arr(inv_freq_host, np.float32)
@@ -310,7 +316,7 @@ def cr_apply_residual_select(target, rep, weights: PackedWeights, yf, n_tokens, 
     st = lib().cr_apply_residual_select(
         ctypes.byref(target), ctypes.byref(rep), ctypes.byref(weights.struct), _p(yf), n_tokens,
         _p(kv_inout), _p(pos), None if f is None else f.ctypes.data, rope_mode, comp, off,
-        _p(keep_chunk_id), _stream(stream))
+        _p(keep_chunk_id), *_ws(workspace), _stream(stream))
     _check("cr_apply_residual_select", st)
 
 
@@ -323,13 +329,13 @@ def cr_rotate_k(target, kv_inout, n_tokens, pos, inv_freq_host, stream=None):
 
 def cr_apply_residual_paged(target, rep, weights: PackedWeights, yf, n_tokens, kv_stale, pos,
                             slot_mapping, paged_cache, num_slots, inv_freq_host=None,
-                            rope_mode=CR_ROPE_NONE, stream=None):
+                            rope_mode=CR_ROPE_NONE, workspace=None, stream=None):
     """Head + residual add, repaired rows written to paged_cache[(2l+kv)*num_slots + slot]."""
     f = None if inv_freq_host is None else _host_arr(inv_freq_host, np.float32)
     st = lib().cr_apply_residual_paged(
         ctypes.byref(target), ctypes.byref(rep), ctypes.byref(weights.struct), _p(yf), n_tokens,
         _p(kv_stale), _p(pos), None if f is None else f.ctypes.data, rope_mode, _p(slot_mapping),
-        _p(paged_cache), num_slots, _stream(stream))
+        _p(paged_cache), num_slots, *_ws(workspace), _stream(stream))
     _check("cr_apply_residual_paged", st)
 
 
@@ -373,6 +379,16 @@ def cr_linear(A, W, bias, out, epi=CR_EPI_BF16, M=None, N=None, K=None, lda=None
     lda = A.stride(0) if lda is None else lda
     ldo = out.stride(0) if ldo is None else ldo
     _check("cr_linear", lib().cr_linear(_p(A), lda, _p(W), _p(bias), M, N, K, _p(out), ldo, epi,
+                                        _stream(stream)))
+
+
+def cr_matmul(A, B, C, a_trans=False, accumulate=False, workspace=None, stream=None):
+    """C [M, N] fp32 (+)= op(A) B; B [K, N] bf16; op(A) = A [M, K] or, with a_trans, A.T for A [K, M].
+    An optional workspace lets the product run as k-parts summed in a fixed order."""
+    K, N = B.shape
+    M = A.shape[1] if a_trans else A.shape[0]
+    _check("cr_matmul", lib().cr_matmul(_p(A), A.stride(0), int(bool(a_trans)), _p(B), B.stride(0), M, N, K,
+                                        _p(C), C.stride(0), int(bool(accumulate)), *_ws(workspace),
                                         _stream(stream)))
 
 

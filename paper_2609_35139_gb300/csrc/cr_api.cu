@@ -669,16 +669,35 @@ cr_status cr_repair_forward_masked(const cr_target_dims* target, const cr_repair
 cr_status cr_apply_residual(const cr_target_dims* target, const cr_repairer_dims* rep,
                             const cr_weights* w, const uint16_t* yf, int64_t n_tokens,
                             void* kv_inout, const int32_t* pos, const float* inv_freq_host,
-                            int32_t rope_mode, void* stream) {
+                            int32_t rope_mode, void* workspace, size_t workspace_bytes,
+                            void* stream) {
     return cr_apply_residual_select(target, rep, w, yf, n_tokens, kv_inout, pos, inv_freq_host,
-                                    rope_mode, CR_APPLY_KV, CR_OFFSET_STALE, nullptr, stream);
+                                    rope_mode, CR_APPLY_KV, CR_OFFSET_STALE, nullptr, workspace,
+                                    workspace_bytes, stream);
+}
+
+// R_M's (cos, sin) for every token and pair index (angle-major, entry q N + t),
+// written once per call into the caller's workspace, so that the head's
+// epilogue reads each row's angles instead of evaluating them for every K
+// segment.  Without a workspace the epilogue evaluates them itself.
+static cr_status target_rope_table(const Dims& d, const int32_t* pos, int64_t n_tokens,
+                                   const float* inv_freq_host, void* workspace,
+                                   size_t workspace_bytes, GemmParams* gp, cudaStream_t st) {
+    if (!workspace) return CR_OK;
+    const size_t bytes = static_cast<size_t>(n_tokens) * static_cast<size_t>(d.dh / 2) * 8;
+    if (!all_aligned(workspace) || workspace_bytes < bytes) return CR_ERR_INVALID_ARG;
+    float2* table = static_cast<float2*>(workspace);
+    const cr_status s = launch_rope_table(pos, n_tokens, static_cast<int>(d.dh / 2), inv_freq_host, table, st);
+    if (s == CR_OK) gp->rope_table = table;
+    return s;
 }
 
 cr_status cr_apply_residual_select(const cr_target_dims* target, const cr_repairer_dims* rep,
                                    const cr_weights* w, const uint16_t* yf, int64_t n_tokens,
                                    void* kv_inout, const int32_t* pos, const float* inv_freq_host,
                                    int32_t rope_mode, int32_t components, int32_t offset,
-                                   const int32_t* keep_chunk_id, void* stream) {
+                                   const int32_t* keep_chunk_id, void* workspace,
+                                   size_t workspace_bytes, void* stream) {
     cr_status s = check_target(target);
     if (s == CR_OK) s = check_repairer(rep);
     if (s != CR_OK) return s;
@@ -715,6 +734,9 @@ cr_status cr_apply_residual_select(const cr_target_dims* target, const cr_repair
     gp.kv_zero = offset == CR_OFFSET_ZERO ? 1 : 0;
     gp.keep_chunk = keep_chunk_id;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (gp.rope_on && components != CR_APPLY_V &&
+        (s = target_rope_table(d, pos, n_tokens, inv_freq_host, workspace, workspace_bytes, &gp, st)) != CR_OK)
+        return s;
     s = launch_gemm(yf, d.db, w->w_out, n_tokens, d.D, d.db, d.f32 ? EPI_KV_F32 : EPI_KV_BF16, gp,
                     kv_inout, d.D, st);
     // V-only under the target's R_M: the K segments the head did not visit are
@@ -743,7 +765,7 @@ cr_status cr_apply_residual_paged(const cr_target_dims* target, const cr_repaire
                                   const void* kv_stale, const int32_t* pos,
                                   const float* inv_freq_host, int32_t rope_mode,
                                   const int64_t* slot_mapping, void* paged_cache, int64_t num_slots,
-                                  void* stream) {
+                                  void* workspace, size_t workspace_bytes, void* stream) {
     cr_status s = check_target(target);
     if (s == CR_OK) s = check_repairer(rep);
     if (s != CR_OK) return s;
@@ -773,9 +795,13 @@ cr_status cr_apply_residual_paged(const cr_target_dims* target, const cr_repaire
     gp.paged = static_cast<uint16_t*>(paged_cache);
     gp.num_slots = num_slots;
     gp.seg_width = static_cast<int32_t>(plane);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (gp.rope_on &&
+        (s = target_rope_table(d, pos, n_tokens, inv_freq_host, workspace, workspace_bytes, &gp, st)) != CR_OK)
+        return s;
     // the stale tile is read through the same tensor map as the in-place update
     return launch_gemm(yf, d.db, w->w_out, n_tokens, d.D, d.db, EPI_KV_PAGED, gp,
-                       const_cast<void*>(kv_stale), d.D, static_cast<cudaStream_t>(stream));
+                       const_cast<void*>(kv_stale), d.D, st);
 }
 
 // ------------------------------------------------------------------ offline preparation
@@ -841,6 +867,27 @@ cr_status cr_linear(const uint16_t* A, int64_t lda, const uint16_t* W, const flo
     static const int map[4] = {EPI_BF16, EPI_GELU_BF16, EPI_ADD_F32, EPI_F32};
     return launch_gemm(A, lda, W, M, N, K, map[epi], gp, nullptr, 0,
                        static_cast<cudaStream_t>(stream));
+}
+
+cr_status cr_matmul(const uint16_t* A, int64_t lda, int32_t a_trans, const uint16_t* B, int64_t ldb,
+                    int64_t M, int64_t N, int64_t K, float* C, int64_t ldc, int32_t accumulate,
+                    void* workspace, size_t workspace_bytes, void* stream) {
+    if (M < 1 || N < 1 || K < 1 || M > INT32_MAX / 2 || N > INT32_MAX / 2 || K > INT32_MAX / 2)
+        return CR_ERR_INVALID_ARG;
+    if (workspace && !all_aligned(workspace)) return CR_ERR_INVALID_ARG;
+    if (!all_aligned(A, B, C) || (lda % 8) != 0 || (ldb % 8) != 0 || (ldc % 4) != 0 || ldb < N ||
+        ldc < N || lda < (a_trans ? M : K))
+        return CR_ERR_INVALID_ARG;
+    if ((N % 64) != 0 || (a_trans && (M % 64) != 0)) return CR_ERR_UNSUPPORTED;
+    unsigned* status = device_status_ptr();
+    if (!status) return CR_ERR_CUDA;
+    GemmParams gp{};
+    gp.status = status;
+    gp.out = C;
+    gp.ldo = ldc;
+    return launch_gemm_lay(A, lda, a_trans ? LAY_MM : LAY_KM, B, ldb, M, N, K,
+                           accumulate ? EPI_ADD_F32 : EPI_F32, gp, static_cast<cudaStream_t>(stream),
+                           static_cast<float*>(workspace), workspace ? workspace_bytes : 0);
 }
 
 cr_status cr_layernorm(const float* x, const float* add, int64_t ld_add, float* x_out,
@@ -1039,10 +1086,9 @@ namespace {
 struct TrainLayout {
     size_t inf, h0, rein, blk, blk_stride, hbuf, yf, rope, dz, rowsq, rowscale, losspart, perreq,
         stats_pad, dh, dxm, du, dtmp, pre, gprod, sig16, dqkv, da, lse, dvec, cstart, dse, dy, colsum, colcnt,
-        norm, blas, total;
+        norm, segw, splitk, total;
     size_t x_in, x_mid, u1, u2, qkv, o, g;   // offsets inside one block's region
 };
-constexpr size_t kBlasBytes = 32ull << 20;
 
 TrainLayout train_layout(const Dims& d, int64_t n) {
     TrainLayout L{};
@@ -1098,7 +1144,8 @@ TrainLayout train_layout(const Dims& d, int64_t n) {
     L.colsum = take(colsum_scratch_floats(n, std::max(d.D, wide)) * 4);
     L.colcnt = take(colsum_counters(std::max(d.D, wide)) * 4);
     L.norm = take(sqnorm_scratch_doubles() * 8);
-    L.blas = take(kBlasBytes);
+    L.segw = take(static_cast<size_t>(d.D) * 128 * 4);   // grouped W_seg gradient blocks
+    L.splitk = take(8 * N * d.db * 4);                     // split-K parts of the backward's products
     L.total = off;
     return L;
 }
@@ -1125,6 +1172,9 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
     if (s != CR_OK) return s;
     const Dims d = dims_of(target, rep);
     if (d.f32) return CR_ERR_UNSUPPORTED;
+    // the backward's products take whole 64-column boxes of every width
+    if (d.dc % 64 != 0 || d.dmodel % 64 != 0 || d.hid % 64 != 0 || (d.S * d.dseg) % 64 != 0)
+        return CR_ERR_UNSUPPORTED;
     if (!hp || !cu_seqlens_host || n_req < 1 || n_req > kMaxReq || n_tokens < 1 ||
         n_tokens > INT32_MAX / 2 || !valid_mask_mode(mask_mode))
         return CR_ERR_INVALID_ARG;
@@ -1234,6 +1284,9 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
     float* CS = at<float>(base, L.colsum);
     unsigned* CCNT = at<unsigned>(base, L.colcnt);
     double* NRM = at<double>(base, L.norm);
+    float* SEGW = at<float>(base, L.segw);
+    float* SPLITK = at<float>(base, L.splitk);
+    const size_t splitk_bytes = 8 * static_cast<size_t>(N) * d.db * 4;
 
     // ---- forward (Sec. 4.1), keeping what the backward needs
     s = cr_compress_features(target, rep, &w, kv_stale, emb, N, h0, rein, inf, IL.total, stream);
@@ -1334,8 +1387,6 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
     if (s != CR_OK) return s;
 
     // ---- backward: the chain rule in reverse, gradients straight into `grads`
-    cublasHandle_t hb;
-    if ((s = blas_handle(st, base + L.blas, kBlasBytes, &hb)) != CR_OK) return s;
     if ((s = cuda_check(cudaMemsetAsync(grads, 0, static_cast<size_t>(P) * 4, st))) != CR_OK) return s;
     // column-sum election counters start at zero (each use leaves them at zero)
     if ((s = cuda_check(cudaMemsetAsync(CCNT, 0, colsum_counters(std::max(d.D, std::max(std::max(d.hid, 3 * d.db),
@@ -1343,7 +1394,17 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
                                                      4,
                                         st))) != CR_OK)
         return s;
-    const cudaDataType_t BF = CUDA_R_16BF, F32 = CUDA_R_32F;
+    // The backward's products on the tensor cores: C [M, N] fp32 (= or, with acc,
+    // +=) op(A) B, B stored [K, N]; op(A) = A [M, K], or A^T for A stored [K, M]
+    auto mm = [&](const uint16_t* A, int64_t lda, bool a_trans, const uint16_t* B, int64_t ldb, int64_t M,
+                  int64_t Nc, int64_t K, float* C, int64_t ldc, bool acc) {
+        GemmParams gp{};
+        gp.status = status;
+        gp.out = C;
+        gp.ldo = ldc;
+        return launch_gemm_lay(A, lda, a_trans ? LAY_MM : LAY_KM, B, ldb, M, Nc, K, acc ? EPI_ADD_F32 : EPI_F32,
+                               gp, st, SPLITK, splitk_bytes);
+    };
     auto colsum = [&](const void* a, bool bf16, int64_t cols, int64_t lda, float* out) {
         return launch_colsum(a, bf16, N, cols, lda, out, false, CS, CCNT, st);
     };
@@ -1357,9 +1418,9 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
         if ((s = (x)) != CR_OK) return s; \
     } while (0)
     // head: dW_out = dz^T y_f, db_out = sum_t dz, dy_f = dz W_out
-    CR_TRY(gemm_rm(hb, true, false, D, db, N, 1.0f, DZ, BF, D, yf, BF, db, 0.0f, gk(W_OUT), F32, db));
+    CR_TRY(mm(DZ, D, true, yf, db, D, db, N, gk(W_OUT), db, false));
     CR_TRY(colsum(DZ, true, D, D, gk(B_OUT)));
-    CR_TRY(gemm_rm(hb, false, false, N, db, D, 1.0f, DZ, BF, D, pb(W_OUT), BF, db, 0.0f, DU, F32, db));
+    CR_TRY(mm(DZ, D, false, pb(W_OUT), db, N, db, D, DU, db, false));
     CR_TRY(launch_ln_backward(H, w.lnf_g, DU, nullptr, eps, N, static_cast<int>(db), DH, GPROD, st));
     CR_TRY(colsum(GPROD, false, db, db, gk(LNFG)));
     CR_TRY(colsum(DU, false, db, db, gk(LNFB)));
@@ -1374,9 +1435,8 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
         const uint16_t* g = reinterpret_cast<const uint16_t*>(blk(b, L.g));
         // h = x_mid + W_fc2 g + b_fc2
         CR_TRY(colsum16(DH, db, SIG, gk(bk(b, BFC2))));
-        CR_TRY(gemm_rm(hb, true, false, db, hid, N, 1.0f, SIG, BF, db, g, BF, hid, 0.0f, gk(bk(b, WFC2)), F32, hid));
-        CR_TRY(gemm_rm(hb, false, false, N, hid, db, 1.0f, SIG, BF, db, pb(bk(b, WFC2)), BF, hid, 0.0f, DTMP, F32,
-                       hid));
+        CR_TRY(mm(SIG, db, true, g, hid, db, hid, N, gk(bk(b, WFC2)), hid, false));
+        CR_TRY(mm(SIG, db, false, pb(bk(b, WFC2)), hid, N, hid, db, DTMP, hid, false));
         // g = GELU(pre), pre = W_fc1 u2 + b_fc1 (recomputed in fp32)
         GemmParams gp{};
         gp.status = status;
@@ -1386,17 +1446,16 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
         CR_TRY(launch_gemm(u2, db, pb(bk(b, WFC1)), N, hid, db, EPI_F32, gp, nullptr, 0, st));
         CR_TRY(launch_gelu_backward(DTMP, PRE, N * hid, st));
         CR_TRY(colsum16(DTMP, hid, SIG, gk(bk(b, BFC1))));
-        CR_TRY(gemm_rm(hb, true, false, hid, db, N, 1.0f, SIG, BF, hid, u2, BF, db, 0.0f, gk(bk(b, WFC1)), F32, db));
-        CR_TRY(gemm_rm(hb, false, false, N, db, hid, 1.0f, SIG, BF, hid, pb(bk(b, WFC1)), BF, db, 0.0f, DU, F32,
-                       db));
+        CR_TRY(mm(SIG, hid, true, u2, db, hid, db, N, gk(bk(b, WFC1)), db, false));
+        CR_TRY(mm(SIG, hid, false, pb(bk(b, WFC1)), db, N, db, hid, DU, db, false));
         // u2 = LN2(x_mid): dx_mid = dh + LN2 backward
         CR_TRY(launch_ln_backward(x_mid, pf(bk(b, LN2G)), DU, DH, eps, N, static_cast<int>(db), DXM, GPROD, st));
         CR_TRY(colsum(GPROD, false, db, db, gk(bk(b, LN2G))));
         CR_TRY(colsum(DU, false, db, db, gk(bk(b, LN2B))));
         // x_mid = x_in + W_o a + b_o
         CR_TRY(colsum16(DXM, db, SIG, gk(bk(b, BO))));
-        CR_TRY(gemm_rm(hb, true, false, db, db, N, 1.0f, SIG, BF, db, o, BF, db, 0.0f, gk(bk(b, WO)), F32, db));
-        CR_TRY(gemm_rm(hb, false, false, N, db, db, 1.0f, SIG, BF, db, pb(bk(b, WO)), BF, db, 0.0f, DA, F32, db));
+        CR_TRY(mm(SIG, db, true, o, db, db, db, N, gk(bk(b, WO)), db, false));
+        CR_TRY(mm(SIG, db, false, pb(bk(b, WO)), db, N, db, db, DA, db, false));
         // attention: the fused backward (P recomputed from the forward's log-sum-exp,
         // dQ, dK, dV into dqkv), dO in bf16 for its MMAs
         CR_TRY(to16(DA, N * db, SIG));
@@ -1406,39 +1465,45 @@ cr_status cr_train_step(const cr_target_dims* target, const cr_repairer_dims* re
         CR_TRY(launch_rope_backward(DQKV, rope, N, static_cast<int>(db), static_cast<int>(hd), st));
         // qkv = W_qkv u1 + b_qkv;  u1 = LN1(x_in): dx_in = dx_mid + LN1 backward
         CR_TRY(colsum16(DQKV, 3 * db, SIG, gk(bk(b, BQKV))));
-        CR_TRY(gemm_rm(hb, true, false, 3 * db, db, N, 1.0f, SIG, BF, 3 * db, u1, BF, db, 0.0f, gk(bk(b, WQKV)),
-                       F32, db));
-        CR_TRY(gemm_rm(hb, false, false, N, db, 3 * db, 1.0f, SIG, BF, 3 * db, pb(bk(b, WQKV)), BF, db, 0.0f, DU,
-                       F32, db));
+        CR_TRY(mm(SIG, 3 * db, true, u1, db, 3 * db, db, N, gk(bk(b, WQKV)), db, false));
+        CR_TRY(mm(SIG, 3 * db, false, pb(bk(b, WQKV)), db, N, db, 3 * db, DU, db, false));
         CR_TRY(launch_ln_backward(x_in, pf(bk(b, LN1G)), DU, DXM, eps, N, static_cast<int>(db), DH, GPROD, st));
         CR_TRY(colsum(GPROD, false, db, db, gk(bk(b, LN1G))));
         CR_TRY(colsum(DU, false, db, db, gk(bk(b, LN1B))));
         // x_in = h^{b-1} + W_rein,b s + b_rein,b: ds += dx_in W_rein,b
         CR_TRY(colsum16(DH, db, SIG, gk(B_REIN) + b * db));
-        CR_TRY(gemm_rm(hb, true, false, db, dc, N, 1.0f, SIG, BF, db, se, BF, 4 * dc, 0.0f, gk(W_REIN) + b * db * dc,
-                       F32, dc));
-        CR_TRY(gemm_rm(hb, false, false, N, dc, db, 1.0f, SIG, BF, db, pb(W_REIN) + b * db * dc, BF, dc, 1.0f, DSE,
-                       F32, 2 * dc));
+        CR_TRY(mm(SIG, db, true, se, 4 * dc, db, dc, N, gk(W_REIN) + b * db * dc, dc, false));
+        CR_TRY(mm(SIG, db, false, pb(W_REIN) + b * db * dc, dc, N, dc, db, DSE, 2 * dc, true));
     }
     // h0 = W_fuse [s; e] + b_fuse
     CR_TRY(colsum16(DH, db, SIG, gk(B_FUSE)));
-    CR_TRY(gemm_rm(hb, true, false, db, 2 * dc, N, 1.0f, SIG, BF, db, se, BF, 4 * dc, 0.0f, gk(W_FUSE), F32, 2 * dc));
-    CR_TRY(gemm_rm(hb, false, false, N, 2 * dc, db, 1.0f, SIG, BF, db, pb(W_FUSE), BF, 2 * dc, 1.0f, DSE, F32,
-                   2 * dc));
+    CR_TRY(mm(SIG, db, true, se, 4 * dc, db, 2 * dc, N, gk(W_FUSE), 2 * dc, false));
+    CR_TRY(mm(SIG, db, false, pb(W_FUSE), 2 * dc, N, 2 * dc, db, DSE, 2 * dc, true));
     // e = W_tok emb + b_tok;  s = W_map y + b_map
     CR_TRY(to16(DSE, N * 2 * dc, SIG));
-    CR_TRY(gemm_rm(hb, true, false, dc, d.dmodel, N, 1.0f, SIG + dc, BF, 2 * dc, emb, BF, d.dmodel, 0.0f, gk(W_TOK),
-                   F32, d.dmodel));
+    CR_TRY(mm(SIG + dc, 2 * dc, true, static_cast<const uint16_t*>(emb), d.dmodel, dc, d.dmodel, N, gk(W_TOK),
+              d.dmodel, false));
     CR_TRY(colsum(DSE + dc, false, dc, 2 * dc, gk(B_TOK)));
     const int64_t Sd = d.S * d.dseg;
-    CR_TRY(gemm_rm(hb, true, false, dc, Sd, N, 1.0f, SIG, BF, 2 * dc, y, BF, 2 * Sd, 0.0f, gk(W_MAP), F32, Sd));
+    CR_TRY(mm(SIG, 2 * dc, true, y, 2 * Sd, dc, Sd, N, gk(W_MAP), Sd, false));
     CR_TRY(colsum(DSE, false, dc, 2 * dc, gk(B_MAP)));
-    CR_TRY(gemm_rm(hb, false, false, N, Sd, dc, 1.0f, SIG, BF, 2 * dc, pb(W_MAP), BF, Sd, 0.0f, DY, F32, Sd));
-    // y_{t,s} = (W_seg,s / sigma_stale) kv_{t,s} + b_seg,s: per segment dy^T kv, then / sigma_stale
+    CR_TRY(mm(SIG, 2 * dc, false, pb(W_MAP), Sd, N, Sd, dc, DY, Sd, false));
+    // y_{t,s} = (W_seg,s / sigma_stale) kv_{t,s} + b_seg,s: per segment kv_s^T dy_s
+    // ([d_h, d_seg], summed over tokens), then / sigma_stale.  One grouped product:
+    // the d_h rows of 128 / d_seg consecutive segments share one 128-column block
+    // of dy, the block holding their own d_seg columns; their other columns are
+    // computed and dropped (the product reads kv once, which bounds it).
     CR_TRY(colsum16(DY, Sd, SIG, gk(B_SEG)));
-    CR_TRY(gemm_rm(hb, true, false, d.dseg, d.dh, N, 1.0f, SIG, BF, Sd, kv_stale, BF, D, 0.0f, gk(W_SEG), F32, d.dh,
-                   d.S, d.dseg, d.dh, d.dseg * d.dh));
-    CR_TRY(launch_scale_seg_grad(gk(W_SEG), d.S, d.dseg, d.dh, sigma_stale, st));
+    {
+        GemmParams gp{};
+        gp.status = status;
+        gp.out = SEGW;
+        gp.ldo = 128;
+        gp.bgroup_rows = static_cast<int32_t>((128 / d.dseg) * d.dh);
+        CR_TRY(launch_gemm_lay(static_cast<const uint16_t*>(kv_stale), D, LAY_MM, SIG, Sd, D, 128, N, EPI_F32, gp,
+                               st));
+    }
+    CR_TRY(launch_seg_grad(SEGW, gk(W_SEG), d.S, d.dseg, d.dh, sigma_stale, st));
 
     // ---- clipping and AdamW (App. A)
     AdamWParams ah{};

@@ -251,6 +251,21 @@ __device__ __forceinline__ int tile_n0(const GemmParams& p, int t) {
     return c * BN;
 }
 
+// The same rotation with (cos, sin) read from a per-call angle-major table
+// (entry q * M + row, written by the RoPE-table kernel with sincos_prod's
+// formula: the same rotation to the last bit of an angle).
+__device__ __forceinline__ void rotate16_tab(float* a, float* b, const float2* tab, int64_t M, int row,
+                                             int j0) {
+    const float2* t = tab + static_cast<int64_t>(j0) * M + row;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        const float2 v = __ldg(t + i * M);
+        const float x = a[i], y = b[i];
+        a[i] = x * v.x - y * v.y;
+        b[i] = y * v.x + x * v.y;
+    }
+}
+
 __device__ __forceinline__ void rotate16(float* a, float* b, float p, const float* inv_freq, int j0) {
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
@@ -262,13 +277,23 @@ __device__ __forceinline__ void rotate16(float* a, float* b, float p, const floa
     }
 }
 
-template <int BN, int EPI, int CG>
+// Operand layouts (LAY, cr_internal.h): LAY_KK = A [M, K] and W [N, K], both
+// K-major (the forward's linears); LAY_KM = A K-major, W stored [K, N]
+// (MN-major: dX = dY W of the backward); LAY_MM = A stored [K, M] and W [K, N],
+// both MN-major (dW = dY^T X).  An MN-major operand arrives as 64-wide boxes of
+// 64 K-rows (128B swizzle): the MMA descriptor steps 16 K-rows (2 KB) per
+// K = 16 MMA and finds the next 64 M (or N) 8 KB further on (leading byte
+// offset).
+
+template <int BN, int EPI, int CG, int LAY>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const __grid_constant__ CUtensorMap tmC, const __grid_constant__ GemmParams p) {
     using Cfg = GemmCfg<BN, EPI, CG>;
     constexpr int STAGES = Cfg::kStages;
-    constexpr uint32_t IDESC = idesc_bf16(BM * CG, BN, false, false);
+    constexpr bool kAMN = (LAY == LAY_MM), kBMN = (LAY != LAY_KK);
+    static_assert(!kBMN || (BN / CG) % 64 == 0, "an MN-major W half must be whole 64-column boxes");
+    constexpr uint32_t IDESC = idesc_bf16(BM * CG, BN, kAMN, kBMN);
 
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -335,9 +360,17 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const uint32_t tmem_base = *tmem_slot;
     const WaitCtx wc{abort_flag, p.status};
 
-    const int total = p.num_m * p.num_n;
+    // split-K (split_k > 1): tile t / split_k, k-blocks of part t % split_k; each
+    // part's fp32 result goes to its own [M, N] slice of the output (rows
+    // (t % split_k) M ..), summed later in a fixed order
+    const int total = p.num_m * p.num_n * p.split_k;
     // a two-term A runs the W k-blocks twice: first against A_hi, then A_lo
     const int num_k = p.split_kb > 0 ? 2 * p.split_kb : (p.K + BK - 1) / BK;
+    const int k_per = (num_k + p.split_k - 1) / p.split_k;
+    auto k_range = [&](int t, int* kb0, int* kb1) {
+        *kb0 = (t % p.split_k) * k_per;
+        *kb1 = min(num_k, *kb0 + k_per);
+    };
     const bool has_bias = p.bias != nullptr;
     // the epilogue consumes a per-tile load (vectors and/or the in-place tile)
     const bool epi_load = Cfg::kInPlace || has_bias;
@@ -361,27 +394,47 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         uint32_t stage = 0, phase = 0;
         bool ok = true;
         for (int t = cta0; t < total && ok; t += ncta) {
-            const int m0 = (t % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-            const int n0 = tile_n0<BN, Cfg::kKV>(p, t);
-            for (int kb = 0; kb < num_k; ++kb) {
+            const int m0 = ((t / p.split_k) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
+            const int n0 = tile_n0<BN, Cfg::kKV>(p, t / p.split_k);
+            int kbeg, kend;
+            k_range(t, &kbeg, &kend);
+            for (int kb = kbeg; kb < kend; ++kb) {
                 if (!(ok = mbar_wait_warp(&empty[stage], phase ^ 1u, wc, 102))) break;
                 uint8_t* sa = smem + stage * Cfg::kStageBytes;
                 if (elect_one()) {
-                    const int nb0 = n0 + static_cast<int>(rank) * (BN / CG);
+                    // W columns of this tile: its own column block, or (grouped
+                    // rows) the block that belongs to its rows' group
+                    const int nw = p.bgroup_rows > 0
+                                       ? (((t / p.split_k) % p.num_m) * (BM * CG) / p.bgroup_rows) * BN : n0;
+                    const int nb0 = nw + static_cast<int>(rank) * (BN / CG);
                     const bool lo = p.split_kb > 0 && kb >= p.split_kb;
                     const CUtensorMap* ma = lo ? &p.tm_alo : &tmA;
                     const int ka = (lo ? kb - p.split_kb : kb) * BK;   // A and W column
-                    if (CG == 1) {
+                    auto load = [&](uint8_t* dst, const CUtensorMap* m, int x, int y, uint32_t fb) {
+                        if constexpr (CG == 1)
+                            tma_load_2d(dst, m, &full[stage], x, y);
+                        else
+                            tma_load_2d_pair(dst, m, fb, x, y);
+                    };
+                    // both CTAs' copies count on the even CTA's barrier, which
+                    // expects the pair's bytes (its own arrive is the only one)
+                    const uint32_t fb = CG == 2 ? mapa_shared(smem_u32(&full[stage]), 0) : 0u;
+                    if (CG == 1)
                         mbar_expect_tx(&full[stage], Cfg::kStageBytes);
-                        tma_load_2d(sa, ma, &full[stage], ka, m0);
-                        tma_load_2d(sa + A_BYTES, &tmB, &full[stage], ka, nb0);
+                    else if (rank == 0)
+                        mbar_expect_tx(&full[stage], CG * Cfg::kStageBytes);
+                    if constexpr (kAMN) {
+                        load(sa, ma, m0, ka, fb);
+                        load(sa + A_BYTES / 2, ma, m0 + 64, ka, fb);
                     } else {
-                        // both CTAs' copies count on the even CTA's barrier, which
-                        // expects the pair's bytes (its own arrive is the only one)
-                        const uint32_t fb = mapa_shared(smem_u32(&full[stage]), 0);
-                        if (rank == 0) mbar_expect_tx(&full[stage], CG * Cfg::kStageBytes);
-                        tma_load_2d_pair(sa, ma, fb, ka, m0);
-                        tma_load_2d_pair(sa + A_BYTES, &tmB, fb, ka, nb0);
+                        load(sa, ma, ka, m0, fb);
+                    }
+                    if constexpr (kBMN) {
+#pragma unroll
+                        for (int i = 0; i < BN / CG / 64; ++i)
+                            load(sa + A_BYTES + i * 8192, &tmB, nb0 + 64 * i, ka, fb);
+                    } else {
+                        load(sa + A_BYTES, &tmB, ka, nb0, fb);
                     }
                 }
                 __syncwarp();
@@ -407,8 +460,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             bool ok = true;
             int i = 0;
             for (int t = cta0; t < total && ok; t += ncta, ++i) {
-                const int m0 = (t % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-                const int n0 = tile_n0<BN, Cfg::kKV>(p, t);
+                const int m0 = ((t / p.split_k) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
+                const int n0 = tile_n0<BN, Cfg::kKV>(p, t / p.split_k);
                 const int nb = min(BN, p.N - n0);
                 const uint32_t vbytes = static_cast<uint32_t>(nb) * 4u;
                 if constexpr (Cfg::kInPlace) {
@@ -466,8 +519,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         uint32_t pk = 0;               // in-place tiles so far
         uint32_t pkg[2] = {0u, 0u};    // boxes of each epilogue group so far
         for (int t = cta0; t < total && ok; t += ncta) {
-            const int m0 = (t % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-            const int n0 = tile_n0<BN, Cfg::kKV>(p, t);
+            const int m0 = ((t / p.split_k) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
+            const int n0 = tile_n0<BN, Cfg::kKV>(p, t / p.split_k);
             const bool rows_in = m0 < p.M;   // a pair tile's second half may lie below M
             if constexpr (Cfg::kInPlace) {
                 // each box as soon as the epilogue has written it; once TMA has read
@@ -493,7 +546,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     const uint32_t b = static_cast<uint32_t>(g) * GB + (pkg[g] % GB);
                     if (!(ok = mbar_wait_warp(&epi_done[b], (pkg[g] / GB) & 1u, wc, 402))) break;
                     if (leader) {
-                        if (rows_in) tma_store_2d(&tmC, tile + b * 16384, n0 + k * Cfg::kBoxCols, m0);
+                        if (rows_in)
+                            tma_store_2d(&tmC, tile + b * 16384, n0 + k * Cfg::kBoxCols,
+                                         m0 + (t % p.split_k) * p.M);
                         tma_store_commit();
                         tma_store_wait_read0();
                         mbar_arrive(&st_free[b]);
@@ -512,27 +567,32 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         // (for a pair: the even CTA, issuing M = 256 MMAs over both CTAs'
         // shared memory and TMEM, committing to the barriers of both)
         // Stage descriptors: a K=16 step adds 32 bytes (2 units of 16 B) to the
-        // start address, a stage kStageBytes, the W operand A_BYTES.
-        const uint64_t da0 = smem_desc(smem_u32(smem), 16, 1024, SWZ_128B);
+        // start address of a K-major operand and 16 rows (2 KB) to an MN-major
+        // one, a stage kStageBytes, the W operand A_BYTES.
+        const uint64_t da0 = smem_desc(smem_u32(smem), kAMN ? 8192 : 16, 1024, SWZ_128B);
+        const uint64_t db0 = smem_desc(smem_u32(smem + A_BYTES), kBMN ? 8192 : 16, 1024, SWZ_128B);
         constexpr uint64_t kStageStep = Cfg::kStageBytes >> 4;
-        constexpr uint64_t kBStep = A_BYTES >> 4;
+        constexpr uint64_t kAK = kAMN ? (2048 >> 4) : 2, kBK = kBMN ? (2048 >> 4) : 2;
         uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
         bool ok = true;
         for (int t = cta0; t < total && ok; t += ncta) {
             if (!(ok = mbar_wait_warp(&tempty[acc], acc_phase ^ 1u, wc, 201))) break;
             tc_fence_after();
             const uint32_t d = tmem_base + acc * BN;
-            for (int kb = 0; kb < num_k; ++kb) {
+            int kbeg, kend;
+            k_range(t, &kbeg, &kend);
+            for (int kb = kbeg; kb < kend; ++kb) {
                 if (!(ok = mbar_wait_warp(&full[stage], phase, wc, 202))) break;
                 tc_fence_after();
                 const uint64_t da = da0 + stage * kStageStep;
+                const uint64_t dw = db0 + stage * kStageStep;
                 if (elect_one()) {
 #pragma unroll
                     for (int k = 0; k < BK / 16; ++k) {
                         if constexpr (CG == 2)
-                            mma_bf16_ss2(d, da + 2 * k, da + kBStep + 2 * k, IDESC, (kb | k) != 0 ? 1u : 0u);
+                            mma_bf16_ss2(d, da + kAK * k, dw + kBK * k, IDESC, (kb != kbeg || k != 0) ? 1u : 0u);
                         else
-                            mma_bf16_ss(d, da + 2 * k, da + kBStep + 2 * k, IDESC, (kb | k) != 0 ? 1u : 0u);
+                            mma_bf16_ss(d, da + kAK * k, dw + kBK * k, IDESC, (kb != kbeg || k != 0) ? 1u : 0u);
                     }
                     if constexpr (CG == 2)
                         mma_commit2_mc(&empty[stage], 0x3);
@@ -588,8 +648,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         bool ok = true;
         int i = 0;
         for (int t = cta0; t < total && ok; t += ncta, ++i) {
-            const int m0 = (t % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-            const int n0 = tile_n0<BN, Cfg::kKV>(p, t);
+            const int m0 = ((t / p.split_k) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
+            const int n0 = tile_n0<BN, Cfg::kKV>(p, t / p.split_k);
             // QKV: the rotation angles depend on (row, pair index) only: cos/sin
             // for every head of the tile, fetched while the MMAs still run
             constexpr int NP = (EPI == EPI_QKV_ROPE) ? 32 : 1;
@@ -743,7 +803,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                                     kb[q] = fmaf(sb_[q], b[q] + bb[q], kb[q]);
                                 }
                             }
-                            if (rot) rotate16(ka, kb, pr, p.inv_freq, j);
+                            if (rot) {
+                                if (p.rope_table)
+                                    rotate16_tab(ka, kb, p.rope_table, p.M, row_ok ? row : 0, j);
+                                else
+                                    rotate16(ka, kb, pr, p.inv_freq, j);
+                            }
                             put16(ta, ka);
                             put16(tb, kb);
                         }
@@ -895,11 +960,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     }
 }
 
-template <int BN, int EPI, int CG>
+template <int BN, int EPI, int CG, int LAY = LAY_KK>
 cr_status launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
                     const GemmParams& p, cudaStream_t st) {
     using Cfg = GemmCfg<BN, EPI, CG>;
-    auto kern = gemm_kernel<BN, EPI, CG>;
+    auto kern = gemm_kernel<BN, EPI, CG, LAY>;
     static unsigned long long attr_done = 0;   // one per template instantiation
     const cr_status sa = ensure_smem_attr(kern, static_cast<int>(Cfg::kSmemBytes), &attr_done);
     if (sa != CR_OK) return sa;
@@ -1001,6 +1066,7 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
     p.K = static_cast<int32_t>(K);
     p.num_m = static_cast<int32_t>((M + BM * kCG - 1) / (BM * kCG));
     p.num_n = static_cast<int32_t>((N + BN - 1) / BN);
+    p.split_k = 1;
     if (kv && p.col_block > 0) {
         // output choice: half of the column blocks, each a whole number of tiles
         if (p.col_block % BN != 0 || N % (2 * static_cast<int64_t>(p.col_block)) != 0)
@@ -1070,6 +1136,139 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
         default:
             return CR_ERR_INVALID_ARG;
     }
+}
+
+namespace {
+// C [M, N] (row stride ldc) = (or += with accumulate) the sum over u < s of
+// part[u] ([M, N] slices, contiguous), in order u = 0, 1, ..: the split-K parts
+// of one product, four columns per thread.
+__global__ void __launch_bounds__(256)
+    splitk_reduce_kernel(const float* __restrict__ part, int s, int64_t M, int64_t N, float* C, int64_t ldc,
+                         int accumulate) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int64_t n4 = N >> 2, total = M * n4;
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t m = i / n4, c = (i - m * n4) << 2;
+        float4 acc = *reinterpret_cast<const float4*>(part + m * N + c);
+        for (int u = 1; u < s; ++u) {
+            const float4 v = *reinterpret_cast<const float4*>(part + (u * M + m) * N + c);
+            acc.x += v.x;
+            acc.y += v.y;
+            acc.z += v.z;
+            acc.w += v.w;
+        }
+        float4* dst = reinterpret_cast<float4*>(C + m * ldc + c);
+        if (accumulate) {
+            const float4 o = *dst;
+            acc.x += o.x;
+            acc.y += o.y;
+            acc.z += o.z;
+            acc.w += o.w;
+        }
+        *dst = acc;
+    }
+}
+}  // namespace
+
+cr_status launch_gemm_lay(const uint16_t* A, int64_t lda, int lay, const uint16_t* W, int64_t ldw,
+                          int64_t M, int64_t N, int64_t K, int epi, GemmParams p, cudaStream_t st,
+                          float* scratch, size_t scratch_bytes) {
+    if (lay != LAY_KM && lay != LAY_MM) return CR_ERR_INVALID_ARG;
+    if (epi != EPI_F32 && epi != EPI_ADD_F32) return CR_ERR_UNSUPPORTED;
+    if (M < 1 || N < 1 || K < 1 || (N % 64) != 0 || (lay == LAY_MM && (M % 64) != 0))
+        return CR_ERR_UNSUPPORTED;
+    // Tile width as in launch_gemm (rounds x (256 + BN)); an MN-major W half is
+    // whole 64-column boxes, so 256 or 128 (the in-place fp32 tile: 128).
+    int BN = 128;
+    if (epi == EPI_F32 && p.bgroup_rows == 0) {
+        const int64_t pairs = num_sms() / kCG > 0 ? num_sms() / kCG : 1;
+        const int64_t mt = (M + BM * kCG - 1) / (BM * kCG);
+        const int64_t c256 = ((mt * ((N + 255) / 256) + pairs - 1) / pairs) * (256 + 256);
+        const int64_t c128 = ((mt * ((N + 127) / 128) + pairs - 1) / pairs) * (256 + 128);
+        BN = c256 <= c128 ? 256 : 128;
+    }
+    p.M = static_cast<int32_t>(M);
+    p.N = static_cast<int32_t>(N);
+    p.K = static_cast<int32_t>(K);
+    p.num_m = static_cast<int32_t>((M + BM * kCG - 1) / (BM * kCG));
+    p.num_n = static_cast<int32_t>((N + BN - 1) / BN);
+    p.col_block = 0;
+    p.split_kb = 0;
+    p.split_k = 1;
+    // Split-K: when the tiles fill the CTA pairs poorly (the last round partly
+    // empty), cut each tile's k-loop into s parts, each written to its own fp32
+    // slice of the scratch and summed in a fixed order by a second kernel.  s
+    // minimises rounds(s) / s x tile time + the sum's traffic, with every part
+    // at least four k-blocks.
+    const int64_t pairs = num_sms() / kCG > 0 ? num_sms() / kCG : 1;
+    const int64_t tiles = static_cast<int64_t>(p.num_m) * p.num_n;
+    const int64_t nkb = (K + BK - 1) / BK;
+    // (whole 128-row boxes only: a part's rows must not spill into the next slice)
+    if (scratch && p.bgroup_rows == 0 && M % BM == 0) {
+        const double tile_us = static_cast<double>(nkb) * (256 + BN) / 1.9e3;   // ~1.9 GHz
+        double best = static_cast<double>((tiles + pairs - 1) / pairs) * tile_us;
+        for (int sk = 2; sk <= 8; sk *= 2) {
+            const int64_t kp = (nkb + sk - 1) / sk;
+            if (kp < 4 || (sk - 1) * kp >= nkb) break;
+            const size_t need = static_cast<size_t>(sk) * M * N * 4;
+            if (need > scratch_bytes) break;
+            const double t = static_cast<double>((tiles * sk + pairs - 1) / pairs) * tile_us / sk +
+                             static_cast<double>(need + static_cast<size_t>(M) * N * 4 * (epi == EPI_ADD_F32 ? 2 : 1)) /
+                                 6.0e6;   // bytes at ~6 TB/s, in microseconds
+            if (t < best * 0.95) {
+                best = t;
+                p.split_k = sk;
+            }
+        }
+    }
+    float* const C = static_cast<float*>(p.out);
+    const int64_t ldc = p.ldo;
+    if (p.split_k > 1) {
+        p.out = scratch;
+        p.ldo = N;
+    }
+    if (p.bgroup_rows > 0) {
+        // grouped rows: one column block per tile, the W block of the tile's group
+        if (p.bgroup_rows % (BM * kCG) != 0 || N != BN) return CR_ERR_UNSUPPORTED;
+        p.num_n = 1;
+    }
+    CUtensorMap ta, tb, tc;
+    const bool amn = (lay == LAY_MM);
+    if (!make_tmap_2d(&ta, A, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, amn ? M : K, amn ? K : M, lda * 2,
+                      amn ? 64 : BK, amn ? BK : BM, CU_TENSOR_MAP_SWIZZLE_128B))
+        return CR_ERR_INVALID_ARG;
+    const int64_t wcols = p.bgroup_rows > 0 ? ldw : N;   // grouped: W blocks of every group
+    if (!make_tmap_2d(&tb, W, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, wcols, K, ldw * 2, 64, BK,
+                      CU_TENSOR_MAP_SWIZZLE_128B))
+        return CR_ERR_INVALID_ARG;
+    if (!make_tmap_2d(&tc, p.out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, N, M * p.split_k, p.ldo * 4, 32, BM,
+                      CU_TENSOR_MAP_SWIZZLE_128B))
+        return CR_ERR_INVALID_ARG;
+    cr_status s;
+    if (p.split_k > 1) {
+        // the parts are plain fp32 products; the sum adds into C for EPI_ADD_F32
+        s = amn ? (BN == 256 ? launch_bn<256, EPI_F32, kCG, LAY_MM>(ta, tb, tc, p, st)
+                             : launch_bn<128, EPI_F32, kCG, LAY_MM>(ta, tb, tc, p, st))
+                : (BN == 256 ? launch_bn<256, EPI_F32, kCG, LAY_KM>(ta, tb, tc, p, st)
+                             : launch_bn<128, EPI_F32, kCG, LAY_KM>(ta, tb, tc, p, st));
+        if (s != CR_OK) return s;
+        const int64_t n4 = M * (N / 4);
+        int64_t blocks = (n4 + 255) / 256;
+        if (blocks > static_cast<int64_t>(num_sms()) * 16) blocks = static_cast<int64_t>(num_sms()) * 16;
+        return launch_pdl(splitk_reduce_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st,
+                          static_cast<const float*>(scratch), static_cast<int>(p.split_k), M, N, C, ldc,
+                          epi == EPI_ADD_F32 ? 1 : 0);
+    }
+    if (epi == EPI_ADD_F32)
+        return amn ? launch_bn<128, EPI_ADD_F32, kCG, LAY_MM>(ta, tb, tc, p, st)
+                   : launch_bn<128, EPI_ADD_F32, kCG, LAY_KM>(ta, tb, tc, p, st);
+    if (amn)
+        return BN == 256 ? launch_bn<256, EPI_F32, kCG, LAY_MM>(ta, tb, tc, p, st)
+                         : launch_bn<128, EPI_F32, kCG, LAY_MM>(ta, tb, tc, p, st);
+    return BN == 256 ? launch_bn<256, EPI_F32, kCG, LAY_KM>(ta, tb, tc, p, st)
+                     : launch_bn<128, EPI_F32, kCG, LAY_KM>(ta, tb, tc, p, st);
 }
 
 }  // namespace cr

@@ -4,8 +4,6 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
-#include <cublas_v2.h>
-
 #include "cr.h"
 #include "cr_ops.h"
 
@@ -62,6 +60,10 @@ enum GemmEpi : int {
                         // and per-row partial sums of r^2 instead of storing r
 };
 
+// Operand layouts of the GEMM: K-major A and W (the forward), K-major A with
+// MN-major W (dX = dY W), MN-major A and W (dW = dY^T X).
+enum GemmLayout : int { LAY_KK = 0, LAY_KM = 1, LAY_MM = 2 };
+
 struct GemmParams {
     int32_t M, N, K;
     int32_t num_m, num_n;
@@ -102,6 +104,13 @@ struct GemmParams {
     // same k-blocks of A_lo (tm_alo) against the same W columns, into one
     // accumulator: A at about 16 significant bits for twice the MMAs.  0 = plain A.
     int32_t split_kb;
+    // split-K (launch_gemm_lay): parts per tile, each writing rows [u M, (u + 1) M)
+    // of the output (1 = off; every launcher sets it)
+    int32_t split_k;
+    // grouped rows (launch_gemm_lay): every bgroup_rows rows of A form a group whose
+    // tile reads W columns [g BN, (g + 1) BN) of the W matrix, g = row / bgroup_rows,
+    // and writes output columns [0, BN); 0 = off
+    int32_t bgroup_rows;
     float inv_freq[64];      // RoPE frequencies, rope_dim / 2 entries
     CUtensorMap tm_joint;    // EPI_KV_LOSS (set by launch_gemm; the type carries its alignment)
     CUtensorMap tm_alo;      // two-term A: the A_lo operand
@@ -239,6 +248,16 @@ cr_status launch_sigma_finalize(const double* sumsq, int64_t D, int64_t count, f
 cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t M, int64_t N,
                       int64_t K, int epi, GemmParams p, void* kv_base, int64_t ld_kv,
                       cudaStream_t st, const uint16_t* A_lo = nullptr);
+// The backward's products, C [M, N] fp32 (out = p.out, row stride p.ldo) =, or
+// += with EPI_ADD_F32, A' W' where W' [K, N] is stored MN-major (row k of W at
+// W + k ldw, N contiguous) and A' [M, K] is A [M, K] K-major (lay LAY_KM = 1) or
+// stored [K, M] MN-major (lay LAY_MM = 2), row stride lda.  N a multiple of 64;
+// with LAY_MM also M.  No bias.
+// scratch (optional, fp32, scratch_bytes long): room for split-K parts; with it
+// the product may run as up to 8 k-parts summed in a fixed order afterwards.
+cr_status launch_gemm_lay(const uint16_t* A, int64_t lda, int lay, const uint16_t* W, int64_t ldw,
+                          int64_t M, int64_t N, int64_t K, int epi, GemmParams p, cudaStream_t st,
+                          float* scratch = nullptr, size_t scratch_bytes = 0);
 cr_status launch_segproj(const uint16_t* kv, int64_t ld_kv, const uint16_t* wfold, int head_dim,
                          SegParams p, cudaStream_t st);
 // The same projection reading the cache tiles straight from the pool (rows
@@ -290,16 +309,14 @@ cr_status launch_ln_backward(const float* x, const float* gamma, const float* dy
                              int64_t N, int D, float* dx, float* gprod, cudaStream_t st);
 cr_status launch_gelu_backward(float* dg, const float* pre, int64_t n, cudaStream_t st);
 cr_status launch_rope_backward(float* dqkv, const float2* table, int64_t N, int db, int hd, cudaStream_t st);
-cr_status launch_scale_seg_grad(float* g, int64_t S, int64_t dseg, int64_t dh, const float* sigma,
-                                cudaStream_t st);
+// The W_seg gradient from the grouped dW GEMM's blocks ([S d_h, 128] fp32, the
+// rows of segment s carrying its d_seg columns at (s mod (128 / d_seg)) d_seg):
+// g [S][d_seg][d_h] = block / sigma_stale (the fold of 1/sigma into W_seg).
+cr_status launch_seg_grad(const float* blocks, float* g, int64_t S, int64_t dseg, int64_t dh,
+                          const float* sigma, cudaStream_t st);
 size_t sqnorm_scratch_doubles();
 cr_status launch_clip_adamw(float* p, float* m, float* v, const float* g, uint16_t* pb, int64_t n,
                             const AdamWParams& hp, float max_norm, double* scratch, float* stats,
                             cudaStream_t st);
-cr_status blas_handle(cudaStream_t st, void* ws, size_t ws_bytes, cublasHandle_t* out);
-cr_status gemm_rm(cublasHandle_t h, bool tA, bool tB, int64_t M, int64_t N, int64_t K, float alpha,
-                  const void* A, cudaDataType_t ta, int64_t lda, const void* B, cudaDataType_t tb, int64_t ldb,
-                  float beta, void* C, cudaDataType_t tc, int64_t ldc, int64_t batch = 1, int64_t sA = 0,
-                  int64_t sB = 0, int64_t sC = 0);
 
 }  // namespace cr

@@ -1,6 +1,6 @@
 // Training-step kernels (Sec. 4.2, App. A): the bandwidth-bound pieces of the
-// backward pass and of the optimizer, plus the row-major GEMM helpers over
-// cuBLAS that the backward's plain (unfused) matrix products use.
+// backward pass and of the optimizer (the backward's matrix products run in
+// the tcgen05 GEMM, launch_gemm_lay).
 //   row_scale_kernel     c_request of every row, for the loss head's epilogue
 //   rowsq_kernel         per row: the loss head's partial sums of r^2 in order
 //   loss_reduce_kernel   per request, rows summed in order (fp64): the loss
@@ -10,7 +10,7 @@
 //   rope_backward_kernel the repairer RoPE's transpose on dQ, dK
 //   sqnorm_*             squared L2 norm of the gradient (fp64, fixed order)
 //   adamw_kernel         clipping coefficient, AdamW, bf16 mirror of the weights
-#include <cublas_v2.h>
+//   seg_grad_kernel      the segment weights' gradient out of the grouped GEMM's blocks
 #include <cuda_bf16.h>
 
 #include "cr_internal.h"
@@ -280,17 +280,22 @@ __global__ void __launch_bounds__(256)
 
 // out[i] = in[i] * scale[i % cols] (dW_seg: the cache's 1 / sigma_stale per column)
 __global__ void __launch_bounds__(256)
-    scale_cols_kernel(float* __restrict__ a, int64_t n, const float* __restrict__ sigma, int64_t period,
-                      int64_t seg_cols, int64_t d_seg) {
+    seg_grad_kernel(const float* __restrict__ blocks, float* __restrict__ g, int64_t S, int64_t d_seg,
+                    int64_t dh, const float* __restrict__ sigma) {
     pdl_launch_dependents();
     pdl_wait();
+    // blocks [S d_h, 128]: row s d_h + d of segment s holds sum_t kv[t, s d_h + d] dy[t, c]
+    // for the 128 columns c of its group; segment s's own d_seg columns start at
+    // (s mod (128 / d_seg)) d_seg.  g = [S][d_seg][d_h], divided by sigma_stale.
+    const int64_t n = S * d_seg * dh;
+    const int64_t spg = 128 / d_seg;
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        // a = [S][d_seg][d_h]: element (s, ., j) divides by sigma[s d_h + j]
-        const int64_t s = i / period;
-        const int64_t j = i % seg_cols;
-        (void)d_seg;
-        a[i] /= __ldg(sigma + s * seg_cols + j);
+        const int64_t s = i / (d_seg * dh);
+        const int64_t r = i - s * d_seg * dh;
+        const int64_t j = r / dh, d = r - j * dh;
+        const int64_t row = s * dh + d;
+        g[i] = __ldg(blocks + row * 128 + (s % spg) * d_seg + j) / __ldg(sigma + row);
     }
 }
 
@@ -458,10 +463,11 @@ cr_status launch_rope_backward(float* dqkv, const float2* table, int64_t N, int 
     return launch_pdl(rope_backward_kernel, grid_for(N * db), dim3(256), 0, st, dqkv, table, N, db, hd);
 }
 
-cr_status launch_scale_seg_grad(float* g, int64_t S, int64_t dseg, int64_t dh, const float* sigma,
-                                cudaStream_t st) {
+cr_status launch_seg_grad(const float* blocks, float* g, int64_t S, int64_t dseg, int64_t dh,
+                          const float* sigma, cudaStream_t st) {
+    if (128 % dseg != 0) return CR_ERR_UNSUPPORTED;
     const int64_t n = S * dseg * dh;
-    return launch_pdl(scale_cols_kernel, grid_for(n), dim3(256), 0, st, g, n, sigma, dseg * dh, dh, dseg);
+    return launch_pdl(seg_grad_kernel, grid_for(n), dim3(256), 0, st, blocks, g, S, dseg, dh, sigma);
 }
 
 size_t sqnorm_scratch_doubles() { return kNormCtas; }
@@ -477,53 +483,6 @@ cr_status launch_clip_adamw(float* p, float* m, float* v, const float* g, uint16
     if (n % 4 != 0) return CR_ERR_UNSUPPORTED;
     return launch_pdl(adamw_kernel, grid_for(n / 4), dim3(256), 0, st, p, m, v, g, pb, n, hp,
                       static_cast<const float*>(stats));
-}
-
-// ------------------------------------------------------------------ cuBLAS, row-major
-// One handle per device, created on first use; its workspace is set to a
-// caller-provided region before every call, so cuBLAS allocates nothing per call.
-namespace {
-cublasHandle_t g_blas[64];
-}
-
-cr_status blas_handle(cudaStream_t st, void* ws, size_t ws_bytes, cublasHandle_t* out) {
-    const int d = current_device_index();
-    if (d < 0 || d >= 64) return CR_ERR_CUDA;
-    if (!g_blas[d]) {
-        cublasHandle_t h;
-        if (cublasCreate(&h) != CUBLAS_STATUS_SUCCESS) return CR_ERR_CUDA;
-        cublasHandle_t expected = nullptr;
-        if (!__atomic_compare_exchange_n(&g_blas[d], &expected, h, false, __ATOMIC_ACQ_REL, __ATOMIC_ACQUIRE))
-            cublasDestroy(h);
-    }
-    cublasHandle_t h = g_blas[d];
-    if (cublasSetStream(h, st) != CUBLAS_STATUS_SUCCESS) return CR_ERR_CUDA;
-    if (cublasSetWorkspace(h, ws, ws_bytes) != CUBLAS_STATUS_SUCCESS) return CR_ERR_CUDA;
-    *out = h;
-    return CR_OK;
-}
-
-// Row-major C[M, N] = alpha op(A) op(B) + beta C, op(A) [M, K], op(B) [K, N]
-// (bf16 operands with fp32 accumulation; fp32 operands would run in TF32);
-// tA: A is stored [K, M] (op(A) = A^T); tB: B is stored [N, K].  In cuBLAS's
-// column-major terms this is C^T = op(B)^T op(A)^T on the same memory.
-cr_status gemm_rm(cublasHandle_t h, bool tA, bool tB, int64_t M, int64_t N, int64_t K, float alpha,
-                  const void* A, cudaDataType_t ta, int64_t lda, const void* B, cudaDataType_t tb, int64_t ldb,
-                  float beta, void* C, cudaDataType_t tc, int64_t ldc, int64_t batch, int64_t sA, int64_t sB,
-                  int64_t sC) {
-    const cublasComputeType_t ct = (ta == CUDA_R_32F) ? CUBLAS_COMPUTE_32F_FAST_TF32 : CUBLAS_COMPUTE_32F;
-    cublasStatus_t e;
-    if (batch <= 1)
-        e = cublasGemmEx(h, tB ? CUBLAS_OP_T : CUBLAS_OP_N, tA ? CUBLAS_OP_T : CUBLAS_OP_N, static_cast<int>(N),
-                         static_cast<int>(M), static_cast<int>(K), &alpha, B, tb, static_cast<int>(ldb), A, ta,
-                         static_cast<int>(lda), &beta, C, tc, static_cast<int>(ldc), ct, CUBLAS_GEMM_DEFAULT);
-    else
-        e = cublasGemmStridedBatchedEx(h, tB ? CUBLAS_OP_T : CUBLAS_OP_N, tA ? CUBLAS_OP_T : CUBLAS_OP_N,
-                                       static_cast<int>(N), static_cast<int>(M), static_cast<int>(K), &alpha, B,
-                                       tb, static_cast<int>(ldb), sB, A, ta, static_cast<int>(lda), sA, &beta, C,
-                                       tc, static_cast<int>(ldc), sC, static_cast<int>(batch), ct,
-                                       CUBLAS_GEMM_DEFAULT);
-    return e == CUBLAS_STATUS_SUCCESS ? CR_OK : CR_ERR_CUDA;
 }
 
 }  // namespace cr

@@ -92,11 +92,13 @@ class RepairSession:
         or keep each request's first chunk stale."""
         if component == "kv" and offset == "stale" and not keep_first_chunk:
             cr.cr_apply_residual(self.target, self.rep, self.weights, self.yf, a.n_tokens, self.kv,
-                                 self.pos, inv_freq_target, rope_mode, stream)
+                                 self.pos, inv_freq_target, rope_mode, workspace=self.workspace,
+                                 stream=stream)
         else:
             cr.cr_apply_residual_select(self.target, self.rep, self.weights, self.yf, a.n_tokens,
                                         self.kv, self.pos, inv_freq_target, rope_mode, component,
-                                        offset, self.chunk_id if keep_first_chunk else None, stream)
+                                        offset, self.chunk_id if keep_first_chunk else None,
+                                        workspace=self.workspace, stream=stream)
 
     def stale_kv(self, a: Assembled, inv_freq_target, stream=None):
         """The stale cache of independent reuse: the assembled canonical cache with K
@@ -109,7 +111,7 @@ class RepairSession:
         ([2 L, num_slots, H_kv d_h] bf16) at slot_mapping[t] (int64, < 0 = skip); kv stays stale."""
         cr.cr_apply_residual_paged(self.target, self.rep, self.weights, self.yf, a.n_tokens, self.kv,
                                    self.pos, slot_mapping, paged_cache, num_slots, inv_freq_target,
-                                   rope_mode, stream)
+                                   rope_mode, workspace=self.workspace, stream=stream)
 
     def repair(self, kv_pool, emb_pool, chunk_start, chunk_len, chunk_idx, cu_chunks,
                inv_freq_target=None, rope_mode=cr.CR_ROPE_NONE, stream=None,

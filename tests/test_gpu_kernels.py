@@ -55,6 +55,40 @@ def test_linear(M, N, K, epi):
         assert_close_bf16(got, ref, 3e-3, f"linear bf16 {M}x{N}x{K}")
 
 
+@pytest.mark.parametrize("M,N,K", [(256, 128, 64), (300, 192, 1000), (1024, 4096, 5120), (16384, 1024, 336),
+                                   (5120, 512, 2048), (128, 64, 8)])
+@pytest.mark.parametrize("a_trans", [False, True])
+@pytest.mark.parametrize("accumulate", [False, True])
+def test_matmul_layouts(M, N, K, a_trans, accumulate):
+    """The backward's products: C (+)= op(A) B with B stored [K, N] and A stored
+    [M, K] or [K, M] (the MN-major operand layouts), against float64 products of
+    the same bf16 values: fp32 accumulation error only.  Ragged K and M (not a
+    multiple of the tile) included."""
+    if a_trans and M % 64:
+        pytest.skip("a transposed A needs whole 64-row blocks")
+    g = np.random.default_rng(M + 3 * N + 7 * K + 2 * a_trans + accumulate)
+    A = _bf16(g, (K, M) if a_trans else (M, K))
+    B = _bf16(g, (K, N), 1.0 / np.sqrt(K))
+    init = g.standard_normal((M, N)).astype(np.float32)
+    C = to_dev(init)
+    cr.cr_matmul(to_dev(A), to_dev(B), C, a_trans=a_trans, accumulate=accumulate)
+    torch.cuda.synchronize()
+    a64 = as_f64(A).T if a_trans else as_f64(A)
+    ref = a64 @ as_f64(B) + (init if accumulate else 0.0)
+    assert_close(to_host(C), ref, 1e-5, 1e-4, f"matmul {M}x{N}x{K} a_trans={a_trans} acc={accumulate}")
+    # with a workspace the poorly filled shapes run as k-parts summed in order: the
+    # same products to fp32 rounding, and the same bits on a rerun
+    ws = torch.empty(8 * M * N * 4, dtype=torch.uint8, device="cuda")
+    outs = []
+    for _ in range(2):
+        C2 = to_dev(init)
+        cr.cr_matmul(to_dev(A), to_dev(B), C2, a_trans=a_trans, accumulate=accumulate, workspace=ws)
+        torch.cuda.synchronize()
+        outs.append(to_host(C2))
+    assert_close(outs[0], ref, 1e-5, 1e-4, f"split matmul {M}x{N}x{K} a_trans={a_trans} acc={accumulate}")
+    assert np.array_equal(outs[0], outs[1])
+
+
 def test_gelu_epilogue_tails():
     """GELU of the GEMM epilogue over [-12, 12]: every row's output equals x, so
     the epilogue sees each bf16 value of the range; compared with the fp64

@@ -72,7 +72,8 @@ def test_paged_write_equals_in_place_repair(rope_mode):
 
     # reference: the in-place repair of a copy of the same stale rows
     ref = stale.clone()
-    cr.cr_apply_residual(sess.target, sess.rep, sess.weights, sess.yf, n, ref, sess.pos, inv, rope_mode)
+    cr.cr_apply_residual(sess.target, sess.rep, sess.weights, sess.yf, n, ref, sess.pos, inv, rope_mode,
+                         workspace=sess.workspace)
     torch.cuda.synchronize()
     assert torch.equal(sess.kv[:n], stale), "the stale cache must stay untouched"
     got = to_host(paged).reshape(planes, num_slots, plane)
@@ -145,3 +146,32 @@ def test_paged_write_matches_oracle(rope_mode):
         worst = max(worst, err)
         assert err <= 2e-2 and cos >= 0.999, f"plane {pl}: max err {err:.3e} x RMS, cosine {cos:.6f}"
     print(f"paged write vs oracle (rope={rope}): worst max err {worst:.3e} x RMS")
+
+
+@pytest.mark.parametrize("name", ["small", "tiny"])
+def test_target_rope_angles_from_table_equal_inline(name):
+    """Under R_M the head reads each row's (cos, sin) from the per-call table written
+    into the workspace; without a workspace it evaluates them in the epilogue.  Both
+    evaluate the same formula (the angle's product error folded back in), compiled
+    in different places, so they may differ in the last bit of an angle: the two
+    repaired caches agree to one bf16 rounding (almost all values equal) or, for an
+    fp32 cache, to 2^-20 of its RMS."""
+    case, sess, a = _prepared(name)
+    n = a.n_tokens
+    stale = sess.kv[:n].clone()
+    outs = []
+    for ws in (sess.workspace, None):
+        kv = stale.clone()
+        cr.cr_apply_residual(sess.target, sess.rep, sess.weights, sess.yf, n, kv, sess.pos,
+                             case.inv_freq_target, cr.CR_ROPE_GLOBAL, workspace=ws)
+        torch.cuda.synchronize()
+        outs.append(to_host(kv))
+    dt = case.target.cache_dtype
+    x, y = as_f64(outs[0]), as_f64(outs[1])
+    if dt == "bf16":   # one rounding of the cache dtype
+        bound = 2.0 * half_ulp(np.maximum(np.abs(x), np.abs(y)), dt)
+    else:              # an angle's last bit moves a rotated pair by ~2^-23 of its size
+        bound = 2.0 ** -20 * np.sqrt(np.mean(x ** 2))
+    assert np.all(np.abs(x - y) <= bound), float(np.abs(x - y).max())
+    if dt == "bf16":   # the coarse rounding absorbs almost every such difference
+        assert np.mean(x != y) < 1e-2

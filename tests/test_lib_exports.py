@@ -106,11 +106,17 @@ def test_other_calls_reject_bad_inputs_on_host(L):
     assert L.cr_compress_features(ctypes.byref(t), ctypes.byref(r), ctypes.byref(w), FAKE, FAKE,
                                   10, FAKE, FAKE, FAKE, 1 << 30, None) == cr.CR_ERR_INVALID_ARG
     assert L.cr_apply_residual(ctypes.byref(t), ctypes.byref(r), ctypes.byref(w), FAKE, 10, FAKE,
-                               FAKE, None, 1, None) == cr.CR_ERR_INVALID_ARG
+                               FAKE, None, 1, None, 0, None) == cr.CR_ERR_INVALID_ARG
     assert L.cr_linear(FAKE, 64, FAKE, None, 10, 30, 64, FAKE, 30, 0, None) == cr.CR_ERR_INVALID_ARG
     assert L.cr_linear(FAKE, 64, FAKE, None, 10, 32, 60, FAKE, 32, 0, None) == cr.CR_ERR_INVALID_ARG
     assert L.cr_layernorm(FAKE, None, 0, None, FAKE, FAKE, 1e-5, 4, 100, FAKE, None) == \
         cr.CR_ERR_INVALID_ARG
+    # cr_matmul: sizes, strides and alignment on the host; widths in 64-column blocks
+    assert L.cr_matmul(FAKE, 64, 0, FAKE, 64, 0, 64, 64, FAKE, 64, 0, None, 0, None) == cr.CR_ERR_INVALID_ARG
+    assert L.cr_matmul(FAKE, 60, 0, FAKE, 64, 10, 64, 60, FAKE, 64, 0, None, 0, None) == cr.CR_ERR_INVALID_ARG
+    assert L.cr_matmul(FAKE + 8, 64, 0, FAKE, 64, 10, 64, 64, FAKE, 64, 0, None, 0, None) == cr.CR_ERR_INVALID_ARG
+    assert L.cr_matmul(FAKE, 64, 0, FAKE, 96, 10, 96, 64, FAKE, 96, 0, None, 0, None) == cr.CR_ERR_UNSUPPORTED
+    assert L.cr_matmul(FAKE, 96, 1, FAKE, 64, 96, 64, 64, FAKE, 64, 0, None, 0, None) == cr.CR_ERR_UNSUPPORTED
     cu = np.array([0, 100], np.int32)
     assert L.cr_chunk_causal_attention(FAKE, 1024, 8, FAKE, cu.ctypes.data, 1, 100, FAKE,
                                        None) == cr.CR_ERR_UNSUPPORTED          # 128-dim heads
@@ -147,7 +153,7 @@ def test_output_choice_calls_reject_bad_inputs_on_host(L):
     w.w_out = w.b_out = w.sigma_delta = FAKE
     sel = lambda tt, comp=3, off=0, keep=None, rope=0, freq=None: L.cr_apply_residual_select(
         ctypes.byref(tt), ctypes.byref(r), ctypes.byref(w), FAKE, 10, FAKE, FAKE, freq, rope, comp,
-        off, keep, None)
+        off, keep, None, 0, None)
     for comp in (0, 4, -1):
         assert sel(t, comp=comp) == cr.CR_ERR_INVALID_ARG
     assert sel(t, off=2) == cr.CR_ERR_INVALID_ARG
@@ -167,7 +173,7 @@ def test_paged_residual_rejects_bad_inputs_on_host(L):
     w.w_out = w.b_out = w.sigma_delta = FAKE
     call = lambda tt, n=10, slots=64, paged=FAKE: L.cr_apply_residual_paged(
         ctypes.byref(tt), ctypes.byref(r), ctypes.byref(w), FAKE, n, FAKE, FAKE, None, 0, FAKE, paged,
-        slots, None)
+        slots, None, 0, None)
     assert call(t, slots=0) == cr.CR_ERR_INVALID_ARG          # no slots
     assert call(t, n=0) == cr.CR_ERR_INVALID_ARG              # no tokens
     assert call(t, paged=FAKE + 8) == cr.CR_ERR_INVALID_ARG   # misaligned cache
