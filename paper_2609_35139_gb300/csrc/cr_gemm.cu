@@ -238,6 +238,23 @@ __device__ __forceinline__ void vec16(const float* v, int col, float* out) {
 // First output column of tile t.  Tiles are walked W-tile-major (t / num_m is
 // the column tile); under an output choice (KV epilogues with col_block > 0)
 // only the K or only the V column blocks are walked.
+// Tile walk of a launch: t -> (linear tile, k-part).  The linear tile c num_m + m
+// names row tile m of column tile c.  Default order: k-parts fastest, then row
+// tiles, then column tiles (W-tile-major: the CTAs running together share a W
+// tile, and the activations stay in L2).  n_fast: column tiles fastest, then
+// row tiles, k-parts slowest, for an A operand much larger than L2: the tiles
+// running together share their A rows and one k-range of W, so A is read once.
+__device__ __forceinline__ int tile_lin(const GemmParams& p, int t) {
+    if (p.n_fast) {
+        const int r = t % (p.num_m * p.num_n);
+        return (r % p.num_n) * p.num_m + r / p.num_n;
+    }
+    return t / p.split_k;
+}
+__device__ __forceinline__ int tile_part(const GemmParams& p, int t) {
+    return p.n_fast ? t / (p.num_m * p.num_n) : t % p.split_k;
+}
+
 template <int BN, bool KV>
 __device__ __forceinline__ int tile_n0(const GemmParams& p, int t) {
     const int c = t / p.num_m;
@@ -368,7 +385,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const int num_k = p.split_kb > 0 ? 2 * p.split_kb : (p.K + BK - 1) / BK;
     const int k_per = (num_k + p.split_k - 1) / p.split_k;
     auto k_range = [&](int t, int* kb0, int* kb1) {
-        *kb0 = (t % p.split_k) * k_per;
+        *kb0 = tile_part(p, t) * k_per;
         *kb1 = min(num_k, *kb0 + k_per);
     };
     const bool has_bias = p.bias != nullptr;
@@ -394,8 +411,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         uint32_t stage = 0, phase = 0;
         bool ok = true;
         for (int t = cta0; t < total && ok; t += ncta) {
-            const int m0 = ((t / p.split_k) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-            const int n0 = tile_n0<BN, Cfg::kKV>(p, t / p.split_k);
+            const int m0 = (tile_lin(p, t) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
+            const int n0 = tile_n0<BN, Cfg::kKV>(p, tile_lin(p, t));
             int kbeg, kend;
             k_range(t, &kbeg, &kend);
             for (int kb = kbeg; kb < kend; ++kb) {
@@ -405,7 +422,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     // W columns of this tile: its own column block, or (grouped
                     // rows) the block that belongs to its rows' group
                     const int nw = p.bgroup_rows > 0
-                                       ? (((t / p.split_k) % p.num_m) * (BM * CG) / p.bgroup_rows) * BN : n0;
+                                       ? ((tile_lin(p, t) % p.num_m) * (BM * CG) / p.bgroup_rows) * BN : n0;
                     const int nb0 = nw + static_cast<int>(rank) * (BN / CG);
                     const bool lo = p.split_kb > 0 && kb >= p.split_kb;
                     const CUtensorMap* ma = lo ? &p.tm_alo : &tmA;
@@ -460,8 +477,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             bool ok = true;
             int i = 0;
             for (int t = cta0; t < total && ok; t += ncta, ++i) {
-                const int m0 = ((t / p.split_k) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-                const int n0 = tile_n0<BN, Cfg::kKV>(p, t / p.split_k);
+                const int m0 = (tile_lin(p, t) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
+                const int n0 = tile_n0<BN, Cfg::kKV>(p, tile_lin(p, t));
                 const int nb = min(BN, p.N - n0);
                 const uint32_t vbytes = static_cast<uint32_t>(nb) * 4u;
                 if constexpr (Cfg::kInPlace) {
@@ -519,8 +536,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         uint32_t pk = 0;               // in-place tiles so far
         uint32_t pkg[2] = {0u, 0u};    // boxes of each epilogue group so far
         for (int t = cta0; t < total && ok; t += ncta) {
-            const int m0 = ((t / p.split_k) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-            const int n0 = tile_n0<BN, Cfg::kKV>(p, t / p.split_k);
+            const int m0 = (tile_lin(p, t) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
+            const int n0 = tile_n0<BN, Cfg::kKV>(p, tile_lin(p, t));
             const bool rows_in = m0 < p.M;   // a pair tile's second half may lie below M
             if constexpr (Cfg::kInPlace) {
                 // each box as soon as the epilogue has written it; once TMA has read
@@ -548,7 +565,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     if (leader) {
                         if (rows_in)
                             tma_store_2d(&tmC, tile + b * 16384, n0 + k * Cfg::kBoxCols,
-                                         m0 + (t % p.split_k) * p.M);
+                                         m0 + tile_part(p, t) * p.M);
                         tma_store_commit();
                         tma_store_wait_read0();
                         mbar_arrive(&st_free[b]);
@@ -648,8 +665,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         bool ok = true;
         int i = 0;
         for (int t = cta0; t < total && ok; t += ncta, ++i) {
-            const int m0 = ((t / p.split_k) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-            const int n0 = tile_n0<BN, Cfg::kKV>(p, t / p.split_k);
+            const int m0 = (tile_lin(p, t) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
+            const int n0 = tile_n0<BN, Cfg::kKV>(p, tile_lin(p, t));
             // QKV: the rotation angles depend on (row, pair index) only: cos/sin
             // for every head of the tile, fetched while the MMAs still run
             constexpr int NP = (EPI == EPI_QKV_ROPE) ? 32 : 1;
@@ -1067,6 +1084,7 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
     p.num_m = static_cast<int32_t>((M + BM * kCG - 1) / (BM * kCG));
     p.num_n = static_cast<int32_t>((N + BN - 1) / BN);
     p.split_k = 1;
+    p.n_fast = 0;
     if (kv && p.col_block > 0) {
         // output choice: half of the column blocks, each a whole number of tiles
         if (p.col_block % BN != 0 || N % (2 * static_cast<int64_t>(p.col_block)) != 0)
@@ -1200,21 +1218,23 @@ cr_status launch_gemm_lay(const uint16_t* A, int64_t lda, int lay, const uint16_
     // Split-K: when the tiles fill the CTA pairs poorly (the last round partly
     // empty), cut each tile's k-loop into s parts, each written to its own fp32
     // slice of the scratch and summed in a fixed order by a second kernel.  s
-    // minimises rounds(s) / s x tile time + the sum's traffic, with every part
-    // at least four k-blocks.
+    // minimises rounds(s) x (tile time / s + a fixed cost per round for the
+    // pipeline's fill and the epilogue's drain) + the sum's traffic, with every
+    // part at least four k-blocks.
     const int64_t pairs = num_sms() / kCG > 0 ? num_sms() / kCG : 1;
     const int64_t tiles = static_cast<int64_t>(p.num_m) * p.num_n;
     const int64_t nkb = (K + BK - 1) / BK;
     // (whole 128-row boxes only: a part's rows must not spill into the next slice)
     if (scratch && p.bgroup_rows == 0 && M % BM == 0) {
         const double tile_us = static_cast<double>(nkb) * (256 + BN) / 1.9e3;   // ~1.9 GHz
-        double best = static_cast<double>((tiles + pairs - 1) / pairs) * tile_us;
+        const double round_us = 6.0;
+        double best = static_cast<double>((tiles + pairs - 1) / pairs) * (tile_us + round_us);
         for (int sk = 2; sk <= 8; sk *= 2) {
             const int64_t kp = (nkb + sk - 1) / sk;
             if (kp < 4 || (sk - 1) * kp >= nkb) break;
             const size_t need = static_cast<size_t>(sk) * M * N * 4;
             if (need > scratch_bytes) break;
-            const double t = static_cast<double>((tiles * sk + pairs - 1) / pairs) * tile_us / sk +
+            const double t = static_cast<double>((tiles * sk + pairs - 1) / pairs) * (tile_us / sk + round_us) +
                              static_cast<double>(need + static_cast<size_t>(M) * N * 4 * (epi == EPI_ADD_F32 ? 2 : 1)) /
                                  6.0e6;   // bytes at ~6 TB/s, in microseconds
             if (t < best * 0.95) {
@@ -1223,6 +1243,8 @@ cr_status launch_gemm_lay(const uint16_t* A, int64_t lda, int lay, const uint16_
             }
         }
     }
+    // an A operand far larger than L2 is walked once: column tiles fastest
+    p.n_fast = (p.bgroup_rows == 0 && p.num_n > 1 && static_cast<double>(M) * K * 2 > 64e6) ? 1 : 0;
     float* const C = static_cast<float*>(p.out);
     const int64_t ldc = p.ldo;
     if (p.split_k > 1) {

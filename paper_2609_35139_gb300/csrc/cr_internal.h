@@ -107,6 +107,9 @@ struct GemmParams {
     // split-K (launch_gemm_lay): parts per tile, each writing rows [u M, (u + 1) M)
     // of the output (1 = off; every launcher sets it)
     int32_t split_k;
+    // tile order: 0 = W-tile-major (row tiles fastest), 1 = column tiles fastest
+    // (k-parts slowest), for an A operand far larger than L2
+    int32_t n_fast;
     // grouped rows (launch_gemm_lay): every bgroup_rows rows of A form a group whose
     // tile reads W columns [g BN, (g + 1) BN) of the W matrix, g = row / bgroup_rows,
     // and writes output columns [0, BN); 0 = off
