@@ -1220,7 +1220,9 @@ cr_status launch_gemm_lay(const uint16_t* A, int64_t lda, int lay, const uint16_
     // slice of the scratch and summed in a fixed order by a second kernel.  s
     // minimises rounds(s) x (tile time / s + a fixed cost per round for the
     // pipeline's fill and the epilogue's drain) + the sum's traffic, with every
-    // part at least four k-blocks.
+    // part at least 64 k-blocks (measured on the training step's shapes: shorter
+    // parts lose more to their fill, drain and sum than the idle CTA pairs cost;
+    // the head's dX product, K = 65536, gains 30 % from 8 parts).
     const int64_t pairs = num_sms() / kCG > 0 ? num_sms() / kCG : 1;
     const int64_t tiles = static_cast<int64_t>(p.num_m) * p.num_n;
     const int64_t nkb = (K + BK - 1) / BK;
@@ -1231,7 +1233,7 @@ cr_status launch_gemm_lay(const uint16_t* A, int64_t lda, int lay, const uint16_
         double best = static_cast<double>((tiles + pairs - 1) / pairs) * (tile_us + round_us);
         for (int sk = 2; sk <= 8; sk *= 2) {
             const int64_t kp = (nkb + sk - 1) / sk;
-            if (kp < 4 || (sk - 1) * kp >= nkb) break;
+            if (kp < 64 || (sk - 1) * kp >= nkb) break;
             const size_t need = static_cast<size_t>(sk) * M * N * 4;
             if (need > scratch_bytes) break;
             const double t = static_cast<double>((tiles * sk + pairs - 1) / pairs) * (tile_us / sk + round_us) +

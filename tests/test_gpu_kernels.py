@@ -56,7 +56,7 @@ def test_linear(M, N, K, epi):
 
 
 @pytest.mark.parametrize("M,N,K", [(256, 128, 64), (300, 192, 1000), (1024, 4096, 5120), (16384, 1024, 336),
-                                   (5120, 512, 2048), (128, 64, 8)])
+                                   (5120, 512, 2048), (128, 64, 8), (256, 128, 16384)])
 @pytest.mark.parametrize("a_trans", [False, True])
 @pytest.mark.parametrize("accumulate", [False, True])
 def test_matmul_layouts(M, N, K, a_trans, accumulate):
@@ -75,9 +75,14 @@ def test_matmul_layouts(M, N, K, a_trans, accumulate):
     torch.cuda.synchronize()
     a64 = as_f64(A).T if a_trans else as_f64(A)
     ref = a64 @ as_f64(B) + (init if accumulate else 0.0)
-    assert_close(to_host(C), ref, 1e-5, 1e-4, f"matmul {M}x{N}x{K} a_trans={a_trans} acc={accumulate}")
-    # with a workspace the poorly filled shapes run as k-parts summed in order: the
-    # same products to fp32 rounding, and the same bits on a rerun
+    # fp32 accumulation: the error grows with the k-loop (measured 1.9e-5 relative RMS
+    # at K = 16384); 1.5x that growth beyond K = 8192
+    g = max(1.0, 1.5 * K / 8192)
+    tol = (1e-5 * g, 1e-4 * g)
+    assert_close(to_host(C), ref, *tol, f"matmul {M}x{N}x{K} a_trans={a_trans} acc={accumulate}")
+    # with a workspace the poorly filled shapes with long k-loops (the last one here)
+    # run as k-parts summed in order: the same products to fp32 rounding, and the
+    # same bits on a rerun
     ws = torch.empty(8 * M * N * 4, dtype=torch.uint8, device="cuda")
     outs = []
     for _ in range(2):
@@ -85,7 +90,7 @@ def test_matmul_layouts(M, N, K, a_trans, accumulate):
         cr.cr_matmul(to_dev(A), to_dev(B), C2, a_trans=a_trans, accumulate=accumulate, workspace=ws)
         torch.cuda.synchronize()
         outs.append(to_host(C2))
-    assert_close(outs[0], ref, 1e-5, 1e-4, f"split matmul {M}x{N}x{K} a_trans={a_trans} acc={accumulate}")
+    assert_close(outs[0], ref, *tol, f"split matmul {M}x{N}x{K} a_trans={a_trans} acc={accumulate}")
     assert np.array_equal(outs[0], outs[1])
 
 
