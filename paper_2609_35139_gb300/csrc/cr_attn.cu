@@ -65,11 +65,12 @@ struct AttnCfg {
 // softmax groups.
 // At launch each thread gets 65536 / 384 = 168 registers (the host checks
 // this); the control warpgroup gives up most of its share so that the softmax
-// threads can hold a whole S row: 72 * 128 + 2 * 216 * 128 = 168 * 384.
+// threads can hold a whole S row: 48 * 128 + 2 * 224 * 128 <= 168 * 384 (the
+// control warps keep only descriptors, counters and phases).
 constexpr int kThreads = 384;
 constexpr uint32_t kRegsLaunch = 168;
-constexpr uint32_t kRegsCtl = 72;
-constexpr uint32_t kRegsSoftmax = 216;
+constexpr uint32_t kRegsCtl = 48;
+constexpr uint32_t kRegsSoftmax = 224;
 static_assert(kRegsCtl * 128 + 2 * kRegsSoftmax * 128 <= kRegsLaunch * kThreads,
               "register split exceeds the launch allocation");
 constexpr float kRescaleLog2 = 8.0f;   // lazy-rescale threshold (log2 units)
