@@ -11,17 +11,18 @@
 //               double-buffered fp32 accumulator and multicasts its commits.
 //   warp 2      epilogue-input loader: per tile, the bias (and sigma_delta)
 //               slice by bulk copy and, for in-place epilogues, the output tile
-//               itself (the stale cache tile, the fp32 residual-stream tile, or
-//               for the training loss head the stale and joint cache tiles) by
-//               TMA, as soon as the epilogue has released its slot.
-//   warp 3      TMA store issuer for the staged output.
+//               itself (the stale cache tile, or for the training loss head the
+//               stale and joint cache tiles) by TMA, as soon as the epilogue has
+//               released its slot.
+//   warp 3      TMA store issuer for the staged output (for the fp32 residual
+//               stream a TMA reduce-add: x += acc + b in L2).
 //   warps 4..11 epilogue, two groups of four warps (one per TMEM lane
 //               quarter) splitting each tile's columns: tcgen05.ld 32 lanes x
 //               16 columns, bias from shared memory, then one of: bf16, GELU,
 //               fp32, RoPE on Q/K (into 128B-swizzled staging buffers, one box
 //               of 128 B-wide columns at a time, double-buffered per group), or
-//               in place on the staged tile: residual stream x += acc + b,
-//               cache kv = kv + sigma_delta (acc + b) (+ R_M on K).  Staged
+//               in place on the staged tile: cache kv = kv + sigma_delta
+//               (acc + b) (+ R_M on K).  Staged
 //               data goes out with TMA stores (coalesced, asynchronous).  The
 //               paged head and the loss head write from registers instead: the
 //               repaired rows into the paged target cache, or the training
@@ -63,7 +64,11 @@ struct GemmCfg {
     // of r^2, from registers (no TMA store)
     static constexpr bool kLoss = (EPI == EPI_KV_LOSS);
     static constexpr bool kDirect = kPaged || kLoss;
-    static constexpr bool kInPlace = kKV || EPI == EPI_ADD_F32;   // tile loaded, updated, stored
+    static constexpr bool kInPlace = kKV;   // tile loaded, updated, stored
+    // the fp32 residual add goes out as a TMA reduce-add of the staged box
+    // (x += acc + bias in L2, one add per element: the same rounding as a
+    // load, add and store, without staging the old tile)
+    static constexpr bool kReduce = (EPI == EPI_ADD_F32);
     static constexpr int kTileEsize = (EPI == EPI_KV_F32 || EPI == EPI_ADD_F32 || EPI == EPI_F32) ? 4 : 2;
     static constexpr int kBoxCols = 128 / kTileEsize;          // one 128-byte swizzle row
     // in-place epilogues stage the whole [BM x BN] tile; store-only epilogues
@@ -85,8 +90,8 @@ struct GemmCfg {
     static constexpr uint32_t kStageBytes = A_BYTES + kBBytes;
     static constexpr uint32_t kFixed = 1024 + kTileBytes + kVecBufs * kVecBytes + 512;
     static constexpr int kStagesFit = static_cast<int>((kSmemLimit - kFixed) / kStageBytes);
-    static constexpr int kStages = kStagesFit > 6 ? 6 : kStagesFit;
-    static_assert(kStages >= 3, "GEMM tile does not fit in shared memory");
+    static constexpr int kStages = kStagesFit > 8 ? 8 : kStagesFit;
+    static_assert(kStages >= 4, "GEMM tile does not fit in shared memory");
     static constexpr uint32_t kSmemBytes = kFixed + kStages * kStageBytes;
     // double-buffered accumulator; TMEM is allocated in powers of two
     static constexpr uint32_t kTmemCols = (2 * BN <= 256) ? 256u : 512u;
@@ -427,19 +432,20 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     const bool lo = p.split_kb > 0 && kb >= p.split_kb;
                     const CUtensorMap* ma = lo ? &p.tm_alo : &tmA;
                     const int ka = (lo ? kb - p.split_kb : kb) * BK;   // A and W column
+                    uint64_t* fq = &full[stage];
                     auto load = [&](uint8_t* dst, const CUtensorMap* m, int x, int y, uint32_t fb) {
                         if constexpr (CG == 1)
-                            tma_load_2d(dst, m, &full[stage], x, y);
+                            tma_load_2d(dst, m, fq, x, y);
                         else
                             tma_load_2d_pair(dst, m, fb, x, y);
                     };
                     // both CTAs' copies count on the even CTA's barrier, which
                     // expects the pair's bytes (its own arrive is the only one)
-                    const uint32_t fb = CG == 2 ? mapa_shared(smem_u32(&full[stage]), 0) : 0u;
+                    const uint32_t fb = CG == 2 ? mapa_shared(smem_u32(fq), 0) : 0u;
                     if (CG == 1)
-                        mbar_expect_tx(&full[stage], Cfg::kStageBytes);
+                        mbar_expect_tx(fq, Cfg::kStageBytes);
                     else if (rank == 0)
-                        mbar_expect_tx(&full[stage], CG * Cfg::kStageBytes);
+                        mbar_expect_tx(fq, CG * Cfg::kStageBytes);
                     if constexpr (kAMN) {
                         load(sa, ma, m0, ka, fb);
                         load(sa + A_BYTES / 2, ma, m0 + 64, ka, fb);
@@ -556,6 +562,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 }
                 ++pk;
             } else {
+                // one box store stays in flight: a buffer goes back to its group
+                // once the next box's store is issued and the older one has
+                // read it; by the end of the tile every store has read its box
+                int prev = -1;
                 for (int k = 0; k < Cfg::kBoxes; ++k) {
                     // box k was staged by epilogue group k & 1 in its buffer pkg & 1
                     constexpr uint32_t GB = Cfg::kGroupBufs;
@@ -563,16 +573,26 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     const uint32_t b = static_cast<uint32_t>(g) * GB + (pkg[g] % GB);
                     if (!(ok = mbar_wait_warp(&epi_done[b], (pkg[g] / GB) & 1u, wc, 402))) break;
                     if (leader) {
-                        if (rows_in)
-                            tma_store_2d(&tmC, tile + b * 16384, n0 + k * Cfg::kBoxCols,
-                                         m0 + tile_part(p, t) * p.M);
+                        if (rows_in) {
+                            const int x = n0 + k * Cfg::kBoxCols, y = m0 + tile_part(p, t) * p.M;
+                            if constexpr (Cfg::kReduce)
+                                tma_reduce_add_2d(&tmC, tile + b * 16384, x, y);
+                            else
+                                tma_store_2d(&tmC, tile + b * 16384, x, y);
+                        }
                         tma_store_commit();
-                        tma_store_wait_read0();
-                        mbar_arrive(&st_free[b]);
+                        tma_store_wait_read<1>();
+                        if (prev >= 0) mbar_arrive(&st_free[prev]);
                     }
                     __syncwarp();
+                    prev = static_cast<int>(b);
                     ++pkg[g];
                 }
+                if (leader) {
+                    tma_store_wait_read0();
+                    if (ok && prev >= 0) mbar_arrive(&st_free[prev]);
+                }
+                __syncwarp();
                 if (ok && epi_load && leader) mbar_arrive(epi_empty);
                 __syncwarp();
             }
@@ -854,16 +874,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                             for (int q = 0; q < 16; ++q) bv[q] = 0.0f;
                         }
                         tmem_wait_ld();
-                        if constexpr (Cfg::kKV) {
-                            if (!keep) {
-                                float sv[16];
-                                vec16(vst, c, sv);
+                        if (!keep) {
+                            float sv[16];
+                            vec16(vst, c, sv);
 #pragma unroll
-                                for (int q = 0; q < 16; ++q) k[q] = fmaf(sv[q], a[q] + bv[q], k[q]);
-                            }
-                        } else {
-#pragma unroll
-                            for (int q = 0; q < 16; ++q) k[q] += a[q] + bv[q];
+                            for (int q = 0; q < 16; ++q) k[q] = fmaf(sv[q], a[q] + bv[q], k[q]);
                         }
                         put16(c, k);
                       }
@@ -1198,7 +1213,7 @@ cr_status launch_gemm_lay(const uint16_t* A, int64_t lda, int lay, const uint16_
     if (M < 1 || N < 1 || K < 1 || (N % 64) != 0 || (lay == LAY_MM && (M % 64) != 0))
         return CR_ERR_UNSUPPORTED;
     // Tile width as in launch_gemm (rounds x (256 + BN)); an MN-major W half is
-    // whole 64-column boxes, so 256 or 128 (the in-place fp32 tile: 128).
+    // whole 64-column boxes, so 256 or 128 (the accumulating form: 128).
     int BN = 128;
     if (epi == EPI_F32 && p.bgroup_rows == 0) {
         const int64_t pairs = num_sms() / kCG > 0 ? num_sms() / kCG : 1;

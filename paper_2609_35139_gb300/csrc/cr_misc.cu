@@ -120,9 +120,14 @@ __global__ void __launch_bounds__(256) gather_emb_kernel(const __grid_constant__
 }
 
 
-// One warp per row, VPL float4 per lane (D = 128 * VPL); two-pass statistics
-// from registers (mean, then mean squared deviation: biased variance).
-template <int VPL>
+// A row of D = 128 VPL values is held by WPR warps (WPR = 2 when VPL is even):
+// each lane keeps VPL / WPR float4 of it in registers, so that a CTA of 256
+// threads keeps 8 / WPR rows in flight with few registers per thread (many
+// resident warps hide the memory latency).  Two-pass statistics from the
+// registers (mean, then mean squared deviation: biased variance); the WPR
+// warps of a row exchange their partial sums through shared memory.  gamma and
+// beta are read after the statistics (they stay in L1).
+template <int VPL, int WPR>
 __global__ void __launch_bounds__(256) layernorm_kernel(const float* x,
                                                         const float* __restrict__ add,
                                                         int64_t ld_add, float* x_out,
@@ -130,63 +135,75 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const float* x,
                                                         const float* __restrict__ b, float eps,
                                                         int64_t M, uint16_t* __restrict__ u) {
     constexpr int D = VPL * 128;
+    constexpr int HV = VPL / WPR;            // float4 per lane
+    constexpr int RPB = 8 / WPR;             // rows per CTA
+    static_assert(VPL % WPR == 0, "a row splits into whole float4 columns per warp");
+    __shared__ float red[2][8];
     pdl_launch_dependents();
     pdl_wait();
-    const int64_t row = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    const int warp = static_cast<int>(threadIdx.x >> 5);
+    const int part = warp % WPR;             // this warp's part of the row
+    const int64_t row = static_cast<int64_t>(blockIdx.x) * RPB + warp / WPR;
     const int lane = threadIdx.x & 31;
-    if (row >= M) return;
-    // every load of the row (x, the reinjection term, gamma, beta) is issued
-    // before the first use: one memory round trip per row
-    float4 v[VPL], gg[VPL], bq[VPL], av[VPL];
-    const float4* xr = reinterpret_cast<const float4*>(x + row * D);
-    const float4* g4 = reinterpret_cast<const float4*>(g);
-    const float4* b4 = reinterpret_cast<const float4*>(b);
+    const bool live = row < M;
+    const int64_t rr = live ? row : 0;       // rows past M read row 0 and write nothing
+    const int c0 = part * (D / 4 / WPR);     // first float4 of this part
+    float4 v[HV];
+    const float4* xr = reinterpret_cast<const float4*>(x + rr * D) + c0;
 #pragma unroll
-    for (int k = 0; k < VPL; ++k) v[k] = xr[lane + 32 * k];
+    for (int k = 0; k < HV; ++k) v[k] = xr[lane + 32 * k];
     if (add) {
-        const float4* ar = reinterpret_cast<const float4*>(add + row * ld_add);
+        float4 av[HV];
+        const float4* ar = reinterpret_cast<const float4*>(add + rr * ld_add) + c0;
 #pragma unroll
-        for (int k = 0; k < VPL; ++k) av[k] = ar[lane + 32 * k];
-    }
+        for (int k = 0; k < HV; ++k) av[k] = ar[lane + 32 * k];
+        float4* xo = reinterpret_cast<float4*>(x_out + rr * D) + c0;
 #pragma unroll
-    for (int k = 0; k < VPL; ++k) {
-        gg[k] = __ldg(g4 + lane + 32 * k);
-        bq[k] = __ldg(b4 + lane + 32 * k);
-    }
-    if (add) {
-        float4* xo = reinterpret_cast<float4*>(x_out + row * D);
-#pragma unroll
-        for (int k = 0; k < VPL; ++k) {
+        for (int k = 0; k < HV; ++k) {
             v[k].x += av[k].x;
             v[k].y += av[k].y;
             v[k].z += av[k].z;
             v[k].w += av[k].w;
-            xo[lane + 32 * k] = v[k];
+            if (live) xo[lane + 32 * k] = v[k];
         }
     }
+    // the row's sum over its WPR warps (the same order in every warp of the row)
+    auto row_sum = [&](float s, int slot) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        if constexpr (WPR == 1) {
+            return s;
+        } else {
+            if (lane == 0) red[slot][warp] = s;
+            __syncthreads();
+            const int w0 = warp - part;
+            float t = red[slot][w0];
+#pragma unroll
+            for (int q = 1; q < WPR; ++q) t += red[slot][w0 + q];
+            return t;
+        }
+    };
     float s = 0.f;
 #pragma unroll
-    for (int k = 0; k < VPL; ++k) s += (v[k].x + v[k].y) + (v[k].z + v[k].w);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    const float mean = s * (1.0f / D);
+    for (int k = 0; k < HV; ++k) s += (v[k].x + v[k].y) + (v[k].z + v[k].w);
+    const float mean = row_sum(s, 0) * (1.0f / D);
     float q = 0.f;
 #pragma unroll
-    for (int k = 0; k < VPL; ++k) {
+    for (int k = 0; k < HV; ++k) {
         const float a = v[k].x - mean, bb = v[k].y - mean, c = v[k].z - mean, d = v[k].w - mean;
         q += (a * a + bb * bb) + (c * c + d * d);
     }
+    const float rstd = rsqrtf(row_sum(q, 1) * (1.0f / D) + eps);
+    if (!live) return;
+    const float4* g4 = reinterpret_cast<const float4*>(g) + c0;
+    const float4* b4 = reinterpret_cast<const float4*>(b) + c0;
+    uint2* ur = reinterpret_cast<uint2*>(u + row * D) + c0;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
-    const float rstd = rsqrtf(q * (1.0f / D) + eps);
-    uint2* ur = reinterpret_cast<uint2*>(u + row * D);
-#pragma unroll
-    for (int k = 0; k < VPL; ++k) {
+    for (int k = 0; k < HV; ++k) {
+        const float4 gg = __ldg(g4 + lane + 32 * k), bq = __ldg(b4 + lane + 32 * k);
         uint2 w;
-        w.x = pack_bf16x2((v[k].x - mean) * rstd * gg[k].x + bq[k].x,
-                          (v[k].y - mean) * rstd * gg[k].y + bq[k].y);
-        w.y = pack_bf16x2((v[k].z - mean) * rstd * gg[k].z + bq[k].z,
-                          (v[k].w - mean) * rstd * gg[k].w + bq[k].w);
+        w.x = pack_bf16x2((v[k].x - mean) * rstd * gg.x + bq.x, (v[k].y - mean) * rstd * gg.y + bq.y);
+        w.y = pack_bf16x2((v[k].z - mean) * rstd * gg.z + bq.z, (v[k].w - mean) * rstd * gg.w + bq.w);
         ur[lane + 32 * k] = w;
     }
 }
@@ -277,13 +294,14 @@ cr_status launch_layernorm(const float* x, const float* add, int64_t ld_add, flo
                            const float* g, const float* b, float eps, int64_t M, int64_t D,
                            uint16_t* u, cudaStream_t st) {
     if (M <= 0) return CR_OK;
-    const int rows_per_block = 8;
-    const int grid = static_cast<int>((M + rows_per_block - 1) / rows_per_block);
     switch (D) {
-#define CR_LN_CASE(V)                                                                       \
-    case V * 128:                                                                           \
-        return launch_pdl(layernorm_kernel<V>, dim3(grid), dim3(256), 0, st, x, add, ld_add, \
-                          x_out, g, b, eps, M, u);
+#define CR_LN_CASE(V)                                                                          \
+    case V * 128: {                                                                            \
+        constexpr int W = (V % 2 == 0) ? 2 : 1;                                                \
+        const int grid = static_cast<int>((M + 8 / W - 1) / (8 / W));                          \
+        return launch_pdl(layernorm_kernel<V, W>, dim3(grid), dim3(256), 0, st, x, add, ld_add, \
+                          x_out, g, b, eps, M, u);                                             \
+    }
         CR_LN_CASE(1)
         CR_LN_CASE(2)
         CR_LN_CASE(3)
