@@ -14,16 +14,17 @@
 //               itself (the stale cache tile, or for the training loss head the
 //               stale and joint cache tiles) by TMA, as soon as the epilogue has
 //               released its slot.
-//   warp 3      TMA store issuer for the staged output (for the fp32 residual
-//               stream a TMA reduce-add: x += acc + b in L2).
+//   warp 3      TMA store issuer for the staged in-place tile.
 //   warps 4..11 epilogue, two groups of four warps (one per TMEM lane
 //               quarter) splitting each tile's columns: tcgen05.ld 32 lanes x
 //               16 columns, bias from shared memory, then one of: bf16, GELU,
 //               fp32, RoPE on Q/K (into 128B-swizzled staging buffers, one box
-//               of 128 B-wide columns at a time, double-buffered per group), or
-//               in place on the staged tile: cache kv = kv + sigma_delta
-//               (acc + b) (+ R_M on K).  Staged
-//               data goes out with TMA stores (coalesced, asynchronous).  The
+//               of 128 B-wide columns at a time, double-buffered per group,
+//               each box stored by one thread of the group after a named
+//               barrier; the fp32 residual stream as a TMA reduce-add,
+//               x += acc + b in L2), or in place on the staged tile: cache
+//               kv = kv + sigma_delta (acc + b) (+ R_M on K), stored by warp 3.
+//               Staged data goes out with TMA (coalesced, asynchronous).  The
 //               paged head and the loss head write from registers instead: the
 //               repaired rows into the paged target cache, or the training
 //               gradient dz = c (acc + b - (joint - stale) / sigma_delta) in
@@ -307,6 +308,20 @@ __device__ __forceinline__ void rotate16(float* a, float* b, float p, const floa
 // K = 16 MMA and finds the next 64 M (or N) 8 KB further on (leading byte
 // offset).
 
+// all n threads at named barrier id agree on v (true only if every one passed true)
+__device__ __forceinline__ bool named_bar_and(uint32_t id, uint32_t n, bool v) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "barrier.cta.red.and.pred q, %2, %3, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"(v ? 1u : 0u), "r"(id), "r"(n)
+        : "memory");
+    return r != 0;
+}
+
 template <int BN, int EPI, int CG, int LAY>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -333,9 +348,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     uint64_t* epi_full = tempty + 2;     // [8]
     uint64_t* epi_empty = epi_full + 8;  // [8] back to the loader: box b (and the vectors) free
     uint64_t* drain = epi_empty + 8;
-    uint64_t* epi_done = drain + 1;      // [8] in-place: box b written; else [group][buffer]
-    uint64_t* st_free = epi_done + 8;    // [group][buffer]: the TMA store has read that buffer
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(st_free + 4);
+    uint64_t* epi_done = drain + 1;      // [8] in-place: box b written (to the store issuer)
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(epi_done + 8);
     int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
     const uint32_t warp = warp_id(), lane = lane_id();
@@ -356,12 +370,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
         for (int b = 0; b < 8; ++b) {
             mbar_init(&epi_full[b], 1);
-            mbar_init(&epi_empty[b], 1);
-            // in-place: one barrier per box for all 256 epilogue threads;
-            // store-only: one per group and buffer for that group's 128 threads
-            mbar_init(&epi_done[b], Cfg::kInPlace ? 256 : 128);
+            // store-only: epi_empty[0] takes one arrive from each epilogue group
+            mbar_init(&epi_empty[b], (!Cfg::kInPlace && b == 0) ? 2 : 1);
+            // in-place: one barrier per box for all 256 epilogue threads
+            mbar_init(&epi_done[b], 256);
         }
-        for (int b = 0; b < 4; ++b) mbar_init(&st_free[b], 1);
         mbar_init(drain, 1);
         *abort_flag = 0;
         fence_barrier_init();
@@ -532,22 +545,20 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             }
         }
     } else if (warp == 3) {
-        // ---------------------------------------------------- TMA store issuer:
-        // writes each staged buffer back once the 128 epilogue threads have
-        // filled it, and hands the buffer (or the in-place tile and the bias
-        // slice) back when TMA has read it.  The bulk-group waits belong to the
-        // elected lane that committed the stores.
-        const bool leader = elect_one();
-        bool ok = true;
-        uint32_t pk = 0;               // in-place tiles so far
-        uint32_t pkg[2] = {0u, 0u};    // boxes of each epilogue group so far
-        for (int t = cta0; t < total && ok; t += ncta) {
-            const int m0 = (tile_lin(p, t) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-            const int n0 = tile_n0<BN, Cfg::kKV>(p, tile_lin(p, t));
-            const bool rows_in = m0 < p.M;   // a pair tile's second half may lie below M
-            if constexpr (Cfg::kInPlace) {
-                // each box as soon as the epilogue has written it; once TMA has read
-                // it, the loader may bring the next tile's copy of that box
+        // ---------------------------------------------------- TMA store issuer
+        // of the in-place epilogues: writes each box of the staged tile back
+        // once the 256 epilogue threads have updated it, and hands the box back
+        // to the loader when TMA has read it (the store-only epilogues issue
+        // their own stores).  The bulk-group waits belong to the elected lane
+        // that committed the stores.
+        if constexpr (Cfg::kInPlace) {
+            const bool leader = elect_one();
+            bool ok = true;
+            uint32_t pk = 0;   // in-place tiles so far
+            for (int t = cta0; t < total && ok; t += ncta) {
+                const int m0 = (tile_lin(p, t) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
+                const int n0 = tile_n0<BN, Cfg::kKV>(p, tile_lin(p, t));
+                const bool rows_in = m0 < p.M;   // a pair tile's second half may lie below M
                 for (int b = 0; b < Cfg::kBoxes && ok; ++b) {
                     if (!(ok = mbar_wait_warp(&epi_done[b], pk & 1u, wc, 401))) break;
                     if (leader) {
@@ -561,44 +572,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     __syncwarp();
                 }
                 ++pk;
-            } else {
-                // one box store stays in flight: a buffer goes back to its group
-                // once the next box's store is issued and the older one has
-                // read it; by the end of the tile every store has read its box
-                int prev = -1;
-                for (int k = 0; k < Cfg::kBoxes; ++k) {
-                    // box k was staged by epilogue group k & 1 in its buffer pkg & 1
-                    constexpr uint32_t GB = Cfg::kGroupBufs;
-                    const int g = k & 1;
-                    const uint32_t b = static_cast<uint32_t>(g) * GB + (pkg[g] % GB);
-                    if (!(ok = mbar_wait_warp(&epi_done[b], (pkg[g] / GB) & 1u, wc, 402))) break;
-                    if (leader) {
-                        if (rows_in) {
-                            const int x = n0 + k * Cfg::kBoxCols, y = m0 + tile_part(p, t) * p.M;
-                            if constexpr (Cfg::kReduce)
-                                tma_reduce_add_2d(&tmC, tile + b * 16384, x, y);
-                            else
-                                tma_store_2d(&tmC, tile + b * 16384, x, y);
-                        }
-                        tma_store_commit();
-                        tma_store_wait_read<1>();
-                        if (prev >= 0) mbar_arrive(&st_free[prev]);
-                    }
-                    __syncwarp();
-                    prev = static_cast<int>(b);
-                    ++pkg[g];
-                }
-                if (leader) {
-                    tma_store_wait_read0();
-                    if (ok && prev >= 0) mbar_arrive(&st_free[prev]);
-                }
-                __syncwarp();
-                if (ok && epi_load && leader) mbar_arrive(epi_empty);
-                __syncwarp();
             }
+            if (leader) tma_store_wait0();
+            __syncwarp();
         }
-        if (leader) tma_store_wait0();
-        __syncwarp();
     } else if (warp == 1 && (CG == 1 || rank == 0)) {
         // ---------------------------------------------------- MMA issuer
         // (for a pair: the even CTA, issuing M = 256 MMAs over both CTAs'
@@ -695,7 +672,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             ok = mbar_wait(&tfull[acc], acc_phase, wc, 301);
             // in-place epilogues wait box by box below
             if (epi_load && !Cfg::kInPlace) ok = ok && mbar_wait(epi_full, static_cast<uint32_t>(i) & 1u, wc, 302);
-            if (!__all_sync(0xffffffffu, ok)) {
+            if constexpr (!Cfg::kInPlace) {
+                // the group's 128 threads take the same path (named barriers follow)
+                if (!(ok = named_bar_and(1 + eg, 128, ok))) break;
+            } else if (!__all_sync(0xffffffffu, ok)) {
                 ok = false;
                 break;
             }
@@ -897,18 +877,21 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 // store-only epilogues: one 128 B-wide box of columns at a time,
                 // into alternating staging buffers
                 constexpr int PC = Cfg::kBoxCols;
+                // one thread of each group issues (and waits on) its stores; the
+                // group meets at a named barrier before and after writing a box
+                const bool glead = (quad == 0 && lane == 0);
                 // boxes alternate between the groups; each group cycles its own
                 // kGroupBufs staging buffers (pk counts this group's boxes)
                 for (int k = eg; k < Cfg::kBoxes && ok; k += 2, ++pk) {
                     constexpr uint32_t GB = Cfg::kGroupBufs;
                     const uint32_t bsel = static_cast<uint32_t>(eg) * GB + (pk % GB);
-                    if (pk >= GB) {
-                        ok = mbar_wait(&st_free[bsel], ((pk / GB) - 1) & 1u, wc, 304);
-                        if (!__all_sync(0xffffffffu, ok)) {
-                            ok = false;
-                            break;
-                        }
+                    // the group's leader stored this buffer GB boxes ago: once that
+                    // store has read it, the group may rewrite it
+                    if (glead && pk >= GB) {
+                        if constexpr (GB == 1) tma_store_wait_read0();
+                        else tma_store_wait_read<1>();
                     }
+                    named_bar_sync(1 + eg, 128);
                     uint8_t* buf = tile + bsel * 16384;
                     const int c0 = k * PC;
                     if constexpr (EPI == EPI_QKV_ROPE) {
@@ -966,15 +949,29 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                         }
                     }
                     fence_async_smem();
-                    mbar_arrive(&epi_done[bsel]);
+                    named_bar_sync(1 + eg, 128);
+                    if (glead) {
+                        if (m0 < p.M) {
+                            const int x = n0 + k * PC, y = m0 + tile_part(p, t) * p.M;
+                            if constexpr (Cfg::kReduce)
+                                tma_reduce_add_2d(&tmC, buf, x, y);
+                            else
+                                tma_store_2d(&tmC, buf, x, y);
+                        }
+                        tma_store_commit();
+                    }
                 }
                 // this group has read its columns of the TMEM buffer
                 tc_fence_before();
                 __syncwarp();
                 if (ok && lane == 0) release_acc(&tempty[acc]);
+                if (ok && glead && epi_load) mbar_arrive(epi_empty);
             }
             acc ^= 1u;
             if (acc == 0) acc_phase ^= 1u;
+        }
+        if constexpr (!Cfg::kInPlace) {
+            if ((warp & 3u) == 0 && lane == 0) tma_store_wait0();
         }
     }
     tc_fence_before();
