@@ -354,33 +354,25 @@ static cr_status compress_stage2(const Dims& d, const cr_weights* w, const uint1
     const int64_t Sd = d.S * d.dseg;
     GemmParams gp{};
     gp.status = status;
-    gp.bias = w->b_map;
-    gp.out = se32;
-    gp.ldo = 2 * d.dc;
-    if ((s = launch_gemm(y, 2 * Sd, w->w_map, N, d.dc, Sd, EPI_F32, gp, nullptr, 0, st,
-                         y + Sd)) != CR_OK)
-        return s;
-    gp.bias = w->b_tok;
-    gp.out = se32 + d.dc;
-    if ((s = launch_gemm(embb, d.dmodel, w->w_tok, N, d.dc, d.dmodel, EPI_F32, gp, nullptr, 0,
-                         st)) != CR_OK)
-        return s;
+    // W_map over [y_hi | y_lo] and P_tok over the embeddings in one launch: the
+    // short P_tok tiles fill the CTA pairs the W_map tiles leave idle
+    const GemmProduct map{y, 2 * Sd, y + Sd, w->w_map, d.dc, Sd, w->b_map, se32, 2 * d.dc};
+    const GemmProduct tok{embb, d.dmodel, nullptr, w->w_tok, d.dc, d.dmodel, w->b_tok, se32 + d.dc,
+                          2 * d.dc};
+    if ((s = launch_gemm_pair(map, tok, N, gp, st)) != CR_OK) return s;
     if ((s = launch_split_bf16(se32, N, 2 * d.dc, se2, st)) != CR_OK) return s;
-    gp.bias = w->b_fuse;
-    gp.out = h0_out;
-    gp.ldo = d.db;
-    if ((s = launch_gemm(se2, 4 * d.dc, w->w_fuse, N, d.db, 2 * d.dc, EPI_F32, gp, nullptr, 0,
-                         st, se2 + 2 * d.dc)) != CR_OK)
-        return s;
+    // the fusion F over [s | e] and the reinjection P_b over s, both two-term
+    const GemmProduct fuse{se2, 4 * d.dc, se2 + 2 * d.dc, w->w_fuse, d.db, 2 * d.dc, w->b_fuse, h0_out,
+                           d.db};
     if (d.B > 0) {
-        gp.bias = w->b_rein;
-        gp.out = rein_out;
-        gp.ldo = d.B * d.db;
-        if ((s = launch_gemm(se2, 4 * d.dc, w->w_rein, N, d.B * d.db, d.dc, EPI_F32, gp, nullptr,
-                             0, st, se2 + 2 * d.dc)) != CR_OK)
-            return s;
+        const GemmProduct rein{se2, 4 * d.dc, se2 + 2 * d.dc, w->w_rein, d.B * d.db, d.dc, w->b_rein,
+                               rein_out, d.B * d.db};
+        return launch_gemm_pair(fuse, rein, N, gp, st);
     }
-    return CR_OK;
+    gp.bias = fuse.bias;
+    gp.out = fuse.out;
+    gp.ldo = fuse.ldo;
+    return launch_gemm(fuse.A, fuse.lda, fuse.W, N, fuse.N, fuse.K, EPI_F32, gp, nullptr, 0, st, fuse.A_lo);
 }
 
 static SegParams seg_params(const Dims& d, const cr_weights* w, int64_t N, uint16_t* y,

@@ -328,7 +328,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 const __grid_constant__ CUtensorMap tmC, const __grid_constant__ GemmParams p) {
     using Cfg = GemmCfg<BN, EPI, CG>;
     constexpr int STAGES = Cfg::kStages;
-    constexpr bool kAMN = (LAY == LAY_MM), kBMN = (LAY != LAY_KK);
+    constexpr bool kAMN = (LAY == LAY_MM), kBMN = (LAY == LAY_KM || LAY == LAY_MM);
+    constexpr bool kPair = (LAY == LAY_KK2);
     static_assert(!kBMN || (BN / CG) % 64 == 0, "an MN-major W half must be whole 64-column boxes");
     constexpr uint32_t IDESC = idesc_bf16(BM * CG, BN, kAMN, kBMN);
 
@@ -401,8 +402,32 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const int total = p.num_m * p.num_n * p.split_k;
     // a two-term A runs the W k-blocks twice: first against A_hi, then A_lo
     const int num_k = p.split_kb > 0 ? 2 * p.split_kb : (p.K + BK - 1) / BK;
+    const int num_k2 = kPair ? (p.split_kb2 > 0 ? 2 * p.split_kb2 : (p.K2 + BK - 1) / BK) : 0;
     const int k_per = (num_k + p.split_k - 1) / p.split_k;
+    // two products (n_split > 0): a tile belongs to the second one when its first
+    // column is at or past n_split
+    auto second = [&](int n0) { return kPair && n0 >= p.n_split; };
+    // Two products, pair c taking tiles c, c + ncta, ...: the first product's H
+    // (longer) tiles come first.  Where the launch has E = tiles - pairs > 0
+    // second tiles to hand out and the second product's tiles can take them all
+    // twice over, E of those lead instead, so that the pairs running two tiles
+    // run two short ones: pairs 0..E-1 short + short, E..E+H-1 one long tile,
+    // the rest one short tile.
+    const int n_long = kPair ? p.num_m * (p.n_split / BN) : 0;
+    const int n_extra = total - ncta;
+    const bool reorder = kPair && n_extra > 0 && 2 * n_extra <= total - n_long && n_long + n_extra <= ncta;
+    auto lin = [&](int t) {
+        if constexpr (kPair) {
+            if (reorder) return t < n_extra ? n_long + t : (t < n_extra + n_long ? t - n_extra : t);
+        }
+        return tile_lin(p, t);
+    };
     auto k_range = [&](int t, int* kb0, int* kb1) {
+        if constexpr (kPair) {
+            *kb0 = 0;
+            *kb1 = second(tile_n0<BN, Cfg::kKV>(p, lin(t))) ? num_k2 : num_k;
+            return;
+        }
         *kb0 = tile_part(p, t) * k_per;
         *kb1 = min(num_k, *kb0 + k_per);
     };
@@ -424,13 +449,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             tma_prefetch(&tmB);
             if (p.split_kb > 0) tma_prefetch(&p.tm_alo);
             if constexpr (Cfg::kInPlace) tma_prefetch(&tmC);
+            if constexpr (kPair) {
+                tma_prefetch(&p.tm_a2);
+                tma_prefetch(&p.tm_b2);
+                if (p.split_kb2 > 0) tma_prefetch(&p.tm_alo2);
+            }
         }
         __syncwarp();
         uint32_t stage = 0, phase = 0;
         bool ok = true;
         for (int t = cta0; t < total && ok; t += ncta) {
-            const int m0 = (tile_lin(p, t) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-            const int n0 = tile_n0<BN, Cfg::kKV>(p, tile_lin(p, t));
+            const int m0 = (lin(t) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
+            const int n0 = tile_n0<BN, Cfg::kKV>(p, lin(t));
             int kbeg, kend;
             k_range(t, &kbeg, &kend);
             for (int kb = kbeg; kb < kend; ++kb) {
@@ -439,12 +469,16 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 if (elect_one()) {
                     // W columns of this tile: its own column block, or (grouped
                     // rows) the block that belongs to its rows' group
+                    const bool g2 = second(n0);
                     const int nw = p.bgroup_rows > 0
-                                       ? ((tile_lin(p, t) % p.num_m) * (BM * CG) / p.bgroup_rows) * BN : n0;
+                                       ? ((lin(t) % p.num_m) * (BM * CG) / p.bgroup_rows) * BN
+                                       : (g2 ? n0 - p.n_split : n0);
                     const int nb0 = nw + static_cast<int>(rank) * (BN / CG);
-                    const bool lo = p.split_kb > 0 && kb >= p.split_kb;
-                    const CUtensorMap* ma = lo ? &p.tm_alo : &tmA;
-                    const int ka = (lo ? kb - p.split_kb : kb) * BK;   // A and W column
+                    const int skb = g2 ? p.split_kb2 : p.split_kb;
+                    const bool lo = skb > 0 && kb >= skb;
+                    const CUtensorMap* ma = g2 ? (lo ? &p.tm_alo2 : &p.tm_a2) : (lo ? &p.tm_alo : &tmA);
+                    const CUtensorMap* mb = g2 ? &p.tm_b2 : &tmB;
+                    const int ka = (lo ? kb - skb : kb) * BK;   // A and W column
                     uint64_t* fq = &full[stage];
                     auto load = [&](uint8_t* dst, const CUtensorMap* m, int x, int y, uint32_t fb) {
                         if constexpr (CG == 1)
@@ -470,7 +504,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                         for (int i = 0; i < BN / CG / 64; ++i)
                             load(sa + A_BYTES + i * 8192, &tmB, nb0 + 64 * i, ka, fb);
                     } else {
-                        load(sa + A_BYTES, &tmB, ka, nb0, fb);
+                        load(sa + A_BYTES, mb, ka, nb0, fb);
                     }
                 }
                 __syncwarp();
@@ -496,8 +530,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             bool ok = true;
             int i = 0;
             for (int t = cta0; t < total && ok; t += ncta, ++i) {
-                const int m0 = (tile_lin(p, t) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-                const int n0 = tile_n0<BN, Cfg::kKV>(p, tile_lin(p, t));
+                const int m0 = (lin(t) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
+                const int n0 = tile_n0<BN, Cfg::kKV>(p, lin(t));
                 const int nb = min(BN, p.N - n0);
                 const uint32_t vbytes = static_cast<uint32_t>(nb) * 4u;
                 if constexpr (Cfg::kInPlace) {
@@ -533,7 +567,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                         break;
                     if (elect_one()) {
                         mbar_expect_tx(epi_full, vbytes);
-                        bulk_load(vec, p.bias + n0, vbytes, epi_full);
+                        bulk_load(vec, second(n0) ? p.bias2 + (n0 - p.n_split) : p.bias + n0, vbytes,
+                                  epi_full);
                     }
                     __syncwarp();
                 }
@@ -556,8 +591,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             bool ok = true;
             uint32_t pk = 0;   // in-place tiles so far
             for (int t = cta0; t < total && ok; t += ncta) {
-                const int m0 = (tile_lin(p, t) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-                const int n0 = tile_n0<BN, Cfg::kKV>(p, tile_lin(p, t));
+                const int m0 = (lin(t) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
+                const int n0 = tile_n0<BN, Cfg::kKV>(p, lin(t));
                 const bool rows_in = m0 < p.M;   // a pair tile's second half may lie below M
                 for (int b = 0; b < Cfg::kBoxes && ok; ++b) {
                     if (!(ok = mbar_wait_warp(&epi_done[b], pk & 1u, wc, 401))) break;
@@ -662,8 +697,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         bool ok = true;
         int i = 0;
         for (int t = cta0; t < total && ok; t += ncta, ++i) {
-            const int m0 = (tile_lin(p, t) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
-            const int n0 = tile_n0<BN, Cfg::kKV>(p, tile_lin(p, t));
+            const int m0 = (lin(t) % p.num_m) * (BM * CG) + static_cast<int>(rank) * BM;
+            const int n0 = tile_n0<BN, Cfg::kKV>(p, lin(t));
             // QKV: the rotation angles depend on (row, pair index) only: cos/sin
             // for every head of the tile, fetched while the MMAs still run
             constexpr int NP = (EPI == EPI_QKV_ROPE) ? 32 : 1;
@@ -952,11 +987,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     named_bar_sync(1 + eg, 128);
                     if (glead) {
                         if (m0 < p.M) {
-                            const int x = n0 + k * PC, y = m0 + tile_part(p, t) * p.M;
+                            const bool g2 = second(n0);
+                            const int x = (g2 ? n0 - p.n_split : n0) + k * PC, y = m0 + tile_part(p, t) * p.M;
                             if constexpr (Cfg::kReduce)
                                 tma_reduce_add_2d(&tmC, buf, x, y);
                             else
-                                tma_store_2d(&tmC, buf, x, y);
+                                tma_store_2d(g2 ? &p.tm_c2 : &tmC, buf, x, y);
                         }
                         tma_store_commit();
                     }
@@ -1097,6 +1133,7 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
     p.num_n = static_cast<int32_t>((N + BN - 1) / BN);
     p.split_k = 1;
     p.n_fast = 0;
+    p.n_split = 0;
     if (kv && p.col_block > 0) {
         // output choice: half of the column blocks, each a whole number of tiles
         if (p.col_block % BN != 0 || N % (2 * static_cast<int64_t>(p.col_block)) != 0)
@@ -1202,6 +1239,65 @@ __global__ void __launch_bounds__(256)
 }
 }  // namespace
 
+cr_status launch_gemm_pair(const GemmProduct& a, const GemmProduct& b, int64_t M, GemmParams p,
+                           cudaStream_t st) {
+    constexpr int BN = 256;
+    if (M < 1 || a.N < 1 || b.N < 1 || a.K < 1 || b.K < 1) return CR_ERR_INVALID_ARG;
+    // tiles of 256 columns must not straddle the two products, and the tile's
+    // vectors come from one bias array or none
+    if (a.N % BN != 0 || (a.bias == nullptr) != (b.bias == nullptr) || a.N + b.N > (1 << 30)) {
+        GemmParams pa = p;
+        pa.bias = a.bias;
+        pa.out = a.out;
+        pa.ldo = a.ldo;
+        const cr_status s = launch_gemm(a.A, a.lda, a.W, M, a.N, a.K, EPI_F32, pa, nullptr, 0, st, a.A_lo);
+        if (s != CR_OK) return s;
+        GemmParams pb = p;
+        pb.bias = b.bias;
+        pb.out = b.out;
+        pb.ldo = b.ldo;
+        return launch_gemm(b.A, b.lda, b.W, M, b.N, b.K, EPI_F32, pb, nullptr, 0, st, b.A_lo);
+    }
+    if ((b.bias && (b.N % 4) != 0)) return CR_ERR_UNSUPPORTED;   // bias slices are 16-byte bulk copies
+    p.M = static_cast<int32_t>(M);
+    p.N = static_cast<int32_t>(a.N + b.N);
+    p.K = static_cast<int32_t>(a.K);
+    p.K2 = static_cast<int32_t>(b.K);
+    p.num_m = static_cast<int32_t>((M + BM * kCG - 1) / (BM * kCG));
+    p.num_n = static_cast<int32_t>((a.N + b.N + BN - 1) / BN);
+    p.split_k = 1;
+    p.n_fast = 0;
+    p.col_block = 0;
+    p.bgroup_rows = 0;
+    p.n_split = static_cast<int32_t>(a.N);
+    p.bias = a.bias;
+    p.bias2 = b.bias;
+    p.out = a.out;
+    p.ldo = a.ldo;
+    const auto BF = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    const auto SW = CU_TENSOR_MAP_SWIZZLE_128B;
+    CUtensorMap ta, tb, tc;
+    // columns past K read as zeros in both terms (TMA bounds)
+    if (!make_tmap_2d(&ta, a.A, BF, a.K, M, a.lda * 2, BK, BM, SW) ||
+        !make_tmap_2d(&tb, a.W, BF, a.K, a.N, a.K * 2, BK, BN / kCG, SW) ||
+        !make_tmap_2d(&tc, a.out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, a.N, M, a.ldo * 4, 32, BM, SW) ||
+        !make_tmap_2d(&p.tm_a2, b.A, BF, b.K, M, b.lda * 2, BK, BM, SW) ||
+        !make_tmap_2d(&p.tm_b2, b.W, BF, b.K, b.N, b.K * 2, BK, BN / kCG, SW) ||
+        !make_tmap_2d(&p.tm_c2, b.out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, b.N, M, b.ldo * 4, 32, BM, SW))
+        return CR_ERR_INVALID_ARG;
+    p.split_kb = 0;
+    if (a.A_lo) {
+        if (!make_tmap_2d(&p.tm_alo, a.A_lo, BF, a.K, M, a.lda * 2, BK, BM, SW)) return CR_ERR_INVALID_ARG;
+        p.split_kb = static_cast<int32_t>((a.K + BK - 1) / BK);
+    }
+    p.split_kb2 = 0;
+    if (b.A_lo) {
+        if (!make_tmap_2d(&p.tm_alo2, b.A_lo, BF, b.K, M, b.lda * 2, BK, BM, SW)) return CR_ERR_INVALID_ARG;
+        p.split_kb2 = static_cast<int32_t>((b.K + BK - 1) / BK);
+    }
+    return launch_bn<BN, EPI_F32, kCG, LAY_KK2>(ta, tb, tc, p, st);
+}
+
 cr_status launch_gemm_lay(const uint16_t* A, int64_t lda, int lay, const uint16_t* W, int64_t ldw,
                           int64_t M, int64_t N, int64_t K, int epi, GemmParams p, cudaStream_t st,
                           float* scratch, size_t scratch_bytes) {
@@ -1227,6 +1323,7 @@ cr_status launch_gemm_lay(const uint16_t* A, int64_t lda, int lay, const uint16_
     p.col_block = 0;
     p.split_kb = 0;
     p.split_k = 1;
+    p.n_split = 0;
     // Split-K: when the tiles fill the CTA pairs poorly (the last round partly
     // empty), cut each tile's k-loop into s parts, each written to its own fp32
     // slice of the scratch and summed in a fixed order by a second kernel.  s

@@ -62,7 +62,9 @@ enum GemmEpi : int {
 
 // Operand layouts of the GEMM: K-major A and W (the forward), K-major A with
 // MN-major W (dX = dY W), MN-major A and W (dW = dY^T X).
-enum GemmLayout : int { LAY_KK = 0, LAY_KM = 1, LAY_MM = 2 };
+// LAY_KK2: both operands K-major, two products in one launch (launch_gemm_pair);
+// its own instantiation, so that the one-product kernels carry none of its logic
+enum GemmLayout : int { LAY_KK = 0, LAY_KM = 1, LAY_MM = 2, LAY_KK2 = 3 };
 
 struct GemmParams {
     int32_t M, N, K;
@@ -114,9 +116,32 @@ struct GemmParams {
     // tile reads W columns [g BN, (g + 1) BN) of the W matrix, g = row / bgroup_rows,
     // and writes output columns [0, BN); 0 = off
     int32_t bgroup_rows;
+    // two products in one launch (launch_gemm_pair, EPI_F32): the output columns
+    // [n_split, N) of the launch belong to a second product with its own A
+    // (tm_a2, two-term through tm_alo2 when split_kb2 > 0), W (tm_b2, its rows
+    // counted from n_split), K2, bias2 and output (tm_c2, its columns counted from
+    // n_split); n_split is a multiple of the tile width.  0 = one product.
+    int32_t n_split;
+    int32_t K2;
+    int32_t split_kb2;
+    const float* bias2;
     float inv_freq[64];      // RoPE frequencies, rope_dim / 2 entries
     CUtensorMap tm_joint;    // EPI_KV_LOSS (set by launch_gemm; the type carries its alignment)
     CUtensorMap tm_alo;      // two-term A: the A_lo operand
+    CUtensorMap tm_a2, tm_alo2, tm_b2, tm_c2;   // the second product (n_split > 0)
+};
+
+// One product of launch_gemm_pair: C[M, N] = A[M, K] W[N, K]^T + bias (fp32 out),
+// A two-term when A_lo is given (as for launch_gemm).
+struct GemmProduct {
+    const uint16_t* A;
+    int64_t lda;
+    const uint16_t* A_lo;
+    const uint16_t* W;
+    int64_t N, K;
+    const float* bias;
+    float* out;
+    int64_t ldo;
 };
 
 // ------------------------------------------------------------------ segment projection
@@ -258,6 +283,12 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
 // with LAY_MM also M.  No bias.
 // scratch (optional, fp32, scratch_bytes long): room for split-K parts; with it
 // the product may run as up to 8 k-parts summed in a fixed order afterwards.
+// Two fp32 products over the same rows in one launch, so that the tiles of the
+// shorter one fill the CTA pairs the other leaves idle.  Falls back to two
+// launch_gemm calls where the first product's width is not a multiple of the
+// tile width.
+cr_status launch_gemm_pair(const GemmProduct& a, const GemmProduct& b, int64_t M, GemmParams p,
+                           cudaStream_t st);
 cr_status launch_gemm_lay(const uint16_t* A, int64_t lda, int lay, const uint16_t* W, int64_t ldw,
                           int64_t M, int64_t N, int64_t K, int epi, GemmParams p, cudaStream_t st,
                           float* scratch = nullptr, size_t scratch_bytes = 0);
