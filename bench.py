@@ -3,8 +3,10 @@
 latency per request, with the roofline fraction of the dominant kernel.
 
 One step = one request through RepairSession.repair on one stream: the C-ABI
-calls cr_assemble_compress (assembly fused with the encoder), cr_repair_forward
-and cr_apply_residual, captured once into a CUDA graph and replayed.
+calls cr_assemble_compress (the encoder reading the chunk pool; for a bf16
+cache the assembled copy is not written), cr_repair_forward and
+cr_apply_residual_pool (the head reading the stale rows from the pool and
+writing the repaired cache), captured once into a CUDA graph and replayed.
 Default workload: the Llama-3.1-8B-shaped cache (32 layers, 8 KV heads,
 head_dim 128, d_model 4096) with the d_c 512 / d_b 1024 / 6-block repairer,
 one request of 10 chunks x 512 tokens.  Inputs are seeded and synthetic; the
@@ -281,6 +283,16 @@ def run_ours(args):
     rope_mode = cr.CR_ROPE_GLOBAL if args.rope else cr.CR_ROPE_NONE
     freq = case.inv_freq_target if args.rope else None
     choice = dict(component=args.component, offset=args.offset, keep_first_chunk=args.keep_first_chunk)
+    # RepairSession.repair's path: for a bf16 cache under the method's output the
+    # encoder and the head read the pool, and no assembled cache is written
+    pooled = (case.target.cache_dtype == "bf16" and args.component == "kv" and args.offset == "stale"
+              and not args.keep_first_chunk)
+
+    def head(f, mode):
+        if pooled:
+            sess.apply_pool(a, kvp, p.chunk_start, p.chunk_len, p.chunk_idx, p.cu_chunks, f, mode)
+        else:
+            sess.apply(a, f, mode, **choice)
 
     def step():
         sess.repair(kvp, embp, p.chunk_start, p.chunk_len, p.chunk_idx, p.cu_chunks, freq, rope_mode,
@@ -288,16 +300,16 @@ def run_ours(args):
 
     # ---- per-call timing (eager), for the stage breakdown and the roofline
     a = sess.assemble(kvp, embp, p.chunk_start, p.chunk_len, p.chunk_idx, p.cu_chunks)
-    # the step runs the fused front (assemble_compress); the two calls it replaces are
-    # timed too, for the breakdown
+    # the step runs the fused front (assemble_compress) and the head as repair() does;
+    # the two calls the front replaces are timed too, for the breakdown
     calls = [("assemble", lambda: sess.assemble(kvp, embp, p.chunk_start, p.chunk_len,
                                                 p.chunk_idx, p.cu_chunks)),
              ("compress", lambda: sess.compress(a)),
              ("assemble_compress", lambda: sess.assemble_compress(kvp, embp, p.chunk_start,
                                                                   p.chunk_len, p.chunk_idx,
-                                                                  p.cu_chunks)),
+                                                                  p.cu_chunks, write_kv=not pooled)),
              ("forward", lambda: sess.forward(a, mask_mode=args.mask)),
-             ("apply", lambda: sess.apply(a, freq, rope_mode, **choice))]
+             ("apply", lambda: head(freq, rope_mode))]
     for _ in range(3):
         for _, fn in calls:
             fn()
@@ -383,7 +395,7 @@ def run_ours(args):
     # above leaves K canonical. The head with R_M, timed like the other calls (after
     # the timed region, so that the launch order before it is unchanged).
     if not args.rope and not args.variant:
-        fn = lambda: sess.apply(a, case.inv_freq_target, cr.CR_ROPE_GLOBAL, **choice)
+        fn = lambda: head(case.inv_freq_target, cr.CR_ROPE_GLOBAL)
         for _ in range(3):
             fn()
         torch.cuda.synchronize()
@@ -397,13 +409,17 @@ def run_ours(args):
         torch.cuda.synchronize()
         stages["apply_rope"] = statistics.median(e0.elapsed_time(e1) for e0, e1 in ev)
     gather_bytes = 2.0 * N * (tg.d_kv + tg.d_model) * es
+    # the fused front's HBM work: the pool's cache rows read (and, without the pool
+    # head, the assembled copy written), the embeddings read and written
+    front_bytes = N * (tg.d_kv + 2 * tg.d_model) * es if pooled else gather_bytes
     kernels = {
         "attn_kernel": dict(name=f"attn_kernel ({args.mask.replace('_', '-')} flash attention)",
                             launches=rp.n_blocks,
                             ms=attn_ms, flops=attn_flops,
                             algorithmic=f"4*d_b per visible (query, key) pair = {attn_flops:.3e} "
                                         f"flop per launch"),
-        "gemm_kernel<256,KV>": dict(name="cr_apply_residual (KV residual head GEMM + residual add)",
+        "gemm_kernel<256,KV>": dict(name=("cr_apply_residual_pool" if pooled else "cr_apply_residual")
+                                    + " (KV residual head GEMM + residual add)",
                                     launches=1, ms=head_ms, flops=head_flops,
                                     algorithmic=f"2*N*d_b*(columns visited) = {head_flops:.3e} "
                                                 f"flop per launch"),
@@ -422,28 +438,29 @@ def run_ours(args):
                 "launches_per_step": dom["launches"]}
     # Whole request: the algorithmic tensor work at the sustained bf16 peak (the step
     # loop keeps the tensor cores busy through the whole timed region) plus the
-    # front's cache traffic (pool read, assembled write) at the measured copy
-    # bandwidth; the segment projection's flops ride on that traffic.
+    # front's HBM work (the pool read; the assembled write where the head does not
+    # read the pool) at the measured copy bandwidth; the segment projection's flops
+    # ride on that traffic.
     S = 2 * tg.n_layers * tg.n_kv_heads
     lin_flops = 2.0 * N * (S * rp.d_seg * rp.d_c + tg.d_model * rp.d_c + 2 * rp.d_c * rp.d_b
                            + rp.n_blocks * rp.d_c * rp.d_b
                            + rp.n_blocks * (4 * rp.d_b * rp.d_b + 2 * rp.d_b * rp.mlp_hidden))
     tensor_flops = lin_flops + rp.n_blocks * attn_flops + head_flops
-    ideal_ms = tensor_flops / (tf_sus * 1e12) * 1e3 + gather_bytes / (hbm * 1e9) * 1e3
+    ideal_ms = tensor_flops / (tf_sus * 1e12) * 1e3 + front_bytes / (hbm * 1e9) * 1e3
     roofline.update({
         "request_frac": ideal_ms / (total_ms / args.steps),
         "request_frac_p50": ideal_ms / statistics.median(per_step),
         "request_ideal_ms": ideal_ms,
         "request_algorithmic": (f"{tensor_flops:.4e} tensor flop (linears {lin_flops:.3e}, attention "
                                 f"{rp.n_blocks * attn_flops:.3e}, head {head_flops:.3e}) at the sustained "
-                                f"{tf_sus} TF/s + {gather_bytes:.4e} front bytes at {hbm} GB/s"),
+                                f"{tf_sus} TF/s + {front_bytes:.4e} front bytes at {hbm} GB/s"),
     })
     stage_roofline = {
         "assemble_hbm_frac": gather_bytes / (stages["assemble"] * 1e-3) / 1e9 / hbm,
         "assemble_hbm_gbs": gather_bytes / (stages["assemble"] * 1e-3) / 1e9,
-        # fused front: the same cache bytes (pool read, assembled write) plus the
-        # encoder's small GEMMs, over the whole call
-        "front_hbm_frac": gather_bytes / (stages["assemble_compress"] * 1e-3) / 1e9 / hbm,
+        # fused front: its cache and embedding bytes plus the encoder's small GEMMs,
+        # over the whole call
+        "front_hbm_frac": front_bytes / (stages["assemble_compress"] * 1e-3) / 1e9 / hbm,
         "front_ms": stages["assemble_compress"],
         "attention_tensor_frac": attn_flops / (attn_ms * 1e-3) / 1e12 / tf_burst,
         "attention_ms_per_launch": attn_ms,
@@ -454,12 +471,16 @@ def run_ours(args):
     if "apply_rope" in stages:
         stage_roofline["head_rope_tensor_frac"] = head_flops / (stages["apply_rope"] * 1e-3) / 1e12 / tf_burst
         stage_roofline["head_rope_ms"] = stages["apply_rope"]
-    # front: gather (embeddings + chunk map), sigma fold, projection, four encoder
-    # GEMMs and the two-term split of s|e (fp32 caches: the two-call path with its
-    # two bf16 conversions); forward: RoPE table, 7 kernels per block, final
-    # LayerNorm; head
-    launches_per_step = 1 + (2 + 5 + (2 if tg.cache_dtype == "f32" else 0) - (1 if rp.n_blocks == 0 else 0)) \
-        + (1 if rp.n_blocks > 0 else 0) + 7 * rp.n_blocks + 1 + 1
+    # front: gather (embeddings + chunk map), sigma fold, projection, the encoder's
+    # GEMMs (W_map with P_tok and F with P_b as two-product launches where d_c and
+    # d_b are whole 256-column tiles, else one launch each) and the two-term split
+    # of s|e (fp32 caches: the two-call path with its two bf16 conversions);
+    # forward: RoPE table, 7 kernels per block, final LayerNorm; head (with the pool
+    # head, the pool-row table first)
+    enc = (1 if rp.d_c % 256 == 0 else 2) + \
+        ((1 if rp.d_b % 256 == 0 else 2) if rp.n_blocks > 0 else 1)
+    launches_per_step = 1 + 2 + enc + 1 + (2 if tg.cache_dtype == "f32" else 0) \
+        + (1 if rp.n_blocks > 0 else 0) + 7 * rp.n_blocks + 1 + 1 + (1 if pooled else 0)
     launches_per_step += 1 if (args.mask == "block_diagonal" and rp.n_blocks > 0) else 0
     launches_per_step += 1 if (args.rope and args.component == "v") else 0
     cpu = None

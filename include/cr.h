@@ -216,7 +216,9 @@ cr_status cr_compress_features(const cr_target_dims* target, const cr_repairer_d
  * cache the segment projection reads its cache tiles straight from kv_pool
  * and writes each tile it reads into kv_out, so the assembly costs one read
  * and one write of the cache instead of two reads and a write; fp32 caches
- * take the two-call path.  The caller sizes kv_out, emb_out and the
+ * take the two-call path.  For a bf16 cache kv_out may be NULL: the assembled
+ * cache is then not written at all (cr_apply_residual_pool writes the repaired
+ * cache from the pool).  The caller sizes kv_out, emb_out and the
  * workspace (cr_workspace_bytes(.., max_tokens)) for max_tokens rows.
  * Errors: those of the two calls, checked before any launch.
  */
@@ -286,6 +288,31 @@ cr_status cr_apply_residual(const cr_target_dims* target, const cr_repairer_dims
                             void* kv_inout, const int32_t* pos, const float* inv_freq_host,
                             int32_t rope_mode, void* workspace, size_t workspace_bytes,
                             void* stream);
+
+/*
+ * cr_apply_residual_pool - cr_apply_residual for a bf16 cache whose stale rows
+ * are read from the chunk pool instead of an assembled cache (Sec. 4.1, KV
+ * residual output): for request token t at pool row src(t),
+ *   kv_out_t = round(kv_pool[src(t)] + sigma_delta * (W_out y_f,t + b_out))
+ * (with R_M on K for CR_ROPE_GLOBAL), the same values bit for bit as
+ * cr_assemble_stale followed by cr_apply_residual.  With cr_assemble_compress
+ * called without kv_out, the request's cache makes one read in the encoder and
+ * one read and one write here, instead of an extra write and read of an
+ * assembled copy.  The chunk arguments are those of that call (host arrays,
+ * the same checks) and must describe exactly n_tokens rows; kv_out [N, D_KV]
+ * receives every row.  workspace: the cr_workspace_bytes(.., >= n_tokens)
+ * workspace (its pool-row tables and, under CR_ROPE_GLOBAL, the R_M table are
+ * written).  Errors: CR_ERR_UNSUPPORTED for fp32 caches; otherwise as the two
+ * calls it replaces.
+ */
+cr_status cr_apply_residual_pool(const cr_target_dims* target, const cr_repairer_dims* rep,
+                                 const cr_weights* w, const uint16_t* yf, int64_t n_tokens,
+                                 const void* kv_pool, int64_t n_pool_tokens,
+                                 const int64_t* chunk_start, const int32_t* chunk_len,
+                                 int32_t n_pool_chunks, const int32_t* chunk_idx,
+                                 const int32_t* cu_chunks, int32_t n_req, void* kv_out,
+                                 const int32_t* pos, const float* inv_freq_host, int32_t rope_mode,
+                                 void* workspace, size_t workspace_bytes, void* stream);
 
 /*
  * cr_apply_residual_select - cr_apply_residual under an output choice of

@@ -26,7 +26,7 @@ EXPORTED = [
     "cr_workspace_bytes", "cr_assemble_stale", "cr_compress_features", "cr_assemble_compress",
     "cr_repair_forward",
     "cr_repair_forward_masked", "cr_apply_residual", "cr_apply_residual_select", "cr_rotate_k",
-    "cr_apply_residual_paged", "cr_canonicalize_chunks",
+    "cr_apply_residual_paged", "cr_apply_residual_pool", "cr_canonicalize_chunks",
     "cr_sigma_workspace_bytes", "cr_sigma_accumulate", "cr_sigma_finalize", "cr_get_device_status",
     "cr_clear_device_status", "cr_status_str", "cr_last_cuda_error",
     "cr_linear", "cr_matmul", "cr_layernorm", "cr_chunk_causal_attention", "cr_masked_attention",
@@ -108,6 +108,9 @@ def lib(build_if_missing: bool = False) -> ctypes.CDLL:
                                     vp, vp, vp, i32, vp, c_size_t, vp]),
         "cr_apply_residual_paged": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp,
                                           i64, vp, vp, vp, i32, vp, vp, i64, vp, c_size_t, vp]),
+        "cr_apply_residual_pool": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp, i64,
+                                         vp, i64, vp, vp, i32, vp, vp, i32, vp, vp, vp, i32, vp, c_size_t,
+                                         vp]),
         "cr_canonicalize_chunks": (i32, [P(cr_target_dims), vp, i64, vp, vp, vp]),
         "cr_rotate_k": (i32, [P(cr_target_dims), vp, i64, vp, vp, vp]),
         "cr_apply_residual_select": (i32, [P(cr_target_dims), P(cr_repairer_dims), P(cr_weights), vp,
@@ -239,7 +242,8 @@ def cr_compress_features(target, rep, weights: PackedWeights, kv, emb, n_tokens,
 def cr_assemble_compress(target, rep, weights: PackedWeights, kv_pool, emb_pool, chunk_start,
                          chunk_len, chunk_idx, cu_chunks, kv_out, emb_out, chunk_id, chunk_end, pos,
                          cu_seqlens_dev, h0_out, rein_out, workspace, stream=None):
-    """cr_assemble_stale + cr_compress_features in one call; returns (n_tokens, cu_seqlens_host)."""
+    """cr_assemble_stale + cr_compress_features in one call; returns (n_tokens, cu_seqlens_host).
+    kv_out None (bf16 caches): the assembled cache is not written (see cr_apply_residual_pool)."""
     cs = _host_arr(chunk_start, np.int64)
     cl = _host_arr(chunk_len, np.int32)
     ci = _host_arr(chunk_idx, np.int32)
@@ -249,7 +253,7 @@ def cr_assemble_compress(target, rep, weights: PackedWeights, kv_pool, emb_pool,
     st = lib().cr_assemble_compress(
         ctypes.byref(target), ctypes.byref(rep), ctypes.byref(weights.struct), _p(kv_pool),
         _p(emb_pool), kv_pool.shape[0], cs.ctypes.data, cl.ctypes.data, len(cl), ci.ctypes.data,
-        cu.ctypes.data, n_req, _p(kv_out), _p(emb_out), kv_out.shape[0], _p(chunk_id),
+        cu.ctypes.data, n_req, _p(kv_out), _p(emb_out), emb_out.shape[0], _p(chunk_id),
         _p(chunk_end), _p(pos), _p(cu_seqlens_dev), cu_host.ctypes.data, _p(h0_out), _p(rein_out),
         _p(workspace), workspace.numel() * workspace.element_size(), _stream(stream))
     _check("cr_assemble_compress", st)
@@ -297,6 +301,23 @@ def cr_apply_residual(target, rep, weights: PackedWeights, yf, n_tokens, kv_inou
         _p(kv_inout), _p(pos), None if f is None else f.ctypes.data, rope_mode, *_ws(workspace),
         _stream(stream))
     _check("cr_apply_residual", st)
+
+
+def cr_apply_residual_pool(target, rep, weights: PackedWeights, yf, n_tokens, kv_pool, chunk_start,
+                           chunk_len, chunk_idx, cu_chunks, kv_out, pos, inv_freq_host=None,
+                           rope_mode=CR_ROPE_NONE, workspace=None, stream=None):
+    """The head with the stale rows read from the pool, the repaired rows written to kv_out."""
+    cs = _host_arr(chunk_start, np.int64)
+    cl = _host_arr(chunk_len, np.int32)
+    ci = _host_arr(chunk_idx, np.int32)
+    cu = _host_arr(cu_chunks, np.int32)
+    f = None if inv_freq_host is None else _host_arr(inv_freq_host, np.float32)
+    st = lib().cr_apply_residual_pool(
+        ctypes.byref(target), ctypes.byref(rep), ctypes.byref(weights.struct), _p(yf), n_tokens,
+        _p(kv_pool), kv_pool.shape[0], cs.ctypes.data, cl.ctypes.data, len(cl), ci.ctypes.data,
+        cu.ctypes.data, len(cu) - 1, _p(kv_out), _p(pos), None if f is None else f.ctypes.data,
+        rope_mode, *_ws(workspace), _stream(stream))
+    _check("cr_apply_residual_pool", st)
 
 
 CR_APPLY_K, CR_APPLY_V, CR_APPLY_KV = 1, 2, 3

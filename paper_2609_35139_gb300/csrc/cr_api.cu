@@ -88,7 +88,7 @@ cr_status check_repairer(const cr_repairer_dims* r) {
 }
 
 struct WsLayout {
-    size_t wfold, kvb, embb, y, se32, se2, x, u, qkv, o, g, rope, kstart, total;
+    size_t wfold, kvb, embb, y, se32, se2, x, u, qkv, o, g, rope, kstart, srcrow, boxsrc, total;
 };
 
 WsLayout ws_layout(const Dims& d, int64_t n) {
@@ -113,6 +113,8 @@ WsLayout ws_layout(const Dims& d, int64_t n) {
     w.g = take(N * d.hid * 2);
     w.rope = take(N * (d.hd / 2) * 8);   // repairer RoPE (cos, sin) per token and pair
     w.kstart = take(N * 4);              // chunk start per token (block-diagonal mask)
+    w.srcrow = take(N * 8);              // pool row per token (cr_apply_residual_pool)
+    w.boxsrc = take((N / 128 + 2) * 8);  // pool row per contiguous 128-row box, or -1
     w.total = off;
     return w;
 }
@@ -131,6 +133,12 @@ bool all_aligned() { return true; }
 template <typename P, typename... R>
 bool all_aligned(const P* p, R... rest) {
     return p != nullptr && aligned16(p) && all_aligned(rest...);
+}
+// the same for optional buffers: NULL passes
+bool aligned_or_null() { return true; }
+template <typename P, typename... R>
+bool aligned_or_null(const P* p, R... rest) {
+    return (p == nullptr || aligned16(p)) && aligned_or_null(rest...);
 }
 
 }  // namespace
@@ -256,7 +264,8 @@ static cr_status build_gather(const Dims& d, const void* kv_pool, const void* em
     if (!chunk_start || !chunk_len || !chunk_idx || !cu_chunks) return CR_ERR_INVALID_ARG;
     if (n_req < 1 || n_req > kMaxReq || n_pool_chunks < 1 || n_pool_tokens < 1)
         return CR_ERR_INVALID_ARG;
-    if (!all_aligned(kv_pool, emb_pool, kv_out, emb_out, chunk_id, chunk_end, pos, cu_seqlens_dev))
+    // (the callers say which of the outputs they need)
+    if (!all_aligned(kv_pool) || !aligned_or_null(emb_pool, kv_out, emb_out, chunk_id, chunk_end, pos, cu_seqlens_dev))
         return CR_ERR_INVALID_ARG;
     if (cu_chunks[0] != 0) return CR_ERR_INVALID_ARG;
     const int64_t es = d.f32 ? 4 : 2;
@@ -315,6 +324,8 @@ cr_status cr_assemble_stale(const cr_target_dims* target, const void* kv_pool,
     cr_status s = check_target(target);
     if (s != CR_OK) return s;
     if (!cu_seqlens_host) return CR_ERR_INVALID_ARG;
+    if (!all_aligned(emb_pool, kv_out, emb_out, chunk_id, chunk_end, pos, cu_seqlens_dev))
+        return CR_ERR_INVALID_ARG;
     const Dims d = dims_of(target, nullptr);
     GatherParams* p = new GatherParams();   // ~17 KB: keep it off the caller's stack
     s = build_gather(d, kv_pool, emb_pool, n_pool_tokens, chunk_start, chunk_len, n_pool_chunks,
@@ -458,12 +469,16 @@ cr_status cr_assemble_compress(const cr_target_dims* target, const cr_repairer_d
                                  workspace_bytes, &d, &L);
     if (s != CR_OK) return s;
     if (!cu_seqlens_host) return CR_ERR_INVALID_ARG;
+    if (!all_aligned(emb_pool, emb_out, chunk_id, chunk_end, pos, cu_seqlens_dev)) return CR_ERR_INVALID_ARG;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     GatherParams* p = new GatherParams();
     s = build_gather(d, kv_pool, emb_pool, n_pool_tokens, chunk_start, chunk_len, n_pool_chunks,
                      chunk_idx, cu_chunks, n_req, kv_out, emb_out, max_tokens, chunk_id, chunk_end,
                      pos, cu_seqlens_dev, p);
     const int64_t N = p->n_tokens;
+    // without kv_out (the repaired cache is written from the pool by
+    // cr_apply_residual_pool) only the bf16 path applies
+    if (s == CR_OK && !kv_out && (d.f32 || n_pool_tokens > INT32_MAX)) s = CR_ERR_UNSUPPORTED;
     if (s == CR_OK && (d.f32 || n_pool_tokens > INT32_MAX)) {
         // fp32 caches go through the bf16 conversion of the two-call form
         for (int r = 0; r <= n_req; ++r) cu_seqlens_host[r] = p->cu_seqlens_host[r];
@@ -738,6 +753,63 @@ cr_status cr_apply_residual_select(const cr_target_dims* target, const cr_repair
                                 static_cast<int>(d.H), static_cast<int>(d.dh), inv_freq_host, st,
                                 -1.0f);
     return s;
+}
+
+cr_status cr_apply_residual_pool(const cr_target_dims* target, const cr_repairer_dims* rep,
+                                 const cr_weights* w, const uint16_t* yf, int64_t n_tokens,
+                                 const void* kv_pool, int64_t n_pool_tokens,
+                                 const int64_t* chunk_start, const int32_t* chunk_len,
+                                 int32_t n_pool_chunks, const int32_t* chunk_idx,
+                                 const int32_t* cu_chunks, int32_t n_req, void* kv_out,
+                                 const int32_t* pos, const float* inv_freq_host, int32_t rope_mode,
+                                 void* workspace, size_t workspace_bytes, void* stream) {
+    cr_status s = check_target(target);
+    if (s == CR_OK) s = check_repairer(rep);
+    if (s != CR_OK) return s;
+    const Dims d = dims_of(target, rep);
+    if (d.f32) return CR_ERR_UNSUPPORTED;   // bf16 caches (the fused front's path)
+    if (!w || !kv_pool || !kv_out || !workspace || n_tokens < 1 || n_tokens > INT32_MAX / 2 ||
+        n_pool_tokens < 1 || n_pool_tokens > INT32_MAX)
+        return CR_ERR_INVALID_ARG;
+    if (rope_mode != CR_ROPE_NONE && rope_mode != CR_ROPE_GLOBAL) return CR_ERR_INVALID_ARG;
+    if (rope_mode == CR_ROPE_GLOBAL && !inv_freq_host) return CR_ERR_INVALID_ARG;
+    if (!all_aligned(yf, kv_pool, kv_out, pos, workspace, w->w_out, w->b_out, w->sigma_delta))
+        return CR_ERR_INVALID_ARG;
+    if (d.D % 256 != 0) return CR_ERR_UNSUPPORTED;
+    const WsLayout L = ws_layout(d, n_tokens);
+    if (workspace_bytes < L.total) return CR_ERR_INVALID_ARG;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    GatherParams* gpl = new GatherParams();
+    s = build_gather(d, kv_pool, nullptr, n_pool_tokens, chunk_start, chunk_len, n_pool_chunks, chunk_idx,
+                     cu_chunks, n_req, nullptr, nullptr, n_tokens, nullptr, nullptr, nullptr, nullptr, gpl);
+    if (s == CR_OK && gpl->n_tokens != n_tokens) s = CR_ERR_INVALID_ARG;
+    int64_t* src_row = at<int64_t>(workspace, L.srcrow);
+    int64_t* box_src = at<int64_t>(workspace, L.boxsrc);
+    if (s == CR_OK) s = launch_src_rows(*gpl, src_row, box_src, st);
+    unsigned* status = gpl->status;
+    delete gpl;
+    if (s != CR_OK) return s;
+    GemmParams gp{};
+    gp.status = status;
+    gp.bias = w->b_out;
+    gp.sigma = w->sigma_delta;
+    gp.pos = pos;
+    gp.rope_dim = static_cast<int32_t>(d.dh);
+    gp.rope_on = rope_mode == CR_ROPE_GLOBAL ? 1 : 0;
+    gp.n_kv_heads = static_cast<int32_t>(d.H);
+    if (gp.rope_on) {
+        for (int i = 0; i < d.dh / 2; ++i) gp.inv_freq[i] = inv_freq_host[i];
+        // (the R_M table sits at the front of the workspace, clear of the row tables)
+        if ((s = target_rope_table(d, pos, n_tokens, inv_freq_host, workspace, workspace_bytes, &gp, st)) != CR_OK)
+            return s;
+    }
+    gp.kv_pool = static_cast<const uint16_t*>(kv_pool);
+    gp.src_row = src_row;
+    gp.box_src = box_src;
+    if (!make_tmap_2d(&gp.tm_pool, kv_pool, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d.D, n_pool_tokens, d.D * 2, 64,
+                      128, CU_TENSOR_MAP_SWIZZLE_128B))
+        return CR_ERR_INVALID_ARG;
+    return launch_gemm(yf, d.db, w->w_out, n_tokens, d.D, d.db, EPI_KV_POOL, gp, kv_out, d.D, st);
 }
 
 cr_status cr_rotate_k(const cr_target_dims* target, void* kv_inout, int64_t n_tokens,

@@ -57,7 +57,11 @@ static_assert(kGemmRegsCtl * 128 + 2 * kGemmRegsEpi * 128 <= kGemmRegsLaunch * k
 template <int BN, int EPI, int CG>
 struct GemmCfg {
     static constexpr bool kKV =
-        (EPI == EPI_KV_BF16 || EPI == EPI_KV_F32 || EPI == EPI_KV_PAGED || EPI == EPI_KV_LOSS);
+        (EPI == EPI_KV_BF16 || EPI == EPI_KV_F32 || EPI == EPI_KV_PAGED || EPI == EPI_KV_LOSS ||
+         EPI == EPI_KV_POOL);
+    // the stale tile comes from the chunk pool (a TMA box where a box's rows are one
+    // contiguous pool range, else row by row), the repaired tile goes to the output
+    static constexpr bool kPoolSrc = (EPI == EPI_KV_POOL);
     // the stale tile is staged as for the in-place update, but the repaired rows
     // go straight from registers to the paged target cache (no TMA store)
     static constexpr bool kPaged = (EPI == EPI_KV_PAGED);
@@ -538,15 +542,40 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     // box by box, each as soon as the previous tile's copy of it has
                     // been stored; box 0 also brings this tile's vectors (buffer i & 1)
                     float* vdst = vec + (i & 1) * (Cfg::kVecBytes / 4);
+                    // pool source: this CTA's 128 rows as one pool box, or -1
+                    const int64_t bsrc = (Cfg::kPoolSrc && load_tile && m0 < p.M) ? p.box_src[m0 / BM] : -1;
                     for (int b = 0; b < Cfg::kBoxes; ++b) {
                         if (!(ok = mbar_wait_warp(&epi_empty[b], (static_cast<uint32_t>(i) & 1u) ^ 1u, wc, 101)))
                             break;
-                        uint32_t bytes = load_tile ? (Cfg::kLoss ? 32768u : 16384u) : 0u;
+                        bool tma_tile = load_tile;
+                        if constexpr (Cfg::kPoolSrc) {
+                            tma_tile = load_tile && bsrc >= 0;
+                            if (load_tile && bsrc < 0) {
+                                // rows from several pool ranges (or past the last row):
+                                // the warp copies them, each 16-byte chunk c of row r to
+                                // r * 128 + ((c ^ (r & 7)) << 4), as TMA would place it
+                                uint8_t* dstb = tile + b * 16384;
+                                const int col0 = n0 + b * Cfg::kBoxCols;
+                                for (int e = static_cast<int>(lane); e < BM * 8; e += 32) {
+                                    const int rr = e >> 3, c = e & 7;
+                                    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+                                    if (m0 + rr < p.M)
+                                        v = __ldg(reinterpret_cast<const uint4*>(
+                                            p.kv_pool + p.src_row[m0 + rr] * p.N + col0 + c * 8));
+                                    *reinterpret_cast<uint4*>(dstb + rr * 128 + ((c ^ (rr & 7)) << 4)) = v;
+                                }
+                                __syncwarp();
+                            }
+                        }
+                        uint32_t bytes = tma_tile ? (Cfg::kLoss ? 32768u : 16384u) : 0u;
                         if (b == 0) bytes += (has_bias ? vbytes : 0u) + (Cfg::kKV ? vbytes : 0u);
                         if (elect_one()) {
                             if (bytes) mbar_expect_tx(&epi_full[b], bytes);
                             else mbar_arrive(&epi_full[b]);
-                            if (load_tile) {
+                            if (Cfg::kPoolSrc && tma_tile) {
+                                tma_load_2d(tile + b * 16384, &p.tm_pool, &epi_full[b], n0 + b * Cfg::kBoxCols,
+                                            static_cast<int>(bsrc));
+                            } else if (tma_tile) {
                                 if constexpr (Cfg::kLoss) {
                                     tma_load_2d(tile + 2 * b * 16384, &tmC, &epi_full[b], n0 + b * Cfg::kBoxCols, m0);
                                     tma_load_2d(tile + (2 * b + 1) * 16384, &p.tm_joint, &epi_full[b],
@@ -1091,7 +1120,8 @@ constexpr int kCG = 2;
 cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t M, int64_t N,
                       int64_t K, int epi, GemmParams p, void* kv_base, int64_t ld_kv,
                       cudaStream_t st, const uint16_t* A_lo) {
-    const bool kv = (epi == EPI_KV_BF16 || epi == EPI_KV_F32 || epi == EPI_KV_PAGED || epi == EPI_KV_LOSS);
+    const bool kv = (epi == EPI_KV_BF16 || epi == EPI_KV_F32 || epi == EPI_KV_PAGED || epi == EPI_KV_LOSS ||
+                     epi == EPI_KV_POOL);
     const bool f32_tile = (epi == EPI_KV_F32 || epi == EPI_ADD_F32);
     // Tile width.  Per 64-deep k-block a CTA of a pair moves 32 KB + 128 BN
     // bytes through shared memory (TMA writes and MMA operand reads of its A
@@ -1200,6 +1230,9 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
         case EPI_KV_PAGED:
             if (p.seg_width <= 0 || p.seg_width % 256 != 0 || p.num_slots < 1) return CR_ERR_UNSUPPORTED;
             return launch_bn<256, EPI_KV_PAGED, kCG>(ta, tb, tc, p, st);
+        case EPI_KV_POOL:
+            if (!p.kv_pool || !p.src_row || !p.box_src) return CR_ERR_INVALID_ARG;
+            return launch_bn<256, EPI_KV_POOL, kCG>(ta, tb, tc, p, st);
         default:
             return CR_ERR_INVALID_ARG;
     }

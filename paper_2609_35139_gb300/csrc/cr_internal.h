@@ -55,9 +55,11 @@ enum GemmEpi : int {
     EPI_KV_F32 = 6,     // same for an fp32 cache
     EPI_KV_PAGED = 7,   // bf16 cache: stale tile read token-major, repaired rows written
                         // to a paged, layer-major target cache through a slot mapping
-    EPI_KV_LOSS = 8     // training head: r = z + b - (joint - stale) / sigma from the staged
+    EPI_KV_LOSS = 8,    // training head: r = z + b - (joint - stale) / sigma from the staged
                         // bf16 stale and joint tiles; writes dz = row_scale[t] r (bf16)
                         // and per-row partial sums of r^2 instead of storing r
+    EPI_KV_POOL = 9     // EPI_KV_BF16 with the stale tile read from the chunk pool (rows
+                        // src_row[t]) and the repaired rows stored into the output cache
 };
 
 // Operand layouts of the GEMM: K-major A and W (the forward), K-major A with
@@ -125,10 +127,18 @@ struct GemmParams {
     int32_t K2;
     int32_t split_kb2;
     const float* bias2;
+    // EPI_KV_POOL: the stale cache rows come from the pool (bf16 [n_pool, N], row
+    // stride N): box_src[b] the pool row of the first of request rows 128 b ..
+    // 128 b + 127 when they are one contiguous pool range (loaded by TMA through
+    // tm_pool), else -1 (each row from src_row[t])
+    const uint16_t* kv_pool;
+    const int64_t* src_row;
+    const int64_t* box_src;
     float inv_freq[64];      // RoPE frequencies, rope_dim / 2 entries
     CUtensorMap tm_joint;    // EPI_KV_LOSS (set by launch_gemm; the type carries its alignment)
     CUtensorMap tm_alo;      // two-term A: the A_lo operand
     CUtensorMap tm_a2, tm_alo2, tm_b2, tm_c2;   // the second product (n_split > 0)
+    CUtensorMap tm_pool;                         // EPI_KV_POOL: the chunk pool
 };
 
 // One product of launch_gemm_pair: C[M, N] = A[M, K] W[N, K]^T + bias (fp32 out),
@@ -263,6 +273,9 @@ constexpr int64_t kSigmaSlice = 64;
 
 // Launchers (validated arguments).
 cr_status launch_gather(const GatherParams& p, cudaStream_t st);
+// the pool row of each request token, and per 128-row box its first token's
+// pool row when the box is one contiguous pool range (else -1)
+cr_status launch_src_rows(const GatherParams& p, int64_t* src_row, int64_t* box_src, cudaStream_t st);
 // K segments rotated in place by R_M(dir * (-pos)): dir = +1 canonicalises
 // (R_M(q)^{-1}), dir = -1 applies R_M(p).
 cr_status launch_canonicalize(void* kv, bool f32, int64_t n, const int32_t* pos, int L, int H, int dh,

@@ -278,6 +278,55 @@ cr_status launch_rope_table(const int32_t* pos, int64_t n, int half_dim, const f
                       half_dim, f, table);
 }
 
+// The pool row of every request token (the gather's segment table), and per
+// 128-row box of the request the pool row of its first token when all 128 rows
+// lie in one chunk (a contiguous pool range), else -1.
+__global__ void __launch_bounds__(256) src_rows_kernel(const __grid_constant__ GatherParams p,
+                                                       int64_t* __restrict__ src_row,
+                                                       int64_t* __restrict__ box_src) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int64_t n_box = (p.n_tokens + 127) / 128;
+    const int64_t n = p.n_tokens > n_box ? p.n_tokens : n_box;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        auto seg_of = [&](int64_t t) {
+            int lo = 0, hi = p.n_seg - 1;
+            while (lo < hi) {
+                const int mid = (lo + hi + 1) >> 1;
+                if (p.seg[mid].dst_row <= t)
+                    lo = mid;
+                else
+                    hi = mid - 1;
+            }
+            return lo;
+        };
+        if (i < p.n_tokens) {
+            const GatherSeg& sg = p.seg[seg_of(i)];
+            const int64_t off = i - sg.dst_row;
+            if (off < 0 || off >= sg.len || sg.src_row + off >= p.n_pool_tokens) {
+                report(p.status, CR_DEV_INDEX, 3);
+                src_row[i] = 0;
+            } else {
+                src_row[i] = sg.src_row + off;
+            }
+        }
+        if (i < n_box) {
+            const int64_t t0 = 128 * i, t1 = t0 + 127;
+            const GatherSeg& sg = p.seg[seg_of(t0)];
+            const bool one = t1 < p.n_tokens && t1 < sg.dst_row + sg.len && t0 >= sg.dst_row;
+            box_src[i] = one ? sg.src_row + (t0 - sg.dst_row) : -1;
+        }
+    }
+}
+
+cr_status launch_src_rows(const GatherParams& p, int64_t* src_row, int64_t* box_src, cudaStream_t st) {
+    if (p.n_tokens <= 0) return CR_OK;
+    const int64_t grid = (p.n_tokens + 255) / 256;
+    return launch_pdl(src_rows_kernel, dim3(static_cast<unsigned>(grid)), dim3(256), 0, st, p, src_row,
+                      box_src);
+}
+
 cr_status launch_gather(const GatherParams& p, cudaStream_t st) {
     if (p.n_tokens <= 0) return CR_OK;
     if (p.kv_row_bytes == 0) {

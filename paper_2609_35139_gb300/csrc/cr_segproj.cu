@@ -253,7 +253,11 @@ __global__ void __launch_bounds__(224, 1)
                     if (!(ok = mbar_wait_warp(&full[stage], phase, wc, 114))) break;
                     const uint8_t* sa = smem + stage * Cfg::kStageBytes;
                     const int col = (s0 + g) * DH;
-                    if (tr.rows == 128) {
+                    if (!p.kv_out) {
+                        // no assembled cache asked for: the projection alone reads the stage
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&empty[stage]);
+                    } else if (tr.rows == 128) {
                         if (lane == 0) {
                             fence_async_smem();
 #pragma unroll
@@ -435,8 +439,10 @@ cr_status launch_segproj_pool(const uint16_t* kv_pool, int64_t n_pool_tokens, ui
                       2 * static_cast<uint64_t>(p.S) * p.d_seg, head_dim * 2, 64, SP_N,
                       CU_TENSOR_MAP_SWIZZLE_128B))
         return CR_ERR_INVALID_ARG;
-    if (!make_tmap_2d(&to, kv_out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dkv, p.M, dkv * 2, 64, 128,
-                      CU_TENSOR_MAP_SWIZZLE_128B))
+    // without an assembled cache the output map is never used (the pool's stands in)
+    if (!make_tmap_2d(&to, kv_out ? static_cast<const void*>(kv_out) : kv_pool, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                      dkv, kv_out ? static_cast<uint64_t>(p.M) : static_cast<uint64_t>(n_pool_tokens), dkv * 2,
+                      64, 128, CU_TENSOR_MAP_SWIZZLE_128B))
         return CR_ERR_INVALID_ARG;
     return head_dim == 128 ? launch_dh<128, true>(tk, tw, to, p, tiles, st)
                            : launch_dh<64, true>(tk, tw, to, p, tiles, st);

@@ -64,13 +64,15 @@ class RepairSession:
                                 self.h0, self.rein, self.workspace, stream)
 
     def assemble_compress(self, kv_pool: torch.Tensor, emb_pool: torch.Tensor, chunk_start,
-                          chunk_len, chunk_idx, cu_chunks, stream=None) -> Assembled:
+                          chunk_len, chunk_idx, cu_chunks, stream=None, write_kv=True) -> Assembled:
         """assemble + compress as one call: the segment projection reads the pool and
-        writes the assembled cache as it goes (same results, one cache read fewer)."""
+        writes the assembled cache as it goes (same results, one cache read fewer);
+        write_kv=False (bf16 caches) leaves kv unwritten, for apply_pool."""
         n, cu = cr.cr_assemble_compress(self.target, self.rep, self.weights, kv_pool, emb_pool,
-                                        chunk_start, chunk_len, chunk_idx, cu_chunks, self.kv,
-                                        self.emb, self.chunk_id, self.chunk_end, self.pos,
-                                        self.cu_seqlens, self.h0, self.rein, self.workspace, stream)
+                                        chunk_start, chunk_len, chunk_idx, cu_chunks,
+                                        self.kv if write_kv else None, self.emb, self.chunk_id,
+                                        self.chunk_end, self.pos, self.cu_seqlens, self.h0,
+                                        self.rein, self.workspace, stream)
         return Assembled(n, cu)
 
     def forward(self, a: Assembled, stream=None, mask_mode="block_causal"):
@@ -100,6 +102,14 @@ class RepairSession:
                                         offset, self.chunk_id if keep_first_chunk else None,
                                         workspace=self.workspace, stream=stream)
 
+    def apply_pool(self, a: Assembled, kv_pool: torch.Tensor, chunk_start, chunk_len, chunk_idx,
+                   cu_chunks, inv_freq_target=None, rope_mode=cr.CR_ROPE_NONE, stream=None):
+        """Head and residual add with the stale rows read from the pool (the chunk map of
+        the assemble call) and the repaired rows written to kv (bf16 caches)."""
+        cr.cr_apply_residual_pool(self.target, self.rep, self.weights, self.yf, a.n_tokens, kv_pool,
+                                  chunk_start, chunk_len, chunk_idx, cu_chunks, self.kv, self.pos,
+                                  inv_freq_target, rope_mode, workspace=self.workspace, stream=stream)
+
     def stale_kv(self, a: Assembled, inv_freq_target, stream=None):
         """The stale cache of independent reuse: the assembled canonical cache with K
         rotated to its request positions (no repair), in place on kv."""
@@ -118,12 +128,21 @@ class RepairSession:
                mask_mode="block_causal", component="kv", offset="stale",
                keep_first_chunk=False) -> Assembled:
         """Assemble, compress, run the blocks and apply the residual; kv holds the result.
-        The keyword options select the App. F mask and output variants (defaults: the method)."""
+        The keyword options select the App. F mask and output variants (defaults: the method).
+        For a bf16 cache under the method's output the stale rows never go through kv: the
+        encoder and the head read them from the pool (the same results, one write and one read
+        of the cache fewer)."""
+        pooled = (self.target.cache_dtype == cr.CR_BF16 and component == "kv" and offset == "stale"
+                  and not keep_first_chunk)
         a = self.assemble_compress(kv_pool, emb_pool, chunk_start, chunk_len, chunk_idx, cu_chunks,
-                                   stream)
+                                   stream, write_kv=not pooled)
         self.forward(a, stream, mask_mode=mask_mode)
-        self.apply(a, inv_freq_target, rope_mode, stream, component=component, offset=offset,
-                   keep_first_chunk=keep_first_chunk)
+        if pooled:
+            self.apply_pool(a, kv_pool, chunk_start, chunk_len, chunk_idx, cu_chunks, inv_freq_target,
+                            rope_mode, stream)
+        else:
+            self.apply(a, inv_freq_target, rope_mode, stream, component=component, offset=offset,
+                       keep_first_chunk=keep_first_chunk)
         return a
 
 

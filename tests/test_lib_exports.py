@@ -62,9 +62,9 @@ def test_workspace_bytes_host_logic(L):
     assert 0 < w1 < w2
     # dominated by per-token buffers: y (two bf16 terms), s|e (fp32, then two bf16
     # terms), x (fp32), u, qkv, o, g (bf16), the repairer RoPE table (32 (cos, sin)
-    # pairs per token) and the chunk start (int32)
+    # pairs per token), the chunk start (int32) and the pool row (int64)
     per_tok = (2 * 512 * 16 * 2 + 2 * 512 * 4 + 4 * 512 * 2 + 1024 * 4 + 1024 * 2 + 3 * 1024 * 2
-               + 1024 * 2 + 4096 * 2 + 32 * 8 + 4)
+               + 1024 * 2 + 4096 * 2 + 32 * 8 + 4 + 8)
     assert abs((w2 - w1) - 5119 * per_tok) < 64 * 256
     bad = cr.repairer_dims(16, 512, 1000, 6, 16, 4096)   # d_b not a multiple of 128
     assert cr.cr_workspace_bytes(t, bad, 10) == 0
