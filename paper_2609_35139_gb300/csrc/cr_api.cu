@@ -88,7 +88,7 @@ cr_status check_repairer(const cr_repairer_dims* r) {
 }
 
 struct WsLayout {
-    size_t wfold, kvb, embb, y, se32, se2, x, u, qkv, o, g, rope, kstart, srcrow, boxsrc, total;
+    size_t wfold, kvb, embb, y, se32, se2, x, u, qkv, o, g, rope, kstart, srcrow, boxsrc, grpsrc, total;
 };
 
 WsLayout ws_layout(const Dims& d, int64_t n) {
@@ -115,6 +115,7 @@ WsLayout ws_layout(const Dims& d, int64_t n) {
     w.kstart = take(N * 4);              // chunk start per token (block-diagonal mask)
     w.srcrow = take(N * 8);              // pool row per token (cr_apply_residual_pool)
     w.boxsrc = take((N / 128 + 2) * 8);  // pool row per contiguous 128-row box, or -1
+    w.grpsrc = take((N / 128 + 2) * 128);  // pool row per contiguous 8-row group, or -1
     w.total = off;
     return w;
 }
@@ -785,7 +786,8 @@ cr_status cr_apply_residual_pool(const cr_target_dims* target, const cr_repairer
     if (s == CR_OK && gpl->n_tokens != n_tokens) s = CR_ERR_INVALID_ARG;
     int64_t* src_row = at<int64_t>(workspace, L.srcrow);
     int64_t* box_src = at<int64_t>(workspace, L.boxsrc);
-    if (s == CR_OK) s = launch_src_rows(*gpl, src_row, box_src, st);
+    int64_t* grp_src = at<int64_t>(workspace, L.grpsrc);
+    if (s == CR_OK) s = launch_src_rows(*gpl, src_row, box_src, grp_src, st);
     unsigned* status = gpl->status;
     delete gpl;
     if (s != CR_OK) return s;
@@ -806,8 +808,11 @@ cr_status cr_apply_residual_pool(const cr_target_dims* target, const cr_repairer
     gp.kv_pool = static_cast<const uint16_t*>(kv_pool);
     gp.src_row = src_row;
     gp.box_src = box_src;
+    gp.grp_src = grp_src;
     if (!make_tmap_2d(&gp.tm_pool, kv_pool, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d.D, n_pool_tokens, d.D * 2, 64,
-                      128, CU_TENSOR_MAP_SWIZZLE_128B))
+                      128, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_tmap_2d(&gp.tm_pool8, kv_pool, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, d.D, n_pool_tokens, d.D * 2, 64,
+                      8, CU_TENSOR_MAP_SWIZZLE_128B))
         return CR_ERR_INVALID_ARG;
     return launch_gemm(yf, d.db, w->w_out, n_tokens, d.D, d.db, EPI_KV_POOL, gp, kv_out, d.D, st);
 }

@@ -542,33 +542,72 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     // box by box, each as soon as the previous tile's copy of it has
                     // been stored; box 0 also brings this tile's vectors (buffer i & 1)
                     float* vdst = vec + (i & 1) * (Cfg::kVecBytes / 4);
-                    // pool source: this CTA's 128 rows as one pool box, or -1
+                    // pool source: this CTA's 128 rows as one pool box, or -1; then
+                    // lane g < 16 holds the pool row of the tile's 8-row group g, or -1
                     const int64_t bsrc = (Cfg::kPoolSrc && load_tile && m0 < p.M) ? p.box_src[m0 / BM] : -1;
+                    const bool straddle = Cfg::kPoolSrc && load_tile && bsrc < 0;
+                    int64_t gsrc = -1;
+                    uint32_t good = 0;   // groups loaded by TMA (8-row boxes)
+                    int hg = -1;         // first group the warp copies, its rows' pool rows below
+                    int64_t hs0 = -1, hs1 = -1;
+                    if (straddle) {
+                        if (lane < 16 && m0 < p.M) gsrc = p.grp_src[m0 / 8 + static_cast<int>(lane)];
+                        good = __ballot_sync(0xffffffffu, gsrc >= 0) & 0xFFFFu;
+                        if (good != 0xFFFFu) {
+                            hg = __ffs(static_cast<int>(~good & 0xFFFFu)) - 1;
+                            const int r0 = 8 * hg + (static_cast<int>(lane) >> 3);
+                            if (m0 + r0 < p.M) hs0 = p.src_row[m0 + r0];
+                            if (m0 + r0 + 4 < p.M) hs1 = p.src_row[m0 + r0 + 4];
+                        }
+                    }
                     for (int b = 0; b < Cfg::kBoxes; ++b) {
                         if (!(ok = mbar_wait_warp(&epi_empty[b], (static_cast<uint32_t>(i) & 1u) ^ 1u, wc, 101)))
                             break;
-                        bool tma_tile = load_tile;
-                        if constexpr (Cfg::kPoolSrc) {
-                            tma_tile = load_tile && bsrc >= 0;
-                            if (load_tile && bsrc < 0) {
-                                // rows from several pool ranges (or past the last row):
-                                // the warp copies them, each 16-byte chunk c of row r to
-                                // r * 128 + ((c ^ (r & 7)) << 4), as TMA would place it
-                                uint8_t* dstb = tile + b * 16384;
-                                const int col0 = n0 + b * Cfg::kBoxCols;
-                                for (int e = static_cast<int>(lane); e < BM * 8; e += 32) {
-                                    const int rr = e >> 3, c = e & 7;
-                                    uint4 v = make_uint4(0u, 0u, 0u, 0u);
-                                    if (m0 + rr < p.M)
-                                        v = __ldg(reinterpret_cast<const uint4*>(
-                                            p.kv_pool + p.src_row[m0 + rr] * p.N + col0 + c * 8));
-                                    *reinterpret_cast<uint4*>(dstb + rr * 128 + ((c ^ (rr & 7)) << 4)) = v;
+                        const uint32_t vb = b == 0 ? (has_bias ? vbytes : 0u) + (Cfg::kKV ? vbytes : 0u) : 0u;
+                        if (straddle) {
+                            // a tile across chunk boundaries: its contiguous 8-row groups
+                            // by TMA, the others copied by the warp, then one arrival
+                            const uint32_t bytes = static_cast<uint32_t>(__popc(good)) * 1024u + vb;
+                            if (elect_one()) {
+                                if (bytes) mbar_add_tx(&epi_full[b], bytes);
+                                if (b == 0) {
+                                    if (has_bias) bulk_load(vdst, p.bias + n0, vbytes, &epi_full[0]);
+                                    if constexpr (Cfg::kKV) bulk_load(vdst + BN, p.sigma + n0, vbytes, &epi_full[0]);
                                 }
-                                __syncwarp();
                             }
+                            __syncwarp();
+                            uint8_t* dstb = tile + b * 16384;
+                            const int col0 = n0 + b * Cfg::kBoxCols;
+                            for (int g = 0; g < 16; ++g) {
+                                const int64_t s = __shfl_sync(0xffffffffu, gsrc, g);
+                                if (s >= 0 && lane == 0)
+                                    tma_load_2d(dstb + g * 1024, &p.tm_pool8, &epi_full[b], col0, static_cast<int>(s));
+                            }
+                            // each 16-byte chunk c of row r to r * 128 + ((c ^ (r & 7)) << 4),
+                            // where TMA places it, by asynchronous copies that the barrier
+                            // waits for; rows past the request are zero-filled
+                            for (uint32_t bad = ~good & 0xFFFFu; bad; bad &= bad - 1) {
+                                const int g = __ffs(static_cast<int>(bad)) - 1;
+                                const int c = static_cast<int>(lane) & 7;
+                                const int r0 = 8 * g + (static_cast<int>(lane) >> 3), r1 = r0 + 4;
+                                int64_t s0 = hs0, s1 = hs1;
+                                if (g != hg) {
+                                    s0 = m0 + r0 < p.M ? p.src_row[m0 + r0] : -1;
+                                    s1 = m0 + r1 < p.M ? p.src_row[m0 + r1] : -1;
+                                }
+                                cp_async16(dstb + r0 * 128 + ((c ^ (r0 & 7)) << 4),
+                                           p.kv_pool + (s0 >= 0 ? s0 : 0) * p.N + col0 + c * 8, s0 >= 0 ? 16u : 0u);
+                                cp_async16(dstb + r1 * 128 + ((c ^ (r1 & 7)) << 4),
+                                           p.kv_pool + (s1 >= 0 ? s1 : 0) * p.N + col0 + c * 8, s1 >= 0 ? 16u : 0u);
+                            }
+                            if (good != 0xFFFFu) cp_async_mbar_arrive(&epi_full[b]);
+                            __syncwarp();
+                            if (elect_one()) mbar_arrive(&epi_full[b]);
+                            __syncwarp();
+                            continue;
                         }
-                        uint32_t bytes = tma_tile ? (Cfg::kLoss ? 32768u : 16384u) : 0u;
-                        if (b == 0) bytes += (has_bias ? vbytes : 0u) + (Cfg::kKV ? vbytes : 0u);
+                        const bool tma_tile = load_tile;
+                        uint32_t bytes = (tma_tile ? (Cfg::kLoss ? 32768u : 16384u) : 0u) + vb;
                         if (elect_one()) {
                             if (bytes) mbar_expect_tx(&epi_full[b], bytes);
                             else mbar_arrive(&epi_full[b]);
@@ -1231,7 +1270,7 @@ cr_status launch_gemm(const uint16_t* A, int64_t lda, const uint16_t* W, int64_t
             if (p.seg_width <= 0 || p.seg_width % 256 != 0 || p.num_slots < 1) return CR_ERR_UNSUPPORTED;
             return launch_bn<256, EPI_KV_PAGED, kCG>(ta, tb, tc, p, st);
         case EPI_KV_POOL:
-            if (!p.kv_pool || !p.src_row || !p.box_src) return CR_ERR_INVALID_ARG;
+            if (!p.kv_pool || !p.src_row || !p.box_src || !p.grp_src) return CR_ERR_INVALID_ARG;
             return launch_bn<256, EPI_KV_POOL, kCG>(ta, tb, tc, p, st);
         default:
             return CR_ERR_INVALID_ARG;

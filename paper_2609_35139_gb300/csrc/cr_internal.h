@@ -129,16 +129,18 @@ struct GemmParams {
     const float* bias2;
     // EPI_KV_POOL: the stale cache rows come from the pool (bf16 [n_pool, N], row
     // stride N): box_src[b] the pool row of the first of request rows 128 b ..
-    // 128 b + 127 when they are one contiguous pool range (loaded by TMA through
-    // tm_pool), else -1 (each row from src_row[t])
+    // 128 b + 127 when they are one contiguous pool range (one TMA box through
+    // tm_pool), else -1; then grp_src[g] the same for rows 8 g .. 8 g + 7 (one
+    // 8-row TMA box through tm_pool8), else -1 (each row from src_row[t])
     const uint16_t* kv_pool;
     const int64_t* src_row;
     const int64_t* box_src;
+    const int64_t* grp_src;
     float inv_freq[64];      // RoPE frequencies, rope_dim / 2 entries
     CUtensorMap tm_joint;    // EPI_KV_LOSS (set by launch_gemm; the type carries its alignment)
     CUtensorMap tm_alo;      // two-term A: the A_lo operand
     CUtensorMap tm_a2, tm_alo2, tm_b2, tm_c2;   // the second product (n_split > 0)
-    CUtensorMap tm_pool;                         // EPI_KV_POOL: the chunk pool
+    CUtensorMap tm_pool, tm_pool8;               // EPI_KV_POOL: the chunk pool, 128- and 8-row boxes
 };
 
 // One product of launch_gemm_pair: C[M, N] = A[M, K] W[N, K]^T + bias (fp32 out),
@@ -275,7 +277,8 @@ constexpr int64_t kSigmaSlice = 64;
 cr_status launch_gather(const GatherParams& p, cudaStream_t st);
 // the pool row of each request token, and per 128-row box its first token's
 // pool row when the box is one contiguous pool range (else -1)
-cr_status launch_src_rows(const GatherParams& p, int64_t* src_row, int64_t* box_src, cudaStream_t st);
+cr_status launch_src_rows(const GatherParams& p, int64_t* src_row, int64_t* box_src, int64_t* grp_src,
+                          cudaStream_t st);
 // K segments rotated in place by R_M(dir * (-pos)): dir = +1 canonicalises
 // (R_M(q)^{-1}), dir = -1 applies R_M(p).
 cr_status launch_canonicalize(void* kv, bool f32, int64_t n, const int32_t* pos, int L, int H, int dh,

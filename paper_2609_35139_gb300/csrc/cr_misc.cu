@@ -278,29 +278,41 @@ cr_status launch_rope_table(const int32_t* pos, int64_t n, int half_dim, const f
                       half_dim, f, table);
 }
 
-// The pool row of every request token (the gather's segment table), and per
+// The pool row of every request token (the gather's segment table); per
 // 128-row box of the request the pool row of its first token when all 128 rows
-// lie in one chunk (a contiguous pool range), else -1.
+// lie in one chunk (a contiguous pool range), else -1; and the same per 8-row
+// group, for the boxes that straddle chunks (16 groups per box, -1 for groups
+// past the request's end).
 __global__ void __launch_bounds__(256) src_rows_kernel(const __grid_constant__ GatherParams p,
                                                        int64_t* __restrict__ src_row,
-                                                       int64_t* __restrict__ box_src) {
+                                                       int64_t* __restrict__ box_src,
+                                                       int64_t* __restrict__ grp_src) {
     pdl_launch_dependents();
     pdl_wait();
     const int64_t n_box = (p.n_tokens + 127) / 128;
-    const int64_t n = p.n_tokens > n_box ? p.n_tokens : n_box;
+    const int64_t n_grp = 16 * n_box;
+    const int64_t n = p.n_tokens > n_grp ? p.n_tokens : n_grp;
+    auto seg_of = [&](int64_t t) {
+        int lo = 0, hi = p.n_seg - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (p.seg[mid].dst_row <= t)
+                lo = mid;
+            else
+                hi = mid - 1;
+        }
+        return lo;
+    };
+    // first row of rows [t0, t0 + len) in the pool when they are one chunk's, else -1
+    auto run_src = [&](int64_t t0, int64_t len) -> int64_t {
+        const int64_t t1 = t0 + len - 1;
+        if (t1 >= p.n_tokens) return -1;
+        const GatherSeg& sg = p.seg[seg_of(t0)];
+        const bool one = t1 < sg.dst_row + sg.len && t0 >= sg.dst_row;
+        return one ? sg.src_row + (t0 - sg.dst_row) : -1;
+    };
     for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        auto seg_of = [&](int64_t t) {
-            int lo = 0, hi = p.n_seg - 1;
-            while (lo < hi) {
-                const int mid = (lo + hi + 1) >> 1;
-                if (p.seg[mid].dst_row <= t)
-                    lo = mid;
-                else
-                    hi = mid - 1;
-            }
-            return lo;
-        };
         if (i < p.n_tokens) {
             const GatherSeg& sg = p.seg[seg_of(i)];
             const int64_t off = i - sg.dst_row;
@@ -311,20 +323,19 @@ __global__ void __launch_bounds__(256) src_rows_kernel(const __grid_constant__ G
                 src_row[i] = sg.src_row + off;
             }
         }
-        if (i < n_box) {
-            const int64_t t0 = 128 * i, t1 = t0 + 127;
-            const GatherSeg& sg = p.seg[seg_of(t0)];
-            const bool one = t1 < p.n_tokens && t1 < sg.dst_row + sg.len && t0 >= sg.dst_row;
-            box_src[i] = one ? sg.src_row + (t0 - sg.dst_row) : -1;
-        }
+        if (i < n_box) box_src[i] = run_src(128 * i, 128);
+        if (i < n_grp) grp_src[i] = run_src(8 * i, 8);
     }
 }
 
-cr_status launch_src_rows(const GatherParams& p, int64_t* src_row, int64_t* box_src, cudaStream_t st) {
+cr_status launch_src_rows(const GatherParams& p, int64_t* src_row, int64_t* box_src, int64_t* grp_src,
+                          cudaStream_t st) {
     if (p.n_tokens <= 0) return CR_OK;
-    const int64_t grid = (p.n_tokens + 255) / 256;
+    const int64_t n_grp = 16 * ((p.n_tokens + 127) / 128);
+    const int64_t n = p.n_tokens > n_grp ? p.n_tokens : n_grp;
+    const int64_t grid = (n + 255) / 256;
     return launch_pdl(src_rows_kernel, dim3(static_cast<unsigned>(grid)), dim3(256), 0, st, p, src_row,
-                      box_src);
+                      box_src, grp_src);
 }
 
 cr_status launch_gather(const GatherParams& p, cudaStream_t st) {

@@ -64,6 +64,24 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
                  "r"(bytes)
                  : "memory");
 }
+// Raise the barrier's expected transaction bytes without arriving (the arrival
+// follows once the caller's own writes to the guarded buffer are done).
+__device__ __forceinline__ void mbar_add_tx(uint64_t* bar, uint32_t bytes) {
+    asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+}
+// 16-byte asynchronous copy global -> shared (zero-filled where src_bytes is
+// 0), and the arrival on a barrier once this thread's earlier such copies have
+// landed (the barrier's pending count is raised first, so the phase also waits
+// for them).
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc, uint32_t src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(smem_dst)), "l"(gsrc),
+                 "r"(src_bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_mbar_arrive(uint64_t* bar) {
+    asm volatile("cp.async.mbarrier.arrive.shared::cta.b64 [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
 // Non-blocking probe of the phase (no suspend): the fast path of a wait.
 __device__ __forceinline__ bool mbar_test_wait(uint32_t addr, uint32_t parity) {
     uint32_t ok;
