@@ -445,6 +445,8 @@ def run_ours(args):
     lin_flops = 2.0 * N * (S * rp.d_seg * rp.d_c + tg.d_model * rp.d_c + 2 * rp.d_c * rp.d_b
                            + rp.n_blocks * rp.d_c * rp.d_b
                            + rp.n_blocks * (4 * rp.d_b * rp.d_b + 2 * rp.d_b * rp.mlp_hidden))
+    enc_flops = 2.0 * N * (S * rp.d_seg * rp.d_c + tg.d_model * rp.d_c + 2 * rp.d_c * rp.d_b
+                           + rp.n_blocks * rp.d_c * rp.d_b)
     tensor_flops = lin_flops + rp.n_blocks * attn_flops + head_flops
     ideal_ms = tensor_flops / (tf_sus * 1e12) * 1e3 + front_bytes / (hbm * 1e9) * 1e3
     roofline.update({
@@ -461,6 +463,10 @@ def run_ours(args):
         # fused front: its cache and embedding bytes plus the encoder's small GEMMs,
         # over the whole call
         "front_hbm_frac": front_bytes / (stages["assemble_compress"] * 1e-3) / 1e9 / hbm,
+        # the front against its own floor: its HBM bytes at the copy bandwidth plus the
+        # encoder's algorithmic flops (W_map, P_tok, F, P_b) at the burst peak
+        "front_frac": (front_bytes / (hbm * 1e9) + enc_flops / (tf_burst * 1e12)) * 1e3 /
+                      stages["assemble_compress"],
         "front_ms": stages["assemble_compress"],
         "attention_tensor_frac": attn_flops / (attn_ms * 1e-3) / 1e12 / tf_burst,
         "attention_ms_per_launch": attn_ms,
