@@ -218,3 +218,33 @@ def test_fused_front_rejects_bad_inputs_on_host(L):
                                   60, None, None, 3, None, None, 1, *([FAKE] * 2), 100,
                                   *([FAKE] * 4), None, FAKE, FAKE, FAKE, ws, None) == \
         cr.CR_ERR_UNSUPPORTED
+
+
+def test_pool_head_rejects_bad_inputs_on_host(L):
+    """cr_apply_residual_pool checks its dims, pointers, RoPE mode and workspace before
+    it reads the chunk map or launches anything."""
+    c, (t, r) = _dims()
+    w = cr.cr_weights()
+    w.w_out = w.b_out = w.sigma_delta = FAKE
+    ws = cr.cr_workspace_bytes(t, r, 100)
+    freq = np.ones(64, np.float32)
+
+    def call(tt=t, n=100, n_pool=60, yf=FAKE, kv_pool=FAKE, kv_out=FAKE, rope=cr.CR_ROPE_NONE,
+             inv_freq=None, workspace=FAKE, ws_bytes=ws, weights=w):
+        return L.cr_apply_residual_pool(ctypes.byref(tt), ctypes.byref(r), ctypes.byref(weights), yf, n,
+                                        kv_pool, n_pool, None, None, 3, None, None, 1, kv_out, FAKE,
+                                        inv_freq, rope, workspace, ws_bytes, None)
+
+    assert call(tt=cr.target_dims(4, 2, 128, 512, "f32")) == cr.CR_ERR_UNSUPPORTED   # bf16 caches only
+    assert call(n=0) == cr.CR_ERR_INVALID_ARG                      # no tokens
+    assert call(n_pool=0) == cr.CR_ERR_INVALID_ARG                 # empty pool
+    assert call(kv_pool=None) == cr.CR_ERR_INVALID_ARG             # no pool
+    assert call(kv_out=None) == cr.CR_ERR_INVALID_ARG              # no output
+    assert call(workspace=None) == cr.CR_ERR_INVALID_ARG           # no workspace
+    assert call(yf=FAKE + 8) == cr.CR_ERR_INVALID_ARG              # misaligned
+    assert call(rope=7) == cr.CR_ERR_INVALID_ARG                   # unknown RoPE mode
+    assert call(rope=cr.CR_ROPE_GLOBAL) == cr.CR_ERR_INVALID_ARG   # R_M without frequencies
+    assert call(ws_bytes=ws - 256) == cr.CR_ERR_INVALID_ARG        # workspace short
+    assert call(weights=cr.cr_weights()) == cr.CR_ERR_INVALID_ARG  # no head weights
+    odd = cr.target_dims(3, 1, 64, 512, "bf16")                    # D_KV = 384: not whole 256-column tiles
+    assert call(tt=odd, inv_freq=freq.ctypes.data) == cr.CR_ERR_UNSUPPORTED
