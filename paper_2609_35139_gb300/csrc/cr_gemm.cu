@@ -87,7 +87,12 @@ struct GemmCfg {
     // 16 KB boxes, column box b at boxes 2 b and 2 b + 1)
     static constexpr uint32_t kTileBytes =
         kInPlace ? BM * BN * kTileEsize * (kLoss ? 2 : 1) : 2 * kGroupBufs * 16384;
-    static constexpr uint32_t kVecBytes = BN * 4 * (kKV ? 2 : 1);   // bias (+ sigma)
+    // the 256-wide bf16 heads read their bias and sigma slices straight from global
+    // memory (every thread of a warp the same address: one broadcast load from L1),
+    // so that the 4 KB of staged vectors go to a fifth operand stage beside the
+    // 64 KB staged tile
+    static constexpr bool kVecGlobal = (EPI == EPI_KV_BF16 || EPI == EPI_KV_POOL || EPI == EPI_KV_PAGED);
+    static constexpr uint32_t kVecBytes = kVecGlobal ? 0u : BN * 4 * (kKV ? 2 : 1);   // bias (+ sigma)
     // in-place epilogues recycle the staged tile box by box, so the next tile's
     // vectors may land while this tile is still being finished: two buffers
     static constexpr int kVecBufs = kInPlace ? 2 : 1;
@@ -563,14 +568,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     for (int b = 0; b < Cfg::kBoxes; ++b) {
                         if (!(ok = mbar_wait_warp(&epi_empty[b], (static_cast<uint32_t>(i) & 1u) ^ 1u, wc, 101)))
                             break;
-                        const uint32_t vb = b == 0 ? (has_bias ? vbytes : 0u) + (Cfg::kKV ? vbytes : 0u) : 0u;
+                        const uint32_t vb =
+                            (b == 0 && !Cfg::kVecGlobal) ? (has_bias ? vbytes : 0u) + (Cfg::kKV ? vbytes : 0u) : 0u;
                         if (straddle) {
                             // a tile across chunk boundaries: its contiguous 8-row groups
                             // by TMA, the others copied by the warp, then one arrival
                             const uint32_t bytes = static_cast<uint32_t>(__popc(good)) * 1024u + vb;
                             if (elect_one()) {
                                 if (bytes) mbar_add_tx(&epi_full[b], bytes);
-                                if (b == 0) {
+                                if (b == 0 && !Cfg::kVecGlobal) {
                                     if (has_bias) bulk_load(vdst, p.bias + n0, vbytes, &epi_full[0]);
                                     if constexpr (Cfg::kKV) bulk_load(vdst + BN, p.sigma + n0, vbytes, &epi_full[0]);
                                 }
@@ -623,7 +629,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                                     tma_load_2d(tile + b * 16384, &tmC, &epi_full[b], n0 + b * Cfg::kBoxCols, m0);
                                 }
                             }
-                            if (b == 0) {
+                            if (b == 0 && !Cfg::kVecGlobal) {
                                 if (has_bias) bulk_load(vdst, p.bias + n0, vbytes, &epi_full[0]);
                                 if constexpr (Cfg::kKV) bulk_load(vdst + BN, p.sigma + n0, vbytes, &epi_full[0]);
                             }
@@ -839,8 +845,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 // this tile's vectors, and the per-box hand-over: box b of the
                 // staged tile is waited for before it is read and released to the
                 // store as soon as both groups have written their part of it
-                const float* vbt = vb + (i & 1) * (Cfg::kVecBytes / 4);
-                const float* vst = vbt + BN;
+                const float* vbt = Cfg::kVecGlobal ? p.bias + n0 : vb + (i & 1) * (Cfg::kVecBytes / 4);
+                const float* vst = Cfg::kVecGlobal ? p.sigma + n0 : vbt + BN;
                 auto wait_box = [&](int b) -> bool {
                     const bool w = mbar_wait(&epi_full[b], static_cast<uint32_t>(i) & 1u, wc, 302);
                     return __all_sync(0xffffffffu, w);
