@@ -778,6 +778,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             constexpr int NP = (EPI == EPI_QKV_ROPE) ? 32 : 1;
             float cs[NP], sn[NP];
             if constexpr (EPI == EPI_QKV_ROPE) rope_angles<NP>(p, m0 + r, cs, sn);
+            if constexpr (Cfg::kVecGlobal) {
+                // the tile's bias and sigma slices (BN fp32 each, 128-byte lines)
+                // into L1 while the MMAs still run
+                constexpr int kLines = BN * 4 / 128;
+                if (lane < kLines) {
+                    if (has_bias) prefetch_l1(p.bias + n0 + lane * 32);
+                    prefetch_l1(p.sigma + n0 + lane * 32);
+                }
+            }
             ok = mbar_wait(&tfull[acc], acc_phase, wc, 301);
             // in-place epilogues wait box by box below
             if (epi_load && !Cfg::kInPlace) ok = ok && mbar_wait(epi_full, static_cast<uint32_t>(i) & 1u, wc, 302);

@@ -183,6 +183,11 @@ __device__ __forceinline__ bool elect_one() {
 }
 
 // ----------------------------------------------------------------- TMA
+// Bring the 128-byte line holding p into this SM's L1 (a hint; no fault on any
+// address the caller may read).
+__device__ __forceinline__ void prefetch_l1(const void* p) {
+    asm volatile("prefetch.global.L1 [%0];" ::"l"(p));
+}
 __device__ __forceinline__ void tma_prefetch(const CUtensorMap* m) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(m)) : "memory");
 }
