@@ -302,8 +302,8 @@ cr_status cr_apply_residual(const cr_target_dims* target, const cr_repairer_dims
  * the same checks) and must describe exactly n_tokens rows; kv_out [N, D_KV]
  * receives every row.  workspace: the cr_workspace_bytes(.., >= n_tokens)
  * workspace (its pool-row tables and, under CR_ROPE_GLOBAL, the R_M table are
- * written).  Errors: CR_ERR_UNSUPPORTED for fp32 caches; otherwise as the two
- * calls it replaces.
+ * written).  Errors: CR_ERR_UNSUPPORTED for fp32 caches and for D_KV not a
+ * multiple of 256; otherwise as the two calls it replaces.
  */
 cr_status cr_apply_residual_pool(const cr_target_dims* target, const cr_repairer_dims* rep,
                                  const cr_weights* w, const uint16_t* yf, int64_t n_tokens,

@@ -59,8 +59,9 @@ struct GemmCfg {
     static constexpr bool kKV =
         (EPI == EPI_KV_BF16 || EPI == EPI_KV_F32 || EPI == EPI_KV_PAGED || EPI == EPI_KV_LOSS ||
          EPI == EPI_KV_POOL);
-    // the stale tile comes from the chunk pool (a TMA box where a box's rows are one
-    // contiguous pool range, else row by row), the repaired tile goes to the output
+    // the stale tile comes from the chunk pool (a 128-row TMA box where a box's rows
+    // are one chunk's; across a chunk boundary 8-row TMA boxes, and cp.async for the
+    // rows of the 8-row group that crosses it), the repaired tile goes to the output
     static constexpr bool kPoolSrc = (EPI == EPI_KV_POOL);
     // the stale tile is staged as for the in-place update, but the repaired rows
     // go straight from registers to the paged target cache (no TMA store)

@@ -275,8 +275,8 @@ constexpr int64_t kSigmaSlice = 64;
 
 // Launchers (validated arguments).
 cr_status launch_gather(const GatherParams& p, cudaStream_t st);
-// the pool row of each request token, and per 128-row box its first token's
-// pool row when the box is one contiguous pool range (else -1)
+// the pool row of each request token, and per 128-row box and per 8-row group
+// its first token's pool row when its rows are one chunk's (else -1)
 cr_status launch_src_rows(const GatherParams& p, int64_t* src_row, int64_t* box_src, int64_t* grp_src,
                           cudaStream_t st);
 // K segments rotated in place by R_M(dir * (-pos)): dir = +1 canonicalises
