@@ -373,3 +373,134 @@ def test_constant_head_adds_sigma_times_bias():
     kv = O.dtype_to_f64(a["kv"], "bf16")
     want = kv + c.weights["sigma_delta"].astype(np.float64) * bias.astype(np.float64)
     np.testing.assert_array_equal(res.repaired, want)
+
+
+# ------------------------------------------------------------------ whole method, brute force
+def _lin(W, x, b):
+    """Plain-Python affine map: out[i] = sum_k W[i][k] x[k] + b[i]."""
+    return [sum(W[i][k] * x[k] for k in range(len(x))) + b[i] for i in range(len(W))]
+
+
+def _ln(x, g, b, eps):
+    n = len(x)
+    mu = sum(x) / n
+    var = sum((a - mu) ** 2 for a in x) / n
+    return [(a - mu) / math.sqrt(var + eps) * g[i] + b[i] for i, a in enumerate(x)]
+
+
+def _repair_brute_force(kv, emb, cid, pos, w, *, L, H, dh, n_heads, eps, theta):
+    """The repair forward of Sec. 4.1 written out token by token with Python floats:
+    StaleEncoder (one d_h -> d_seg map per segment on kv / sigma_stale, then W_map),
+    token fusion F([s; P_tok e]), B pre-LN Repair Blocks whose input is h + P_b(s),
+    each with rotate-half RoPE on q and k, softmax attention over keys j with
+    c(j) <= c(i), an erf-GELU MLP, then LN_f, the head and kv + sigma_Delta z."""
+    n, D = len(kv), len(kv[0])
+    S = D // dh
+    lst = lambda a: np.asarray(a, np.float64).tolist()
+    sig = lst(w["sigma_stale"])
+    s_feat = []
+    for t in range(n):
+        y = []
+        for s in range(S):
+            x = [kv[t][s * dh + d] / sig[s * dh + d] for d in range(dh)]
+            y += _lin(lst(w["w_seg"][s]), x, lst(w["b_seg"][s]))
+        s_feat.append(_lin(lst(w["w_map"]), y, lst(w["b_map"])))
+    h = []
+    for t in range(n):
+        e = _lin(lst(w["w_tok"]), emb[t], lst(w["b_tok"]))
+        h.append(_lin(lst(w["w_fuse"]), s_feat[t] + e, lst(w["b_fuse"])))
+    db = len(h[0])
+    hd = db // n_heads
+    B = w["w_rein"].shape[0]
+    for b in range(B):
+        p = f"blk{b}."
+        x = [[a + r for a, r in zip(h[t], _lin(lst(w["w_rein"][b]), s_feat[t], lst(w["b_rein"][b])))]
+             for t in range(n)]
+        q, k, v = [], [], []
+        for t in range(n):
+            u = _ln(x[t], lst(w[p + "ln1_g"]), lst(w[p + "ln1_b"]), eps)
+            o = _lin(lst(w[p + "w_qkv"]), u, lst(w[p + "b_qkv"]))
+            qt, kt = [], []
+            for hh in range(n_heads):
+                for src, dst in ((o[hh * hd:(hh + 1) * hd], qt), (o[db + hh * hd:db + (hh + 1) * hd], kt)):
+                    half = hd // 2
+                    for i in range(half):
+                        ang = pos[t] * theta ** (-2.0 * i / hd)
+                        c, sn = math.cos(ang), math.sin(ang)
+                        dst.append(src[i] * c - src[i + half] * sn)
+                    for i in range(half):
+                        ang = pos[t] * theta ** (-2.0 * i / hd)
+                        c, sn = math.cos(ang), math.sin(ang)
+                        dst.append(src[i + half] * c + src[i] * sn)
+            q.append(qt)
+            k.append(kt)
+            v.append(o[2 * db:])
+        x2 = []
+        for i in range(n):
+            att = [0.0] * db
+            for hh in range(n_heads):
+                sl = slice(hh * hd, (hh + 1) * hd)
+                sc = [(j, sum(a * c for a, c in zip(q[i][sl], k[j][sl])) / math.sqrt(hd))
+                      for j in range(n) if cid[j] <= cid[i]]
+                m = max(s for _, s in sc)
+                den = sum(math.exp(s - m) for _, s in sc)
+                for j, s in sc:
+                    for d in range(hd):
+                        att[hh * hd + d] += math.exp(s - m) / den * v[j][hh * hd + d]
+            x2.append([a + c for a, c in zip(x[i], _lin(lst(w[p + "w_o"]), att, lst(w[p + "b_o"])))])
+        h = []
+        for t in range(n):
+            u = _ln(x2[t], lst(w[p + "ln2_g"]), lst(w[p + "ln2_b"]), eps)
+            g = [0.5 * a * (1.0 + math.erf(a / math.sqrt(2.0)))
+                 for a in _lin(lst(w[p + "w_fc1"]), u, lst(w[p + "b_fc1"]))]
+            h.append([a + c for a, c in zip(x2[t], _lin(lst(w[p + "w_fc2"]), g, lst(w[p + "b_fc2"])))])
+    sd = lst(w["sigma_delta"])
+    out = []
+    for t in range(n):
+        yf = _ln(h[t], lst(w["lnf_g"]), lst(w["lnf_b"]), eps)
+        z = _lin(lst(w["w_out"]), yf, lst(w["b_out"]))
+        out.append([kv[t][c] + sd[c] * z[c] for c in range(D)])
+    return np.array(s_feat), np.array(out)
+
+
+def test_whole_repair_brute_force_tiny():
+    """The oracle's repair of a 7-token, 3-chunk request equals the token-by-token
+    Python-float restatement of Sec. 4.1 (every weight, bias and LayerNorm affine
+    random and nonzero, two blocks, two heads, two segments)."""
+    g = np.random.default_rng(11)
+    L, H, dh, dm = 1, 1, 4, 5          # D_KV = 2 L H d_h = 8: segments K and V of layer 0
+    ds, dc, db, B, nh, hid = 2, 3, 4, 2, 2, 6
+    S, D = 2 * L * H, 2 * L * H * dh
+    r = lambda *shape: g.normal(size=shape) * 0.5
+    w = {"w_seg": r(S, ds, dh), "b_seg": r(S, ds), "w_map": r(dc, S * ds), "b_map": r(dc),
+         "w_tok": r(dc, dm), "b_tok": r(dc), "w_fuse": r(db, 2 * dc), "b_fuse": r(db),
+         "w_rein": r(B, db, dc), "b_rein": r(B, db), "lnf_g": 1 + r(db), "lnf_b": r(db),
+         "w_out": r(D, db), "b_out": r(D), "sigma_stale": 0.5 + g.random(D),
+         "sigma_delta": 0.5 + g.random(D)}
+    for b in range(B):
+        p = f"blk{b}."
+        w.update({p + "ln1_g": 1 + r(db), p + "ln1_b": r(db), p + "w_qkv": r(3 * db, db),
+                  p + "b_qkv": r(3 * db), p + "w_o": r(db, db), p + "b_o": r(db),
+                  p + "ln2_g": 1 + r(db), p + "ln2_b": r(db), p + "w_fc1": r(hid, db),
+                  p + "b_fc1": r(hid), p + "w_fc2": r(db, hid), p + "b_fc2": r(db)})
+    n = 7
+    cid = np.array([0, 0, 1, 1, 1, 2, 2], np.int32)
+    pos = np.arange(n)
+    kv = g.normal(size=(n, D))
+    emb = g.normal(size=(n, dm))
+    eps, theta = 1e-5, 1e4
+    res = O.repair_request(kv, emb, cid, pos, w, cache_dtype="f32", n_layers=L, n_kv_heads=H,
+                           head_dim=dh, n_heads=nh, eps=eps, rope_theta=theta)
+    s_bf, rep_bf = _repair_brute_force(kv.tolist(), emb.tolist(), cid.tolist(), pos.tolist(), w, L=L,
+                                       H=H, dh=dh, n_heads=nh, eps=eps, theta=theta)
+    np.testing.assert_allclose(res.s, s_bf, rtol=1e-11, atol=1e-12)
+    np.testing.assert_allclose(res.repaired, rep_bf, rtol=1e-10, atol=1e-11)
+    # and the restatement is sensitive to what it checks: V and K swapped in the
+    # qkv split, or the mask reversed, move the result well outside the tolerance
+    w_sw = dict(w)
+    for b in range(B):
+        q_, k_, v_ = np.split(w[f"blk{b}.w_qkv"], 3)
+        w_sw[f"blk{b}.w_qkv"] = np.concatenate([q_, v_, k_])
+    res_sw = O.repair_request(kv, emb, cid, pos, w_sw, cache_dtype="f32", n_layers=L, n_kv_heads=H,
+                              head_dim=dh, n_heads=nh, eps=eps, rope_theta=theta)
+    assert np.abs(res_sw.repaired - rep_bf).max() > 1e-3
