@@ -220,7 +220,8 @@ cr_status cr_compress_features(const cr_target_dims* target, const cr_repairer_d
  * cache is then not written at all (cr_apply_residual_pool writes the repaired
  * cache from the pool).  The caller sizes kv_out, emb_out and the
  * workspace (cr_workspace_bytes(.., max_tokens)) for max_tokens rows.
- * Errors: those of the two calls, checked before any launch.
+ * Errors: those of the two calls, checked before any launch;
+ * CR_ERR_UNSUPPORTED for a NULL kv_out with an fp32 cache.
  */
 cr_status cr_assemble_compress(const cr_target_dims* target, const cr_repairer_dims* rep,
                                const cr_weights* w, const void* kv_pool, const void* emb_pool,
