@@ -10,8 +10,8 @@ writing the repaired cache), captured once into a CUDA graph and replayed.
 Default workload: the Llama-3.1-8B-shaped cache (32 layers, 8 KV heads,
 head_dim 128, d_model 4096) with the d_c 512 / d_b 1024 / 6-block repairer,
 one request of 10 chunks x 512 tokens.  Inputs are seeded and synthetic; the
-pool (1 GiB) and the assembled cache (0.67 GB) exceed the 129 MB L2, so no
-explicit L2 flush is needed between steps.
+pool (1 GiB) and the request's cache (0.67 GB, read from the pool and written
+repaired) exceed the 129 MB L2, so no explicit L2 flush is needed between steps.
 
     python bench.py [--gpus N --steps K --warmup W] [--impl reference]
                     [--mask MODE] [--component kv|k|v] [--offset stale|zero]
@@ -369,9 +369,9 @@ def run_ours(args):
     total_ms = max_over_ranks(sum(per_step), "cuda")
     value = whole_job_rate(world, N, args.steps, total_ms)
     l2_note = (f"L2 flushed between steps (512 MB written outside the timed events): the "
-               f"assembled cache ({cache_bytes / 1e6:.0f} MB) is under twice the 129 MB L2"
+               f"request's cache ({cache_bytes / 1e6:.0f} MB) is under twice the 129 MB L2"
                if flush is not None else
-               f"no flush: the assembled cache ({cache_bytes / 1e6:.0f} MB) and the pool exceed the "
+               f"no flush: the request's cache ({cache_bytes / 1e6:.0f} MB) and the pool exceed the "
                f"129 MB L2")
     st, word = cr.cr_get_device_status()
     if st != cr.CR_OK:
